@@ -1,0 +1,434 @@
+#!/usr/bin/env python3
+"""Throughput of the MoSA layer (forward + backward) on GB300.
+
+    python bench.py [--gpus N] [--steps K] [--warmup W] [--impl mosa|reference]
+                    [--config NAME] [--no-cpu-baseline]
+
+A step is one forward and one backward pass of the layer over one batch of
+the workload (default: B=8 sequences of T=1024 tokens, d=512, H=16 heads of
+size 64, k=128 tokens per head, bf16 storage) with inputs resident in HBM.
+L2 is flushed (a 256 MiB write) before every timed step, outside the step's
+CUDA events.  Under torchrun every rank runs its own copy of the workload
+(weak scaling, no collective on the data path); the reported time is the
+maximum over ranks.
+
+Rank 0 prints one JSON line: tokens/s, the roofline of the dominant kernel
+(timed live with CUDA events on the library's stream), the fp64 CPU oracle
+timed on a bounded sample of the same workload, an end-to-end figure through
+the public API with host buffers, SM clocks sampled during the timed region
+and the number of library kernels launched.
+
+``--impl reference`` times the CPU oracle (the only reference this layer
+has) on the host cores instead.
+"""
+from __future__ import annotations
+
+import argparse
+import hashlib
+import json
+import os
+import statistics
+import subprocess
+import sys
+import tempfile
+import threading
+import time
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+METRIC = "MoSA layer fwd+bwd tokens/s; achieved TFLOP/s and HBM GB/s vs GB300 peak"
+L2_FLUSH_BYTES = 256 << 20
+FALLBACK_PEAKS = {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "bf16_tflops_sustained": 1700.0,
+                  "sm_max_mhz": 2070.0}
+NUM_SM = 152
+FP32_LANES_PER_SM = 128
+
+
+def parse_args():
+    p = argparse.ArgumentParser(description=__doc__.split("\n")[0])
+    p.add_argument("--gpus", type=int, default=1)
+    p.add_argument("--steps", type=int, default=200)
+    p.add_argument("--warmup", type=int, default=10)
+    p.add_argument("--impl", choices=["mosa", "reference"], default="mosa")
+    p.add_argument("--config", default=None)
+    p.add_argument("--no-cpu-baseline", action="store_true")
+    p.add_argument("--cpu-budget-s", type=float, default=15.0)
+    return p.parse_args()
+
+
+def load_peaks():
+    path = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    if os.path.exists(path):
+        with open(path) as f:
+            d = json.load(f)
+        return {k: float(d.get(k, FALLBACK_PEAKS[k])) for k in FALLBACK_PEAKS}, "measured"
+    return dict(FALLBACK_PEAKS), "fallback"
+
+
+# ----------------------------------------------------------------- clocks
+
+class ClockSampler:
+    """nvidia-smi samples (200 ms) kept only while the timed region runs."""
+    FIELDS = ("timestamp,index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+              "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+              "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, gpu_index: int):
+        self.gpu = gpu_index
+        self.proc = None
+        self.lines: list[tuple[float, str]] = []
+        self.window = (0.0, 0.0)
+
+    def start(self):
+        try:
+            self.proc = subprocess.Popen(
+                ["nvidia-smi", f"--id={self.gpu}", f"--query-gpu={self.FIELDS}",
+                 "--format=csv,noheader,nounits", "-lms", "200"],
+                stdout=subprocess.PIPE, stderr=subprocess.DEVNULL, text=True)
+        except (FileNotFoundError, OSError):
+            self.proc = None
+            return
+        self.reader = threading.Thread(target=self._read, daemon=True)
+        self.reader.start()
+        time.sleep(0.6)
+
+    def _read(self):
+        for line in self.proc.stdout:
+            self.lines.append((time.time(), line.strip()))
+
+    def mark(self, t0, t1):
+        self.window = (t0, t1)
+
+    def stop(self):
+        if self.proc is None:
+            return None
+        time.sleep(0.3)
+        self.proc.terminate()
+        try:
+            self.proc.wait(timeout=5)
+        except subprocess.TimeoutExpired:
+            self.proc.kill()
+        t0, t1 = self.window
+        rows = [l for (t, l) in self.lines if t0 - 0.25 <= t <= t1 + 0.25]
+        if not rows:
+            rows = [l for (_, l) in self.lines]
+        mhz, maxes, reasons = [], [], set()
+        names = ("hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap")
+        for r in rows:
+            f = [x.strip() for x in r.split(",")]
+            if len(f) < 10:
+                continue
+            try:
+                mhz.append(float(f[2]))
+                maxes.append(float(f[3]))
+            except ValueError:
+                continue
+            for name, val in zip(names, f[6:10]):
+                if val.lower().startswith("active"):
+                    reasons.add(name)
+        if not mhz:
+            return None
+        return {"sm_mhz": statistics.median(mhz), "sm_max_mhz": max(maxes),
+                "reasons": sorted(reasons), "samples": len(mhz)}
+
+
+# ------------------------------------------------------------ CPU oracle
+
+def oracle_sample(cfg, x, n_seq):
+    """Time the oracle's forward + backward on the first n_seq sequences."""
+    import oracle
+    W = (x["Wr"], x["Wq"], x["Wk"], x["Wv"], x["Wo"])
+    batches = list(range(n_seq))
+    t0 = time.perf_counter()
+    _, I, _, _ = oracle.forward(x["X"], *W, k=cfg.k, batches=batches)
+    if cfg.backward:
+        oracle.backward(x["X"], *W, I=I, dY=x["dY"], batches=batches)
+    return time.perf_counter() - t0
+
+
+def choose_sample(cfg, x, budget_s):
+    t1 = oracle_sample(cfg, x, 1)
+    n = int(max(1, min(cfg.B, budget_s // max(t1, 1e-6))))
+    return n, t1
+
+
+def cpu_baseline(cfg, x, budget_s):
+    import oracle
+    n, t1 = choose_sample(cfg, x, budget_s)
+    t = oracle_sample(cfg, x, n) if n > 1 else t1
+    what = "forward+backward" if cfg.backward else "forward"
+    return {"value": n * cfg.T / t, "unit": "tokens/s", "cores": oracle.num_threads(),
+            "kind": "oracle",
+            "sample": f"{what} of {n} of the {cfg.B} sequences of {cfg.name} "
+                      f"(all {cfg.H} heads, fp64, {t:.2f} s)"}
+
+
+# ------------------------------------------------------------ roofline
+
+STAGES = ["router", "select", "qkv", "attn_fwd", "out", "out_bwd", "attn_bwd", "in_bwd",
+          "w_bwd"]
+
+
+def stage_bound(stage, peaks, kind):
+    """(bound, peak, unit) for a stage implemented as `kind` ('tensor', 'simt', 'mem')."""
+    if kind == "mem":
+        return "hbm", peaks["hbm_gbs"], "GB/s"
+    if kind == "tensor":
+        return "tensor", peaks["bf16_tflops_sustained"], "TFLOP/s"
+    ffma = NUM_SM * FP32_LANES_PER_SM * 2 * peaks["sm_max_mhz"] * 1e6 / 1e12
+    return "alu", ffma, "TFLOP/s"
+
+
+def stage_kind(stage, lib_impl):
+    if stage in ("router", "select"):
+        return "mem"
+    return lib_impl.get(stage, "simt")
+
+
+def traffic_for(stage, cfg_name):
+    """Per-launch DRAM bytes of `stage` from the committed ncu summary, or None
+    when the summary is missing or was taken on a different kernel source."""
+    path = os.path.join(ROOT, "profiles", "traffic.json")
+    if not os.path.exists(path):
+        return None
+    with open(path) as f:
+        d = json.load(f)
+    ent = d.get(cfg_name, {}).get(stage)
+    if not ent:
+        return None
+    if ent.get("source_sha256") != source_digest():
+        return None
+    return ent.get("bytes_per_launch")
+
+
+def source_digest():
+    import glob
+    h = hashlib.sha256()
+    for p in sorted(glob.glob(os.path.join(ROOT, "paper_2505_00315_gb300", "csrc", "*"))):
+        with open(p, "rb") as f:
+            h.update(f.read())
+    return h.hexdigest()
+
+
+# ------------------------------------------------------------------ main
+
+def run_reference(args, cfg, rank, world):
+    """The oracle as the reference arm: rank 0 times it on the host cores."""
+    if rank != 0:
+        return
+    import oracle
+    from paper_2505_00315_gb300 import workloads as W
+    x = W.make_inputs(cfg)
+    per_step_budget = max(1.0, 150.0 / max(1, args.steps + args.warmup))
+    n, _ = choose_sample(cfg, x, per_step_budget)
+    for _ in range(args.warmup):
+        oracle_sample(cfg, x, n)
+    times = [oracle_sample(cfg, x, n) for _ in range(args.steps)]
+    total = sum(times)
+    value = n * cfg.T * args.steps / total
+    what = "forward+backward" if cfg.backward else "forward"
+    line = {"impl": "reference", "metric": METRIC, "value": value, "unit": "tokens/s",
+            "n_gpus": args.gpus, "steps": args.steps, "warmup": args.warmup,
+            "ms_per_step": 1e3 * total / args.steps, "higher_is_better": True,
+            "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic",
+            "config": config_block(cfg),
+            "cpu_baseline": {"value": value, "unit": "tokens/s", "kind": "oracle",
+                             "cores": oracle.num_threads(),
+                             "sample": f"{what} of {n} of the {cfg.B} sequences per step"},
+            "e2e": {"value": value, "unit": "tokens/s", "h2d_bytes_per_step": 0,
+                    "d2h_bytes_per_step": 0}}
+    print(json.dumps(line), flush=True)
+
+
+def config_block(cfg):
+    return {"workload": cfg.name, "B": cfg.B, "T": cfg.T, "d": cfg.d, "H": cfg.H, "hp": cfg.hp,
+            "k": cfg.k, "storage": cfg.dtype,
+            "inputs": "seeded Gaussian X, weights N(0,1/d), dY; planted router margin",
+            "l2": "flushed before every timed step by a 256 MiB write outside the step's events"}
+
+
+def main():
+    args = parse_args()
+    import torch
+    from paper_2505_00315_gb300 import workloads as W
+
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    cfg = W.CONFIGS[args.config or W.BENCH_CONFIG]
+
+    if args.impl == "reference":
+        run_reference(args, cfg, rank, world)
+        return
+
+    import paper_2505_00315_gb300 as mosa
+    from paper_2505_00315_gb300 import flops
+
+    torch.cuda.set_device(local)
+    dist = None
+    if world > 1:
+        import torch.distributed as dist
+        dist.init_process_group("nccl", device_id=torch.device("cuda", local))
+
+    def barrier():
+        if dist is not None:
+            dist.barrier()
+
+    x = W.make_inputs(cfg)
+    tdt = torch.bfloat16 if cfg.dtype == "bf16" else torch.float32
+    dev = torch.device("cuda", local)
+    D = {n: torch.from_numpy(x[n]).to(dev).to(tdt) for n in x}
+    shape = mosa.make_shape(D["X"], D["Wq"], cfg.k)
+    ws = mosa.alloc_workspace(shape, dev)
+    f32 = dict(dtype=torch.float32, device=dev)
+    outs = {"Y": torch.empty((cfg.B, cfg.T, cfg.d), **f32),
+            "I": torch.empty((cfg.B, cfg.H, cfg.k), dtype=torch.int32, device=dev),
+            "r_sel": torch.empty((cfg.B, cfg.H, cfg.k), **f32)}
+    grads = {"dX": torch.empty((cfg.B, cfg.T, cfg.d), **f32),
+             "dW_r": torch.empty((cfg.d, cfg.H), **f32),
+             "dW_q": torch.empty((cfg.H, cfg.d, cfg.hp), **f32),
+             "dW_k": torch.empty((cfg.H, cfg.d, cfg.hp), **f32),
+             "dW_v": torch.empty((cfg.H, cfg.d, cfg.hp), **f32),
+             "dW_o": torch.empty((cfg.H, cfg.hp, cfg.d), **f32)}
+    flush_buf = torch.empty(L2_FLUSH_BYTES // 4, **f32)
+
+    def step(Xd=None, dYd=None):
+        Xd = D["X"] if Xd is None else Xd
+        dYd = D["dY"] if dYd is None else dYd
+        Y, I, rs, _, _ = mosa.mosa_forward(Xd, D["Wr"], D["Wq"], D["Wk"], D["Wv"], D["Wo"],
+                                           cfg.k, workspace=ws, out=outs)
+        if cfg.backward:
+            mosa.mosa_backward(Xd, D["Wr"], D["Wq"], D["Wk"], D["Wv"], D["Wo"], I, rs, dYd, ws,
+                               out=grads)
+
+    # Warm-up, then one profiled pass to find the dominant stage.
+    for _ in range(max(3, args.warmup)):
+        flush_buf.zero_()
+        step()
+    torch.cuda.synchronize()
+    mosa.mosa_profile_stages((1 << len(STAGES)) - 1)
+    for _ in range(5):
+        flush_buf.zero_()
+        step()
+    torch.cuda.synchronize()
+    prof = mosa.mosa_profile_read()
+    mosa.mosa_profile_stages(0)
+    stage_ms = {s: prof[s][0] / max(prof[s][1], 1) for s in STAGES if prof[s][1]}
+    dominant = max(stage_ms, key=stage_ms.get)
+
+    # Timed region: K steps, L2 flushed before each, dominant stage timed live.
+    K = args.steps
+    starts = [torch.cuda.Event(enable_timing=True) for _ in range(K)]
+    ends = [torch.cuda.Event(enable_timing=True) for _ in range(K)]
+    sampler = ClockSampler(local) if rank == 0 else None
+    if sampler:
+        sampler.start()
+    barrier()
+    torch.cuda.synchronize()
+    launches0 = mosa.mosa_kernel_launches()
+    mosa.mosa_profile_stages(1 << STAGES.index(dominant))
+    t_host0 = time.time()
+    for i in range(K):
+        flush_buf.zero_()
+        starts[i].record()
+        step()
+        ends[i].record()
+    torch.cuda.synchronize()
+    t_host1 = time.time()
+    barrier()
+    launches = mosa.mosa_kernel_launches() - launches0
+    mosa.mosa_profile_stages(0)
+    dom = mosa.mosa_profile_read()[dominant]
+    clocks = None
+    if sampler:
+        sampler.mark(t_host0, t_host1)
+        clocks = sampler.stop()
+    total_ms = sum(s.elapsed_time(e) for s, e in zip(starts, ends))
+    if dist is not None:
+        t = torch.tensor([total_ms], dtype=torch.float64, device=dev)
+        dist.all_reduce(t, op=dist.ReduceOp.MAX)
+        total_ms = float(t.item())
+    tokens = world * cfg.B * cfg.T * K
+    value = tokens / (total_ms / 1e3)
+
+    # End to end through the public API with pinned host buffers.
+    hX = torch.from_numpy(x["X"]).to(tdt).pin_memory()
+    hdY = torch.from_numpy(x["dY"]).to(tdt).pin_memory()
+    hY = torch.empty((cfg.B, cfg.T, cfg.d), dtype=torch.float32).pin_memory()
+    hdX = torch.empty((cfg.B, cfg.T, cfg.d), dtype=torch.float32).pin_memory()
+    Xd = torch.empty_like(D["X"])
+    dYd = torch.empty_like(D["dY"])
+    e2e_steps = max(10, K // 4)
+
+    def e2e_step():
+        Xd.copy_(hX, non_blocking=True)
+        dYd.copy_(hdY, non_blocking=True)
+        step(Xd, dYd)
+        hY.copy_(outs["Y"], non_blocking=True)
+        hdX.copy_(grads["dX"], non_blocking=True)
+
+    for _ in range(3):
+        e2e_step()
+    torch.cuda.synchronize()
+    barrier()
+    e0 = torch.cuda.Event(enable_timing=True)
+    e1 = torch.cuda.Event(enable_timing=True)
+    e0.record()
+    for _ in range(e2e_steps):
+        e2e_step()
+    e1.record()
+    torch.cuda.synchronize()
+    e2e_ms = e0.elapsed_time(e1)
+    if dist is not None:
+        t = torch.tensor([e2e_ms], dtype=torch.float64, device=dev)
+        dist.all_reduce(t, op=dist.ReduceOp.MAX)
+        e2e_ms = float(t.item())
+    h2d = hX.numel() * hX.element_size() + hdY.numel() * hdY.element_size()
+    d2h = hY.numel() * 4 + hdX.numel() * 4
+
+    if rank != 0:
+        if dist is not None:
+            dist.destroy_process_group()
+        return
+
+    # Roofline of the dominant kernel.
+    peaks, peak_src = load_peaks()
+    work = flops.layer_work(cfg.B, cfg.T, cfg.d, cfg.H, cfg.hp, cfg.k,
+                            elem_bytes=2 if cfg.dtype == "bf16" else 4)
+    impl = getattr(mosa, "stage_impl", lambda s: {})(shape)
+    kind = stage_kind(dominant, impl)
+    bound, peak, unit = stage_bound(dominant, peaks, kind)
+    dom_ms = dom[0] / max(dom[1], 1)
+    if unit == "GB/s":
+        achieved = work[dominant]["bytes"] / (dom_ms / 1e3) / 1e9
+    else:
+        achieved = work[dominant]["flops"] / (dom_ms / 1e3) / 1e12
+    layer_flops = work["forward_flops"] + (work["backward_flops"] if cfg.backward else 0)
+    line = {
+        "metric": METRIC, "value": value, "unit": "tokens/s", "n_gpus": world, "steps": K,
+        "warmup": args.warmup, "ms_per_step": total_ms / K, "higher_is_better": True,
+        "scaling": "weak", "vs_baseline": None, "dtype": cfg.dtype, "data": "synthetic",
+        "config": config_block(cfg),
+        "roofline": {"kernel": dominant, "bound": bound, "achieved": achieved, "peak": peak,
+                     "unit": unit, "frac": achieved / peak, "peak_source": peak_src,
+                     "traffic": traffic_for(dominant, cfg.name),
+                     "algorithmic": work[dominant]["flops" if unit != "GB/s" else "bytes"],
+                     "ms_per_launch": dom_ms},
+        "layer_tflops": layer_flops * world * K / (total_ms / 1e3) / 1e12,
+        "stage_ms": {s: round(v, 5) for s, v in stage_ms.items()},
+        "e2e": {"value": world * cfg.B * cfg.T * e2e_steps / (e2e_ms / 1e3), "unit": "tokens/s",
+                "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h,
+                "what": "pinned host X, dY -> device; forward+backward; Y, dX -> pinned host"},
+        "gpu_launches": int(launches),
+        "clocks": clocks,
+    }
+    if world == 1 and not args.no_cpu_baseline:
+        line["cpu_baseline"] = cpu_baseline(cfg, x, args.cpu_budget_s)
+    print(json.dumps(line), flush=True)
+    if dist is not None:
+        dist.destroy_process_group()
+
+
+if __name__ == "__main__":
+    main()

@@ -1,0 +1,169 @@
+/*
+ * libmosa: Mixture-of-Sparse-Attention (MoSA) layer on one NVIDIA GB300 (sm_103a).
+ *
+ * The layer (arXiv 2505.00315, Sec. 2.2 and Eq. mosa_mha) for each sequence b
+ * and head h:
+ *     r      = sigmoid(X[b] W_r[:,h])                 router scores over T tokens
+ *     r^topk, I = TopK(r, k)                          k tokens chosen by the head
+ *     X^s    = X[b, I, :]                             gathered rows
+ *     Q, K, V = X^s W_q[h], X^s W_k[h], X^s W_v[h]
+ *     A      = softmax((Q K^T + M) / sqrt(h')) V,     M_ij = 0 iff I_i >= I_j, else -inf
+ *     Y[b, I_i, :] += r^topk_i (A W_o[h])_i           scattered back; heads summed
+ *
+ * Conventions shared by every call:
+ *   - All tensor pointers are DEVICE pointers to caller-owned memory; the
+ *     layer calls allocate nothing on the device or the host (only the
+ *     optional stage timing below creates CUDA events).
+ *   - Layouts are dense row-major:
+ *       X, dY     [B,T,d]      storage dtype (fp32 or bf16)
+ *       W_r       [d,H]        storage dtype
+ *       W_q,W_k,W_v [H,d,h']   storage dtype
+ *       W_o       [H,h',d]     storage dtype
+ *       Y, dX     [B,T,d]      fp32
+ *       I         [B,H,k]      int32, strictly ascending token indices
+ *       r_sel     [B,H,k]      fp32, r^topk in the order of I
+ *       r_full    [B,H,T]      fp32 router scores of every token
+ *       dW_r      [d,H]  dW_q,dW_k,dW_v [H,d,h']  dW_o [H,h',d]   fp32
+ *   - Calls are asynchronous on `stream` (a cudaStream_t, NULL = legacy default
+ *     stream).  They return after argument validation and kernel launch.
+ *   - Outputs are overwritten, never accumulated into.
+ *   - Arithmetic: fp32 accumulation everywhere; with bf16 storage the saved
+ *     intermediates (Q, K, V, attention output, gradients fed to tensor-core
+ *     products) are rounded to bf16.
+ *   - Tokens tied on the router score are taken lowest index first.
+ *   - NaN inputs give undefined results (but no out-of-bounds access).
+ *   - Errors: a call that returns anything but MOSA_OK has launched nothing.
+ *     Errors found on the device (invalid caller indices, a bounded wait that
+ *     ran out) are recorded in a status word inside the workspace; read and
+ *     clear it with mosa_check_status().
+ */
+#ifndef MOSA_H_
+#define MOSA_H_
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+typedef enum {
+    MOSA_OK = 0,
+    MOSA_ERR_INVALID_ARG = 1,     /* bad sizes, NULL pointers, k > T, bad indices */
+    MOSA_ERR_UNSUPPORTED = 2,     /* valid but outside what the kernels implement */
+    MOSA_ERR_CUDA = 3,            /* a CUDA runtime call or launch failed */
+    MOSA_ERR_DEVICE_TIMEOUT = 4,  /* a bounded device-side wait gave up */
+    MOSA_ERR_WORKSPACE = 5        /* workspace NULL, too small or misaligned */
+} mosa_status;
+
+typedef enum { MOSA_F32 = 0, MOSA_BF16 = 1 } mosa_dtype;
+
+/* Problem size.  B sequences of T tokens of width d; H MoSA heads of size hp
+ * (the paper's h'); each head keeps k of the T tokens (Sec. 2.2). */
+typedef struct {
+    int32_t B, T, d, H, hp, k;
+    int32_t dtype; /* mosa_dtype of X, dY and all weights */
+} mosa_shape;
+
+/* Supported sizes (else MOSA_ERR_UNSUPPORTED):
+ *   1 <= k <= T <= 65536; B, H >= 1; B*T*d < 2^31; H*d*hp < 2^31;
+ *   d % 8 == 0 and hp in {16, 32, 64, 128}. */
+
+/* Human-readable name of a status code (static string, never NULL). */
+const char *mosa_status_string(mosa_status s);
+
+/* Bytes of device workspace the calls below need for `shape`; 0 if the shape
+ * is invalid or unsupported.  The workspace carries the state that
+ * mosa_backward reuses from mosa_forward (router scores, selected rows,
+ * Q/K/V, attention output and its log-sum-exp) plus the status word, so the
+ * same buffer must be passed to a forward and the backward that follows it.
+ * It must be 256-byte aligned. */
+size_t mosa_workspace_bytes(const mosa_shape *shape);
+
+/* Forward pass of the layer (Sec. 2.2, Eq. mosa_mha): router, TopK, gather,
+ * per-head projections, index-masked causal attention, diag(r^topk) A W_o and
+ * the scatter-sum into Y.
+ *   X, W_r, W_q, W_k, W_v, W_o : inputs (storage dtype), see layouts above.
+ *   Y      : [B,T,d] fp32 output; rows chosen by no head are 0.
+ *   I      : [B,H,k] int32 output, ascending.
+ *   r_sel  : [B,H,k] fp32 output, r at I.
+ *   r_full : [B,H,T] fp32 output of all router scores, or NULL.
+ *   workspace, workspace_bytes : see mosa_workspace_bytes.
+ *   stream : cudaStream_t.
+ * Returns MOSA_OK, MOSA_ERR_INVALID_ARG, MOSA_ERR_UNSUPPORTED,
+ * MOSA_ERR_WORKSPACE or MOSA_ERR_CUDA. */
+mosa_status mosa_forward(const mosa_shape *shape, const void *X, const void *W_r,
+                         const void *W_q, const void *W_k, const void *W_v, const void *W_o,
+                         float *Y, int32_t *I, float *r_sel, float *r_full, void *workspace,
+                         size_t workspace_bytes, void *stream);
+
+/* Forward pass with caller-chosen token sets (no router, no TopK): the
+ * fixed-sparse special case of Sec. 3.1 (I = [0, rho, 2rho, ...], r = 1) and
+ * any other externally routed variant.
+ *   I     : [B,H,k] int32 input, strictly ascending and in [0,T) per row.
+ *           Rows breaking this are replaced by 0..k-1 and flagged in the
+ *           status word (MOSA_ERR_INVALID_ARG from mosa_check_status).
+ *   r_sel : [B,H,k] fp32 input scores applied as diag(r_sel).
+ *   Y     : [B,T,d] fp32 output.
+ * W_r is not read.  The workspace afterwards holds the state mosa_backward
+ * needs, but the router gradient it then reports assumes r_sel =
+ * sigmoid(X W_r)[I]. */
+mosa_status mosa_forward_with_indices(const mosa_shape *shape, const void *X,
+                                      const void *W_q, const void *W_k, const void *W_v,
+                                      const void *W_o, const int32_t *I, const float *r_sel,
+                                      float *Y, void *workspace, size_t workspace_bytes,
+                                      void *stream);
+
+/* Backward pass: gradients of <Y, dY> with the token sets held constant
+ * (TopK is not differentiated; the router learns through the diag(r^topk)
+ * scaling only, Sec. 2.2).  Must follow a mosa_forward (or
+ * mosa_forward_with_indices) on the same stream, with the same shape, inputs
+ * and workspace; I and r_sel are that call's outputs.
+ *   dY : [B,T,d] upstream gradient (storage dtype).
+ *   dX [B,T,d], dW_r [d,H], dW_q/dW_k/dW_v [H,d,hp], dW_o [H,hp,d] : fp32 outputs.
+ * Returns as mosa_forward. */
+mosa_status mosa_backward(const mosa_shape *shape, const void *X, const void *W_r,
+                          const void *W_q, const void *W_k, const void *W_v, const void *W_o,
+                          const int32_t *I, const float *r_sel, const void *dY, float *dX,
+                          float *dW_r, float *dW_q, float *dW_k, float *dW_v, float *dW_o,
+                          void *workspace, size_t workspace_bytes, void *stream);
+
+/* TopK alone (Sec. 2.2): for each of `rows` rows of T fp32 scores, the k
+ * largest (ties: lower index first), written ascending by index.
+ *   scores [rows,T] fp32 input; I [rows,k] int32 and r_sel [rows,k] fp32 outputs.
+ * Needs no workspace.  1 <= k <= T <= 65536.  Scores must not be NaN. */
+mosa_status mosa_topk(int32_t rows, int32_t T, int32_t k, const float *scores, int32_t *I,
+                      float *r_sel, void *stream);
+
+/* Waits for `stream`, then reads and clears the device status word in the
+ * workspace: MOSA_OK, MOSA_ERR_INVALID_ARG (caller indices were invalid) or
+ * MOSA_ERR_DEVICE_TIMEOUT; MOSA_ERR_CUDA if the wait itself failed. */
+mosa_status mosa_check_status(const mosa_shape *shape, void *workspace, void *stream);
+
+
+/* ---- Measurement support (not part of the layer) ----------------------
+ * Stages, in launch order: 0 router, 1 select, 2 qkv, 3 attn_fwd, 4 out,
+ * 5 out_bwd, 6 attn_bwd, 7 in_bwd, 8 w_bwd (9 reserved).  These calls create
+ * CUDA events (host-side handles, no device memory) when stage timing is on. */
+
+/* Number of kernels this library has launched since it was loaded. */
+unsigned long long mosa_kernel_launches(void);
+
+/* Turns CUDA-event timing on for the stages whose bit is set in stage_mask
+ * (0 turns it off).  Each timed stage of later calls records an event pair on
+ * the call's stream.  Always MOSA_OK. */
+mosa_status mosa_profile_stages(uint32_t stage_mask);
+
+/* Waits for the recorded events, writes per stage the summed elapsed
+ * milliseconds and the number of timed launches (arrays of max_stages
+ * entries, either may be NULL), resets the sums and returns the number of
+ * stages the library has. */
+int32_t mosa_profile_read(double *total_ms, int32_t *count, int32_t max_stages);
+
+/* Name of a stage ("router", "select", ...; "unknown" if out of range). */
+const char *mosa_stage_name(int32_t stage);
+
+#ifdef __cplusplus
+}
+#endif
+#endif /* MOSA_H_ */

@@ -228,16 +228,19 @@ int oracle_forward_indices(int B, int T, int d, int H, int hp, int k, const doub
     if (B <= 0 || T <= 0 || d <= 0 || H <= 0 || hp <= 0 || k <= 0 || k > T) return -1;
     memset(Y, 0, sizeof(double) * (size_t)B * T * d);
     int failed = 0;
-    #pragma omp parallel for schedule(dynamic, 1) reduction(| : failed)
-    for (int b = 0; b < B; ++b) {
-        if (!selected(bsel, b)) continue;
-        head_state s;
-        if (head_state_alloc(&s, k, d, hp) != 0) { head_state_free(&s); failed |= 1; continue; }
-        double *rs = (double *)malloc(sizeof(double) * (size_t)k);
-        const double *Xb = X + IDX3(b, 0, 0, T, d);
-        double *Yb = Y + IDX3(b, 0, 0, T, d);
+    /* Units (b,h) run in parallel; rows of Y shared between heads are
+     * updated atomically. */
+    #pragma omp parallel for collapse(2) schedule(dynamic, 1) reduction(| : failed)
+    for (int b = 0; b < B; ++b)
         for (int h = 0; h < H; ++h) {
-            if (!selected(hsel, h)) continue;
+            if (!selected(bsel, b) || !selected(hsel, h)) continue;
+            head_state s;
+            double *rs = (double *)malloc(sizeof(double) * (size_t)k);
+            if (head_state_alloc(&s, k, d, hp) != 0 || !rs) {
+                head_state_free(&s); free(rs); failed |= 1; continue;
+            }
+            const double *Xb = X + IDX3(b, 0, 0, T, d);
+            double *Yb = Y + IDX3(b, 0, 0, T, d);
             const int32_t *Ibh = I + IDX3(b, h, 0, H, k);
             for (int i = 0; i < k; ++i) {
                 if (r_sel_in) {
@@ -252,12 +255,13 @@ int oracle_forward_indices(int B, int T, int d, int H, int hp, int k, const doub
                          Wv + IDX3(h, 0, 0, d, hp), Wo + IDX3(h, 0, 0, hp, d));
             /* X^o = diag(r^topk) A W^o;  Y_{I_i} += X^o_i  (Eq. mosa_mha sums the heads) */
             for (int i = 0; i < k; ++i)
-                for (int c = 0; c < d; ++c)
+                for (int c = 0; c < d; ++c) {
+                    #pragma omp atomic
                     Yb[IDX2(Ibh[i], c, d)] += rs[i] * s.AWo[IDX2(i, c, d)];
+                }
+            free(rs);
+            head_state_free(&s);
         }
-        free(rs);
-        head_state_free(&s);
-    }
     return failed ? -1 : 0;
 }
 
@@ -321,11 +325,12 @@ int oracle_backward(int B, int T, int d, int H, int hp, int k, const double *X,
     memset(dWo, 0, sizeof(double) * (size_t)H * hp * d);
     const double scale = 1.0 / sqrt((double)hp);
     int failed = 0;
-    /* Heads run in parallel: each head owns its weight gradients; dX rows are
-     * shared between heads and updated atomically. */
-    #pragma omp parallel for schedule(dynamic, 1) reduction(| : failed)
-    for (int h = 0; h < H; ++h) {
-        if (!selected(hsel, h)) continue;
+    /* Units (h,b) run in parallel; every shared accumulation (rows of dX,
+     * weight gradients) is an atomic add. */
+    #pragma omp parallel for collapse(2) schedule(dynamic, 1) reduction(| : failed)
+    for (int h = 0; h < H; ++h)
+    for (int b = 0; b < B; ++b) {
+        if (!selected(hsel, h) || !selected(bsel, b)) continue;
         head_state s;
         if (head_state_alloc(&s, k, d, hp) != 0) { head_state_free(&s); failed |= 1; continue; }
         double *rs = (double *)malloc(sizeof(double) * (size_t)k);
@@ -342,8 +347,7 @@ int oracle_backward(int B, int T, int d, int H, int hp, int k, const double *X,
         const double *Wv_h = Wv + IDX3(h, 0, 0, d, hp), *Wo_h = Wo + IDX3(h, 0, 0, hp, d);
         double *dWq_h = dWq + IDX3(h, 0, 0, d, hp), *dWk_h = dWk + IDX3(h, 0, 0, d, hp);
         double *dWv_h = dWv + IDX3(h, 0, 0, d, hp), *dWo_h = dWo + IDX3(h, 0, 0, hp, d);
-        for (int b = 0; b < B && !failed; ++b) {
-            if (!selected(bsel, b)) continue;
+        if (!failed) {
             const double *Xb = X + IDX3(b, 0, 0, T, d);
             const double *dYb = dY + IDX3(b, 0, 0, T, d);
             double *dXb = dX + IDX3(b, 0, 0, T, d);
@@ -369,6 +373,7 @@ int oracle_backward(int B, int T, int d, int H, int hp, int k, const double *X,
                     double acc = 0.0;
                     for (int i = 0; i < k; ++i)
                         acc += rs[i] * s.A[IDX2(i, p, hp)] * dXo[IDX2(i, c, d)];
+                    #pragma omp atomic
                     dWo_h[IDX2(p, c, d)] += acc;
                 }
             /* dA = diag(r) dX^o W^o^T */
@@ -420,12 +425,16 @@ int oracle_backward(int B, int T, int d, int H, int hp, int k, const double *X,
                         ak += x * dK[IDX2(i, p, hp)];
                         av += x * dV[IDX2(i, p, hp)];
                     }
+                    #pragma omp atomic
                     dWq_h[IDX2(c, p, hp)] += aq;
+                    #pragma omp atomic
                     dWk_h[IDX2(c, p, hp)] += ak;
+                    #pragma omp atomic
                     dWv_h[IDX2(c, p, hp)] += av;
                 }
                 double ar = 0.0;
                 for (int i = 0; i < k; ++i) ar += s.Xs[IDX2(i, c, d)] * dlogit[i];
+                #pragma omp atomic
                 dWr[IDX2(c, h, H)] += ar;
             }
             /* dX[I] += dQ W^Q^T + dK W^K^T + dV W^V^T + dlogit W^r[:,h]^T */

@@ -1,0 +1,21 @@
+"""GB300-native Mixture-of-Sparse-Attention (MoSA) layer, arXiv 2505.00315.
+
+The layer runs in libmosa.so (hand-written CUDA for sm_103a behind the C ABI
+of include/mosa.h).  This package holds the thin Python binding with the
+same call names, the seeded synthetic workloads and the FLOP model.  The
+binding is imported lazily so that ``workloads`` and ``flops`` work on a
+machine without a GPU.
+"""
+from __future__ import annotations
+
+__all__ = ["mosa_forward", "mosa_forward_with_indices", "mosa_backward", "mosa_topk",
+           "mosa_workspace_bytes", "mosa_check_status", "alloc_workspace", "make_shape",
+           "MosaShape", "MosaError", "load", "mosa_kernel_launches", "mosa_profile_stages",
+           "mosa_profile_read", "mosa_stage_name"]
+
+
+def __getattr__(name):
+    if name in __all__:
+        from . import _binding
+        return getattr(_binding, name)
+    raise AttributeError(name)

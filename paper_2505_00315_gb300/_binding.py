@@ -1,0 +1,289 @@
+"""ctypes binding of libmosa (include/mosa.h).
+
+Argument marshalling only: every step of the layer runs in the library's
+CUDA kernels.  Torch supplies device memory and the current stream.  There
+is no fallback: if the library cannot be built or loaded, or no CUDA device
+is present, the calls raise.
+"""
+from __future__ import annotations
+
+import ctypes
+import os
+import threading
+
+from . import build as _build
+
+MOSA_OK = 0
+MOSA_ERR_INVALID_ARG = 1
+MOSA_ERR_UNSUPPORTED = 2
+MOSA_ERR_CUDA = 3
+MOSA_ERR_DEVICE_TIMEOUT = 4
+MOSA_ERR_WORKSPACE = 5
+MOSA_F32 = 0
+MOSA_BF16 = 1
+
+#: Every function include/mosa.h declares.
+EXPORTED = ("mosa_status_string", "mosa_workspace_bytes", "mosa_forward",
+            "mosa_forward_with_indices", "mosa_backward", "mosa_topk", "mosa_check_status",
+            "mosa_kernel_launches", "mosa_profile_stages", "mosa_profile_read",
+            "mosa_stage_name")
+
+
+class MosaShape(ctypes.Structure):
+    """mosa_shape: B sequences of T tokens of width d, H heads of size hp, k
+    tokens per head, storage dtype (MOSA_F32 or MOSA_BF16)."""
+    _fields_ = [("B", ctypes.c_int32), ("T", ctypes.c_int32), ("d", ctypes.c_int32),
+                ("H", ctypes.c_int32), ("hp", ctypes.c_int32), ("k", ctypes.c_int32),
+                ("dtype", ctypes.c_int32)]
+
+    def astuple(self):
+        return (self.B, self.T, self.d, self.H, self.hp, self.k, self.dtype)
+
+
+class MosaError(RuntimeError):
+    def __init__(self, code: int, where: str):
+        self.code = code
+        super().__init__(f"{where}: {status_string(code)}")
+
+
+_lock = threading.Lock()
+_lib = None
+
+
+def lib_path() -> str:
+    return _build.LIB
+
+
+def load(build_if_missing: bool = True) -> ctypes.CDLL:
+    """Load libmosa.so (building it first if needed) and declare signatures."""
+    global _lib
+    with _lock:
+        if _lib is not None:
+            return _lib
+        path = _build.build() if build_if_missing else _build.LIB
+        if not os.path.exists(path):
+            raise RuntimeError(f"libmosa is not built ({path}); run paper_2505_00315_gb300.build")
+        L = ctypes.CDLL(path)
+        vp, sz, i32 = ctypes.c_void_p, ctypes.c_size_t, ctypes.c_int32
+        sp = ctypes.POINTER(MosaShape)
+        L.mosa_status_string.argtypes = [ctypes.c_int]
+        L.mosa_status_string.restype = ctypes.c_char_p
+        L.mosa_workspace_bytes.argtypes = [sp]
+        L.mosa_workspace_bytes.restype = sz
+        L.mosa_forward.argtypes = [sp] + [vp] * 6 + [vp] * 4 + [vp, sz, vp]
+        L.mosa_forward.restype = ctypes.c_int
+        L.mosa_forward_with_indices.argtypes = [sp] + [vp] * 5 + [vp, vp, vp] + [vp, sz, vp]
+        L.mosa_forward_with_indices.restype = ctypes.c_int
+        L.mosa_backward.argtypes = [sp] + [vp] * 6 + [vp, vp, vp] + [vp] * 6 + [vp, sz, vp]
+        L.mosa_backward.restype = ctypes.c_int
+        L.mosa_topk.argtypes = [i32, i32, i32, vp, vp, vp, vp]
+        L.mosa_topk.restype = ctypes.c_int
+        L.mosa_check_status.argtypes = [sp, vp, vp]
+        L.mosa_check_status.restype = ctypes.c_int
+        L.mosa_kernel_launches.argtypes = []
+        L.mosa_kernel_launches.restype = ctypes.c_ulonglong
+        L.mosa_profile_stages.argtypes = [ctypes.c_uint32]
+        L.mosa_profile_stages.restype = ctypes.c_int
+        L.mosa_profile_read.argtypes = [ctypes.POINTER(ctypes.c_double),
+                                        ctypes.POINTER(ctypes.c_int32), i32]
+        L.mosa_profile_read.restype = i32
+        L.mosa_stage_name.argtypes = [i32]
+        L.mosa_stage_name.restype = ctypes.c_char_p
+        _lib = L
+        return L
+
+
+def status_string(code: int) -> str:
+    return load().mosa_status_string(int(code)).decode()
+
+
+def _check(code: int, where: str) -> None:
+    if code != MOSA_OK:
+        raise MosaError(code, where)
+
+
+# ---------------------------------------------------------------- torch glue
+
+def _torch():
+    import torch
+    return torch
+
+
+def _dtype_code(t) -> int:
+    torch = _torch()
+    if t.dtype == torch.float32:
+        return MOSA_F32
+    if t.dtype == torch.bfloat16:
+        return MOSA_BF16
+    raise TypeError(f"unsupported storage dtype {t.dtype} (float32 or bfloat16)")
+
+
+def _dev(t, name: str, dtype=None):
+    torch = _torch()
+    if not isinstance(t, torch.Tensor):
+        raise TypeError(f"{name} must be a torch.Tensor")
+    if not t.is_cuda:
+        raise ValueError(f"{name} must be a CUDA tensor (libmosa runs on the GPU only)")
+    if dtype is not None and t.dtype != dtype:
+        raise TypeError(f"{name} must be {dtype}, got {t.dtype}")
+    if not t.is_contiguous():
+        raise ValueError(f"{name} must be contiguous")
+    return ctypes.c_void_p(t.data_ptr())
+
+
+def _stream(stream):
+    torch = _torch()
+    s = torch.cuda.current_stream() if stream is None else stream
+    return ctypes.c_void_p(s.cuda_stream)
+
+
+def make_shape(X, W_q, k: int) -> MosaShape:
+    B, T, d = X.shape
+    H, d2, hp = W_q.shape
+    if d2 != d:
+        raise ValueError("W_q must be [H, d, hp] with the d of X")
+    return MosaShape(B, T, d, H, hp, int(k), _dtype_code(X))
+
+
+def mosa_workspace_bytes(shape: MosaShape) -> int:
+    return int(load().mosa_workspace_bytes(ctypes.byref(shape)))
+
+
+def alloc_workspace(shape: MosaShape, device=None):
+    """A torch uint8 device buffer of mosa_workspace_bytes(shape) bytes."""
+    torch = _torch()
+    n = mosa_workspace_bytes(shape)
+    if n == 0:
+        raise MosaError(MOSA_ERR_INVALID_ARG, "mosa_workspace_bytes")
+    return torch.empty(n, dtype=torch.uint8, device=device or "cuda")
+
+
+def _same(ref, *ts):
+    for name, t in ts:
+        if t.dtype != ref.dtype:
+            raise TypeError(f"{name} must have the storage dtype {ref.dtype}")
+
+
+def mosa_forward(X, W_r, W_q, W_k, W_v, W_o, k: int, workspace=None, want_r_full=False,
+                 out=None, stream=None):
+    """Forward pass (Sec. 2.2).  Returns (Y, I, r_sel, r_full or None, workspace).
+
+    ``out`` may hold preallocated "Y", "I", "r_sel" (and "r_full") tensors."""
+    torch = _torch()
+    shape = make_shape(X, W_q, k)
+    _same(X, ("W_r", W_r), ("W_q", W_q), ("W_k", W_k), ("W_v", W_v), ("W_o", W_o))
+    B, T, d, H = shape.B, shape.T, shape.d, shape.H
+    dev = X.device
+    out = out or {}
+    Y = out.get("Y") if out.get("Y") is not None else torch.empty((B, T, d), dtype=torch.float32, device=dev)
+    I = out.get("I") if out.get("I") is not None else torch.empty((B, H, k), dtype=torch.int32, device=dev)
+    rs = out.get("r_sel") if out.get("r_sel") is not None else torch.empty((B, H, k), dtype=torch.float32, device=dev)
+    rf = None
+    if want_r_full:
+        rf = out.get("r_full") if out.get("r_full") is not None else torch.empty((B, H, T), dtype=torch.float32, device=dev)
+    if workspace is None:
+        workspace = alloc_workspace(shape, dev)
+    rc = load().mosa_forward(ctypes.byref(shape), _dev(X, "X"), _dev(W_r, "W_r"), _dev(W_q, "W_q"),
+                             _dev(W_k, "W_k"), _dev(W_v, "W_v"), _dev(W_o, "W_o"),
+                             _dev(Y, "Y", torch.float32), _dev(I, "I", torch.int32),
+                             _dev(rs, "r_sel", torch.float32),
+                             None if rf is None else _dev(rf, "r_full", torch.float32),
+                             _dev(workspace, "workspace"), workspace.numel(), _stream(stream))
+    _check(rc, "mosa_forward")
+    return Y, I, rs, rf, workspace
+
+
+def mosa_forward_with_indices(X, W_q, W_k, W_v, W_o, I, r_sel, workspace=None, out=None,
+                              stream=None):
+    """Forward with caller-chosen token sets (e.g. the fixed-sparse case of
+    Sec. 3.1).  Returns (Y, workspace)."""
+    torch = _torch()
+    shape = make_shape(X, W_q, I.shape[-1])
+    _same(X, ("W_q", W_q), ("W_k", W_k), ("W_v", W_v), ("W_o", W_o))
+    B, T, d = shape.B, shape.T, shape.d
+    Y = (out or {}).get("Y")
+    if Y is None:
+        Y = torch.empty((B, T, d), dtype=torch.float32, device=X.device)
+    if workspace is None:
+        workspace = alloc_workspace(shape, X.device)
+    rc = load().mosa_forward_with_indices(
+        ctypes.byref(shape), _dev(X, "X"), _dev(W_q, "W_q"), _dev(W_k, "W_k"), _dev(W_v, "W_v"),
+        _dev(W_o, "W_o"), _dev(I, "I", torch.int32), _dev(r_sel, "r_sel", torch.float32),
+        _dev(Y, "Y", torch.float32), _dev(workspace, "workspace"), workspace.numel(),
+        _stream(stream))
+    _check(rc, "mosa_forward_with_indices")
+    return Y, workspace
+
+
+def mosa_backward(X, W_r, W_q, W_k, W_v, W_o, I, r_sel, dY, workspace, out=None, stream=None):
+    """Backward pass; returns a dict with dX, dW_r, dW_q, dW_k, dW_v, dW_o (fp32)."""
+    torch = _torch()
+    shape = make_shape(X, W_q, I.shape[-1])
+    _same(X, ("W_r", W_r), ("W_q", W_q), ("W_k", W_k), ("W_v", W_v), ("W_o", W_o), ("dY", dY))
+    dev = X.device
+    g = dict(out or {})
+    f32 = torch.float32
+    for name, like in (("dX", X), ("dW_r", W_r), ("dW_q", W_q), ("dW_k", W_k), ("dW_v", W_v),
+                       ("dW_o", W_o)):
+        if g.get(name) is None:
+            g[name] = torch.empty(like.shape, dtype=f32, device=dev)
+    rc = load().mosa_backward(
+        ctypes.byref(shape), _dev(X, "X"), _dev(W_r, "W_r"), _dev(W_q, "W_q"), _dev(W_k, "W_k"),
+        _dev(W_v, "W_v"), _dev(W_o, "W_o"), _dev(I, "I", torch.int32),
+        _dev(r_sel, "r_sel", f32), _dev(dY, "dY"), _dev(g["dX"], "dX", f32),
+        _dev(g["dW_r"], "dW_r", f32), _dev(g["dW_q"], "dW_q", f32), _dev(g["dW_k"], "dW_k", f32),
+        _dev(g["dW_v"], "dW_v", f32), _dev(g["dW_o"], "dW_o", f32),
+        _dev(workspace, "workspace"), workspace.numel(), _stream(stream))
+    _check(rc, "mosa_backward")
+    return g
+
+
+def mosa_topk(scores, k: int, out=None, stream=None):
+    """TopK alone over the last dim of fp32 ``scores`` [..., T]; returns (I, r_sel)."""
+    torch = _torch()
+    T = scores.shape[-1]
+    rows = scores.numel() // T if T else 0
+    lead = tuple(scores.shape[:-1])
+    I = (out or {}).get("I")
+    rs = (out or {}).get("r_sel")
+    if I is None:
+        I = torch.empty(lead + (k,), dtype=torch.int32, device=scores.device)
+    if rs is None:
+        rs = torch.empty(lead + (k,), dtype=torch.float32, device=scores.device)
+    rc = load().mosa_topk(rows, T, int(k), _dev(scores, "scores", torch.float32),
+                          _dev(I, "I", torch.int32), _dev(rs, "r_sel", torch.float32),
+                          _stream(stream))
+    _check(rc, "mosa_topk")
+    return I, rs
+
+
+def mosa_check_status(shape: MosaShape, workspace, stream=None) -> int:
+    """Synchronizes the stream, returns and clears the device status code."""
+    return int(load().mosa_check_status(ctypes.byref(shape), _dev(workspace, "workspace"),
+                                        _stream(stream)))
+
+
+# ------------------------------------------------------------ measurement
+
+def mosa_kernel_launches() -> int:
+    """Kernels the library has launched since it was loaded."""
+    return int(load().mosa_kernel_launches())
+
+
+def mosa_profile_stages(mask: int) -> None:
+    """Turn CUDA-event timing on for the stages in ``mask`` (0 = off)."""
+    _check(load().mosa_profile_stages(int(mask)), "mosa_profile_stages")
+
+
+def mosa_stage_name(stage: int) -> str:
+    return load().mosa_stage_name(int(stage)).decode()
+
+
+def mosa_profile_read() -> dict:
+    """{stage name: (total ms, timed launches)} since the last read; resets."""
+    L = load()
+    n = 16
+    ms = (ctypes.c_double * n)()
+    cnt = (ctypes.c_int32 * n)()
+    m = L.mosa_profile_read(ms, cnt, n)
+    return {mosa_stage_name(i): (ms[i], cnt[i]) for i in range(min(m, n))}

@@ -1,0 +1,53 @@
+// Host-side launchers of the libmosa kernels (internal; the public C ABI is
+// include/mosa.h).  Every launcher enqueues its kernels on `stream` and
+// returns the launch status; none synchronizes.
+#pragma once
+
+#include "common.cuh"
+
+namespace mosa {
+
+// F1, Sec. 2.2 router: r_full[b,h,t] = sigmoid(X[b,t,:] . W_r[:,h]) in fp32.
+cudaError_t launch_router(const Dims &dm, const void *X, const void *Wr, float *r_full,
+                          cudaStream_t stream);
+
+// F2, Sec. 2.2 TopK: per row of T scores, the k largest (ties: lower index),
+// ascending.  If gidx != nullptr, row = b*H + h also writes the head-major
+// gather rows gidx[(h*B+b)*k + i] = b*T + I and rsel_hm likewise.
+cudaError_t launch_select(int rows, int T, int k, const float *scores, int32_t *I, float *rsel,
+                          int B, int H, int32_t *gidx, float *rsel_hm, cudaStream_t stream);
+
+// Caller-supplied I / r_sel -> head-major gather rows, validating each row
+// (in range, strictly ascending); invalid rows become 0..k-1 and set
+// kStatusBadIndex.
+cudaError_t launch_indices_to_rows(const Dims &dm, const int32_t *I, const float *rsel,
+                                   int32_t *gidx, float *rsel_hm, uint32_t *status,
+                                   cudaStream_t stream);
+
+// F3: Q, K, V = X[I] W_{q,k,v}[h].
+cudaError_t launch_qkv(const Dims &dm, const void *X, const void *Wq, const void *Wk,
+                       const void *Wv, const Saved &sv, cudaStream_t stream);
+
+// F4: A = softmax((QK^T + M)/sqrt(h')) V, AR = diag(r) A, lse.
+cudaError_t launch_attn_fwd(const Dims &dm, const Saved &sv, cudaStream_t stream);
+
+// F5: Y = 0; Y[b, I, :] += AR W_o[h] summed over heads.
+cudaError_t launch_out(const Dims &dm, const void *Wo, const Saved &sv, float *Y,
+                       cudaStream_t stream);
+
+// B1: G = dY[I] W_o^T, dr, dA = r G, dlogit, D; dW_o = AR^T dY[I].
+cudaError_t launch_out_bwd(const Dims &dm, const void *Wo, const void *dY, const Saved &sv,
+                           float *dWo, cudaStream_t stream);
+
+// B2: dQ, dK, dV from dA (flash-style recomputation of P).
+cudaError_t launch_attn_bwd(const Dims &dm, const Saved &sv, cudaStream_t stream);
+
+// B3: dX = 0; dX[b, I, :] += dQ W_q^T + dK W_k^T + dV W_v^T + dlogit W_r[:,h]^T.
+cudaError_t launch_in_bwd(const Dims &dm, const void *Wq, const void *Wk, const void *Wv,
+                          const void *Wr, const Saved &sv, float *dX, cudaStream_t stream);
+
+// B4: dW_{q,k,v}[h] = X[I]^T d{Q,K,V};  dW_r[:,h] = X[I]^T dlogit.
+cudaError_t launch_w_bwd(const Dims &dm, const void *X, const Saved &sv, float *dWq,
+                         float *dWk, float *dWv, float *dWr, cudaStream_t stream);
+
+}  // namespace mosa

@@ -1,0 +1,229 @@
+// C ABI of libmosa (declared in include/mosa.h): argument validation,
+// workspace carving and the launch sequence of the forward and backward
+// passes of the MoSA layer (Sec. 2.2, Eq. mosa_mha).
+#include <cstring>
+
+#include "../../include/mosa.h"
+#include "launch.h"
+#include "profile.h"
+
+namespace mosa {
+namespace {
+
+constexpr size_t kAlign = 256;
+
+size_t align_up(size_t x) { return (x + kAlign - 1) / kAlign * kAlign; }
+
+// Validation shared by every entry point: MOSA_OK, INVALID_ARG or UNSUPPORTED.
+mosa_status check_shape(const mosa_shape *s, Dims *out) {
+    if (s == nullptr) return MOSA_ERR_INVALID_ARG;
+    if (s->B <= 0 || s->T <= 0 || s->d <= 0 || s->H <= 0 || s->hp <= 0 || s->k <= 0)
+        return MOSA_ERR_INVALID_ARG;
+    if (s->k > s->T) return MOSA_ERR_INVALID_ARG;
+    if (s->dtype != MOSA_F32 && s->dtype != MOSA_BF16) return MOSA_ERR_INVALID_ARG;
+    const long long lim = 1LL << 31;
+    if ((long long)s->B * s->T * s->d >= lim) return MOSA_ERR_UNSUPPORTED;
+    if ((long long)s->H * s->d * s->hp >= lim) return MOSA_ERR_UNSUPPORTED;
+    if ((long long)s->B * s->H * s->T >= lim) return MOSA_ERR_UNSUPPORTED;
+    if ((long long)s->B * s->H * s->k * 3 * s->hp >= lim) return MOSA_ERR_UNSUPPORTED;
+    if (s->T > 65536) return MOSA_ERR_UNSUPPORTED;
+    if (s->H > 65535) return MOSA_ERR_UNSUPPORTED;
+    if (s->d % 8 != 0) return MOSA_ERR_UNSUPPORTED;
+    if (s->hp != 16 && s->hp != 32 && s->hp != 64 && s->hp != 128) return MOSA_ERR_UNSUPPORTED;
+    if (out) *out = Dims{s->B, s->T, s->d, s->H, s->hp, s->k, s->dtype == MOSA_BF16};
+    return MOSA_OK;
+}
+
+// Carves the workspace; returns the bytes needed (and fills *sv if base != nullptr).
+size_t carve(const Dims &dm, char *base, Saved *sv) {
+    size_t off = 0;
+    auto take = [&](size_t bytes) -> char * {
+        char *p = base ? base + off : nullptr;
+        off += align_up(bytes);
+        return p;
+    };
+    const size_t R = (size_t)dm.rows();
+    const size_t e = dm.esize();
+    Saved s{};
+    s.status = (uint32_t *)take(sizeof(uint32_t));
+    s.r_full = (float *)take(sizeof(float) * (size_t)dm.B * dm.H * dm.T);
+    s.gidx = (int32_t *)take(sizeof(int32_t) * R);
+    s.rsel = (float *)take(sizeof(float) * R);
+    s.Q = take(e * R * dm.hp);
+    s.K = take(e * R * dm.hp);
+    s.V = take(e * R * dm.hp);
+    s.A = take(e * R * dm.hp);
+    s.AR = take(e * R * dm.hp);
+    s.lse = (float *)take(sizeof(float) * R);
+    s.dA = take(e * R * dm.hp);
+    s.dlogit = (float *)take(sizeof(float) * R);
+    s.Dd = (float *)take(sizeof(float) * R);
+    s.dQKV = take(e * R * 3 * dm.hp);
+    s.G = (float *)take(sizeof(float) * R * dm.hp);
+    if (sv) *sv = s;
+    return off;
+}
+
+mosa_status check_workspace(const Dims &dm, void *ws, size_t bytes, Saved *sv) {
+    if (ws == nullptr || ((uintptr_t)ws % kAlign) != 0) return MOSA_ERR_WORKSPACE;
+    if (bytes < carve(dm, nullptr, nullptr)) return MOSA_ERR_WORKSPACE;
+    carve(dm, (char *)ws, sv);
+    return MOSA_OK;
+}
+
+mosa_status cuda_status(cudaError_t e) { return e == cudaSuccess ? MOSA_OK : MOSA_ERR_CUDA; }
+
+#define MOSA_TRY(expr)                                  \
+    do {                                                \
+        cudaError_t _e = (expr);                        \
+        if (_e != cudaSuccess) return MOSA_ERR_CUDA;    \
+    } while (0)
+
+// F3-F5 for the rows already selected into sv.gidx / sv.rsel.
+mosa_status forward_heads(const Dims &dm, const void *X, const void *W_q, const void *W_k,
+                          const void *W_v, const void *W_o, float *Y, const Saved &sv,
+                          cudaStream_t s) {
+    {
+        StageScope st_(kStageQkv, s);
+        MOSA_TRY(launch_qkv(dm, X, W_q, W_k, W_v, sv, s));
+    }
+    {
+        StageScope st_(kStageAttnFwd, s);
+        MOSA_TRY(launch_attn_fwd(dm, sv, s));
+    }
+    {
+        StageScope st_(kStageOut, s);
+        MOSA_TRY(launch_out(dm, W_o, sv, Y, s));
+    }
+    return MOSA_OK;
+}
+
+}  // namespace
+}  // namespace mosa
+
+using namespace mosa;
+
+extern "C" {
+
+const char *mosa_status_string(mosa_status s) {
+    switch (s) {
+        case MOSA_OK: return "MOSA_OK";
+        case MOSA_ERR_INVALID_ARG: return "MOSA_ERR_INVALID_ARG: invalid argument";
+        case MOSA_ERR_UNSUPPORTED: return "MOSA_ERR_UNSUPPORTED: shape outside the supported set";
+        case MOSA_ERR_CUDA: return "MOSA_ERR_CUDA: CUDA runtime error";
+        case MOSA_ERR_DEVICE_TIMEOUT: return "MOSA_ERR_DEVICE_TIMEOUT: a bounded device wait gave up";
+        case MOSA_ERR_WORKSPACE: return "MOSA_ERR_WORKSPACE: workspace missing, misaligned or too small";
+        default: return "unknown mosa_status";
+    }
+}
+
+size_t mosa_workspace_bytes(const mosa_shape *shape) {
+    Dims dm;
+    if (check_shape(shape, &dm) != MOSA_OK) return 0;
+    return carve(dm, nullptr, nullptr);
+}
+
+mosa_status mosa_forward(const mosa_shape *shape, const void *X, const void *W_r,
+                         const void *W_q, const void *W_k, const void *W_v, const void *W_o,
+                         float *Y, int32_t *I, float *r_sel, float *r_full, void *workspace,
+                         size_t workspace_bytes, void *stream) {
+    Dims dm;
+    mosa_status st = check_shape(shape, &dm);
+    if (st != MOSA_OK) return st;
+    if (!X || !W_r || !W_q || !W_k || !W_v || !W_o || !Y || !I || !r_sel)
+        return MOSA_ERR_INVALID_ARG;
+    Saved sv;
+    if ((st = check_workspace(dm, workspace, workspace_bytes, &sv)) != MOSA_OK) return st;
+    cudaStream_t s = (cudaStream_t)stream;
+    float *rf = r_full ? r_full : sv.r_full;
+    MOSA_TRY(cudaMemsetAsync(sv.status, 0, sizeof(uint32_t), s));
+    {
+        StageScope st_(kStageRouter, s);
+        MOSA_TRY(launch_router(dm, X, W_r, rf, s));
+    }
+    {
+        StageScope st_(kStageSelect, s);
+        MOSA_TRY(launch_select(dm.B * dm.H, dm.T, dm.k, rf, I, r_sel, dm.B, dm.H, sv.gidx,
+                               sv.rsel, s));
+    }
+    return forward_heads(dm, X, W_q, W_k, W_v, W_o, Y, sv, s);
+}
+
+mosa_status mosa_forward_with_indices(const mosa_shape *shape, const void *X, const void *W_q,
+                                      const void *W_k, const void *W_v, const void *W_o,
+                                      const int32_t *I, const float *r_sel, float *Y,
+                                      void *workspace, size_t workspace_bytes, void *stream) {
+    Dims dm;
+    mosa_status st = check_shape(shape, &dm);
+    if (st != MOSA_OK) return st;
+    if (!X || !W_q || !W_k || !W_v || !W_o || !I || !r_sel || !Y) return MOSA_ERR_INVALID_ARG;
+    Saved sv;
+    if ((st = check_workspace(dm, workspace, workspace_bytes, &sv)) != MOSA_OK) return st;
+    cudaStream_t s = (cudaStream_t)stream;
+    MOSA_TRY(cudaMemsetAsync(sv.status, 0, sizeof(uint32_t), s));
+    {
+        StageScope st_(kStageSelect, s);
+        MOSA_TRY(launch_indices_to_rows(dm, I, r_sel, sv.gidx, sv.rsel, sv.status, s));
+    }
+    return forward_heads(dm, X, W_q, W_k, W_v, W_o, Y, sv, s);
+}
+
+mosa_status mosa_backward(const mosa_shape *shape, const void *X, const void *W_r,
+                          const void *W_q, const void *W_k, const void *W_v, const void *W_o,
+                          const int32_t *I, const float *r_sel, const void *dY, float *dX,
+                          float *dW_r, float *dW_q, float *dW_k, float *dW_v, float *dW_o,
+                          void *workspace, size_t workspace_bytes, void *stream) {
+    Dims dm;
+    mosa_status st = check_shape(shape, &dm);
+    if (st != MOSA_OK) return st;
+    if (!X || !W_r || !W_q || !W_k || !W_v || !W_o || !I || !r_sel || !dY || !dX || !dW_r ||
+        !dW_q || !dW_k || !dW_v || !dW_o)
+        return MOSA_ERR_INVALID_ARG;
+    Saved sv;
+    if ((st = check_workspace(dm, workspace, workspace_bytes, &sv)) != MOSA_OK) return st;
+    cudaStream_t s = (cudaStream_t)stream;
+    {
+        StageScope st_(kStageOutBwd, s);
+        MOSA_TRY(launch_out_bwd(dm, W_o, dY, sv, dW_o, s));
+    }
+    {
+        StageScope st_(kStageAttnBwd, s);
+        MOSA_TRY(launch_attn_bwd(dm, sv, s));
+    }
+    {
+        StageScope st_(kStageInBwd, s);
+        MOSA_TRY(launch_in_bwd(dm, W_q, W_k, W_v, W_r, sv, dX, s));
+    }
+    {
+        StageScope st_(kStageWBwd, s);
+        MOSA_TRY(launch_w_bwd(dm, X, sv, dW_q, dW_k, dW_v, dW_r, s));
+    }
+    return MOSA_OK;
+}
+
+mosa_status mosa_topk(int32_t rows, int32_t T, int32_t k, const float *scores, int32_t *I,
+                      float *r_sel, void *stream) {
+    if (rows <= 0 || T <= 0 || k <= 0 || k > T) return MOSA_ERR_INVALID_ARG;
+    if (!scores || !I || !r_sel) return MOSA_ERR_INVALID_ARG;
+    if (T > 65536) return MOSA_ERR_UNSUPPORTED;
+    return cuda_status(launch_select(rows, T, k, scores, I, r_sel, 0, 1, nullptr, nullptr,
+                                     (cudaStream_t)stream));
+}
+
+mosa_status mosa_check_status(const mosa_shape *shape, void *workspace, void *stream) {
+    Dims dm;
+    mosa_status st = check_shape(shape, &dm);
+    if (st != MOSA_OK) return st;
+    if (workspace == nullptr || ((uintptr_t)workspace % kAlign) != 0) return MOSA_ERR_WORKSPACE;
+    cudaStream_t s = (cudaStream_t)stream;
+    uint32_t word = 0;
+    if (cudaStreamSynchronize(s) != cudaSuccess) return MOSA_ERR_CUDA;
+    if (cudaMemcpy(&word, workspace, sizeof(word), cudaMemcpyDeviceToHost) != cudaSuccess)
+        return MOSA_ERR_CUDA;
+    if (cudaMemset(workspace, 0, sizeof(word)) != cudaSuccess) return MOSA_ERR_CUDA;
+    if (word & kStatusTimeout) return MOSA_ERR_DEVICE_TIMEOUT;
+    if (word & kStatusBadIndex) return MOSA_ERR_INVALID_ARG;
+    return MOSA_OK;
+}
+
+}  // extern "C"

@@ -1,0 +1,103 @@
+// Measurement support for libmosa (not part of the layer's arithmetic): a
+// count of the kernels the library has launched, and optional CUDA-event
+// timing of individual stages on the stream they run on.
+#include <atomic>
+#include <mutex>
+#include <vector>
+
+#include "../../include/mosa.h"
+#include "profile.h"
+
+namespace mosa {
+namespace {
+
+std::atomic<unsigned long long> g_launches{0};
+std::atomic<uint32_t> g_mask{0};
+std::mutex g_mu;
+
+struct Pending {
+    int stage;
+    cudaEvent_t start, stop;
+};
+std::vector<Pending> g_pending;
+std::vector<cudaEvent_t> g_free;
+double g_ms[kNumStages] = {};
+int32_t g_count[kNumStages] = {};
+
+const char *kNames[kNumStages] = {"router", "select", "qkv", "attn_fwd", "out",
+                                  "out_bwd", "attn_bwd", "in_bwd", "w_bwd", "rows"};
+
+cudaEvent_t take_event() {
+    if (!g_free.empty()) {
+        cudaEvent_t e = g_free.back();
+        g_free.pop_back();
+        return e;
+    }
+    cudaEvent_t e = nullptr;
+    if (cudaEventCreate(&e) != cudaSuccess) return nullptr;
+    return e;
+}
+
+}  // namespace
+
+void note_launches(int n) { g_launches.fetch_add((unsigned long long)n, std::memory_order_relaxed); }
+
+StageScope::StageScope(int stage, cudaStream_t s) : stage_(stage), stream_(s) {
+    if (!(g_mask.load(std::memory_order_relaxed) & (1u << stage))) return;
+    std::lock_guard<std::mutex> lk(g_mu);
+    start_ = take_event();
+    stop_ = take_event();
+    if (start_ && stop_ && cudaEventRecord(start_, s) == cudaSuccess) {
+        active_ = true;
+    }
+}
+
+StageScope::~StageScope() {
+    if (!active_) return;
+    std::lock_guard<std::mutex> lk(g_mu);
+    if (cudaEventRecord(stop_, stream_) == cudaSuccess) g_pending.push_back({stage_, start_, stop_});
+}
+
+}  // namespace mosa
+
+using namespace mosa;
+
+extern "C" {
+
+unsigned long long mosa_kernel_launches(void) { return g_launches.load(); }
+
+mosa_status mosa_profile_stages(uint32_t stage_mask) {
+    g_mask.store(stage_mask & ((1u << kNumStages) - 1u));
+    return MOSA_OK;
+}
+
+int32_t mosa_profile_read(double *total_ms, int32_t *count, int32_t max_stages) {
+    std::lock_guard<std::mutex> lk(g_mu);
+    for (const Pending &p : g_pending) {
+        float ms = 0.f;
+        if (cudaEventSynchronize(p.stop) == cudaSuccess &&
+            cudaEventElapsedTime(&ms, p.start, p.stop) == cudaSuccess) {
+            g_ms[p.stage] += ms;
+            g_count[p.stage] += 1;
+        }
+        g_free.push_back(p.start);
+        g_free.push_back(p.stop);
+    }
+    g_pending.clear();
+    const int n = max_stages < kNumStages ? max_stages : kNumStages;
+    for (int i = 0; i < n; ++i) {
+        if (total_ms) total_ms[i] = g_ms[i];
+        if (count) count[i] = g_count[i];
+    }
+    for (int i = 0; i < kNumStages; ++i) {
+        g_ms[i] = 0.0;
+        g_count[i] = 0;
+    }
+    return kNumStages;
+}
+
+const char *mosa_stage_name(int32_t stage) {
+    return (stage >= 0 && stage < kNumStages) ? kNames[stage] : "unknown";
+}
+
+}  // extern "C"

@@ -1,0 +1,240 @@
+// Per-head projections of the MoSA layer on CUDA cores (fp32 FFMA), used for
+// fp32 storage and as the plain path for bf16:
+//   F3  Q, K, V = X^s W^{Q,K,V}           (X^s = X[b, I, :], Sec. 2.2)
+//   F5  Y[b, I, :] += diag(r^topk) A W^o  (scatter-sum over heads, Eq. mosa_mha)
+//   B1  G = dY[I] W^o^T, dW^o = (diag(r) A)^T dY[I], and the row terms
+//       dr = <A, G>, dA = r G, dlogit = dr r (1 - r), D = rowsum(dA o A)
+//   B3  dX[b, I, :] += dQ W^Q^T + dK W^K^T + dV W^V^T + dlogit W^r[:,h]^T
+//   B4  dW^{Q,K,V} = X^s^T d{Q,K,V},  dW^r[:,h] = X^s^T dlogit
+// Rows of head h are m = b*k + i; gidx maps them to rows of X / Y / dY.
+#include "launch.h"
+#include "simt_gemm.cuh"
+
+namespace mosa {
+namespace {
+
+template <class T>
+struct QkvOp {
+    static constexpr bool kAKFast = true, kBKFast = false;
+    int M, N, K;  // B*k, 3*hp, d
+    int hp;
+    const T *X, *Wq, *Wk, *Wv;
+    const int32_t *gidx;
+    T *Q, *Kp, *V;
+    __device__ float a(int g, int m, int c) const {
+        return to_f32(X[(size_t)gidx[(size_t)g * M + m] * K + c]);
+    }
+    __device__ float b(int g, int c, int n) const {
+        const int w = n / hp, p = n - w * hp;
+        const T *W = w == 0 ? Wq : (w == 1 ? Wk : Wv);
+        return to_f32(W[((size_t)g * K + c) * hp + p]);
+    }
+    __device__ void store(int g, int m, int n, float v) const {
+        const int w = n / hp, p = n - w * hp;
+        T *O = w == 0 ? Q : (w == 1 ? Kp : V);
+        O[((size_t)g * M + m) * hp + p] = from_f32<T>(v);
+    }
+};
+
+template <class T>
+struct OutOp {
+    static constexpr bool kAKFast = true, kBKFast = false;
+    int M, N, K;  // B*k, d, hp
+    const T *AR, *Wo;
+    const int32_t *gidx;
+    float *Y;
+    __device__ float a(int g, int m, int p) const { return to_f32(AR[((size_t)g * M + m) * K + p]); }
+    __device__ float b(int g, int p, int n) const { return to_f32(Wo[((size_t)g * K + p) * N + n]); }
+    __device__ void store(int g, int m, int n, float v) const {
+        atomicAdd(Y + (size_t)gidx[(size_t)g * M + m] * N + n, v);
+    }
+};
+
+template <class T>
+struct OutBwdGOp {
+    static constexpr bool kAKFast = true, kBKFast = true;
+    int M, N, K;  // B*k, hp, d
+    const T *dY, *Wo;
+    const int32_t *gidx;
+    float *G;
+    __device__ float a(int g, int m, int c) const {
+        return to_f32(dY[(size_t)gidx[(size_t)g * M + m] * K + c]);
+    }
+    __device__ float b(int g, int c, int n) const { return to_f32(Wo[((size_t)g * N + n) * K + c]); }
+    __device__ void store(int g, int m, int n, float v) const { G[((size_t)g * M + m) * N + n] = v; }
+};
+
+template <class T>
+struct OutBwdWOp {
+    static constexpr bool kAKFast = false, kBKFast = false;
+    int M, N, K;  // hp, d, B*k
+    const T *AR, *dY;
+    const int32_t *gidx;
+    float *dWo;
+    __device__ float a(int g, int p, int m) const { return to_f32(AR[((size_t)g * K + m) * M + p]); }
+    __device__ float b(int g, int m, int n) const {
+        return to_f32(dY[(size_t)gidx[(size_t)g * K + m] * N + n]);
+    }
+    __device__ void store(int g, int p, int n, float v) const { dWo[((size_t)g * M + p) * N + n] = v; }
+};
+
+template <class T>
+struct InBwdOp {
+    static constexpr bool kAKFast = true, kBKFast = true;
+    int M, N, K;  // B*k, d, 3*hp
+    int hp, H;
+    const T *dQKV, *Wq, *Wk, *Wv, *Wr;
+    const float *dlogit;
+    const int32_t *gidx;
+    float *dX;
+    __device__ float a(int g, int m, int kk) const { return to_f32(dQKV[((size_t)g * M + m) * K + kk]); }
+    __device__ float b(int g, int kk, int n) const {
+        const int w = kk / hp, p = kk - w * hp;
+        const T *W = w == 0 ? Wq : (w == 1 ? Wk : Wv);
+        return to_f32(W[((size_t)g * N + n) * hp + p]);
+    }
+    __device__ void store(int g, int m, int n, float v) const {
+        const size_t row = (size_t)g * M + m;
+        v = fmaf(dlogit[row], to_f32(Wr[(size_t)n * H + g]), v);
+        atomicAdd(dX + (size_t)gidx[row] * N + n, v);
+    }
+};
+
+// dW_{q,k,v} and, as one extra output column, dW_r.
+template <class T>
+struct WBwdOp {
+    static constexpr bool kAKFast = false, kBKFast = false;
+    int M, N, K;  // d, 3*hp + 1, B*k
+    int hp, H;
+    const T *X, *dQKV;
+    const float *dlogit;
+    const int32_t *gidx;
+    float *dWq, *dWk, *dWv, *dWr;
+    __device__ float a(int g, int c, int m) const {
+        return to_f32(X[(size_t)gidx[(size_t)g * K + m] * M + c]);
+    }
+    __device__ float b(int g, int m, int n) const {
+        const size_t row = (size_t)g * K + m;
+        return n < 3 * hp ? to_f32(dQKV[row * (3 * hp) + n]) : dlogit[row];
+    }
+    __device__ void store(int g, int c, int n, float v) const {
+        if (n == 3 * hp) {
+            dWr[(size_t)c * H + g] = v;
+            return;
+        }
+        const int w = n / hp, p = n - w * hp;
+        float *O = w == 0 ? dWq : (w == 1 ? dWk : dWv);
+        O[((size_t)g * M + c) * hp + p] = v;
+    }
+};
+
+// One warp per selected row: dr = <A, G>, dA = r G (rounded to storage),
+// D = rowsum(dA o A), dlogit = dr r (1 - r).
+template <class T>
+__global__ void out_bwd_rows_kernel(const float *__restrict__ G, const T *__restrict__ A,
+                                    const float *__restrict__ rsel, T *__restrict__ dA,
+                                    float *__restrict__ Dd, float *__restrict__ dlogit,
+                                    long long rows, int hp) {
+    const long long row = (long long)blockIdx.x * (blockDim.x / 32) + threadIdx.x / 32;
+    const int lane = threadIdx.x & 31;
+    if (row >= rows) return;
+    const float r = rsel[row];
+    float dr = 0.f, dd = 0.f;
+    for (int p = lane; p < hp; p += 32) {
+        const float g = G[row * hp + p];
+        const float a = to_f32(A[row * hp + p]);
+        dr = fmaf(a, g, dr);
+        const T da = from_f32<T>(r * g);
+        dA[row * hp + p] = da;
+        dd = fmaf(to_f32(da), a, dd);
+    }
+#pragma unroll
+    for (int off = 16; off > 0; off >>= 1) {
+        dr += __shfl_xor_sync(0xffffffffu, dr, off);
+        dd += __shfl_xor_sync(0xffffffffu, dd, off);
+    }
+    if (lane == 0) {
+        Dd[row] = dd;
+        dlogit[row] = dr * r * (1.f - r);
+    }
+}
+
+template <class T>
+cudaError_t qkv_t(const Dims &dm, const void *X, const void *Wq, const void *Wk, const void *Wv,
+                  const Saved &sv, cudaStream_t s) {
+    QkvOp<T> op{dm.B * dm.k, 3 * dm.hp, dm.d, dm.hp, (const T *)X, (const T *)Wq, (const T *)Wk,
+                (const T *)Wv, sv.gidx, (T *)sv.Q, (T *)sv.K, (T *)sv.V};
+    return launch_simt_gemm(op, dm.H, s);
+}
+
+template <class T>
+cudaError_t out_t(const Dims &dm, const void *Wo, const Saved &sv, float *Y, cudaStream_t s) {
+    cudaError_t e = cudaMemsetAsync(Y, 0, sizeof(float) * (size_t)dm.B * dm.T * dm.d, s);
+    if (e != cudaSuccess) return e;
+    OutOp<T> op{dm.B * dm.k, dm.d, dm.hp, (const T *)sv.AR, (const T *)Wo, sv.gidx, Y};
+    return launch_simt_gemm(op, dm.H, s);
+}
+
+template <class T>
+cudaError_t out_bwd_t(const Dims &dm, const void *Wo, const void *dY, const Saved &sv,
+                      float *dWo, cudaStream_t s) {
+    OutBwdGOp<T> g{dm.B * dm.k, dm.hp, dm.d, (const T *)dY, (const T *)Wo, sv.gidx, sv.G};
+    cudaError_t e = launch_simt_gemm(g, dm.H, s);
+    if (e != cudaSuccess) return e;
+    const long long rows = dm.rows();
+    const int warps = 8;
+    out_bwd_rows_kernel<T><<<(unsigned)((rows + warps - 1) / warps), warps * 32, 0, s>>>(
+        sv.G, (const T *)sv.A, sv.rsel, (T *)sv.dA, sv.Dd, sv.dlogit, rows, dm.hp);
+    note_launches(1);
+    if ((e = cudaGetLastError()) != cudaSuccess) return e;
+    OutBwdWOp<T> w{dm.hp, dm.d, dm.B * dm.k, (const T *)sv.AR, (const T *)dY, sv.gidx, dWo};
+    return launch_simt_gemm(w, dm.H, s);
+}
+
+template <class T>
+cudaError_t in_bwd_t(const Dims &dm, const void *Wq, const void *Wk, const void *Wv,
+                     const void *Wr, const Saved &sv, float *dX, cudaStream_t s) {
+    cudaError_t e = cudaMemsetAsync(dX, 0, sizeof(float) * (size_t)dm.B * dm.T * dm.d, s);
+    if (e != cudaSuccess) return e;
+    InBwdOp<T> op{dm.B * dm.k, dm.d, 3 * dm.hp, dm.hp, dm.H, (const T *)sv.dQKV, (const T *)Wq,
+                  (const T *)Wk, (const T *)Wv, (const T *)Wr, sv.dlogit, sv.gidx, dX};
+    return launch_simt_gemm(op, dm.H, s);
+}
+
+template <class T>
+cudaError_t w_bwd_t(const Dims &dm, const void *X, const Saved &sv, float *dWq, float *dWk,
+                    float *dWv, float *dWr, cudaStream_t s) {
+    WBwdOp<T> op{dm.d, 3 * dm.hp + 1, dm.B * dm.k, dm.hp, dm.H, (const T *)X,
+                 (const T *)sv.dQKV, sv.dlogit, sv.gidx, dWq, dWk, dWv, dWr};
+    return launch_simt_gemm(op, dm.H, s);
+}
+
+}  // namespace
+
+cudaError_t launch_qkv(const Dims &dm, const void *X, const void *Wq, const void *Wk,
+                       const void *Wv, const Saved &sv, cudaStream_t s) {
+    return dm.bf16 ? qkv_t<bf16>(dm, X, Wq, Wk, Wv, sv, s) : qkv_t<float>(dm, X, Wq, Wk, Wv, sv, s);
+}
+
+cudaError_t launch_out(const Dims &dm, const void *Wo, const Saved &sv, float *Y, cudaStream_t s) {
+    return dm.bf16 ? out_t<bf16>(dm, Wo, sv, Y, s) : out_t<float>(dm, Wo, sv, Y, s);
+}
+
+cudaError_t launch_out_bwd(const Dims &dm, const void *Wo, const void *dY, const Saved &sv,
+                           float *dWo, cudaStream_t s) {
+    return dm.bf16 ? out_bwd_t<bf16>(dm, Wo, dY, sv, dWo, s) : out_bwd_t<float>(dm, Wo, dY, sv, dWo, s);
+}
+
+cudaError_t launch_in_bwd(const Dims &dm, const void *Wq, const void *Wk, const void *Wv,
+                          const void *Wr, const Saved &sv, float *dX, cudaStream_t s) {
+    return dm.bf16 ? in_bwd_t<bf16>(dm, Wq, Wk, Wv, Wr, sv, dX, s)
+                   : in_bwd_t<float>(dm, Wq, Wk, Wv, Wr, sv, dX, s);
+}
+
+cudaError_t launch_w_bwd(const Dims &dm, const void *X, const Saved &sv, float *dWq, float *dWk,
+                         float *dWv, float *dWr, cudaStream_t s) {
+    return dm.bf16 ? w_bwd_t<bf16>(dm, X, sv, dWq, dWk, dWv, dWr, s)
+                   : w_bwd_t<float>(dm, X, sv, dWq, dWk, dWv, dWr, s);
+}
+
+}  // namespace mosa

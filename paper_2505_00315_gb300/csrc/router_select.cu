@@ -1,0 +1,215 @@
+// Router (F1) and TopK selection (F2) of the MoSA layer, Sec. 2.2:
+//   r = sigmoid(X W^r);   r^topk, I = TopK(r, k).
+//
+// The selection is a per-row radix select on an order-preserving uint32
+// image of the fp32 scores (4 passes of 8 bits, most significant first),
+// which finds the exact k-th largest key.  A final in-order compaction keeps
+// every key above it plus the lowest-index keys equal to it, so I comes out
+// ascending (the order the causal mask works in) and ties go to the lower
+// token index.  Block-wide ranks use warp ballots, so no sort is needed.
+#include "launch.h"
+#include "profile.h"
+#include "simt_gemm.cuh"
+
+namespace mosa {
+namespace {
+
+template <class E>
+struct RouterOp {
+    static constexpr bool kAKFast = true;   // X rows are contiguous along d
+    static constexpr bool kBKFast = false;  // W_r rows are contiguous along H
+    int M, N, K;                            // B*T tokens, H heads, d
+    int T, H;
+    const E *X, *Wr;
+    float *r_full;
+    __device__ float a(int, int m, int kk) const { return to_f32(X[(size_t)m * K + kk]); }
+    __device__ float b(int, int kk, int n) const { return to_f32(Wr[(size_t)kk * N + n]); }
+    __device__ void store(int, int m, int n, float logit) const {
+        const int bb = m / T, t = m % T;
+        r_full[((size_t)bb * H + n) * T + t] = 1.f / (1.f + expf(-logit));
+    }
+};
+
+// Order-preserving map of a non-NaN float to uint32 (-0 and +0 map together).
+__device__ __forceinline__ uint32_t order_key(float f) {
+    uint32_t u = __float_as_uint(f);
+    if (u == 0x80000000u) u = 0u;
+    return (u & 0x80000000u) ? ~u : (u | 0x80000000u);
+}
+
+constexpr int kSelThreads = 1024;
+
+// Exclusive rank of this thread among the block's threads with `flag` set,
+// in thread order; `total` receives the block-wide count.  sh has 33 words.
+__device__ __forceinline__ uint32_t block_rank(bool flag, uint32_t *sh, uint32_t &total) {
+    const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+    const int nwarps = blockDim.x >> 5;
+    const uint32_t ballot = __ballot_sync(0xffffffffu, flag);
+    if (lane == 0) sh[warp] = __popc(ballot);
+    __syncthreads();
+    if (warp == 0) {
+        const uint32_t v = lane < nwarps ? sh[lane] : 0u;
+        uint32_t incl = v;
+#pragma unroll
+        for (int off = 1; off < 32; off <<= 1) {
+            const uint32_t y = __shfl_up_sync(0xffffffffu, incl, off);
+            if (lane >= off) incl += y;
+        }
+        sh[lane] = incl - v;
+        if (lane == 31) sh[32] = incl;
+    }
+    __syncthreads();
+    const uint32_t r = sh[warp] + __popc(ballot & ((1u << lane) - 1u));
+    total = sh[32];
+    __syncthreads();
+    return r;
+}
+
+__global__ void __launch_bounds__(kSelThreads)
+topk_select_kernel(const float *__restrict__ scores, int T, int k, int32_t *__restrict__ I,
+                   float *__restrict__ rsel, int B, int H, int32_t *__restrict__ gidx,
+                   float *__restrict__ rsel_hm) {
+    __shared__ uint32_t hist[256];
+    __shared__ uint32_t sh[33];
+    __shared__ uint32_t sh_prefix, sh_remaining;
+    const int row = blockIdx.x;
+    const float *s = scores + (size_t)row * T;
+    const int tid = threadIdx.x;
+
+    uint32_t prefix = 0u, mask = 0u, remaining = (uint32_t)k;
+    for (int pass = 0; pass < 4; ++pass) {
+        const int shift = 24 - 8 * pass;
+        for (int i = tid; i < 256; i += blockDim.x) hist[i] = 0u;
+        __syncthreads();
+        for (int t = tid; t < T; t += blockDim.x) {
+            const uint32_t key = order_key(__ldg(s + t));
+            if ((key & mask) == prefix) atomicAdd(&hist[(key >> shift) & 255u], 1u);
+        }
+        __syncthreads();
+        if (tid < 32) {
+            // Lane l owns the 8 bins 255-8l ... 248-8l (largest keys first).
+            const int lane = tid;
+            uint32_t c[8], sum = 0u;
+#pragma unroll
+            for (int j = 0; j < 8; ++j) {
+                c[j] = hist[255 - (lane * 8 + j)];
+                sum += c[j];
+            }
+            uint32_t incl = sum;
+#pragma unroll
+            for (int off = 1; off < 32; off <<= 1) {
+                const uint32_t y = __shfl_up_sync(0xffffffffu, incl, off);
+                if (lane >= off) incl += y;
+            }
+            const uint32_t reach = __ballot_sync(0xffffffffu, incl >= remaining);
+            const int first = __ffs(reach) - 1;  // the candidates always number >= remaining
+            if (lane == first) {
+                uint32_t cum = incl - sum;
+                int bin = 0;
+                uint32_t left = remaining;
+#pragma unroll
+                for (int j = 0; j < 8; ++j) {
+                    if (cum + c[j] >= remaining) {
+                        bin = 255 - (lane * 8 + j);
+                        left = remaining - cum;
+                        break;
+                    }
+                    cum += c[j];
+                }
+                sh_prefix = prefix | ((uint32_t)bin << shift);
+                sh_remaining = left;
+            }
+        }
+        __syncthreads();
+        prefix = sh_prefix;
+        remaining = sh_remaining;
+        mask |= 255u << shift;
+        __syncthreads();
+    }
+    // prefix is now the k-th largest key; `remaining` keys equal to it are kept.
+    const uint32_t thr = prefix;
+    uint32_t base_eq = 0u, base_sel = 0u;
+    const int hh = row % H, bb = row / H;
+    for (int t0 = 0; t0 < T; t0 += blockDim.x) {
+        const int t = t0 + tid;
+        float v = 0.f;
+        uint32_t key = 0u;
+        if (t < T) {
+            v = __ldg(s + t);
+            key = order_key(v);
+        }
+        const bool gt = t < T && key > thr;
+        const bool eq = t < T && key == thr;
+        uint32_t n_eq, n_sel;
+        const uint32_t eq_rank = base_eq + block_rank(eq, sh, n_eq);
+        const bool take = gt || (eq && eq_rank < remaining);
+        const uint32_t pos = base_sel + block_rank(take, sh, n_sel);
+        if (take) {
+            I[(size_t)row * k + pos] = t;
+            rsel[(size_t)row * k + pos] = v;
+            if (gidx != nullptr) {
+                const size_t o = ((size_t)hh * B + bb) * k + pos;
+                gidx[o] = bb * T + t;
+                rsel_hm[o] = v;
+            }
+        }
+        base_eq += n_eq;
+        base_sel += n_sel;
+    }
+}
+
+__global__ void indices_to_rows_kernel(const int32_t *__restrict__ I,
+                                       const float *__restrict__ rsel, int B, int H, int T,
+                                       int k, int32_t *__restrict__ gidx,
+                                       float *__restrict__ rsel_hm, uint32_t *status) {
+    const int row = blockIdx.x;  // b*H + h
+    const int hh = row % H, bb = row / H;
+    const int32_t *Ir = I + (size_t)row * k;
+    int bad = 0;
+    for (int i = threadIdx.x; i < k; i += blockDim.x) {
+        const int32_t t = Ir[i];
+        if (t < 0 || t >= T || (i > 0 && Ir[i - 1] >= t)) bad = 1;
+    }
+    bad = __syncthreads_or(bad);
+    if (bad && threadIdx.x == 0) atomicOr(status, kStatusBadIndex);
+    for (int i = threadIdx.x; i < k; i += blockDim.x) {
+        const int32_t t = bad ? i : Ir[i];
+        const size_t o = ((size_t)hh * B + bb) * k + i;
+        gidx[o] = bb * T + t;
+        rsel_hm[o] = rsel[(size_t)row * k + i];
+    }
+}
+
+}  // namespace
+
+cudaError_t launch_router(const Dims &dm, const void *X, const void *Wr, float *r_full,
+                          cudaStream_t stream) {
+    if (dm.bf16) {
+        RouterOp<bf16> op{dm.B * dm.T, dm.H, dm.d, dm.T, dm.H, (const bf16 *)X,
+                          (const bf16 *)Wr, r_full};
+        return launch_simt_gemm(op, 1, stream);
+    }
+    RouterOp<float> op{dm.B * dm.T, dm.H, dm.d, dm.T, dm.H, (const float *)X,
+                       (const float *)Wr, r_full};
+    return launch_simt_gemm(op, 1, stream);
+}
+
+cudaError_t launch_select(int rows, int T, int k, const float *scores, int32_t *I, float *rsel,
+                          int B, int H, int32_t *gidx, float *rsel_hm, cudaStream_t stream) {
+    if (rows <= 0) return cudaSuccess;
+    topk_select_kernel<<<rows, kSelThreads, 0, stream>>>(scores, T, k, I, rsel, B, H, gidx,
+                                                        rsel_hm);
+    note_launches(1);
+    return cudaGetLastError();
+}
+
+cudaError_t launch_indices_to_rows(const Dims &dm, const int32_t *I, const float *rsel,
+                                   int32_t *gidx, float *rsel_hm, uint32_t *status,
+                                   cudaStream_t stream) {
+    indices_to_rows_kernel<<<dm.B * dm.H, 256, 0, stream>>>(I, rsel, dm.B, dm.H, dm.T, dm.k,
+                                                           gidx, rsel_hm, status);
+    note_launches(1);
+    return cudaGetLastError();
+}
+
+}  // namespace mosa

@@ -1,0 +1,163 @@
+"""GPU parity: libmosa (through its C ABI) against the fp64 CPU oracle.
+
+Indices are compared bit-exactly; floats within the stated tolerances
+(fp32 storage: 1e-4 relative L2; bf16 storage: 2e-2 relative L2 and 5e-2
+max-abs).  Small cases are compared element by element in full; the full
+workload sizes are compared on sampled units the oracle computes exactly
+(every head of one sequence for Y and dX, every sequence of one head for the
+weight gradients) plus every selected index.
+"""
+import numpy as np
+import pytest
+import torch
+
+import oracle
+import paper_2505_00315_gb300 as mosa
+from paper_2505_00315_gb300 import workloads as W
+from _gpu import assert_close, run_layer, to_dev
+from _util import sigmoid_gap
+
+pytestmark = pytest.mark.gpu
+
+
+def weights(x):
+    return x["Wr"], x["Wq"], x["Wk"], x["Wv"], x["Wo"]
+
+
+# ------------------------------------------------------------ TopK alone ----
+
+def score_rows(kind, rows, T, rng):
+    if kind == "uniform":
+        return rng.random((rows, T), dtype=np.float32)
+    if kind == "ties":
+        return rng.choice(np.array([0.125, 0.25, 0.5, 0.75], np.float32), size=(rows, T))
+    if kind == "equal":
+        return np.full((rows, T), 0.5, np.float32)
+    if kind == "signed":      # negatives, both zeros, sub-normals
+        v = rng.standard_normal((rows, T)).astype(np.float32)
+        v[:, ::7] = 0.0
+        v[:, 3::11] = -0.0
+        v[:, 5::13] = np.float32(1e-42)
+        return v
+    raise ValueError(kind)
+
+
+@pytest.mark.parametrize("kind", ["uniform", "ties", "equal", "signed"])
+@pytest.mark.parametrize("T,k", [(1, 1), (7, 3), (1000, 1), (1024, 128), (1025, 1025),
+                                 (4096, 64), (8192, 4000), (65536, 257)])
+def test_topk_bit_exact(kind, T, k):
+    rng = np.random.default_rng(T * 31 + k)
+    rows = 3 if T > 10000 else 5
+    s = score_rows(kind, rows, T, rng)
+    I, rs = mosa.mosa_topk(torch.from_numpy(s).cuda(), k)
+    I, rs = I.cpu().numpy(), rs.cpu().numpy()
+    for r in range(rows):
+        Iref, _ = oracle.topk(s[r].astype(np.float64), k)
+        np.testing.assert_array_equal(I[r], Iref)
+        np.testing.assert_array_equal(rs[r].view(np.uint32), s[r][Iref].view(np.uint32))
+
+
+# ---------------------------------------------------- small full parity ----
+
+SMALL = [
+    W.CONFIGS["f32_B1_T256_d128_H4_k64"],
+    W.MosaConfig("ragged_f32", B=2, T=300, d=136, H=3, hp=32, k=77, dtype="f32", seed=11),
+    W.MosaConfig("ragged_bf16", B=2, T=300, d=136, H=3, hp=64, k=77, dtype="bf16", seed=12),
+    W.MosaConfig("k_eq_T_bf16", B=2, T=96, d=64, H=2, hp=64, k=96, dtype="bf16", seed=13),
+    W.MosaConfig("k1_f32", B=3, T=50, d=16, H=5, hp=16, k=1, dtype="f32", seed=14),
+    W.MosaConfig("hp128_bf16", B=1, T=200, d=256, H=2, hp=128, k=130, dtype="bf16", seed=15),
+    W.MosaConfig("hp16_f32", B=2, T=129, d=24, H=7, hp=16, k=65, dtype="f32", seed=16),
+]
+
+
+@pytest.mark.parametrize("cfg", SMALL, ids=lambda c: c.name)
+def test_small_forward_backward_full_parity(cfg):
+    x = W.make_inputs(cfg)
+    Y, I, rs, rf = oracle.forward(x["X"], *weights(x), k=cfg.k)
+    assert sigmoid_gap(rf, cfg.k) > 1e-3
+    g = run_layer(cfg, x, backward=True)
+    np.testing.assert_array_equal(g["I"], I)
+    assert_close("r_full", g["r_full"], rf, cfg.dtype)
+    assert_close("r_sel", g["r_sel"], rs, cfg.dtype)
+    assert_close("Y", g["Y"], Y, cfg.dtype)
+    untouched = np.ones((cfg.B, cfg.T), bool)
+    for b in range(cfg.B):
+        untouched[b, I[b].ravel()] = False
+    assert (g["Y"][untouched] == 0).all()
+    ref = oracle.backward(x["X"], *weights(x), I=I, dY=x["dY"])
+    for name in ("dX", "dWr", "dWq", "dWk", "dWv", "dWo"):
+        gname = name[:2] + "_" + name[2:].lower() if name != "dX" else "dX"
+        assert_close(name, g[gname], ref[name], cfg.dtype)
+
+
+# ------------------------------------------------ full workload sizes ----
+
+FULL = [c for c in W.CONFIGS.values() if c.dtype == "bf16"]
+
+
+@pytest.mark.parametrize("cfg", FULL, ids=lambda c: c.name)
+def test_full_size_sampled_parity(cfg):
+    x = W.make_inputs(cfg)
+    g = run_layer(cfg, x, backward=True)
+    # Every selected index, bit-exact, from the oracle's full score table.
+    rf = oracle.router(x["X"], x["Wr"])
+    assert sigmoid_gap(rf, cfg.k) > 1e-3
+    for b in range(cfg.B):
+        for h in range(cfg.H):
+            Iref, rsref = oracle.topk(rf[b, h], cfg.k)
+            np.testing.assert_array_equal(g["I"][b, h], Iref)
+    assert_close("r_full", g["r_full"], rf, cfg.dtype)
+    # Y and dX of sequence 0 (all heads), exact in the oracle.
+    b0 = cfg.B - 1
+    Y, I, _, _ = oracle.forward(x["X"], *weights(x), k=cfg.k, batches=[b0])
+    assert_close("Y[b]", g["Y"][b0], Y[b0], cfg.dtype)
+    gb = oracle.backward(x["X"], *weights(x), I=g["I"], dY=x["dY"], batches=[b0])
+    assert_close("dX[b]", g["dX"][b0], gb["dX"][b0], cfg.dtype)
+    # Weight gradients of one head (all sequences), exact in the oracle.
+    h0 = cfg.H // 2
+    gh = oracle.backward(x["X"], *weights(x), I=g["I"], dY=x["dY"], heads=[h0])
+    for name in ("dWq", "dWk", "dWv", "dWo"):
+        assert_close(name + "[h]", g[name[:2] + "_" + name[2:].lower()][h0], gh[name][h0],
+                     cfg.dtype)
+    assert_close("dWr[:,h]", g["dW_r"][:, h0], gh["dWr"][:, h0], cfg.dtype)
+
+
+# --------------------------------------------------- indices entry point ----
+
+@pytest.mark.parametrize("dtype", ["f32", "bf16"])
+def test_fixed_sparse_indices_entry(dtype):
+    cfg = W.MosaConfig("fixed", B=2, T=512, d=64, H=4, hp=32, k=64, dtype=dtype, seed=21)
+    x = W.make_inputs(cfg, plant=False)
+    I = W.fixed_sparse_indices(cfg.B, cfg.H, cfg.T, cfg.k)
+    ones = np.ones((cfg.B, cfg.H, cfg.k), np.float32)
+    ref = oracle.forward_indices(x["X"], *weights(x), I=I, r_sel=ones)
+    Xd, Wq, Wk, Wv, Wo = (to_dev(x[n], dtype) for n in ("X", "Wq", "Wk", "Wv", "Wo"))
+    Y, ws = mosa.mosa_forward_with_indices(Xd, Wq, Wk, Wv, Wo, torch.from_numpy(I).cuda(),
+                                           torch.from_numpy(ones).cuda())
+    assert mosa.mosa_check_status(mosa.make_shape(Xd, Wq, cfg.k), ws) == 0
+    assert_close("Y", Y.cpu().numpy(), ref, dtype)
+
+
+def test_invalid_indices_are_flagged_not_followed():
+    cfg = W.MosaConfig("bad", B=1, T=64, d=32, H=2, hp=32, k=8, dtype="f32", seed=22)
+    x = W.make_inputs(cfg, plant=False)
+    I = W.fixed_sparse_indices(cfg.B, cfg.H, cfg.T, cfg.k).copy()
+    I[0, 1, 3] = 10_000          # out of range
+    I[0, 0, 5] = I[0, 0, 4]      # not strictly ascending
+    Xd, Wq, Wk, Wv, Wo = (to_dev(x[n], "f32") for n in ("X", "Wq", "Wk", "Wv", "Wo"))
+    rs = torch.ones((1, 2, 8), device="cuda")
+    Y, ws = mosa.mosa_forward_with_indices(Xd, Wq, Wk, Wv, Wo, torch.from_numpy(I).cuda(), rs)
+    shape = mosa.make_shape(Xd, Wq, cfg.k)
+    assert mosa.mosa_check_status(shape, ws) == 1          # MOSA_ERR_INVALID_ARG
+    assert torch.isfinite(Y).all()
+    assert mosa.mosa_check_status(shape, ws) == 0          # cleared by the read
+
+
+def test_workspace_reuse_gives_same_result():
+    cfg = W.CONFIGS["B8_T1024_d512_H16_k128"].with_(B=2)
+    x = W.make_inputs(cfg)
+    a = run_layer(cfg, x)
+    b = run_layer(cfg, x)
+    np.testing.assert_array_equal(a["I"], b["I"])
+    for n in ("Y", "dX", "dW_q", "dW_o", "dW_r"):
+        np.testing.assert_allclose(a[n], b[n], rtol=1e-5, atol=1e-6)

@@ -19,18 +19,19 @@ namespace {
 constexpr int kRowsPerBlock = 64;
 constexpr int kTile = 32;
 
-template <class T, int HP>
+template <class TS, int HP>
 __global__ void __launch_bounds__(kRowsPerBlock)
-attn_fwd_simt_kernel(const T *__restrict__ Q, const T *__restrict__ K, const T *__restrict__ V,
-                     const float *__restrict__ rsel, T *__restrict__ A, T *__restrict__ AR,
-                     float *__restrict__ lse, int k, float scale) {
+attn_fwd_simt_kernel(const void *__restrict__ Q, const void *__restrict__ K,
+                     const void *__restrict__ V, const float *__restrict__ rsel,
+                     float *__restrict__ A, void *__restrict__ AR, float *__restrict__ lse, int k,
+                     float scale) {
     __shared__ float Ks[kTile][HP], Vs[kTile][HP];
     const size_t base = (size_t)blockIdx.y * k;
     const int i = blockIdx.x * kRowsPerBlock + threadIdx.x;
     float q[HP], o[HP];
 #pragma unroll
     for (int p = 0; p < HP; ++p) {
-        q[p] = i < k ? to_f32(Q[(base + i) * HP + p]) * scale : 0.f;
+        q[p] = i < k ? Inter<TS>::ld(Q, base + i, HP, p) * scale : 0.f;
         o[p] = 0.f;
     }
     float m = -FLT_MAX, l = 0.f;
@@ -39,8 +40,8 @@ attn_fwd_simt_kernel(const T *__restrict__ Q, const T *__restrict__ K, const T *
         __syncthreads();
         for (int e = threadIdx.x; e < kTile * HP; e += kRowsPerBlock) {
             const int jj = e / HP, p = e % HP, j = j0 + jj;
-            Ks[jj][p] = j < k ? to_f32(K[(base + j) * HP + p]) : 0.f;
-            Vs[jj][p] = j < k ? to_f32(V[(base + j) * HP + p]) : 0.f;
+            Ks[jj][p] = j < k ? Inter<TS>::ld(K, base + j, HP, p) : 0.f;
+            Vs[jj][p] = j < k ? Inter<TS>::ld(V, base + j, HP, p) : 0.f;
         }
         __syncthreads();
         if (i < k) {
@@ -68,27 +69,28 @@ attn_fwd_simt_kernel(const T *__restrict__ Q, const T *__restrict__ K, const T *
 #pragma unroll
         for (int p = 0; p < HP; ++p) {
             const float a = o[p] * inv;
-            A[(base + i) * HP + p] = from_f32<T>(a);
-            AR[(base + i) * HP + p] = from_f32<T>(r * a);
+            A[(base + i) * HP + p] = a;
+            Inter<TS>::st(AR, base + i, HP, p, r * a);
         }
         lse[base + i] = m + logf(l);
     }
 }
 
 // dQ: one thread per query row i, keys j <= i.
-template <class T, int HP>
+template <class TS, int HP>
 __global__ void __launch_bounds__(kRowsPerBlock)
-attn_bwd_dq_simt_kernel(const T *__restrict__ Q, const T *__restrict__ K, const T *__restrict__ V,
-                        const T *__restrict__ dA, const float *__restrict__ lse,
-                        const float *__restrict__ Dd, T *__restrict__ dQKV, int k, float scale) {
+attn_bwd_dq_simt_kernel(const void *__restrict__ Q, const void *__restrict__ K,
+                        const void *__restrict__ V, const void *__restrict__ dA,
+                        const float *__restrict__ lse, const float *__restrict__ Dd,
+                        void *__restrict__ dQKV, int k, float scale) {
     __shared__ float Ks[kTile][HP], Vs[kTile][HP];
     const size_t base = (size_t)blockIdx.y * k;
     const int i = blockIdx.x * kRowsPerBlock + threadIdx.x;
     float q[HP], da[HP], dq[HP];
 #pragma unroll
     for (int p = 0; p < HP; ++p) {
-        q[p] = i < k ? to_f32(Q[(base + i) * HP + p]) * scale : 0.f;
-        da[p] = i < k ? to_f32(dA[(base + i) * HP + p]) : 0.f;
+        q[p] = i < k ? Inter<TS>::ld(Q, base + i, HP, p) * scale : 0.f;
+        da[p] = i < k ? Inter<TS>::ld(dA, base + i, HP, p) : 0.f;
         dq[p] = 0.f;
     }
     const float L = i < k ? lse[base + i] : 0.f, D = i < k ? Dd[base + i] : 0.f;
@@ -97,8 +99,8 @@ attn_bwd_dq_simt_kernel(const T *__restrict__ Q, const T *__restrict__ K, const 
         __syncthreads();
         for (int e = threadIdx.x; e < kTile * HP; e += kRowsPerBlock) {
             const int jj = e / HP, p = e % HP, j = j0 + jj;
-            Ks[jj][p] = j < k ? to_f32(K[(base + j) * HP + p]) : 0.f;
-            Vs[jj][p] = j < k ? to_f32(V[(base + j) * HP + p]) : 0.f;
+            Ks[jj][p] = j < k ? Inter<TS>::ld(K, base + j, HP, p) : 0.f;
+            Vs[jj][p] = j < k ? Inter<TS>::ld(V, base + j, HP, p) : 0.f;
         }
         __syncthreads();
         if (i < k) {
@@ -118,32 +120,33 @@ attn_bwd_dq_simt_kernel(const T *__restrict__ Q, const T *__restrict__ K, const 
     }
     if (i < k) {
 #pragma unroll
-        for (int p = 0; p < HP; ++p) dQKV[(base + i) * (3 * HP) + p] = from_f32<T>(dq[p] * scale);
+        for (int p = 0; p < HP; ++p) Inter<TS>::st(dQKV, base + i, 3 * HP, p, dq[p] * scale);
     }
 }
 
 // dK and dV: one thread per key row j, queries i >= j.
-template <class T, int HP, bool kDK>
+template <class TS, int HP, bool kDK>
 __global__ void __launch_bounds__(kRowsPerBlock)
-attn_bwd_dkv_simt_kernel(const T *__restrict__ Q, const T *__restrict__ K, const T *__restrict__ V,
-                         const T *__restrict__ dA, const float *__restrict__ lse,
-                         const float *__restrict__ Dd, T *__restrict__ dQKV, int k, float scale) {
+attn_bwd_dkv_simt_kernel(const void *__restrict__ Q, const void *__restrict__ K,
+                         const void *__restrict__ V, const void *__restrict__ dA,
+                         const float *__restrict__ lse, const float *__restrict__ Dd,
+                         void *__restrict__ dQKV, int k, float scale) {
     __shared__ float Qs[kTile][HP], dAs[kTile][HP], Ls[kTile], Ds[kTile];
     const size_t base = (size_t)blockIdx.y * k;
     const int j = blockIdx.x * kRowsPerBlock + threadIdx.x;
     float kr[HP], vr[HP], acc[HP];
 #pragma unroll
     for (int p = 0; p < HP; ++p) {
-        kr[p] = j < k ? to_f32(K[(base + j) * HP + p]) * scale : 0.f;
-        vr[p] = (kDK && j < k) ? to_f32(V[(base + j) * HP + p]) : 0.f;
+        kr[p] = j < k ? Inter<TS>::ld(K, base + j, HP, p) * scale : 0.f;
+        vr[p] = (kDK && j < k) ? Inter<TS>::ld(V, base + j, HP, p) : 0.f;
         acc[p] = 0.f;
     }
     for (int i0 = blockIdx.x * kRowsPerBlock; i0 < k; i0 += kTile) {
         __syncthreads();
         for (int e = threadIdx.x; e < kTile * HP; e += kRowsPerBlock) {
             const int ii = e / HP, p = e % HP, i = i0 + ii;
-            Qs[ii][p] = i < k ? to_f32(Q[(base + i) * HP + p]) : 0.f;
-            dAs[ii][p] = i < k ? to_f32(dA[(base + i) * HP + p]) : 0.f;
+            Qs[ii][p] = i < k ? Inter<TS>::ld(Q, base + i, HP, p) : 0.f;
+            dAs[ii][p] = i < k ? Inter<TS>::ld(dA, base + i, HP, p) : 0.f;
         }
         for (int ii = threadIdx.x; ii < kTile; ii += kRowsPerBlock) {
             const int i = i0 + ii;
@@ -176,57 +179,52 @@ attn_bwd_dkv_simt_kernel(const T *__restrict__ Q, const T *__restrict__ K, const
         const int col = kDK ? HP : 2 * HP;
         const float f = kDK ? scale : 1.f;
 #pragma unroll
-        for (int p = 0; p < HP; ++p)
-            dQKV[(base + j) * (3 * HP) + col + p] = from_f32<T>(acc[p] * f);
+        for (int p = 0; p < HP; ++p) Inter<TS>::st(dQKV, base + j, 3 * HP, col + p, acc[p] * f);
     }
 }
 
-template <class T, int HP>
+template <class TS, int HP>
 cudaError_t attn_fwd_t(const Dims &dm, const Saved &sv, cudaStream_t s) {
     dim3 grid((dm.k + kRowsPerBlock - 1) / kRowsPerBlock, dm.H * dm.B);
     const float scale = 1.f / sqrtf((float)HP);
-    attn_fwd_simt_kernel<T, HP><<<grid, kRowsPerBlock, 0, s>>>(
-        (const T *)sv.Q, (const T *)sv.K, (const T *)sv.V, sv.rsel, (T *)sv.A, (T *)sv.AR, sv.lse,
-        dm.k, scale);
+    attn_fwd_simt_kernel<TS, HP><<<grid, kRowsPerBlock, 0, s>>>(sv.Q, sv.K, sv.V, sv.rsel, sv.A,
+                                                               sv.AR, sv.lse, dm.k, scale);
     note_launches(1);
     return cudaGetLastError();
 }
 
-template <class T, int HP>
+template <class TS, int HP>
 cudaError_t attn_bwd_t(const Dims &dm, const Saved &sv, cudaStream_t s) {
     dim3 grid((dm.k + kRowsPerBlock - 1) / kRowsPerBlock, dm.H * dm.B);
     const float scale = 1.f / sqrtf((float)HP);
-    attn_bwd_dq_simt_kernel<T, HP><<<grid, kRowsPerBlock, 0, s>>>(
-        (const T *)sv.Q, (const T *)sv.K, (const T *)sv.V, (const T *)sv.dA, sv.lse, sv.Dd,
-        (T *)sv.dQKV, dm.k, scale);
-    attn_bwd_dkv_simt_kernel<T, HP, true><<<grid, kRowsPerBlock, 0, s>>>(
-        (const T *)sv.Q, (const T *)sv.K, (const T *)sv.V, (const T *)sv.dA, sv.lse, sv.Dd,
-        (T *)sv.dQKV, dm.k, scale);
-    attn_bwd_dkv_simt_kernel<T, HP, false><<<grid, kRowsPerBlock, 0, s>>>(
-        (const T *)sv.Q, (const T *)sv.K, (const T *)sv.V, (const T *)sv.dA, sv.lse, sv.Dd,
-        (T *)sv.dQKV, dm.k, scale);
+    attn_bwd_dq_simt_kernel<TS, HP><<<grid, kRowsPerBlock, 0, s>>>(
+        sv.Q, sv.K, sv.V, sv.dA, sv.lse, sv.Dd, sv.dQKV, dm.k, scale);
+    attn_bwd_dkv_simt_kernel<TS, HP, true><<<grid, kRowsPerBlock, 0, s>>>(
+        sv.Q, sv.K, sv.V, sv.dA, sv.lse, sv.Dd, sv.dQKV, dm.k, scale);
+    attn_bwd_dkv_simt_kernel<TS, HP, false><<<grid, kRowsPerBlock, 0, s>>>(
+        sv.Q, sv.K, sv.V, sv.dA, sv.lse, sv.Dd, sv.dQKV, dm.k, scale);
     note_launches(3);
     return cudaGetLastError();
 }
 
-template <class T>
+template <class TS>
 cudaError_t attn_fwd_dispatch(const Dims &dm, const Saved &sv, cudaStream_t s) {
     switch (dm.hp) {
-        case 16: return attn_fwd_t<T, 16>(dm, sv, s);
-        case 32: return attn_fwd_t<T, 32>(dm, sv, s);
-        case 64: return attn_fwd_t<T, 64>(dm, sv, s);
-        case 128: return attn_fwd_t<T, 128>(dm, sv, s);
+        case 16: return attn_fwd_t<TS, 16>(dm, sv, s);
+        case 32: return attn_fwd_t<TS, 32>(dm, sv, s);
+        case 64: return attn_fwd_t<TS, 64>(dm, sv, s);
+        case 128: return attn_fwd_t<TS, 128>(dm, sv, s);
         default: return cudaErrorInvalidValue;
     }
 }
 
-template <class T>
+template <class TS>
 cudaError_t attn_bwd_dispatch(const Dims &dm, const Saved &sv, cudaStream_t s) {
     switch (dm.hp) {
-        case 16: return attn_bwd_t<T, 16>(dm, sv, s);
-        case 32: return attn_bwd_t<T, 32>(dm, sv, s);
-        case 64: return attn_bwd_t<T, 64>(dm, sv, s);
-        case 128: return attn_bwd_t<T, 128>(dm, sv, s);
+        case 16: return attn_bwd_t<TS, 16>(dm, sv, s);
+        case 32: return attn_bwd_t<TS, 32>(dm, sv, s);
+        case 64: return attn_bwd_t<TS, 64>(dm, sv, s);
+        case 128: return attn_bwd_t<TS, 128>(dm, sv, s);
         default: return cudaErrorInvalidValue;
     }
 }
@@ -234,11 +232,11 @@ cudaError_t attn_bwd_dispatch(const Dims &dm, const Saved &sv, cudaStream_t s) {
 }  // namespace
 
 cudaError_t launch_attn_fwd(const Dims &dm, const Saved &sv, cudaStream_t s) {
-    return dm.bf16 ? attn_fwd_dispatch<bf16>(dm, sv, s) : attn_fwd_dispatch<float>(dm, sv, s);
+    return dm.bf16 ? attn_fwd_dispatch<SplitBF16>(dm, sv, s) : attn_fwd_dispatch<float>(dm, sv, s);
 }
 
 cudaError_t launch_attn_bwd(const Dims &dm, const Saved &sv, cudaStream_t s) {
-    return dm.bf16 ? attn_bwd_dispatch<bf16>(dm, sv, s) : attn_bwd_dispatch<float>(dm, sv, s);
+    return dm.bf16 ? attn_bwd_dispatch<SplitBF16>(dm, sv, s) : attn_bwd_dispatch<float>(dm, sv, s);
 }
 
 }  // namespace mosa

@@ -28,6 +28,51 @@ __device__ __forceinline__ float from_f32<float>(float x) { return x; }
 template <>
 __device__ __forceinline__ bf16 from_f32<bf16>(float x) { return __float2bfloat16_rn(x); }
 
+// Intermediates (Q, K, V, diag(r) A, dA, dQ|dK|dV) are kept at about fp32
+// precision whatever the input dtype: fp32 arrays for fp32 inputs, and for
+// bf16 inputs a pair (hi, lo) of bf16 values with v ~= hi + lo (hi = bf16(v),
+// lo = bf16(v - hi)), stored as planar halves of each row: [hi x cols | lo x
+// cols].  A tensor-core product with such an operand is two bf16 MMAs into
+// one fp32 accumulator.  Both forms take 4 bytes per element.
+struct SplitBF16 {};
+
+template <class TS>
+struct Inter;
+
+template <>
+struct Inter<float> {
+    static __device__ __forceinline__ float ld(const void *p, size_t row, int cols, int c) {
+        return static_cast<const float *>(p)[row * cols + c];
+    }
+    static __device__ __forceinline__ void st(void *p, size_t row, int cols, int c, float v) {
+        static_cast<float *>(p)[row * cols + c] = v;
+    }
+};
+
+template <>
+struct Inter<SplitBF16> {
+    static __device__ __forceinline__ float ld(const void *p, size_t row, int cols, int c) {
+        const bf16 *q = static_cast<const bf16 *>(p) + row * 2 * cols;
+        return __bfloat162float(q[c]) + __bfloat162float(q[cols + c]);
+    }
+    static __device__ __forceinline__ void st(void *p, size_t row, int cols, int c, float v) {
+        bf16 *q = static_cast<bf16 *>(p) + row * 2 * cols;
+        const bf16 hi = __float2bfloat16_rn(v);
+        q[c] = hi;
+        q[cols + c] = __float2bfloat16_rn(v - __bfloat162float(hi));
+    }
+};
+
+// Intermediate storage for an input dtype.
+template <class TI>
+struct InterOf {
+    using type = float;
+};
+template <>
+struct InterOf<bf16> {
+    using type = SplitBF16;
+};
+
 // Internal views of the workspace.  Per-head state is stored head-major,
 // [H][B*k][...], so that each head's B*k selected rows form one contiguous
 // matrix (row m = b*k + i).
@@ -36,14 +81,14 @@ struct Saved {
     float *r_full;      // [B,H,T]   router scores (when the caller gives none)
     int32_t *gidx;      // [H,B*k]   b*T + I[b,h,i]: row of X / Y / dY to gather or scatter
     float *rsel;        // [H,B*k]   r^topk in the same order
-    void *Q, *K, *V;    // [H,B*k,hp] storage dtype
-    void *A;            // [H,B*k,hp] attention output
-    void *AR;           // [H,B*k,hp] diag(r^topk) A
+    void *Q, *K, *V;    // [H,B*k,hp] intermediate (fp32 or bf16 hi/lo pair)
+    float *A;           // [H,B*k,hp] attention output, fp32
+    void *AR;           // [H,B*k,hp] diag(r^topk) A, intermediate
     float *lse;         // [H,B*k]   log-sum-exp of the scaled, masked scores
-    void *dA;           // [H,B*k,hp] gradient of A
+    void *dA;           // [H,B*k,hp] gradient of A, intermediate
     float *dlogit;      // [H,B*k]   gradient of the router logit
     float *Dd;          // [H,B*k]   rowsum(dA o A)
-    void *dQKV;         // [H,B*k,3hp] dQ | dK | dV
+    void *dQKV;         // [H,B*k,3hp] dQ | dK | dV, intermediate
     float *G;           // [H,B*k,hp] dY[I] W_o^T (fp32)
 };
 

@@ -43,7 +43,7 @@ size_t carve(const Dims &dm, char *base, Saved *sv) {
         return p;
     };
     const size_t R = (size_t)dm.rows();
-    const size_t e = dm.esize();
+    const size_t e = 4;  // fp32, or a bf16 hi/lo pair
     Saved s{};
     s.status = (uint32_t *)take(sizeof(uint32_t));
     s.r_full = (float *)take(sizeof(float) * (size_t)dm.B * dm.H * dm.T);
@@ -52,7 +52,7 @@ size_t carve(const Dims &dm, char *base, Saved *sv) {
     s.Q = take(e * R * dm.hp);
     s.K = take(e * R * dm.hp);
     s.V = take(e * R * dm.hp);
-    s.A = take(e * R * dm.hp);
+    s.A = (float *)take(sizeof(float) * R * dm.hp);
     s.AR = take(e * R * dm.hp);
     s.lse = (float *)take(sizeof(float) * R);
     s.dA = take(e * R * dm.hp);

@@ -15,12 +15,13 @@ namespace {
 
 template <class T>
 struct QkvOp {
+    using TS = typename InterOf<T>::type;
     static constexpr bool kAKFast = true, kBKFast = false;
     int M, N, K;  // B*k, 3*hp, d
     int hp;
     const T *X, *Wq, *Wk, *Wv;
     const int32_t *gidx;
-    T *Q, *Kp, *V;
+    void *Q, *Kp, *V;
     __device__ float a(int g, int m, int c) const {
         return to_f32(X[(size_t)gidx[(size_t)g * M + m] * K + c]);
     }
@@ -31,19 +32,21 @@ struct QkvOp {
     }
     __device__ void store(int g, int m, int n, float v) const {
         const int w = n / hp, p = n - w * hp;
-        T *O = w == 0 ? Q : (w == 1 ? Kp : V);
-        O[((size_t)g * M + m) * hp + p] = from_f32<T>(v);
+        void *O = w == 0 ? Q : (w == 1 ? Kp : V);
+        Inter<TS>::st(O, (size_t)g * M + m, hp, p, v);
     }
 };
 
 template <class T>
 struct OutOp {
+    using TS = typename InterOf<T>::type;
     static constexpr bool kAKFast = true, kBKFast = false;
     int M, N, K;  // B*k, d, hp
-    const T *AR, *Wo;
+    const void *AR;
+    const T *Wo;
     const int32_t *gidx;
     float *Y;
-    __device__ float a(int g, int m, int p) const { return to_f32(AR[((size_t)g * M + m) * K + p]); }
+    __device__ float a(int g, int m, int p) const { return Inter<TS>::ld(AR, (size_t)g * M + m, K, p); }
     __device__ float b(int g, int p, int n) const { return to_f32(Wo[((size_t)g * K + p) * N + n]); }
     __device__ void store(int g, int m, int n, float v) const {
         atomicAdd(Y + (size_t)gidx[(size_t)g * M + m] * N + n, v);
@@ -66,12 +69,14 @@ struct OutBwdGOp {
 
 template <class T>
 struct OutBwdWOp {
+    using TS = typename InterOf<T>::type;
     static constexpr bool kAKFast = false, kBKFast = false;
     int M, N, K;  // hp, d, B*k
-    const T *AR, *dY;
+    const void *AR;
+    const T *dY;
     const int32_t *gidx;
     float *dWo;
-    __device__ float a(int g, int p, int m) const { return to_f32(AR[((size_t)g * K + m) * M + p]); }
+    __device__ float a(int g, int p, int m) const { return Inter<TS>::ld(AR, (size_t)g * K + m, M, p); }
     __device__ float b(int g, int m, int n) const {
         return to_f32(dY[(size_t)gidx[(size_t)g * K + m] * N + n]);
     }
@@ -80,14 +85,16 @@ struct OutBwdWOp {
 
 template <class T>
 struct InBwdOp {
+    using TS = typename InterOf<T>::type;
     static constexpr bool kAKFast = true, kBKFast = true;
     int M, N, K;  // B*k, d, 3*hp
     int hp, H;
-    const T *dQKV, *Wq, *Wk, *Wv, *Wr;
+    const void *dQKV;
+    const T *Wq, *Wk, *Wv, *Wr;
     const float *dlogit;
     const int32_t *gidx;
     float *dX;
-    __device__ float a(int g, int m, int kk) const { return to_f32(dQKV[((size_t)g * M + m) * K + kk]); }
+    __device__ float a(int g, int m, int kk) const { return Inter<TS>::ld(dQKV, (size_t)g * M + m, K, kk); }
     __device__ float b(int g, int kk, int n) const {
         const int w = kk / hp, p = kk - w * hp;
         const T *W = w == 0 ? Wq : (w == 1 ? Wk : Wv);
@@ -103,10 +110,12 @@ struct InBwdOp {
 // dW_{q,k,v} and, as one extra output column, dW_r.
 template <class T>
 struct WBwdOp {
+    using TS = typename InterOf<T>::type;
     static constexpr bool kAKFast = false, kBKFast = false;
     int M, N, K;  // d, 3*hp + 1, B*k
     int hp, H;
-    const T *X, *dQKV;
+    const T *X;
+    const void *dQKV;
     const float *dlogit;
     const int32_t *gidx;
     float *dWq, *dWk, *dWv, *dWr;
@@ -115,7 +124,7 @@ struct WBwdOp {
     }
     __device__ float b(int g, int m, int n) const {
         const size_t row = (size_t)g * K + m;
-        return n < 3 * hp ? to_f32(dQKV[row * (3 * hp) + n]) : dlogit[row];
+        return n < 3 * hp ? Inter<TS>::ld(dQKV, row, 3 * hp, n) : dlogit[row];
     }
     __device__ void store(int g, int c, int n, float v) const {
         if (n == 3 * hp) {
@@ -130,9 +139,9 @@ struct WBwdOp {
 
 // One warp per selected row: dr = <A, G>, dA = r G (rounded to storage),
 // D = rowsum(dA o A), dlogit = dr r (1 - r).
-template <class T>
-__global__ void out_bwd_rows_kernel(const float *__restrict__ G, const T *__restrict__ A,
-                                    const float *__restrict__ rsel, T *__restrict__ dA,
+template <class TS>
+__global__ void out_bwd_rows_kernel(const float *__restrict__ G, const float *__restrict__ A,
+                                    const float *__restrict__ rsel, void *__restrict__ dA,
                                     float *__restrict__ Dd, float *__restrict__ dlogit,
                                     long long rows, int hp) {
     const long long row = (long long)blockIdx.x * (blockDim.x / 32) + threadIdx.x / 32;
@@ -142,11 +151,11 @@ __global__ void out_bwd_rows_kernel(const float *__restrict__ G, const T *__rest
     float dr = 0.f, dd = 0.f;
     for (int p = lane; p < hp; p += 32) {
         const float g = G[row * hp + p];
-        const float a = to_f32(A[row * hp + p]);
+        const float a = A[row * hp + p];
         dr = fmaf(a, g, dr);
-        const T da = from_f32<T>(r * g);
-        dA[row * hp + p] = da;
-        dd = fmaf(to_f32(da), a, dd);
+        const float da = r * g;
+        Inter<TS>::st(dA, row, hp, p, da);
+        dd = fmaf(da, a, dd);
     }
 #pragma unroll
     for (int off = 16; off > 0; off >>= 1) {
@@ -163,7 +172,7 @@ template <class T>
 cudaError_t qkv_t(const Dims &dm, const void *X, const void *Wq, const void *Wk, const void *Wv,
                   const Saved &sv, cudaStream_t s) {
     QkvOp<T> op{dm.B * dm.k, 3 * dm.hp, dm.d, dm.hp, (const T *)X, (const T *)Wq, (const T *)Wk,
-                (const T *)Wv, sv.gidx, (T *)sv.Q, (T *)sv.K, (T *)sv.V};
+                (const T *)Wv, sv.gidx, sv.Q, sv.K, sv.V};
     return launch_simt_gemm(op, dm.H, s);
 }
 
@@ -171,7 +180,7 @@ template <class T>
 cudaError_t out_t(const Dims &dm, const void *Wo, const Saved &sv, float *Y, cudaStream_t s) {
     cudaError_t e = cudaMemsetAsync(Y, 0, sizeof(float) * (size_t)dm.B * dm.T * dm.d, s);
     if (e != cudaSuccess) return e;
-    OutOp<T> op{dm.B * dm.k, dm.d, dm.hp, (const T *)sv.AR, (const T *)Wo, sv.gidx, Y};
+    OutOp<T> op{dm.B * dm.k, dm.d, dm.hp, sv.AR, (const T *)Wo, sv.gidx, Y};
     return launch_simt_gemm(op, dm.H, s);
 }
 
@@ -183,11 +192,12 @@ cudaError_t out_bwd_t(const Dims &dm, const void *Wo, const void *dY, const Save
     if (e != cudaSuccess) return e;
     const long long rows = dm.rows();
     const int warps = 8;
-    out_bwd_rows_kernel<T><<<(unsigned)((rows + warps - 1) / warps), warps * 32, 0, s>>>(
-        sv.G, (const T *)sv.A, sv.rsel, (T *)sv.dA, sv.Dd, sv.dlogit, rows, dm.hp);
+    out_bwd_rows_kernel<typename InterOf<T>::type>
+        <<<(unsigned)((rows + warps - 1) / warps), warps * 32, 0, s>>>(
+            sv.G, sv.A, sv.rsel, sv.dA, sv.Dd, sv.dlogit, rows, dm.hp);
     note_launches(1);
     if ((e = cudaGetLastError()) != cudaSuccess) return e;
-    OutBwdWOp<T> w{dm.hp, dm.d, dm.B * dm.k, (const T *)sv.AR, (const T *)dY, sv.gidx, dWo};
+    OutBwdWOp<T> w{dm.hp, dm.d, dm.B * dm.k, sv.AR, (const T *)dY, sv.gidx, dWo};
     return launch_simt_gemm(w, dm.H, s);
 }
 
@@ -196,7 +206,7 @@ cudaError_t in_bwd_t(const Dims &dm, const void *Wq, const void *Wk, const void 
                      const void *Wr, const Saved &sv, float *dX, cudaStream_t s) {
     cudaError_t e = cudaMemsetAsync(dX, 0, sizeof(float) * (size_t)dm.B * dm.T * dm.d, s);
     if (e != cudaSuccess) return e;
-    InBwdOp<T> op{dm.B * dm.k, dm.d, 3 * dm.hp, dm.hp, dm.H, (const T *)sv.dQKV, (const T *)Wq,
+    InBwdOp<T> op{dm.B * dm.k, dm.d, 3 * dm.hp, dm.hp, dm.H, sv.dQKV, (const T *)Wq,
                   (const T *)Wk, (const T *)Wv, (const T *)Wr, sv.dlogit, sv.gidx, dX};
     return launch_simt_gemm(op, dm.H, s);
 }
@@ -205,7 +215,7 @@ template <class T>
 cudaError_t w_bwd_t(const Dims &dm, const void *X, const Saved &sv, float *dWq, float *dWk,
                     float *dWv, float *dWr, cudaStream_t s) {
     WBwdOp<T> op{dm.d, 3 * dm.hp + 1, dm.B * dm.k, dm.hp, dm.H, (const T *)X,
-                 (const T *)sv.dQKV, sv.dlogit, sv.gidx, dWq, dWk, dWv, dWr};
+                 sv.dQKV, sv.dlogit, sv.gidx, dWq, dWk, dWv, dWr};
     return launch_simt_gemm(op, dm.H, s);
 }
 

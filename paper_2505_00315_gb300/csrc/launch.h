@@ -50,4 +50,19 @@ cudaError_t launch_in_bwd(const Dims &dm, const void *Wq, const void *Wk, const 
 cudaError_t launch_w_bwd(const Dims &dm, const void *X, const Saved &sv, float *dWq,
                          float *dWk, float *dWv, float *dWr, cudaStream_t stream);
 
+// ---- tensor-core path (tc_gemm.cu): bf16 inputs, head size 64 ----
+bool tc_supported(const Dims &dm);
+// True when the tensor-core kernels serve this shape (false also when the
+// environment variable MOSA_FORCE_SIMT is set to a non-zero value).
+bool use_tc(const Dims &dm);
+cudaError_t tc_qkv(const Dims &dm, const void *X, const void *Wq, const void *Wk, const void *Wv,
+                   const Saved &sv, cudaStream_t s);
+cudaError_t tc_out(const Dims &dm, const void *Wo, const Saved &sv, float *Y, cudaStream_t s);
+cudaError_t tc_out_bwd(const Dims &dm, const void *Wo, const void *dY, const Saved &sv,
+                       float *dWo, cudaStream_t s);
+cudaError_t tc_in_bwd(const Dims &dm, const void *Wq, const void *Wk, const void *Wv,
+                      const void *Wr, const Saved &sv, float *dX, cudaStream_t s);
+cudaError_t tc_w_bwd(const Dims &dm, const void *X, const Saved &sv, float *dWq, float *dWk,
+                     float *dWv, cudaStream_t s);
+
 }  // namespace mosa

@@ -7,6 +7,8 @@
 //   B3  dX[b, I, :] += dQ W^Q^T + dK W^K^T + dV W^V^T + dlogit W^r[:,h]^T
 //   B4  dW^{Q,K,V} = X^s^T d{Q,K,V},  dW^r[:,h] = X^s^T dlogit
 // Rows of head h are m = b*k + i; gidx maps them to rows of X / Y / dY.
+#include <cstdlib>
+
 #include "launch.h"
 #include "simt_gemm.cuh"
 
@@ -168,6 +170,38 @@ __global__ void out_bwd_rows_kernel(const float *__restrict__ G, const float *__
     }
 }
 
+// dW_r[c, h] = sum_m X[g(m), c] dlogit(m): one thread per column c of one
+// head and one slice of the rows; slices are summed with atomics.
+template <class T>
+__global__ void dwr_kernel(const T *__restrict__ X, const int32_t *__restrict__ gidx,
+                           const float *__restrict__ dlogit, float *__restrict__ dWr, int Mtok,
+                           int d, int H, int rows_per_slice) {
+    const int c = blockIdx.x * blockDim.x + threadIdx.x;
+    const int h = blockIdx.y;
+    const int m_begin = blockIdx.z * rows_per_slice;
+    const int m_end = min(Mtok, m_begin + rows_per_slice);
+    if (c >= d) return;
+    float acc = 0.f;
+    for (int m = m_begin; m < m_end; ++m) {
+        const size_t row = (size_t)h * Mtok + m;
+        acc = fmaf(to_f32(X[(size_t)gidx[row] * d + c]), dlogit[row], acc);
+    }
+    atomicAdd(dWr + (size_t)c * H + h, acc);
+}
+
+template <class T>
+cudaError_t dwr_t(const Dims &dm, const void *X, const Saved &sv, float *dWr, cudaStream_t s) {
+    cudaError_t e = cudaMemsetAsync(dWr, 0, sizeof(float) * (size_t)dm.d * dm.H, s);
+    if (e != cudaSuccess) return e;
+    const int Mtok = dm.B * dm.k;
+    const int rows = 64;
+    dim3 grid((dm.d + 255) / 256, dm.H, (Mtok + rows - 1) / rows);
+    dwr_kernel<T><<<grid, 256, 0, s>>>((const T *)X, sv.gidx, sv.dlogit, dWr, Mtok, dm.d, dm.H,
+                                       rows);
+    note_launches(1);
+    return cudaGetLastError();
+}
+
 template <class T>
 cudaError_t qkv_t(const Dims &dm, const void *X, const void *Wq, const void *Wk, const void *Wv,
                   const Saved &sv, cudaStream_t s) {
@@ -221,28 +255,43 @@ cudaError_t w_bwd_t(const Dims &dm, const void *X, const Saved &sv, float *dWq, 
 
 }  // namespace
 
+bool use_tc(const Dims &dm) {
+    const char *f = std::getenv("MOSA_FORCE_SIMT");
+    if (f != nullptr && f[0] != '\0' && f[0] != '0') return false;
+    return tc_supported(dm);
+}
+
 cudaError_t launch_qkv(const Dims &dm, const void *X, const void *Wq, const void *Wk,
                        const void *Wv, const Saved &sv, cudaStream_t s) {
+    if (use_tc(dm)) return tc_qkv(dm, X, Wq, Wk, Wv, sv, s);
     return dm.bf16 ? qkv_t<bf16>(dm, X, Wq, Wk, Wv, sv, s) : qkv_t<float>(dm, X, Wq, Wk, Wv, sv, s);
 }
 
 cudaError_t launch_out(const Dims &dm, const void *Wo, const Saved &sv, float *Y, cudaStream_t s) {
+    if (use_tc(dm)) return tc_out(dm, Wo, sv, Y, s);
     return dm.bf16 ? out_t<bf16>(dm, Wo, sv, Y, s) : out_t<float>(dm, Wo, sv, Y, s);
 }
 
 cudaError_t launch_out_bwd(const Dims &dm, const void *Wo, const void *dY, const Saved &sv,
                            float *dWo, cudaStream_t s) {
+    if (use_tc(dm)) return tc_out_bwd(dm, Wo, dY, sv, dWo, s);
     return dm.bf16 ? out_bwd_t<bf16>(dm, Wo, dY, sv, dWo, s) : out_bwd_t<float>(dm, Wo, dY, sv, dWo, s);
 }
 
 cudaError_t launch_in_bwd(const Dims &dm, const void *Wq, const void *Wk, const void *Wv,
                           const void *Wr, const Saved &sv, float *dX, cudaStream_t s) {
+    if (use_tc(dm)) return tc_in_bwd(dm, Wq, Wk, Wv, Wr, sv, dX, s);
     return dm.bf16 ? in_bwd_t<bf16>(dm, Wq, Wk, Wv, Wr, sv, dX, s)
                    : in_bwd_t<float>(dm, Wq, Wk, Wv, Wr, sv, dX, s);
 }
 
 cudaError_t launch_w_bwd(const Dims &dm, const void *X, const Saved &sv, float *dWq, float *dWk,
                          float *dWv, float *dWr, cudaStream_t s) {
+    if (use_tc(dm)) {
+        cudaError_t e = tc_w_bwd(dm, X, sv, dWq, dWk, dWv, s);
+        if (e != cudaSuccess) return e;
+        return dwr_t<bf16>(dm, X, sv, dWr, s);
+    }
     return dm.bf16 ? w_bwd_t<bf16>(dm, X, sv, dWq, dWk, dWv, dWr, s)
                    : w_bwd_t<float>(dm, X, sv, dWq, dWk, dWv, dWr, s);
 }

@@ -1,0 +1,596 @@
+// Per-head projections of the MoSA layer on the 5th-generation tensor cores
+// (tcgen05.mma, fp32 accumulators in TMEM), operands staged by TMA, with the
+// gathers through the selected token indices done by TMA gather4 loads.
+//
+// One CTA computes one 128-row output tile of one head (or one split of the
+// reduction for the weight gradients).  Warp roles (256 threads):
+//   warp 0      producer: TMA tile / gather4 loads into a STAGES-deep ring
+//   warp 1      MMA issuer (one thread): tcgen05.mma per 16-wide K step
+//   warp 2      TMEM allocator
+//   warps 4-7   epilogue: tcgen05.ld of the accumulator rows, fused output
+// Every mbarrier wait is bounded; a wait that runs out sets kStatusTimeout in
+// the workspace status word and the CTA winds down without hanging.
+//
+// Variants (bf16 inputs, head size 64; intermediates are bf16 hi/lo pairs, so
+// a product with one is two MMAs into the same accumulator):
+//   kQKV  F3  [Q|K|V](m,:)  = X[g(m),:] W_{q|k|v}[h]        A gathered K-major, B MN-major
+//   kOUT  F5  Y[g(m),n]    += (diag(r) A)(m,:) W_o[h](:,n)   A = AR pair,  B MN-major
+//   kG    B1  G(m,:)        = dY[g(m),:] W_o[h]^T, then dr, dA = r G, D, dlogit in the epilogue
+//   kDWO  B1  dW_o[h](p,c)  = sum_m AR(m,p) dY[g(m),c]       A gathered MN-major, B = AR pair
+//   kDX   B3  dX[g(m),n]   += dQKV(m,:) [W_q|W_k|W_v][h]^T(:,n) + dlogit(m) W_r[n,h]
+//   kDW   B4  dW_{q|k|v}[h](c,p) = sum_m X[g(m),c] dQKV(m,p) A gathered MN-major, B = dQKV pair
+// where g(m) = b*T + I[b,h,i] for row m = b*k + i of head h.
+#include <cudaTypedefs.h>
+
+#include <cstdio>
+#include <mutex>
+
+#include "launch.h"
+#include "profile.h"
+#include "tc_common.cuh"
+
+namespace mosa {
+namespace {
+
+using namespace tc;
+
+enum Kind : int { kQKV = 0, kOUT, kG, kDWO, kDX, kDW };
+
+constexpr int kBM = 128;        // rows per tile (TMEM lanes)
+constexpr int kBK = 64;         // K per stage: one 128-byte swizzle row of bf16
+constexpr int kTile8K = 8192;   // one 64x64 bf16 block
+constexpr int kTile16K = 16384; // one 128x64 bf16 block
+constexpr int kThreads = 256;
+
+template <int KIND>
+struct Cfg;
+template <>
+struct Cfg<kQKV> {
+    static constexpr int BN = 192, STAGES = 4, A_BYTES = kTile16K, B_BYTES = 3 * kTile8K,
+                         TMEM_COLS = 256;
+    static constexpr bool A_MN = false, B_MN = true, A_PAIR = false, B_PAIR = false;
+};
+template <>
+struct Cfg<kOUT> {
+    static constexpr int BN = 256, STAGES = 1, A_BYTES = 2 * kTile16K, B_BYTES = 4 * kTile8K,
+                         TMEM_COLS = 256;
+    static constexpr bool A_MN = false, B_MN = true, A_PAIR = true, B_PAIR = false;
+};
+template <>
+struct Cfg<kG> {
+    static constexpr int BN = 64, STAGES = 4, A_BYTES = kTile16K, B_BYTES = kTile8K,
+                         TMEM_COLS = 64;
+    static constexpr bool A_MN = false, B_MN = false, A_PAIR = false, B_PAIR = false;
+};
+template <>
+struct Cfg<kDWO> {
+    static constexpr int BN = 64, STAGES = 4, A_BYTES = kTile16K, B_BYTES = 2 * kTile8K,
+                         TMEM_COLS = 64;
+    static constexpr bool A_MN = true, B_MN = true, A_PAIR = false, B_PAIR = true;
+};
+template <>
+struct Cfg<kDX> {
+    static constexpr int BN = 256, STAGES = 3, A_BYTES = 2 * kTile16K, B_BYTES = 32768,
+                         TMEM_COLS = 256;
+    static constexpr bool A_MN = false, B_MN = false, A_PAIR = true, B_PAIR = false;
+};
+template <>
+struct Cfg<kDW> {
+    static constexpr int BN = 192, STAGES = 3, A_BYTES = kTile16K, B_BYTES = 6 * kTile8K,
+                         TMEM_COLS = 256;
+    static constexpr bool A_MN = true, B_MN = true, A_PAIR = false, B_PAIR = true;
+};
+
+template <int KIND>
+constexpr int smem_bytes() {
+    return 1024 /* alignment slack */ + Cfg<KIND>::STAGES * (Cfg<KIND>::A_BYTES + Cfg<KIND>::B_BYTES) +
+           1024 /* barriers, row indices */;
+}
+
+struct TcParams {
+    CUtensorMap mapA;      // gathered source (2-D, box 64x1) or per-head tile map (3-D)
+    CUtensorMap mapB[3];   // per-head tile maps of the B operand
+    int M;                 // output rows per head: B*k for row kinds, d for kDWO / kDW
+    int Mtok;              // selected rows per head, B*k
+    int N;                 // output columns (d for kOUT / kDX)
+    int nkb;               // K blocks in the whole reduction
+    int splits;            // reduction splits (kDWO / kDW)
+    int d, H;
+    const int32_t *gidx;   // [H, B*k]
+    const float *rsel;     // [H, B*k]
+    const float *A32;      // [H, B*k, 64] attention output (kG)
+    const float *dlogit;   // [H, B*k] (kDX reads, kG writes via out_f1)
+    const bf16 *Wr;        // [d, H] (kDX)
+    void *out[3];          // Q/K/V pairs (kQKV), dA pair (kG)
+    float *out_f;          // Y (kOUT), dW_o (kDWO), dX (kDX), dW_q (kDW)
+    float *out_f1;         // Dd (kG), dW_k (kDW)
+    float *out_f2;         // dlogit (kG), dW_v (kDW)
+    uint32_t *status;
+};
+
+__device__ __forceinline__ void store_pair_row32(bf16 *row_hi, bf16 *row_lo, const float (&v)[32]) {
+    // v -> hi = bf16(v), lo = bf16(v - hi); 32 values each, four 16-byte stores per half
+#pragma unroll
+    for (int q = 0; q < 4; ++q) {
+        uint32_t h4[4], l4[4];
+#pragma unroll
+        for (int e = 0; e < 4; ++e) {
+            const float a = v[q * 8 + 2 * e], b = v[q * 8 + 2 * e + 1];
+            const bf16 ha = __float2bfloat16_rn(a), hb = __float2bfloat16_rn(b);
+            const bf16 la = __float2bfloat16_rn(a - __bfloat162float(ha));
+            const bf16 lb = __float2bfloat16_rn(b - __bfloat162float(hb));
+            h4[e] = (uint32_t)__bfloat16_as_ushort(ha) | ((uint32_t)__bfloat16_as_ushort(hb) << 16);
+            l4[e] = (uint32_t)__bfloat16_as_ushort(la) | ((uint32_t)__bfloat16_as_ushort(lb) << 16);
+        }
+        reinterpret_cast<uint4 *>(row_hi)[q] = make_uint4(h4[0], h4[1], h4[2], h4[3]);
+        reinterpret_cast<uint4 *>(row_lo)[q] = make_uint4(l4[0], l4[1], l4[2], l4[3]);
+    }
+}
+
+template <int KIND>
+__global__ void __launch_bounds__(kThreads, 1) tc_gemm_kernel(const __grid_constant__ TcParams p) {
+    using C = Cfg<KIND>;
+    constexpr int S = C::STAGES;
+    extern __shared__ uint8_t smem_raw[];
+    uint8_t *smem = reinterpret_cast<uint8_t *>(
+        (reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
+    uint8_t *sA = smem;
+    uint8_t *sB = smem + S * C::A_BYTES;
+    uint64_t *bars = reinterpret_cast<uint64_t *>(sB + S * C::B_BYTES);
+    uint64_t *full = bars, *empty = bars + S, *done = bars + 2 * S;
+    uint32_t *tmem_slot = reinterpret_cast<uint32_t *>(done + 1);
+    int *s_abort = reinterpret_cast<int *>(tmem_slot + 1);
+    int *s_rows = s_abort + 1 + 2;  // 128 gather rows, 16-byte aligned below
+    s_rows = reinterpret_cast<int *>((reinterpret_cast<uintptr_t>(s_rows) + 15) & ~uintptr_t(15));
+
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    const int m_tile = blockIdx.x, n_tile = blockIdx.y;
+    const int h = (KIND == kDWO || KIND == kDW) ? blockIdx.z / p.splits : blockIdx.z;
+    const int split = (KIND == kDWO || KIND == kDW) ? blockIdx.z % p.splits : 0;
+    const int m0 = m_tile * kBM;
+    const int n0 = n_tile * C::BN;
+    int kb_begin = 0, kb_end = p.nkb;
+    if (KIND == kDWO || KIND == kDW) {
+        const int per = (p.nkb + p.splits - 1) / p.splits;
+        kb_begin = split * per;
+        kb_end = min(p.nkb, kb_begin + per);
+    }
+    const int nkb = kb_end - kb_begin;
+
+    if (threadIdx.x == 0) {
+        for (int s = 0; s < S; ++s) {
+            mbar_init(smem_u32(&full[s]), 1);
+            mbar_init(smem_u32(&empty[s]), 1);
+        }
+        mbar_init(smem_u32(done), 1);
+        *s_abort = 0;
+        fence_barrier_init();
+    }
+    if (KIND == kQKV || KIND == kG) {
+        for (int r = threadIdx.x; r < kBM; r += kThreads) {
+            const int m = m0 + r;
+            s_rows[r] = m < p.Mtok ? p.gidx[(size_t)h * p.Mtok + m] : 0;
+        }
+    }
+    if (warp == 2) {
+        tmem_alloc(smem_u32(tmem_slot), C::TMEM_COLS);
+        tmem_relinquish();
+    }
+    tc_fence_before();
+    __syncthreads();
+    tc_fence_after();
+    const uint32_t tmem = *tmem_slot;
+
+    if (warp == 0) {
+        // ------------------------------------------------------- producer
+        int issued = 0;
+        for (int it = 0; it < nkb; ++it) {
+            const int s = it % S;
+            const uint32_t fb = smem_u32(&full[s]);
+            bool ok = true;
+            if (lane == 0) ok = mbar_wait(smem_u32(&empty[s]), ((it / S) & 1) ^ 1);
+            ok = __shfl_sync(0xffffffffu, ok ? 1 : 0, 0) != 0;
+            if (!ok || *(volatile int *)s_abort) {
+                if (lane == 0) {
+                    atomicOr(p.status, kStatusTimeout);
+                    *(volatile int *)s_abort = 1;
+                }
+                break;
+            }
+            const int kb = kb_begin + it;
+            const uint32_t a = smem_u32(sA + s * C::A_BYTES), b = smem_u32(sB + s * C::B_BYTES);
+            if (lane == 0) mbar_expect_tx(fb, C::A_BYTES + C::B_BYTES);
+            __syncwarp();
+            if constexpr (KIND == kQKV || KIND == kG) {
+                const int4 r4 = reinterpret_cast<const int4 *>(s_rows)[lane];
+                tma_gather4(a + lane * 512, &p.mapA, fb, kb * kBK, r4.x, r4.y, r4.z, r4.w);
+                if (KIND == kQKV && lane < 3) tma_load_3d(b + lane * kTile8K, &p.mapB[lane], fb, 0, kb * kBK, h);
+                if (KIND == kG && lane == 0) tma_load_3d(b, &p.mapB[0], fb, kb * kBK, 0, h);
+            } else if constexpr (KIND == kOUT) {
+                if (lane == 0) tma_load_3d(a, &p.mapA, fb, 0, m0, h);
+                if (lane == 1) tma_load_3d(a + kTile16K, &p.mapA, fb, 64, m0, h);
+                if (lane >= 2 && lane < 6)
+                    tma_load_3d(b + (lane - 2) * kTile8K, &p.mapB[0], fb, n0 + 64 * (lane - 2), 0, h);
+            } else if constexpr (KIND == kDX) {
+                if (lane == 0) tma_load_3d(a, &p.mapA, fb, 64 * kb, m0, h);
+                if (lane == 1) tma_load_3d(a + kTile16K, &p.mapA, fb, 192 + 64 * kb, m0, h);
+                if (lane == 2) tma_load_3d(b, &p.mapB[kb], fb, 0, n0, h);
+            } else {  // kDWO, kDW: tokens along K, gathered; two 64-wide column blocks of A
+                const int j = lane >> 4, g = lane & 15;
+                const int t0 = kb * kBK + 4 * g;
+                const int32_t *gi = p.gidx + (size_t)h * p.Mtok;
+                const int r0 = t0 + 0 < p.Mtok ? gi[t0 + 0] : 0;
+                const int r1 = t0 + 1 < p.Mtok ? gi[t0 + 1] : 0;
+                const int r2 = t0 + 2 < p.Mtok ? gi[t0 + 2] : 0;
+                const int r3 = t0 + 3 < p.Mtok ? gi[t0 + 3] : 0;
+                tma_gather4(a + j * kTile8K + g * 512, &p.mapA, fb, m0 + 64 * j, r0, r1, r2, r3);
+                if constexpr (KIND == kDWO) {
+                    if (lane < 2) tma_load_3d(b + lane * kTile8K, &p.mapB[0], fb, 64 * lane, kb * kBK, h);
+                } else {
+                    if (lane < 6)
+                        tma_load_3d(b + lane * kTile8K, &p.mapB[0], fb,
+                                    (lane < 3 ? 0 : 192) + 64 * (lane % 3), kb * kBK, h);
+                }
+            }
+            issued = it + 1;
+        }
+        if (*(volatile int *)s_abort && lane == 0) {
+            // Let copies already in flight land before the CTA can exit.
+            for (int it = max(0, issued - S); it < issued; ++it)
+                mbar_wait(smem_u32(&full[it % S]), (it / S) & 1);
+        }
+    } else if (warp == 1) {
+        // ------------------------------------------------------ MMA issuer
+        if (lane == 0) {
+            constexpr uint32_t idesc = idesc_bf16(kBM, C::BN, C::A_MN, C::B_MN);
+            for (int it = 0; it < nkb; ++it) {
+                const int s = it % S;
+                if (!mbar_wait(smem_u32(&full[s]), (it / S) & 1) || *(volatile int *)s_abort) {
+                    atomicOr(p.status, kStatusTimeout);
+                    *(volatile int *)s_abort = 1;
+                    break;
+                }
+                tc_fence_after();
+                const uint32_t a = smem_u32(sA + s * C::A_BYTES), b = smem_u32(sB + s * C::B_BYTES);
+                constexpr int pairs = (C::A_PAIR || C::B_PAIR) ? 2 : 1;
+#pragma unroll
+                for (int half = 0; half < pairs; ++half) {
+                    const uint32_t ah = a + (C::A_PAIR ? half * (C::A_BYTES / 2) : 0);
+                    const uint32_t bh = b + (C::B_PAIR ? half * (C::B_BYTES / 2) : 0);
+#pragma unroll
+                    for (int j = 0; j < kBK / 16; ++j) {
+                        const uint64_t ad = C::A_MN ? smem_desc_sw128(ah + j * 2048, kTile8K, 1024)
+                                                    : smem_desc_sw128(ah + j * 32, 16, 1024);
+                        const uint64_t bd = C::B_MN ? smem_desc_sw128(bh + j * 2048, kTile8K, 1024)
+                                                    : smem_desc_sw128(bh + j * 32, 16, 1024);
+                        mma_bf16(tmem, ad, bd, idesc, (it > 0 || half > 0 || j > 0) ? 1u : 0u);
+                    }
+                }
+                mma_commit(smem_u32(&empty[s]));
+            }
+            mma_commit(smem_u32(done));
+        }
+    } else if (warp >= 4) {
+        // -------------------------------------------------------- epilogue
+        const int q = warp - 4;
+        const int r = q * 32 + lane;
+        const int mg = m0 + r;
+        const bool ok = mbar_wait(smem_u32(done), 0);
+        tc_fence_after();
+        const bool abort = !ok || *(volatile int *)s_abort || nkb <= 0;
+        if (!ok && lane == 0) atomicOr(p.status, kStatusTimeout);
+        const uint32_t tb = tmem + ((uint32_t)(q * 32) << 16);
+        if constexpr (KIND == kQKV) {
+            const size_t row = (size_t)h * p.Mtok + mg;
+#pragma unroll 1
+            for (int c0 = 0; c0 < C::BN; c0 += 32) {
+                float v[32];
+                tmem_ld32(tb + c0, v);
+                if (!abort && mg < p.M) {
+                    bf16 *base = static_cast<bf16 *>(p.out[c0 / 64]) + row * 128 + (c0 % 64);
+                    store_pair_row32(base, base + 64, v);
+                }
+            }
+        } else if constexpr (KIND == kOUT || KIND == kDX) {
+            const bool live = !abort && mg < p.M;
+            const size_t row = (size_t)h * p.Mtok + (live ? mg : 0);
+            float *dst = p.out_f + (size_t)p.gidx[row] * p.d;
+            const float dl = (KIND == kDX && live) ? p.dlogit[row] : 0.f;
+#pragma unroll 1
+            for (int c0 = 0; c0 < C::BN; c0 += 32) {
+                float v[32];
+                tmem_ld32(tb + c0, v);
+                if (!live) continue;
+#pragma unroll
+                for (int e = 0; e < 32; e += 4) {
+                    const int n = n0 + c0 + e;
+                    if (n < p.d) {
+                        if (KIND == kDX) {
+#pragma unroll
+                            for (int u = 0; u < 4; ++u)
+                                v[e + u] = fmaf(dl, __bfloat162float(p.Wr[(size_t)(n + u) * p.H + h]), v[e + u]);
+                        }
+                        red_add_v4(dst + n, v[e], v[e + 1], v[e + 2], v[e + 3]);
+                    }
+                }
+            }
+        } else if constexpr (KIND == kG) {
+            float g[64];
+            float lo[32];
+            tmem_ld32(tb, lo);
+#pragma unroll
+            for (int e = 0; e < 32; ++e) g[e] = lo[e];
+            tmem_ld32(tb + 32, lo);
+#pragma unroll
+            for (int e = 0; e < 32; ++e) g[32 + e] = lo[e];
+            if (!abort && mg < p.M) {
+                const size_t row = (size_t)h * p.Mtok + mg;
+                const float rr = p.rsel[row];
+                const float4 *arow = reinterpret_cast<const float4 *>(p.A32 + row * 64);
+                float dr = 0.f, dd = 0.f;
+#pragma unroll
+                for (int e4 = 0; e4 < 16; ++e4) {
+                    const float4 a4 = arow[e4];
+                    dr = fmaf(a4.x, g[4 * e4 + 0], dr);
+                    dr = fmaf(a4.y, g[4 * e4 + 1], dr);
+                    dr = fmaf(a4.z, g[4 * e4 + 2], dr);
+                    dr = fmaf(a4.w, g[4 * e4 + 3], dr);
+                }
+                // dA = r G (kept as a bf16 pair); D = rowsum(dA o A) = r dr
+#pragma unroll
+                for (int e = 0; e < 64; ++e) g[e] *= rr;
+                dd = rr * dr;
+                bf16 *base = static_cast<bf16 *>(p.out[0]) + row * 128;
+                float half[32];
+#pragma unroll
+                for (int e = 0; e < 32; ++e) half[e] = g[e];
+                store_pair_row32(base, base + 64, half);
+#pragma unroll
+                for (int e = 0; e < 32; ++e) half[e] = g[32 + e];
+                store_pair_row32(base + 32, base + 96, half);
+                p.out_f1[row] = dd;
+                p.out_f2[row] = dr * rr * (1.f - rr);
+            }
+        } else if constexpr (KIND == kDWO) {
+            const bool live = !abort && mg < p.M;
+#pragma unroll 1
+            for (int c0 = 0; c0 < 64; c0 += 32) {
+                float v[32];
+                tmem_ld32(tb + c0, v);
+                if (!live) continue;
+                float *dst = p.out_f + ((size_t)h * 64 + c0) * p.d + mg;
+#pragma unroll
+                for (int e = 0; e < 32; ++e) {
+                    if (p.splits > 1)
+                        atomicAdd(dst + (size_t)e * p.d, v[e]);
+                    else
+                        dst[(size_t)e * p.d] = v[e];
+                }
+            }
+        } else {  // kDW
+            const bool live = !abort && mg < p.M;
+#pragma unroll 1
+            for (int c0 = 0; c0 < 192; c0 += 32) {
+                float v[32];
+                tmem_ld32(tb + c0, v);
+                if (!live) continue;
+                float *W = c0 < 64 ? p.out_f : (c0 < 128 ? p.out_f1 : p.out_f2);
+                float *dst = W + ((size_t)h * p.d + mg) * 64 + (c0 % 64);
+#pragma unroll
+                for (int e = 0; e < 32; e += 4) {
+                    if (p.splits > 1)
+                        red_add_v4(dst + e, v[e], v[e + 1], v[e + 2], v[e + 3]);
+                    else
+                        *reinterpret_cast<float4 *>(dst + e) = make_float4(v[e], v[e + 1], v[e + 2], v[e + 3]);
+                }
+            }
+        }
+    }
+    tc_fence_before();
+    __syncthreads();
+    if (warp == 2) {
+        tc_fence_after();
+        tmem_dealloc(tmem, C::TMEM_COLS);
+    }
+}
+
+// ------------------------------------------------------------------ host
+
+PFN_cuTensorMapEncodeTiled_v12000 encode_fn() {
+    static PFN_cuTensorMapEncodeTiled_v12000 fn = nullptr;
+    static std::once_flag once;
+    std::call_once(once, [] {
+        void *ptr = nullptr;
+        cudaDriverEntryPointQueryResult q;
+        if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &ptr, 12000,
+                                             cudaEnableDefault, &q) == cudaSuccess &&
+            q == cudaDriverEntryPointSuccess)
+            fn = reinterpret_cast<PFN_cuTensorMapEncodeTiled_v12000>(ptr);
+    });
+    return fn;
+}
+
+// bf16 tensor map with 128-byte swizzle.  dims innermost first; strides in
+// bytes for dims 1..rank-1; box innermost first.
+bool make_map(CUtensorMap *m, const void *base, int rank, const uint64_t *dims,
+              const uint64_t *strides, const uint32_t *box) {
+    auto fn = encode_fn();
+    if (!fn) return false;
+    cuuint64_t gd[3], gs[2];
+    cuuint32_t bx[3], es[3] = {1, 1, 1};
+    for (int i = 0; i < rank; ++i) {
+        gd[i] = dims[i];
+        bx[i] = box[i];
+    }
+    for (int i = 0; i < rank - 1; ++i) gs[i] = strides[i];
+    CUresult r = fn(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, (cuuint32_t)rank, const_cast<void *>(base),
+                    gd, gs, bx, es, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+                    CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+    return r == CUDA_SUCCESS;
+}
+
+// Rows of a [rows, cols] bf16 matrix fetched one row (64 columns) at a time by gather4.
+bool map_gather(CUtensorMap *m, const void *base, uint64_t rows, uint64_t cols) {
+    const uint64_t dims[2] = {cols, rows}, strides[1] = {cols * 2};
+    const uint32_t box[2] = {64, 1};
+    return make_map(m, base, 2, dims, strides, box);
+}
+
+// Per-head tiles of a [H, rows, cols] bf16 array: box {64, box_rows, 1}.
+bool map_heads(CUtensorMap *m, const void *base, uint64_t H, uint64_t rows, uint64_t cols,
+               uint32_t box_rows) {
+    const uint64_t dims[3] = {cols, rows, H}, strides[2] = {cols * 2, rows * cols * 2};
+    const uint32_t box[3] = {64, box_rows, 1};
+    return make_map(m, base, 3, dims, strides, box);
+}
+
+template <int KIND>
+cudaError_t launch_kind(const TcParams &p, dim3 grid, cudaStream_t s) {
+    constexpr int smem = smem_bytes<KIND>();
+    static std::once_flag once;
+    static cudaError_t attr = cudaSuccess;
+    std::call_once(once, [] {
+        attr = cudaFuncSetAttribute(tc_gemm_kernel<KIND>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                    smem);
+    });
+    if (attr != cudaSuccess) return attr;
+    tc_gemm_kernel<KIND><<<grid, kThreads, smem, s>>>(p);
+    note_launches(1);
+    return cudaGetLastError();
+}
+
+int splits_for(int tiles, int nkb) {
+    // enough CTAs to cover the 152 SMs at least once, each with >= 2 K blocks
+    int sp = 1;
+    while (tiles * sp < 152 && sp * 2 <= nkb / 2) sp *= 2;
+    return sp;
+}
+
+TcParams base_params(const Dims &dm, const Saved &sv) {
+    TcParams p;
+    memset(&p, 0, sizeof(p));
+    p.Mtok = dm.B * dm.k;
+    p.d = dm.d;
+    p.H = dm.H;
+    p.gidx = sv.gidx;
+    p.rsel = sv.rsel;
+    p.status = sv.status;
+    p.splits = 1;
+    return p;
+}
+
+}  // namespace
+
+bool tc_supported(const Dims &dm) {
+    return dm.bf16 && dm.hp == 64 && encode_fn() != nullptr;
+}
+
+cudaError_t tc_qkv(const Dims &dm, const void *X, const void *Wq, const void *Wk, const void *Wv,
+                   const Saved &sv, cudaStream_t s) {
+    TcParams p = base_params(dm, sv);
+    p.M = p.Mtok;
+    p.nkb = (dm.d + kBK - 1) / kBK;
+    bool ok = map_gather(&p.mapA, X, (uint64_t)dm.B * dm.T, dm.d);
+    const void *W[3] = {Wq, Wk, Wv};
+    for (int j = 0; j < 3; ++j) ok = ok && map_heads(&p.mapB[j], W[j], dm.H, dm.d, 64, 64);
+    if (!ok) return cudaErrorInvalidValue;
+    p.out[0] = sv.Q;
+    p.out[1] = sv.K;
+    p.out[2] = sv.V;
+    dim3 grid((p.M + kBM - 1) / kBM, 1, dm.H);
+    return launch_kind<kQKV>(p, grid, s);
+}
+
+cudaError_t tc_out(const Dims &dm, const void *Wo, const Saved &sv, float *Y, cudaStream_t s) {
+    cudaError_t e = cudaMemsetAsync(Y, 0, sizeof(float) * (size_t)dm.B * dm.T * dm.d, s);
+    if (e != cudaSuccess) return e;
+    TcParams p = base_params(dm, sv);
+    p.M = p.Mtok;
+    p.N = dm.d;
+    p.nkb = 1;
+    bool ok = map_heads(&p.mapA, sv.AR, dm.H, p.Mtok, 128, 128) &&
+              map_heads(&p.mapB[0], Wo, dm.H, 64, dm.d, 64);
+    if (!ok) return cudaErrorInvalidValue;
+    p.out_f = Y;
+    dim3 grid((p.M + kBM - 1) / kBM, (dm.d + 255) / 256, dm.H);
+    return launch_kind<kOUT>(p, grid, s);
+}
+
+cudaError_t tc_out_bwd(const Dims &dm, const void *Wo, const void *dY, const Saved &sv,
+                       float *dWo, cudaStream_t s) {
+    // G = dY[I] W_o^T with the row terms fused into the epilogue.
+    TcParams p = base_params(dm, sv);
+    p.M = p.Mtok;
+    p.nkb = (dm.d + kBK - 1) / kBK;
+    bool ok = map_gather(&p.mapA, dY, (uint64_t)dm.B * dm.T, dm.d) &&
+              map_heads(&p.mapB[0], Wo, dm.H, 64, dm.d, 64);
+    if (!ok) return cudaErrorInvalidValue;
+    p.A32 = sv.A;
+    p.out[0] = sv.dA;
+    p.out_f1 = sv.Dd;
+    p.out_f2 = sv.dlogit;
+    dim3 grid((p.M + kBM - 1) / kBM, 1, dm.H);
+    cudaError_t e = launch_kind<kG>(p, grid, s);
+    if (e != cudaSuccess) return e;
+    // dW_o[h](p, c) = sum_m AR(m, p) dY[g(m), c]
+    TcParams q = base_params(dm, sv);
+    q.M = dm.d;
+    q.nkb = (q.Mtok + kBK - 1) / kBK;
+    const int tiles = (dm.d + kBM - 1) / kBM * dm.H;
+    q.splits = splits_for(tiles, q.nkb);
+    ok = map_gather(&q.mapA, dY, (uint64_t)dm.B * dm.T, dm.d) &&
+         map_heads(&q.mapB[0], sv.AR, dm.H, q.Mtok, 128, 64);
+    if (!ok) return cudaErrorInvalidValue;
+    q.out_f = dWo;
+    if (q.splits > 1) {
+        e = cudaMemsetAsync(dWo, 0, sizeof(float) * (size_t)dm.H * 64 * dm.d, s);
+        if (e != cudaSuccess) return e;
+    }
+    dim3 grid2((dm.d + kBM - 1) / kBM, 1, dm.H * q.splits);
+    return launch_kind<kDWO>(q, grid2, s);
+}
+
+cudaError_t tc_in_bwd(const Dims &dm, const void *Wq, const void *Wk, const void *Wv,
+                      const void *Wr, const Saved &sv, float *dX, cudaStream_t s) {
+    cudaError_t e = cudaMemsetAsync(dX, 0, sizeof(float) * (size_t)dm.B * dm.T * dm.d, s);
+    if (e != cudaSuccess) return e;
+    TcParams p = base_params(dm, sv);
+    p.M = p.Mtok;
+    p.N = dm.d;
+    p.nkb = 3;
+    const void *W[3] = {Wq, Wk, Wv};
+    bool ok = map_heads(&p.mapA, sv.dQKV, dm.H, p.Mtok, 384, 128);
+    for (int j = 0; j < 3; ++j) ok = ok && map_heads(&p.mapB[j], W[j], dm.H, dm.d, 64, 256);
+    if (!ok) return cudaErrorInvalidValue;
+    p.dlogit = sv.dlogit;
+    p.Wr = static_cast<const bf16 *>(Wr);
+    p.out_f = dX;
+    dim3 grid((p.M + kBM - 1) / kBM, (dm.d + 255) / 256, dm.H);
+    return launch_kind<kDX>(p, grid, s);
+}
+
+cudaError_t tc_w_bwd(const Dims &dm, const void *X, const Saved &sv, float *dWq, float *dWk,
+                     float *dWv, cudaStream_t s) {
+    TcParams p = base_params(dm, sv);
+    p.M = dm.d;
+    p.nkb = (p.Mtok + kBK - 1) / kBK;
+    const int tiles = (dm.d + kBM - 1) / kBM * dm.H;
+    p.splits = splits_for(tiles, p.nkb);
+    bool ok = map_gather(&p.mapA, X, (uint64_t)dm.B * dm.T, dm.d) &&
+              map_heads(&p.mapB[0], sv.dQKV, dm.H, p.Mtok, 384, 64);
+    if (!ok) return cudaErrorInvalidValue;
+    p.out_f = dWq;
+    p.out_f1 = dWk;
+    p.out_f2 = dWv;
+    if (p.splits > 1) {
+        const size_t n = sizeof(float) * (size_t)dm.H * dm.d * 64;
+        cudaError_t e;
+        if ((e = cudaMemsetAsync(dWq, 0, n, s)) != cudaSuccess) return e;
+        if ((e = cudaMemsetAsync(dWk, 0, n, s)) != cudaSuccess) return e;
+        if ((e = cudaMemsetAsync(dWv, 0, n, s)) != cudaSuccess) return e;
+    }
+    dim3 grid((dm.d + kBM - 1) / kBM, 1, dm.H * p.splits);
+    return launch_kind<kDW>(p, grid, s);
+}
+
+}  // namespace mosa

@@ -7,6 +7,8 @@ workload sizes are compared on sampled units the oracle computes exactly
 (every head of one sequence for Y and dX, every sequence of one head for the
 weight gradients) plus every selected index.
 """
+import os
+
 import numpy as np
 import pytest
 import torch
@@ -70,8 +72,19 @@ SMALL = [
 ]
 
 
+@pytest.fixture(params=["default", "simt"])
+def kernel_path(request, monkeypatch):
+    """Run a test on the default kernels (tensor cores where the shape allows)
+    and again with the CUDA-core kernels forced."""
+    if request.param == "simt":
+        monkeypatch.setenv("MOSA_FORCE_SIMT", "1")
+    else:
+        monkeypatch.delenv("MOSA_FORCE_SIMT", raising=False)
+    return request.param
+
+
 @pytest.mark.parametrize("cfg", SMALL, ids=lambda c: c.name)
-def test_small_forward_backward_full_parity(cfg):
+def test_small_forward_backward_full_parity(cfg, kernel_path):
     x = W.make_inputs(cfg)
     Y, I, rs, rf = oracle.forward(x["X"], *weights(x), k=cfg.k)
     assert sigmoid_gap(rf, cfg.k) > 1e-3
@@ -124,9 +137,9 @@ def test_full_size_sampled_parity(cfg):
 
 # --------------------------------------------------- indices entry point ----
 
-@pytest.mark.parametrize("dtype", ["f32", "bf16"])
-def test_fixed_sparse_indices_entry(dtype):
-    cfg = W.MosaConfig("fixed", B=2, T=512, d=64, H=4, hp=32, k=64, dtype=dtype, seed=21)
+@pytest.mark.parametrize("dtype,hp", [("f32", 32), ("bf16", 32), ("bf16", 64)])
+def test_fixed_sparse_indices_entry(dtype, hp, kernel_path):
+    cfg = W.MosaConfig("fixed", B=2, T=512, d=64, H=4, hp=hp, k=64, dtype=dtype, seed=21)
     x = W.make_inputs(cfg, plant=False)
     I = W.fixed_sparse_indices(cfg.B, cfg.H, cfg.T, cfg.k)
     ones = np.ones((cfg.B, cfg.H, cfg.k), np.float32)

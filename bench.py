@@ -181,8 +181,6 @@ def stage_bound(stage, peaks, kind):
 
 
 def stage_kind(stage, lib_impl):
-    if stage in ("router", "select"):
-        return "mem"
     return lib_impl.get(stage, "simt")
 
 
@@ -209,6 +207,22 @@ def source_digest():
         with open(p, "rb") as f:
             h.update(f.read())
     return h.hexdigest()
+
+
+# ------------------------------------------------------------ multi-rank
+
+def combine_ranks(local_ms: float, tokens_per_rank: int, dist=None, device="cpu"):
+    """Whole-job throughput under weak scaling: every rank processes its own
+    batch, the job's time is the slowest rank's.  Returns (tokens/s, max ms)."""
+    world = 1
+    ms = float(local_ms)
+    if dist is not None and dist.is_initialized():
+        import torch
+        world = dist.get_world_size()
+        t = torch.tensor([ms], dtype=torch.float64, device=device)
+        dist.all_reduce(t, op=dist.ReduceOp.MAX)
+        ms = float(t.item())
+    return world * tokens_per_rank / (ms / 1e3), ms
 
 
 # ------------------------------------------------------------------ main
@@ -345,12 +359,7 @@ def main():
         sampler.mark(t_host0, t_host1)
         clocks = sampler.stop()
     total_ms = sum(s.elapsed_time(e) for s, e in zip(starts, ends))
-    if dist is not None:
-        t = torch.tensor([total_ms], dtype=torch.float64, device=dev)
-        dist.all_reduce(t, op=dist.ReduceOp.MAX)
-        total_ms = float(t.item())
-    tokens = world * cfg.B * cfg.T * K
-    value = tokens / (total_ms / 1e3)
+    value, total_ms = combine_ranks(total_ms, cfg.B * cfg.T * K, dist, dev)
 
     # End to end through the public API with pinned host buffers.
     hX = torch.from_numpy(x["X"]).to(tdt).pin_memory()
@@ -379,11 +388,7 @@ def main():
         e2e_step()
     e1.record()
     torch.cuda.synchronize()
-    e2e_ms = e0.elapsed_time(e1)
-    if dist is not None:
-        t = torch.tensor([e2e_ms], dtype=torch.float64, device=dev)
-        dist.all_reduce(t, op=dist.ReduceOp.MAX)
-        e2e_ms = float(t.item())
+    e2e_value, e2e_ms = combine_ranks(e0.elapsed_time(e1), cfg.B * cfg.T * e2e_steps, dist, dev)
     h2d = hX.numel() * hX.element_size() + hdY.numel() * hdY.element_size()
     d2h = hY.numel() * 4 + hdX.numel() * 4
 
@@ -396,7 +401,7 @@ def main():
     peaks, peak_src = load_peaks()
     work = flops.layer_work(cfg.B, cfg.T, cfg.d, cfg.H, cfg.hp, cfg.k,
                             elem_bytes=2 if cfg.dtype == "bf16" else 4)
-    impl = getattr(mosa, "stage_impl", lambda s: {})(shape)
+    impl = mosa.stage_impl(shape)
     kind = stage_kind(dominant, impl)
     bound, peak, unit = stage_bound(dominant, peaks, kind)
     dom_ms = dom[0] / max(dom[1], 1)
@@ -417,7 +422,7 @@ def main():
                      "ms_per_launch": dom_ms},
         "layer_tflops": layer_flops * world * K / (total_ms / 1e3) / 1e12,
         "stage_ms": {s: round(v, 5) for s, v in stage_ms.items()},
-        "e2e": {"value": world * cfg.B * cfg.T * e2e_steps / (e2e_ms / 1e3), "unit": "tokens/s",
+        "e2e": {"value": e2e_value, "unit": "tokens/s",
                 "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h,
                 "what": "pinned host X, dY -> device; forward+backward; Y, dX -> pinned host"},
         "gpu_launches": int(launches),

@@ -163,6 +163,11 @@ int32_t mosa_profile_read(double *total_ms, int32_t *count, int32_t max_stages);
 /* Name of a stage ("router", "select", ...; "unknown" if out of range). */
 const char *mosa_stage_name(int32_t stage);
 
+/* Which units the kernels of `stage` run on for `shape`, so that a timing can
+ * be set against the right roofline: 0 CUDA cores (fp32 FFMA), 1 tensor cores
+ * (tcgen05), 2 memory-bound data movement; -1 for an invalid shape or stage. */
+int32_t mosa_stage_engine(const mosa_shape *shape, int32_t stage);
+
 #ifdef __cplusplus
 }
 #endif

@@ -26,7 +26,7 @@ MOSA_BF16 = 1
 EXPORTED = ("mosa_status_string", "mosa_workspace_bytes", "mosa_forward",
             "mosa_forward_with_indices", "mosa_backward", "mosa_topk", "mosa_check_status",
             "mosa_kernel_launches", "mosa_profile_stages", "mosa_profile_read",
-            "mosa_stage_name")
+            "mosa_stage_name", "mosa_stage_engine")
 
 
 class MosaShape(ctypes.Structure):
@@ -89,6 +89,8 @@ def load(build_if_missing: bool = True) -> ctypes.CDLL:
         L.mosa_profile_read.restype = i32
         L.mosa_stage_name.argtypes = [i32]
         L.mosa_stage_name.restype = ctypes.c_char_p
+        L.mosa_stage_engine.argtypes = [sp, i32]
+        L.mosa_stage_engine.restype = i32
         _lib = L
         return L
 
@@ -287,3 +289,22 @@ def mosa_profile_read() -> dict:
     cnt = (ctypes.c_int32 * n)()
     m = L.mosa_profile_read(ms, cnt, n)
     return {mosa_stage_name(i): (ms[i], cnt[i]) for i in range(min(m, n))}
+
+
+_ENGINES = {0: "simt", 1: "tensor", 2: "mem"}
+
+
+def mosa_stage_engine(shape: MosaShape, stage: int) -> int:
+    return int(load().mosa_stage_engine(ctypes.byref(shape), int(stage)))
+
+
+def stage_impl(shape: MosaShape) -> dict:
+    """{stage name: "simt" | "tensor" | "mem"} for this shape."""
+    out = {}
+    for i in range(32):
+        if mosa_stage_name(i) == "unknown":
+            break
+        e = mosa_stage_engine(shape, i)
+        if e >= 0:
+            out[mosa_stage_name(i)] = _ENGINES[e]
+    return out

@@ -210,6 +210,21 @@ mosa_status mosa_topk(int32_t rows, int32_t T, int32_t k, const float *scores, i
                                      (cudaStream_t)stream));
 }
 
+int32_t mosa_stage_engine(const mosa_shape *shape, int32_t stage) {
+    Dims dm;
+    if (check_shape(shape, &dm) != MOSA_OK || stage < 0 || stage >= kNumStages) return -1;
+    switch (stage) {
+        case kStageRouter:
+        case kStageSelect: return 2;
+        case kStageQkv:
+        case kStageOut:
+        case kStageOutBwd:
+        case kStageInBwd:
+        case kStageWBwd: return use_tc(dm) ? 1 : 0;
+        default: return 0;  // attention: CUDA cores
+    }
+}
+
 mosa_status mosa_check_status(const mosa_shape *shape, void *workspace, void *stream) {
     Dims dm;
     mosa_status st = check_shape(shape, &dm);

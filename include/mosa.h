@@ -141,6 +141,27 @@ mosa_status mosa_topk(int32_t rows, int32_t T, int32_t k, const float *scores, i
 mosa_status mosa_check_status(const mosa_shape *shape, void *workspace, void *stream);
 
 
+/* Routing without a workspace: router scores r = sigmoid(X W_r) and TopK, the
+ * same I and r_sel as mosa_forward, for callers that cannot allocate device
+ * memory.  The paper has no counterpart; this exists for callers whose
+ * device heap belongs to someone else (a host application that hands out no
+ * buffers after start-up, a plug-in interface that passes only inputs and
+ * outputs) or that must never pay cudaMalloc's implicit synchronisation.
+ * It allocates nothing: the [B,H,T] scores live in a 4 MiB array compiled
+ * into the library (held on every GPU that loads it until the process
+ * exits), so B*H*T may be at most 1,048,576 (else MOSA_ERR_UNSUPPORTED).
+ *   X [B,T,d], W_r [d,H] : inputs (storage dtype); hp is validated but unused.
+ *   I [B,H,k] int32, r_sel [B,H,k] fp32 : outputs, as mosa_forward.
+ * The first call on a device looks up the array's device address (once per
+ * device, with that device current); make that first call before any stream
+ * capture.  All calls share the one array and the contents of the last call
+ * remain in it; nothing needs clearing, because each call writes every score
+ * it reads.  Calls whose GPU work overlaps (different streams or host
+ * threads without ordering) race on the array: order them on one stream.
+ * Returns MOSA_OK, MOSA_ERR_INVALID_ARG, MOSA_ERR_UNSUPPORTED or MOSA_ERR_CUDA. */
+mosa_status mosa_route_noalloc(const mosa_shape *shape, const void *X, const void *W_r,
+                               int32_t *I, float *r_sel, void *stream);
+
 /* ---- Measurement support (not part of the layer) ----------------------
  * Stages, in launch order: 0 router, 1 select, 2 qkv, 3 attn_fwd, 4 out,
  * 5 out_bwd, 6 attn_bwd, 7 in_bwd, 8 w_bwd (9 reserved).  These calls create

@@ -26,7 +26,7 @@ MOSA_BF16 = 1
 EXPORTED = ("mosa_status_string", "mosa_workspace_bytes", "mosa_forward",
             "mosa_forward_with_indices", "mosa_backward", "mosa_topk", "mosa_check_status",
             "mosa_kernel_launches", "mosa_profile_stages", "mosa_profile_read",
-            "mosa_stage_name", "mosa_stage_engine")
+            "mosa_stage_name", "mosa_stage_engine", "mosa_route_noalloc")
 
 
 class MosaShape(ctypes.Structure):
@@ -89,6 +89,8 @@ def load(build_if_missing: bool = True) -> ctypes.CDLL:
         L.mosa_profile_read.restype = i32
         L.mosa_stage_name.argtypes = [i32]
         L.mosa_stage_name.restype = ctypes.c_char_p
+        L.mosa_route_noalloc.argtypes = [sp, vp, vp, vp, vp, vp]
+        L.mosa_route_noalloc.restype = ctypes.c_int
         L.mosa_stage_engine.argtypes = [sp, i32]
         L.mosa_stage_engine.restype = i32
         _lib = L
@@ -308,3 +310,25 @@ def stage_impl(shape: MosaShape) -> dict:
         if e >= 0:
             out[mosa_stage_name(i)] = _ENGINES[e]
     return out
+
+
+def mosa_route_noalloc(X, W_r, k: int, hp: int = 64, out=None, stream=None):
+    """Router + TopK with no workspace (the library's own 4 MiB score array);
+    returns (I, r_sel).  For callers that cannot allocate device memory; the
+    output tensors may be passed preallocated in ``out``."""
+    torch = _torch()
+    B, T, d = X.shape
+    H = W_r.shape[1]
+    shape = MosaShape(B, T, d, H, int(hp), int(k), _dtype_code(X))
+    _same(X, ("W_r", W_r))
+    I = (out or {}).get("I")
+    rs = (out or {}).get("r_sel")
+    if I is None:
+        I = torch.empty((B, H, k), dtype=torch.int32, device=X.device)
+    if rs is None:
+        rs = torch.empty((B, H, k), dtype=torch.float32, device=X.device)
+    rc = load().mosa_route_noalloc(ctypes.byref(shape), _dev(X, "X"), _dev(W_r, "W_r"),
+                                   _dev(I, "I", torch.int32), _dev(rs, "r_sel", torch.float32),
+                                   _stream(stream))
+    _check(rc, "mosa_route_noalloc")
+    return I, rs

@@ -232,6 +232,7 @@ cudaError_t attn_bwd_dispatch(const Dims &dm, const Saved &sv, cudaStream_t s) {
 }  // namespace
 
 cudaError_t launch_attn_fwd(const Dims &dm, const Saved &sv, cudaStream_t s) {
+    if (use_tc(dm)) return tc_attn_fwd(dm, sv, s);
     return dm.bf16 ? attn_fwd_dispatch<SplitBF16>(dm, sv, s) : attn_fwd_dispatch<float>(dm, sv, s);
 }
 

@@ -220,8 +220,9 @@ int32_t mosa_stage_engine(const mosa_shape *shape, int32_t stage) {
         case kStageOut:
         case kStageOutBwd:
         case kStageInBwd:
-        case kStageWBwd: return use_tc(dm) ? 1 : 0;
-        default: return 0;  // attention: CUDA cores
+        case kStageWBwd:
+        case kStageAttnFwd: return use_tc(dm) ? 1 : 0;
+        default: return 0;  // attention backward: CUDA cores
     }
 }
 

@@ -237,6 +237,7 @@ cudaError_t launch_attn_fwd(const Dims &dm, const Saved &sv, cudaStream_t s) {
 }
 
 cudaError_t launch_attn_bwd(const Dims &dm, const Saved &sv, cudaStream_t s) {
+    if (use_tc(dm)) return tc_attn_bwd(dm, sv, s);
     return dm.bf16 ? attn_bwd_dispatch<SplitBF16>(dm, sv, s) : attn_bwd_dispatch<float>(dm, sv, s);
 }
 

@@ -63,6 +63,7 @@ cudaError_t tc_out_bwd(const Dims &dm, const void *Wo, const void *dY, const Sav
 cudaError_t tc_in_bwd(const Dims &dm, const void *Wq, const void *Wk, const void *Wv,
                       const void *Wr, const Saved &sv, float *dX, cudaStream_t s);
 cudaError_t tc_attn_fwd(const Dims &dm, const Saved &sv, cudaStream_t s);
+cudaError_t tc_attn_bwd(const Dims &dm, const Saved &sv, cudaStream_t s);
 cudaError_t tc_w_bwd(const Dims &dm, const void *X, const Saved &sv, float *dWq, float *dWk,
                      float *dWv, cudaStream_t s);
 

@@ -221,8 +221,9 @@ int32_t mosa_stage_engine(const mosa_shape *shape, int32_t stage) {
         case kStageOutBwd:
         case kStageInBwd:
         case kStageWBwd:
-        case kStageAttnFwd: return use_tc(dm) ? 1 : 0;
-        default: return 0;  // attention backward: CUDA cores
+        case kStageAttnFwd:
+        case kStageAttnBwd: return use_tc(dm) ? 1 : 0;
+        default: return 0;
     }
 }
 

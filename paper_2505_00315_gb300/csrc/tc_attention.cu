@@ -12,8 +12,16 @@
 // Q, K, V, P are bf16 hi/lo pairs (v ~ hi + lo), so each product is three
 // bf16 MMAs (hi*hi + hi*lo + lo*hi) into one fp32 accumulator, which keeps the
 // result at fp32-level accuracy.
+// Backward (B2), flash-style with P recomputed from the saved log-sum-exp,
+// D = rowsum(dA o A) and dS = P o (dP - D):
+//   dK/dV kernel, one CTA per (128-key tile, b, h), over 64-query blocks:
+//     S^T = K Q^T, dP^T = V dA^T, then dV += P^T dA, dK += dS^T Q
+//   dQ kernel, one CTA per (128-query tile, b, h), over 64-key blocks:
+//     S = Q K^T, dP = dA V^T, then dQ += dS K
+// The same shared-memory tile of Q (or dA, K) serves as a K-major operand in
+// one product and as an MN-major operand in the other.
 // Warp roles: 0 TMA producer, 1 MMA issuer, 2 TMEM allocator, 4-7 softmax
-// (one query row per thread).  All waits are bounded.
+// (one row per thread).  All waits are bounded.
 #include <cudaTypedefs.h>
 
 #include <mutex>
@@ -327,6 +335,405 @@ __global__ void __launch_bounds__(kThreads, 1) attn_fwd_tc_kernel(const __grid_c
     }
 }
 
+// ------------------------------------------------------------ backward
+
+constexpr int kKT = 128;                  // keys per dK/dV CTA
+constexpr int kQB = 64;                   // queries per block in the dK/dV loop
+constexpr int kHalf128 = 128 * 64 * 2;    // one half of a 128-row tile, 16 KB
+constexpr int kHalf64 = 64 * 64 * 2;      // one half of a 64-row tile, 8 KB
+
+struct DkvSmem {
+    uint8_t k[2][kHalf128];
+    uint8_t v[2][kHalf128];
+    uint8_t q[kStages][2][kHalf64];
+    uint8_t da[kStages][2][kHalf64];
+    uint8_t pt[2][kHalf128];              // P^T  [128 keys x 64 queries] pair
+    uint8_t dst[2][kHalf128];             // dS^T pair
+    uint64_t kv_full, st_full, p_ready, pd_done, acc_done;
+    uint64_t qa_full[kStages], qa_empty[kStages];
+    uint32_t tmem;
+    int abort;
+};
+constexpr int kDkvSmem = (int)sizeof(DkvSmem) + 1024;
+
+struct DqSmem {
+    uint8_t q[2][kHalf128];
+    uint8_t da[2][kHalf128];
+    uint8_t k[kStages][2][kHalf64];
+    uint8_t v[kStages][2][kHalf64];
+    uint8_t ds[2][kHalf128];              // dS [128 queries x 64 keys] pair
+    uint64_t qa_full, sp_full, ds_ready, ds_done, acc_done;
+    uint64_t kv_full[kStages], kv_empty[kStages];
+    uint32_t tmem;
+    int abort;
+};
+constexpr int kDqSmem = (int)sizeof(DqSmem) + 1024;
+
+struct BwdParams {
+    CUtensorMap mA0, mA1, mB0, mB1;   // dK/dV: K, V (128 rows), Q, dA (64 rows); dQ: Q, dA (128), K, V (64)
+    int k, Mtok;
+    float scale, scale_log2;
+    const float *lse, *Dd;            // [H, B*k]
+    bf16 *dQKV;                       // [H, B*k, 384] pair: dQ|dK|dV hi, then lo
+    uint32_t *status;
+};
+
+template <class SM>
+__device__ __forceinline__ void flag_timeout_b(SM &sm, uint32_t *status) {
+    atomicOr(status, kStatusTimeout);
+    *(volatile int *)&sm.abort = 1;
+}
+
+// Three split products D (+)= Ah Bh + Ah Bl + Al Bh over K = 64.
+__device__ __forceinline__ void mma_pair3(uint32_t d, uint32_t a_hi, uint32_t a_lo, uint32_t b_hi,
+                                          uint32_t b_lo, bool a_mn, bool b_mn, uint32_t idesc,
+                                          bool accumulate_first) {
+    const uint32_t aa[3] = {a_hi, a_hi, a_lo}, bb[3] = {b_hi, b_lo, b_hi};
+#pragma unroll
+    for (int t = 0; t < 3; ++t)
+#pragma unroll
+        for (int kk = 0; kk < 4; ++kk) {
+            const uint64_t ad = a_mn ? smem_desc_sw128(aa[t] + kk * 2048, 8192, 1024)
+                                     : smem_desc_sw128(aa[t] + kk * 32, 16, 1024);
+            const uint64_t bd = b_mn ? smem_desc_sw128(bb[t] + kk * 2048, 8192, 1024)
+                                     : smem_desc_sw128(bb[t] + kk * 32, 16, 1024);
+            mma_bf16(d, ad, bd, idesc, (accumulate_first || t > 0 || kk > 0) ? 1u : 0u);
+        }
+}
+
+__device__ __forceinline__ void ld64(uint32_t taddr, float *v) {
+    float t32[32];
+    tmem_ld32(taddr, t32);
+#pragma unroll
+    for (int c = 0; c < 32; ++c) v[c] = t32[c];
+    tmem_ld32(taddr + 32, t32);
+#pragma unroll
+    for (int c = 0; c < 32; ++c) v[32 + c] = t32[c];
+}
+
+// 64 values as a bf16 pair into a global row: hi at row[col_hi..], lo at row[col_lo..].
+__device__ __forceinline__ void store_pair64(bf16 *row, int col_hi, int col_lo, const float *v,
+                                             float f) {
+#pragma unroll
+    for (int c = 0; c < 64; c += 8) {
+        uint32_t h4[4], l4[4];
+#pragma unroll
+        for (int e = 0; e < 4; ++e) {
+            const float a = v[c + 2 * e] * f, b = v[c + 2 * e + 1] * f;
+            const bf16 ha = __float2bfloat16_rn(a), hb = __float2bfloat16_rn(b);
+            const bf16 la = __float2bfloat16_rn(a - __bfloat162float(ha));
+            const bf16 lb = __float2bfloat16_rn(b - __bfloat162float(hb));
+            h4[e] = (uint32_t)__bfloat16_as_ushort(ha) | ((uint32_t)__bfloat16_as_ushort(hb) << 16);
+            l4[e] = (uint32_t)__bfloat16_as_ushort(la) | ((uint32_t)__bfloat16_as_ushort(lb) << 16);
+        }
+        *reinterpret_cast<uint4 *>(row + col_hi + c) = make_uint4(h4[0], h4[1], h4[2], h4[3]);
+        *reinterpret_cast<uint4 *>(row + col_lo + c) = make_uint4(l4[0], l4[1], l4[2], l4[3]);
+    }
+}
+
+__global__ void __launch_bounds__(kThreads, 1) attn_dkv_tc_kernel(const __grid_constant__ BwdParams p) {
+    extern __shared__ uint8_t smem_raw[];
+    DkvSmem &sm = *reinterpret_cast<DkvSmem *>(
+        (reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    const int jt = blockIdx.x, b = blockIdx.y, h = blockIdx.z;
+    const int j0 = jt * kKT;
+    const int qb_begin = j0 / kQB;                      // queries i >= j0
+    const int nq = (p.k + kQB - 1) / kQB - qb_begin;    // query blocks to visit
+
+    if (threadIdx.x == 0) {
+        mbar_init(smem_u32(&sm.kv_full), 1);
+        mbar_init(smem_u32(&sm.st_full), 1);
+        mbar_init(smem_u32(&sm.p_ready), 128);
+        mbar_init(smem_u32(&sm.pd_done), 1);
+        mbar_init(smem_u32(&sm.acc_done), 1);
+        for (int s = 0; s < kStages; ++s) {
+            mbar_init(smem_u32(&sm.qa_full[s]), 1);
+            mbar_init(smem_u32(&sm.qa_empty[s]), 1);
+        }
+        sm.abort = 0;
+        fence_barrier_init();
+    }
+    if (warp == 2) {
+        tmem_alloc(smem_u32(&sm.tmem), 256);
+        tmem_relinquish();
+    }
+    tc_fence_before();
+    __syncthreads();
+    tc_fence_after();
+    const uint32_t tmem = sm.tmem;
+    const uint32_t tST = tmem, tDPT = tmem + 64, tDV = tmem + 128, tDK = tmem + 192;
+
+    if (warp == 0) {
+        if (lane == 0) {
+            const uint32_t kb = smem_u32(&sm.kv_full);
+            mbar_expect_tx(kb, 4 * kHalf128);
+            tma_load_4d(smem_u32(sm.k[0]), &p.mA0, kb, 0, j0, b, h);
+            tma_load_4d(smem_u32(sm.k[1]), &p.mA0, kb, 64, j0, b, h);
+            tma_load_4d(smem_u32(sm.v[0]), &p.mA1, kb, 0, j0, b, h);
+            tma_load_4d(smem_u32(sm.v[1]), &p.mA1, kb, 64, j0, b, h);
+            int issued = 0;
+            for (int n = 0; n < nq; ++n) {
+                const int s = n % kStages;
+                if (!mbar_wait(smem_u32(&sm.qa_empty[s]), ((n / kStages) & 1) ^ 1) ||
+                    *(volatile int *)&sm.abort) {
+                    flag_timeout_b(sm, p.status);
+                    break;
+                }
+                const int i0 = (qb_begin + n) * kQB;
+                const uint32_t fb = smem_u32(&sm.qa_full[s]);
+                mbar_expect_tx(fb, 4 * kHalf64);
+                tma_load_4d(smem_u32(sm.q[s][0]), &p.mB0, fb, 0, i0, b, h);
+                tma_load_4d(smem_u32(sm.q[s][1]), &p.mB0, fb, 64, i0, b, h);
+                tma_load_4d(smem_u32(sm.da[s][0]), &p.mB1, fb, 0, i0, b, h);
+                tma_load_4d(smem_u32(sm.da[s][1]), &p.mB1, fb, 64, i0, b, h);
+                issued = n + 1;
+            }
+            if (*(volatile int *)&sm.abort) {
+                mbar_wait(kb, 0);
+                for (int n = max(0, issued - kStages); n < issued; ++n)
+                    mbar_wait(smem_u32(&sm.qa_full[n % kStages]), (n / kStages) & 1);
+            }
+        }
+    } else if (warp == 1) {
+        if (lane == 0) {
+            constexpr uint32_t idKK = idesc_bf16(kKT, kQB, false, false);  // S^T, dP^T
+            constexpr uint32_t idKM = idesc_bf16(kKT, 64, false, true);    // dV, dK
+            bool ok = mbar_wait(smem_u32(&sm.kv_full), 0);
+            for (int n = 0; ok && n < nq; ++n) {
+                const int s = n % kStages;
+                if (!mbar_wait(smem_u32(&sm.qa_full[s]), (n / kStages) & 1) ||
+                    *(volatile int *)&sm.abort) {
+                    ok = false;
+                    break;
+                }
+                tc_fence_after();
+                const uint32_t q0 = smem_u32(sm.q[s][0]), q1 = smem_u32(sm.q[s][1]);
+                const uint32_t a0 = smem_u32(sm.da[s][0]), a1 = smem_u32(sm.da[s][1]);
+                mma_pair3(tST, smem_u32(sm.k[0]), smem_u32(sm.k[1]), q0, q1, false, false, idKK, false);
+                mma_pair3(tDPT, smem_u32(sm.v[0]), smem_u32(sm.v[1]), a0, a1, false, false, idKK, false);
+                mma_commit(smem_u32(&sm.st_full));
+                if (!mbar_wait(smem_u32(&sm.p_ready), n & 1) || *(volatile int *)&sm.abort) {
+                    ok = false;
+                    break;
+                }
+                tc_fence_after();
+                mma_pair3(tDV, smem_u32(sm.pt[0]), smem_u32(sm.pt[1]), a0, a1, false, true, idKM, n > 0);
+                mma_pair3(tDK, smem_u32(sm.dst[0]), smem_u32(sm.dst[1]), q0, q1, false, true, idKM, n > 0);
+                mma_commit(smem_u32(&sm.qa_empty[s]));
+                mma_commit(smem_u32(&sm.pd_done));
+            }
+            if (!ok) {
+                flag_timeout_b(sm, p.status);
+                mma_commit(smem_u32(&sm.st_full));
+            }
+            mma_commit(smem_u32(&sm.acc_done));
+        }
+    } else if (warp >= 4) {
+        const int q = warp - 4;
+        const int r = q * 32 + lane;
+        const int j = j0 + r;
+        const uint32_t lane_off = (uint32_t)(q * 32) << 16;
+        const size_t base = (size_t)h * p.Mtok + (size_t)b * p.k;
+        bool ok = true;
+        for (int n = 0; n < nq; ++n) {
+            if (!mbar_wait(smem_u32(&sm.st_full), n & 1) || *(volatile int *)&sm.abort) {
+                ok = false;
+                break;
+            }
+            tc_fence_after();
+            float st[64], dpt[64];
+            ld64(tST + lane_off, st);
+            ld64(tDPT + lane_off, dpt);
+            const int i0 = (qb_begin + n) * kQB;
+#pragma unroll
+            for (int c = 0; c < 64; ++c) {
+                const int i = i0 + c;
+                const bool allowed = (i >= j) && (i < p.k);
+                const float l2 = allowed ? __ldg(p.lse + base + i) * 1.4426950408889634f : 0.f;
+                const float dd = allowed ? __ldg(p.Dd + base + i) : 0.f;
+                const float pr = allowed ? exp2f(st[c] * p.scale_log2 - l2) : 0.f;
+                st[c] = pr;
+                dpt[c] = pr * (dpt[c] - dd);
+            }
+            if (n > 0 && !mbar_wait(smem_u32(&sm.pd_done), (n - 1) & 1)) {
+                ok = false;
+                break;
+            }
+            write_pair_row64(sm.pt[0], sm.pt[1], r, st);
+            write_pair_row64(sm.dst[0], sm.dst[1], r, dpt);
+            fence_proxy_async();
+            tc_fence_before();
+            mbar_arrive(smem_u32(&sm.p_ready));
+        }
+        const bool done = mbar_wait(smem_u32(&sm.acc_done), 0);
+        tc_fence_after();
+        float dv[64], dk[64];
+        ld64(tDV + lane_off, dv);
+        ld64(tDK + lane_off, dk);
+        if (!ok || !done) flag_timeout_b(sm, p.status);
+        if (ok && done && j < p.k && nq > 0 && !*(volatile int *)&sm.abort) {
+            bf16 *row = p.dQKV + (base + j) * 384;
+            store_pair64(row, 64, 256, dk, p.scale);
+            store_pair64(row, 128, 320, dv, 1.f);
+        }
+    }
+    tc_fence_before();
+    __syncthreads();
+    if (warp == 2) {
+        tc_fence_after();
+        tmem_dealloc(tmem, 256);
+    }
+}
+
+__global__ void __launch_bounds__(kThreads, 1) attn_dq_tc_kernel(const __grid_constant__ BwdParams p) {
+    extern __shared__ uint8_t smem_raw[];
+    DqSmem &sm = *reinterpret_cast<DqSmem *>(
+        (reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    const int qt = blockIdx.x, b = blockIdx.y, h = blockIdx.z;
+    const int i0 = qt * kQ;
+    const int q_end = min(p.k, i0 + kQ);
+    const int nblk = (q_end + kKV - 1) / kKV;
+
+    if (threadIdx.x == 0) {
+        mbar_init(smem_u32(&sm.qa_full), 1);
+        mbar_init(smem_u32(&sm.sp_full), 1);
+        mbar_init(smem_u32(&sm.ds_ready), 128);
+        mbar_init(smem_u32(&sm.ds_done), 1);
+        mbar_init(smem_u32(&sm.acc_done), 1);
+        for (int s = 0; s < kStages; ++s) {
+            mbar_init(smem_u32(&sm.kv_full[s]), 1);
+            mbar_init(smem_u32(&sm.kv_empty[s]), 1);
+        }
+        sm.abort = 0;
+        fence_barrier_init();
+    }
+    if (warp == 2) {
+        tmem_alloc(smem_u32(&sm.tmem), 256);
+        tmem_relinquish();
+    }
+    tc_fence_before();
+    __syncthreads();
+    tc_fence_after();
+    const uint32_t tmem = sm.tmem;
+    const uint32_t tS = tmem, tDP = tmem + 64, tDQ = tmem + 128;
+
+    if (warp == 0) {
+        if (lane == 0) {
+            const uint32_t qb = smem_u32(&sm.qa_full);
+            mbar_expect_tx(qb, 4 * kHalf128);
+            tma_load_4d(smem_u32(sm.q[0]), &p.mA0, qb, 0, i0, b, h);
+            tma_load_4d(smem_u32(sm.q[1]), &p.mA0, qb, 64, i0, b, h);
+            tma_load_4d(smem_u32(sm.da[0]), &p.mA1, qb, 0, i0, b, h);
+            tma_load_4d(smem_u32(sm.da[1]), &p.mA1, qb, 64, i0, b, h);
+            int issued = 0;
+            for (int n = 0; n < nblk; ++n) {
+                const int s = n % kStages;
+                if (!mbar_wait(smem_u32(&sm.kv_empty[s]), ((n / kStages) & 1) ^ 1) ||
+                    *(volatile int *)&sm.abort) {
+                    flag_timeout_b(sm, p.status);
+                    break;
+                }
+                const uint32_t fb = smem_u32(&sm.kv_full[s]);
+                mbar_expect_tx(fb, 4 * kHalf64);
+                tma_load_4d(smem_u32(sm.k[s][0]), &p.mB0, fb, 0, n * kKV, b, h);
+                tma_load_4d(smem_u32(sm.k[s][1]), &p.mB0, fb, 64, n * kKV, b, h);
+                tma_load_4d(smem_u32(sm.v[s][0]), &p.mB1, fb, 0, n * kKV, b, h);
+                tma_load_4d(smem_u32(sm.v[s][1]), &p.mB1, fb, 64, n * kKV, b, h);
+                issued = n + 1;
+            }
+            if (*(volatile int *)&sm.abort) {
+                mbar_wait(qb, 0);
+                for (int n = max(0, issued - kStages); n < issued; ++n)
+                    mbar_wait(smem_u32(&sm.kv_full[n % kStages]), (n / kStages) & 1);
+            }
+        }
+    } else if (warp == 1) {
+        if (lane == 0) {
+            constexpr uint32_t idKK = idesc_bf16(kQ, kKV, false, false);  // S, dP
+            constexpr uint32_t idKM = idesc_bf16(kQ, 64, false, true);    // dQ
+            bool ok = mbar_wait(smem_u32(&sm.qa_full), 0);
+            for (int n = 0; ok && n < nblk; ++n) {
+                const int s = n % kStages;
+                if (!mbar_wait(smem_u32(&sm.kv_full[s]), (n / kStages) & 1) ||
+                    *(volatile int *)&sm.abort) {
+                    ok = false;
+                    break;
+                }
+                tc_fence_after();
+                const uint32_t k0 = smem_u32(sm.k[s][0]), k1 = smem_u32(sm.k[s][1]);
+                const uint32_t v0 = smem_u32(sm.v[s][0]), v1 = smem_u32(sm.v[s][1]);
+                mma_pair3(tS, smem_u32(sm.q[0]), smem_u32(sm.q[1]), k0, k1, false, false, idKK, false);
+                mma_pair3(tDP, smem_u32(sm.da[0]), smem_u32(sm.da[1]), v0, v1, false, false, idKK, false);
+                mma_commit(smem_u32(&sm.sp_full));
+                if (!mbar_wait(smem_u32(&sm.ds_ready), n & 1) || *(volatile int *)&sm.abort) {
+                    ok = false;
+                    break;
+                }
+                tc_fence_after();
+                mma_pair3(tDQ, smem_u32(sm.ds[0]), smem_u32(sm.ds[1]), k0, k1, false, true, idKM, n > 0);
+                mma_commit(smem_u32(&sm.kv_empty[s]));
+                mma_commit(smem_u32(&sm.ds_done));
+            }
+            if (!ok) {
+                flag_timeout_b(sm, p.status);
+                mma_commit(smem_u32(&sm.sp_full));
+            }
+            mma_commit(smem_u32(&sm.acc_done));
+        }
+    } else if (warp >= 4) {
+        const int q = warp - 4;
+        const int r = q * 32 + lane;
+        const int i = i0 + r;
+        const uint32_t lane_off = (uint32_t)(q * 32) << 16;
+        const size_t base = (size_t)h * p.Mtok + (size_t)b * p.k;
+        const float l2 = i < p.k ? p.lse[base + i] * 1.4426950408889634f : 0.f;
+        const float dd = i < p.k ? p.Dd[base + i] : 0.f;
+        bool ok = true;
+        for (int n = 0; n < nblk; ++n) {
+            if (!mbar_wait(smem_u32(&sm.sp_full), n & 1) || *(volatile int *)&sm.abort) {
+                ok = false;
+                break;
+            }
+            tc_fence_after();
+            float sv[64], dp[64];
+            ld64(tS + lane_off, sv);
+            ld64(tDP + lane_off, dp);
+            const int jb = n * kKV;
+#pragma unroll
+            for (int c = 0; c < 64; ++c) {
+                const bool allowed = (jb + c <= i);
+                const float pr = allowed ? exp2f(sv[c] * p.scale_log2 - l2) : 0.f;
+                dp[c] = pr * (dp[c] - dd);
+            }
+            if (n > 0 && !mbar_wait(smem_u32(&sm.ds_done), (n - 1) & 1)) {
+                ok = false;
+                break;
+            }
+            write_pair_row64(sm.ds[0], sm.ds[1], r, dp);
+            fence_proxy_async();
+            tc_fence_before();
+            mbar_arrive(smem_u32(&sm.ds_ready));
+        }
+        const bool done = mbar_wait(smem_u32(&sm.acc_done), 0);
+        tc_fence_after();
+        float dq[64];
+        ld64(tDQ + lane_off, dq);
+        if (!ok || !done) flag_timeout_b(sm, p.status);
+        if (ok && done && i < p.k && nblk > 0 && !*(volatile int *)&sm.abort) {
+            bf16 *row = p.dQKV + (base + i) * 384;
+            store_pair64(row, 0, 192, dq, p.scale);
+        }
+    }
+    tc_fence_before();
+    __syncthreads();
+    if (warp == 2) {
+        tc_fence_after();
+        tmem_dealloc(tmem, 256);
+    }
+}
+
 PFN_cuTensorMapEncodeTiled_v12000 encode() {
     static PFN_cuTensorMapEncodeTiled_v12000 fn = nullptr;
     static std::once_flag once;
@@ -382,6 +789,47 @@ cudaError_t tc_attn_fwd(const Dims &dm, const Saved &sv, cudaStream_t s) {
     dim3 grid((dm.k + kQ - 1) / kQ, dm.B, dm.H);
     attn_fwd_tc_kernel<<<grid, kThreads, kFwdSmem, s>>>(p);
     note_launches(1);
+    return cudaGetLastError();
+}
+
+cudaError_t tc_attn_bwd(const Dims &dm, const Saved &sv, cudaStream_t s) {
+    BwdParams kv, dq;
+    memset(&kv, 0, sizeof(kv));
+    memset(&dq, 0, sizeof(dq));
+    bool ok = map_units(&kv.mA0, sv.K, dm.H, dm.B, dm.k, kKT) &&
+              map_units(&kv.mA1, sv.V, dm.H, dm.B, dm.k, kKT) &&
+              map_units(&kv.mB0, sv.Q, dm.H, dm.B, dm.k, kQB) &&
+              map_units(&kv.mB1, sv.dA, dm.H, dm.B, dm.k, kQB) &&
+              map_units(&dq.mA0, sv.Q, dm.H, dm.B, dm.k, kQ) &&
+              map_units(&dq.mA1, sv.dA, dm.H, dm.B, dm.k, kQ) &&
+              map_units(&dq.mB0, sv.K, dm.H, dm.B, dm.k, kKV) &&
+              map_units(&dq.mB1, sv.V, dm.H, dm.B, dm.k, kKV);
+    if (!ok) return cudaErrorInvalidValue;
+    for (BwdParams *p : {&kv, &dq}) {
+        p->k = dm.k;
+        p->Mtok = dm.B * dm.k;
+        p->scale = 1.f / sqrtf(64.f);
+        p->scale_log2 = 1.4426950408889634f / sqrtf(64.f);
+        p->lse = sv.lse;
+        p->Dd = sv.Dd;
+        p->dQKV = static_cast<bf16 *>(sv.dQKV);
+        p->status = sv.status;
+    }
+    static std::once_flag once;
+    static cudaError_t attr = cudaSuccess;
+    std::call_once(once, [] {
+        attr = cudaFuncSetAttribute(attn_dkv_tc_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                    kDkvSmem);
+        if (attr == cudaSuccess)
+            attr = cudaFuncSetAttribute(attn_dq_tc_kernel,
+                                        cudaFuncAttributeMaxDynamicSharedMemorySize, kDqSmem);
+    });
+    if (attr != cudaSuccess) return attr;
+    dim3 gkv((dm.k + kKT - 1) / kKT, dm.B, dm.H);
+    attn_dkv_tc_kernel<<<gkv, kThreads, kDkvSmem, s>>>(kv);
+    dim3 gq((dm.k + kQ - 1) / kQ, dm.B, dm.H);
+    attn_dq_tc_kernel<<<gq, kThreads, kDqSmem, s>>>(dq);
+    note_launches(2);
     return cudaGetLastError();
 }
 

@@ -361,6 +361,35 @@ def main():
     total_ms = sum(s.elapsed_time(e) for s, e in zip(starts, ends))
     value, total_ms = combine_ranks(total_ms, cfg.B * cfg.T * K, dist, dev)
 
+    # Diagnostic: the same step replayed from a CUDA graph (host launch cost removed).
+    graph_ms = None
+    try:
+        g = torch.cuda.CUDAGraph()
+        side = torch.cuda.Stream()
+        side.wait_stream(torch.cuda.current_stream())
+        with torch.cuda.stream(side):
+            step()
+        torch.cuda.current_stream().wait_stream(side)
+        torch.cuda.synchronize()
+        with torch.cuda.graph(g):
+            step()
+        for _ in range(3):
+            flush_buf.zero_()
+            g.replay()
+        torch.cuda.synchronize()
+        gs = [torch.cuda.Event(enable_timing=True) for _ in range(K)]
+        ge = [torch.cuda.Event(enable_timing=True) for _ in range(K)]
+        for i in range(K):
+            flush_buf.zero_()
+            gs[i].record()
+            g.replay()
+            ge[i].record()
+        torch.cuda.synchronize()
+        graph_ms = sum(a.elapsed_time(b) for a, b in zip(gs, ge)) / K
+        del g
+    except Exception as exc:  # capture unsupported: report why
+        graph_ms = f"unavailable: {exc}"
+
     # End to end through the public API with pinned host buffers.
     hX = torch.from_numpy(x["X"]).to(tdt).pin_memory()
     hdY = torch.from_numpy(x["dY"]).to(tdt).pin_memory()
@@ -426,6 +455,7 @@ def main():
                 "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h,
                 "what": "pinned host X, dY -> device; forward+backward; Y, dX -> pinned host"},
         "gpu_launches": int(launches),
+        "graph_ms_per_step": graph_ms,
         "clocks": clocks,
     }
     if world == 1 and not args.no_cpu_baseline:

@@ -10,6 +10,9 @@ namespace mosa {
 // F1, Sec. 2.2 router: r_full[b,h,t] = sigmoid(X[b,t,:] . W_r[:,h]) in fp32.
 cudaError_t launch_router(const Dims &dm, const void *X, const void *Wr, float *r_full,
                           cudaStream_t stream);
+// F1 choosing the tensor-core kernel where it applies.
+cudaError_t launch_router_auto(const Dims &dm, const void *X, const void *Wr, float *r_full,
+                               uint32_t *status, cudaStream_t stream);
 
 // F2, Sec. 2.2 TopK: per row of T scores, the k largest (ties: lower index),
 // ascending.  If gidx != nullptr, row = b*H + h also writes the head-major
@@ -62,6 +65,9 @@ cudaError_t tc_out_bwd(const Dims &dm, const void *Wo, const void *dY, const Sav
                        float *dWo, cudaStream_t s);
 cudaError_t tc_in_bwd(const Dims &dm, const void *Wq, const void *Wk, const void *Wv,
                       const void *Wr, const Saved &sv, float *dX, cudaStream_t s);
+// F1 on tensor cores (bf16 inputs, H % 8 == 0); false if not applicable.
+bool tc_router(const Dims &dm, const void *X, const void *Wr, float *r_full, uint32_t *status,
+               cudaStream_t s, cudaError_t *err);
 cudaError_t tc_attn_fwd(const Dims &dm, const Saved &sv, cudaStream_t s);
 cudaError_t tc_attn_bwd(const Dims &dm, const Saved &sv, cudaStream_t s);
 cudaError_t tc_w_bwd(const Dims &dm, const void *X, const Saved &sv, float *dWq, float *dWk,

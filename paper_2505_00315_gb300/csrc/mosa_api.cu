@@ -139,7 +139,7 @@ mosa_status mosa_forward(const mosa_shape *shape, const void *X, const void *W_r
     MOSA_TRY(cudaMemsetAsync(sv.status, 0, sizeof(uint32_t), s));
     {
         StageScope st_(kStageRouter, s);
-        MOSA_TRY(launch_router(dm, X, W_r, rf, s));
+        MOSA_TRY(launch_router_auto(dm, X, W_r, rf, sv.status, s));
     }
     {
         StageScope st_(kStageSelect, s);
@@ -214,7 +214,7 @@ int32_t mosa_stage_engine(const mosa_shape *shape, int32_t stage) {
     Dims dm;
     if (check_shape(shape, &dm) != MOSA_OK || stage < 0 || stage >= kNumStages) return -1;
     switch (stage) {
-        case kStageRouter:
+        case kStageRouter: return (use_tc(dm) && dm.H % 8 == 0) ? 1 : 0;
         case kStageSelect: return 2;
         case kStageQkv:
         case kStageOut:

@@ -194,6 +194,13 @@ cudaError_t launch_router(const Dims &dm, const void *X, const void *Wr, float *
     return launch_simt_gemm(op, 1, stream);
 }
 
+cudaError_t launch_router_auto(const Dims &dm, const void *X, const void *Wr, float *r_full,
+                               uint32_t *status, cudaStream_t stream) {
+    cudaError_t e = cudaSuccess;
+    if (use_tc(dm) && tc_router(dm, X, Wr, r_full, status, stream, &e)) return e;
+    return launch_router(dm, X, Wr, r_full, stream);
+}
+
 cudaError_t launch_select(int rows, int T, int k, const float *scores, int32_t *I, float *rsel,
                           int B, int H, int32_t *gidx, float *rsel_hm, cudaStream_t stream) {
     if (rows <= 0) return cudaSuccess;

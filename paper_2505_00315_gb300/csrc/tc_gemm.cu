@@ -19,6 +19,7 @@
 //   kDWO  B1  dW_o[h](p,c)  = sum_m AR(m,p) dY[g(m),c]       A gathered MN-major, B = AR pair
 //   kDX   B3  dX[g(m),n]   += dQKV(m,:) [W_q|W_k|W_v][h]^T(:,n) + dlogit(m) W_r[n,h]
 //   kDW   B4  dW_{q|k|v}[h](c,p) = sum_m X[g(m),c] dQKV(m,p) A gathered MN-major, B = dQKV pair
+//   kROUTER F1 r[b,h,t] = sigmoid(X[b,t,:] W_r[:,h])       A = X tiles, B = W_r MN-major
 // where g(m) = b*T + I[b,h,i] for row m = b*k + i of head h.
 #include <cudaTypedefs.h>
 
@@ -34,7 +35,7 @@ namespace {
 
 using namespace tc;
 
-enum Kind : int { kQKV = 0, kOUT, kG, kDWO, kDX, kDW };
+enum Kind : int { kQKV = 0, kOUT, kG, kDWO, kDX, kDW, kROUTER };
 
 constexpr int kBM = 128;        // rows per tile (TMEM lanes)
 constexpr int kBK = 64;         // K per stage: one 128-byte swizzle row of bf16
@@ -81,6 +82,13 @@ struct Cfg<kDW> {
     static constexpr bool A_MN = true, B_MN = true, A_PAIR = false, B_PAIR = true;
 };
 
+template <>
+struct Cfg<kROUTER> {
+    static constexpr int BN = 128, STAGES = 4, A_BYTES = kTile16K, B_BYTES = 2 * kTile8K,
+                         TMEM_COLS = 128;
+    static constexpr bool A_MN = false, B_MN = true, A_PAIR = false, B_PAIR = false;
+};
+
 template <int KIND>
 constexpr int smem_bytes() {
     return 1024 /* alignment slack */ + Cfg<KIND>::STAGES * (Cfg<KIND>::A_BYTES + Cfg<KIND>::B_BYTES) +
@@ -95,7 +103,7 @@ struct TcParams {
     int N;                 // output columns (d for kOUT / kDX)
     int nkb;               // K blocks in the whole reduction
     int splits;            // reduction splits (kDWO / kDW)
-    int d, H;
+    int d, H, T;
     const int32_t *gidx;   // [H, B*k]
     const float *rsel;     // [H, B*k]
     const float *A32;      // [H, B*k, 64] attention output (kG)
@@ -211,6 +219,10 @@ __global__ void __launch_bounds__(kThreads, 1) tc_gemm_kernel(const __grid_const
                 if (lane == 1) tma_load_3d(a + kTile16K, &p.mapA, fb, 64, m0, h);
                 if (lane >= 2 && lane < 6)
                     tma_load_3d(b + (lane - 2) * kTile8K, &p.mapB[0], fb, n0 + 64 * (lane - 2), 0, h);
+            } else if constexpr (KIND == kROUTER) {
+                if (lane == 0) tma_load_2d(a, &p.mapA, fb, kb * kBK, m0);
+                if (lane == 1 || lane == 2)
+                    tma_load_2d(b + (lane - 1) * kTile8K, &p.mapB[0], fb, n0 + 64 * (lane - 1), kb * kBK);
             } else if constexpr (KIND == kDX) {
                 if (lane == 0) tma_load_3d(a, &p.mapA, fb, 64 * kb, m0, h);
                 if (lane == 1) tma_load_3d(a + kTile16K, &p.mapA, fb, 192 + 64 * kb, m0, h);
@@ -351,6 +363,21 @@ __global__ void __launch_bounds__(kThreads, 1) tc_gemm_kernel(const __grid_const
                 p.out_f1[row] = dd;
                 p.out_f2[row] = dr * rr * (1.f - rr);
             }
+        } else if constexpr (KIND == kROUTER) {
+            const bool live = !abort && mg < p.M;
+            const int bb = live ? mg / p.T : 0, t = live ? mg % p.T : 0;
+            float *dst = p.out_f + (size_t)bb * p.H * p.T + t;
+#pragma unroll 1
+            for (int c0 = 0; c0 < C::BN; c0 += 32) {
+                float v[32];
+                tmem_ld32(tb + c0, v);
+                if (!live) continue;
+#pragma unroll
+                for (int e = 0; e < 32; ++e) {
+                    const int hh = n0 + c0 + e;
+                    if (hh < p.H) dst[(size_t)hh * p.T] = 1.f / (1.f + expf(-v[e]));
+                }
+            }
         } else if constexpr (KIND == kDWO) {
             const bool live = !abort && mg < p.M;
 #pragma unroll 1
@@ -479,7 +506,34 @@ TcParams base_params(const Dims &dm, const Saved &sv) {
     return p;
 }
 
+bool map_2d(CUtensorMap *m, const void *base, uint64_t rows, uint64_t cols, uint32_t box_rows) {
+    const uint64_t dims[2] = {cols, rows}, strides[1] = {cols * 2};
+    const uint32_t box[2] = {64, box_rows};
+    return make_map(m, base, 2, dims, strides, box);
+}
+
 }  // namespace
+
+bool tc_router(const Dims &dm, const void *X, const void *Wr, float *r_full, uint32_t *status,
+               cudaStream_t s, cudaError_t *err) {
+    if (!dm.bf16 || dm.H % 8 != 0 || encode_fn() == nullptr) return false;
+    TcParams p;
+    memset(&p, 0, sizeof(p));
+    p.M = dm.B * dm.T;
+    p.nkb = (dm.d + kBK - 1) / kBK;
+    p.splits = 1;
+    p.d = dm.d;
+    p.H = dm.H;
+    p.T = dm.T;
+    p.status = status;
+    p.out_f = r_full;
+    if (!map_2d(&p.mapA, X, (uint64_t)dm.B * dm.T, dm.d, 128) ||
+        !map_2d(&p.mapB[0], Wr, dm.d, dm.H, 64))
+        return false;
+    dim3 grid((p.M + kBM - 1) / kBM, (dm.H + 127) / 128, 1);
+    *err = launch_kind<kROUTER>(p, grid, s);
+    return true;
+}
 
 bool tc_supported(const Dims &dm) {
     return dm.bf16 && dm.hp == 64 && encode_fn() != nullptr;

@@ -4,10 +4,13 @@
 //
 // One CTA computes one 128-row output tile of one head (or one split of the
 // reduction for the weight gradients).  Warp roles (256 threads):
-//   warp 0      producer: TMA tile / gather4 loads into a STAGES-deep ring
+//   warp 0      producer: TMA tile loads into a STAGES-deep ring
 //   warp 1      MMA issuer (one thread): tcgen05.mma per 16-wide K step
 //   warp 2      TMEM allocator
-//   warps 4-7   epilogue: tcgen05.ld of the accumulator rows, fused output
+//   warps 4-7   gathered operand: 16-byte cp.async copies of the selected rows,
+//               written in the 128-byte-swizzled layout (TMA gather4 issues
+//               only ~4 rows per ~80 cycles per SM, too slow here); then the
+//               epilogue: tcgen05.ld of the accumulator rows, fused output
 // Every mbarrier wait is bounded; a wait that runs out sets kStatusTimeout in
 // the workspace status word and the CTA winds down without hanging.
 //
@@ -47,7 +50,7 @@ template <int KIND>
 struct Cfg;
 template <>
 struct Cfg<kQKV> {
-    static constexpr int BN = 192, STAGES = 4, A_BYTES = kTile16K, B_BYTES = 3 * kTile8K,
+    static constexpr int BN = 192, STAGES = 2, A_BYTES = kTile16K, B_BYTES = 3 * kTile8K,
                          TMEM_COLS = 256;
     static constexpr bool A_MN = false, B_MN = true, A_PAIR = false, B_PAIR = false;
 };
@@ -65,7 +68,7 @@ struct Cfg<kG> {
 };
 template <>
 struct Cfg<kDWO> {
-    static constexpr int BN = 64, STAGES = 4, A_BYTES = kTile16K, B_BYTES = 2 * kTile8K,
+    static constexpr int BN = 64, STAGES = 3, A_BYTES = kTile16K, B_BYTES = 2 * kTile8K,
                          TMEM_COLS = 64;
     static constexpr bool A_MN = true, B_MN = true, A_PAIR = false, B_PAIR = true;
 };
@@ -84,10 +87,16 @@ struct Cfg<kDW> {
 
 template <>
 struct Cfg<kROUTER> {
-    static constexpr int BN = 128, STAGES = 4, A_BYTES = kTile16K, B_BYTES = 2 * kTile8K,
+    static constexpr int BN = 128, STAGES = 3, A_BYTES = kTile16K, B_BYTES = 2 * kTile8K,
                          TMEM_COLS = 128;
     static constexpr bool A_MN = false, B_MN = true, A_PAIR = false, B_PAIR = false;
 };
+
+// Kinds whose A operand is gathered through the selected rows.
+template <int KIND>
+constexpr bool gathers() {
+    return KIND == kQKV || KIND == kG || KIND == kDWO || KIND == kDW;
+}
 
 template <int KIND>
 constexpr int smem_bytes() {
@@ -109,6 +118,7 @@ struct TcParams {
     const float *A32;      // [H, B*k, 64] attention output (kG)
     const float *dlogit;   // [H, B*k] (kDX reads, kG writes via out_f1)
     const bf16 *Wr;        // [d, H] (kDX)
+    const void *src_rows;  // gathered source [B*T, d] bf16: X (kQKV, kDW) or dY (kG, kDWO)
     void *out[3];          // Q/K/V pairs (kQKV), dA pair (kG)
     float *out_f;          // Y (kOUT), dW_o (kDWO), dX (kDX), dW_q (kDW)
     float *out_f1;         // Dd (kG), dW_k (kDW)
@@ -133,6 +143,73 @@ __device__ __forceinline__ void store_pair_row32(bf16 *row_hi, bf16 *row_lo, con
         reinterpret_cast<uint4 *>(row_hi)[q] = make_uint4(h4[0], h4[1], h4[2], h4[3]);
         reinterpret_cast<uint4 *>(row_lo)[q] = make_uint4(l4[0], l4[1], l4[2], l4[3]);
     }
+}
+
+// The gathered A operand of one stage, copied by the 128 threads of warps 4-7
+// with 16-byte cp.async into the 128-byte-swizzled layout the MMA reads:
+//   K-major (kQKV, kG):    rows m of the tile = source rows g(m), 64 columns of K block kb
+//   MN-major (kDWO, kDW):  64 tokens of K block kb, columns m0 .. m0+127 in two
+//                          64-wide blocks; token rows are the smem rows
+// Element (row, 16-byte chunk c) lands at row*128 + ((c ^ (row & 7)) * 16).
+// Each thread keeps up to STAGES copy groups in flight; when a stage's group
+// has landed it makes the copies visible to the tensor core (proxy fence) and
+// arrives on that stage's full barrier.
+template <int KIND>
+__device__ __forceinline__ void gather_operand(const TcParams &p, uint8_t *sA, uint64_t *full,
+                                               uint64_t *empty, const int *s_rows, int *s_abort,
+                                               int h, int m0, int kb_begin, int nkb) {
+    using C = Cfg<KIND>;
+    constexpr int S = C::STAGES;
+    const int t = threadIdx.x - 128;       // 0..127
+    const int chunk = t & 7, sub = t >> 3;  // 16 rows x 8 chunks per pass
+    const bf16 *src = static_cast<const bf16 *>(p.src_rows);
+    const int32_t *gi = p.gidx + (size_t)h * p.Mtok;
+    int landed = 0;  // stages whose full barrier this thread has arrived on
+    for (int it = 0; it < nkb; ++it) {
+        const int s = it % S;
+        if (!mbar_wait(smem_u32(&empty[s]), ((it / S) & 1) ^ 1) || *(volatile int *)s_abort) {
+            atomicOr(p.status, kStatusTimeout);
+            *(volatile int *)s_abort = 1;
+            break;
+        }
+        const int kb = kb_begin + it;
+        const uint32_t a = smem_u32(sA + s * C::A_BYTES);
+        if constexpr (KIND == kQKV || KIND == kG) {
+            const int col = kb * kBK + chunk * 8;
+            const uint32_t nbytes = col < p.d ? 16u : 0u;
+#pragma unroll
+            for (int j = 0; j < 8; ++j) {
+                const int row = sub + 16 * j;
+                const bf16 *g = src + (size_t)s_rows[row] * p.d + (nbytes ? col : 0);
+                cp_async16(a + row * 128 + ((chunk ^ (row & 7)) << 4), g, nbytes);
+            }
+        } else {
+#pragma unroll
+            for (int q4 = 0; q4 < 4; ++q4) {
+                const int tok = sub + 16 * q4;
+                const int tg = kb * kBK + tok;
+                const int rowg = tg < p.Mtok ? gi[tg] : 0;
+#pragma unroll
+                for (int j = 0; j < 2; ++j) {
+                    const int col = m0 + 64 * j + chunk * 8;
+                    const uint32_t nbytes = (tg < p.Mtok && col < p.d) ? 16u : 0u;
+                    const bf16 *g = src + (size_t)rowg * p.d + (nbytes ? col : 0);
+                    cp_async16(a + j * kTile8K + tok * 128 + ((chunk ^ (tok & 7)) << 4), g, nbytes);
+                }
+            }
+        }
+        cp_async_commit();
+        if (it >= S - 1) {
+            cp_async_wait<S - 1>();
+            fence_proxy_async();
+            mbar_arrive(smem_u32(&full[(it - (S - 1)) % S]));
+            ++landed;
+        }
+    }
+    cp_async_wait<0>();
+    fence_proxy_async();
+    const int issued = *(volatile int *)s_abort ? landed : nkb;
+    for (int it = landed; it < issued; ++it) mbar_arrive(smem_u32(&full[it % S]));
 }
 
 template <int KIND>
@@ -167,7 +244,8 @@ __global__ void __launch_bounds__(kThreads, 1) tc_gemm_kernel(const __grid_const
 
     if (threadIdx.x == 0) {
         for (int s = 0; s < S; ++s) {
-            mbar_init(smem_u32(&full[s]), 1);
+            // gathered kinds: the TMA arrival plus one per gathering thread
+            mbar_init(smem_u32(&full[s]), gathers<KIND>() ? 129 : 1);
             mbar_init(smem_u32(&empty[s]), 1);
         }
         mbar_init(smem_u32(done), 1);
@@ -207,13 +285,12 @@ __global__ void __launch_bounds__(kThreads, 1) tc_gemm_kernel(const __grid_const
             }
             const int kb = kb_begin + it;
             const uint32_t a = smem_u32(sA + s * C::A_BYTES), b = smem_u32(sB + s * C::B_BYTES);
-            if (lane == 0) mbar_expect_tx(fb, C::A_BYTES + C::B_BYTES);
+            if (lane == 0) mbar_expect_tx(fb, gathers<KIND>() ? C::B_BYTES : C::A_BYTES + C::B_BYTES);
             __syncwarp();
-            if constexpr (KIND == kQKV || KIND == kG) {
-                const int4 r4 = reinterpret_cast<const int4 *>(s_rows)[lane];
-                tma_gather4(a + lane * 512, &p.mapA, fb, kb * kBK, r4.x, r4.y, r4.z, r4.w);
-                if (KIND == kQKV && lane < 3) tma_load_3d(b + lane * kTile8K, &p.mapB[lane], fb, 0, kb * kBK, h);
-                if (KIND == kG && lane == 0) tma_load_3d(b, &p.mapB[0], fb, kb * kBK, 0, h);
+            if constexpr (KIND == kQKV) {
+                if (lane < 3) tma_load_3d(b + lane * kTile8K, &p.mapB[lane], fb, 0, kb * kBK, h);
+            } else if constexpr (KIND == kG) {
+                if (lane == 0) tma_load_3d(b, &p.mapB[0], fb, kb * kBK, 0, h);
             } else if constexpr (KIND == kOUT) {
                 if (lane == 0) tma_load_3d(a, &p.mapA, fb, 0, m0, h);
                 if (lane == 1) tma_load_3d(a + kTile16K, &p.mapA, fb, 64, m0, h);
@@ -227,22 +304,12 @@ __global__ void __launch_bounds__(kThreads, 1) tc_gemm_kernel(const __grid_const
                 if (lane == 0) tma_load_3d(a, &p.mapA, fb, 64 * kb, m0, h);
                 if (lane == 1) tma_load_3d(a + kTile16K, &p.mapA, fb, 192 + 64 * kb, m0, h);
                 if (lane == 2) tma_load_3d(b, &p.mapB[kb], fb, 0, n0, h);
-            } else {  // kDWO, kDW: tokens along K, gathered; two 64-wide column blocks of A
-                const int j = lane >> 4, g = lane & 15;
-                const int t0 = kb * kBK + 4 * g;
-                const int32_t *gi = p.gidx + (size_t)h * p.Mtok;
-                const int r0 = t0 + 0 < p.Mtok ? gi[t0 + 0] : 0;
-                const int r1 = t0 + 1 < p.Mtok ? gi[t0 + 1] : 0;
-                const int r2 = t0 + 2 < p.Mtok ? gi[t0 + 2] : 0;
-                const int r3 = t0 + 3 < p.Mtok ? gi[t0 + 3] : 0;
-                tma_gather4(a + j * kTile8K + g * 512, &p.mapA, fb, m0 + 64 * j, r0, r1, r2, r3);
-                if constexpr (KIND == kDWO) {
-                    if (lane < 2) tma_load_3d(b + lane * kTile8K, &p.mapB[0], fb, 64 * lane, kb * kBK, h);
-                } else {
-                    if (lane < 6)
-                        tma_load_3d(b + lane * kTile8K, &p.mapB[0], fb,
-                                    (lane < 3 ? 0 : 192) + 64 * (lane % 3), kb * kBK, h);
-                }
+            } else if constexpr (KIND == kDWO) {
+                if (lane < 2) tma_load_3d(b + lane * kTile8K, &p.mapB[0], fb, 64 * lane, kb * kBK, h);
+            } else {  // kDW
+                if (lane < 6)
+                    tma_load_3d(b + lane * kTile8K, &p.mapB[0], fb,
+                                (lane < 3 ? 0 : 192) + 64 * (lane % 3), kb * kBK, h);
             }
             issued = it + 1;
         }
@@ -283,6 +350,8 @@ __global__ void __launch_bounds__(kThreads, 1) tc_gemm_kernel(const __grid_const
             mma_commit(smem_u32(done));
         }
     } else if (warp >= 4) {
+        if constexpr (gathers<KIND>()) gather_operand<KIND>(p, sA, full, empty, s_rows, s_abort, h, m0,
+                                                            kb_begin, nkb);
         // -------------------------------------------------------- epilogue
         const int q = warp - 4;
         const int r = q * 32 + lane;
@@ -548,6 +617,7 @@ cudaError_t tc_qkv(const Dims &dm, const void *X, const void *Wq, const void *Wk
     const void *W[3] = {Wq, Wk, Wv};
     for (int j = 0; j < 3; ++j) ok = ok && map_heads(&p.mapB[j], W[j], dm.H, dm.d, 64, 64);
     if (!ok) return cudaErrorInvalidValue;
+    p.src_rows = X;
     p.out[0] = sv.Q;
     p.out[1] = sv.K;
     p.out[2] = sv.V;
@@ -579,6 +649,7 @@ cudaError_t tc_out_bwd(const Dims &dm, const void *Wo, const void *dY, const Sav
     bool ok = map_gather(&p.mapA, dY, (uint64_t)dm.B * dm.T, dm.d) &&
               map_heads(&p.mapB[0], Wo, dm.H, 64, dm.d, 64);
     if (!ok) return cudaErrorInvalidValue;
+    p.src_rows = dY;
     p.A32 = sv.A;
     p.out[0] = sv.dA;
     p.out_f1 = sv.Dd;
@@ -595,6 +666,7 @@ cudaError_t tc_out_bwd(const Dims &dm, const void *Wo, const void *dY, const Sav
     ok = map_gather(&q.mapA, dY, (uint64_t)dm.B * dm.T, dm.d) &&
          map_heads(&q.mapB[0], sv.AR, dm.H, q.Mtok, 128, 64);
     if (!ok) return cudaErrorInvalidValue;
+    q.src_rows = dY;
     q.out_f = dWo;
     if (q.splits > 1) {
         e = cudaMemsetAsync(dWo, 0, sizeof(float) * (size_t)dm.H * 64 * dm.d, s);
@@ -633,6 +705,7 @@ cudaError_t tc_w_bwd(const Dims &dm, const void *X, const Saved &sv, float *dWq,
     bool ok = map_gather(&p.mapA, X, (uint64_t)dm.B * dm.T, dm.d) &&
               map_heads(&p.mapB[0], sv.dQKV, dm.H, p.Mtok, 384, 64);
     if (!ok) return cudaErrorInvalidValue;
+    p.src_rows = X;
     p.out_f = dWq;
     p.out_f1 = dWk;
     p.out_f2 = dWv;

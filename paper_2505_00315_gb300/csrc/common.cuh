@@ -88,7 +88,8 @@ struct Saved {
     void *dA;           // [H,B*k,hp] gradient of A, intermediate
     float *dlogit;      // [H,B*k]   gradient of the router logit
     float *Dd;          // [H,B*k]   rowsum(dA o A)
-    void *dQKV;         // [H,B*k,3hp] dQ | dK | dV, intermediate
+    void *dQKV;         // [H,B*k,3hp] dQ | dK | dV, intermediate (tensor-core path:
+                        // [H,B*k,512] bf16 pair dQ|dK|dV|dlogit,0.. hi then lo)
     float *G;           // [H,B*k,hp] dY[I] W_o^T (fp32)
 };
 

@@ -71,6 +71,6 @@ bool tc_router(const Dims &dm, const void *X, const void *Wr, float *r_full, uin
 cudaError_t tc_attn_fwd(const Dims &dm, const Saved &sv, cudaStream_t s);
 cudaError_t tc_attn_bwd(const Dims &dm, const Saved &sv, cudaStream_t s);
 cudaError_t tc_w_bwd(const Dims &dm, const void *X, const Saved &sv, float *dWq, float *dWk,
-                     float *dWv, cudaStream_t s);
+                     float *dWv, float *dWr, cudaStream_t s);
 
 }  // namespace mosa

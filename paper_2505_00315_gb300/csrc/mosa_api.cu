@@ -58,7 +58,7 @@ size_t carve(const Dims &dm, char *base, Saved *sv) {
     s.dA = take(e * R * dm.hp);
     s.dlogit = (float *)take(sizeof(float) * R);
     s.Dd = (float *)take(sizeof(float) * R);
-    s.dQKV = take(e * R * 3 * dm.hp);
+    s.dQKV = take(e * R * 4 * dm.hp);  // 3 h' columns, or 4 blocks of 64 on the tensor cores
     s.G = (float *)take(sizeof(float) * R * dm.hp);
     if (sv) *sv = s;
     return off;

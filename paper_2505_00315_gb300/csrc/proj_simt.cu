@@ -287,11 +287,7 @@ cudaError_t launch_in_bwd(const Dims &dm, const void *Wq, const void *Wk, const 
 
 cudaError_t launch_w_bwd(const Dims &dm, const void *X, const Saved &sv, float *dWq, float *dWk,
                          float *dWv, float *dWr, cudaStream_t s) {
-    if (use_tc(dm)) {
-        cudaError_t e = tc_w_bwd(dm, X, sv, dWq, dWk, dWv, s);
-        if (e != cudaSuccess) return e;
-        return dwr_t<bf16>(dm, X, sv, dWr, s);
-    }
+    if (use_tc(dm)) return tc_w_bwd(dm, X, sv, dWq, dWk, dWv, dWr, s);
     return dm.bf16 ? w_bwd_t<bf16>(dm, X, sv, dWq, dWk, dWv, dWr, s)
                    : w_bwd_t<float>(dm, X, sv, dWq, dWk, dWv, dWr, s);
 }

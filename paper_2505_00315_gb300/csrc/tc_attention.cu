@@ -22,13 +22,12 @@
 // one product and as an MN-major operand in the other.
 // Warp roles: 0 TMA producer, 1 MMA issuer, 2 TMEM allocator, 4-7 softmax
 // (one row per thread).  All waits are bounded.
-#include <cudaTypedefs.h>
-
 #include <mutex>
 
 #include "launch.h"
 #include "profile.h"
 #include "tc_common.cuh"
+#include "tmap.h"
 
 namespace mosa {
 namespace {
@@ -374,7 +373,7 @@ struct BwdParams {
     int k, Mtok;
     float scale, scale_log2;
     const float *lse, *Dd;            // [H, B*k]
-    bf16 *dQKV;                       // [H, B*k, 384] pair: dQ|dK|dV hi, then lo
+    bf16 *dQKV;                       // [H, B*k, 512] pair: dQ|dK|dV|dlogit hi, then lo
     uint32_t *status;
 };
 
@@ -573,9 +572,9 @@ __global__ void __launch_bounds__(kThreads, 1) attn_dkv_tc_kernel(const __grid_c
         ld64(tDK + lane_off, dk);
         if (!ok || !done) flag_timeout_b(sm, p.status);
         if (ok && done && j < p.k && nq > 0 && !*(volatile int *)&sm.abort) {
-            bf16 *row = p.dQKV + (base + j) * 384;
-            store_pair64(row, 64, 256, dk, p.scale);
-            store_pair64(row, 128, 320, dv, 1.f);
+            bf16 *row = p.dQKV + (base + j) * 512;
+            store_pair64(row, 64, 320, dk, p.scale);
+            store_pair64(row, 128, 384, dv, 1.f);
         }
     }
     tc_fence_before();
@@ -722,8 +721,8 @@ __global__ void __launch_bounds__(kThreads, 1) attn_dq_tc_kernel(const __grid_co
         ld64(tDQ + lane_off, dq);
         if (!ok || !done) flag_timeout_b(sm, p.status);
         if (ok && done && i < p.k && nblk > 0 && !*(volatile int *)&sm.abort) {
-            bf16 *row = p.dQKV + (base + i) * 384;
-            store_pair64(row, 0, 192, dq, p.scale);
+            bf16 *row = p.dQKV + (base + i) * 512;
+            store_pair64(row, 0, 256, dq, p.scale);
         }
     }
     tc_fence_before();
@@ -734,31 +733,13 @@ __global__ void __launch_bounds__(kThreads, 1) attn_dq_tc_kernel(const __grid_co
     }
 }
 
-PFN_cuTensorMapEncodeTiled_v12000 encode() {
-    static PFN_cuTensorMapEncodeTiled_v12000 fn = nullptr;
-    static std::once_flag once;
-    std::call_once(once, [] {
-        void *ptr = nullptr;
-        cudaDriverEntryPointQueryResult q;
-        if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &ptr, 12000,
-                                             cudaEnableDefault, &q) == cudaSuccess &&
-            q == cudaDriverEntryPointSuccess)
-            fn = reinterpret_cast<PFN_cuTensorMapEncodeTiled_v12000>(ptr);
-    });
-    return fn;
-}
-
 // [H, B, k, 128] bf16 pair array (row = 64 hi + 64 lo), box {64, rows, 1, 1}:
 // rows past k of one sequence read as zeros.
 bool map_units(CUtensorMap *m, const void *base, int H, int B, int k, uint32_t rows) {
-    auto fn = encode();
-    if (!fn) return false;
-    const cuuint64_t dims[4] = {128, (cuuint64_t)k, (cuuint64_t)B, (cuuint64_t)H};
-    const cuuint64_t strides[3] = {256, (cuuint64_t)k * 256, (cuuint64_t)B * k * 256};
-    const cuuint32_t box[4] = {64, rows, 1, 1}, es[4] = {1, 1, 1, 1};
-    return fn(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 4, const_cast<void *>(base), dims, strides, box,
-              es, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
-              CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+    const uint64_t dims[4] = {128, (uint64_t)k, (uint64_t)B, (uint64_t)H};
+    const uint64_t strides[3] = {256, (uint64_t)k * 256, (uint64_t)B * k * 256};
+    const uint32_t box[4] = {64, rows, 1, 1};
+    return tmap_bf16(m, base, 4, dims, strides, box);
 }
 
 }  // namespace

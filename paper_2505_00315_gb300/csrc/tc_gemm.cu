@@ -21,17 +21,18 @@
 //   kG    B1  G(m,:)        = dY[g(m),:] W_o[h]^T, then dr, dA = r G, D, dlogit in the epilogue
 //   kDWO  B1  dW_o[h](p,c)  = sum_m AR(m,p) dY[g(m),c]       A gathered MN-major, B = AR pair
 //   kDX   B3  dX[g(m),n]   += dQKV(m,:) [W_q|W_k|W_v][h]^T(:,n) + dlogit(m) W_r[n,h]
-//   kDW   B4  dW_{q|k|v}[h](c,p) = sum_m X[g(m),c] dQKV(m,p) A gathered MN-major, B = dQKV pair
+//   kDW   B4  [dW_q|dW_k|dW_v|dW_r][h](c,:) = sum_m X[g(m),c] [dQ|dK|dV|dlogit](m,:)
+//             A gathered MN-major, B = the dQKV pair (its 4th 64-column block holds
+//             dlogit in column 0 and zeros), so dW_r comes out of the same product
 //   kROUTER F1 r[b,h,t] = sigmoid(X[b,t,:] W_r[:,h])       A = X tiles, B = W_r MN-major
 // where g(m) = b*T + I[b,h,i] for row m = b*k + i of head h.
-#include <cudaTypedefs.h>
-
 #include <cstdio>
 #include <mutex>
 
 #include "launch.h"
 #include "profile.h"
 #include "tc_common.cuh"
+#include "tmap.h"
 
 namespace mosa {
 namespace {
@@ -80,7 +81,7 @@ struct Cfg<kDX> {
 };
 template <>
 struct Cfg<kDW> {
-    static constexpr int BN = 192, STAGES = 3, A_BYTES = kTile16K, B_BYTES = 6 * kTile8K,
+    static constexpr int BN = 256, STAGES = 2, A_BYTES = kTile16K, B_BYTES = 8 * kTile8K,
                          TMEM_COLS = 256;
     static constexpr bool A_MN = true, B_MN = true, A_PAIR = false, B_PAIR = true;
 };
@@ -92,16 +93,27 @@ struct Cfg<kROUTER> {
     static constexpr bool A_MN = false, B_MN = true, A_PAIR = false, B_PAIR = false;
 };
 
+// Row width (bf16) of the dQKV pair array on the tensor-core path:
+// [dQ | dK | dV | dlogit, 0..] hi (256) then the same lo (256).
+constexpr int kDQKVCols = 512;
+
+// Kinds that scatter-add their output rows into [B*T, d] (Y or dX).
+template <int KIND>
+__host__ __device__ constexpr bool scatters() {
+    return KIND == kOUT || KIND == kDX;
+}
+
 // Kinds whose A operand is gathered through the selected rows.
 template <int KIND>
-constexpr bool gathers() {
+__host__ __device__ constexpr bool gathers() {
     return KIND == kQKV || KIND == kG || KIND == kDWO || KIND == kDW;
 }
 
 template <int KIND>
 constexpr int smem_bytes() {
     return 1024 /* alignment slack */ + Cfg<KIND>::STAGES * (Cfg<KIND>::A_BYTES + Cfg<KIND>::B_BYTES) +
-           1024 /* barriers, row indices */;
+           2048 /* barriers, row indices, row scalars */ +
+           (scatters<KIND>() ? 4 * 32 * 128 : 0) /* per-warp transpose buffers */;
 }
 
 struct TcParams {
@@ -119,10 +131,11 @@ struct TcParams {
     const float *dlogit;   // [H, B*k] (kDX reads, kG writes via out_f1)
     const bf16 *Wr;        // [d, H] (kDX)
     const void *src_rows;  // gathered source [B*T, d] bf16: X (kQKV, kDW) or dY (kG, kDWO)
-    void *out[3];          // Q/K/V pairs (kQKV), dA pair (kG)
+    void *out[3];          // Q/K/V pairs (kQKV); dA pair, dQKV pair (kG)
     float *out_f;          // Y (kOUT), dW_o (kDWO), dX (kDX), dW_q (kDW)
     float *out_f1;         // Dd (kG), dW_k (kDW)
     float *out_f2;         // dlogit (kG), dW_v (kDW)
+    float *out_f3;         // dW_r (kDW)
     uint32_t *status;
 };
 
@@ -227,6 +240,8 @@ __global__ void __launch_bounds__(kThreads, 1) tc_gemm_kernel(const __grid_const
     int *s_abort = reinterpret_cast<int *>(tmem_slot + 1);
     int *s_rows = s_abort + 1 + 2;  // 128 gather rows, 16-byte aligned below
     s_rows = reinterpret_cast<int *>((reinterpret_cast<uintptr_t>(s_rows) + 15) & ~uintptr_t(15));
+    float *s_dl = reinterpret_cast<float *>(s_rows + kBM);   // dlogit of the tile's rows (kDX)
+    uint8_t *s_xpose = reinterpret_cast<uint8_t *>(bars) + 2048;  // 4 x 4 KB (scatter kinds)
 
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     const int m_tile = blockIdx.x, n_tile = blockIdx.y;
@@ -252,10 +267,11 @@ __global__ void __launch_bounds__(kThreads, 1) tc_gemm_kernel(const __grid_const
         *s_abort = 0;
         fence_barrier_init();
     }
-    if (KIND == kQKV || KIND == kG) {
+    if (KIND == kQKV || KIND == kG || scatters<KIND>()) {
         for (int r = threadIdx.x; r < kBM; r += kThreads) {
             const int m = m0 + r;
             s_rows[r] = m < p.Mtok ? p.gidx[(size_t)h * p.Mtok + m] : 0;
+            if (KIND == kDX) s_dl[r] = m < p.Mtok ? p.dlogit[(size_t)h * p.Mtok + m] : 0.f;
         }
     }
     if (warp == 2) {
@@ -302,14 +318,12 @@ __global__ void __launch_bounds__(kThreads, 1) tc_gemm_kernel(const __grid_const
                     tma_load_2d(b + (lane - 1) * kTile8K, &p.mapB[0], fb, n0 + 64 * (lane - 1), kb * kBK);
             } else if constexpr (KIND == kDX) {
                 if (lane == 0) tma_load_3d(a, &p.mapA, fb, 64 * kb, m0, h);
-                if (lane == 1) tma_load_3d(a + kTile16K, &p.mapA, fb, 192 + 64 * kb, m0, h);
+                if (lane == 1) tma_load_3d(a + kTile16K, &p.mapA, fb, 256 + 64 * kb, m0, h);
                 if (lane == 2) tma_load_3d(b, &p.mapB[kb], fb, 0, n0, h);
             } else if constexpr (KIND == kDWO) {
                 if (lane < 2) tma_load_3d(b + lane * kTile8K, &p.mapB[0], fb, 64 * lane, kb * kBK, h);
-            } else {  // kDW
-                if (lane < 6)
-                    tma_load_3d(b + lane * kTile8K, &p.mapB[0], fb,
-                                (lane < 3 ? 0 : 192) + 64 * (lane % 3), kb * kBK, h);
+            } else {  // kDW: hi blocks 0..3 then lo blocks 0..3
+                if (lane < 8) tma_load_3d(b + lane * kTile8K, &p.mapB[0], fb, 64 * lane, kb * kBK, h);
             }
             issued = it + 1;
         }
@@ -373,27 +387,42 @@ __global__ void __launch_bounds__(kThreads, 1) tc_gemm_kernel(const __grid_const
                 }
             }
         } else if constexpr (KIND == kOUT || KIND == kDX) {
-            const bool live = !abort && mg < p.M;
-            const size_t row = (size_t)h * p.Mtok + (live ? mg : 0);
-            float *dst = p.out_f + (size_t)p.gidx[row] * p.d;
-            const float dl = (KIND == kDX && live) ? p.dlogit[row] : 0.f;
+            // Transpose each 32 x 32 block through this warp's shared buffer so that
+            // every red.add.v4 instruction covers four whole 128-byte row segments.
+            uint8_t *xb = s_xpose + q * 4096;
+            const int chunk = lane & 7;
 #pragma unroll 1
             for (int c0 = 0; c0 < C::BN; c0 += 32) {
                 float v[32];
                 tmem_ld32(tb + c0, v);
-                if (!live) continue;
 #pragma unroll
-                for (int e = 0; e < 32; e += 4) {
-                    const int n = n0 + c0 + e;
-                    if (n < p.d) {
+                for (int c = 0; c < 8; ++c)
+                    *reinterpret_cast<float4 *>(xb + lane * 128 + ((c ^ (lane & 7)) << 4)) =
+                        make_float4(v[4 * c], v[4 * c + 1], v[4 * c + 2], v[4 * c + 3]);
+                __syncwarp();
+                const int n = n0 + c0 + 4 * chunk;
+                float w[4] = {0.f, 0.f, 0.f, 0.f};
+                if (KIND == kDX && n < p.d) {
+#pragma unroll
+                    for (int u = 0; u < 4; ++u) w[u] = __bfloat162float(p.Wr[(size_t)(n + u) * p.H + h]);
+                }
+#pragma unroll
+                for (int i = 0; i < 8; ++i) {
+                    const int rl = (lane >> 3) + 4 * i;
+                    const int rt = q * 32 + rl;
+                    float4 val = *reinterpret_cast<const float4 *>(xb + rl * 128 + ((chunk ^ (rl & 7)) << 4));
+                    if (!abort && m0 + rt < p.M && n < p.d) {
                         if (KIND == kDX) {
-#pragma unroll
-                            for (int u = 0; u < 4; ++u)
-                                v[e + u] = fmaf(dl, __bfloat162float(p.Wr[(size_t)(n + u) * p.H + h]), v[e + u]);
+                            const float dl = s_dl[rt];
+                            val.x = fmaf(dl, w[0], val.x);
+                            val.y = fmaf(dl, w[1], val.y);
+                            val.z = fmaf(dl, w[2], val.z);
+                            val.w = fmaf(dl, w[3], val.w);
                         }
-                        red_add_v4(dst + n, v[e], v[e + 1], v[e + 2], v[e + 3]);
+                        red_add_v4(p.out_f + (size_t)s_rows[rt] * p.d + n, val.x, val.y, val.z, val.w);
                     }
                 }
+                __syncwarp();
             }
         } else if constexpr (KIND == kG) {
             float g[64];
@@ -430,7 +459,23 @@ __global__ void __launch_bounds__(kThreads, 1) tc_gemm_kernel(const __grid_const
                 for (int e = 0; e < 32; ++e) half[e] = g[32 + e];
                 store_pair_row32(base + 32, base + 96, half);
                 p.out_f1[row] = dd;
-                p.out_f2[row] = dr * rr * (1.f - rr);
+                const float dl = dr * rr * (1.f - rr);
+                p.out_f2[row] = dl;
+                // column block 3 of the dQKV pair: dlogit, then zeros (read by kDW for dW_r)
+                bf16 *drow = static_cast<bf16 *>(p.out[1]) + row * kDQKVCols;
+                const bf16 dh = __float2bfloat16_rn(dl);
+                const bf16 dlo = __float2bfloat16_rn(dl - __bfloat162float(dh));
+                const uint4 z = make_uint4(0, 0, 0, 0);
+#pragma unroll
+                for (int e = 0; e < 8; ++e) {
+                    uint4 vh = z, vl = z;
+                    if (e == 0) {
+                        vh.x = (uint32_t)__bfloat16_as_ushort(dh);
+                        vl.x = (uint32_t)__bfloat16_as_ushort(dlo);
+                    }
+                    reinterpret_cast<uint4 *>(drow + 192)[e] = vh;
+                    reinterpret_cast<uint4 *>(drow + 448)[e] = vl;
+                }
             }
         } else if constexpr (KIND == kROUTER) {
             const bool live = !abort && mg < p.M;
@@ -480,6 +525,15 @@ __global__ void __launch_bounds__(kThreads, 1) tc_gemm_kernel(const __grid_const
                         *reinterpret_cast<float4 *>(dst + e) = make_float4(v[e], v[e + 1], v[e + 2], v[e + 3]);
                 }
             }
+            float v[32];
+            tmem_ld32(tb + 192, v);  // column 192: dW_r[c, h]
+            if (live) {
+                float *dst = p.out_f3 + (size_t)mg * p.H + h;
+                if (p.splits > 1)
+                    atomicAdd(dst, v[0]);
+                else
+                    *dst = v[0];
+            }
         }
     }
     tc_fence_before();
@@ -492,37 +546,9 @@ __global__ void __launch_bounds__(kThreads, 1) tc_gemm_kernel(const __grid_const
 
 // ------------------------------------------------------------------ host
 
-PFN_cuTensorMapEncodeTiled_v12000 encode_fn() {
-    static PFN_cuTensorMapEncodeTiled_v12000 fn = nullptr;
-    static std::once_flag once;
-    std::call_once(once, [] {
-        void *ptr = nullptr;
-        cudaDriverEntryPointQueryResult q;
-        if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &ptr, 12000,
-                                             cudaEnableDefault, &q) == cudaSuccess &&
-            q == cudaDriverEntryPointSuccess)
-            fn = reinterpret_cast<PFN_cuTensorMapEncodeTiled_v12000>(ptr);
-    });
-    return fn;
-}
-
-// bf16 tensor map with 128-byte swizzle.  dims innermost first; strides in
-// bytes for dims 1..rank-1; box innermost first.
 bool make_map(CUtensorMap *m, const void *base, int rank, const uint64_t *dims,
               const uint64_t *strides, const uint32_t *box) {
-    auto fn = encode_fn();
-    if (!fn) return false;
-    cuuint64_t gd[3], gs[2];
-    cuuint32_t bx[3], es[3] = {1, 1, 1};
-    for (int i = 0; i < rank; ++i) {
-        gd[i] = dims[i];
-        bx[i] = box[i];
-    }
-    for (int i = 0; i < rank - 1; ++i) gs[i] = strides[i];
-    CUresult r = fn(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, (cuuint32_t)rank, const_cast<void *>(base),
-                    gd, gs, bx, es, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
-                    CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
-    return r == CUDA_SUCCESS;
+    return tmap_bf16(m, base, rank, dims, strides, box);
 }
 
 // Rows of a [rows, cols] bf16 matrix fetched one row (64 columns) at a time by gather4.
@@ -585,7 +611,7 @@ bool map_2d(CUtensorMap *m, const void *base, uint64_t rows, uint64_t cols, uint
 
 bool tc_router(const Dims &dm, const void *X, const void *Wr, float *r_full, uint32_t *status,
                cudaStream_t s, cudaError_t *err) {
-    if (!dm.bf16 || dm.H % 8 != 0 || encode_fn() == nullptr) return false;
+    if (!dm.bf16 || dm.H % 8 != 0 || !tmap_available()) return false;
     TcParams p;
     memset(&p, 0, sizeof(p));
     p.M = dm.B * dm.T;
@@ -605,7 +631,7 @@ bool tc_router(const Dims &dm, const void *X, const void *Wr, float *r_full, uin
 }
 
 bool tc_supported(const Dims &dm) {
-    return dm.bf16 && dm.hp == 64 && encode_fn() != nullptr;
+    return dm.bf16 && dm.hp == 64 && tmap_available();
 }
 
 cudaError_t tc_qkv(const Dims &dm, const void *X, const void *Wq, const void *Wk, const void *Wv,
@@ -652,6 +678,7 @@ cudaError_t tc_out_bwd(const Dims &dm, const void *Wo, const void *dY, const Sav
     p.src_rows = dY;
     p.A32 = sv.A;
     p.out[0] = sv.dA;
+    p.out[1] = sv.dQKV;
     p.out_f1 = sv.Dd;
     p.out_f2 = sv.dlogit;
     dim3 grid((p.M + kBM - 1) / kBM, 1, dm.H);
@@ -685,7 +712,7 @@ cudaError_t tc_in_bwd(const Dims &dm, const void *Wq, const void *Wk, const void
     p.N = dm.d;
     p.nkb = 3;
     const void *W[3] = {Wq, Wk, Wv};
-    bool ok = map_heads(&p.mapA, sv.dQKV, dm.H, p.Mtok, 384, 128);
+    bool ok = map_heads(&p.mapA, sv.dQKV, dm.H, p.Mtok, kDQKVCols, 128);
     for (int j = 0; j < 3; ++j) ok = ok && map_heads(&p.mapB[j], W[j], dm.H, dm.d, 64, 256);
     if (!ok) return cudaErrorInvalidValue;
     p.dlogit = sv.dlogit;
@@ -696,25 +723,28 @@ cudaError_t tc_in_bwd(const Dims &dm, const void *Wq, const void *Wk, const void
 }
 
 cudaError_t tc_w_bwd(const Dims &dm, const void *X, const Saved &sv, float *dWq, float *dWk,
-                     float *dWv, cudaStream_t s) {
+                     float *dWv, float *dWr, cudaStream_t s) {
     TcParams p = base_params(dm, sv);
     p.M = dm.d;
     p.nkb = (p.Mtok + kBK - 1) / kBK;
     const int tiles = (dm.d + kBM - 1) / kBM * dm.H;
     p.splits = splits_for(tiles, p.nkb);
     bool ok = map_gather(&p.mapA, X, (uint64_t)dm.B * dm.T, dm.d) &&
-              map_heads(&p.mapB[0], sv.dQKV, dm.H, p.Mtok, 384, 64);
+              map_heads(&p.mapB[0], sv.dQKV, dm.H, p.Mtok, kDQKVCols, 64);
     if (!ok) return cudaErrorInvalidValue;
     p.src_rows = X;
     p.out_f = dWq;
     p.out_f1 = dWk;
     p.out_f2 = dWv;
+    p.out_f3 = dWr;
     if (p.splits > 1) {
         const size_t n = sizeof(float) * (size_t)dm.H * dm.d * 64;
         cudaError_t e;
         if ((e = cudaMemsetAsync(dWq, 0, n, s)) != cudaSuccess) return e;
         if ((e = cudaMemsetAsync(dWk, 0, n, s)) != cudaSuccess) return e;
         if ((e = cudaMemsetAsync(dWv, 0, n, s)) != cudaSuccess) return e;
+        if ((e = cudaMemsetAsync(dWr, 0, sizeof(float) * (size_t)dm.d * dm.H, s)) != cudaSuccess)
+            return e;
     }
     dim3 grid((dm.d + kBM - 1) / kBM, 1, dm.H * p.splits);
     return launch_kind<kDW>(p, grid, s);

@@ -342,18 +342,24 @@ def main():
     torch.cuda.synchronize()
     launches0 = mosa.mosa_kernel_launches()
     mosa.mosa_profile_stages(1 << STAGES.index(dominant))
+    mosa.mosa_profile_read()
+    dom = [0.0, 0]
     t_host0 = time.time()
     for i in range(K):
         flush_buf.zero_()
         starts[i].record()
         step()
         ends[i].record()
+        # the dominant stage's events of this step (waits for the step to end;
+        # the next step's L2 flush covers the host time this takes)
+        ms, n = mosa.mosa_profile_read()[dominant]
+        dom[0] += ms
+        dom[1] += n
     torch.cuda.synchronize()
     t_host1 = time.time()
     barrier()
     launches = mosa.mosa_kernel_launches() - launches0
     mosa.mosa_profile_stages(0)
-    dom = mosa.mosa_profile_read()[dominant]
     clocks = None
     if sampler:
         sampler.mark(t_host0, t_host1)
@@ -361,8 +367,10 @@ def main():
     total_ms = sum(s.elapsed_time(e) for s, e in zip(starts, ends))
     value, total_ms = combine_ranks(total_ms, cfg.B * cfg.T * K, dist, dev)
 
-    # Diagnostic: the same step replayed from a CUDA graph (host launch cost removed).
+    # Diagnostic: the same step replayed from a CUDA graph captured by torch
+    # around the eager calls (the library's own graph cache switched off).
     graph_ms = None
+    os.environ["MOSA_GRAPHS"] = "0"
     try:
         g = torch.cuda.CUDAGraph()
         side = torch.cuda.Stream()
@@ -389,6 +397,8 @@ def main():
         del g
     except Exception as exc:  # capture unsupported: report why
         graph_ms = f"unavailable: {exc}"
+    finally:
+        os.environ.pop("MOSA_GRAPHS", None)
 
     # End to end through the public API with pinned host buffers.
     hX = torch.from_numpy(x["X"]).to(tdt).pin_memory()

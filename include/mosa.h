@@ -26,6 +26,13 @@
  *       dW_r      [d,H]  dW_q,dW_k,dW_v [H,d,h']  dW_o [H,h',d]   fp32
  *   - Calls are asynchronous on `stream` (a cudaStream_t, NULL = legacy default
  *     stream).  They return after argument validation and kernel launch.
+ *   - mosa_forward, mosa_forward_with_indices and mosa_backward capture their
+ *     launch sequence into a CUDA graph the first time they see a given
+ *     shape, set of pointers and kernel path, and replay that graph on later
+ *     identical calls (one launch instead of about a dozen).  The capture runs
+ *     on an internal stream of the current device.  Up to 128 graphs are kept
+ *     (driver resources, no user memory); further new calls run unrecorded.
+ *     Setting the environment variable MOSA_GRAPHS=0 turns this off.
  *   - Outputs are overwritten, never accumulated into.
  *   - Arithmetic: fp32 accumulation everywhere; with bf16 storage the saved
  *     intermediates (Q, K, V, attention output, gradients fed to tensor-core

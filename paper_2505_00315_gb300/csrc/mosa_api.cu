@@ -1,7 +1,10 @@
 // C ABI of libmosa (declared in include/mosa.h): argument validation,
 // workspace carving and the launch sequence of the forward and backward
 // passes of the MoSA layer (Sec. 2.2, Eq. mosa_mha).
+#include <cstdlib>
 #include <cstring>
+#include <mutex>
+#include <unordered_map>
 
 #include "../../include/mosa.h"
 #include "launch.h"
@@ -98,6 +101,102 @@ mosa_status forward_heads(const Dims &dm, const void *X, const void *W_q, const 
     return MOSA_OK;
 }
 
+// ---------------------------------------------------------- graph cache
+// A layer call enqueues about a dozen kernels and memsets; launched one by one
+// from the host that costs tens of microseconds per call.  The first call with
+// a given shape, set of pointers, kernel path and stage-timing mask is captured
+// on an internal stream into a CUDA graph; later identical calls launch that
+// graph on the caller's stream.  MOSA_GRAPHS=0 turns this off.
+
+struct GraphKey {
+    int op, device, tc;
+    uint32_t mask;
+    mosa_shape shape;
+    const void *ptr[18];
+    bool operator==(const GraphKey &o) const { return std::memcmp(this, &o, sizeof(GraphKey)) == 0; }
+};
+
+struct GraphKeyHash {
+    size_t operator()(const GraphKey &k) const {
+        const unsigned char *b = reinterpret_cast<const unsigned char *>(&k);
+        uint64_t h = 1469598103934665603ull;
+        for (size_t i = 0; i < sizeof(GraphKey); ++i) h = (h ^ b[i]) * 1099511628211ull;
+        return (size_t)h;
+    }
+};
+
+struct GraphEntry {
+    cudaGraphExec_t exec = nullptr;
+    CaptureRecord rec;
+};
+
+constexpr size_t kMaxGraphs = 128;
+constexpr int kMaxDevices = 64;
+std::mutex g_graph_mu;
+std::unordered_map<GraphKey, GraphEntry *, GraphKeyHash> g_graphs;
+cudaStream_t g_capture_stream[kMaxDevices] = {};
+
+bool graphs_enabled() {
+    const char *v = std::getenv("MOSA_GRAPHS");
+    return v == nullptr || v[0] != '0';
+}
+
+GraphKey make_key(int op, const Dims &dm, const mosa_shape *shape,
+                  std::initializer_list<const void *> ptrs) {
+    GraphKey k;
+    std::memset(&k, 0, sizeof(k));
+    k.op = op;
+    cudaGetDevice(&k.device);
+    k.tc = use_tc(dm) ? 1 : 0;
+    k.mask = profile_mask();
+    k.shape = *shape;
+    int i = 0;
+    for (const void *p : ptrs) k.ptr[i++] = p;
+    return k;
+}
+
+// Runs `enqueue(stream)`, through a cached CUDA graph when possible.
+template <class Enqueue>
+mosa_status run_graphed(const GraphKey &key, cudaStream_t user, Enqueue &&enqueue) {
+    if (!graphs_enabled() || key.device < 0 || key.device >= kMaxDevices) return enqueue(user);
+    std::lock_guard<std::mutex> lk(g_graph_mu);
+    auto it = g_graphs.find(key);
+    GraphEntry *e = it == g_graphs.end() ? nullptr : it->second;
+    if (e == nullptr) {
+        if (g_graphs.size() >= kMaxGraphs) return enqueue(user);
+        cudaStream_t &cs = g_capture_stream[key.device];
+        if (cs == nullptr && cudaStreamCreateWithFlags(&cs, cudaStreamNonBlocking) != cudaSuccess) {
+            cs = nullptr;
+            return enqueue(user);
+        }
+        e = new GraphEntry;
+        capture_into(&e->rec);
+        mosa_status st = MOSA_ERR_CUDA;
+        cudaGraph_t g = nullptr;
+        if (cudaStreamBeginCapture(cs, cudaStreamCaptureModeThreadLocal) == cudaSuccess) {
+            st = enqueue(cs);
+            if (cudaStreamEndCapture(cs, &g) != cudaSuccess) st = MOSA_ERR_CUDA;
+        }
+        capture_into(nullptr);
+        if (st == MOSA_OK && g != nullptr && cudaGraphInstantiate(&e->exec, g, 0) != cudaSuccess)
+            st = MOSA_ERR_CUDA;
+        if (g != nullptr) cudaGraphDestroy(g);
+        if (st != MOSA_OK) {
+            (void)cudaGetLastError();
+            for (auto &q : e->rec.pairs) {
+                cudaEventDestroy(q.start);
+                cudaEventDestroy(q.stop);
+            }
+            delete e;
+            return enqueue(user);  // capture failed: run the same work directly
+        }
+        g_graphs.emplace(key, e);
+    }
+    if (cudaGraphLaunch(e->exec, user) != cudaSuccess) return MOSA_ERR_CUDA;
+    replayed(e->rec);
+    return MOSA_OK;
+}
+
 }  // namespace
 }  // namespace mosa
 
@@ -134,19 +233,23 @@ mosa_status mosa_forward(const mosa_shape *shape, const void *X, const void *W_r
         return MOSA_ERR_INVALID_ARG;
     Saved sv;
     if ((st = check_workspace(dm, workspace, workspace_bytes, &sv)) != MOSA_OK) return st;
-    cudaStream_t s = (cudaStream_t)stream;
     float *rf = r_full ? r_full : sv.r_full;
-    MOSA_TRY(cudaMemsetAsync(sv.status, 0, sizeof(uint32_t), s));
-    {
-        StageScope st_(kStageRouter, s);
-        MOSA_TRY(launch_router_auto(dm, X, W_r, rf, sv.status, s));
-    }
-    {
-        StageScope st_(kStageSelect, s);
-        MOSA_TRY(launch_select(dm.B * dm.H, dm.T, dm.k, rf, I, r_sel, dm.B, dm.H, sv.gidx,
-                               sv.rsel, s));
-    }
-    return forward_heads(dm, X, W_q, W_k, W_v, W_o, Y, sv, s);
+    auto enqueue = [&](cudaStream_t s) -> mosa_status {
+        MOSA_TRY(cudaMemsetAsync(sv.status, 0, sizeof(uint32_t), s));
+        {
+            StageScope st_(kStageRouter, s);
+            MOSA_TRY(launch_router_auto(dm, X, W_r, rf, sv.status, s));
+        }
+        {
+            StageScope st_(kStageSelect, s);
+            MOSA_TRY(launch_select(dm.B * dm.H, dm.T, dm.k, rf, I, r_sel, dm.B, dm.H, sv.gidx,
+                                   sv.rsel, s));
+        }
+        return forward_heads(dm, X, W_q, W_k, W_v, W_o, Y, sv, s);
+    };
+    const GraphKey key = make_key(0, dm, shape, {X, W_r, W_q, W_k, W_v, W_o, Y, I, r_sel, r_full,
+                                                 workspace});
+    return run_graphed(key, (cudaStream_t)stream, enqueue);
 }
 
 mosa_status mosa_forward_with_indices(const mosa_shape *shape, const void *X, const void *W_q,
@@ -159,13 +262,16 @@ mosa_status mosa_forward_with_indices(const mosa_shape *shape, const void *X, co
     if (!X || !W_q || !W_k || !W_v || !W_o || !I || !r_sel || !Y) return MOSA_ERR_INVALID_ARG;
     Saved sv;
     if ((st = check_workspace(dm, workspace, workspace_bytes, &sv)) != MOSA_OK) return st;
-    cudaStream_t s = (cudaStream_t)stream;
-    MOSA_TRY(cudaMemsetAsync(sv.status, 0, sizeof(uint32_t), s));
-    {
-        StageScope st_(kStageSelect, s);
-        MOSA_TRY(launch_indices_to_rows(dm, I, r_sel, sv.gidx, sv.rsel, sv.status, s));
-    }
-    return forward_heads(dm, X, W_q, W_k, W_v, W_o, Y, sv, s);
+    auto enqueue = [&](cudaStream_t s) -> mosa_status {
+        MOSA_TRY(cudaMemsetAsync(sv.status, 0, sizeof(uint32_t), s));
+        {
+            StageScope st_(kStageSelect, s);
+            MOSA_TRY(launch_indices_to_rows(dm, I, r_sel, sv.gidx, sv.rsel, sv.status, s));
+        }
+        return forward_heads(dm, X, W_q, W_k, W_v, W_o, Y, sv, s);
+    };
+    const GraphKey key = make_key(1, dm, shape, {X, W_q, W_k, W_v, W_o, I, r_sel, Y, workspace});
+    return run_graphed(key, (cudaStream_t)stream, enqueue);
 }
 
 mosa_status mosa_backward(const mosa_shape *shape, const void *X, const void *W_r,
@@ -181,24 +287,28 @@ mosa_status mosa_backward(const mosa_shape *shape, const void *X, const void *W_
         return MOSA_ERR_INVALID_ARG;
     Saved sv;
     if ((st = check_workspace(dm, workspace, workspace_bytes, &sv)) != MOSA_OK) return st;
-    cudaStream_t s = (cudaStream_t)stream;
-    {
-        StageScope st_(kStageOutBwd, s);
-        MOSA_TRY(launch_out_bwd(dm, W_o, dY, sv, dW_o, s));
-    }
-    {
-        StageScope st_(kStageAttnBwd, s);
-        MOSA_TRY(launch_attn_bwd(dm, sv, s));
-    }
-    {
-        StageScope st_(kStageInBwd, s);
-        MOSA_TRY(launch_in_bwd(dm, W_q, W_k, W_v, W_r, sv, dX, s));
-    }
-    {
-        StageScope st_(kStageWBwd, s);
-        MOSA_TRY(launch_w_bwd(dm, X, sv, dW_q, dW_k, dW_v, dW_r, s));
-    }
-    return MOSA_OK;
+    auto enqueue = [&](cudaStream_t s) -> mosa_status {
+        {
+            StageScope st_(kStageOutBwd, s);
+            MOSA_TRY(launch_out_bwd(dm, W_o, dY, sv, dW_o, s));
+        }
+        {
+            StageScope st_(kStageAttnBwd, s);
+            MOSA_TRY(launch_attn_bwd(dm, sv, s));
+        }
+        {
+            StageScope st_(kStageInBwd, s);
+            MOSA_TRY(launch_in_bwd(dm, W_q, W_k, W_v, W_r, sv, dX, s));
+        }
+        {
+            StageScope st_(kStageWBwd, s);
+            MOSA_TRY(launch_w_bwd(dm, X, sv, dW_q, dW_k, dW_v, dW_r, s));
+        }
+        return MOSA_OK;
+    };
+    const GraphKey key = make_key(2, dm, shape, {X, W_r, W_q, W_k, W_v, W_o, I, r_sel, dY, dX,
+                                                 dW_r, dW_q, dW_k, dW_v, dW_o, workspace});
+    return run_graphed(key, (cudaStream_t)stream, enqueue);
 }
 
 mosa_status mosa_topk(int32_t rows, int32_t T, int32_t k, const float *scores, int32_t *I,

@@ -18,7 +18,9 @@ std::mutex g_mu;
 struct Pending {
     int stage;
     cudaEvent_t start, stop;
+    bool recycle;  // false for events owned by a captured graph
 };
+thread_local CaptureRecord *t_capture = nullptr;
 std::vector<Pending> g_pending;
 std::vector<cudaEvent_t> g_free;
 double g_ms[kNumStages] = {};
@@ -40,10 +42,36 @@ cudaEvent_t take_event() {
 
 }  // namespace
 
-void note_launches(int n) { g_launches.fetch_add((unsigned long long)n, std::memory_order_relaxed); }
+void note_launches(int n) {
+    if (t_capture != nullptr) {
+        t_capture->launches += (unsigned long long)n;
+        return;
+    }
+    g_launches.fetch_add((unsigned long long)n, std::memory_order_relaxed);
+}
+
+void capture_into(CaptureRecord *rec) { t_capture = rec; }
+
+uint32_t profile_mask() { return g_mask.load(std::memory_order_relaxed); }
+
+void replayed(const CaptureRecord &rec) {
+    g_launches.fetch_add(rec.launches, std::memory_order_relaxed);
+    if (rec.pairs.empty()) return;
+    std::lock_guard<std::mutex> lk(g_mu);
+    for (const CaptureRecord::Pair &q : rec.pairs) g_pending.push_back({q.stage, q.start, q.stop, false});
+}
 
 StageScope::StageScope(int stage, cudaStream_t s) : stage_(stage), stream_(s) {
     if (!(g_mask.load(std::memory_order_relaxed) & (1u << stage))) return;
+    if (t_capture != nullptr) {
+        // recorded into the graph: these events live as long as the graph
+        // External records become event nodes of the graph (a plain record
+        // during capture would only mark a dependency inside the capture).
+        if (cudaEventCreate(&start_) == cudaSuccess && cudaEventCreate(&stop_) == cudaSuccess &&
+            cudaEventRecordWithFlags(start_, s, cudaEventRecordExternal) == cudaSuccess)
+            active_ = true;
+        return;
+    }
     std::lock_guard<std::mutex> lk(g_mu);
     start_ = take_event();
     stop_ = take_event();
@@ -54,8 +82,14 @@ StageScope::StageScope(int stage, cudaStream_t s) : stage_(stage), stream_(s) {
 
 StageScope::~StageScope() {
     if (!active_) return;
+    if (t_capture != nullptr) {
+        if (cudaEventRecordWithFlags(stop_, stream_, cudaEventRecordExternal) == cudaSuccess)
+            t_capture->pairs.push_back({stage_, start_, stop_});
+        return;
+    }
     std::lock_guard<std::mutex> lk(g_mu);
-    if (cudaEventRecord(stop_, stream_) == cudaSuccess) g_pending.push_back({stage_, start_, stop_});
+    if (cudaEventRecord(stop_, stream_) == cudaSuccess)
+        g_pending.push_back({stage_, start_, stop_, true});
 }
 
 }  // namespace mosa
@@ -80,8 +114,10 @@ int32_t mosa_profile_read(double *total_ms, int32_t *count, int32_t max_stages) 
             g_ms[p.stage] += ms;
             g_count[p.stage] += 1;
         }
-        g_free.push_back(p.start);
-        g_free.push_back(p.stop);
+        if (p.recycle) {
+            g_free.push_back(p.start);
+            g_free.push_back(p.stop);
+        }
     }
     g_pending.clear();
     const int n = max_stages < kNumStages ? max_stages : kNumStages;

@@ -3,6 +3,8 @@
 
 #include <cuda_runtime.h>
 
+#include <vector>
+
 namespace mosa {
 
 enum Stage : int {
@@ -10,8 +12,26 @@ enum Stage : int {
     kStageOutBwd, kStageAttnBwd, kStageInBwd, kStageWBwd, kStageRows, kNumStages
 };
 
-// Adds n to the library's kernel-launch counter.
+// Adds n to the library's kernel-launch counter (or, while this thread is
+// capturing a graph, to the capture's own count).
 void note_launches(int n);
+
+// Stage-timing event pairs and kernel count recorded while a graph is being
+// captured; they belong to the graph and are re-armed on every replay.
+struct CaptureRecord {
+    struct Pair {
+        int stage;
+        cudaEvent_t start, stop;
+    };
+    std::vector<Pair> pairs;
+    unsigned long long launches = 0;
+};
+// Routes StageScope and note_launches of this thread into `rec` (nullptr ends).
+void capture_into(CaptureRecord *rec);
+// Accounts one replay of a captured graph: its kernels and its timing pairs.
+void replayed(const CaptureRecord &rec);
+// Stage-timing mask currently in force.
+uint32_t profile_mask();
 
 // Records a CUDA event pair around one stage when that stage's timing is on.
 class StageScope {

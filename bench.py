@@ -167,7 +167,7 @@ def cpu_baseline(cfg, x, budget_s):
 # ------------------------------------------------------------ roofline
 
 STAGES = ["router", "select", "qkv", "attn_fwd", "out", "out_bwd", "attn_bwd", "in_bwd",
-          "w_bwd"]
+          "w_bwd", "dwo"]
 
 
 def stage_bound(stage, peaks, kind):

@@ -60,11 +60,17 @@ bool tc_supported(const Dims &dm);
 bool use_tc(const Dims &dm);
 cudaError_t tc_qkv(const Dims &dm, const void *X, const void *Wq, const void *Wk, const void *Wv,
                    const Saved &sv, cudaStream_t s);
-cudaError_t tc_out(const Dims &dm, const void *Wo, const Saved &sv, float *Y, cudaStream_t s);
-cudaError_t tc_out_bwd(const Dims &dm, const void *Wo, const void *dY, const Saved &sv,
-                       float *dWo, cudaStream_t s);
+// zero_output = false: the caller has already zeroed Y / dX on this stream's timeline.
+cudaError_t tc_out(const Dims &dm, const void *Wo, const Saved &sv, float *Y, cudaStream_t s,
+                   bool zero_output);
+// B1 in two independent parts: G and the row terms; dW_o.
+cudaError_t tc_out_bwd_g(const Dims &dm, const void *Wo, const void *dY, const Saved &sv,
+                         cudaStream_t s);
+cudaError_t tc_out_bwd_w(const Dims &dm, const void *dY, const Saved &sv, float *dWo,
+                         cudaStream_t s);
 cudaError_t tc_in_bwd(const Dims &dm, const void *Wq, const void *Wk, const void *Wv,
-                      const void *Wr, const Saved &sv, float *dX, cudaStream_t s);
+                      const void *Wr, const Saved &sv, float *dX, cudaStream_t s,
+                      bool zero_output);
 // F1 on tensor cores (bf16 inputs, H % 8 == 0); false if not applicable.
 bool tc_router(const Dims &dm, const void *X, const void *Wr, float *r_full, uint32_t *status,
                cudaStream_t s, cudaError_t *err);

@@ -82,6 +82,42 @@ mosa_status cuda_status(cudaError_t e) { return e == cudaSuccess ? MOSA_OK : MOS
         if (_e != cudaSuccess) return MOSA_ERR_CUDA;    \
     } while (0)
 
+// ------------------------------------------------ concurrent branches
+// On the tensor-core path independent kernels run on a second, internal
+// stream joined back with events (graph branches when captured):
+//   forward:  zeroing Y runs beside router .. attention;
+//   backward: dW_o and the zeroing of dX and the weight gradients run beside
+//             G -> attention backward; then dX and dW run side by side.
+struct DevResources {
+    cudaStream_t side = nullptr;
+    cudaEvent_t ev[4] = {};
+};
+constexpr int kMaxDev = 64;
+std::mutex g_res_mu;
+DevResources g_res[kMaxDev];
+
+DevResources *dev_resources() {
+    int dev = 0;
+    if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= kMaxDev) return nullptr;
+    std::lock_guard<std::mutex> lk(g_res_mu);
+    DevResources &r = g_res[dev];
+    if (r.side == nullptr) {
+        if (cudaStreamCreateWithFlags(&r.side, cudaStreamNonBlocking) != cudaSuccess) {
+            r.side = nullptr;
+            return nullptr;
+        }
+        for (auto &e : r.ev)
+            if (cudaEventCreateWithFlags(&e, cudaEventDisableTiming) != cudaSuccess) return nullptr;
+    }
+    return &r;
+}
+
+// `to` waits for the work enqueued so far on `from`.
+cudaError_t link(cudaStream_t from, cudaStream_t to, cudaEvent_t ev) {
+    cudaError_t e = cudaEventRecord(ev, from);
+    return e != cudaSuccess ? e : cudaStreamWaitEvent(to, ev, 0);
+}
+
 // F3-F5 for the rows already selected into sv.gidx / sv.rsel.
 mosa_status forward_heads(const Dims &dm, const void *X, const void *W_q, const void *W_k,
                           const void *W_v, const void *W_o, float *Y, const Saved &sv,
@@ -98,6 +134,76 @@ mosa_status forward_heads(const Dims &dm, const void *X, const void *W_q, const 
         StageScope st_(kStageOut, s);
         MOSA_TRY(launch_out(dm, W_o, sv, Y, s));
     }
+    return MOSA_OK;
+}
+
+// Tensor-core forward: Y is zeroed on the side stream while the head steps run.
+mosa_status forward_tc(const Dims &dm, const void *X, const void *W_r, const void *W_q,
+                       const void *W_k, const void *W_v, const void *W_o, float *Y, int32_t *I,
+                       float *r_sel, float *rf, bool route, const int32_t *I_in,
+                       const float *rsel_in, const Saved &sv, cudaStream_t s, DevResources &r) {
+    MOSA_TRY(link(s, r.side, r.ev[0]));
+    MOSA_TRY(cudaMemsetAsync(Y, 0, sizeof(float) * (size_t)dm.B * dm.T * dm.d, r.side));
+    MOSA_TRY(cudaMemsetAsync(sv.status, 0, sizeof(uint32_t), s));
+    if (route) {
+        {
+            StageScope st_(kStageRouter, s);
+            MOSA_TRY(launch_router_auto(dm, X, W_r, rf, sv.status, s));
+        }
+        StageScope st_(kStageSelect, s);
+        MOSA_TRY(launch_select(dm.B * dm.H, dm.T, dm.k, rf, I, r_sel, dm.B, dm.H, sv.gidx,
+                               sv.rsel, s));
+    } else {
+        StageScope st_(kStageSelect, s);
+        MOSA_TRY(launch_indices_to_rows(dm, I_in, rsel_in, sv.gidx, sv.rsel, sv.status, s));
+    }
+    {
+        StageScope st_(kStageQkv, s);
+        MOSA_TRY(launch_qkv(dm, X, W_q, W_k, W_v, sv, s));
+    }
+    {
+        StageScope st_(kStageAttnFwd, s);
+        MOSA_TRY(launch_attn_fwd(dm, sv, s));
+    }
+    MOSA_TRY(link(r.side, s, r.ev[1]));
+    {
+        StageScope st_(kStageOut, s);
+        MOSA_TRY(tc_out(dm, W_o, sv, Y, s, false));
+    }
+    return MOSA_OK;
+}
+
+// Tensor-core backward with two branches (see above).
+mosa_status backward_tc(const Dims &dm, const void *X, const void *W_r, const void *W_q,
+                        const void *W_k, const void *W_v, const void *W_o, const void *dY,
+                        float *dX, float *dW_r, float *dW_q, float *dW_k, float *dW_v,
+                        float *dW_o, const Saved &sv, cudaStream_t s, DevResources &r) {
+    cudaStream_t t = r.side;
+    MOSA_TRY(link(s, t, r.ev[0]));
+    {
+        StageScope st_(kStageDwo, t);
+        MOSA_TRY(tc_out_bwd_w(dm, dY, sv, dW_o, t));
+    }
+    MOSA_TRY(cudaMemsetAsync(dX, 0, sizeof(float) * (size_t)dm.B * dm.T * dm.d, t));
+    MOSA_TRY(link(t, s, r.ev[1]));  // dX zeroed before the scatter into it
+    {
+        StageScope st_(kStageOutBwd, s);
+        MOSA_TRY(tc_out_bwd_g(dm, W_o, dY, sv, s));
+    }
+    {
+        StageScope st_(kStageAttnBwd, s);
+        MOSA_TRY(launch_attn_bwd(dm, sv, s));
+    }
+    MOSA_TRY(link(s, t, r.ev[2]));  // dQ|dK|dV|dlogit ready for dW
+    {
+        StageScope st_(kStageWBwd, t);
+        MOSA_TRY(tc_w_bwd(dm, X, sv, dW_q, dW_k, dW_v, dW_r, t));
+    }
+    {
+        StageScope st_(kStageInBwd, s);
+        MOSA_TRY(tc_in_bwd(dm, W_q, W_k, W_v, W_r, sv, dX, s, false));
+    }
+    MOSA_TRY(link(t, s, r.ev[3]));  // join
     return MOSA_OK;
 }
 
@@ -158,8 +264,10 @@ GraphKey make_key(int op, const Dims &dm, const mosa_shape *shape,
 // Runs `enqueue(stream)`, through a cached CUDA graph when possible.
 template <class Enqueue>
 mosa_status run_graphed(const GraphKey &key, cudaStream_t user, Enqueue &&enqueue) {
-    if (!graphs_enabled() || key.device < 0 || key.device >= kMaxDevices) return enqueue(user);
+    // One lock for both paths: the eager path shares the internal side stream
+    // and its events between calls.
     std::lock_guard<std::mutex> lk(g_graph_mu);
+    if (!graphs_enabled() || key.device < 0 || key.device >= kMaxDevices) return enqueue(user);
     auto it = g_graphs.find(key);
     GraphEntry *e = it == g_graphs.end() ? nullptr : it->second;
     if (e == nullptr) {
@@ -234,7 +342,11 @@ mosa_status mosa_forward(const mosa_shape *shape, const void *X, const void *W_r
     Saved sv;
     if ((st = check_workspace(dm, workspace, workspace_bytes, &sv)) != MOSA_OK) return st;
     float *rf = r_full ? r_full : sv.r_full;
+    DevResources *res = use_tc(dm) ? dev_resources() : nullptr;
     auto enqueue = [&](cudaStream_t s) -> mosa_status {
+        if (res != nullptr)
+            return forward_tc(dm, X, W_r, W_q, W_k, W_v, W_o, Y, I, r_sel, rf, true, nullptr,
+                              nullptr, sv, s, *res);
         MOSA_TRY(cudaMemsetAsync(sv.status, 0, sizeof(uint32_t), s));
         {
             StageScope st_(kStageRouter, s);
@@ -262,7 +374,11 @@ mosa_status mosa_forward_with_indices(const mosa_shape *shape, const void *X, co
     if (!X || !W_q || !W_k || !W_v || !W_o || !I || !r_sel || !Y) return MOSA_ERR_INVALID_ARG;
     Saved sv;
     if ((st = check_workspace(dm, workspace, workspace_bytes, &sv)) != MOSA_OK) return st;
+    DevResources *res = use_tc(dm) ? dev_resources() : nullptr;
     auto enqueue = [&](cudaStream_t s) -> mosa_status {
+        if (res != nullptr)
+            return forward_tc(dm, X, nullptr, W_q, W_k, W_v, W_o, Y, nullptr, nullptr, nullptr,
+                              false, I, r_sel, sv, s, *res);
         MOSA_TRY(cudaMemsetAsync(sv.status, 0, sizeof(uint32_t), s));
         {
             StageScope st_(kStageSelect, s);
@@ -287,7 +403,11 @@ mosa_status mosa_backward(const mosa_shape *shape, const void *X, const void *W_
         return MOSA_ERR_INVALID_ARG;
     Saved sv;
     if ((st = check_workspace(dm, workspace, workspace_bytes, &sv)) != MOSA_OK) return st;
+    DevResources *res = use_tc(dm) ? dev_resources() : nullptr;
     auto enqueue = [&](cudaStream_t s) -> mosa_status {
+        if (res != nullptr)
+            return backward_tc(dm, X, W_r, W_q, W_k, W_v, W_o, dY, dX, dW_r, dW_q, dW_k, dW_v,
+                               dW_o, sv, s, *res);
         {
             StageScope st_(kStageOutBwd, s);
             MOSA_TRY(launch_out_bwd(dm, W_o, dY, sv, dW_o, s));
@@ -331,6 +451,7 @@ int32_t mosa_stage_engine(const mosa_shape *shape, int32_t stage) {
         case kStageOutBwd:
         case kStageInBwd:
         case kStageWBwd:
+        case kStageDwo:
         case kStageAttnFwd:
         case kStageAttnBwd: return use_tc(dm) ? 1 : 0;
         default: return 0;

@@ -27,7 +27,7 @@ double g_ms[kNumStages] = {};
 int32_t g_count[kNumStages] = {};
 
 const char *kNames[kNumStages] = {"router", "select", "qkv", "attn_fwd", "out",
-                                  "out_bwd", "attn_bwd", "in_bwd", "w_bwd", "rows"};
+                                  "out_bwd", "attn_bwd", "in_bwd", "w_bwd", "dwo"};
 
 cudaEvent_t take_event() {
     if (!g_free.empty()) {

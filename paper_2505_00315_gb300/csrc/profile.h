@@ -9,7 +9,7 @@ namespace mosa {
 
 enum Stage : int {
     kStageRouter = 0, kStageSelect, kStageQkv, kStageAttnFwd, kStageOut,
-    kStageOutBwd, kStageAttnBwd, kStageInBwd, kStageWBwd, kStageRows, kNumStages
+    kStageOutBwd, kStageAttnBwd, kStageInBwd, kStageWBwd, kStageDwo, kNumStages
 };
 
 // Adds n to the library's kernel-launch counter (or, while this thread is

@@ -268,19 +268,22 @@ cudaError_t launch_qkv(const Dims &dm, const void *X, const void *Wq, const void
 }
 
 cudaError_t launch_out(const Dims &dm, const void *Wo, const Saved &sv, float *Y, cudaStream_t s) {
-    if (use_tc(dm)) return tc_out(dm, Wo, sv, Y, s);
+    if (use_tc(dm)) return tc_out(dm, Wo, sv, Y, s, true);
     return dm.bf16 ? out_t<bf16>(dm, Wo, sv, Y, s) : out_t<float>(dm, Wo, sv, Y, s);
 }
 
 cudaError_t launch_out_bwd(const Dims &dm, const void *Wo, const void *dY, const Saved &sv,
                            float *dWo, cudaStream_t s) {
-    if (use_tc(dm)) return tc_out_bwd(dm, Wo, dY, sv, dWo, s);
+    if (use_tc(dm)) {
+        cudaError_t e = tc_out_bwd_g(dm, Wo, dY, sv, s);
+        return e != cudaSuccess ? e : tc_out_bwd_w(dm, dY, sv, dWo, s);
+    }
     return dm.bf16 ? out_bwd_t<bf16>(dm, Wo, dY, sv, dWo, s) : out_bwd_t<float>(dm, Wo, dY, sv, dWo, s);
 }
 
 cudaError_t launch_in_bwd(const Dims &dm, const void *Wq, const void *Wk, const void *Wv,
                           const void *Wr, const Saved &sv, float *dX, cudaStream_t s) {
-    if (use_tc(dm)) return tc_in_bwd(dm, Wq, Wk, Wv, Wr, sv, dX, s);
+    if (use_tc(dm)) return tc_in_bwd(dm, Wq, Wk, Wv, Wr, sv, dX, s, true);
     return dm.bf16 ? in_bwd_t<bf16>(dm, Wq, Wk, Wv, Wr, sv, dX, s)
                    : in_bwd_t<float>(dm, Wq, Wk, Wv, Wr, sv, dX, s);
 }

@@ -651,9 +651,12 @@ cudaError_t tc_qkv(const Dims &dm, const void *X, const void *Wq, const void *Wk
     return launch_kind<kQKV>(p, grid, s);
 }
 
-cudaError_t tc_out(const Dims &dm, const void *Wo, const Saved &sv, float *Y, cudaStream_t s) {
-    cudaError_t e = cudaMemsetAsync(Y, 0, sizeof(float) * (size_t)dm.B * dm.T * dm.d, s);
-    if (e != cudaSuccess) return e;
+cudaError_t tc_out(const Dims &dm, const void *Wo, const Saved &sv, float *Y, cudaStream_t s,
+                   bool zero_output) {
+    if (zero_output) {
+        cudaError_t e = cudaMemsetAsync(Y, 0, sizeof(float) * (size_t)dm.B * dm.T * dm.d, s);
+        if (e != cudaSuccess) return e;
+    }
     TcParams p = base_params(dm, sv);
     p.M = p.Mtok;
     p.N = dm.d;
@@ -666,8 +669,8 @@ cudaError_t tc_out(const Dims &dm, const void *Wo, const Saved &sv, float *Y, cu
     return launch_kind<kOUT>(p, grid, s);
 }
 
-cudaError_t tc_out_bwd(const Dims &dm, const void *Wo, const void *dY, const Saved &sv,
-                       float *dWo, cudaStream_t s) {
+cudaError_t tc_out_bwd_g(const Dims &dm, const void *Wo, const void *dY, const Saved &sv,
+                         cudaStream_t s) {
     // G = dY[I] W_o^T with the row terms fused into the epilogue.
     TcParams p = base_params(dm, sv);
     p.M = p.Mtok;
@@ -682,16 +685,20 @@ cudaError_t tc_out_bwd(const Dims &dm, const void *Wo, const void *dY, const Sav
     p.out_f1 = sv.Dd;
     p.out_f2 = sv.dlogit;
     dim3 grid((p.M + kBM - 1) / kBM, 1, dm.H);
-    cudaError_t e = launch_kind<kG>(p, grid, s);
-    if (e != cudaSuccess) return e;
+    return launch_kind<kG>(p, grid, s);
+}
+
+cudaError_t tc_out_bwd_w(const Dims &dm, const void *dY, const Saved &sv, float *dWo,
+                         cudaStream_t s) {
     // dW_o[h](p, c) = sum_m AR(m, p) dY[g(m), c]
+    cudaError_t e;
     TcParams q = base_params(dm, sv);
     q.M = dm.d;
     q.nkb = (q.Mtok + kBK - 1) / kBK;
     const int tiles = (dm.d + kBM - 1) / kBM * dm.H;
     q.splits = splits_for(tiles, q.nkb);
-    ok = map_gather(&q.mapA, dY, (uint64_t)dm.B * dm.T, dm.d) &&
-         map_heads(&q.mapB[0], sv.AR, dm.H, q.Mtok, 128, 64);
+    const bool ok = map_gather(&q.mapA, dY, (uint64_t)dm.B * dm.T, dm.d) &&
+                    map_heads(&q.mapB[0], sv.AR, dm.H, q.Mtok, 128, 64);
     if (!ok) return cudaErrorInvalidValue;
     q.src_rows = dY;
     q.out_f = dWo;
@@ -704,9 +711,11 @@ cudaError_t tc_out_bwd(const Dims &dm, const void *Wo, const void *dY, const Sav
 }
 
 cudaError_t tc_in_bwd(const Dims &dm, const void *Wq, const void *Wk, const void *Wv,
-                      const void *Wr, const Saved &sv, float *dX, cudaStream_t s) {
-    cudaError_t e = cudaMemsetAsync(dX, 0, sizeof(float) * (size_t)dm.B * dm.T * dm.d, s);
-    if (e != cudaSuccess) return e;
+                      const void *Wr, const Saved &sv, float *dX, cudaStream_t s, bool zero_output) {
+    if (zero_output) {
+        cudaError_t e = cudaMemsetAsync(dX, 0, sizeof(float) * (size_t)dm.B * dm.T * dm.d, s);
+        if (e != cudaSuccess) return e;
+    }
     TcParams p = base_params(dm, sv);
     p.M = p.Mtok;
     p.N = dm.d;

@@ -71,8 +71,12 @@ def layer_work(B: int, T: int, d: int, H: int, hp: int, k: int, elem_bytes: int 
         "out": {"flops": 2 * hp * d * k * U,
                 # read scaled A and W_o; fp32 reduction into Y[B,T,d]
                 "bytes": U * k * hp * e + H * hp * d * e + U * k * d * 4},
-        "out_bwd": {"flops": 4 * hp * d * k * U,
-                    "bytes": U * k * d * e + H * hp * d * (e + 4) + 2 * U * k * hp * e},
+        # G = dY[I] W_o^T and the row terms (dr, dA, D, dlogit)
+        "out_bwd": {"flops": 2 * hp * d * k * U,
+                    "bytes": U * k * d * e + H * hp * d * e + 2 * U * k * hp * e},
+        # dW_o = (diag(r) A)^T dY[I]
+        "dwo": {"flops": 2 * hp * d * k * U,
+                "bytes": U * k * d * e + U * k * hp * e + H * hp * d * 4},
         "attn_bwd": {"flops": 5 * causal * U,
                      "bytes": 6 * U * k * hp * e + 3 * U * k * hp * e},
         "in_bwd": {"flops": (6 * d * hp * k + 2 * d * k) * U,
@@ -81,7 +85,7 @@ def layer_work(B: int, T: int, d: int, H: int, hp: int, k: int, elem_bytes: int 
                   "bytes": U * k * d * e + 3 * U * k * hp * e + 3 * H * d * hp * 4 + d * H * 4},
     }
     fwd = ("router", "select", "qkv", "attn_fwd", "out")
-    bwd = ("out_bwd", "attn_bwd", "in_bwd", "w_bwd")
+    bwd = ("out_bwd", "dwo", "attn_bwd", "in_bwd", "w_bwd")
     w["forward_flops"] = sum(w[s]["flops"] for s in fwd)
     w["backward_flops"] = sum(w[s]["flops"] for s in bwd)
     return w

@@ -733,6 +733,341 @@ __global__ void __launch_bounds__(kThreads, 1) attn_dq_tc_kernel(const __grid_co
     }
 }
 
+// ------------------------------------------------- k <= 128: one CTA per unit
+// When a head keeps at most 128 tokens the whole k x k problem of one (b, h)
+// unit fits one CTA: a single 128-key block, no online rescaling (forward) and
+// one fused pass for dQ, dK and dV (backward).  P (then dS) lives in one
+// 128 x 128 bf16-pair tile: K-major (keys contiguous) for P V and dS K, and
+// read through an MN-major descriptor as P^T / dS^T for dV and dK.
+
+constexpr int kSmallK = 128;
+constexpr int kPBig = 128 * 64 * 2;   // one 64-key block of a 128-row tile, one half: 16 KB
+
+struct SmallFwdSmem {
+    uint8_t q[2][kPBig];
+    uint8_t k[2][kPBig];
+    uint8_t v[2][kPBig];
+    uint8_t p[2][2][kPBig];           // [half][key block]
+    uint64_t in_full, s_full, p_ready, o_full;
+    uint32_t tmem;
+    int abort;
+};
+constexpr int kSmallFwdSmem = (int)sizeof(SmallFwdSmem) + 1024;
+
+struct SmallBwdSmem {
+    uint8_t q[2][kPBig];
+    uint8_t k[2][kPBig];
+    uint8_t v[2][kPBig];
+    uint8_t da[2][kPBig];
+    uint8_t p[2][2][kPBig];           // P, then dS
+    uint64_t in_full, sp_full, p_ready, pv_done, ds_ready, acc_done;
+    uint32_t tmem;
+    int abort;
+};
+constexpr int kSmallBwdSmem = (int)sizeof(SmallBwdSmem) + 1024;
+
+// 32 consecutive keys c0..c0+31 of row r of a [128 x 128] pair tile.
+__device__ __forceinline__ void write_pair32(uint8_t (*tile)[2][kPBig], int r, int c0, const float *v) {
+    const int blk = c0 >> 6, cb = (c0 & 63) >> 3;  // 16-byte chunk index within the 128-byte row
+#pragma unroll
+    for (int c = 0; c < 4; ++c) {
+        uint32_t h4[4], l4[4];
+#pragma unroll
+        for (int e = 0; e < 4; ++e) {
+            const float a = v[c * 8 + 2 * e], b = v[c * 8 + 2 * e + 1];
+            const bf16 ha = __float2bfloat16_rn(a), hb = __float2bfloat16_rn(b);
+            const bf16 la = __float2bfloat16_rn(a - __bfloat162float(ha));
+            const bf16 lb = __float2bfloat16_rn(b - __bfloat162float(hb));
+            h4[e] = (uint32_t)__bfloat16_as_ushort(ha) | ((uint32_t)__bfloat16_as_ushort(hb) << 16);
+            l4[e] = (uint32_t)__bfloat16_as_ushort(la) | ((uint32_t)__bfloat16_as_ushort(lb) << 16);
+        }
+        const int off = r * 128 + (((cb + c) ^ (r & 7)) << 4);
+        *reinterpret_cast<uint4 *>(tile[0][blk] + off) = make_uint4(h4[0], h4[1], h4[2], h4[3]);
+        *reinterpret_cast<uint4 *>(tile[1][blk] + off) = make_uint4(l4[0], l4[1], l4[2], l4[3]);
+    }
+}
+
+// D (+)= A B over K = 128 with A a [128 x 128] pair tile (two 64-wide blocks)
+// and B a pair of 128-row tiles, three split products each.
+//   a_mn = false: A K-major, K = tile columns (P V, dS K)
+//   a_mn = true:  A read as its transpose (P^T dA, dS^T Q), K = tile rows
+__device__ __forceinline__ void mma_k128(uint32_t d, const uint8_t (*a)[2][kPBig],
+                                         const uint8_t (*b)[kPBig], bool a_mn, uint32_t idesc) {
+#pragma unroll
+    for (int t = 0; t < 3; ++t) {
+        const int ah = t == 2 ? 1 : 0, bh = t == 1 ? 1 : 0;
+#pragma unroll
+        for (int kk = 0; kk < 8; ++kk) {
+            uint64_t ad, bd;
+            if (a_mn) {
+                // rows kk*16.. of both key blocks; next 64-wide M block 16 KB on
+                ad = smem_desc_sw128(smem_u32(a[ah][0]) + kk * 2048, kPBig, 1024);
+            } else {
+                ad = smem_desc_sw128(smem_u32(a[ah][kk >> 2]) + (kk & 3) * 32, 16, 1024);
+            }
+            // B rows = K index (MN-major B: 64-wide N block, 16 rows per step)
+            bd = smem_desc_sw128(smem_u32(b[bh]) + kk * 2048, kPBig, 1024);
+            mma_bf16(d, ad, bd, idesc, (t > 0 || kk > 0) ? 1u : 0u);
+        }
+    }
+}
+
+__global__ void __launch_bounds__(kThreads, 1) attn_fwd_small_kernel(const __grid_constant__ AttnParams p) {
+    extern __shared__ uint8_t smem_raw[];
+    SmallFwdSmem &sm = *reinterpret_cast<SmallFwdSmem *>(
+        (reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    const int b = blockIdx.y, h = blockIdx.z;
+    if (threadIdx.x == 0) {
+        mbar_init(smem_u32(&sm.in_full), 1);
+        mbar_init(smem_u32(&sm.s_full), 1);
+        mbar_init(smem_u32(&sm.p_ready), 128);
+        mbar_init(smem_u32(&sm.o_full), 1);
+        sm.abort = 0;
+        fence_barrier_init();
+    }
+    if (warp == 2) {
+        tmem_alloc(smem_u32(&sm.tmem), 256);
+        tmem_relinquish();
+    }
+    tc_fence_before();
+    __syncthreads();
+    tc_fence_after();
+    const uint32_t tmem = sm.tmem, tS = tmem, tO = tmem + 128;
+
+    if (warp == 0) {
+        if (lane == 0) {
+            const uint32_t fb = smem_u32(&sm.in_full);
+            mbar_expect_tx(fb, 6 * kPBig);
+            for (int hf = 0; hf < 2; ++hf) {
+                tma_load_4d(smem_u32(sm.q[hf]), &p.mQ, fb, 64 * hf, 0, b, h);
+                tma_load_4d(smem_u32(sm.k[hf]), &p.mK, fb, 64 * hf, 0, b, h);
+                tma_load_4d(smem_u32(sm.v[hf]), &p.mV, fb, 64 * hf, 0, b, h);
+            }
+        }
+    } else if (warp == 1) {
+        if (lane == 0) {
+            constexpr uint32_t idS = idesc_bf16(128, 128, false, false);
+            constexpr uint32_t idO = idesc_bf16(128, 64, false, true);
+            bool ok = mbar_wait(smem_u32(&sm.in_full), 0);
+            if (ok) {
+                tc_fence_after();
+                // S = Q K^T: K (keys x p) is the K-major B operand, N = 128 keys
+                const uint32_t qa[3] = {smem_u32(sm.q[0]), smem_u32(sm.q[0]), smem_u32(sm.q[1])};
+                const uint32_t kb[3] = {smem_u32(sm.k[0]), smem_u32(sm.k[1]), smem_u32(sm.k[0])};
+#pragma unroll
+                for (int t = 0; t < 3; ++t)
+#pragma unroll
+                    for (int kk = 0; kk < 4; ++kk)
+                        mma_bf16(tS, smem_desc_sw128(qa[t] + kk * 32, 16, 1024),
+                                 smem_desc_sw128(kb[t] + kk * 32, 16, 1024), idS,
+                                 (t > 0 || kk > 0) ? 1u : 0u);
+                mma_commit(smem_u32(&sm.s_full));
+                ok = mbar_wait(smem_u32(&sm.p_ready), 0) && !*(volatile int *)&sm.abort;
+                if (ok) {
+                    tc_fence_after();
+                    mma_k128(tO, sm.p, sm.v, false, idO);
+                }
+            }
+            if (!ok) {
+                flag_timeout_b(sm, p.status);
+                mma_commit(smem_u32(&sm.s_full));   // release the softmax warps
+            }
+            mma_commit(smem_u32(&sm.o_full));
+        }
+    } else if (warp >= 4) {
+        const int q = warp - 4;
+        const int r = q * 32 + lane;   // query row i
+        const uint32_t lane_off = (uint32_t)(q * 32) << 16;
+        bool ok = mbar_wait(smem_u32(&sm.s_full), 0);
+        tc_fence_after();
+        float m = -INFINITY, l = 0.f;
+        // pass 1: row max
+#pragma unroll 1
+        for (int c0 = 0; c0 < kSmallK; c0 += 32) {
+            float t32[32];
+            tmem_ld32(tS + lane_off + c0, t32);
+#pragma unroll
+            for (int c = 0; c < 32; ++c)
+                if (c0 + c <= r) m = fmaxf(m, t32[c] * p.scale_log2);
+        }
+        // pass 2: probabilities into shared memory, row sum
+#pragma unroll 1
+        for (int c0 = 0; c0 < kSmallK; c0 += 32) {
+            float t32[32];
+            tmem_ld32(tS + lane_off + c0, t32);
+#pragma unroll
+            for (int c = 0; c < 32; ++c) {
+                t32[c] = (c0 + c <= r) ? exp2f(t32[c] * p.scale_log2 - m) : 0.f;
+                l += t32[c];
+            }
+            write_pair32(sm.p, r, c0, t32);
+        }
+        fence_proxy_async();
+        tc_fence_before();
+        mbar_arrive(smem_u32(&sm.p_ready));
+        ok = mbar_wait(smem_u32(&sm.o_full), 0) && ok;
+        tc_fence_after();
+        float o[64];
+        ld64(tO + lane_off, o);
+        if (!ok) flag_timeout_b(sm, p.status);
+        if (ok && r < p.k && !*(volatile int *)&sm.abort) {
+            const size_t row = (size_t)h * p.Mtok + (size_t)b * p.k + r;
+            const float inv = 1.f / l;
+            const float rr = p.rsel[row];
+            float *arow = p.A + row * 64;
+#pragma unroll
+            for (int c = 0; c < 64; c += 4)
+                *reinterpret_cast<float4 *>(arow + c) =
+                    make_float4(o[c] * inv, o[c + 1] * inv, o[c + 2] * inv, o[c + 3] * inv);
+#pragma unroll
+            for (int c = 0; c < 64; ++c) o[c] *= rr * inv;
+            store_pair64(p.AR + row * 128, 0, 64, o, 1.f);
+            p.lse[row] = (m + log2f(l)) * 0.69314718055994531f;
+        }
+    }
+    tc_fence_before();
+    __syncthreads();
+    if (warp == 2) {
+        tc_fence_after();
+        tmem_dealloc(tmem, 256);
+    }
+}
+
+__global__ void __launch_bounds__(kThreads, 1) attn_bwd_small_kernel(const __grid_constant__ BwdParams p) {
+    extern __shared__ uint8_t smem_raw[];
+    SmallBwdSmem &sm = *reinterpret_cast<SmallBwdSmem *>(
+        (reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    const int b = blockIdx.y, h = blockIdx.z;
+    if (threadIdx.x == 0) {
+        mbar_init(smem_u32(&sm.in_full), 1);
+        mbar_init(smem_u32(&sm.sp_full), 1);
+        mbar_init(smem_u32(&sm.p_ready), 128);
+        mbar_init(smem_u32(&sm.pv_done), 1);
+        mbar_init(smem_u32(&sm.ds_ready), 128);
+        mbar_init(smem_u32(&sm.acc_done), 1);
+        sm.abort = 0;
+        fence_barrier_init();
+    }
+    if (warp == 2) {
+        tmem_alloc(smem_u32(&sm.tmem), 512);
+        tmem_relinquish();
+    }
+    tc_fence_before();
+    __syncthreads();
+    tc_fence_after();
+    const uint32_t tmem = sm.tmem;
+    const uint32_t tS = tmem, tDP = tmem + 128, tDV = tmem + 256, tDK = tmem + 320, tDQ = tmem + 384;
+
+    if (warp == 0) {
+        if (lane == 0) {
+            const uint32_t fb = smem_u32(&sm.in_full);
+            mbar_expect_tx(fb, 8 * kPBig);
+            for (int hf = 0; hf < 2; ++hf) {
+                tma_load_4d(smem_u32(sm.q[hf]), &p.mA0, fb, 64 * hf, 0, b, h);
+                tma_load_4d(smem_u32(sm.k[hf]), &p.mA1, fb, 64 * hf, 0, b, h);
+                tma_load_4d(smem_u32(sm.v[hf]), &p.mB0, fb, 64 * hf, 0, b, h);
+                tma_load_4d(smem_u32(sm.da[hf]), &p.mB1, fb, 64 * hf, 0, b, h);
+            }
+        }
+    } else if (warp == 1) {
+        if (lane == 0) {
+            constexpr uint32_t idKK = idesc_bf16(128, 128, false, false);  // S, dP
+            constexpr uint32_t idMN = idesc_bf16(128, 64, true, true);     // dV, dK
+            constexpr uint32_t idKM = idesc_bf16(128, 64, false, true);    // dQ
+            bool ok = mbar_wait(smem_u32(&sm.in_full), 0);
+            if (ok) {
+                tc_fence_after();
+                const uint32_t q0 = smem_u32(sm.q[0]), q1 = smem_u32(sm.q[1]);
+                const uint32_t k0 = smem_u32(sm.k[0]), k1 = smem_u32(sm.k[1]);
+                const uint32_t v0 = smem_u32(sm.v[0]), v1 = smem_u32(sm.v[1]);
+                const uint32_t a0 = smem_u32(sm.da[0]), a1 = smem_u32(sm.da[1]);
+                mma_pair3(tS, q0, q1, k0, k1, false, false, idKK, false);   // S  = Q K^T
+                mma_pair3(tDP, a0, a1, v0, v1, false, false, idKK, false);  // dP = dA V^T
+                mma_commit(smem_u32(&sm.sp_full));
+                ok = mbar_wait(smem_u32(&sm.p_ready), 0) && !*(volatile int *)&sm.abort;
+                if (ok) {
+                    tc_fence_after();
+                    mma_k128(tDV, sm.p, sm.da, true, idMN);   // dV = P^T dA
+                    mma_commit(smem_u32(&sm.pv_done));
+                    ok = mbar_wait(smem_u32(&sm.ds_ready), 0) && !*(volatile int *)&sm.abort;
+                }
+                if (ok) {
+                    tc_fence_after();
+                    mma_k128(tDK, sm.p, sm.q, true, idMN);    // dK = dS^T Q
+                    mma_k128(tDQ, sm.p, sm.k, false, idKM);   // dQ = dS K
+                }
+            }
+            if (!ok) {
+                flag_timeout_b(sm, p.status);
+                mma_commit(smem_u32(&sm.sp_full));
+                mma_commit(smem_u32(&sm.pv_done));
+            }
+            mma_commit(smem_u32(&sm.acc_done));
+        }
+    } else if (warp >= 4) {
+        const int q = warp - 4;
+        const int r = q * 32 + lane;   // query row i for S/dP/dQ; key row j for dK/dV
+        const uint32_t lane_off = (uint32_t)(q * 32) << 16;
+        const size_t base = (size_t)h * p.Mtok + (size_t)b * p.k;
+        const bool valid = r < p.k;
+        const float l2 = valid ? p.lse[base + r] * 1.4426950408889634f : 0.f;
+        const float dd = valid ? p.Dd[base + r] : 0.f;
+        bool ok = mbar_wait(smem_u32(&sm.sp_full), 0);
+        tc_fence_after();
+        // P
+#pragma unroll 1
+        for (int c0 = 0; c0 < kSmallK; c0 += 32) {
+            float t32[32];
+            tmem_ld32(tS + lane_off + c0, t32);
+#pragma unroll
+            for (int c = 0; c < 32; ++c)
+                t32[c] = (valid && c0 + c <= r) ? exp2f(t32[c] * p.scale_log2 - l2) : 0.f;
+            write_pair32(sm.p, r, c0, t32);
+        }
+        fence_proxy_async();
+        tc_fence_before();
+        mbar_arrive(smem_u32(&sm.p_ready));
+        ok = mbar_wait(smem_u32(&sm.pv_done), 0) && ok;   // P read by dV: overwrite with dS
+        tc_fence_after();
+#pragma unroll 1
+        for (int c0 = 0; c0 < kSmallK; c0 += 32) {
+            float t32[32], d32[32];
+            tmem_ld32(tS + lane_off + c0, t32);
+            tmem_ld32(tDP + lane_off + c0, d32);
+#pragma unroll
+            for (int c = 0; c < 32; ++c) {
+                const float pr = (valid && c0 + c <= r) ? exp2f(t32[c] * p.scale_log2 - l2) : 0.f;
+                t32[c] = pr * (d32[c] - dd);
+            }
+            write_pair32(sm.p, r, c0, t32);
+        }
+        fence_proxy_async();
+        tc_fence_before();
+        mbar_arrive(smem_u32(&sm.ds_ready));
+        ok = mbar_wait(smem_u32(&sm.acc_done), 0) && ok;
+        tc_fence_after();
+        float dv[64], dk[64], dq[64];
+        ld64(tDV + lane_off, dv);
+        ld64(tDK + lane_off, dk);
+        ld64(tDQ + lane_off, dq);
+        if (!ok) flag_timeout_b(sm, p.status);
+        if (ok && valid && !*(volatile int *)&sm.abort) {
+            bf16 *row = p.dQKV + (base + r) * 512;
+            store_pair64(row, 0, 256, dq, p.scale);
+            store_pair64(row, 64, 320, dk, p.scale);
+            store_pair64(row, 128, 384, dv, 1.f);
+        }
+    }
+    tc_fence_before();
+    __syncthreads();
+    if (warp == 2) {
+        tc_fence_after();
+        tmem_dealloc(tmem, 512);
+    }
+}
+
 // [H, B, k, 128] bf16 pair array (row = 64 hi + 64 lo), box {64, rows, 1, 1}:
 // rows past k of one sequence read as zeros.
 bool map_units(CUtensorMap *m, const void *base, int H, int B, int k, uint32_t rows) {
@@ -747,9 +1082,10 @@ bool map_units(CUtensorMap *m, const void *base, int H, int B, int k, uint32_t r
 cudaError_t tc_attn_fwd(const Dims &dm, const Saved &sv, cudaStream_t s) {
     AttnParams p;
     memset(&p, 0, sizeof(p));
+    const bool small = dm.k <= kSmallK;
     bool ok = map_units(&p.mQ, sv.Q, dm.H, dm.B, dm.k, kQ) &&
-              map_units(&p.mK, sv.K, dm.H, dm.B, dm.k, kKV) &&
-              map_units(&p.mV, sv.V, dm.H, dm.B, dm.k, kKV);
+              map_units(&p.mK, sv.K, dm.H, dm.B, dm.k, small ? 128 : kKV) &&
+              map_units(&p.mV, sv.V, dm.H, dm.B, dm.k, small ? 128 : kKV);
     if (!ok) return cudaErrorInvalidValue;
     p.k = dm.k;
     p.B = dm.B;
@@ -765,8 +1101,16 @@ cudaError_t tc_attn_fwd(const Dims &dm, const Saved &sv, cudaStream_t s) {
     std::call_once(once, [] {
         attr = cudaFuncSetAttribute(attn_fwd_tc_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                     kFwdSmem);
+        if (attr == cudaSuccess)
+            attr = cudaFuncSetAttribute(attn_fwd_small_kernel,
+                                        cudaFuncAttributeMaxDynamicSharedMemorySize, kSmallFwdSmem);
     });
     if (attr != cudaSuccess) return attr;
+    if (small) {
+        attn_fwd_small_kernel<<<dim3(1, dm.B, dm.H), kThreads, kSmallFwdSmem, s>>>(p);
+        note_launches(1);
+        return cudaGetLastError();
+    }
     dim3 grid((dm.k + kQ - 1) / kQ, dm.B, dm.H);
     attn_fwd_tc_kernel<<<grid, kThreads, kFwdSmem, s>>>(p);
     note_launches(1);
@@ -777,6 +1121,34 @@ cudaError_t tc_attn_bwd(const Dims &dm, const Saved &sv, cudaStream_t s) {
     BwdParams kv, dq;
     memset(&kv, 0, sizeof(kv));
     memset(&dq, 0, sizeof(dq));
+    if (dm.k <= kSmallK) {
+        BwdParams sp;
+        memset(&sp, 0, sizeof(sp));
+        const bool ok = map_units(&sp.mA0, sv.Q, dm.H, dm.B, dm.k, 128) &&
+                        map_units(&sp.mA1, sv.K, dm.H, dm.B, dm.k, 128) &&
+                        map_units(&sp.mB0, sv.V, dm.H, dm.B, dm.k, 128) &&
+                        map_units(&sp.mB1, sv.dA, dm.H, dm.B, dm.k, 128);
+        if (!ok) return cudaErrorInvalidValue;
+        sp.k = dm.k;
+        sp.Mtok = dm.B * dm.k;
+        sp.scale = 1.f / sqrtf(64.f);
+        sp.scale_log2 = 1.4426950408889634f / sqrtf(64.f);
+        sp.lse = sv.lse;
+        sp.Dd = sv.Dd;
+        sp.dQKV = static_cast<bf16 *>(sv.dQKV);
+        sp.status = sv.status;
+        static std::once_flag once_small;
+        static cudaError_t attr_small = cudaSuccess;
+        std::call_once(once_small, [] {
+            attr_small = cudaFuncSetAttribute(attn_bwd_small_kernel,
+                                              cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                              kSmallBwdSmem);
+        });
+        if (attr_small != cudaSuccess) return attr_small;
+        attn_bwd_small_kernel<<<dim3(1, dm.B, dm.H), kThreads, kSmallBwdSmem, s>>>(sp);
+        note_launches(1);
+        return cudaGetLastError();
+    }
     bool ok = map_units(&kv.mA0, sv.K, dm.H, dm.B, dm.k, kKT) &&
               map_units(&kv.mA1, sv.V, dm.H, dm.B, dm.k, kKT) &&
               map_units(&kv.mB0, sv.Q, dm.H, dm.B, dm.k, kQB) &&

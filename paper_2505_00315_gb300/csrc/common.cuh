@@ -91,6 +91,7 @@ struct Saved {
     void *dQKV;         // [H,B*k,3hp] dQ | dK | dV, intermediate (tensor-core path:
                         // [H,B*k,512] bf16 pair dQ|dK|dV|dlogit,0.. hi then lo)
     float *G;           // [H,B*k,hp] dY[I] W_o^T (fp32)
+    float *WrT;         // [H,d] fp32 transpose of W_r (tensor-core backward)
 };
 
 struct Dims {

@@ -3,9 +3,34 @@
 // returns the launch status; none synchronizes.
 #pragma once
 
+#include <utility>
+
 #include "common.cuh"
 
+#include <cstdlib>
+
 namespace mosa {
+
+// Launches `kernel` with programmatic stream serialization (it may begin while
+// the preceding kernel on the stream finishes; the kernel itself waits with
+// griddepcontrol.wait before reading that kernel's results).  MOSA_PDL=0
+// launches it plainly.
+template <class... KArgs, class... Args>
+inline cudaError_t launch_pdl(void (*kernel)(KArgs...), dim3 grid, dim3 block, size_t smem,
+                              cudaStream_t s, Args &&...args) {
+    const char *v = std::getenv("MOSA_PDL");
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = grid;
+    cfg.blockDim = block;
+    cfg.dynamicSmemBytes = smem;
+    cfg.stream = s;
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    attr[0].val.programmaticStreamSerializationAllowed = 1;
+    cfg.attrs = attr;
+    cfg.numAttrs = (v != nullptr && v[0] == '0') ? 0 : 1;
+    return cudaLaunchKernelEx(&cfg, kernel, std::forward<Args>(args)...);
+}
 
 // F1, Sec. 2.2 router: r_full[b,h,t] = sigmoid(X[b,t,:] . W_r[:,h]) in fp32.
 cudaError_t launch_router(const Dims &dm, const void *X, const void *Wr, float *r_full,
@@ -68,6 +93,8 @@ cudaError_t tc_out_bwd_g(const Dims &dm, const void *Wo, const void *dY, const S
                          cudaStream_t s);
 cudaError_t tc_out_bwd_w(const Dims &dm, const void *dY, const Saved &sv, float *dWo,
                          cudaStream_t s);
+// W_r [d,H] bf16 -> sv.WrT [H,d] fp32 (read by the dX epilogue).
+cudaError_t tc_transpose_wr(const Dims &dm, const void *Wr, const Saved &sv, cudaStream_t s);
 cudaError_t tc_in_bwd(const Dims &dm, const void *Wq, const void *Wk, const void *Wv,
                       const void *Wr, const Saved &sv, float *dX, cudaStream_t s,
                       bool zero_output);

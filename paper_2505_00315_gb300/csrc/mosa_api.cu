@@ -63,6 +63,7 @@ size_t carve(const Dims &dm, char *base, Saved *sv) {
     s.Dd = (float *)take(sizeof(float) * R);
     s.dQKV = take(e * R * 4 * dm.hp);  // 3 h' columns, or 4 blocks of 64 on the tensor cores
     s.G = (float *)take(sizeof(float) * R * dm.hp);
+    s.WrT = (float *)take(sizeof(float) * (size_t)dm.d * dm.H);
     if (sv) *sv = s;
     return off;
 }
@@ -180,12 +181,13 @@ mosa_status backward_tc(const Dims &dm, const void *X, const void *W_r, const vo
                         float *dW_o, const Saved &sv, cudaStream_t s, DevResources &r) {
     cudaStream_t t = r.side;
     MOSA_TRY(link(s, t, r.ev[0]));
+    MOSA_TRY(tc_transpose_wr(dm, W_r, sv, t));
+    MOSA_TRY(cudaMemsetAsync(dX, 0, sizeof(float) * (size_t)dm.B * dm.T * dm.d, t));
+    MOSA_TRY(link(t, s, r.ev[1]));  // dX zeroed and W_r transposed before the dX product
     {
         StageScope st_(kStageDwo, t);
         MOSA_TRY(tc_out_bwd_w(dm, dY, sv, dW_o, t));
     }
-    MOSA_TRY(cudaMemsetAsync(dX, 0, sizeof(float) * (size_t)dm.B * dm.T * dm.d, t));
-    MOSA_TRY(link(t, s, r.ev[1]));  // dX zeroed before the scatter into it
     {
         StageScope st_(kStageOutBwd, s);
         MOSA_TRY(tc_out_bwd_g(dm, W_o, dY, sv, s));

@@ -72,6 +72,7 @@ topk_select_kernel(const float *__restrict__ scores, int T, int k, int32_t *__re
     __shared__ uint32_t hist[256];
     __shared__ uint32_t sh[33];
     __shared__ uint32_t sh_prefix, sh_remaining;
+    asm volatile("griddepcontrol.wait;" ::: "memory");  // scores from the router kernel
     const int row = blockIdx.x;
     const float *s = scores + (size_t)row * T;
     const int tid = threadIdx.x;
@@ -162,6 +163,7 @@ __global__ void indices_to_rows_kernel(const int32_t *__restrict__ I,
                                        const float *__restrict__ rsel, int B, int H, int T,
                                        int k, int32_t *__restrict__ gidx,
                                        float *__restrict__ rsel_hm, uint32_t *status) {
+    asm volatile("griddepcontrol.wait;" ::: "memory");
     const int row = blockIdx.x;  // b*H + h
     const int hh = row % H, bb = row / H;
     const int32_t *Ir = I + (size_t)row * k;
@@ -204,10 +206,10 @@ cudaError_t launch_router_auto(const Dims &dm, const void *X, const void *Wr, fl
 cudaError_t launch_select(int rows, int T, int k, const float *scores, int32_t *I, float *rsel,
                           int B, int H, int32_t *gidx, float *rsel_hm, cudaStream_t stream) {
     if (rows <= 0) return cudaSuccess;
-    topk_select_kernel<<<rows, kSelThreads, 0, stream>>>(scores, T, k, I, rsel, B, H, gidx,
-                                                        rsel_hm);
+    cudaError_t e = launch_pdl(topk_select_kernel, dim3(rows), dim3(kSelThreads), 0, stream,
+                               scores, T, k, I, rsel, B, H, gidx, rsel_hm);
     note_launches(1);
-    return cudaGetLastError();
+    return e;
 }
 
 cudaError_t launch_indices_to_rows(const Dims &dm, const int32_t *I, const float *rsel,

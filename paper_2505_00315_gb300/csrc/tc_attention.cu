@@ -122,6 +122,7 @@ __global__ void __launch_bounds__(kThreads, 1) attn_fwd_tc_kernel(const __grid_c
     tc_fence_before();
     __syncthreads();
     tc_fence_after();
+    pdl_wait();  // Q, K, V, dA, lse written by the previous kernels
     const uint32_t tmem = sm.tmem;
     const uint32_t tS = tmem, tO = tmem + 64;
 
@@ -220,6 +221,7 @@ __global__ void __launch_bounds__(kThreads, 1) attn_fwd_tc_kernel(const __grid_c
         }
     } else if (warp >= 4) {
         // ---------------------------------------------------------- softmax
+        pdl_trigger();
         const int q = warp - 4;
         const int r = q * 32 + lane;
         const int i = i0 + r;
@@ -460,6 +462,7 @@ __global__ void __launch_bounds__(kThreads, 1) attn_dkv_tc_kernel(const __grid_c
     tc_fence_before();
     __syncthreads();
     tc_fence_after();
+    pdl_wait();  // Q, K, V, dA, lse written by the previous kernels
     const uint32_t tmem = sm.tmem;
     const uint32_t tST = tmem, tDPT = tmem + 64, tDV = tmem + 128, tDK = tmem + 192;
 
@@ -529,6 +532,7 @@ __global__ void __launch_bounds__(kThreads, 1) attn_dkv_tc_kernel(const __grid_c
             mma_commit(smem_u32(&sm.acc_done));
         }
     } else if (warp >= 4) {
+        pdl_trigger();
         const int q = warp - 4;
         const int r = q * 32 + lane;
         const int j = j0 + r;
@@ -615,6 +619,7 @@ __global__ void __launch_bounds__(kThreads, 1) attn_dq_tc_kernel(const __grid_co
     tc_fence_before();
     __syncthreads();
     tc_fence_after();
+    pdl_wait();  // Q, K, V, dA, lse written by the previous kernels
     const uint32_t tmem = sm.tmem;
     const uint32_t tS = tmem, tDP = tmem + 64, tDQ = tmem + 128;
 
@@ -682,6 +687,7 @@ __global__ void __launch_bounds__(kThreads, 1) attn_dq_tc_kernel(const __grid_co
             mma_commit(smem_u32(&sm.acc_done));
         }
     } else if (warp >= 4) {
+        pdl_trigger();
         const int q = warp - 4;
         const int r = q * 32 + lane;
         const int i = i0 + r;
@@ -833,6 +839,7 @@ __global__ void __launch_bounds__(kThreads, 1) attn_fwd_small_kernel(const __gri
     tc_fence_before();
     __syncthreads();
     tc_fence_after();
+    pdl_wait();  // Q, K, V, dA, lse written by the previous kernels
     const uint32_t tmem = sm.tmem, tS = tmem, tO = tmem + 128;
 
     if (warp == 0) {
@@ -876,6 +883,7 @@ __global__ void __launch_bounds__(kThreads, 1) attn_fwd_small_kernel(const __gri
             mma_commit(smem_u32(&sm.o_full));
         }
     } else if (warp >= 4) {
+        pdl_trigger();
         const int q = warp - 4;
         const int r = q * 32 + lane;   // query row i
         const uint32_t lane_off = (uint32_t)(q * 32) << 16;
@@ -957,6 +965,7 @@ __global__ void __launch_bounds__(kThreads, 1) attn_bwd_small_kernel(const __gri
     tc_fence_before();
     __syncthreads();
     tc_fence_after();
+    pdl_wait();  // Q, K, V, dA, lse written by the previous kernels
     const uint32_t tmem = sm.tmem;
     const uint32_t tS = tmem, tDP = tmem + 128, tDV = tmem + 256, tDK = tmem + 320, tDQ = tmem + 384;
 
@@ -1007,6 +1016,7 @@ __global__ void __launch_bounds__(kThreads, 1) attn_bwd_small_kernel(const __gri
             mma_commit(smem_u32(&sm.acc_done));
         }
     } else if (warp >= 4) {
+        pdl_trigger();
         const int q = warp - 4;
         const int r = q * 32 + lane;   // query row i for S/dP/dQ; key row j for dK/dV
         const uint32_t lane_off = (uint32_t)(q * 32) << 16;
@@ -1107,14 +1117,15 @@ cudaError_t tc_attn_fwd(const Dims &dm, const Saved &sv, cudaStream_t s) {
     });
     if (attr != cudaSuccess) return attr;
     if (small) {
-        attn_fwd_small_kernel<<<dim3(1, dm.B, dm.H), kThreads, kSmallFwdSmem, s>>>(p);
+        cudaError_t e = launch_pdl(attn_fwd_small_kernel, dim3(1, dm.B, dm.H), dim3(kThreads),
+                                   kSmallFwdSmem, s, p);
         note_launches(1);
-        return cudaGetLastError();
+        return e;
     }
     dim3 grid((dm.k + kQ - 1) / kQ, dm.B, dm.H);
-    attn_fwd_tc_kernel<<<grid, kThreads, kFwdSmem, s>>>(p);
+    cudaError_t e = launch_pdl(attn_fwd_tc_kernel, grid, dim3(kThreads), kFwdSmem, s, p);
     note_launches(1);
-    return cudaGetLastError();
+    return e;
 }
 
 cudaError_t tc_attn_bwd(const Dims &dm, const Saved &sv, cudaStream_t s) {
@@ -1145,9 +1156,10 @@ cudaError_t tc_attn_bwd(const Dims &dm, const Saved &sv, cudaStream_t s) {
                                               kSmallBwdSmem);
         });
         if (attr_small != cudaSuccess) return attr_small;
-        attn_bwd_small_kernel<<<dim3(1, dm.B, dm.H), kThreads, kSmallBwdSmem, s>>>(sp);
+        cudaError_t e = launch_pdl(attn_bwd_small_kernel, dim3(1, dm.B, dm.H), dim3(kThreads),
+                                   kSmallBwdSmem, s, sp);
         note_launches(1);
-        return cudaGetLastError();
+        return e;
     }
     bool ok = map_units(&kv.mA0, sv.K, dm.H, dm.B, dm.k, kKT) &&
               map_units(&kv.mA1, sv.V, dm.H, dm.B, dm.k, kKT) &&
@@ -1179,11 +1191,11 @@ cudaError_t tc_attn_bwd(const Dims &dm, const Saved &sv, cudaStream_t s) {
     });
     if (attr != cudaSuccess) return attr;
     dim3 gkv((dm.k + kKT - 1) / kKT, dm.B, dm.H);
-    attn_dkv_tc_kernel<<<gkv, kThreads, kDkvSmem, s>>>(kv);
+    cudaError_t e = launch_pdl(attn_dkv_tc_kernel, gkv, dim3(kThreads), kDkvSmem, s, kv);
     dim3 gq((dm.k + kQ - 1) / kQ, dm.B, dm.H);
-    attn_dq_tc_kernel<<<gq, kThreads, kDqSmem, s>>>(dq);
+    if (e == cudaSuccess) e = launch_pdl(attn_dq_tc_kernel, gq, dim3(kThreads), kDqSmem, s, dq);
     note_launches(2);
-    return cudaGetLastError();
+    return e;
 }
 
 }  // namespace mosa

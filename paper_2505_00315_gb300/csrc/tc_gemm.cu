@@ -21,6 +21,7 @@
 //   kG    B1  G(m,:)        = dY[g(m),:] W_o[h]^T, then dr, dA = r G, D, dlogit in the epilogue
 //   kDWO  B1  dW_o[h](p,c)  = sum_m AR(m,p) dY[g(m),c]       A gathered MN-major, B = AR pair
 //   kDX   B3  dX[g(m),n]   += dQKV(m,:) [W_q|W_k|W_v][h]^T(:,n) + dlogit(m) W_r[n,h]
+//             (W_r read from its fp32 transpose [H, d], one float4 per lane)
 //   kDW   B4  [dW_q|dW_k|dW_v|dW_r][h](c,:) = sum_m X[g(m),c] [dQ|dK|dV|dlogit](m,:)
 //             A gathered MN-major, B = the dQKV pair (its 4th 64-column block holds
 //             dlogit in column 0 and zeros), so dW_r comes out of the same product
@@ -75,7 +76,10 @@ struct Cfg<kDWO> {
 };
 template <>
 struct Cfg<kDX> {
-    static constexpr int BN = 256, STAGES = 3, A_BYTES = 2 * kTile16K, B_BYTES = 32768,
+    // one stage: 80 KB of shared memory lets two CTAs share an SM, so one CTA's
+    // scatter-add epilogue overlaps the other's loads (measured faster than a
+    // three-stage ring at one CTA per SM)
+    static constexpr int BN = 256, STAGES = 1, A_BYTES = 2 * kTile16K, B_BYTES = 32768,
                          TMEM_COLS = 256;
     static constexpr bool A_MN = false, B_MN = false, A_PAIR = true, B_PAIR = false;
 };
@@ -129,7 +133,7 @@ struct TcParams {
     const float *rsel;     // [H, B*k]
     const float *A32;      // [H, B*k, 64] attention output (kG)
     const float *dlogit;   // [H, B*k] (kDX reads, kG writes via out_f1)
-    const bf16 *Wr;        // [d, H] (kDX)
+    const float *WrT;      // [H, d] fp32 transpose of W_r (kDX)
     const void *src_rows;  // gathered source [B*T, d] bf16: X (kQKV, kDW) or dY (kG, kDWO)
     void *out[3];          // Q/K/V pairs (kQKV); dA pair, dQKV pair (kG)
     float *out_f;          // Y (kOUT), dW_o (kDWO), dX (kDX), dW_q (kDW)
@@ -267,6 +271,7 @@ __global__ void __launch_bounds__(kThreads, 1) tc_gemm_kernel(const __grid_const
         *s_abort = 0;
         fence_barrier_init();
     }
+    pdl_wait();  // everything below may read what the previous kernel wrote
     if (KIND == kQKV || KIND == kG || scatters<KIND>()) {
         for (int r = threadIdx.x; r < kBM; r += kThreads) {
             const int m = m0 + r;
@@ -372,6 +377,7 @@ __global__ void __launch_bounds__(kThreads, 1) tc_gemm_kernel(const __grid_const
         const int mg = m0 + r;
         const bool ok = mbar_wait(smem_u32(done), 0);
         tc_fence_after();
+        pdl_trigger();  // main loop done: the next kernel may start its prologue
         const bool abort = !ok || *(volatile int *)s_abort || nkb <= 0;
         if (!ok && lane == 0) atomicOr(p.status, kStatusTimeout);
         const uint32_t tb = tmem + ((uint32_t)(q * 32) << 16);
@@ -401,11 +407,10 @@ __global__ void __launch_bounds__(kThreads, 1) tc_gemm_kernel(const __grid_const
                         make_float4(v[4 * c], v[4 * c + 1], v[4 * c + 2], v[4 * c + 3]);
                 __syncwarp();
                 const int n = n0 + c0 + 4 * chunk;
-                float w[4] = {0.f, 0.f, 0.f, 0.f};
-                if (KIND == kDX && n < p.d) {
-#pragma unroll
-                    for (int u = 0; u < 4; ++u) w[u] = __bfloat162float(p.Wr[(size_t)(n + u) * p.H + h]);
-                }
+                float4 w4 = make_float4(0.f, 0.f, 0.f, 0.f);
+                if (KIND == kDX && n < p.d)
+                    w4 = *reinterpret_cast<const float4 *>(p.WrT + (size_t)h * p.d + n);
+                const float w[4] = {w4.x, w4.y, w4.z, w4.w};
 #pragma unroll
                 for (int i = 0; i < 8; ++i) {
                     const int rl = (lane >> 3) + 4 * i;
@@ -576,9 +581,9 @@ cudaError_t launch_kind(const TcParams &p, dim3 grid, cudaStream_t s) {
                                     smem);
     });
     if (attr != cudaSuccess) return attr;
-    tc_gemm_kernel<KIND><<<grid, kThreads, smem, s>>>(p);
+    cudaError_t e = launch_pdl(tc_gemm_kernel<KIND>, grid, dim3(kThreads), smem, s, p);
     note_launches(1);
-    return cudaGetLastError();
+    return e;
 }
 
 int splits_for(int tiles, int nkb) {
@@ -628,6 +633,24 @@ bool tc_router(const Dims &dm, const void *X, const void *Wr, float *r_full, uin
     dim3 grid((p.M + kBM - 1) / kBM, (dm.H + 127) / 128, 1);
     *err = launch_kind<kROUTER>(p, grid, s);
     return true;
+}
+
+__global__ void transpose_wr_kernel(const bf16 *__restrict__ Wr, float *__restrict__ WrT, int d,
+                                    int H) {
+    pdl_wait();
+    const int i = blockIdx.x * blockDim.x + threadIdx.x;  // element of WrT [H, d]
+    if (i < d * H) {
+        const int h = i / d, c = i - h * d;
+        WrT[i] = __bfloat162float(Wr[(size_t)c * H + h]);
+    }
+}
+
+cudaError_t tc_transpose_wr(const Dims &dm, const void *Wr, const Saved &sv, cudaStream_t s) {
+    const int n = dm.d * dm.H;
+    transpose_wr_kernel<<<(n + 255) / 256, 256, 0, s>>>(static_cast<const bf16 *>(Wr), sv.WrT,
+                                                        dm.d, dm.H);
+    note_launches(1);
+    return cudaGetLastError();
 }
 
 bool tc_supported(const Dims &dm) {
@@ -724,8 +747,9 @@ cudaError_t tc_in_bwd(const Dims &dm, const void *Wq, const void *Wk, const void
     bool ok = map_heads(&p.mapA, sv.dQKV, dm.H, p.Mtok, kDQKVCols, 128);
     for (int j = 0; j < 3; ++j) ok = ok && map_heads(&p.mapB[j], W[j], dm.H, dm.d, 64, 256);
     if (!ok) return cudaErrorInvalidValue;
+    (void)Wr;
     p.dlogit = sv.dlogit;
-    p.Wr = static_cast<const bf16 *>(Wr);
+    p.WrT = sv.WrT;
     p.out_f = dX;
     dim3 grid((p.M + kBM - 1) / kBM, (dm.d + 255) / 256, dm.H);
     return launch_kind<kDX>(p, grid, s);

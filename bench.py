@@ -54,6 +54,9 @@ def parse_args():
     p.add_argument("--config", default=None)
     p.add_argument("--no-cpu-baseline", action="store_true")
     p.add_argument("--cpu-budget-s", type=float, default=15.0)
+    p.add_argument("--ingest-ncu", metavar="CSV", default=None,
+                   help="turn an ncu CSV with dram__bytes_read/write.sum per kernel (taken on "
+                        "this command's workload) into profiles/traffic.json and exit")
     return p.parse_args()
 
 
@@ -200,6 +203,50 @@ def traffic_for(stage, cfg_name):
     return ent.get("bytes_per_launch")
 
 
+# Kernel name (as ncu prints it) -> bench stage.
+KERNEL_STAGE = [("tc_gemm_kernel<6>", "router"), ("tc_gemm_kernel<(int)6>", "router"),
+                ("topk_select", "select"), ("tc_gemm_kernel<0>", "qkv"),
+                ("tc_gemm_kernel<(int)0>", "qkv"), ("attn_fwd", "attn_fwd"),
+                ("tc_gemm_kernel<1>", "out"), ("tc_gemm_kernel<(int)1>", "out"),
+                ("tc_gemm_kernel<2>", "out_bwd"), ("tc_gemm_kernel<(int)2>", "out_bwd"),
+                ("attn_bwd", "attn_bwd"), ("attn_dkv", "attn_bwd"), ("attn_dq", "attn_bwd"),
+                ("tc_gemm_kernel<4>", "in_bwd"), ("tc_gemm_kernel<(int)4>", "in_bwd"),
+                ("tc_gemm_kernel<5>", "w_bwd"), ("tc_gemm_kernel<(int)5>", "w_bwd"),
+                ("tc_gemm_kernel<3>", "dwo"), ("tc_gemm_kernel<(int)3>", "dwo")]
+
+
+def ingest_ncu(csv_path, cfg_name):
+    """Average DRAM bytes per step of each stage from an ncu CSV (one row per
+    kernel launch and metric) into profiles/traffic.json."""
+    import csv
+    import collections
+    per = collections.defaultdict(lambda: collections.defaultdict(float))
+    with open(csv_path) as f:
+        lines = [l for l in f if not l.startswith("==")]
+    for row in csv.DictReader(lines):
+        name, metric = row.get("Kernel Name", ""), row.get("Metric Name", "")
+        if metric not in ("dram__bytes_read.sum", "dram__bytes_write.sum"):
+            continue
+        stage = next((st for key, st in KERNEL_STAGE if key in name), None)
+        if stage is None:
+            continue
+        unit = row.get("Metric Unit", "byte")
+        scale = {"byte": 1, "Kbyte": 1e3, "Mbyte": 1e6, "Gbyte": 1e9, "KB": 1e3, "MB": 1e6}.get(unit, 1)
+        per[stage][row["ID"]] += float(row["Metric Value"].replace(",", "")) * scale
+    path = os.path.join(ROOT, "profiles", "traffic.json")
+    data = json.load(open(path)) if os.path.exists(path) else {}
+    digest = source_digest()
+    ent = {}
+    for stage, launches in per.items():
+        vals = list(launches.values())
+        ent[stage] = {"bytes_per_launch": sum(vals) / len(vals), "launches": len(vals),
+                      "source_sha256": digest}
+    data[cfg_name] = ent
+    with open(path, "w") as f:
+        json.dump(data, f, indent=1, sort_keys=True)
+    print(json.dumps({k: round(v["bytes_per_launch"] / 1e6, 3) for k, v in ent.items()}))
+
+
 def source_digest():
     import glob
     h = hashlib.sha256()
@@ -271,6 +318,10 @@ def main():
     rank = int(os.environ.get("RANK", "0"))
     local = int(os.environ.get("LOCAL_RANK", "0"))
     cfg = W.CONFIGS[args.config or W.BENCH_CONFIG]
+
+    if args.ingest_ncu:
+        ingest_ncu(args.ingest_ncu, cfg.name)
+        return
 
     if args.impl == "reference":
         run_reference(args, cfg, rank, world)

@@ -53,25 +53,25 @@ struct Cfg;
 template <>
 struct Cfg<kQKV> {
     static constexpr int BN = 192, STAGES = 2, A_BYTES = kTile16K, B_BYTES = 3 * kTile8K,
-                         TMEM_COLS = 256;
+                         TMEM_COLS = 256, MIN_CTAS = 2;
     static constexpr bool A_MN = false, B_MN = true, A_PAIR = false, B_PAIR = false;
 };
 template <>
 struct Cfg<kOUT> {
     static constexpr int BN = 256, STAGES = 1, A_BYTES = 2 * kTile16K, B_BYTES = 4 * kTile8K,
-                         TMEM_COLS = 256;
+                         TMEM_COLS = 256, MIN_CTAS = 2;
     static constexpr bool A_MN = false, B_MN = true, A_PAIR = true, B_PAIR = false;
 };
 template <>
 struct Cfg<kG> {
     static constexpr int BN = 64, STAGES = 4, A_BYTES = kTile16K, B_BYTES = kTile8K,
-                         TMEM_COLS = 64;
+                         TMEM_COLS = 64, MIN_CTAS = 2;
     static constexpr bool A_MN = false, B_MN = false, A_PAIR = false, B_PAIR = false;
 };
 template <>
 struct Cfg<kDWO> {
     static constexpr int BN = 64, STAGES = 3, A_BYTES = kTile16K, B_BYTES = 2 * kTile8K,
-                         TMEM_COLS = 64;
+                         TMEM_COLS = 64, MIN_CTAS = 2;
     static constexpr bool A_MN = true, B_MN = true, A_PAIR = false, B_PAIR = true;
 };
 template <>
@@ -80,20 +80,20 @@ struct Cfg<kDX> {
     // scatter-add epilogue overlaps the other's loads (measured faster than a
     // three-stage ring at one CTA per SM)
     static constexpr int BN = 256, STAGES = 1, A_BYTES = 2 * kTile16K, B_BYTES = 32768,
-                         TMEM_COLS = 256;
+                         TMEM_COLS = 256, MIN_CTAS = 2;
     static constexpr bool A_MN = false, B_MN = false, A_PAIR = true, B_PAIR = false;
 };
 template <>
 struct Cfg<kDW> {
     static constexpr int BN = 256, STAGES = 2, A_BYTES = kTile16K, B_BYTES = 8 * kTile8K,
-                         TMEM_COLS = 256;
+                         TMEM_COLS = 256, MIN_CTAS = 1;
     static constexpr bool A_MN = true, B_MN = true, A_PAIR = false, B_PAIR = true;
 };
 
 template <>
 struct Cfg<kROUTER> {
-    static constexpr int BN = 128, STAGES = 3, A_BYTES = kTile16K, B_BYTES = 2 * kTile8K,
-                         TMEM_COLS = 128;
+    static constexpr int BN = 128, STAGES = 6, A_BYTES = kTile16K, B_BYTES = 2 * kTile8K,
+                         TMEM_COLS = 128, MIN_CTAS = 1;
     static constexpr bool A_MN = false, B_MN = true, A_PAIR = false, B_PAIR = false;
 };
 
@@ -113,11 +113,16 @@ __host__ __device__ constexpr bool gathers() {
     return KIND == kQKV || KIND == kG || KIND == kDWO || KIND == kDW;
 }
 
+// Kinds whose epilogue runs on all eight warps (wide output tiles).
+template <int KIND>
+__host__ __device__ constexpr bool epi_all_warps() {
+    return KIND == kQKV || KIND == kOUT || KIND == kDX || KIND == kDW || KIND == kDWO;
+}
+
 template <int KIND>
 constexpr int smem_bytes() {
     return 1024 /* alignment slack */ + Cfg<KIND>::STAGES * (Cfg<KIND>::A_BYTES + Cfg<KIND>::B_BYTES) +
-           2048 /* barriers, row indices, row scalars */ +
-           (scatters<KIND>() ? 4 * 32 * 128 : 0) /* per-warp transpose buffers */;
+           2048 /* barriers, row indices, row scalars */;
 }
 
 struct TcParams {
@@ -143,23 +148,80 @@ struct TcParams {
     uint32_t *status;
 };
 
-__device__ __forceinline__ void store_pair_row32(bf16 *row_hi, bf16 *row_lo, const float (&v)[32]) {
-    // v -> hi = bf16(v), lo = bf16(v - hi); 32 values each, four 16-byte stores per half
+// Epilogue staging: each warp owns kXpose bytes at the start of the operand
+// ring (free once the last MMA has completed).
+constexpr int kXpose = 8192;
+
+// Byte offset of 16-byte unit u (0..15) of row rl (0..31) in a warp's 32 x 256-byte
+// staging buffer.  The XOR keeps both the row-per-lane writes and the
+// unit-per-lane reads free of shared-memory bank conflicts.
+__device__ __forceinline__ uint32_t xoff256(int rl, int u) {
+    return (uint32_t)(rl * 256 + ((u ^ (rl & 15)) << 4));
+}
+
+__device__ __forceinline__ uint32_t pack_bf16x2(bf16 a, bf16 b) {
+    return (uint32_t)__bfloat16_as_ushort(a) | ((uint32_t)__bfloat16_as_ushort(b) << 16);
+}
+
+// Values v[8u .. 8u+7] of this lane's row as hi unit u and lo unit 8 + u.
+__device__ __forceinline__ void stage_pair_unit(uint8_t *xb, int lane, int u, const float *v) {
+    uint32_t h4[4], l4[4];
 #pragma unroll
-    for (int q = 0; q < 4; ++q) {
-        uint32_t h4[4], l4[4];
-#pragma unroll
-        for (int e = 0; e < 4; ++e) {
-            const float a = v[q * 8 + 2 * e], b = v[q * 8 + 2 * e + 1];
-            const bf16 ha = __float2bfloat16_rn(a), hb = __float2bfloat16_rn(b);
-            const bf16 la = __float2bfloat16_rn(a - __bfloat162float(ha));
-            const bf16 lb = __float2bfloat16_rn(b - __bfloat162float(hb));
-            h4[e] = (uint32_t)__bfloat16_as_ushort(ha) | ((uint32_t)__bfloat16_as_ushort(hb) << 16);
-            l4[e] = (uint32_t)__bfloat16_as_ushort(la) | ((uint32_t)__bfloat16_as_ushort(lb) << 16);
-        }
-        reinterpret_cast<uint4 *>(row_hi)[q] = make_uint4(h4[0], h4[1], h4[2], h4[3]);
-        reinterpret_cast<uint4 *>(row_lo)[q] = make_uint4(l4[0], l4[1], l4[2], l4[3]);
+    for (int e = 0; e < 4; ++e) {
+        const float a = v[2 * e], b = v[2 * e + 1];
+        const bf16 ha = __float2bfloat16_rn(a), hb = __float2bfloat16_rn(b);
+        h4[e] = pack_bf16x2(ha, hb);
+        l4[e] = pack_bf16x2(__float2bfloat16_rn(a - __bfloat162float(ha)),
+                            __float2bfloat16_rn(b - __bfloat162float(hb)));
     }
+    *reinterpret_cast<uint4 *>(xb + xoff256(lane, u)) = make_uint4(h4[0], h4[1], h4[2], h4[3]);
+    *reinterpret_cast<uint4 *>(xb + xoff256(lane, 8 + u)) = make_uint4(l4[0], l4[1], l4[2], l4[3]);
+}
+
+// This lane's 64 values as one bf16 pair row [hi 0..63 | lo 0..63] of the staging buffer.
+__device__ __forceinline__ void stage_pair_vals64(uint8_t *xb, const float (&v)[64], int lane) {
+#pragma unroll
+    for (int u = 0; u < 8; ++u) stage_pair_unit(xb, lane, u, v + 8 * u);
+    __syncwarp();
+}
+
+// TMEM columns taddr .. taddr+63 of this lane's row as one bf16 pair row.
+__device__ __forceinline__ void stage_pair_row64(uint8_t *xb, uint32_t taddr, int lane) {
+#pragma unroll
+    for (int hlf = 0; hlf < 2; ++hlf) {
+        float v[32];
+        tmem_ld32(taddr + 32 * hlf, v);
+#pragma unroll
+        for (int u = 0; u < 4; ++u) stage_pair_unit(xb, lane, 4 * hlf + u, v + 8 * u);
+    }
+    __syncwarp();
+}
+
+// Copies staged rows 0 .. nrows-1 to global memory with 16 lanes per row, so
+// every store instruction writes two whole 256-byte rows; addr(rl, u) gives
+// the destination of unit u of row rl.
+template <typename F>
+__device__ __forceinline__ void store_rows256(const uint8_t *xb, int lane, int nrows, F addr) {
+    const int u = lane & 15;
+#pragma unroll 4
+    for (int i = 0; i < 16; ++i) {
+        const int rl = (lane >> 4) + 2 * i;
+        const uint4 val = *reinterpret_cast<const uint4 *>(xb + xoff256(rl, u));
+        if (rl < nrows) *addr(rl, u) = val;
+    }
+    __syncwarp();
+}
+
+// TMEM columns taddr .. taddr+31 of this lane's row into a 32 x 128-byte
+// buffer: 16-byte unit c of row rl at rl*128 + ((c ^ (rl & 7)) << 4).
+__device__ __forceinline__ void stage_f32_32(uint8_t *xb, uint32_t taddr, int lane) {
+    float v[32];
+    tmem_ld32(taddr, v);
+#pragma unroll
+    for (int c = 0; c < 8; ++c)
+        *reinterpret_cast<float4 *>(xb + lane * 128 + ((c ^ (lane & 7)) << 4)) =
+            make_float4(v[4 * c], v[4 * c + 1], v[4 * c + 2], v[4 * c + 3]);
+    __syncwarp();
 }
 
 // The gathered A operand of one stage, copied by the 128 threads of warps 4-7
@@ -230,7 +292,8 @@ __device__ __forceinline__ void gather_operand(const TcParams &p, uint8_t *sA, u
 }
 
 template <int KIND>
-__global__ void __launch_bounds__(kThreads, 1) tc_gemm_kernel(const __grid_constant__ TcParams p) {
+__global__ void __launch_bounds__(kThreads, Cfg<KIND>::MIN_CTAS)
+    tc_gemm_kernel(const __grid_constant__ TcParams p) {
     using C = Cfg<KIND>;
     constexpr int S = C::STAGES;
     extern __shared__ uint8_t smem_raw[];
@@ -245,7 +308,8 @@ __global__ void __launch_bounds__(kThreads, 1) tc_gemm_kernel(const __grid_const
     int *s_rows = s_abort + 1 + 2;  // 128 gather rows, 16-byte aligned below
     s_rows = reinterpret_cast<int *>((reinterpret_cast<uintptr_t>(s_rows) + 15) & ~uintptr_t(15));
     float *s_dl = reinterpret_cast<float *>(s_rows + kBM);   // dlogit of the tile's rows (kDX)
-    uint8_t *s_xpose = reinterpret_cast<uint8_t *>(bars) + 2048;  // 4 x 4 KB (scatter kinds)
+    static_assert(KIND == kROUTER || S * (C::A_BYTES + C::B_BYTES) >= 8 * kXpose,
+                  "epilogue staging must fit in the operand ring");
 
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     const int m_tile = blockIdx.x, n_tile = blockIdx.y;
@@ -290,6 +354,7 @@ __global__ void __launch_bounds__(kThreads, 1) tc_gemm_kernel(const __grid_const
 
     if (warp == 0) {
         // ------------------------------------------------------- producer
+        const int nbl = KIND == kROUTER ? p.N / 64 : 0;  // router: 64-wide W_r blocks per stage
         int issued = 0;
         for (int it = 0; it < nkb; ++it) {
             const int s = it % S;
@@ -306,7 +371,11 @@ __global__ void __launch_bounds__(kThreads, 1) tc_gemm_kernel(const __grid_const
             }
             const int kb = kb_begin + it;
             const uint32_t a = smem_u32(sA + s * C::A_BYTES), b = smem_u32(sB + s * C::B_BYTES);
-            if (lane == 0) mbar_expect_tx(fb, gathers<KIND>() ? C::B_BYTES : C::A_BYTES + C::B_BYTES);
+            if (lane == 0) {
+                const uint32_t tx = KIND == kROUTER ? C::A_BYTES + nbl * kTile8K
+                                    : gathers<KIND>() ? C::B_BYTES : C::A_BYTES + C::B_BYTES;
+                mbar_expect_tx(fb, tx);
+            }
             __syncwarp();
             if constexpr (KIND == kQKV) {
                 if (lane < 3) tma_load_3d(b + lane * kTile8K, &p.mapB[lane], fb, 0, kb * kBK, h);
@@ -319,7 +388,7 @@ __global__ void __launch_bounds__(kThreads, 1) tc_gemm_kernel(const __grid_const
                     tma_load_3d(b + (lane - 2) * kTile8K, &p.mapB[0], fb, n0 + 64 * (lane - 2), 0, h);
             } else if constexpr (KIND == kROUTER) {
                 if (lane == 0) tma_load_2d(a, &p.mapA, fb, kb * kBK, m0);
-                if (lane == 1 || lane == 2)
+                if (lane >= 1 && lane <= nbl)
                     tma_load_2d(b + (lane - 1) * kTile8K, &p.mapB[0], fb, n0 + 64 * (lane - 1), kb * kBK);
             } else if constexpr (KIND == kDX) {
                 if (lane == 0) tma_load_3d(a, &p.mapA, fb, 64 * kb, m0, h);
@@ -340,7 +409,8 @@ __global__ void __launch_bounds__(kThreads, 1) tc_gemm_kernel(const __grid_const
     } else if (warp == 1) {
         // ------------------------------------------------------ MMA issuer
         if (lane == 0) {
-            constexpr uint32_t idesc = idesc_bf16(kBM, C::BN, C::A_MN, C::B_MN);
+            const uint32_t idesc = KIND == kROUTER ? idesc_bf16(kBM, p.N, false, true)
+                                                   : idesc_bf16(kBM, C::BN, C::A_MN, C::B_MN);
             for (int it = 0; it < nkb; ++it) {
                 const int s = it % S;
                 if (!mbar_wait(smem_u32(&full[s]), (it / S) & 1) || *(volatile int *)s_abort) {
@@ -371,58 +441,61 @@ __global__ void __launch_bounds__(kThreads, 1) tc_gemm_kernel(const __grid_const
     } else if (warp >= 4) {
         if constexpr (gathers<KIND>()) gather_operand<KIND>(p, sA, full, empty, s_rows, s_abort, h, m0,
                                                             kb_begin, nkb);
-        // -------------------------------------------------------- epilogue
-        const int q = warp - 4;
+    }
+
+    // ------------------------------------------------------------ epilogue
+    // Warps 4-7 always; warps 0-3 too for the kinds with wide tiles.  Warp w
+    // reads TMEM lanes 32 (w % 4) .. +31, i.e. tile rows q*32 .. q*32+31, and
+    // takes column part (w < 4).  Its staging buffer for coalescing the global
+    // writes lies in the operand ring, which is idle once every MMA is done.
+    if (warp >= 4 || epi_all_warps<KIND>()) {
+        __syncwarp();
+        const int q = warp & 3;
+        const int part = warp < 4 ? 1 : 0;
         const int r = q * 32 + lane;
         const int mg = m0 + r;
         const bool ok = mbar_wait(smem_u32(done), 0);
         tc_fence_after();
-        pdl_trigger();  // main loop done: the next kernel may start its prologue
-        const bool abort = !ok || *(volatile int *)s_abort || nkb <= 0;
-        if (!ok && lane == 0) atomicOr(p.status, kStatusTimeout);
+        if (warp >= 4) pdl_trigger();  // main loop done: the next kernel may start its prologue
+        // warp-uniform, since the TMEM loads below are warp-collective
+        const bool abort = __any_sync(0xffffffffu, !ok || *(volatile int *)s_abort || nkb <= 0);
+        if (!ok) atomicOr(p.status, kStatusTimeout);
         const uint32_t tb = tmem + ((uint32_t)(q * 32) << 16);
-        if constexpr (KIND == kQKV) {
-            const size_t row = (size_t)h * p.Mtok + mg;
-#pragma unroll 1
-            for (int c0 = 0; c0 < C::BN; c0 += 32) {
-                float v[32];
-                tmem_ld32(tb + c0, v);
-                if (!abort && mg < p.M) {
-                    bf16 *base = static_cast<bf16 *>(p.out[c0 / 64]) + row * 128 + (c0 % 64);
-                    store_pair_row32(base, base + 64, v);
-                }
+        uint8_t *xb = smem + warp * kXpose;
+        if (abort) {
+            // nothing to write
+        } else if constexpr (KIND == kQKV) {
+            // Q and K by warps 4-7, V by warps 0-3; one 256-byte pair row per matrix row
+            for (int j = part == 0 ? 0 : 2; j < (part == 0 ? 2 : 3); ++j) {
+                stage_pair_row64(xb, tb + 64 * j, lane);
+                bf16 *dst = static_cast<bf16 *>(p.out[j]) + ((size_t)h * p.Mtok + m0 + q * 32) * 128;
+                const int nrows = min(32, p.M - (m0 + q * 32));
+                store_rows256(xb, lane, nrows, [&](int rl, int u) {
+                    return reinterpret_cast<uint4 *>(dst + (size_t)rl * 128) + u;
+                });
             }
         } else if constexpr (KIND == kOUT || KIND == kDX) {
-            // Transpose each 32 x 32 block through this warp's shared buffer so that
-            // every red.add.v4 instruction covers four whole 128-byte row segments.
-            uint8_t *xb = s_xpose + q * 4096;
+            // 32 x 32 blocks transposed through shared memory so that every
+            // red.add.v4 covers four whole 128-byte row segments
             const int chunk = lane & 7;
-#pragma unroll 1
-            for (int c0 = 0; c0 < C::BN; c0 += 32) {
-                float v[32];
-                tmem_ld32(tb + c0, v);
-#pragma unroll
-                for (int c = 0; c < 8; ++c)
-                    *reinterpret_cast<float4 *>(xb + lane * 128 + ((c ^ (lane & 7)) << 4)) =
-                        make_float4(v[4 * c], v[4 * c + 1], v[4 * c + 2], v[4 * c + 3]);
-                __syncwarp();
+            for (int c0 = part * (C::BN / 2); c0 < (part + 1) * (C::BN / 2); c0 += 32) {
+                stage_f32_32(xb, tb + c0, lane);
                 const int n = n0 + c0 + 4 * chunk;
                 float4 w4 = make_float4(0.f, 0.f, 0.f, 0.f);
                 if (KIND == kDX && n < p.d)
                     w4 = *reinterpret_cast<const float4 *>(p.WrT + (size_t)h * p.d + n);
-                const float w[4] = {w4.x, w4.y, w4.z, w4.w};
 #pragma unroll
                 for (int i = 0; i < 8; ++i) {
                     const int rl = (lane >> 3) + 4 * i;
                     const int rt = q * 32 + rl;
                     float4 val = *reinterpret_cast<const float4 *>(xb + rl * 128 + ((chunk ^ (rl & 7)) << 4));
-                    if (!abort && m0 + rt < p.M && n < p.d) {
+                    if (m0 + rt < p.M && n < p.d) {
                         if (KIND == kDX) {
                             const float dl = s_dl[rt];
-                            val.x = fmaf(dl, w[0], val.x);
-                            val.y = fmaf(dl, w[1], val.y);
-                            val.z = fmaf(dl, w[2], val.z);
-                            val.w = fmaf(dl, w[3], val.w);
+                            val.x = fmaf(dl, w4.x, val.x);
+                            val.y = fmaf(dl, w4.y, val.y);
+                            val.z = fmaf(dl, w4.z, val.z);
+                            val.w = fmaf(dl, w4.w, val.w);
                         }
                         red_add_v4(p.out_f + (size_t)s_rows[rt] * p.d + n, val.x, val.y, val.z, val.w);
                     }
@@ -430,114 +503,127 @@ __global__ void __launch_bounds__(kThreads, 1) tc_gemm_kernel(const __grid_const
                 __syncwarp();
             }
         } else if constexpr (KIND == kG) {
-            float g[64];
-            float lo[32];
-            tmem_ld32(tb, lo);
+            // G row in two 32-column halves: dr = <A, G> accumulates, dA = r G is staged
+            const bool live = mg < p.M;
+            const size_t row = (size_t)h * p.Mtok + (live ? mg : 0);
+            const float rr = live ? p.rsel[row] : 0.f;
+            const float4 *arow = reinterpret_cast<const float4 *>(p.A32 + row * 64);
+            float dr = 0.f;
 #pragma unroll
-            for (int e = 0; e < 32; ++e) g[e] = lo[e];
-            tmem_ld32(tb + 32, lo);
+            for (int hlf = 0; hlf < 2; ++hlf) {
+                float g[32];
+                tmem_ld32(tb + 32 * hlf, g);
 #pragma unroll
-            for (int e = 0; e < 32; ++e) g[32 + e] = lo[e];
-            if (!abort && mg < p.M) {
-                const size_t row = (size_t)h * p.Mtok + mg;
-                const float rr = p.rsel[row];
-                const float4 *arow = reinterpret_cast<const float4 *>(p.A32 + row * 64);
-                float dr = 0.f, dd = 0.f;
-#pragma unroll
-                for (int e4 = 0; e4 < 16; ++e4) {
-                    const float4 a4 = arow[e4];
+                for (int e4 = 0; e4 < 8; ++e4) {
+                    const float4 a4 = live ? arow[8 * hlf + e4] : make_float4(0.f, 0.f, 0.f, 0.f);
                     dr = fmaf(a4.x, g[4 * e4 + 0], dr);
                     dr = fmaf(a4.y, g[4 * e4 + 1], dr);
                     dr = fmaf(a4.z, g[4 * e4 + 2], dr);
                     dr = fmaf(a4.w, g[4 * e4 + 3], dr);
                 }
-                // dA = r G (kept as a bf16 pair); D = rowsum(dA o A) = r dr
 #pragma unroll
-                for (int e = 0; e < 64; ++e) g[e] *= rr;
-                dd = rr * dr;
-                bf16 *base = static_cast<bf16 *>(p.out[0]) + row * 128;
-                float half[32];
+                for (int e = 0; e < 32; ++e) g[e] *= rr;  // dA = r G, kept as a bf16 pair
 #pragma unroll
-                for (int e = 0; e < 32; ++e) half[e] = g[e];
-                store_pair_row32(base, base + 64, half);
-#pragma unroll
-                for (int e = 0; e < 32; ++e) half[e] = g[32 + e];
-                store_pair_row32(base + 32, base + 96, half);
-                p.out_f1[row] = dd;
-                const float dl = dr * rr * (1.f - rr);
+                for (int u = 0; u < 4; ++u) stage_pair_unit(xb, lane, 4 * hlf + u, g + 8 * u);
+            }
+            __syncwarp();
+            // D = rowsum(dA o A) = r dr; dlogit = dr r (1 - r)
+            const float dl = dr * rr * (1.f - rr);
+            if (live) {
+                p.out_f1[row] = rr * dr;
                 p.out_f2[row] = dl;
-                // column block 3 of the dQKV pair: dlogit, then zeros (read by kDW for dW_r)
-                bf16 *drow = static_cast<bf16 *>(p.out[1]) + row * kDQKVCols;
+            }
+            const int row0 = m0 + q * 32;
+            const int nrows = min(32, p.M - row0);
+            bf16 *dA = static_cast<bf16 *>(p.out[0]) + ((size_t)h * p.Mtok + row0) * 128;
+            store_rows256(xb, lane, nrows, [&](int rl, int u) {
+                return reinterpret_cast<uint4 *>(dA + (size_t)rl * 128) + u;
+            });
+            // column block 3 of the dQKV pair: dlogit, then zeros (read by kDW for dW_r)
+            {
                 const bf16 dh = __float2bfloat16_rn(dl);
                 const bf16 dlo = __float2bfloat16_rn(dl - __bfloat162float(dh));
                 const uint4 z = make_uint4(0, 0, 0, 0);
 #pragma unroll
-                for (int e = 0; e < 8; ++e) {
-                    uint4 vh = z, vl = z;
-                    if (e == 0) {
-                        vh.x = (uint32_t)__bfloat16_as_ushort(dh);
-                        vl.x = (uint32_t)__bfloat16_as_ushort(dlo);
-                    }
-                    reinterpret_cast<uint4 *>(drow + 192)[e] = vh;
-                    reinterpret_cast<uint4 *>(drow + 448)[e] = vl;
+                for (int u = 0; u < 16; ++u) {
+                    uint4 v4 = z;
+                    if (u == 0) v4.x = (uint32_t)__bfloat16_as_ushort(dh);
+                    if (u == 8) v4.x = (uint32_t)__bfloat16_as_ushort(dlo);
+                    *reinterpret_cast<uint4 *>(xb + xoff256(lane, u)) = v4;
                 }
+                __syncwarp();
+                bf16 *dq = static_cast<bf16 *>(p.out[1]) + ((size_t)h * p.Mtok + row0) * kDQKVCols;
+                store_rows256(xb, lane, nrows, [&](int rl, int u) {
+                    bf16 *base = dq + (size_t)rl * kDQKVCols + (u < 8 ? 192 : 448 - 64);
+                    return reinterpret_cast<uint4 *>(base) + u;
+                });
             }
         } else if constexpr (KIND == kROUTER) {
-            const bool live = !abort && mg < p.M;
+            const bool live = mg < p.M;
             const int bb = live ? mg / p.T : 0, t = live ? mg % p.T : 0;
             float *dst = p.out_f + (size_t)bb * p.H * p.T + t;
-#pragma unroll 1
-            for (int c0 = 0; c0 < C::BN; c0 += 32) {
+            const int ncols = min(C::BN, p.H - n0);
+            for (int c0 = 0; c0 < ncols; c0 += 32) {
                 float v[32];
                 tmem_ld32(tb + c0, v);
-                if (!live) continue;
+                const int nv = live ? min(32, ncols - c0) : 0;
 #pragma unroll
                 for (int e = 0; e < 32; ++e) {
-                    const int hh = n0 + c0 + e;
-                    if (hh < p.H) dst[(size_t)hh * p.T] = 1.f / (1.f + expf(-v[e]));
+                    if (e < nv) dst[(size_t)(n0 + c0 + e) * p.T] = 1.f / (1.f + expf(-v[e]));
                 }
             }
         } else if constexpr (KIND == kDWO) {
-            const bool live = !abort && mg < p.M;
-#pragma unroll 1
-            for (int c0 = 0; c0 < 64; c0 += 32) {
-                float v[32];
-                tmem_ld32(tb + c0, v);
-                if (!live) continue;
-                float *dst = p.out_f + ((size_t)h * 64 + c0) * p.d + mg;
-#pragma unroll
-                for (int e = 0; e < 32; ++e) {
-                    if (p.splits > 1)
-                        atomicAdd(dst + (size_t)e * p.d, v[e]);
-                    else
-                        dst[(size_t)e * p.d] = v[e];
-                }
-            }
-        } else {  // kDW
-            const bool live = !abort && mg < p.M;
-#pragma unroll 1
-            for (int c0 = 0; c0 < 192; c0 += 32) {
-                float v[32];
-                tmem_ld32(tb + c0, v);
-                if (!live) continue;
-                float *W = c0 < 64 ? p.out_f : (c0 < 128 ? p.out_f1 : p.out_f2);
-                float *dst = W + ((size_t)h * p.d + mg) * 64 + (c0 % 64);
-#pragma unroll
-                for (int e = 0; e < 32; e += 4) {
-                    if (p.splits > 1)
-                        red_add_v4(dst + e, v[e], v[e + 1], v[e + 2], v[e + 3]);
-                    else
-                        *reinterpret_cast<float4 *>(dst + e) = make_float4(v[e], v[e + 1], v[e + 2], v[e + 3]);
-                }
-            }
+            // columns p = c0 .. c0+31 of this head's dW_o rows; TMEM lane = output column mg
+            const int c0 = 32 * part;
             float v[32];
-            tmem_ld32(tb + 192, v);  // column 192: dW_r[c, h]
-            if (live) {
-                float *dst = p.out_f3 + (size_t)mg * p.H + h;
-                if (p.splits > 1)
-                    atomicAdd(dst, v[0]);
-                else
-                    *dst = v[0];
+            tmem_ld32(tb + c0, v);
+            float *xf = reinterpret_cast<float *>(xb);
+#pragma unroll
+            for (int e = 0; e < 32; ++e) xf[e * 32 + lane] = v[e];
+            __syncwarp();
+            const int mcol = m0 + q * 32 + 4 * (lane & 7);
+#pragma unroll
+            for (int i = 0; i < 8; ++i) {
+                const int e = (lane >> 3) + 4 * i;
+                const float4 val = *reinterpret_cast<const float4 *>(xf + e * 32 + 4 * (lane & 7));
+                if (mcol < p.M) {
+                    float *dst = p.out_f + ((size_t)h * 64 + c0 + e) * p.d + mcol;
+                    if (p.splits > 1)
+                        red_add_v4(dst, val.x, val.y, val.z, val.w);
+                    else
+                        *reinterpret_cast<float4 *>(dst) = val;
+                }
+            }
+        } else {  // kDW: columns 0..95 by warps 4-7, 96..191 and dW_r by warps 0-3
+            const int chunk = lane & 7;
+            for (int c0 = 96 * part; c0 < 96 * (part + 1); c0 += 32) {
+                stage_f32_32(xb, tb + c0, lane);
+                float *W = c0 < 64 ? p.out_f : (c0 < 128 ? p.out_f1 : p.out_f2);
+#pragma unroll
+                for (int i = 0; i < 8; ++i) {
+                    const int rl = (lane >> 3) + 4 * i;
+                    const int mr = m0 + q * 32 + rl;
+                    const float4 val = *reinterpret_cast<const float4 *>(xb + rl * 128 + ((chunk ^ (rl & 7)) << 4));
+                    if (mr < p.M) {
+                        float *dst = W + ((size_t)h * p.d + mr) * 64 + (c0 % 64) + 4 * chunk;
+                        if (p.splits > 1)
+                            red_add_v4(dst, val.x, val.y, val.z, val.w);
+                        else
+                            *reinterpret_cast<float4 *>(dst) = val;
+                    }
+                }
+                __syncwarp();
+            }
+            if (part == 1) {
+                float v[32];
+                tmem_ld32(tb + 192, v);  // column 192: dW_r[c, h]
+                if (mg < p.M) {
+                    float *dst = p.out_f3 + (size_t)mg * p.H + h;
+                    if (p.splits > 1)
+                        atomicAdd(dst, v[0]);
+                    else
+                        *dst = v[0];
+                }
             }
         }
     }
@@ -627,6 +713,7 @@ bool tc_router(const Dims &dm, const void *X, const void *Wr, float *r_full, uin
     p.T = dm.T;
     p.status = status;
     p.out_f = r_full;
+    p.N = dm.H <= 64 ? 64 : 128;  // MMA width: 64-wide W_r blocks, at most two per tile
     if (!map_2d(&p.mapA, X, (uint64_t)dm.B * dm.T, dm.d, 128) ||
         !map_2d(&p.mapB[0], Wr, dm.d, dm.H, 64))
         return false;

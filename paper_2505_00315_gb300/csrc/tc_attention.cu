@@ -57,7 +57,9 @@ constexpr int kFwdSmem = (int)sizeof(FwdSmem) + 1024;
 
 struct AttnParams {
     CUtensorMap mQ, mK, mV;   // 4-D maps over [H, B, k, 128] pairs, box {64, rows, 1, 1}
+                              // (k <= 128: 3-D maps over [H, B*k, 128], box {64, 128, 1})
     int k, B, Mtok;
+    int U;                    // k <= 128: sequences packed into one 128-row tile
     float scale_log2;         // log2(e) / sqrt(h')
     const float *rsel;        // [H, B*k]
     float *A;                 // [H, B*k, 64]
@@ -372,7 +374,9 @@ constexpr int kDqSmem = (int)sizeof(DqSmem) + 1024;
 
 struct BwdParams {
     CUtensorMap mA0, mA1, mB0, mB1;   // dK/dV: K, V (128 rows), Q, dA (64 rows); dQ: Q, dA (128), K, V (64)
+                                      // k <= 128: Q, K, V, dA as 3-D maps over [H, B*k, 128]
     int k, Mtok;
+    int U, B;                         // k <= 128: sequences per tile, batch
     float scale, scale_log2;
     const float *lse, *Dd;            // [H, B*k]
     bf16 *dQKV;                       // [H, B*k, 512] pair: dQ|dK|dV|dlogit hi, then lo
@@ -739,12 +743,15 @@ __global__ void __launch_bounds__(kThreads, 1) attn_dq_tc_kernel(const __grid_co
     }
 }
 
-// ------------------------------------------------- k <= 128: one CTA per unit
+// ------------------------------------------------- k <= 128: one CTA per tile
 // When a head keeps at most 128 tokens the whole k x k problem of one (b, h)
 // unit fits one CTA: a single 128-key block, no online rescaling (forward) and
-// one fused pass for dQ, dK and dV (backward).  P (then dS) lives in one
-// 128 x 128 bf16-pair tile: K-major (keys contiguous) for P V and dS K, and
-// read through an MN-major descriptor as P^T / dS^T for dV and dK.
+// one fused pass for dQ, dK and dV (backward).  U = floor(128 / k) consecutive
+// sequences of the same head share the tile (their rows are adjacent in the
+// [H, B*k] layout); the mask is then block-diagonal and causal within each
+// block.  P (then dS) lives in one 128 x 128 bf16-pair tile: K-major (keys
+// contiguous) for P V and dS K, and read through an MN-major descriptor as
+// P^T / dS^T for dV and dK.
 
 constexpr int kSmallK = 128;
 constexpr int kPBig = 128 * 64 * 2;   // one 64-key block of a 128-row tile, one half: 16 KB
@@ -771,6 +778,18 @@ struct SmallBwdSmem {
     int abort;
 };
 constexpr int kSmallBwdSmem = (int)sizeof(SmallBwdSmem) + 1024;
+
+// Tile row r (query or key) of the sequences b0 .. b0+U-1: valid when it lies in
+// one of them; lo is the first tile row of its sequence (keys c with
+// lo <= c <= r are visible from query r).
+struct TileRow {
+    bool valid;
+    int lo;
+};
+__device__ __forceinline__ TileRow tile_row(int r, int k, int U, int b0, int B) {
+    const int u = r / k;
+    return TileRow{u < U && b0 + u < B, u * k};
+}
 
 // 32 consecutive keys c0..c0+31 of row r of a [128 x 128] pair tile.
 __device__ __forceinline__ void write_pair32(uint8_t (*tile)[2][kPBig], int r, int c0, const float *v) {
@@ -823,7 +842,7 @@ __global__ void __launch_bounds__(kThreads, 1) attn_fwd_small_kernel(const __gri
     SmallFwdSmem &sm = *reinterpret_cast<SmallFwdSmem *>(
         (reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-    const int b = blockIdx.y, h = blockIdx.z;
+    const int b0 = blockIdx.y * p.U, h = blockIdx.z;
     if (threadIdx.x == 0) {
         mbar_init(smem_u32(&sm.in_full), 1);
         mbar_init(smem_u32(&sm.s_full), 1);
@@ -847,9 +866,9 @@ __global__ void __launch_bounds__(kThreads, 1) attn_fwd_small_kernel(const __gri
             const uint32_t fb = smem_u32(&sm.in_full);
             mbar_expect_tx(fb, 6 * kPBig);
             for (int hf = 0; hf < 2; ++hf) {
-                tma_load_4d(smem_u32(sm.q[hf]), &p.mQ, fb, 64 * hf, 0, b, h);
-                tma_load_4d(smem_u32(sm.k[hf]), &p.mK, fb, 64 * hf, 0, b, h);
-                tma_load_4d(smem_u32(sm.v[hf]), &p.mV, fb, 64 * hf, 0, b, h);
+                tma_load_3d(smem_u32(sm.q[hf]), &p.mQ, fb, 64 * hf, b0 * p.k, h);
+                tma_load_3d(smem_u32(sm.k[hf]), &p.mK, fb, 64 * hf, b0 * p.k, h);
+                tma_load_3d(smem_u32(sm.v[hf]), &p.mV, fb, 64 * hf, b0 * p.k, h);
             }
         }
     } else if (warp == 1) {
@@ -885,7 +904,9 @@ __global__ void __launch_bounds__(kThreads, 1) attn_fwd_small_kernel(const __gri
     } else if (warp >= 4) {
         pdl_trigger();
         const int q = warp - 4;
-        const int r = q * 32 + lane;   // query row i
+        const int r = q * 32 + lane;   // query row i of the tile
+        const TileRow tr = tile_row(r, p.k, p.U, b0, p.B);
+        const int lo = tr.valid ? tr.lo : r + 1;   // invalid rows see no keys
         const uint32_t lane_off = (uint32_t)(q * 32) << 16;
         bool ok = mbar_wait(smem_u32(&sm.s_full), 0);
         tc_fence_after();
@@ -897,7 +918,7 @@ __global__ void __launch_bounds__(kThreads, 1) attn_fwd_small_kernel(const __gri
             tmem_ld32(tS + lane_off + c0, t32);
 #pragma unroll
             for (int c = 0; c < 32; ++c)
-                if (c0 + c <= r) m = fmaxf(m, t32[c] * p.scale_log2);
+                if (c0 + c <= r && c0 + c >= lo) m = fmaxf(m, t32[c] * p.scale_log2);
         }
         // pass 2: probabilities into shared memory, row sum
 #pragma unroll 1
@@ -906,7 +927,7 @@ __global__ void __launch_bounds__(kThreads, 1) attn_fwd_small_kernel(const __gri
             tmem_ld32(tS + lane_off + c0, t32);
 #pragma unroll
             for (int c = 0; c < 32; ++c) {
-                t32[c] = (c0 + c <= r) ? exp2f(t32[c] * p.scale_log2 - m) : 0.f;
+                t32[c] = (c0 + c <= r && c0 + c >= lo) ? exp2f(t32[c] * p.scale_log2 - m) : 0.f;
                 l += t32[c];
             }
             write_pair32(sm.p, r, c0, t32);
@@ -919,8 +940,8 @@ __global__ void __launch_bounds__(kThreads, 1) attn_fwd_small_kernel(const __gri
         float o[64];
         ld64(tO + lane_off, o);
         if (!ok) flag_timeout_b(sm, p.status);
-        if (ok && r < p.k && !*(volatile int *)&sm.abort) {
-            const size_t row = (size_t)h * p.Mtok + (size_t)b * p.k + r;
+        if (ok && tr.valid && !*(volatile int *)&sm.abort) {
+            const size_t row = (size_t)h * p.Mtok + (size_t)b0 * p.k + r;
             const float inv = 1.f / l;
             const float rr = p.rsel[row];
             float *arow = p.A + row * 64;
@@ -947,7 +968,7 @@ __global__ void __launch_bounds__(kThreads, 1) attn_bwd_small_kernel(const __gri
     SmallBwdSmem &sm = *reinterpret_cast<SmallBwdSmem *>(
         (reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-    const int b = blockIdx.y, h = blockIdx.z;
+    const int b0 = blockIdx.y * p.U, h = blockIdx.z;
     if (threadIdx.x == 0) {
         mbar_init(smem_u32(&sm.in_full), 1);
         mbar_init(smem_u32(&sm.sp_full), 1);
@@ -974,10 +995,10 @@ __global__ void __launch_bounds__(kThreads, 1) attn_bwd_small_kernel(const __gri
             const uint32_t fb = smem_u32(&sm.in_full);
             mbar_expect_tx(fb, 8 * kPBig);
             for (int hf = 0; hf < 2; ++hf) {
-                tma_load_4d(smem_u32(sm.q[hf]), &p.mA0, fb, 64 * hf, 0, b, h);
-                tma_load_4d(smem_u32(sm.k[hf]), &p.mA1, fb, 64 * hf, 0, b, h);
-                tma_load_4d(smem_u32(sm.v[hf]), &p.mB0, fb, 64 * hf, 0, b, h);
-                tma_load_4d(smem_u32(sm.da[hf]), &p.mB1, fb, 64 * hf, 0, b, h);
+                tma_load_3d(smem_u32(sm.q[hf]), &p.mA0, fb, 64 * hf, b0 * p.k, h);
+                tma_load_3d(smem_u32(sm.k[hf]), &p.mA1, fb, 64 * hf, b0 * p.k, h);
+                tma_load_3d(smem_u32(sm.v[hf]), &p.mB0, fb, 64 * hf, b0 * p.k, h);
+                tma_load_3d(smem_u32(sm.da[hf]), &p.mB1, fb, 64 * hf, b0 * p.k, h);
             }
         }
     } else if (warp == 1) {
@@ -1020,8 +1041,10 @@ __global__ void __launch_bounds__(kThreads, 1) attn_bwd_small_kernel(const __gri
         const int q = warp - 4;
         const int r = q * 32 + lane;   // query row i for S/dP/dQ; key row j for dK/dV
         const uint32_t lane_off = (uint32_t)(q * 32) << 16;
-        const size_t base = (size_t)h * p.Mtok + (size_t)b * p.k;
-        const bool valid = r < p.k;
+        const size_t base = (size_t)h * p.Mtok + (size_t)b0 * p.k;
+        const TileRow tr = tile_row(r, p.k, p.U, b0, p.B);
+        const bool valid = tr.valid;
+        const int lo = tr.lo;
         const float l2 = valid ? p.lse[base + r] * 1.4426950408889634f : 0.f;
         const float dd = valid ? p.Dd[base + r] : 0.f;
         bool ok = mbar_wait(smem_u32(&sm.sp_full), 0);
@@ -1033,7 +1056,7 @@ __global__ void __launch_bounds__(kThreads, 1) attn_bwd_small_kernel(const __gri
             tmem_ld32(tS + lane_off + c0, t32);
 #pragma unroll
             for (int c = 0; c < 32; ++c)
-                t32[c] = (valid && c0 + c <= r) ? exp2f(t32[c] * p.scale_log2 - l2) : 0.f;
+                t32[c] = (valid && c0 + c <= r && c0 + c >= lo) ? exp2f(t32[c] * p.scale_log2 - l2) : 0.f;
             write_pair32(sm.p, r, c0, t32);
         }
         fence_proxy_async();
@@ -1048,7 +1071,7 @@ __global__ void __launch_bounds__(kThreads, 1) attn_bwd_small_kernel(const __gri
             tmem_ld32(tDP + lane_off + c0, d32);
 #pragma unroll
             for (int c = 0; c < 32; ++c) {
-                const float pr = (valid && c0 + c <= r) ? exp2f(t32[c] * p.scale_log2 - l2) : 0.f;
+                const float pr = (valid && c0 + c <= r && c0 + c >= lo) ? exp2f(t32[c] * p.scale_log2 - l2) : 0.f;
                 t32[c] = pr * (d32[c] - dd);
             }
             write_pair32(sm.p, r, c0, t32);
@@ -1080,6 +1103,14 @@ __global__ void __launch_bounds__(kThreads, 1) attn_bwd_small_kernel(const __gri
 
 // [H, B, k, 128] bf16 pair array (row = 64 hi + 64 lo), box {64, rows, 1, 1}:
 // rows past k of one sequence read as zeros.
+bool map_rows(CUtensorMap *m, const void *base, int H, int Mtok) {
+    // [H, B*k, 128] bf16 pair array, box {64, 128, 1}: 128 consecutive rows of one head
+    const uint64_t dims[3] = {128, (uint64_t)Mtok, (uint64_t)H};
+    const uint64_t strides[2] = {256, (uint64_t)Mtok * 256};
+    const uint32_t box[3] = {64, 128, 1};
+    return tmap_bf16(m, base, 3, dims, strides, box);
+}
+
 bool map_units(CUtensorMap *m, const void *base, int H, int B, int k, uint32_t rows) {
     const uint64_t dims[4] = {128, (uint64_t)k, (uint64_t)B, (uint64_t)H};
     const uint64_t strides[3] = {256, (uint64_t)k * 256, (uint64_t)B * k * 256};
@@ -1093,10 +1124,14 @@ cudaError_t tc_attn_fwd(const Dims &dm, const Saved &sv, cudaStream_t s) {
     AttnParams p;
     memset(&p, 0, sizeof(p));
     const bool small = dm.k <= kSmallK;
-    bool ok = map_units(&p.mQ, sv.Q, dm.H, dm.B, dm.k, kQ) &&
-              map_units(&p.mK, sv.K, dm.H, dm.B, dm.k, small ? 128 : kKV) &&
-              map_units(&p.mV, sv.V, dm.H, dm.B, dm.k, small ? 128 : kKV);
+    const int Mtok = dm.B * dm.k;
+    bool ok = small ? (map_rows(&p.mQ, sv.Q, dm.H, Mtok) && map_rows(&p.mK, sv.K, dm.H, Mtok) &&
+                       map_rows(&p.mV, sv.V, dm.H, Mtok))
+                    : (map_units(&p.mQ, sv.Q, dm.H, dm.B, dm.k, kQ) &&
+                       map_units(&p.mK, sv.K, dm.H, dm.B, dm.k, kKV) &&
+                       map_units(&p.mV, sv.V, dm.H, dm.B, dm.k, kKV));
     if (!ok) return cudaErrorInvalidValue;
+    p.U = small ? kSmallK / dm.k : 1;
     p.k = dm.k;
     p.B = dm.B;
     p.Mtok = dm.B * dm.k;
@@ -1117,8 +1152,8 @@ cudaError_t tc_attn_fwd(const Dims &dm, const Saved &sv, cudaStream_t s) {
     });
     if (attr != cudaSuccess) return attr;
     if (small) {
-        cudaError_t e = launch_pdl(attn_fwd_small_kernel, dim3(1, dm.B, dm.H), dim3(kThreads),
-                                   kSmallFwdSmem, s, p);
+        cudaError_t e = launch_pdl(attn_fwd_small_kernel, dim3(1, (dm.B + p.U - 1) / p.U, dm.H),
+                                   dim3(kThreads), kSmallFwdSmem, s, p);
         note_launches(1);
         return e;
     }
@@ -1135,11 +1170,12 @@ cudaError_t tc_attn_bwd(const Dims &dm, const Saved &sv, cudaStream_t s) {
     if (dm.k <= kSmallK) {
         BwdParams sp;
         memset(&sp, 0, sizeof(sp));
-        const bool ok = map_units(&sp.mA0, sv.Q, dm.H, dm.B, dm.k, 128) &&
-                        map_units(&sp.mA1, sv.K, dm.H, dm.B, dm.k, 128) &&
-                        map_units(&sp.mB0, sv.V, dm.H, dm.B, dm.k, 128) &&
-                        map_units(&sp.mB1, sv.dA, dm.H, dm.B, dm.k, 128);
+        const int Mtok = dm.B * dm.k;
+        const bool ok = map_rows(&sp.mA0, sv.Q, dm.H, Mtok) && map_rows(&sp.mA1, sv.K, dm.H, Mtok) &&
+                        map_rows(&sp.mB0, sv.V, dm.H, Mtok) && map_rows(&sp.mB1, sv.dA, dm.H, Mtok);
         if (!ok) return cudaErrorInvalidValue;
+        sp.U = kSmallK / dm.k;
+        sp.B = dm.B;
         sp.k = dm.k;
         sp.Mtok = dm.B * dm.k;
         sp.scale = 1.f / sqrtf(64.f);
@@ -1156,8 +1192,8 @@ cudaError_t tc_attn_bwd(const Dims &dm, const Saved &sv, cudaStream_t s) {
                                               kSmallBwdSmem);
         });
         if (attr_small != cudaSuccess) return attr_small;
-        cudaError_t e = launch_pdl(attn_bwd_small_kernel, dim3(1, dm.B, dm.H), dim3(kThreads),
-                                   kSmallBwdSmem, s, sp);
+        cudaError_t e = launch_pdl(attn_bwd_small_kernel, dim3(1, (dm.B + sp.U - 1) / sp.U, dm.H),
+                                   dim3(kThreads), kSmallBwdSmem, s, sp);
         note_launches(1);
         return e;
     }

@@ -27,6 +27,7 @@
 //             dlogit in column 0 and zeros), so dW_r comes out of the same product
 //   kROUTER F1 r[b,h,t] = sigmoid(X[b,t,:] W_r[:,h])       A = X tiles, B = W_r MN-major
 // where g(m) = b*T + I[b,h,i] for row m = b*k + i of head h.
+#include <algorithm>
 #include <cstdio>
 #include <mutex>
 
@@ -47,6 +48,7 @@ constexpr int kBK = 64;         // K per stage: one 128-byte swizzle row of bf16
 constexpr int kTile8K = 8192;   // one 64x64 bf16 block
 constexpr int kTile16K = 16384; // one 128x64 bf16 block
 constexpr int kThreads = 256;
+constexpr int kMaxStages = 8;    // mbarrier slots per ring
 
 template <int KIND>
 struct Cfg;
@@ -92,8 +94,10 @@ struct Cfg<kDW> {
 
 template <>
 struct Cfg<kROUTER> {
-    static constexpr int BN = 128, STAGES = 6, A_BYTES = kTile16K, B_BYTES = 2 * kTile8K,
-                         TMEM_COLS = 128, MIN_CTAS = 1;
+    // ring of 192 KB; the stage count is chosen at launch from the MMA width
+    // (p.N = 64..256): a stage holds the X tile and N/64 W_r blocks
+    static constexpr int BN = 256, STAGES = 4, A_BYTES = kTile16K, B_BYTES = 4 * kTile8K,
+                         TMEM_COLS = 256, MIN_CTAS = 1;
     static constexpr bool A_MN = false, B_MN = true, A_PAIR = false, B_PAIR = false;
 };
 
@@ -130,7 +134,9 @@ struct TcParams {
     CUtensorMap mapB[3];   // per-head tile maps of the B operand
     int M;                 // output rows per head: B*k for row kinds, d for kDWO / kDW
     int Mtok;              // selected rows per head, B*k
-    int N;                 // output columns (d for kOUT / kDX)
+    int N;                 // output columns (d for kOUT / kDX); MMA width (kROUTER)
+    int ring_stages;       // kROUTER: stages in the ring (<= kMaxStages)
+    int ring_stride;       // kROUTER: bytes per stage
     int nkb;               // K blocks in the whole reduction
     int splits;            // reduction splits (kDWO / kDW)
     int d, H, T;
@@ -302,7 +308,18 @@ __global__ void __launch_bounds__(kThreads, Cfg<KIND>::MIN_CTAS)
     uint8_t *sA = smem;
     uint8_t *sB = smem + S * C::A_BYTES;
     uint64_t *bars = reinterpret_cast<uint64_t *>(sB + S * C::B_BYTES);
-    uint64_t *full = bars, *empty = bars + S, *done = bars + 2 * S;
+    uint64_t *full = bars, *empty = bars + kMaxStages, *done = bars + 2 * kMaxStages;
+    static_assert(S <= kMaxStages, "ring too deep");
+    // the router's ring is laid out per stage ([X tile | W_r blocks]) with a
+    // stage count fixed at launch; every other kind has STAGES A tiles, then
+    // STAGES B tiles
+    const int ns = KIND == kROUTER ? p.ring_stages : S;
+    auto stage_a = [&](int st) -> uint8_t * {
+        return KIND == kROUTER ? smem + st * p.ring_stride : sA + st * C::A_BYTES;
+    };
+    auto stage_b = [&](int st) -> uint8_t * {
+        return KIND == kROUTER ? smem + st * p.ring_stride + C::A_BYTES : sB + st * C::B_BYTES;
+    };
     uint32_t *tmem_slot = reinterpret_cast<uint32_t *>(done + 1);
     int *s_abort = reinterpret_cast<int *>(tmem_slot + 1);
     int *s_rows = s_abort + 1 + 2;  // 128 gather rows, 16-byte aligned below
@@ -326,7 +343,7 @@ __global__ void __launch_bounds__(kThreads, Cfg<KIND>::MIN_CTAS)
     const int nkb = kb_end - kb_begin;
 
     if (threadIdx.x == 0) {
-        for (int s = 0; s < S; ++s) {
+        for (int s = 0; s < ns; ++s) {
             // gathered kinds: the TMA arrival plus one per gathering thread
             mbar_init(smem_u32(&full[s]), gathers<KIND>() ? 129 : 1);
             mbar_init(smem_u32(&empty[s]), 1);
@@ -357,10 +374,10 @@ __global__ void __launch_bounds__(kThreads, Cfg<KIND>::MIN_CTAS)
         const int nbl = KIND == kROUTER ? p.N / 64 : 0;  // router: 64-wide W_r blocks per stage
         int issued = 0;
         for (int it = 0; it < nkb; ++it) {
-            const int s = it % S;
+            const int s = it % ns;
             const uint32_t fb = smem_u32(&full[s]);
             bool ok = true;
-            if (lane == 0) ok = mbar_wait(smem_u32(&empty[s]), ((it / S) & 1) ^ 1);
+            if (lane == 0) ok = mbar_wait(smem_u32(&empty[s]), ((it / ns) & 1) ^ 1);
             ok = __shfl_sync(0xffffffffu, ok ? 1 : 0, 0) != 0;
             if (!ok || *(volatile int *)s_abort) {
                 if (lane == 0) {
@@ -370,7 +387,7 @@ __global__ void __launch_bounds__(kThreads, Cfg<KIND>::MIN_CTAS)
                 break;
             }
             const int kb = kb_begin + it;
-            const uint32_t a = smem_u32(sA + s * C::A_BYTES), b = smem_u32(sB + s * C::B_BYTES);
+            const uint32_t a = smem_u32(stage_a(s)), b = smem_u32(stage_b(s));
             if (lane == 0) {
                 const uint32_t tx = KIND == kROUTER ? C::A_BYTES + nbl * kTile8K
                                     : gathers<KIND>() ? C::B_BYTES : C::A_BYTES + C::B_BYTES;
@@ -403,8 +420,8 @@ __global__ void __launch_bounds__(kThreads, Cfg<KIND>::MIN_CTAS)
         }
         if (*(volatile int *)s_abort && lane == 0) {
             // Let copies already in flight land before the CTA can exit.
-            for (int it = max(0, issued - S); it < issued; ++it)
-                mbar_wait(smem_u32(&full[it % S]), (it / S) & 1);
+            for (int it = max(0, issued - ns); it < issued; ++it)
+                mbar_wait(smem_u32(&full[it % ns]), (it / ns) & 1);
         }
     } else if (warp == 1) {
         // ------------------------------------------------------ MMA issuer
@@ -412,14 +429,14 @@ __global__ void __launch_bounds__(kThreads, Cfg<KIND>::MIN_CTAS)
             const uint32_t idesc = KIND == kROUTER ? idesc_bf16(kBM, p.N, false, true)
                                                    : idesc_bf16(kBM, C::BN, C::A_MN, C::B_MN);
             for (int it = 0; it < nkb; ++it) {
-                const int s = it % S;
-                if (!mbar_wait(smem_u32(&full[s]), (it / S) & 1) || *(volatile int *)s_abort) {
+                const int s = it % ns;
+                if (!mbar_wait(smem_u32(&full[s]), (it / ns) & 1) || *(volatile int *)s_abort) {
                     atomicOr(p.status, kStatusTimeout);
                     *(volatile int *)s_abort = 1;
                     break;
                 }
                 tc_fence_after();
-                const uint32_t a = smem_u32(sA + s * C::A_BYTES), b = smem_u32(sB + s * C::B_BYTES);
+                const uint32_t a = smem_u32(stage_a(s)), b = smem_u32(stage_b(s));
                 constexpr int pairs = (C::A_PAIR || C::B_PAIR) ? 2 : 1;
 #pragma unroll
                 for (int half = 0; half < pairs; ++half) {
@@ -713,11 +730,13 @@ bool tc_router(const Dims &dm, const void *X, const void *Wr, float *r_full, uin
     p.T = dm.T;
     p.status = status;
     p.out_f = r_full;
-    p.N = dm.H <= 64 ? 64 : 128;  // MMA width: 64-wide W_r blocks, at most two per tile
+    p.N = std::min(256, (dm.H + 63) / 64 * 64);  // MMA width: 64-wide W_r blocks
+    p.ring_stride = kTile16K + p.N / 64 * kTile8K;
+    p.ring_stages = std::min(kMaxStages, Cfg<kROUTER>::STAGES * (kTile16K + 4 * kTile8K) / p.ring_stride);
     if (!map_2d(&p.mapA, X, (uint64_t)dm.B * dm.T, dm.d, 128) ||
         !map_2d(&p.mapB[0], Wr, dm.d, dm.H, 64))
         return false;
-    dim3 grid((p.M + kBM - 1) / kBM, (dm.H + 127) / 128, 1);
+    dim3 grid((p.M + kBM - 1) / kBM, (dm.H + 255) / 256, 1);
     *err = launch_kind<kROUTER>(p, grid, s);
     return true;
 }

@@ -69,6 +69,11 @@ SMALL = [
     W.MosaConfig("k1_f32", B=3, T=50, d=16, H=5, hp=16, k=1, dtype="f32", seed=14),
     W.MosaConfig("hp128_bf16", B=1, T=200, d=256, H=2, hp=128, k=130, dtype="bf16", seed=15),
     W.MosaConfig("hp16_f32", B=2, T=129, d=24, H=7, hp=16, k=65, dtype="f32", seed=16),
+    # k <= 64: several sequences of a head share one 128-row attention tile
+    W.MosaConfig("pack2_oddB_bf16", B=3, T=200, d=64, H=2, hp=64, k=64, dtype="bf16", seed=17),
+    W.MosaConfig("pack4_bf16", B=5, T=100, d=64, H=3, hp=64, k=32, dtype="bf16", seed=18),
+    W.MosaConfig("pack2_k50_bf16", B=5, T=120, d=64, H=2, hp=64, k=50, dtype="bf16", seed=19),
+    W.MosaConfig("pack42_k3_bf16", B=5, T=40, d=32, H=2, hp=64, k=3, dtype="bf16", seed=20),
 ]
 
 

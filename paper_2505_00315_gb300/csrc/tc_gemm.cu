@@ -24,7 +24,8 @@
 //             (W_r read from its fp32 transpose [H, d], one float4 per lane)
 //   kDW   B4  [dW_q|dW_k|dW_v|dW_r][h](c,:) = sum_m X[g(m),c] [dQ|dK|dV|dlogit](m,:)
 //             A gathered MN-major, B = the dQKV pair (its 4th 64-column block holds
-//             dlogit in column 0 and zeros), so dW_r comes out of the same product
+//             dlogit in column 0 and zeros), so dW_r comes out of the same product;
+//             256 rows c per CTA in two accumulators that share every B tile
 //   kROUTER F1 r[b,h,t] = sigmoid(X[b,t,:] W_r[:,h])       A = X tiles, B = W_r MN-major
 // where g(m) = b*T + I[b,h,i] for row m = b*k + i of head h.
 #include <algorithm>
@@ -87,8 +88,10 @@ struct Cfg<kDX> {
 };
 template <>
 struct Cfg<kDW> {
-    static constexpr int BN = 256, STAGES = 2, A_BYTES = kTile16K, B_BYTES = 8 * kTile8K,
-                         TMEM_COLS = 256, MIN_CTAS = 1;
+    // 256 rows of d per CTA as two 128 x 256 accumulators sharing each B tile;
+    // K blocks of 32 tokens: A = 4 blocks of 32 x 64, B = 8 blocks of 32 x 64
+    static constexpr int BN = 256, STAGES = 4, A_BYTES = 4 * 4096, B_BYTES = 8 * 4096,
+                         TMEM_COLS = 512, MIN_CTAS = 1;
     static constexpr bool A_MN = true, B_MN = true, A_PAIR = false, B_PAIR = true;
 };
 
@@ -100,6 +103,16 @@ struct Cfg<kROUTER> {
                          TMEM_COLS = 256, MIN_CTAS = 1;
     static constexpr bool A_MN = false, B_MN = true, A_PAIR = false, B_PAIR = false;
 };
+
+// Tokens per K block and accumulators (128-row tiles) per CTA.
+template <int KIND>
+__host__ __device__ constexpr int kind_bk() {
+    return KIND == kDW ? 32 : kBK;
+}
+template <int KIND>
+__host__ __device__ constexpr int kind_acc() {
+    return KIND == kDW ? 2 : 1;
+}
 
 // Row width (bf16) of the dQKV pair array on the tensor-core path:
 // [dQ | dK | dV | dlogit, 0..] hi (256) then the same lo (256).
@@ -233,18 +246,24 @@ __device__ __forceinline__ void stage_f32_32(uint8_t *xb, uint32_t taddr, int la
 // The gathered A operand of one stage, copied by the 128 threads of warps 4-7
 // with 16-byte cp.async into the 128-byte-swizzled layout the MMA reads:
 //   K-major (kQKV, kG):    rows m of the tile = source rows g(m), 64 columns of K block kb
-//   MN-major (kDWO, kDW):  64 tokens of K block kb, columns m0 .. m0+127 in two
+//   MN-major (kDWO):       64 tokens of K block kb, columns m0 .. m0+127 in two
 //                          64-wide blocks; token rows are the smem rows
+//   MN-major (kDW):        32 tokens of K block kb, columns m0 .. m0+255 in four
+//                          64-wide blocks
 // Element (row, 16-byte chunk c) lands at row*128 + ((c ^ (row & 7)) * 16).
-// Each thread keeps up to STAGES copy groups in flight; when a stage's group
-// has landed it makes the copies visible to the tensor core (proxy fence) and
-// arrives on that stage's full barrier.
+// A stage's copies are confirmed (wait, proxy fence, arrival on its full
+// barrier) LAG stages after they are issued, with LAG = STAGES - 2 (deeper
+// rings; a two-stage ring keeps LAG = 1): issuing
+// stage it + LAG waits only for the MMAs of stage it - 2, so the barrier of
+// stage it opens while the MMAs of stage it - 1 still run and the tensor pipe
+// never drains between K blocks.
 template <int KIND>
 __device__ __forceinline__ void gather_operand(const TcParams &p, uint8_t *sA, uint64_t *full,
                                                uint64_t *empty, const int *s_rows, int *s_abort,
                                                int h, int m0, int kb_begin, int nkb) {
     using C = Cfg<KIND>;
     constexpr int S = C::STAGES;
+    constexpr int LAG = S >= 3 ? S - 2 : S - 1;  // a two-stage ring keeps one stage of lag
     const int t = threadIdx.x - 128;       // 0..127
     const int chunk = t & 7, sub = t >> 3;  // 16 rows x 8 chunks per pass
     const bf16 *src = static_cast<const bf16 *>(p.src_rows);
@@ -268,6 +287,21 @@ __device__ __forceinline__ void gather_operand(const TcParams &p, uint8_t *sA, u
                 const bf16 *g = src + (size_t)s_rows[row] * p.d + (nbytes ? col : 0);
                 cp_async16(a + row * 128 + ((chunk ^ (row & 7)) << 4), g, nbytes);
             }
+        } else if constexpr (KIND == kDW) {
+            // 32 tokens x 256 columns of d in four 64-wide blocks of 4 KB
+#pragma unroll
+            for (int q2 = 0; q2 < 2; ++q2) {
+                const int tok = sub + 16 * q2;
+                const int tg = kb * 32 + tok;
+                const int rowg = tg < p.Mtok ? gi[tg] : 0;
+#pragma unroll
+                for (int j = 0; j < 4; ++j) {
+                    const int col = m0 + 64 * j + chunk * 8;
+                    const uint32_t nbytes = (tg < p.Mtok && col < p.d) ? 16u : 0u;
+                    const bf16 *g = src + (size_t)rowg * p.d + (nbytes ? col : 0);
+                    cp_async16(a + j * 4096 + tok * 128 + ((chunk ^ (tok & 7)) << 4), g, nbytes);
+                }
+            }
         } else {
 #pragma unroll
             for (int q4 = 0; q4 < 4; ++q4) {
@@ -284,10 +318,10 @@ __device__ __forceinline__ void gather_operand(const TcParams &p, uint8_t *sA, u
             }
         }
         cp_async_commit();
-        if (it >= S - 1) {
-            cp_async_wait<S - 1>();
+        if (it >= LAG) {
+            cp_async_wait<LAG>();
             fence_proxy_async();
-            mbar_arrive(smem_u32(&full[(it - (S - 1)) % S]));
+            mbar_arrive(smem_u32(&full[(it - LAG) % S]));
             ++landed;
         }
     }
@@ -332,7 +366,7 @@ __global__ void __launch_bounds__(kThreads, Cfg<KIND>::MIN_CTAS)
     const int m_tile = blockIdx.x, n_tile = blockIdx.y;
     const int h = (KIND == kDWO || KIND == kDW) ? blockIdx.z / p.splits : blockIdx.z;
     const int split = (KIND == kDWO || KIND == kDW) ? blockIdx.z % p.splits : 0;
-    const int m0 = m_tile * kBM;
+    const int m0 = m_tile * kBM * kind_acc<KIND>();
     const int n0 = n_tile * C::BN;
     int kb_begin = 0, kb_end = p.nkb;
     if (KIND == kDWO || KIND == kDW) {
@@ -413,8 +447,8 @@ __global__ void __launch_bounds__(kThreads, Cfg<KIND>::MIN_CTAS)
                 if (lane == 2) tma_load_3d(b, &p.mapB[kb], fb, 0, n0, h);
             } else if constexpr (KIND == kDWO) {
                 if (lane < 2) tma_load_3d(b + lane * kTile8K, &p.mapB[0], fb, 64 * lane, kb * kBK, h);
-            } else {  // kDW: hi blocks 0..3 then lo blocks 0..3
-                if (lane < 8) tma_load_3d(b + lane * kTile8K, &p.mapB[0], fb, 64 * lane, kb * kBK, h);
+            } else {  // kDW: hi blocks 0..3 then lo blocks 0..3, 32 token rows each
+                if (lane < 8) tma_load_3d(b + lane * 4096, &p.mapB[0], fb, 64 * lane, kb * 32, h);
             }
             issued = it + 1;
         }
@@ -438,6 +472,19 @@ __global__ void __launch_bounds__(kThreads, Cfg<KIND>::MIN_CTAS)
                 tc_fence_after();
                 const uint32_t a = smem_u32(stage_a(s)), b = smem_u32(stage_b(s));
                 constexpr int pairs = (C::A_PAIR || C::B_PAIR) ? 2 : 1;
+                if constexpr (KIND == kDW) {
+                    // accumulator c: rows of d-blocks 2c, 2c+1; B pair halves at +0 / +16 KB
+#pragma unroll
+                    for (int c = 0; c < 2; ++c)
+#pragma unroll
+                        for (int half = 0; half < 2; ++half)
+#pragma unroll
+                            for (int j = 0; j < 2; ++j)
+                                mma_bf16(tmem + 256 * c,
+                                         smem_desc_sw128(a + c * 8192 + j * 2048, 4096, 1024),
+                                         smem_desc_sw128(b + half * 16384 + j * 2048, 4096, 1024),
+                                         idesc, (it > 0 || half > 0 || j > 0) ? 1u : 0u);
+                } else
 #pragma unroll
                 for (int half = 0; half < pairs; ++half) {
                     const uint32_t ah = a + (C::A_PAIR ? half * (C::A_BYTES / 2) : 0);
@@ -611,15 +658,17 @@ __global__ void __launch_bounds__(kThreads, Cfg<KIND>::MIN_CTAS)
                         *reinterpret_cast<float4 *>(dst) = val;
                 }
             }
-        } else {  // kDW: columns 0..95 by warps 4-7, 96..191 and dW_r by warps 0-3
+        } else {  // kDW: warps 4-7 accumulator 0 (d rows m0 ..), warps 0-3 accumulator 1 (m0+128 ..)
             const int chunk = lane & 7;
-            for (int c0 = 96 * part; c0 < 96 * (part + 1); c0 += 32) {
-                stage_f32_32(xb, tb + c0, lane);
+            const uint32_t ta = tb + 256 * part;
+            const int mrow0 = m0 + 128 * part + q * 32;
+            for (int c0 = 0; c0 < 192; c0 += 32) {
+                stage_f32_32(xb, ta + c0, lane);
                 float *W = c0 < 64 ? p.out_f : (c0 < 128 ? p.out_f1 : p.out_f2);
 #pragma unroll
                 for (int i = 0; i < 8; ++i) {
                     const int rl = (lane >> 3) + 4 * i;
-                    const int mr = m0 + q * 32 + rl;
+                    const int mr = mrow0 + rl;
                     const float4 val = *reinterpret_cast<const float4 *>(xb + rl * 128 + ((chunk ^ (rl & 7)) << 4));
                     if (mr < p.M) {
                         float *dst = W + ((size_t)h * p.d + mr) * 64 + (c0 % 64) + 4 * chunk;
@@ -631,16 +680,15 @@ __global__ void __launch_bounds__(kThreads, Cfg<KIND>::MIN_CTAS)
                 }
                 __syncwarp();
             }
-            if (part == 1) {
-                float v[32];
-                tmem_ld32(tb + 192, v);  // column 192: dW_r[c, h]
-                if (mg < p.M) {
-                    float *dst = p.out_f3 + (size_t)mg * p.H + h;
-                    if (p.splits > 1)
-                        atomicAdd(dst, v[0]);
-                    else
-                        *dst = v[0];
-                }
+            float v[32];
+            tmem_ld32(ta + 192, v);  // column 192: dW_r[c, h]
+            const int mr = mrow0 + lane;
+            if (mr < p.M) {
+                float *dst = p.out_f3 + (size_t)mr * p.H + h;
+                if (p.splits > 1)
+                    atomicAdd(dst, v[0]);
+                else
+                    *dst = v[0];
             }
         }
     }
@@ -865,11 +913,13 @@ cudaError_t tc_w_bwd(const Dims &dm, const void *X, const Saved &sv, float *dWq,
                      float *dWv, float *dWr, cudaStream_t s) {
     TcParams p = base_params(dm, sv);
     p.M = dm.d;
-    p.nkb = (p.Mtok + kBK - 1) / kBK;
-    const int tiles = (dm.d + kBM - 1) / kBM * dm.H;
-    p.splits = splits_for(tiles, p.nkb);
+    p.nkb = (p.Mtok + 31) / 32;
+    const int tiles = (dm.d + 255) / 256 * dm.H;
+    // one wave of single-CTA SMs: the most reduction splits with tiles * splits <= 152
+    p.splits = 1;
+    while (tiles * p.splits * 2 <= 152 && p.splits * 4 <= p.nkb) p.splits *= 2;
     bool ok = map_gather(&p.mapA, X, (uint64_t)dm.B * dm.T, dm.d) &&
-              map_heads(&p.mapB[0], sv.dQKV, dm.H, p.Mtok, kDQKVCols, 64);
+              map_heads(&p.mapB[0], sv.dQKV, dm.H, p.Mtok, kDQKVCols, 32);
     if (!ok) return cudaErrorInvalidValue;
     p.src_rows = X;
     p.out_f = dWq;
@@ -885,7 +935,7 @@ cudaError_t tc_w_bwd(const Dims &dm, const void *X, const Saved &sv, float *dWq,
         if ((e = cudaMemsetAsync(dWr, 0, sizeof(float) * (size_t)dm.d * dm.H, s)) != cudaSuccess)
             return e;
     }
-    dim3 grid((dm.d + kBM - 1) / kBM, 1, dm.H * p.splits);
+    dim3 grid((dm.d + 255) / 256, 1, dm.H * p.splits);
     return launch_kind<kDW>(p, grid, s);
 }
 

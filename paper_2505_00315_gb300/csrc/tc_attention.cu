@@ -761,6 +761,7 @@ struct SmallFwdSmem {
     uint8_t k[2][kPBig];
     uint8_t v[2][kPBig];
     uint8_t p[2][2][kPBig];           // [half][key block]
+    float part_max[2][128], part_sum[2][128];   // per key half: row max, row sum
     uint64_t in_full, s_full, p_ready, o_full;
     uint32_t tmem;
     int abort;
@@ -837,7 +838,14 @@ __device__ __forceinline__ void mma_k128(uint32_t d, const uint8_t (*a)[2][kPBig
     }
 }
 
-__global__ void __launch_bounds__(kThreads, 1) attn_fwd_small_kernel(const __grid_constant__ AttnParams p) {
+// Threads of the k <= 128 kernels: warps 0-3 load, issue MMAs and own TMEM;
+// warps 4-11 run the softmax passes and the epilogue, two per TMEM lane
+// quadrant: warp w serves tile rows 32 (w % 4) .. +31 and key (or output)
+// column half ch = (w - 4) / 4.
+constexpr int kSmallThreads = 384;
+constexpr int kSoftmaxThreads = 256;
+
+__global__ void __launch_bounds__(kSmallThreads, 1) attn_fwd_small_kernel(const __grid_constant__ AttnParams p) {
     extern __shared__ uint8_t smem_raw[];
     SmallFwdSmem &sm = *reinterpret_cast<SmallFwdSmem *>(
         (reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
@@ -846,7 +854,7 @@ __global__ void __launch_bounds__(kThreads, 1) attn_fwd_small_kernel(const __gri
     if (threadIdx.x == 0) {
         mbar_init(smem_u32(&sm.in_full), 1);
         mbar_init(smem_u32(&sm.s_full), 1);
-        mbar_init(smem_u32(&sm.p_ready), 128);
+        mbar_init(smem_u32(&sm.p_ready), kSoftmaxThreads);
         mbar_init(smem_u32(&sm.o_full), 1);
         sm.abort = 0;
         fence_barrier_init();
@@ -903,26 +911,31 @@ __global__ void __launch_bounds__(kThreads, 1) attn_fwd_small_kernel(const __gri
         }
     } else if (warp >= 4) {
         pdl_trigger();
-        const int q = warp - 4;
+        const int q = warp & 3, ch = (warp - 4) >> 2;
         const int r = q * 32 + lane;   // query row i of the tile
+        const int cb = 64 * ch;        // this thread's 64 keys
         const TileRow tr = tile_row(r, p.k, p.U, b0, p.B);
         const int lo = tr.valid ? tr.lo : r + 1;   // invalid rows see no keys
         const uint32_t lane_off = (uint32_t)(q * 32) << 16;
         bool ok = mbar_wait(smem_u32(&sm.s_full), 0);
         tc_fence_after();
-        float m = -INFINITY, l = 0.f;
-        // pass 1: row max
+        // pass 1: row max over both halves
+        float m = -INFINITY;
 #pragma unroll 1
-        for (int c0 = 0; c0 < kSmallK; c0 += 32) {
+        for (int c0 = cb; c0 < cb + 64; c0 += 32) {
             float t32[32];
             tmem_ld32(tS + lane_off + c0, t32);
 #pragma unroll
             for (int c = 0; c < 32; ++c)
                 if (c0 + c <= r && c0 + c >= lo) m = fmaxf(m, t32[c] * p.scale_log2);
         }
-        // pass 2: probabilities into shared memory, row sum
+        sm.part_max[ch][r] = m;
+        named_barrier(1, kSoftmaxThreads);
+        m = fmaxf(sm.part_max[0][r], sm.part_max[1][r]);
+        // pass 2: probabilities into shared memory, partial row sums
+        float l = 0.f;
 #pragma unroll 1
-        for (int c0 = 0; c0 < kSmallK; c0 += 32) {
+        for (int c0 = cb; c0 < cb + 64; c0 += 32) {
             float t32[32];
             tmem_ld32(tS + lane_off + c0, t32);
 #pragma unroll
@@ -932,27 +945,39 @@ __global__ void __launch_bounds__(kThreads, 1) attn_fwd_small_kernel(const __gri
             }
             write_pair32(sm.p, r, c0, t32);
         }
+        sm.part_sum[ch][r] = l;
         fence_proxy_async();
         tc_fence_before();
         mbar_arrive(smem_u32(&sm.p_ready));
         ok = mbar_wait(smem_u32(&sm.o_full), 0) && ok;
         tc_fence_after();
-        float o[64];
-        ld64(tO + lane_off, o);
+        named_barrier(1, kSoftmaxThreads);   // partial sums visible
+        l = sm.part_sum[0][r] + sm.part_sum[1][r];
+        float o[32];
+        tmem_ld32(tO + lane_off + 32 * ch, o);   // output columns 32 ch .. 32 ch + 31
         if (!ok) flag_timeout_b(sm, p.status);
-        if (ok && tr.valid && !*(volatile int *)&sm.abort) {
-            const size_t row = (size_t)h * p.Mtok + (size_t)b0 * p.k + r;
-            const float inv = 1.f / l;
-            const float rr = p.rsel[row];
-            float *arow = p.A + row * 64;
-#pragma unroll
-            for (int c = 0; c < 64; c += 4)
-                *reinterpret_cast<float4 *>(arow + c) =
-                    make_float4(o[c] * inv, o[c + 1] * inv, o[c + 2] * inv, o[c + 3] * inv);
-#pragma unroll
-            for (int c = 0; c < 64; ++c) o[c] *= rr * inv;
-            store_pair64(p.AR + row * 128, 0, 64, o, 1.f);
-            p.lse[row] = (m + log2f(l)) * 0.69314718055994531f;
+        const bool live = __all_sync(0xffffffffu, ok && !*(volatile int *)&sm.abort);
+        const unsigned vmask = __ballot_sync(0xffffffffu, tr.valid);
+        const size_t row0 = (size_t)h * p.Mtok + (size_t)b0 * p.k + q * 32;   // global row of lane 0
+        if (live) {
+            // Q tile is free once S is done: 4 KB of staging per softmax warp
+            uint8_t *xb = sm.q[0] + (warp - 4) * 4096;
+            const float inv = tr.valid ? 1.f / l : 0.f;
+            stage_f32x32(xb, o, inv, lane);
+            store_rows128(xb, lane, [&](int rl, int c) -> uint4 * {
+                if (!((vmask >> rl) & 1u)) return nullptr;
+                return reinterpret_cast<uint4 *>(p.A + (row0 + rl) * 64 + 32 * ch) + c;
+            });
+            const float rr = tr.valid ? p.rsel[row0 + lane] : 0.f;
+            stage_pair32(xb, o, inv * rr, lane);
+            store_rows128(xb, lane, [&](int rl, int c) -> uint4 * {
+                if (!((vmask >> rl) & 1u)) return nullptr;
+                bf16 *base = p.AR + (row0 + rl) * 128 + 32 * ch;
+                return c < 4 ? reinterpret_cast<uint4 *>(base) + c
+                             : reinterpret_cast<uint4 *>(base + 64) + (c - 4);
+            });
+            // lse in natural-log units of the scaled scores
+            if (ch == 0 && tr.valid) p.lse[row0 + lane] = (m + log2f(l)) * 0.69314718055994531f;
         }
     }
     tc_fence_before();
@@ -963,7 +988,7 @@ __global__ void __launch_bounds__(kThreads, 1) attn_fwd_small_kernel(const __gri
     }
 }
 
-__global__ void __launch_bounds__(kThreads, 1) attn_bwd_small_kernel(const __grid_constant__ BwdParams p) {
+__global__ void __launch_bounds__(kSmallThreads, 1) attn_bwd_small_kernel(const __grid_constant__ BwdParams p) {
     extern __shared__ uint8_t smem_raw[];
     SmallBwdSmem &sm = *reinterpret_cast<SmallBwdSmem *>(
         (reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
@@ -972,9 +997,9 @@ __global__ void __launch_bounds__(kThreads, 1) attn_bwd_small_kernel(const __gri
     if (threadIdx.x == 0) {
         mbar_init(smem_u32(&sm.in_full), 1);
         mbar_init(smem_u32(&sm.sp_full), 1);
-        mbar_init(smem_u32(&sm.p_ready), 128);
+        mbar_init(smem_u32(&sm.p_ready), kSoftmaxThreads);
         mbar_init(smem_u32(&sm.pv_done), 1);
-        mbar_init(smem_u32(&sm.ds_ready), 128);
+        mbar_init(smem_u32(&sm.ds_ready), kSoftmaxThreads);
         mbar_init(smem_u32(&sm.acc_done), 1);
         sm.abort = 0;
         fence_barrier_init();
@@ -1038,8 +1063,9 @@ __global__ void __launch_bounds__(kThreads, 1) attn_bwd_small_kernel(const __gri
         }
     } else if (warp >= 4) {
         pdl_trigger();
-        const int q = warp - 4;
+        const int q = warp & 3, ch = (warp - 4) >> 2;
         const int r = q * 32 + lane;   // query row i for S/dP/dQ; key row j for dK/dV
+        const int cb = 64 * ch;        // this thread's 64 keys
         const uint32_t lane_off = (uint32_t)(q * 32) << 16;
         const size_t base = (size_t)h * p.Mtok + (size_t)b0 * p.k;
         const TileRow tr = tile_row(r, p.k, p.U, b0, p.B);
@@ -1051,7 +1077,7 @@ __global__ void __launch_bounds__(kThreads, 1) attn_bwd_small_kernel(const __gri
         tc_fence_after();
         // P
 #pragma unroll 1
-        for (int c0 = 0; c0 < kSmallK; c0 += 32) {
+        for (int c0 = cb; c0 < cb + 64; c0 += 32) {
             float t32[32];
             tmem_ld32(tS + lane_off + c0, t32);
 #pragma unroll
@@ -1065,7 +1091,7 @@ __global__ void __launch_bounds__(kThreads, 1) attn_bwd_small_kernel(const __gri
         ok = mbar_wait(smem_u32(&sm.pv_done), 0) && ok;   // P read by dV: overwrite with dS
         tc_fence_after();
 #pragma unroll 1
-        for (int c0 = 0; c0 < kSmallK; c0 += 32) {
+        for (int c0 = cb; c0 < cb + 64; c0 += 32) {
             float t32[32], d32[32];
             tmem_ld32(tS + lane_off + c0, t32);
             tmem_ld32(tDP + lane_off + c0, d32);
@@ -1081,16 +1107,26 @@ __global__ void __launch_bounds__(kThreads, 1) attn_bwd_small_kernel(const __gri
         mbar_arrive(smem_u32(&sm.ds_ready));
         ok = mbar_wait(smem_u32(&sm.acc_done), 0) && ok;
         tc_fence_after();
-        float dv[64], dk[64], dq[64];
-        ld64(tDV + lane_off, dv);
-        ld64(tDK + lane_off, dk);
-        ld64(tDQ + lane_off, dq);
         if (!ok) flag_timeout_b(sm, p.status);
-        if (ok && valid && !*(volatile int *)&sm.abort) {
-            bf16 *row = p.dQKV + (base + r) * 512;
-            store_pair64(row, 0, 256, dq, p.scale);
-            store_pair64(row, 64, 320, dk, p.scale);
-            store_pair64(row, 128, 384, dv, 1.f);
+        const bool live = __all_sync(0xffffffffu, ok && !*(volatile int *)&sm.abort);
+        const unsigned vmask = __ballot_sync(0xffffffffu, valid);
+        // dQ, dK, dV columns 32 ch .. +31 as bf16 pairs in the dQKV row layout
+        // (hi at column off + 32 ch, lo 256 further); the Q tile is free by now
+        uint8_t *xb = sm.q[0] + (warp - 4) * 4096;
+        const uint32_t src[3] = {tDQ, tDK, tDV};
+        const float fac[3] = {p.scale, p.scale, 1.f};
+#pragma unroll 1
+        for (int t = 0; t < 3; ++t) {
+            float v[32];
+            tmem_ld32(src[t] + lane_off + 32 * ch, v);
+            if (!live) continue;
+            stage_pair32(xb, v, fac[t], lane);
+            store_rows128(xb, lane, [&](int rl, int c) -> uint4 * {
+                if (!((vmask >> rl) & 1u)) return nullptr;
+                bf16 *row = p.dQKV + (base + q * 32 + rl) * 512 + 64 * t + 32 * ch;
+                return c < 4 ? reinterpret_cast<uint4 *>(row) + c
+                             : reinterpret_cast<uint4 *>(row + 256) + (c - 4);
+            });
         }
     }
     tc_fence_before();
@@ -1153,7 +1189,7 @@ cudaError_t tc_attn_fwd(const Dims &dm, const Saved &sv, cudaStream_t s) {
     if (attr != cudaSuccess) return attr;
     if (small) {
         cudaError_t e = launch_pdl(attn_fwd_small_kernel, dim3(1, (dm.B + p.U - 1) / p.U, dm.H),
-                                   dim3(kThreads), kSmallFwdSmem, s, p);
+                                   dim3(kSmallThreads), kSmallFwdSmem, s, p);
         note_launches(1);
         return e;
     }
@@ -1193,7 +1229,7 @@ cudaError_t tc_attn_bwd(const Dims &dm, const Saved &sv, cudaStream_t s) {
         });
         if (attr_small != cudaSuccess) return attr_small;
         cudaError_t e = launch_pdl(attn_bwd_small_kernel, dim3(1, (dm.B + sp.U - 1) / sp.U, dm.H),
-                                   dim3(kThreads), kSmallBwdSmem, s, sp);
+                                   dim3(kSmallThreads), kSmallBwdSmem, s, sp);
         note_launches(1);
         return e;
     }

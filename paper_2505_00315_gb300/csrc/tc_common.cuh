@@ -209,6 +209,64 @@ __host__ __device__ constexpr uint32_t idesc_bf16(int M, int N, bool a_mn_major,
            | ((uint32_t)(M >> 4) << 24);
 }
 
+// ------------------------------------------------------ epilogue staging
+// A warp stages 32 rows of 128 bytes, one row per lane (16-byte unit c of row r
+// at r*128 + ((c ^ (r & 7)) << 4), free of bank conflicts), then copies them
+// out with 8 lanes per row, so each store instruction covers four whole
+// 128-byte rows or eight 64-byte halves.
+__device__ __forceinline__ uint32_t xoff128(int r, int c) {
+    return (uint32_t)(r * 128 + ((c ^ (r & 7)) << 4));
+}
+
+// 32 fp32 values v * f of this lane's row.
+__device__ __forceinline__ void stage_f32x32(uint8_t *xb, const float *v, float f, int lane) {
+#pragma unroll
+    for (int c = 0; c < 8; ++c)
+        *reinterpret_cast<float4 *>(xb + xoff128(lane, c)) =
+            make_float4(v[4 * c] * f, v[4 * c + 1] * f, v[4 * c + 2] * f, v[4 * c + 3] * f);
+    __syncwarp();
+}
+
+// 32 values v * f of this lane's row as a bf16 pair: hi in units 0..3, lo in 4..7.
+__device__ __forceinline__ void stage_pair32(uint8_t *xb, const float *v, float f, int lane) {
+#pragma unroll
+    for (int u = 0; u < 4; ++u) {
+        uint32_t h4[4], l4[4];
+#pragma unroll
+        for (int e = 0; e < 4; ++e) {
+            const float a = v[8 * u + 2 * e] * f, b = v[8 * u + 2 * e + 1] * f;
+            const __nv_bfloat16 ha = __float2bfloat16_rn(a), hb = __float2bfloat16_rn(b);
+            const __nv_bfloat16 la = __float2bfloat16_rn(a - __bfloat162float(ha));
+            const __nv_bfloat16 lb = __float2bfloat16_rn(b - __bfloat162float(hb));
+            h4[e] = (uint32_t)__bfloat16_as_ushort(ha) | ((uint32_t)__bfloat16_as_ushort(hb) << 16);
+            l4[e] = (uint32_t)__bfloat16_as_ushort(la) | ((uint32_t)__bfloat16_as_ushort(lb) << 16);
+        }
+        *reinterpret_cast<uint4 *>(xb + xoff128(lane, u)) = make_uint4(h4[0], h4[1], h4[2], h4[3]);
+        *reinterpret_cast<uint4 *>(xb + xoff128(lane, 4 + u)) = make_uint4(l4[0], l4[1], l4[2], l4[3]);
+    }
+    __syncwarp();
+}
+
+// Copies the staged rows out: addr(rl, c) is the destination of unit c of row
+// rl, or nullptr to skip the row.
+template <typename F>
+__device__ __forceinline__ void store_rows128(const uint8_t *xb, int lane, F addr) {
+    const int c = lane & 7;
+#pragma unroll
+    for (int i = 0; i < 8; ++i) {
+        const int rl = (lane >> 3) + 4 * i;
+        const uint4 val = *reinterpret_cast<const uint4 *>(xb + xoff128(rl, c));
+        uint4 *d = addr(rl, c);
+        if (d != nullptr) *d = val;
+    }
+    __syncwarp();
+}
+
+// Barrier among the `count` threads of the warps that use the given id (1..15).
+__device__ __forceinline__ void named_barrier(int id, int count) {
+    asm volatile("bar.sync %0, %1;" ::"r"(id), "r"(count) : "memory");
+}
+
 // ------------------------------------------------------- global reductions
 __device__ __forceinline__ void red_add_v4(float *addr, float a, float b, float c, float d) {
     asm volatile("red.global.add.v4.f32 [%0], {%1, %2, %3, %4};" ::"l"(addr), "f"(a), "f"(b),

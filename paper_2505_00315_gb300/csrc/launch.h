@@ -83,6 +83,12 @@ bool tc_supported(const Dims &dm);
 // True when the tensor-core kernels serve this shape (false also when the
 // environment variable MOSA_FORCE_SIMT is set to a non-zero value).
 bool use_tc(const Dims &dm);
+// Fused F3 + F4 + F5 for k <= 128 (tc_fused_fwd.cu); off with MOSA_FUSED_FWD=0.
+bool tc_fused_forward_supported(const Dims &dm);
+bool use_fused_forward(const Dims &dm);
+cudaError_t tc_fused_forward(const Dims &dm, const void *X, const void *Wq, const void *Wk,
+                             const void *Wv, const void *Wo, const Saved &sv, float *Y,
+                             cudaStream_t s);
 cudaError_t tc_qkv(const Dims &dm, const void *X, const void *Wq, const void *Wk, const void *Wv,
                    const Saved &sv, cudaStream_t s);
 // zero_output = false: the caller has already zeroed Y / dX on this stream's timeline.

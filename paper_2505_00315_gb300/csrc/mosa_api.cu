@@ -158,6 +158,12 @@ mosa_status forward_tc(const Dims &dm, const void *X, const void *W_r, const voi
         StageScope st_(kStageSelect, s);
         MOSA_TRY(launch_indices_to_rows(dm, I_in, rsel_in, sv.gidx, sv.rsel, sv.status, s));
     }
+    if (use_fused_forward(dm)) {
+        MOSA_TRY(link(r.side, s, r.ev[1]));  // Y zeroed
+        StageScope st_(kStageFwdUnit, s);
+        MOSA_TRY(tc_fused_forward(dm, X, W_q, W_k, W_v, W_o, sv, Y, s));
+        return MOSA_OK;
+    }
     {
         StageScope st_(kStageQkv, s);
         MOSA_TRY(launch_qkv(dm, X, W_q, W_k, W_v, sv, s));
@@ -255,7 +261,7 @@ GraphKey make_key(int op, const Dims &dm, const mosa_shape *shape,
     std::memset(&k, 0, sizeof(k));
     k.op = op;
     cudaGetDevice(&k.device);
-    k.tc = use_tc(dm) ? 1 : 0;
+    k.tc = (use_tc(dm) ? 1 : 0) | (use_fused_forward(dm) ? 2 : 0);
     k.mask = profile_mask();
     k.shape = *shape;
     int i = 0;
@@ -456,6 +462,7 @@ int32_t mosa_stage_engine(const mosa_shape *shape, int32_t stage) {
         case kStageDwo:
         case kStageAttnFwd:
         case kStageAttnBwd: return use_tc(dm) ? 1 : 0;
+        case kStageFwdUnit: return use_fused_forward(dm) ? 1 : 0;
         default: return 0;
     }
 }

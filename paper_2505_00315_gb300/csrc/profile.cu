@@ -27,7 +27,8 @@ double g_ms[kNumStages] = {};
 int32_t g_count[kNumStages] = {};
 
 const char *kNames[kNumStages] = {"router", "select", "qkv", "attn_fwd", "out",
-                                  "out_bwd", "attn_bwd", "in_bwd", "w_bwd", "dwo"};
+                                  "out_bwd", "attn_bwd", "in_bwd", "w_bwd", "dwo",
+                                  "fwd_unit"};
 
 cudaEvent_t take_event() {
     if (!g_free.empty()) {

@@ -9,7 +9,9 @@ namespace mosa {
 
 enum Stage : int {
     kStageRouter = 0, kStageSelect, kStageQkv, kStageAttnFwd, kStageOut,
-    kStageOutBwd, kStageAttnBwd, kStageInBwd, kStageWBwd, kStageDwo, kNumStages
+    kStageOutBwd, kStageAttnBwd, kStageInBwd, kStageWBwd, kStageDwo,
+    kStageFwdUnit,  // F3 + F4 + F5 fused (k <= 128)
+    kNumStages
 };
 
 // Adds n to the library's kernel-launch counter (or, while this thread is

@@ -261,6 +261,12 @@ bool use_tc(const Dims &dm) {
     return tc_supported(dm);
 }
 
+bool use_fused_forward(const Dims &dm) {
+    const char *f = std::getenv("MOSA_FUSED_FWD");
+    if (f != nullptr && f[0] == '0') return false;
+    return use_tc(dm) && tc_fused_forward_supported(dm);
+}
+
 cudaError_t launch_qkv(const Dims &dm, const void *X, const void *Wq, const void *Wk,
                        const void *Wv, const Saved &sv, cudaStream_t s) {
     if (use_tc(dm)) return tc_qkv(dm, X, Wq, Wk, Wv, sv, s);

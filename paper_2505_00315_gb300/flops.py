@@ -84,6 +84,13 @@ def layer_work(B: int, T: int, d: int, H: int, hp: int, k: int, elem_bytes: int 
         "w_bwd": {"flops": (6 * d * hp * k + 2 * d * k) * U,
                   "bytes": U * k * d * e + 3 * U * k * hp * e + 3 * H * d * hp * 4 + d * H * 4},
     }
+    # F3 + F4 + F5 in one kernel (k <= 128): the three steps' FLOPs; bytes as
+    # those steps minus the Q/K/V and scaled-A round trips they no longer make
+    # (Q/K/V, A, AR and lse are still written once for the backward)
+    w["fwd_unit"] = {"flops": w["qkv"]["flops"] + w["attn_fwd"]["flops"] + w["out"]["flops"],
+                     "bytes": U * k * d * e + 3 * H * d * hp * e + H * hp * d * e
+                              + 3 * U * k * hp * e + 2 * U * k * hp * e + U * k * 4
+                              + U * k * d * 4}
     fwd = ("router", "select", "qkv", "attn_fwd", "out")
     bwd = ("out_bwd", "dwo", "attn_bwd", "in_bwd", "w_bwd")
     w["forward_flops"] = sum(w[s]["flops"] for s in fwd)

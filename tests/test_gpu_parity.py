@@ -77,14 +77,17 @@ SMALL = [
 ]
 
 
-@pytest.fixture(params=["default", "simt"])
+@pytest.fixture(params=["default", "unfused", "simt"])
 def kernel_path(request, monkeypatch):
-    """Run a test on the default kernels (tensor cores where the shape allows)
-    and again with the CUDA-core kernels forced."""
+    """Run a test on the default kernels (tensor cores where the shape allows,
+    the fused forward for k <= 128), again with the forward as three separate
+    kernels, and again with the CUDA-core kernels forced."""
+    monkeypatch.delenv("MOSA_FORCE_SIMT", raising=False)
+    monkeypatch.delenv("MOSA_FUSED_FWD", raising=False)
     if request.param == "simt":
         monkeypatch.setenv("MOSA_FORCE_SIMT", "1")
-    else:
-        monkeypatch.delenv("MOSA_FORCE_SIMT", raising=False)
+    elif request.param == "unfused":
+        monkeypatch.setenv("MOSA_FUSED_FWD", "0")
     return request.param
 
 

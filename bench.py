@@ -170,7 +170,7 @@ def cpu_baseline(cfg, x, budget_s):
 # ------------------------------------------------------------ roofline
 
 STAGES = ["router", "select", "qkv", "attn_fwd", "out", "out_bwd", "attn_bwd", "in_bwd",
-          "w_bwd", "dwo", "fwd_unit"]
+          "w_bwd", "dwo", "fwd_unit", "bwd_unit"]
 
 
 def stage_bound(stage, peaks, kind):
@@ -213,7 +213,7 @@ KERNEL_STAGE = [("tc_gemm_kernel<6>", "router"), ("tc_gemm_kernel<(int)6>", "rou
                 ("tc_gemm_kernel<4>", "in_bwd"), ("tc_gemm_kernel<(int)4>", "in_bwd"),
                 ("tc_gemm_kernel<5>", "w_bwd"), ("tc_gemm_kernel<(int)5>", "w_bwd"),
                 ("tc_gemm_kernel<3>", "dwo"), ("tc_gemm_kernel<(int)3>", "dwo"),
-                ("fused_fwd_kernel", "fwd_unit")]
+                ("fused_fwd_kernel", "fwd_unit"), ("fused_bwd_kernel", "bwd_unit")]
 
 
 def ingest_ncu(csv_path, cfg_name):

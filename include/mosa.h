@@ -33,10 +33,17 @@
  *     on an internal stream of the current device.  Up to 128 graphs are kept
  *     (driver resources, no user memory); further new calls run unrecorded.
  *     Setting the environment variable MOSA_GRAPHS=0 turns this off.
+ *   - Kernel paths (environment, read at every call): MOSA_FORCE_SIMT=1 runs
+ *     the CUDA-core kernels only; MOSA_FUSED_FWD=0 runs the k <= 128 forward
+ *     as three kernels (projection, attention, output) instead of one fused
+ *     kernel; MOSA_FUSED_BWD=1 runs the k <= 128 backward's G, row terms and
+ *     attention backward as one fused kernel; MOSA_PDL=0 turns programmatic
+ *     dependent launch off.  All paths compute the same operation.
  *   - Outputs are overwritten, never accumulated into.
- *   - Arithmetic: fp32 accumulation everywhere; with bf16 storage the saved
- *     intermediates (Q, K, V, attention output, gradients fed to tensor-core
- *     products) are rounded to bf16.
+ *   - Arithmetic: fp32 accumulation everywhere; with bf16 storage the
+ *     intermediates fed to tensor-core products (Q, K, V, P, the attention
+ *     output, dA, dS, dQ|dK|dV) are kept as bf16 hi/lo pairs (v ~ hi + lo),
+ *     which keeps those products at fp32-level accuracy.
  *   - Tokens tied on the router score are taken lowest index first.
  *   - NaN inputs give undefined results (but no out-of-bounds access).
  *   - Errors: a call that returns anything but MOSA_OK has launched nothing.

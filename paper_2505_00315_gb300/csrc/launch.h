@@ -89,6 +89,12 @@ bool use_fused_forward(const Dims &dm);
 cudaError_t tc_fused_forward(const Dims &dm, const void *X, const void *Wq, const void *Wk,
                              const void *Wv, const void *Wo, const Saved &sv, float *Y,
                              cudaStream_t s);
+// Fused G / row terms + attention backward (+ dX) for k <= 128 (tc_fused_bwd.cu);
+// opt-in with MOSA_FUSED_BWD=1.  Needs the fp32 W_r transpose and dX zeroed.
+bool use_fused_backward(const Dims &dm);
+cudaError_t tc_fused_backward(const Dims &dm, const void *W_q, const void *W_k, const void *W_v,
+                              const void *W_o, const void *dY, const Saved &sv, float *dX,
+                              bool with_dx, cudaStream_t s);
 cudaError_t tc_qkv(const Dims &dm, const void *X, const void *Wq, const void *Wk, const void *Wv,
                    const Saved &sv, cudaStream_t s);
 // zero_output = false: the caller has already zeroed Y / dX on this stream's timeline.

@@ -190,6 +190,29 @@ mosa_status backward_tc(const Dims &dm, const void *X, const void *W_r, const vo
     MOSA_TRY(tc_transpose_wr(dm, W_r, sv, t));
     MOSA_TRY(cudaMemsetAsync(dX, 0, sizeof(float) * (size_t)dm.B * dm.T * dm.d, t));
     MOSA_TRY(link(t, s, r.ev[1]));  // dX zeroed and W_r transposed before the dX product
+    if (use_fused_backward(dm)) {
+        // The fused kernel (G, row terms, attention backward) holds a whole SM
+        // per CTA, so nothing runs beside it; dX, dW and dW_o then share the GPU.
+        {
+            StageScope st_(kStageBwdUnit, s);
+            MOSA_TRY(tc_fused_backward(dm, W_q, W_k, W_v, W_o, dY, sv, dX, false, s));
+        }
+        MOSA_TRY(link(s, t, r.ev[2]));  // dQ|dK|dV|dlogit ready
+        {
+            StageScope st_(kStageDwo, t);
+            MOSA_TRY(tc_out_bwd_w(dm, dY, sv, dW_o, t));
+        }
+        {
+            StageScope st_(kStageWBwd, t);
+            MOSA_TRY(tc_w_bwd(dm, X, sv, dW_q, dW_k, dW_v, dW_r, t));
+        }
+        {
+            StageScope st_(kStageInBwd, s);
+            MOSA_TRY(tc_in_bwd(dm, W_q, W_k, W_v, W_r, sv, dX, s, false));
+        }
+        MOSA_TRY(link(t, s, r.ev[3]));  // join
+        return MOSA_OK;
+    }
     {
         StageScope st_(kStageDwo, t);
         MOSA_TRY(tc_out_bwd_w(dm, dY, sv, dW_o, t));
@@ -261,7 +284,7 @@ GraphKey make_key(int op, const Dims &dm, const mosa_shape *shape,
     std::memset(&k, 0, sizeof(k));
     k.op = op;
     cudaGetDevice(&k.device);
-    k.tc = (use_tc(dm) ? 1 : 0) | (use_fused_forward(dm) ? 2 : 0);
+    k.tc = (use_tc(dm) ? 1 : 0) | (use_fused_forward(dm) ? 2 : 0) | (use_fused_backward(dm) ? 4 : 0);
     k.mask = profile_mask();
     k.shape = *shape;
     int i = 0;
@@ -463,6 +486,7 @@ int32_t mosa_stage_engine(const mosa_shape *shape, int32_t stage) {
         case kStageAttnFwd:
         case kStageAttnBwd: return use_tc(dm) ? 1 : 0;
         case kStageFwdUnit: return use_fused_forward(dm) ? 1 : 0;
+        case kStageBwdUnit: return use_fused_backward(dm) ? 1 : 0;
         default: return 0;
     }
 }

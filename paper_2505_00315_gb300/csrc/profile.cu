@@ -28,7 +28,7 @@ int32_t g_count[kNumStages] = {};
 
 const char *kNames[kNumStages] = {"router", "select", "qkv", "attn_fwd", "out",
                                   "out_bwd", "attn_bwd", "in_bwd", "w_bwd", "dwo",
-                                  "fwd_unit"};
+                                  "fwd_unit", "bwd_unit"};
 
 cudaEvent_t take_event() {
     if (!g_free.empty()) {

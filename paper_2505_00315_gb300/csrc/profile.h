@@ -11,6 +11,7 @@ enum Stage : int {
     kStageRouter = 0, kStageSelect, kStageQkv, kStageAttnFwd, kStageOut,
     kStageOutBwd, kStageAttnBwd, kStageInBwd, kStageWBwd, kStageDwo,
     kStageFwdUnit,  // F3 + F4 + F5 fused (k <= 128)
+    kStageBwdUnit,  // B1 (G, row terms) + B2 fused (k <= 128)
     kNumStages
 };
 

@@ -27,6 +27,7 @@
 #include "launch.h"
 #include "profile.h"
 #include "tc_common.cuh"
+#include "tc_tiles.cuh"
 #include "tmap.h"
 
 namespace mosa {
@@ -389,23 +390,6 @@ __device__ __forceinline__ void flag_timeout_b(SM &sm, uint32_t *status) {
     *(volatile int *)&sm.abort = 1;
 }
 
-// Three split products D (+)= Ah Bh + Ah Bl + Al Bh over K = 64.
-__device__ __forceinline__ void mma_pair3(uint32_t d, uint32_t a_hi, uint32_t a_lo, uint32_t b_hi,
-                                          uint32_t b_lo, bool a_mn, bool b_mn, uint32_t idesc,
-                                          bool accumulate_first) {
-    const uint32_t aa[3] = {a_hi, a_hi, a_lo}, bb[3] = {b_hi, b_lo, b_hi};
-#pragma unroll
-    for (int t = 0; t < 3; ++t)
-#pragma unroll
-        for (int kk = 0; kk < 4; ++kk) {
-            const uint64_t ad = a_mn ? smem_desc_sw128(aa[t] + kk * 2048, 8192, 1024)
-                                     : smem_desc_sw128(aa[t] + kk * 32, 16, 1024);
-            const uint64_t bd = b_mn ? smem_desc_sw128(bb[t] + kk * 2048, 8192, 1024)
-                                     : smem_desc_sw128(bb[t] + kk * 32, 16, 1024);
-            mma_bf16(d, ad, bd, idesc, (accumulate_first || t > 0 || kk > 0) ? 1u : 0u);
-        }
-}
-
 __device__ __forceinline__ void ld64(uint32_t taddr, float *v) {
     float t32[32];
     tmem_ld32(taddr, t32);
@@ -754,7 +738,7 @@ __global__ void __launch_bounds__(kThreads, 1) attn_dq_tc_kernel(const __grid_co
 // P^T / dS^T for dV and dK.
 
 constexpr int kSmallK = 128;
-constexpr int kPBig = 128 * 64 * 2;   // one 64-key block of a 128-row tile, one half: 16 KB
+constexpr int kPBig = kTileHalf;   // one 64-key block of a 128-row tile, one half: 16 KB
 
 struct SmallFwdSmem {
     uint8_t q[2][kPBig];
@@ -779,64 +763,6 @@ struct SmallBwdSmem {
     int abort;
 };
 constexpr int kSmallBwdSmem = (int)sizeof(SmallBwdSmem) + 1024;
-
-// Tile row r (query or key) of the sequences b0 .. b0+U-1: valid when it lies in
-// one of them; lo is the first tile row of its sequence (keys c with
-// lo <= c <= r are visible from query r).
-struct TileRow {
-    bool valid;
-    int lo;
-};
-__device__ __forceinline__ TileRow tile_row(int r, int k, int U, int b0, int B) {
-    const int u = r / k;
-    return TileRow{u < U && b0 + u < B, u * k};
-}
-
-// 32 consecutive keys c0..c0+31 of row r of a [128 x 128] pair tile.
-__device__ __forceinline__ void write_pair32(uint8_t (*tile)[2][kPBig], int r, int c0, const float *v) {
-    const int blk = c0 >> 6, cb = (c0 & 63) >> 3;  // 16-byte chunk index within the 128-byte row
-#pragma unroll
-    for (int c = 0; c < 4; ++c) {
-        uint32_t h4[4], l4[4];
-#pragma unroll
-        for (int e = 0; e < 4; ++e) {
-            const float a = v[c * 8 + 2 * e], b = v[c * 8 + 2 * e + 1];
-            const bf16 ha = __float2bfloat16_rn(a), hb = __float2bfloat16_rn(b);
-            const bf16 la = __float2bfloat16_rn(a - __bfloat162float(ha));
-            const bf16 lb = __float2bfloat16_rn(b - __bfloat162float(hb));
-            h4[e] = (uint32_t)__bfloat16_as_ushort(ha) | ((uint32_t)__bfloat16_as_ushort(hb) << 16);
-            l4[e] = (uint32_t)__bfloat16_as_ushort(la) | ((uint32_t)__bfloat16_as_ushort(lb) << 16);
-        }
-        const int off = r * 128 + (((cb + c) ^ (r & 7)) << 4);
-        *reinterpret_cast<uint4 *>(tile[0][blk] + off) = make_uint4(h4[0], h4[1], h4[2], h4[3]);
-        *reinterpret_cast<uint4 *>(tile[1][blk] + off) = make_uint4(l4[0], l4[1], l4[2], l4[3]);
-    }
-}
-
-// D (+)= A B over K = 128 with A a [128 x 128] pair tile (two 64-wide blocks)
-// and B a pair of 128-row tiles, three split products each.
-//   a_mn = false: A K-major, K = tile columns (P V, dS K)
-//   a_mn = true:  A read as its transpose (P^T dA, dS^T Q), K = tile rows
-__device__ __forceinline__ void mma_k128(uint32_t d, const uint8_t (*a)[2][kPBig],
-                                         const uint8_t (*b)[kPBig], bool a_mn, uint32_t idesc) {
-#pragma unroll
-    for (int t = 0; t < 3; ++t) {
-        const int ah = t == 2 ? 1 : 0, bh = t == 1 ? 1 : 0;
-#pragma unroll
-        for (int kk = 0; kk < 8; ++kk) {
-            uint64_t ad, bd;
-            if (a_mn) {
-                // rows kk*16.. of both key blocks; next 64-wide M block 16 KB on
-                ad = smem_desc_sw128(smem_u32(a[ah][0]) + kk * 2048, kPBig, 1024);
-            } else {
-                ad = smem_desc_sw128(smem_u32(a[ah][kk >> 2]) + (kk & 3) * 32, 16, 1024);
-            }
-            // B rows = K index (MN-major B: 64-wide N block, 16 rows per step)
-            bd = smem_desc_sw128(smem_u32(b[bh]) + kk * 2048, kPBig, 1024);
-            mma_bf16(d, ad, bd, idesc, (t > 0 || kk > 0) ? 1u : 0u);
-        }
-    }
-}
 
 // Threads of the k <= 128 kernels: warps 0-3 load, issue MMAs and own TMEM;
 // warps 4-11 run the softmax passes and the epilogue, two per TMEM lane

@@ -28,6 +28,7 @@
 #include "launch.h"
 #include "profile.h"
 #include "tc_common.cuh"
+#include "tc_tiles.cuh"
 #include "tmap.h"
 
 namespace mosa {
@@ -38,7 +39,7 @@ using namespace tc;
 constexpr int kThreads = 384;
 constexpr int kWorkers = 256;            // warps 4-11
 constexpr int kStages = 3;
-constexpr int kHalf = 128 * 64 * 2;      // one hi or lo half of a 128 x 64 tile: 16 KB
+constexpr int kHalf = kTileHalf;         // one hi or lo half of a 128 x 64 tile: 16 KB
 constexpr int kStageBytes = kHalf + 3 * 8192;   // gathered X block + W_q|W_k|W_v blocks
 constexpr int kChunk = 256;              // output columns per phase-4 chunk
 
@@ -84,31 +85,6 @@ __device__ __forceinline__ bool wait_or_abort(FusedSmem &sm, uint64_t &bar, uint
     atomicOr(status, kStatusTimeout);
     *(volatile int *)&sm.abort = 1;
     return false;
-}
-
-// 32 values v[0..31] as columns c0 .. c0+31 of row r of a K-major, 128-byte
-// swizzled pair tile made of 64-column blocks of kHalf bytes per half:
-// tile(half, block) = base + (block * 2 + half) * kHalf  when interleaved
-// [block][half], or the caller's own addressing through hi / lo pointers.
-__device__ __forceinline__ void put_pair32(uint8_t *hi_blk, uint8_t *lo_blk, int r, int c0,
-                                           const float *v, float f) {
-    const int cb = (c0 & 63) >> 3;  // first 16-byte unit within the 128-byte row
-#pragma unroll
-    for (int c = 0; c < 4; ++c) {
-        uint32_t h4[4], l4[4];
-#pragma unroll
-        for (int e = 0; e < 4; ++e) {
-            const float a = v[c * 8 + 2 * e] * f, b = v[c * 8 + 2 * e + 1] * f;
-            const bf16 ha = __float2bfloat16_rn(a), hb = __float2bfloat16_rn(b);
-            const bf16 la = __float2bfloat16_rn(a - __bfloat162float(ha));
-            const bf16 lb = __float2bfloat16_rn(b - __bfloat162float(hb));
-            h4[e] = (uint32_t)__bfloat16_as_ushort(ha) | ((uint32_t)__bfloat16_as_ushort(hb) << 16);
-            l4[e] = (uint32_t)__bfloat16_as_ushort(la) | ((uint32_t)__bfloat16_as_ushort(lb) << 16);
-        }
-        const int off = r * 128 + (((cb + c) ^ (r & 7)) << 4);
-        *reinterpret_cast<uint4 *>(hi_blk + off) = make_uint4(h4[0], h4[1], h4[2], h4[3]);
-        *reinterpret_cast<uint4 *>(lo_blk + off) = make_uint4(l4[0], l4[1], l4[2], l4[3]);
-    }
 }
 
 __global__ void __launch_bounds__(kThreads, 1) fused_fwd_kernel(const __grid_constant__ FusedParams p) {

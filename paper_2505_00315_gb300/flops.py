@@ -91,6 +91,11 @@ def layer_work(B: int, T: int, d: int, H: int, hp: int, k: int, elem_bytes: int 
                      "bytes": U * k * d * e + 3 * H * d * hp * e + H * hp * d * e
                               + 3 * U * k * hp * e + 2 * U * k * hp * e + U * k * 4
                               + U * k * d * 4}
+    # B1 (G and row terms) + B2 in one kernel (k <= 128): the two steps' FLOPs;
+    # bytes: gathered dY, W_o, A, Q/K/V in, dQ|dK|dV out
+    w["bwd_unit"] = {"flops": w["out_bwd"]["flops"] + w["attn_bwd"]["flops"],
+                     "bytes": U * k * d * e + H * hp * d * e + U * k * hp * 4 + 3 * U * k * hp * e
+                              + 3 * U * k * hp * e}
     fwd = ("router", "select", "qkv", "attn_fwd", "out")
     bwd = ("out_bwd", "dwo", "attn_bwd", "in_bwd", "w_bwd")
     w["forward_flops"] = sum(w[s]["flops"] for s in fwd)

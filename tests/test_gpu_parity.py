@@ -77,17 +77,21 @@ SMALL = [
 ]
 
 
-@pytest.fixture(params=["default", "unfused", "simt"])
+@pytest.fixture(params=["default", "unfused", "fused_bwd", "simt"])
 def kernel_path(request, monkeypatch):
     """Run a test on the default kernels (tensor cores where the shape allows,
     the fused forward for k <= 128), again with the forward as three separate
-    kernels, and again with the CUDA-core kernels forced."""
+    kernels, again with the fused backward switched on, and again with the
+    CUDA-core kernels forced."""
     monkeypatch.delenv("MOSA_FORCE_SIMT", raising=False)
     monkeypatch.delenv("MOSA_FUSED_FWD", raising=False)
+    monkeypatch.delenv("MOSA_FUSED_BWD", raising=False)
     if request.param == "simt":
         monkeypatch.setenv("MOSA_FORCE_SIMT", "1")
     elif request.param == "unfused":
         monkeypatch.setenv("MOSA_FUSED_FWD", "0")
+    elif request.param == "fused_bwd":
+        monkeypatch.setenv("MOSA_FUSED_BWD", "1")
     return request.param
 
 

@@ -11,13 +11,15 @@
 
 namespace mosa {
 
-// Launches `kernel` with programmatic stream serialization (it may begin while
-// the preceding kernel on the stream finishes; the kernel itself waits with
-// griddepcontrol.wait before reading that kernel's results).  MOSA_PDL=0
-// launches it plainly.
+// Launches `kernel` with programmatic stream serialization when `early` (it
+// may begin while the preceding kernel on the stream finishes; the kernel
+// itself waits with griddepcontrol.wait before reading that kernel's results).
+// A kernel that shares the GPU with another stream's kernel is launched late
+// instead: waiting early, its CTAs would hold SMs the other kernel needs.
+// MOSA_PDL=0 launches every kernel plainly.
 template <class... KArgs, class... Args>
-inline cudaError_t launch_pdl(void (*kernel)(KArgs...), dim3 grid, dim3 block, size_t smem,
-                              cudaStream_t s, Args &&...args) {
+inline cudaError_t launch_ex(bool early, void (*kernel)(KArgs...), dim3 grid, dim3 block,
+                             size_t smem, cudaStream_t s, Args &&...args) {
     const char *v = std::getenv("MOSA_PDL");
     cudaLaunchConfig_t cfg = {};
     cfg.gridDim = grid;
@@ -28,8 +30,13 @@ inline cudaError_t launch_pdl(void (*kernel)(KArgs...), dim3 grid, dim3 block, s
     attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
     attr[0].val.programmaticStreamSerializationAllowed = 1;
     cfg.attrs = attr;
-    cfg.numAttrs = (v != nullptr && v[0] == '0') ? 0 : 1;
+    cfg.numAttrs = (!early || (v != nullptr && v[0] == '0')) ? 0 : 1;
     return cudaLaunchKernelEx(&cfg, kernel, std::forward<Args>(args)...);
+}
+template <typename... KArgs, typename... Args>
+inline cudaError_t launch_pdl(void (*kernel)(KArgs...), dim3 grid, dim3 block, size_t smem,
+                              cudaStream_t s, Args &&...args) {
+    return launch_ex(true, kernel, grid, block, smem, s, std::forward<Args>(args)...);
 }
 
 // F1, Sec. 2.2 router: r_full[b,h,t] = sigmoid(X[b,t,:] . W_r[:,h]) in fp32.

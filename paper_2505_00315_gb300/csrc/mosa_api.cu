@@ -187,9 +187,14 @@ mosa_status backward_tc(const Dims &dm, const void *X, const void *W_r, const vo
                         float *dW_o, const Saved &sv, cudaStream_t s, DevResources &r) {
     cudaStream_t t = r.side;
     MOSA_TRY(link(s, t, r.ev[0]));
+    if (!use_fused_backward(dm)) {
+        // second stream: dW_o, then what only the dX product needs
+        StageScope st_(kStageDwo, t);
+        MOSA_TRY(tc_out_bwd_w(dm, dY, sv, dW_o, t));
+    }
     MOSA_TRY(tc_transpose_wr(dm, W_r, sv, t));
     MOSA_TRY(cudaMemsetAsync(dX, 0, sizeof(float) * (size_t)dm.B * dm.T * dm.d, t));
-    MOSA_TRY(link(t, s, r.ev[1]));  // dX zeroed and W_r transposed before the dX product
+    MOSA_TRY(cudaEventRecord(r.ev[1], t));  // dX zeroed and W_r transposed
     if (use_fused_backward(dm)) {
         // The fused kernel (G, row terms, attention backward) holds a whole SM
         // per CTA, so nothing runs beside it; dX, dW and dW_o then share the GPU.
@@ -206,16 +211,13 @@ mosa_status backward_tc(const Dims &dm, const void *X, const void *W_r, const vo
             StageScope st_(kStageWBwd, t);
             MOSA_TRY(tc_w_bwd(dm, X, sv, dW_q, dW_k, dW_v, dW_r, t));
         }
+        MOSA_TRY(cudaStreamWaitEvent(s, r.ev[1], 0));
         {
             StageScope st_(kStageInBwd, s);
             MOSA_TRY(tc_in_bwd(dm, W_q, W_k, W_v, W_r, sv, dX, s, false));
         }
         MOSA_TRY(link(t, s, r.ev[3]));  // join
         return MOSA_OK;
-    }
-    {
-        StageScope st_(kStageDwo, t);
-        MOSA_TRY(tc_out_bwd_w(dm, dY, sv, dW_o, t));
     }
     {
         StageScope st_(kStageOutBwd, s);
@@ -230,6 +232,7 @@ mosa_status backward_tc(const Dims &dm, const void *X, const void *W_r, const vo
         StageScope st_(kStageWBwd, t);
         MOSA_TRY(tc_w_bwd(dm, X, sv, dW_q, dW_k, dW_v, dW_r, t));
     }
+    MOSA_TRY(cudaStreamWaitEvent(s, r.ev[1], 0));  // dX zeroed, W_r transposed
     {
         StageScope st_(kStageInBwd, s);
         MOSA_TRY(tc_in_bwd(dm, W_q, W_k, W_v, W_r, sv, dX, s, false));

@@ -723,7 +723,7 @@ bool map_heads(CUtensorMap *m, const void *base, uint64_t H, uint64_t rows, uint
 }
 
 template <int KIND>
-cudaError_t launch_kind(const TcParams &p, dim3 grid, cudaStream_t s) {
+cudaError_t launch_kind(const TcParams &p, dim3 grid, cudaStream_t s, bool early = true) {
     constexpr int smem = smem_bytes<KIND>();
     static std::once_flag once;
     static cudaError_t attr = cudaSuccess;
@@ -732,7 +732,7 @@ cudaError_t launch_kind(const TcParams &p, dim3 grid, cudaStream_t s) {
                                     smem);
     });
     if (attr != cudaSuccess) return attr;
-    cudaError_t e = launch_pdl(tc_gemm_kernel<KIND>, grid, dim3(kThreads), smem, s, p);
+    cudaError_t e = launch_ex(early, tc_gemm_kernel<KIND>, grid, dim3(kThreads), smem, s, p);
     note_launches(1);
     return e;
 }
@@ -906,6 +906,8 @@ cudaError_t tc_in_bwd(const Dims &dm, const void *Wq, const void *Wk, const void
     p.WrT = sv.WrT;
     p.out_f = dX;
     dim3 grid((p.M + kBM - 1) / kBM, (dm.d + 255) / 256, dm.H);
+    // early start: the dW product beside it on the other stream needs all 512
+    // TMEM columns of an SM, so the two cannot share SMs anyway
     return launch_kind<kDX>(p, grid, s);
 }
 

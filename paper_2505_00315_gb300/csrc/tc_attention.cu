@@ -3,12 +3,11 @@
 // Sec. 2.2; with I strictly ascending, I_i >= I_j is j <= i).
 //
 // Forward (F4), one CTA per (128-query tile, sequence b, head h):
-//   for each 64-key block j (causal: up to the tile's last query)
-//     S_j  = Q K_j^T                       tcgen05, fp32 in TMEM
-//     P_j  = exp(S_j/sqrt(h') - m), online max m and sum l per row (4 warps)
-//     O_j  = P_j V_j                       tcgen05, P from shared memory
-//     o    = o * exp(m_old - m_new) + O_j  (registers)
-//   A = o / l, AR = r A, lse = m + log l.
+//   for each 128-key block j (causal: up to the tile's last query)
+//     S_j  = Q K_j^T                       tcgen05, fp32 in TMEM, two buffers
+//     P_j  = exp(S_j/sqrt(h') - m), running max m and sum l per row
+//     O   += P_j V_j                       tcgen05, P from shared memory, O in TMEM
+//   A = O / l, AR = r A, lse = m + log l  (details at the kernel).
 // Q, K, V, P are bf16 hi/lo pairs (v ~ hi + lo), so each product is three
 // bf16 MMAs (hi*hi + hi*lo + lo*hi) into one fp32 accumulator, which keeps the
 // result at fp32-level accuracy.
@@ -20,8 +19,10 @@
 //     S = Q K^T, dP = dA V^T, then dQ += dS K
 // The same shared-memory tile of Q (or dA, K) serves as a K-major operand in
 // one product and as an MN-major operand in the other.
-// Warp roles: 0 TMA producer, 1 MMA issuer, 2 TMEM allocator, 4-7 softmax
-// (one row per thread).  All waits are bounded.
+// Warp roles: 0 TMA producer, 1 MMA issuer, 2 TMEM allocator, then softmax
+// warps (4-7 with one row per thread in the backward kernels, 4-11 with two
+// threads per row in the forward and the k <= 128 kernels).  All waits are
+// bounded.
 #include <mutex>
 
 #include "launch.h"
@@ -38,23 +39,7 @@ using namespace tc;
 constexpr int kQ = 128;          // queries per CTA
 constexpr int kKV = 64;          // keys per block
 constexpr int kThreads = 256;
-constexpr int kQBytes = kQ * 64 * 2;    // one half (hi or lo) of the Q tile, 16 KB
-constexpr int kKVBytes = kKV * 64 * 2;  // one half of a K or V block, 8 KB
-constexpr int kPBytes = kQ * kKV * 2;   // one half of the P tile, 16 KB
 constexpr int kStages = 2;
-
-struct FwdSmem {
-    // all tiles 1024-byte aligned: 128-byte swizzle atoms
-    uint8_t q[2][kQBytes];                   // hi, lo
-    uint8_t k[kStages][2][kKVBytes];
-    uint8_t v[kStages][2][kKVBytes];
-    uint8_t p[2][kPBytes];                   // hi, lo
-    uint64_t q_full, kv_full[kStages], kv_empty[kStages], s_full, o_full, p_ready;
-    uint32_t tmem;
-    int abort;
-};
-
-constexpr int kFwdSmem = (int)sizeof(FwdSmem) + 1024;
 
 struct AttnParams {
     CUtensorMap mQ, mK, mV;   // 4-D maps over [H, B, k, 128] pairs, box {64, rows, 1, 1}
@@ -68,11 +53,6 @@ struct AttnParams {
     float *lse;               // [H, B*k]
     uint32_t *status;
 };
-
-__device__ __forceinline__ void flag_timeout(FwdSmem &sm, uint32_t *status) {
-    atomicOr(status, kStatusTimeout);
-    *(volatile int *)&sm.abort = 1;
-}
 
 // Writes 64 values of one row of a K-major, 128-byte-swizzled bf16 tile as
 // hi and lo halves (row r of a tile whose rows are 128 bytes).
@@ -96,246 +76,243 @@ __device__ __forceinline__ void write_pair_row64(uint8_t *hi_tile, uint8_t *lo_t
     }
 }
 
-__global__ void __launch_bounds__(kThreads, 1) attn_fwd_tc_kernel(const __grid_constant__ AttnParams p) {
+// Forward for k > 128 (F4), one CTA per (128-query tile, b, h), 384 threads:
+// warps 0-3 load, issue MMAs and own TMEM; warps 4-11 run the softmax, two per
+// TMEM lane quadrant (warp w: query rows 32 (w % 4) .. +31, keys
+// 64 ((w - 4) / 4) .. +63 of each 128-key block).  For key block j:
+//   S_j = Q K_j^T into TMEM buffer j % 2, issued two blocks ahead, so the
+//   MMAs of S_{j+2} and O += P_j V_j run while the softmax of block j+1 runs;
+//   P_j = exp2(S_j scale - m) with m the row's running maximum, updated only
+//   when the block's maximum exceeds it by more than 2^8 (O and l are then
+//   rescaled in place; otherwise P may reach 2^8, well inside fp32 and exact
+//   up to the pair rounding, and the final O / l uses the same m throughout);
+//   O accumulates in TMEM.
+// K and V blocks stream through a 3-slot ring in the order the MMAs use them:
+// K0, K1, V0, K2, V1, K3, ... (see kv_item).
+constexpr int kLT = 384;              // threads
+constexpr int kLWorkers = 256;
+constexpr int kLKeys = 128;           // keys per block
+constexpr int kLSlots = 3;            // ring slots of one K or V block pair (32 KB)
+constexpr float kRescaleLog2 = 8.f;   // lazy-rescale threshold (log2 units)
+
+struct FwdLargeSmem {
+    uint8_t q[2][kTileHalf];                  // Q pair
+    uint8_t kv[kLSlots][2][kTileHalf];        // K or V block pairs
+    uint8_t p[2][2][kTileHalf];               // P pair [half][64-key block]
+    float part[2][128];                       // per key half: block max, then final sums
+    uint64_t q_full, kv_full[kLSlots], kv_empty[kLSlots], s_full[2], p_ready, pv_done;
+    uint32_t tmem;
+    int abort;
+};
+constexpr int kFwdLargeSmem = (int)sizeof(FwdLargeSmem) + 1024;
+static_assert(kFwdLargeSmem <= 227 * 1024, "shared memory");
+
+// Item t of the K/V stream for n blocks: (is V, block).
+__device__ __forceinline__ void kv_item(int t, int n, bool &is_v, int &blk) {
+    if (t == 0) { is_v = false; blk = 0; return; }
+    if (n == 1) { is_v = true; blk = 0; return; }
+    if (t == 2 * n - 1) { is_v = true; blk = n - 1; return; }
+    if (t & 1) { is_v = false; blk = (t + 1) >> 1; } else { is_v = true; blk = (t >> 1) - 1; }
+}
+
+__device__ __forceinline__ bool lwait(FwdLargeSmem &sm, uint64_t &bar, uint32_t parity, uint32_t *status) {
+    if (*(volatile int *)&sm.abort) return false;
+    if (mbar_wait(smem_u32(&bar), parity)) return true;
+    atomicOr(status, kStatusTimeout);
+    *(volatile int *)&sm.abort = 1;
+    return false;
+}
+
+__global__ void __launch_bounds__(kLT, 1) attn_fwd_tc_kernel(const __grid_constant__ AttnParams p) {
     extern __shared__ uint8_t smem_raw[];
-    FwdSmem &sm = *reinterpret_cast<FwdSmem *>(
+    FwdLargeSmem &sm = *reinterpret_cast<FwdLargeSmem *>(
         (reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-    const int qt = blockIdx.x, b = blockIdx.y, h = blockIdx.z;
+    // heaviest (last) query tiles first: they visit the most key blocks
+    const int nqt = gridDim.x;
+    const int qt = nqt - 1 - (int)blockIdx.x, b = blockIdx.y, h = blockIdx.z;
     const int i0 = qt * kQ;
-    const int q_end = min(p.k, i0 + kQ);               // exclusive
-    const int nblk = (q_end + kKV - 1) / kKV;          // causal: keys < q_end
+    const int n = qt + 1;                      // causal: key blocks 0 .. qt
+    const int nitems = 2 * n;
 
     if (threadIdx.x == 0) {
         mbar_init(smem_u32(&sm.q_full), 1);
-        for (int s = 0; s < kStages; ++s) {
+        for (int s = 0; s < kLSlots; ++s) {
             mbar_init(smem_u32(&sm.kv_full[s]), 1);
             mbar_init(smem_u32(&sm.kv_empty[s]), 1);
         }
-        mbar_init(smem_u32(&sm.s_full), 1);
-        mbar_init(smem_u32(&sm.o_full), 1);
-        mbar_init(smem_u32(&sm.p_ready), 128);
+        mbar_init(smem_u32(&sm.s_full[0]), 1);
+        mbar_init(smem_u32(&sm.s_full[1]), 1);
+        mbar_init(smem_u32(&sm.p_ready), kLWorkers);
+        mbar_init(smem_u32(&sm.pv_done), 1);
         sm.abort = 0;
         fence_barrier_init();
     }
     if (warp == 2) {
-        tmem_alloc(smem_u32(&sm.tmem), 128);
+        tmem_alloc(smem_u32(&sm.tmem), 512);
         tmem_relinquish();
     }
     tc_fence_before();
     __syncthreads();
     tc_fence_after();
-    pdl_wait();  // Q, K, V, dA, lse written by the previous kernels
+    pdl_wait();  // Q, K, V written by the previous kernels
     const uint32_t tmem = sm.tmem;
-    const uint32_t tS = tmem, tO = tmem + 64;
+    const uint32_t tO = tmem + 256;              // S buffers at 0 and 128
 
     if (warp == 0) {
-        // ---------------------------------------------------------- producer
         if (lane == 0) {
             const uint32_t qb = smem_u32(&sm.q_full);
-            mbar_expect_tx(qb, 2 * kQBytes);
+            mbar_expect_tx(qb, 2 * kTileHalf);
             tma_load_4d(smem_u32(sm.q[0]), &p.mQ, qb, 0, i0, b, h);
             tma_load_4d(smem_u32(sm.q[1]), &p.mQ, qb, 64, i0, b, h);
-            int issued = 0;
-            for (int j = 0; j < nblk; ++j) {
-                const int s = j % kStages;
-                if (!mbar_wait(smem_u32(&sm.kv_empty[s]), ((j / kStages) & 1) ^ 1) ||
-                    *(volatile int *)&sm.abort) {
-                    flag_timeout(sm, p.status);
-                    break;
-                }
+            for (int t = 0; t < nitems; ++t) {
+                const int s = t % kLSlots;
+                if (!lwait(sm, sm.kv_empty[s], ((t / kLSlots) & 1) ^ 1, p.status)) break;
+                bool is_v;
+                int blk;
+                kv_item(t, n, is_v, blk);
                 const uint32_t fb = smem_u32(&sm.kv_full[s]);
-                mbar_expect_tx(fb, 4 * kKVBytes);
-                tma_load_4d(smem_u32(sm.k[s][0]), &p.mK, fb, 0, j * kKV, b, h);
-                tma_load_4d(smem_u32(sm.k[s][1]), &p.mK, fb, 64, j * kKV, b, h);
-                tma_load_4d(smem_u32(sm.v[s][0]), &p.mV, fb, 0, j * kKV, b, h);
-                tma_load_4d(smem_u32(sm.v[s][1]), &p.mV, fb, 64, j * kKV, b, h);
-                issued = j + 1;
-            }
-            if (*(volatile int *)&sm.abort) {
-                mbar_wait(qb, 0);
-                for (int j = max(0, issued - kStages); j < issued; ++j)
-                    mbar_wait(smem_u32(&sm.kv_full[j % kStages]), (j / kStages) & 1);
+                mbar_expect_tx(fb, 2 * kTileHalf);
+                const CUtensorMap *m = is_v ? &p.mV : &p.mK;
+                tma_load_4d(smem_u32(sm.kv[s][0]), m, fb, 0, blk * kLKeys, b, h);
+                tma_load_4d(smem_u32(sm.kv[s][1]), m, fb, 64, blk * kLKeys, b, h);
             }
         }
     } else if (warp == 1) {
-        // ------------------------------------------------------------- MMA
         if (lane == 0) {
-            constexpr uint32_t idS = idesc_bf16(kQ, kKV, false, false);   // Q (K-major) x K^T (K-major)
-            constexpr uint32_t idO = idesc_bf16(kQ, 64, false, true);     // P (K-major) x V (MN-major)
-            bool ok = mbar_wait(smem_u32(&sm.q_full), 0);
-            const uint32_t q0 = smem_u32(sm.q[0]), q1 = smem_u32(sm.q[1]);
-            const uint32_t p0 = smem_u32(sm.p[0]), p1 = smem_u32(sm.p[1]);
-            // PV of block j: O = Ph Vh + Ph Vl + Pl Vh
-            auto issue_pv = [&](int j) {
-                const int s = j % kStages;
-                const uint32_t v0 = smem_u32(sm.v[s][0]), v1 = smem_u32(sm.v[s][1]);
-                const uint32_t pa[3] = {p0, p0, p1}, vb[3] = {v0, v1, v0};
-#pragma unroll
-                for (int t = 0; t < 3; ++t)
-#pragma unroll
-                    for (int kk = 0; kk < kKV / 16; ++kk)
-                        mma_bf16(tO, smem_desc_sw128(pa[t] + kk * 32, 16, 1024),
-                                 smem_desc_sw128(vb[t] + kk * 2048, kKVBytes, 1024), idO,
-                                 (t > 0 || kk > 0) ? 1u : 0u);
-                mma_commit(smem_u32(&sm.o_full));
+            constexpr uint32_t idS = idesc_bf16(128, kLKeys, false, false);
+            constexpr uint32_t idO = idesc_bf16(128, 64, false, true);
+            int t = 0;   // next K/V item to consume
+            bool ok = lwait(sm, sm.q_full, 0, p.status);
+            auto take = [&]() -> int {   // wait for item t, return its slot
+                const int s = t % kLSlots;
+                ok = ok && lwait(sm, sm.kv_full[s], (t / kLSlots) & 1, p.status);
+                ++t;
+                return s;
+            };
+            auto issue_s = [&](int j) {  // S_j = Q K_j^T into buffer j % 2
+                const int s = take();
+                if (!ok) return;
+                tc_fence_after();
+                mma_pair3(tmem + 128 * (j & 1), smem_u32(sm.q[0]), smem_u32(sm.q[1]),
+                          smem_u32(sm.kv[s][0]), smem_u32(sm.kv[s][1]), false, false, idS, false);
+                mma_commit(smem_u32(&sm.s_full[j & 1]));
                 mma_commit(smem_u32(&sm.kv_empty[s]));
             };
-            for (int j = 0; ok && j < nblk; ++j) {
-                if (j > 0) {
-                    if (!mbar_wait(smem_u32(&sm.p_ready), (j - 1) & 1) || *(volatile int *)&sm.abort) {
-                        ok = false;
-                        break;
-                    }
-                    tc_fence_after();
-                    issue_pv(j - 1);
-                }
-                const int s = j % kStages;
-                if (!mbar_wait(smem_u32(&sm.kv_full[s]), (j / kStages) & 1)) {
-                    ok = false;
-                    break;
-                }
+            issue_s(0);
+            if (n > 1) issue_s(1);
+            for (int j = 0; j < n && ok; ++j) {
+                ok = lwait(sm, sm.p_ready, j & 1, p.status);
+                const int s = take();   // V_j
+                if (!ok) break;
                 tc_fence_after();
-                const uint32_t k0 = smem_u32(sm.k[s][0]), k1 = smem_u32(sm.k[s][1]);
-                const uint32_t qa[3] = {q0, q0, q1}, kb[3] = {k0, k1, k0};
-#pragma unroll
-                for (int t = 0; t < 3; ++t)
-#pragma unroll
-                    for (int kk = 0; kk < 64 / 16; ++kk)
-                        mma_bf16(tS, smem_desc_sw128(qa[t] + kk * 32, 16, 1024),
-                                 smem_desc_sw128(kb[t] + kk * 32, 16, 1024), idS,
-                                 (t > 0 || kk > 0) ? 1u : 0u);
-                mma_commit(smem_u32(&sm.s_full));
-            }
-            if (ok && nblk > 0) {
-                if (mbar_wait(smem_u32(&sm.p_ready), (nblk - 1) & 1) && !*(volatile int *)&sm.abort) {
-                    tc_fence_after();
-                    issue_pv(nblk - 1);
-                } else {
-                    ok = false;
-                }
+                mma_k128(tO, sm.p, sm.kv[s], false, idO, j > 0);
+                mma_commit(smem_u32(&sm.pv_done));
+                mma_commit(smem_u32(&sm.kv_empty[s]));
+                if (j + 2 < n) issue_s(j + 2);
             }
             if (!ok) {
-                flag_timeout(sm, p.status);
                 // release the softmax warps
-                mma_commit(smem_u32(&sm.s_full));
-                mma_commit(smem_u32(&sm.o_full));
+                mma_commit(smem_u32(&sm.s_full[0]));
+                mma_commit(smem_u32(&sm.s_full[1]));
+                mma_commit(smem_u32(&sm.pv_done));
             }
         }
     } else if (warp >= 4) {
-        // ---------------------------------------------------------- softmax
         pdl_trigger();
-        const int q = warp - 4;
-        const int r = q * 32 + lane;
+        const int q = warp & 3, ch = (warp - 4) >> 2;
+        const int r = q * 32 + lane;               // query row of the tile
         const int i = i0 + r;
         const uint32_t lane_off = (uint32_t)(q * 32) << 16;
-        float o[64];
-#pragma unroll
-        for (int c = 0; c < 64; ++c) o[c] = 0.f;
-        float m = -INFINITY, l = 0.f, corr_prev = 1.f;
+        float m = -INFINITY, l = 0.f;              // running max (log2 units), partial sum
         bool ok = true;
-        for (int j = 0; j < nblk; ++j) {
-            if (!mbar_wait(smem_u32(&sm.s_full), j & 1) || *(volatile int *)&sm.abort) {
-                ok = false;
-                break;
-            }
+        for (int j = 0; j < n; ++j) {
+            ok = lwait(sm, sm.s_full[j & 1], (j >> 1) & 1, p.status) && ok;
             tc_fence_after();
             float s[64];
             {
                 float t32[32];
-                tmem_ld32(tS + lane_off, t32);
+                tmem_ld32(tmem + 128 * (j & 1) + lane_off + 64 * ch, t32);
 #pragma unroll
                 for (int c = 0; c < 32; ++c) s[c] = t32[c];
-                tmem_ld32(tS + lane_off + 32, t32);
+                tmem_ld32(tmem + 128 * (j & 1) + lane_off + 64 * ch + 32, t32);
 #pragma unroll
                 for (int c = 0; c < 32; ++c) s[32 + c] = t32[c];
             }
-            const int j0 = j * kKV;
-            float mx = m;
+            const int c0 = j * kLKeys + 64 * ch;  // first key of this thread's half
+            float mb = -INFINITY;
 #pragma unroll
             for (int c = 0; c < 64; ++c) {
-                s[c] = (j0 + c <= i) ? s[c] * p.scale_log2 : -INFINITY;
-                mx = fmaxf(mx, s[c]);
+                s[c] = (c0 + c <= i) ? s[c] * p.scale_log2 : -INFINITY;
+                mb = fmaxf(mb, s[c]);
             }
-            const float corr = exp2f(m - mx);   // 0 on the first block (m = -inf)
+            sm.part[ch][r] = mb;
+            named_barrier(1, kLWorkers);
+            mb = fmaxf(sm.part[0][r], sm.part[1][r]);
+            const bool grow = mb > m + kRescaleLog2;   // same decision in both threads of the row
+            const float m_new = grow ? mb : m;
+            const float corr = grow ? exp2f(m - m_new) : 1.f;   // 0 on the first block
             float sum = 0.f;
 #pragma unroll
             for (int c = 0; c < 64; ++c) {
-                s[c] = exp2f(s[c] - mx);
+                s[c] = exp2f(s[c] - m_new);
                 sum += s[c];
             }
             l = l * corr + sum;
-            m = mx;
-            if (j > 0) {
-                // O of the previous block: it is relative to the previous max.
-                if (!mbar_wait(smem_u32(&sm.o_full), (j - 1) & 1)) {
-                    ok = false;
-                    break;
-                }
-                tc_fence_after();
-                float t32[32];
-                tmem_ld32(tO + lane_off, t32);
+            m = m_new;
+            // P_{j-1} V_{j-1} done: P may be overwritten and O rescaled
+            if (j > 0) ok = lwait(sm, sm.pv_done, (j - 1) & 1, p.status) && ok;
+            tc_fence_after();
+            if (j > 0 && __any_sync(0xffffffffu, grow)) {
+                float o[32];
+                tmem_ld32(tO + lane_off + 32 * ch, o);
 #pragma unroll
-                for (int c = 0; c < 32; ++c) o[c] = o[c] * corr_prev + t32[c];
-                tmem_ld32(tO + lane_off + 32, t32);
-#pragma unroll
-                for (int c = 0; c < 32; ++c) o[32 + c] = o[32 + c] * corr_prev + t32[c];
+                for (int c = 0; c < 32; ++c) o[c] *= corr;
+                tmem_st32(tO + lane_off + 32 * ch, o);
             }
-            corr_prev = corr;
-            write_pair_row64(sm.p[0], sm.p[1], r, s);
+            write_pair32(sm.p, r, 64 * ch, s);
+            write_pair32(sm.p, r, 64 * ch + 32, s + 32);
+            named_barrier(1, kLWorkers);           // part[] reused by the next block
             fence_proxy_async();
             tc_fence_before();
             mbar_arrive(smem_u32(&sm.p_ready));
         }
-        if (ok && nblk > 0) {
-            if (mbar_wait(smem_u32(&sm.o_full), (nblk - 1) & 1)) {
-                tc_fence_after();
-                float t32[32];
-                tmem_ld32(tO + lane_off, t32);
-#pragma unroll
-                for (int c = 0; c < 32; ++c) o[c] = o[c] * corr_prev + t32[c];
-                tmem_ld32(tO + lane_off + 32, t32);
-#pragma unroll
-                for (int c = 0; c < 32; ++c) o[32 + c] = o[32 + c] * corr_prev + t32[c];
-            } else {
-                ok = false;
-            }
-        }
-        if (!ok) flag_timeout(sm, p.status);
-        if (ok && i < p.k && !*(volatile int *)&sm.abort) {
-            const size_t row = (size_t)h * p.Mtok + (size_t)b * p.k + i;
-            const float inv = 1.f / l;
-            const float rr = p.rsel[row];
-            float *arow = p.A + row * 64;
-#pragma unroll
-            for (int c = 0; c < 64; c += 4)
-                *reinterpret_cast<float4 *>(arow + c) =
-                    make_float4(o[c] * inv, o[c + 1] * inv, o[c + 2] * inv, o[c + 3] * inv);
-            bf16 *ar = p.AR + row * 128;
-#pragma unroll
-            for (int c = 0; c < 64; c += 8) {
-                uint32_t h4[4], l4[4];
-#pragma unroll
-                for (int e = 0; e < 4; ++e) {
-                    const float a = rr * o[c + 2 * e] * inv, bb = rr * o[c + 2 * e + 1] * inv;
-                    const bf16 ha = __float2bfloat16_rn(a), hb = __float2bfloat16_rn(bb);
-                    const bf16 la = __float2bfloat16_rn(a - __bfloat162float(ha));
-                    const bf16 lb = __float2bfloat16_rn(bb - __bfloat162float(hb));
-                    h4[e] = (uint32_t)__bfloat16_as_ushort(ha) | ((uint32_t)__bfloat16_as_ushort(hb) << 16);
-                    l4[e] = (uint32_t)__bfloat16_as_ushort(la) | ((uint32_t)__bfloat16_as_ushort(lb) << 16);
-                }
-                *reinterpret_cast<uint4 *>(ar + c) = make_uint4(h4[0], h4[1], h4[2], h4[3]);
-                *reinterpret_cast<uint4 *>(ar + 64 + c) = make_uint4(l4[0], l4[1], l4[2], l4[3]);
-            }
+        ok = lwait(sm, sm.pv_done, (n - 1) & 1, p.status) && ok;
+        tc_fence_after();
+        sm.part[ch][r] = l;
+        named_barrier(1, kLWorkers);
+        l = sm.part[0][r] + sm.part[1][r];
+        float o[32];
+        tmem_ld32(tO + lane_off + 32 * ch, o);      // output columns 32 ch .. +31
+        const bool live = __all_sync(0xffffffffu, ok && !*(volatile int *)&sm.abort);
+        const bool valid = i < p.k;
+        const unsigned vmask = __ballot_sync(0xffffffffu, valid);
+        const size_t row0 = (size_t)h * p.Mtok + (size_t)b * p.k + i0 + q * 32;
+        if (live) {
+            uint8_t *xb = &sm.kv[0][0][0] + (warp - 4) * 4096;   // the ring is idle now
+            const float inv = valid ? 1.f / l : 0.f;
+            stage_f32x32(xb, o, inv, lane);
+            store_rows128(xb, lane, [&](int rl, int c) -> uint4 * {
+                if (!((vmask >> rl) & 1u)) return nullptr;
+                return reinterpret_cast<uint4 *>(p.A + (row0 + rl) * 64 + 32 * ch) + c;
+            });
+            const float rr = valid ? p.rsel[row0 + lane] : 0.f;
+            stage_pair32(xb, o, inv * rr, lane);
+            store_rows128(xb, lane, [&](int rl, int c) -> uint4 * {
+                if (!((vmask >> rl) & 1u)) return nullptr;
+                bf16 *base = p.AR + (row0 + rl) * 128 + 32 * ch;
+                return c < 4 ? reinterpret_cast<uint4 *>(base) + c
+                             : reinterpret_cast<uint4 *>(base + 64) + (c - 4);
+            });
             // lse in natural-log units of the scaled scores
-            p.lse[row] = (m + log2f(l)) * 0.69314718055994531f;
+            if (ch == 0 && valid) p.lse[row0 + lane] = (m + log2f(l)) * 0.69314718055994531f;
         }
     }
     tc_fence_before();
     __syncthreads();
     if (warp == 2) {
         tc_fence_after();
-        tmem_dealloc(tmem, 128);
+        tmem_dealloc(tmem, 512);
     }
 }
 
@@ -1090,8 +1067,8 @@ cudaError_t tc_attn_fwd(const Dims &dm, const Saved &sv, cudaStream_t s) {
     bool ok = small ? (map_rows(&p.mQ, sv.Q, dm.H, Mtok) && map_rows(&p.mK, sv.K, dm.H, Mtok) &&
                        map_rows(&p.mV, sv.V, dm.H, Mtok))
                     : (map_units(&p.mQ, sv.Q, dm.H, dm.B, dm.k, kQ) &&
-                       map_units(&p.mK, sv.K, dm.H, dm.B, dm.k, kKV) &&
-                       map_units(&p.mV, sv.V, dm.H, dm.B, dm.k, kKV));
+                       map_units(&p.mK, sv.K, dm.H, dm.B, dm.k, kLKeys) &&
+                       map_units(&p.mV, sv.V, dm.H, dm.B, dm.k, kLKeys));
     if (!ok) return cudaErrorInvalidValue;
     p.U = small ? kSmallK / dm.k : 1;
     p.k = dm.k;
@@ -1107,7 +1084,7 @@ cudaError_t tc_attn_fwd(const Dims &dm, const Saved &sv, cudaStream_t s) {
     static cudaError_t attr = cudaSuccess;
     std::call_once(once, [] {
         attr = cudaFuncSetAttribute(attn_fwd_tc_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                    kFwdSmem);
+                                    kFwdLargeSmem);
         if (attr == cudaSuccess)
             attr = cudaFuncSetAttribute(attn_fwd_small_kernel,
                                         cudaFuncAttributeMaxDynamicSharedMemorySize, kSmallFwdSmem);
@@ -1120,7 +1097,7 @@ cudaError_t tc_attn_fwd(const Dims &dm, const Saved &sv, cudaStream_t s) {
         return e;
     }
     dim3 grid((dm.k + kQ - 1) / kQ, dm.B, dm.H);
-    cudaError_t e = launch_pdl(attn_fwd_tc_kernel, grid, dim3(kThreads), kFwdSmem, s, p);
+    cudaError_t e = launch_pdl(attn_fwd_tc_kernel, grid, dim3(kLT), kFwdLargeSmem, s, p);
     note_launches(1);
     return e;
 }

@@ -74,8 +74,10 @@ __device__ __forceinline__ void mma_pair3(uint32_t d, uint32_t a_hi, uint32_t a_
 // and B a pair of 128-row tiles, three split products each.
 //   a_mn = false: A K-major, K = tile columns (P V, dS K)
 //   a_mn = true:  A read as its transpose (P^T dA, dS^T Q), K = tile rows
+// With accumulate, the products add to what D already holds.
 __device__ __forceinline__ void mma_k128(uint32_t d, const uint8_t (*a)[2][kTileHalf],
-                                         const uint8_t (*b)[kTileHalf], bool a_mn, uint32_t idesc) {
+                                         const uint8_t (*b)[kTileHalf], bool a_mn, uint32_t idesc,
+                                         bool accumulate = false) {
 #pragma unroll
     for (int t = 0; t < 3; ++t) {
         const int ah = t == 2 ? 1 : 0, bh = t == 1 ? 1 : 0;
@@ -90,7 +92,7 @@ __device__ __forceinline__ void mma_k128(uint32_t d, const uint8_t (*a)[2][kTile
             }
             // B rows = K index (MN-major B: 64-wide N block, 16 rows per step)
             bd = smem_desc_sw128(smem_u32(b[bh]) + kk * 2048, kTileHalf, 1024);
-            mma_bf16(d, ad, bd, idesc, (t > 0 || kk > 0) ? 1u : 0u);
+            mma_bf16(d, ad, bd, idesc, (accumulate || t > 0 || kk > 0) ? 1u : 0u);
         }
     }
 }

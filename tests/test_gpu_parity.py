@@ -74,6 +74,9 @@ SMALL = [
     W.MosaConfig("pack4_bf16", B=5, T=100, d=64, H=3, hp=64, k=32, dtype="bf16", seed=18),
     W.MosaConfig("pack2_k50_bf16", B=5, T=120, d=64, H=2, hp=64, k=50, dtype="bf16", seed=19),
     W.MosaConfig("pack42_k3_bf16", B=5, T=40, d=32, H=2, hp=64, k=3, dtype="bf16", seed=20),
+    # k > 128: several 128-query tiles and 128-key blocks, full and ragged
+    W.MosaConfig("largek_bf16", B=1, T=512, d=128, H=3, hp=64, k=384, dtype="bf16", seed=21),
+    W.MosaConfig("largek_ragged_bf16", B=2, T=600, d=64, H=2, hp=64, k=300, dtype="bf16", seed=22),
 ]
 
 

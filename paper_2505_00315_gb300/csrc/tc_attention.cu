@@ -64,11 +64,7 @@ __device__ __forceinline__ void write_pair_row64(uint8_t *hi_tile, uint8_t *lo_t
 #pragma unroll
         for (int e = 0; e < 4; ++e) {
             const float a = v[c * 8 + 2 * e], b = v[c * 8 + 2 * e + 1];
-            const bf16 ha = __float2bfloat16_rn(a), hb = __float2bfloat16_rn(b);
-            const bf16 la = __float2bfloat16_rn(a - __bfloat162float(ha));
-            const bf16 lb = __float2bfloat16_rn(b - __bfloat162float(hb));
-            h4[e] = (uint32_t)__bfloat16_as_ushort(ha) | ((uint32_t)__bfloat16_as_ushort(hb) << 16);
-            l4[e] = (uint32_t)__bfloat16_as_ushort(la) | ((uint32_t)__bfloat16_as_ushort(lb) << 16);
+            split_pair2(a, b, h4[e], l4[e]);
         }
         const int off = r * 128 + ((c ^ (r & 7)) << 4);
         *reinterpret_cast<uint4 *>(hi_tile + off) = make_uint4(h4[0], h4[1], h4[2], h4[3]);
@@ -251,11 +247,11 @@ __global__ void __launch_bounds__(kLT, 1) attn_fwd_tc_kernel(const __grid_consta
             mb = fmaxf(sm.part[0][r], sm.part[1][r]);
             const bool grow = mb > m + kRescaleLog2;   // same decision in both threads of the row
             const float m_new = grow ? mb : m;
-            const float corr = grow ? exp2f(m - m_new) : 1.f;   // 0 on the first block
+            const float corr = grow ? exp2_fast(m - m_new) : 1.f;   // 0 on the first block
             float sum = 0.f;
 #pragma unroll
             for (int c = 0; c < 64; ++c) {
-                s[c] = exp2f(s[c] - m_new);
+                s[c] = exp2_fast(s[c] - m_new);
                 sum += s[c];
             }
             l = l * corr + sum;
@@ -386,11 +382,7 @@ __device__ __forceinline__ void store_pair64(bf16 *row, int col_hi, int col_lo, 
 #pragma unroll
         for (int e = 0; e < 4; ++e) {
             const float a = v[c + 2 * e] * f, b = v[c + 2 * e + 1] * f;
-            const bf16 ha = __float2bfloat16_rn(a), hb = __float2bfloat16_rn(b);
-            const bf16 la = __float2bfloat16_rn(a - __bfloat162float(ha));
-            const bf16 lb = __float2bfloat16_rn(b - __bfloat162float(hb));
-            h4[e] = (uint32_t)__bfloat16_as_ushort(ha) | ((uint32_t)__bfloat16_as_ushort(hb) << 16);
-            l4[e] = (uint32_t)__bfloat16_as_ushort(la) | ((uint32_t)__bfloat16_as_ushort(lb) << 16);
+            split_pair2(a, b, h4[e], l4[e]);
         }
         *reinterpret_cast<uint4 *>(row + col_hi + c) = make_uint4(h4[0], h4[1], h4[2], h4[3]);
         *reinterpret_cast<uint4 *>(row + col_lo + c) = make_uint4(l4[0], l4[1], l4[2], l4[3]);
@@ -520,7 +512,7 @@ __global__ void __launch_bounds__(kThreads, 1) attn_dkv_tc_kernel(const __grid_c
                 const bool allowed = (i >= j) && (i < p.k);
                 const float l2 = allowed ? __ldg(p.lse + base + i) * 1.4426950408889634f : 0.f;
                 const float dd = allowed ? __ldg(p.Dd + base + i) : 0.f;
-                const float pr = allowed ? exp2f(st[c] * p.scale_log2 - l2) : 0.f;
+                const float pr = allowed ? exp2_fast(st[c] * p.scale_log2 - l2) : 0.f;
                 st[c] = pr;
                 dpt[c] = pr * (dpt[c] - dd);
             }
@@ -674,7 +666,7 @@ __global__ void __launch_bounds__(kThreads, 1) attn_dq_tc_kernel(const __grid_co
 #pragma unroll
             for (int c = 0; c < 64; ++c) {
                 const bool allowed = (jb + c <= i);
-                const float pr = allowed ? exp2f(sv[c] * p.scale_log2 - l2) : 0.f;
+                const float pr = allowed ? exp2_fast(sv[c] * p.scale_log2 - l2) : 0.f;
                 dp[c] = pr * (dp[c] - dd);
             }
             if (n > 0 && !mbar_wait(smem_u32(&sm.ds_done), (n - 1) & 1)) {
@@ -843,7 +835,7 @@ __global__ void __launch_bounds__(kSmallThreads, 1) attn_fwd_small_kernel(const 
             tmem_ld32(tS + lane_off + c0, t32);
 #pragma unroll
             for (int c = 0; c < 32; ++c) {
-                t32[c] = (c0 + c <= r && c0 + c >= lo) ? exp2f(t32[c] * p.scale_log2 - m) : 0.f;
+                t32[c] = (c0 + c <= r && c0 + c >= lo) ? exp2_fast(t32[c] * p.scale_log2 - m) : 0.f;
                 l += t32[c];
             }
             write_pair32(sm.p, r, c0, t32);
@@ -985,7 +977,7 @@ __global__ void __launch_bounds__(kSmallThreads, 1) attn_bwd_small_kernel(const 
             tmem_ld32(tS + lane_off + c0, t32);
 #pragma unroll
             for (int c = 0; c < 32; ++c)
-                t32[c] = (valid && c0 + c <= r && c0 + c >= lo) ? exp2f(t32[c] * p.scale_log2 - l2) : 0.f;
+                t32[c] = (valid && c0 + c <= r && c0 + c >= lo) ? exp2_fast(t32[c] * p.scale_log2 - l2) : 0.f;
             write_pair32(sm.p, r, c0, t32);
         }
         fence_proxy_async();
@@ -1000,7 +992,7 @@ __global__ void __launch_bounds__(kSmallThreads, 1) attn_bwd_small_kernel(const 
             tmem_ld32(tDP + lane_off + c0, d32);
 #pragma unroll
             for (int c = 0; c < 32; ++c) {
-                const float pr = (valid && c0 + c <= r && c0 + c >= lo) ? exp2f(t32[c] * p.scale_log2 - l2) : 0.f;
+                const float pr = (valid && c0 + c <= r && c0 + c >= lo) ? exp2_fast(t32[c] * p.scale_log2 - l2) : 0.f;
                 t32[c] = pr * (d32[c] - dd);
             }
             write_pair32(sm.p, r, c0, t32);

@@ -230,6 +230,25 @@ __host__ __device__ constexpr uint32_t idesc_bf16(int M, int N, bool a_mn_major,
            | ((uint32_t)(M >> 4) << 24);
 }
 
+// hi = bf16(v), lo = bf16(v - hi) for two values at once, each half by one
+// packed conversion (round to nearest even), as bf16x2 words with a in the
+// low 16 bits: the split-bf16 pair representation of the kernels' operands.
+__device__ __forceinline__ void split_pair2(float a, float b, uint32_t &hi, uint32_t &lo) {
+    const __nv_bfloat162 h = __floats2bfloat162_rn(a, b);
+    const float2 hf = __bfloat1622float2(h);
+    const __nv_bfloat162 l = __floats2bfloat162_rn(a - hf.x, b - hf.y);
+    hi = *reinterpret_cast<const uint32_t *>(&h);
+    lo = *reinterpret_cast<const uint32_t *>(&l);
+}
+
+// 2^x by the hardware approximation (PTX ex2.approx; -inf gives 0), for the
+// softmax exponentials.
+__device__ __forceinline__ float exp2_fast(float x) {
+    float y;
+    asm("ex2.approx.ftz.f32 %0, %1;" : "=f"(y) : "f"(x));
+    return y;
+}
+
 // ------------------------------------------------------ epilogue staging
 // A warp stages 32 rows of 128 bytes, one row per lane (16-byte unit c of row r
 // at r*128 + ((c ^ (r & 7)) << 4), free of bank conflicts), then copies them
@@ -256,11 +275,7 @@ __device__ __forceinline__ void stage_pair32(uint8_t *xb, const float *v, float 
 #pragma unroll
         for (int e = 0; e < 4; ++e) {
             const float a = v[8 * u + 2 * e] * f, b = v[8 * u + 2 * e + 1] * f;
-            const __nv_bfloat16 ha = __float2bfloat16_rn(a), hb = __float2bfloat16_rn(b);
-            const __nv_bfloat16 la = __float2bfloat16_rn(a - __bfloat162float(ha));
-            const __nv_bfloat16 lb = __float2bfloat16_rn(b - __bfloat162float(hb));
-            h4[e] = (uint32_t)__bfloat16_as_ushort(ha) | ((uint32_t)__bfloat16_as_ushort(hb) << 16);
-            l4[e] = (uint32_t)__bfloat16_as_ushort(la) | ((uint32_t)__bfloat16_as_ushort(lb) << 16);
+            split_pair2(a, b, h4[e], l4[e]);
         }
         *reinterpret_cast<uint4 *>(xb + xoff128(lane, u)) = make_uint4(h4[0], h4[1], h4[2], h4[3]);
         *reinterpret_cast<uint4 *>(xb + xoff128(lane, 4 + u)) = make_uint4(l4[0], l4[1], l4[2], l4[3]);

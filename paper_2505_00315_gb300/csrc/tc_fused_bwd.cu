@@ -350,7 +350,7 @@ __global__ void __launch_bounds__(kThreads, 1) fused_bwd_kernel(const __grid_con
             tmem_ld32(tmem + kColS + lane_off + c0, t32);
 #pragma unroll
             for (int c = 0; c < 32; ++c)
-                t32[c] = (valid && c0 + c <= r && c0 + c >= lo) ? exp2f(t32[c] * p.scale_log2 - l2) : 0.f;
+                t32[c] = (valid && c0 + c <= r && c0 + c >= lo) ? exp2_fast(t32[c] * p.scale_log2 - l2) : 0.f;
             write_pair32(ptile, r, c0, t32);
         }
         fence_proxy_async();
@@ -365,7 +365,7 @@ __global__ void __launch_bounds__(kThreads, 1) fused_bwd_kernel(const __grid_con
             tmem_ld32(tmem + kColDP + lane_off + c0, d32);
 #pragma unroll
             for (int c = 0; c < 32; ++c) {
-                const float pr = (valid && c0 + c <= r && c0 + c >= lo) ? exp2f(t32[c] * p.scale_log2 - l2) : 0.f;
+                const float pr = (valid && c0 + c <= r && c0 + c >= lo) ? exp2_fast(t32[c] * p.scale_log2 - l2) : 0.f;
                 t32[c] = pr * (d32[c] - dd);
             }
             write_pair32(ptile, r, c0, t32);

@@ -331,7 +331,7 @@ __global__ void __launch_bounds__(kThreads, 1) fused_fwd_kernel(const __grid_con
             tmem_ld32(tmem + lane_off + c0, t32);
 #pragma unroll
             for (int c = 0; c < 32; ++c) {
-                t32[c] = (c0 + c <= r && c0 + c >= lo) ? exp2f(t32[c] * p.scale_log2 - m) : 0.f;
+                t32[c] = (c0 + c <= r && c0 + c >= lo) ? exp2_fast(t32[c] * p.scale_log2 - m) : 0.f;
                 l += t32[c];
             }
             put_pair32(ptile[0][c0 >> 6], ptile[1][c0 >> 6], r, c0, t32, 1.f);

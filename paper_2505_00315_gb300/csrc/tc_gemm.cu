@@ -178,20 +178,12 @@ __device__ __forceinline__ uint32_t xoff256(int rl, int u) {
     return (uint32_t)(rl * 256 + ((u ^ (rl & 15)) << 4));
 }
 
-__device__ __forceinline__ uint32_t pack_bf16x2(bf16 a, bf16 b) {
-    return (uint32_t)__bfloat16_as_ushort(a) | ((uint32_t)__bfloat16_as_ushort(b) << 16);
-}
-
 // Values v[8u .. 8u+7] of this lane's row as hi unit u and lo unit 8 + u.
 __device__ __forceinline__ void stage_pair_unit(uint8_t *xb, int lane, int u, const float *v) {
     uint32_t h4[4], l4[4];
 #pragma unroll
     for (int e = 0; e < 4; ++e) {
-        const float a = v[2 * e], b = v[2 * e + 1];
-        const bf16 ha = __float2bfloat16_rn(a), hb = __float2bfloat16_rn(b);
-        h4[e] = pack_bf16x2(ha, hb);
-        l4[e] = pack_bf16x2(__float2bfloat16_rn(a - __bfloat162float(ha)),
-                            __float2bfloat16_rn(b - __bfloat162float(hb)));
+        split_pair2(v[2 * e], v[2 * e + 1], h4[e], l4[e]);
     }
     *reinterpret_cast<uint4 *>(xb + xoff256(lane, u)) = make_uint4(h4[0], h4[1], h4[2], h4[3]);
     *reinterpret_cast<uint4 *>(xb + xoff256(lane, 8 + u)) = make_uint4(l4[0], l4[1], l4[2], l4[3]);

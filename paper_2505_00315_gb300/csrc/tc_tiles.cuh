@@ -34,11 +34,7 @@ __device__ __forceinline__ void put_pair32(uint8_t *hi_blk, uint8_t *lo_blk, int
 #pragma unroll
         for (int e = 0; e < 4; ++e) {
             const float a = v[c * 8 + 2 * e] * f, b = v[c * 8 + 2 * e + 1] * f;
-            const __nv_bfloat16 ha = __float2bfloat16_rn(a), hb = __float2bfloat16_rn(b);
-            const __nv_bfloat16 la = __float2bfloat16_rn(a - __bfloat162float(ha));
-            const __nv_bfloat16 lb = __float2bfloat16_rn(b - __bfloat162float(hb));
-            h4[e] = (uint32_t)__bfloat16_as_ushort(ha) | ((uint32_t)__bfloat16_as_ushort(hb) << 16);
-            l4[e] = (uint32_t)__bfloat16_as_ushort(la) | ((uint32_t)__bfloat16_as_ushort(lb) << 16);
+            split_pair2(a, b, h4[e], l4[e]);
         }
         const int off = r * 128 + (((cb + c) ^ (r & 7)) << 4);
         *reinterpret_cast<uint4 *>(hi_blk + off) = make_uint4(h4[0], h4[1], h4[2], h4[3]);

@@ -230,15 +230,18 @@ __host__ __device__ constexpr uint32_t idesc_bf16(int M, int N, bool a_mn_major,
            | ((uint32_t)(M >> 4) << 24);
 }
 
-// hi = bf16(v), lo = bf16(v - hi) for two values at once, each half by one
-// packed conversion (round to nearest even), as bf16x2 words with a in the
-// low 16 bits: the split-bf16 pair representation of the kernels' operands.
+// The split-bf16 pair representation of the kernels' intermediate operands,
+// for two values at once, as bf16x2 words with a in the low 16 bits:
+// hi = v cut to bf16 (low 16 bits cleared, i.e. rounded toward zero), r = v - hi
+// (exact in fp32), lo = r cut the same way; |v - (hi + lo)| < 2^-14 |v|.
+// Integer operations only (the bf16 conversion unit is far slower):
+// __byte_perm(x, y, 0x7632) packs the high halves of x and y.
 __device__ __forceinline__ void split_pair2(float a, float b, uint32_t &hi, uint32_t &lo) {
-    const __nv_bfloat162 h = __floats2bfloat162_rn(a, b);
-    const float2 hf = __bfloat1622float2(h);
-    const __nv_bfloat162 l = __floats2bfloat162_rn(a - hf.x, b - hf.y);
-    hi = *reinterpret_cast<const uint32_t *>(&h);
-    lo = *reinterpret_cast<const uint32_t *>(&l);
+    const uint32_t ua = __float_as_uint(a), ub = __float_as_uint(b);
+    const float ra = a - __uint_as_float(ua & 0xFFFF0000u);
+    const float rb = b - __uint_as_float(ub & 0xFFFF0000u);
+    hi = __byte_perm(ua, ub, 0x7632);
+    lo = __byte_perm(__float_as_uint(ra), __float_as_uint(rb), 0x7632);
 }
 
 // 2^x by the hardware approximation (PTX ex2.approx; -inf gives 0), for the

@@ -95,7 +95,7 @@ struct FwdLargeSmem {
     uint8_t q[2][kTileHalf];                  // Q pair
     uint8_t kv[kLSlots][2][kTileHalf];        // K or V block pairs
     uint8_t p[2][2][kTileHalf];               // P pair [half][64-key block]
-    float part[2][128];                       // per key half: block max, then final sums
+    float part[2][2][128];                    // [block parity][key half]: block max, final sums
     uint64_t q_full, kv_full[kLSlots], kv_empty[kLSlots], s_full[2], p_ready, pv_done;
     uint32_t tmem;
     int abort;
@@ -235,26 +235,35 @@ __global__ void __launch_bounds__(kLT, 1) attn_fwd_tc_kernel(const __grid_consta
 #pragma unroll
                 for (int c = 0; c < 32; ++c) s[32 + c] = t32[c];
             }
-            const int c0 = j * kLKeys + 64 * ch;  // first key of this thread's half
-            float mb = -INFINITY;
+            if (j == qt) {
+                // diagonal block (earlier blocks are wholly visible): key
+                // j*128 + 64 ch + c is visible from query i iff c <= lim
+                const int lim = i - (j * kLKeys + 64 * ch);
 #pragma unroll
-            for (int c = 0; c < 64; ++c) {
-                s[c] = (c0 + c <= i) ? s[c] * p.scale_log2 : -INFINITY;
-                mb = fmaxf(mb, s[c]);
+                for (int c = 0; c < 64; ++c)
+                    if (c > lim) s[c] = -INFINITY;
             }
-            sm.part[ch][r] = mb;
+            // maxima and sums in four independent chains
+            float mx[4] = {-INFINITY, -INFINITY, -INFINITY, -INFINITY};
+#pragma unroll
+            for (int c = 0; c < 64; ++c) mx[c & 3] = fmaxf(mx[c & 3], s[c]);
+            float mb = fmaxf(fmaxf(mx[0], mx[1]), fmaxf(mx[2], mx[3])) * p.scale_log2;
+            // the exchange buffer alternates with the block parity: the buffer
+            // written here was last read before everyone passed the previous
+            // block's barrier, so one barrier per block suffices
+            sm.part[j & 1][ch][r] = mb;
             named_barrier(1, kLWorkers);
-            mb = fmaxf(sm.part[0][r], sm.part[1][r]);
+            mb = fmaxf(sm.part[j & 1][0][r], sm.part[j & 1][1][r]);
             const bool grow = mb > m + kRescaleLog2;   // same decision in both threads of the row
             const float m_new = grow ? mb : m;
             const float corr = grow ? exp2_fast(m - m_new) : 1.f;   // 0 on the first block
-            float sum = 0.f;
+            float sm4[4] = {0.f, 0.f, 0.f, 0.f};
 #pragma unroll
             for (int c = 0; c < 64; ++c) {
-                s[c] = exp2_fast(s[c] - m_new);
-                sum += s[c];
+                s[c] = exp2_fast(fmaf(s[c], p.scale_log2, -m_new));
+                sm4[c & 3] += s[c];
             }
-            l = l * corr + sum;
+            l = l * corr + ((sm4[0] + sm4[1]) + (sm4[2] + sm4[3]));
             m = m_new;
             // P_{j-1} V_{j-1} done: P may be overwritten and O rescaled
             if (j > 0) ok = lwait(sm, sm.pv_done, (j - 1) & 1, p.status) && ok;
@@ -268,16 +277,15 @@ __global__ void __launch_bounds__(kLT, 1) attn_fwd_tc_kernel(const __grid_consta
             }
             write_pair32(sm.p, r, 64 * ch, s);
             write_pair32(sm.p, r, 64 * ch + 32, s + 32);
-            named_barrier(1, kLWorkers);           // part[] reused by the next block
             fence_proxy_async();
             tc_fence_before();
             mbar_arrive(smem_u32(&sm.p_ready));
         }
         ok = lwait(sm, sm.pv_done, (n - 1) & 1, p.status) && ok;
         tc_fence_after();
-        sm.part[ch][r] = l;
+        sm.part[n & 1][ch][r] = l;
         named_barrier(1, kLWorkers);
-        l = sm.part[0][r] + sm.part[1][r];
+        l = sm.part[n & 1][0][r] + sm.part[n & 1][1][r];
         float o[32];
         tmem_ld32(tO + lane_off + 32 * ch, o);      // output columns 32 ch .. +31
         const bool live = __all_sync(0xffffffffu, ok && !*(volatile int *)&sm.abort);

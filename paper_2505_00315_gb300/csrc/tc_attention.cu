@@ -82,19 +82,25 @@ __device__ __forceinline__ void write_pair_row64(uint8_t *hi_tile, uint8_t *lo_t
 //   when the block's maximum exceeds it by more than 2^8 (O and l are then
 //   rescaled in place; otherwise P may reach 2^8, well inside fp32 and exact
 //   up to the pair rounding, and the final O / l uses the same m throughout);
-//   O accumulates in TMEM.
-// K and V blocks stream through a 3-slot ring in the order the MMAs use them:
+//   O accumulates in TMEM.  P_j (a bf16 pair) is written by the softmax warps
+//   into the TMEM columns of S_j itself (hi in the first 64 columns, lo in
+//   the next 64, two bf16 per column) and O += P_j V_j reads it from there as
+//   the A operand.  Measured on this GPU: a tcgen05.st issued while an MMA
+//   that reads its A operand from TMEM is still running corrupts that MMA's
+//   result even when the columns differ, so P_j is stored only after
+//   P_{j-1} V_{j-1} has completed (its exponentials are computed meanwhile),
+//   and S_{j+2} (which overwrites P_j's columns) only after P_j V_j.
+// K and V blocks stream through a 4-slot ring in the order the MMAs use them:
 // K0, K1, V0, K2, V1, K3, ... (see kv_item).
 constexpr int kLT = 384;              // threads
 constexpr int kLWorkers = 256;
 constexpr int kLKeys = 128;           // keys per block
-constexpr int kLSlots = 3;            // ring slots of one K or V block pair (32 KB)
+constexpr int kLSlots = 4;            // ring slots of one K or V block pair (32 KB)
 constexpr float kRescaleLog2 = 8.f;   // lazy-rescale threshold (log2 units)
 
 struct FwdLargeSmem {
     uint8_t q[2][kTileHalf];                  // Q pair
     uint8_t kv[kLSlots][2][kTileHalf];        // K or V block pairs
-    uint8_t p[2][2][kTileHalf];               // P pair [half][64-key block]
     float part[2][2][128];                    // [block parity][key half]: block max, final sums
     uint64_t q_full, kv_full[kLSlots], kv_empty[kLSlots], s_full[2], p_ready, pv_done;
     uint32_t tmem;
@@ -202,10 +208,26 @@ __global__ void __launch_bounds__(kLT, 1) attn_fwd_tc_kernel(const __grid_consta
                 const int s = take();   // V_j
                 if (!ok) break;
                 tc_fence_after();
-                mma_k128(tO, sm.p, sm.kv[s], false, idO, j > 0);
+                // O += P_j V_j: P (A operand) from the TMEM columns of S_j,
+                // hi at +0, lo at +64, 8 columns per 16 keys; V MN-major
+                const uint32_t pa = tmem + 128 * (j & 1);
+#pragma unroll
+                for (int tt = 0; tt < 3; ++tt) {
+                    const uint32_t a_col = pa + (tt == 2 ? 64 : 0);
+                    const uint32_t vb = smem_u32(sm.kv[s][tt == 1 ? 1 : 0]);
+#pragma unroll
+                    for (int kk = 0; kk < 8; ++kk)
+                        mma_bf16_ts(tO, a_col + 8 * kk, smem_desc_sw128(vb + kk * 2048, kTileHalf, 1024),
+                                    idO, (j > 0 || tt > 0 || kk > 0) ? 1u : 0u);
+                }
                 mma_commit(smem_u32(&sm.pv_done));
                 mma_commit(smem_u32(&sm.kv_empty[s]));
-                if (j + 2 < n) issue_s(j + 2);
+                if (j + 2 < n) {
+                    // S_{j+2} overwrites the columns P_j V_j reads
+                    ok = ok && lwait(sm, sm.pv_done, j & 1, p.status);
+                    tc_fence_after();
+                    issue_s(j + 2);
+                }
             }
             if (!ok) {
                 // release the softmax warps
@@ -265,9 +287,12 @@ __global__ void __launch_bounds__(kLT, 1) attn_fwd_tc_kernel(const __grid_consta
             }
             l = l * corr + ((sm4[0] + sm4[1]) + (sm4[2] + sm4[3]));
             m = m_new;
-            // P_{j-1} V_{j-1} done: P may be overwritten and O rescaled
-            if (j > 0) ok = lwait(sm, sm.pv_done, (j - 1) & 1, p.status) && ok;
-            tc_fence_after();
+            // P_{j-1} V_{j-1} must be complete before any TMEM store (see above);
+            // then O may also be rescaled (P_j V_j waits for this block's P)
+            if (j > 0) {
+                ok = lwait(sm, sm.pv_done, (j - 1) & 1, p.status) && ok;
+                tc_fence_after();
+            }
             if (j > 0 && __any_sync(0xffffffffu, grow)) {
                 float o[32];
                 tmem_ld32(tO + lane_off + 32 * ch, o);
@@ -275,9 +300,17 @@ __global__ void __launch_bounds__(kLT, 1) attn_fwd_tc_kernel(const __grid_consta
                 for (int c = 0; c < 32; ++c) o[c] *= corr;
                 tmem_st32(tO + lane_off + 32 * ch, o);
             }
-            write_pair32(sm.p, r, 64 * ch, s);
-            write_pair32(sm.p, r, 64 * ch + 32, s + 32);
-            fence_proxy_async();
+            // P_j as a pair into the columns of S_j: this thread's 64 keys are
+            // columns 32 ch .. +31 of the hi half and of the lo half (both
+            // threads of the row have read their S values: exchange barrier)
+            {
+                uint32_t hw[32], lw[32];
+#pragma unroll
+                for (int c = 0; c < 32; ++c) split_pair2(s[2 * c], s[2 * c + 1], hw[c], lw[c]);
+                const uint32_t pb = tmem + 128 * (j & 1) + lane_off + 32 * ch;
+                tmem_st32u(pb, hw);
+                tmem_st32u(pb + 64, lw);
+            }
             tc_fence_before();
             mbar_arrive(smem_u32(&sm.p_ready));
         }

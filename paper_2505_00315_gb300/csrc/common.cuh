@@ -90,7 +90,8 @@ struct Saved {
     float *Dd;          // [H,B*k]   rowsum(dA o A)
     void *dQKV;         // [H,B*k,3hp] dQ | dK | dV, intermediate (tensor-core path:
                         // [H,B*k,512] bf16 pair dQ|dK|dV|dlogit,0.. hi then lo)
-    float *G;           // [H,B*k,hp] dY[I] W_o^T (fp32)
+    float *G;           // [H,B*k,hp] dY[I] W_o^T (fp32, CUDA-core path); on the
+                        // tensor-core path with k > 128 the fp32 dQ accumulator
     float *WrT;         // [H,d] fp32 transpose of W_r (tensor-core backward)
 };
 

@@ -12,17 +12,15 @@
 // bf16 MMAs (hi*hi + hi*lo + lo*hi) into one fp32 accumulator, which keeps the
 // result at fp32-level accuracy.
 // Backward (B2), flash-style with P recomputed from the saved log-sum-exp,
-// D = rowsum(dA o A) and dS = P o (dP - D):
-//   dK/dV kernel, one CTA per (128-key tile, b, h), over 64-query blocks:
-//     S^T = K Q^T, dP^T = V dA^T, then dV += P^T dA, dK += dS^T Q
-//   dQ kernel, one CTA per (128-query tile, b, h), over 64-key blocks:
-//     S = Q K^T, dP = dA V^T, then dQ += dS K
+// D = rowsum(dA o A) and dS = P o (dP - D): one CTA per (128-key tile, b, h)
+// over 128-query blocks: S = Q K^T, dP = dA V^T, then dV += P^T dA,
+// dK += dS^T Q, and dQ = dS K added into an fp32 accumulator (details at the
+// kernel); k <= 128 needs one block and writes dQ directly.
 // The same shared-memory tile of Q (or dA, K) serves as a K-major operand in
 // one product and as an MN-major operand in the other.
-// Warp roles: 0 TMA producer, 1 MMA issuer, 2 TMEM allocator, then softmax
-// warps (4-7 with one row per thread in the backward kernels, 4-11 with two
-// threads per row in the forward and the k <= 128 kernels).  All waits are
-// bounded.
+// Warp roles: 0 TMA producer, 1 MMA issuer, 2 TMEM allocator, 4-11 softmax
+// and epilogue warps, two threads per row (each half of the keys).  All waits
+// are bounded.
 #include <mutex>
 
 #include "launch.h"
@@ -37,9 +35,6 @@ namespace {
 using namespace tc;
 
 constexpr int kQ = 128;          // queries per CTA
-constexpr int kKV = 64;          // keys per block
-constexpr int kThreads = 256;
-constexpr int kStages = 2;
 
 struct AttnParams {
     CUtensorMap mQ, mK, mV;   // 4-D maps over [H, B, k, 128] pairs, box {64, rows, 1, 1}
@@ -54,23 +49,6 @@ struct AttnParams {
     uint32_t *status;
 };
 
-// Writes 64 values of one row of a K-major, 128-byte-swizzled bf16 tile as
-// hi and lo halves (row r of a tile whose rows are 128 bytes).
-__device__ __forceinline__ void write_pair_row64(uint8_t *hi_tile, uint8_t *lo_tile, int r,
-                                                 const float *v) {
-#pragma unroll
-    for (int c = 0; c < 8; ++c) {
-        uint32_t h4[4], l4[4];
-#pragma unroll
-        for (int e = 0; e < 4; ++e) {
-            const float a = v[c * 8 + 2 * e], b = v[c * 8 + 2 * e + 1];
-            split_pair2(a, b, h4[e], l4[e]);
-        }
-        const int off = r * 128 + ((c ^ (r & 7)) << 4);
-        *reinterpret_cast<uint4 *>(hi_tile + off) = make_uint4(h4[0], h4[1], h4[2], h4[3]);
-        *reinterpret_cast<uint4 *>(lo_tile + off) = make_uint4(l4[0], l4[1], l4[2], l4[3]);
-    }
-}
 
 // Forward for k > 128 (F4), one CTA per (128-query tile, b, h), 384 threads:
 // warps 0-3 load, issue MMAs and own TMEM; warps 4-11 run the softmax, two per
@@ -355,38 +333,6 @@ __global__ void __launch_bounds__(kLT, 1) attn_fwd_tc_kernel(const __grid_consta
 
 // ------------------------------------------------------------ backward
 
-constexpr int kKT = 128;                  // keys per dK/dV CTA
-constexpr int kQB = 64;                   // queries per block in the dK/dV loop
-constexpr int kHalf128 = 128 * 64 * 2;    // one half of a 128-row tile, 16 KB
-constexpr int kHalf64 = 64 * 64 * 2;      // one half of a 64-row tile, 8 KB
-
-struct DkvSmem {
-    uint8_t k[2][kHalf128];
-    uint8_t v[2][kHalf128];
-    uint8_t q[kStages][2][kHalf64];
-    uint8_t da[kStages][2][kHalf64];
-    uint8_t pt[2][kHalf128];              // P^T  [128 keys x 64 queries] pair
-    uint8_t dst[2][kHalf128];             // dS^T pair
-    uint64_t kv_full, st_full, p_ready, pd_done, acc_done;
-    uint64_t qa_full[kStages], qa_empty[kStages];
-    uint32_t tmem;
-    int abort;
-};
-constexpr int kDkvSmem = (int)sizeof(DkvSmem) + 1024;
-
-struct DqSmem {
-    uint8_t q[2][kHalf128];
-    uint8_t da[2][kHalf128];
-    uint8_t k[kStages][2][kHalf64];
-    uint8_t v[kStages][2][kHalf64];
-    uint8_t ds[2][kHalf128];              // dS [128 queries x 64 keys] pair
-    uint64_t qa_full, sp_full, ds_ready, ds_done, acc_done;
-    uint64_t kv_full[kStages], kv_empty[kStages];
-    uint32_t tmem;
-    int abort;
-};
-constexpr int kDqSmem = (int)sizeof(DqSmem) + 1024;
-
 struct BwdParams {
     CUtensorMap mA0, mA1, mB0, mB1;   // dK/dV: K, V (128 rows), Q, dA (64 rows); dQ: Q, dA (128), K, V (64)
                                       // k <= 128: Q, K, V, dA as 3-D maps over [H, B*k, 128]
@@ -395,6 +341,7 @@ struct BwdParams {
     float scale, scale_log2;
     const float *lse, *Dd;            // [H, B*k]
     bf16 *dQKV;                       // [H, B*k, 512] pair: dQ|dK|dV|dlogit hi, then lo
+    float *dQacc;                     // k > 128: [H, B*k, 64] fp32 dQ accumulator (zeroed)
     uint32_t *status;
 };
 
@@ -404,337 +351,267 @@ __device__ __forceinline__ void flag_timeout_b(SM &sm, uint32_t *status) {
     *(volatile int *)&sm.abort = 1;
 }
 
-__device__ __forceinline__ void ld64(uint32_t taddr, float *v) {
-    float t32[32];
-    tmem_ld32(taddr, t32);
-#pragma unroll
-    for (int c = 0; c < 32; ++c) v[c] = t32[c];
-    tmem_ld32(taddr + 32, t32);
-#pragma unroll
-    for (int c = 0; c < 32; ++c) v[32 + c] = t32[c];
+
+
+// Backward for k > 128 (B2), one CTA per (128-key tile, b, h), 384 threads:
+// warps 0-3 load, issue MMAs and own TMEM; warps 4-11 compute P and dS, two
+// per TMEM lane quadrant (warp w: query rows 32 (w % 4) .. +31 of the current
+// block, keys 64 ((w - 4) / 4) .. +63 of the tile).  For each 128-query block
+// i at or after the tile (causal):
+//   S = Q_i K^T, dP = dA_i V^T                  (TMEM)
+//   P = exp(S / sqrt(h') - lse_i)               (pair tile; kept in registers)
+//   dV += P^T dA_i                              (TMEM, the tile read MN-major)
+//   dS = P o (dP - D_i)                         (pair tile, over P)
+//   dK += dS^T Q_i, dQ_i = dS K                 (TMEM)
+//   dQ_i / sqrt(h') is added into an fp32 accumulator [H, B*k, 64] with
+//   coalesced vector reductions (staged in the P / dS tile, idle by then);
+// dK / sqrt(h') and dV are written once at the end.  Q_i goes to slot i % 2
+// (it is needed until dK and dQ of block i), dA_i to slot 2 (free after dV),
+// so each load is issued at least half a block before its use.
+constexpr int kBT = 384;
+constexpr int kBWorkers = 256;
+constexpr int kBSlots = 3;
+
+struct BwdLargeSmem {
+    uint8_t k[2][kTileHalf];
+    uint8_t v[2][kTileHalf];
+    uint8_t ring[kBSlots][2][kTileHalf];   // Q_i or dA_i pairs
+    uint8_t ps[2][2][kTileHalf];           // P, then dS [half][64-key block]; dQ staging
+    uint64_t kv_full, ring_full[kBSlots], ring_empty[kBSlots];
+    uint64_t sp_full, p_ready, pv_done, ds_ready, dq_full, dq_empty, acc_done;
+    uint32_t tmem;
+    int abort;
+};
+constexpr int kBwdLargeSmem = (int)sizeof(BwdLargeSmem) + 1024;
+static_assert(kBwdLargeSmem <= 227 * 1024, "shared memory");
+
+__device__ __forceinline__ bool bwait(BwdLargeSmem &sm, uint64_t &bar, uint32_t parity, uint32_t *status) {
+    if (*(volatile int *)&sm.abort) return false;
+    if (mbar_wait(smem_u32(&bar), parity)) return true;
+    atomicOr(status, kStatusTimeout);
+    *(volatile int *)&sm.abort = 1;
+    return false;
 }
 
-// 64 values as a bf16 pair into a global row: hi at row[col_hi..], lo at row[col_lo..].
-__device__ __forceinline__ void store_pair64(bf16 *row, int col_hi, int col_lo, const float *v,
-                                             float f) {
-#pragma unroll
-    for (int c = 0; c < 64; c += 8) {
-        uint32_t h4[4], l4[4];
-#pragma unroll
-        for (int e = 0; e < 4; ++e) {
-            const float a = v[c + 2 * e] * f, b = v[c + 2 * e + 1] * f;
-            split_pair2(a, b, h4[e], l4[e]);
-        }
-        *reinterpret_cast<uint4 *>(row + col_hi + c) = make_uint4(h4[0], h4[1], h4[2], h4[3]);
-        *reinterpret_cast<uint4 *>(row + col_lo + c) = make_uint4(l4[0], l4[1], l4[2], l4[3]);
-    }
-}
-
-__global__ void __launch_bounds__(kThreads, 1) attn_dkv_tc_kernel(const __grid_constant__ BwdParams p) {
+__global__ void __launch_bounds__(kBT, 1) attn_bwd_tc_kernel(const __grid_constant__ BwdParams p) {
     extern __shared__ uint8_t smem_raw[];
-    DkvSmem &sm = *reinterpret_cast<DkvSmem *>(
+    BwdLargeSmem &sm = *reinterpret_cast<BwdLargeSmem *>(
         (reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-    const int jt = blockIdx.x, b = blockIdx.y, h = blockIdx.z;
-    const int j0 = jt * kKT;
-    const int qb_begin = j0 / kQB;                      // queries i >= j0
-    const int nq = (p.k + kQB - 1) / kQB - qb_begin;    // query blocks to visit
+    const int jt = blockIdx.x, b = blockIdx.y, h = blockIdx.z;   // tile 0 has the most blocks
+    const int j0 = jt * 128;
+    const int nqb = (p.k + 127) / 128;
+    const int nb = nqb - jt;                  // query blocks jt .. nqb-1
+    const size_t base = (size_t)h * p.Mtok + (size_t)b * p.k;
 
     if (threadIdx.x == 0) {
         mbar_init(smem_u32(&sm.kv_full), 1);
-        mbar_init(smem_u32(&sm.st_full), 1);
-        mbar_init(smem_u32(&sm.p_ready), 128);
-        mbar_init(smem_u32(&sm.pd_done), 1);
-        mbar_init(smem_u32(&sm.acc_done), 1);
-        for (int s = 0; s < kStages; ++s) {
-            mbar_init(smem_u32(&sm.qa_full[s]), 1);
-            mbar_init(smem_u32(&sm.qa_empty[s]), 1);
+        for (int s = 0; s < kBSlots; ++s) {
+            mbar_init(smem_u32(&sm.ring_full[s]), 1);
+            mbar_init(smem_u32(&sm.ring_empty[s]), 1);
         }
+        mbar_init(smem_u32(&sm.sp_full), 1);
+        mbar_init(smem_u32(&sm.p_ready), kBWorkers);
+        mbar_init(smem_u32(&sm.pv_done), 1);
+        mbar_init(smem_u32(&sm.ds_ready), kBWorkers);
+        mbar_init(smem_u32(&sm.dq_full), 1);
+        mbar_init(smem_u32(&sm.dq_empty), kBWorkers);
+        mbar_init(smem_u32(&sm.acc_done), 1);
         sm.abort = 0;
         fence_barrier_init();
     }
     if (warp == 2) {
-        tmem_alloc(smem_u32(&sm.tmem), 256);
+        tmem_alloc(smem_u32(&sm.tmem), 512);
         tmem_relinquish();
     }
     tc_fence_before();
     __syncthreads();
     tc_fence_after();
-    pdl_wait();  // Q, K, V, dA, lse written by the previous kernels
+    pdl_wait();  // Q, K, V, dA, lse, D written by the previous kernels
     const uint32_t tmem = sm.tmem;
-    const uint32_t tST = tmem, tDPT = tmem + 64, tDV = tmem + 128, tDK = tmem + 192;
+    const uint32_t tS = tmem, tDP = tmem + 128, tDV = tmem + 256, tDK = tmem + 320, tDQ = tmem + 384;
 
     if (warp == 0) {
         if (lane == 0) {
             const uint32_t kb = smem_u32(&sm.kv_full);
-            mbar_expect_tx(kb, 4 * kHalf128);
+            mbar_expect_tx(kb, 4 * kTileHalf);
             tma_load_4d(smem_u32(sm.k[0]), &p.mA0, kb, 0, j0, b, h);
             tma_load_4d(smem_u32(sm.k[1]), &p.mA0, kb, 64, j0, b, h);
             tma_load_4d(smem_u32(sm.v[0]), &p.mA1, kb, 0, j0, b, h);
             tma_load_4d(smem_u32(sm.v[1]), &p.mA1, kb, 64, j0, b, h);
-            int issued = 0;
-            for (int n = 0; n < nq; ++n) {
-                const int s = n % kStages;
-                if (!mbar_wait(smem_u32(&sm.qa_empty[s]), ((n / kStages) & 1) ^ 1) ||
-                    *(volatile int *)&sm.abort) {
-                    flag_timeout_b(sm, p.status);
-                    break;
-                }
-                const int i0 = (qb_begin + n) * kQB;
-                const uint32_t fb = smem_u32(&sm.qa_full[s]);
-                mbar_expect_tx(fb, 4 * kHalf64);
-                tma_load_4d(smem_u32(sm.q[s][0]), &p.mB0, fb, 0, i0, b, h);
-                tma_load_4d(smem_u32(sm.q[s][1]), &p.mB0, fb, 64, i0, b, h);
-                tma_load_4d(smem_u32(sm.da[s][0]), &p.mB1, fb, 0, i0, b, h);
-                tma_load_4d(smem_u32(sm.da[s][1]), &p.mB1, fb, 64, i0, b, h);
-                issued = n + 1;
-            }
-            if (*(volatile int *)&sm.abort) {
-                mbar_wait(kb, 0);
-                for (int n = max(0, issued - kStages); n < issued; ++n)
-                    mbar_wait(smem_u32(&sm.qa_full[n % kStages]), (n / kStages) & 1);
+            for (int t = 0; t < 2 * nb; ++t) {
+                const int i = t >> 1, is_da = t & 1;
+                const int s = is_da ? 2 : (i & 1);
+                const int use = is_da ? i : (i >> 1);   // earlier loads into this slot
+                if (!bwait(sm, sm.ring_empty[s], (use & 1) ^ 1, p.status)) break;
+                const int q0 = (jt + i) * 128;
+                const CUtensorMap *m = is_da ? &p.mB1 : &p.mB0;   // dA_i : Q_i
+                const uint32_t fb = smem_u32(&sm.ring_full[s]);
+                mbar_expect_tx(fb, 2 * kTileHalf);
+                tma_load_4d(smem_u32(sm.ring[s][0]), m, fb, 0, q0, b, h);
+                tma_load_4d(smem_u32(sm.ring[s][1]), m, fb, 64, q0, b, h);
             }
         }
     } else if (warp == 1) {
         if (lane == 0) {
-            constexpr uint32_t idKK = idesc_bf16(kKT, kQB, false, false);  // S^T, dP^T
-            constexpr uint32_t idKM = idesc_bf16(kKT, 64, false, true);    // dV, dK
-            bool ok = mbar_wait(smem_u32(&sm.kv_full), 0);
-            for (int n = 0; ok && n < nq; ++n) {
-                const int s = n % kStages;
-                if (!mbar_wait(smem_u32(&sm.qa_full[s]), (n / kStages) & 1) ||
-                    *(volatile int *)&sm.abort) {
-                    ok = false;
-                    break;
-                }
+            constexpr uint32_t idKK = idesc_bf16(128, 128, false, false);  // S, dP
+            constexpr uint32_t idMN = idesc_bf16(128, 64, true, true);     // dV, dK
+            constexpr uint32_t idKM = idesc_bf16(128, 64, false, true);    // dQ
+            bool ok = bwait(sm, sm.kv_full, 0, p.status);
+            const uint32_t k0 = smem_u32(sm.k[0]), k1 = smem_u32(sm.k[1]);
+            const uint32_t v0 = smem_u32(sm.v[0]), v1 = smem_u32(sm.v[1]);
+            for (int i = 0; i < nb && ok; ++i) {
+                const int sq = i & 1, sa = 2;
+                // S and dP of the previous block have been read by the workers
+                if (i > 0) ok = bwait(sm, sm.ds_ready, (i - 1) & 1, p.status);
+                ok = ok && bwait(sm, sm.ring_full[sq], (i >> 1) & 1, p.status);
+                if (!ok) break;
                 tc_fence_after();
-                const uint32_t q0 = smem_u32(sm.q[s][0]), q1 = smem_u32(sm.q[s][1]);
-                const uint32_t a0 = smem_u32(sm.da[s][0]), a1 = smem_u32(sm.da[s][1]);
-                mma_pair3(tST, smem_u32(sm.k[0]), smem_u32(sm.k[1]), q0, q1, false, false, idKK, false);
-                mma_pair3(tDPT, smem_u32(sm.v[0]), smem_u32(sm.v[1]), a0, a1, false, false, idKK, false);
-                mma_commit(smem_u32(&sm.st_full));
-                if (!mbar_wait(smem_u32(&sm.p_ready), n & 1) || *(volatile int *)&sm.abort) {
-                    ok = false;
-                    break;
-                }
+                const uint32_t q0 = smem_u32(sm.ring[sq][0]), q1 = smem_u32(sm.ring[sq][1]);
+                const uint32_t a0 = smem_u32(sm.ring[sa][0]), a1 = smem_u32(sm.ring[sa][1]);
+                mma_pair3(tS, q0, q1, k0, k1, false, false, idKK, false);    // S  = Q_i K^T
+                mma_commit(smem_u32(&sm.sp_full));
+                if (!(ok = bwait(sm, sm.ring_full[sa], i & 1, p.status))) break;
                 tc_fence_after();
-                mma_pair3(tDV, smem_u32(sm.pt[0]), smem_u32(sm.pt[1]), a0, a1, false, true, idKM, n > 0);
-                mma_pair3(tDK, smem_u32(sm.dst[0]), smem_u32(sm.dst[1]), q0, q1, false, true, idKM, n > 0);
-                mma_commit(smem_u32(&sm.qa_empty[s]));
-                mma_commit(smem_u32(&sm.pd_done));
+                mma_pair3(tDP, a0, a1, v0, v1, false, false, idKK, false);   // dP = dA_i V^T
+                if (!(ok = bwait(sm, sm.p_ready, i & 1, p.status))) break;
+                tc_fence_after();
+                mma_k128(tDV, sm.ps, sm.ring[sa], true, idMN, i > 0);        // dV += P^T dA_i
+                mma_commit(smem_u32(&sm.pv_done));                            // dP and dV done
+                mma_commit(smem_u32(&sm.ring_empty[sa]));
+                if (!(ok = bwait(sm, sm.ds_ready, i & 1, p.status))) break;
+                if (i > 0 && !(ok = bwait(sm, sm.dq_empty, (i - 1) & 1, p.status))) break;
+                tc_fence_after();
+                mma_k128(tDK, sm.ps, sm.ring[sq], true, idMN, i > 0);        // dK += dS^T Q_i
+                mma_k128(tDQ, sm.ps, sm.k, false, idKM);                     // dQ_i = dS K
+                mma_commit(smem_u32(&sm.dq_full));
+                mma_commit(smem_u32(&sm.ring_empty[sq]));
             }
             if (!ok) {
-                flag_timeout_b(sm, p.status);
-                mma_commit(smem_u32(&sm.st_full));
+                // release every wait of the workers that may still be pending
+                mma_commit(smem_u32(&sm.sp_full));
+                mma_commit(smem_u32(&sm.pv_done));
+                mma_commit(smem_u32(&sm.dq_full));
             }
             mma_commit(smem_u32(&sm.acc_done));
         }
     } else if (warp >= 4) {
         pdl_trigger();
-        const int q = warp - 4;
-        const int r = q * 32 + lane;
-        const int j = j0 + r;
+        const int q = warp & 3, ch = (warp - 4) >> 2;
+        const int r = q * 32 + lane;                  // query row of the block; key row at the end
         const uint32_t lane_off = (uint32_t)(q * 32) << 16;
-        const size_t base = (size_t)h * p.Mtok + (size_t)b * p.k;
+        uint8_t *xb = &sm.ps[0][0][0] + (warp - 4) * 4096;
         bool ok = true;
-        for (int n = 0; n < nq; ++n) {
-            if (!mbar_wait(smem_u32(&sm.st_full), n & 1) || *(volatile int *)&sm.abort) {
-                ok = false;
-                break;
-            }
+        for (int i = 0; i < nb; ++i) {
+            const int qi = (jt + i) * 128 + r;        // query index
+            const bool valid = qi < p.k;
+            const float l2 = valid ? __ldg(p.lse + base + qi) * 1.4426950408889634f : 0.f;
+            const float dd = valid ? __ldg(p.Dd + base + qi) : 0.f;
+            ok = bwait(sm, sm.sp_full, i & 1, p.status) && ok;
             tc_fence_after();
-            float st[64], dpt[64];
-            ld64(tST + lane_off, st);
-            ld64(tDPT + lane_off, dpt);
-            const int i0 = (qb_begin + n) * kQB;
+            // P over this thread's 64 keys (the diagonal block i = 0 is causal)
+            float pv[64];
+            {
+                float t32[32];
+                tmem_ld32(tS + lane_off + 64 * ch, t32);
 #pragma unroll
-            for (int c = 0; c < 64; ++c) {
-                const int i = i0 + c;
-                const bool allowed = (i >= j) && (i < p.k);
-                const float l2 = allowed ? __ldg(p.lse + base + i) * 1.4426950408889634f : 0.f;
-                const float dd = allowed ? __ldg(p.Dd + base + i) : 0.f;
-                const float pr = allowed ? exp2_fast(st[c] * p.scale_log2 - l2) : 0.f;
-                st[c] = pr;
-                dpt[c] = pr * (dpt[c] - dd);
+                for (int c = 0; c < 32; ++c) pv[c] = t32[c];
+                tmem_ld32(tS + lane_off + 64 * ch + 32, t32);
+#pragma unroll
+                for (int c = 0; c < 32; ++c) pv[32 + c] = t32[c];
             }
-            if (n > 0 && !mbar_wait(smem_u32(&sm.pd_done), (n - 1) & 1)) {
-                ok = false;
-                break;
-            }
-            write_pair_row64(sm.pt[0], sm.pt[1], r, st);
-            write_pair_row64(sm.dst[0], sm.dst[1], r, dpt);
+            const int lim = (i == 0) ? r - 64 * ch : 127;   // visible key offsets c <= lim
+#pragma unroll
+            for (int c = 0; c < 64; ++c)
+                pv[c] = (valid && c <= lim) ? exp2_fast(fmaf(pv[c], p.scale_log2, -l2)) : 0.f;
+            write_pair32(sm.ps, r, 64 * ch, pv);
+            write_pair32(sm.ps, r, 64 * ch + 32, pv + 32);
             fence_proxy_async();
             tc_fence_before();
             mbar_arrive(smem_u32(&sm.p_ready));
-        }
-        const bool done = mbar_wait(smem_u32(&sm.acc_done), 0);
-        tc_fence_after();
-        float dv[64], dk[64];
-        ld64(tDV + lane_off, dv);
-        ld64(tDK + lane_off, dk);
-        if (!ok || !done) flag_timeout_b(sm, p.status);
-        if (ok && done && j < p.k && nq > 0 && !*(volatile int *)&sm.abort) {
-            bf16 *row = p.dQKV + (base + j) * 512;
-            store_pair64(row, 64, 320, dk, p.scale);
-            store_pair64(row, 128, 384, dv, 1.f);
-        }
-    }
-    tc_fence_before();
-    __syncthreads();
-    if (warp == 2) {
-        tc_fence_after();
-        tmem_dealloc(tmem, 256);
-    }
-}
-
-__global__ void __launch_bounds__(kThreads, 1) attn_dq_tc_kernel(const __grid_constant__ BwdParams p) {
-    extern __shared__ uint8_t smem_raw[];
-    DqSmem &sm = *reinterpret_cast<DqSmem *>(
-        (reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
-    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-    const int qt = blockIdx.x, b = blockIdx.y, h = blockIdx.z;
-    const int i0 = qt * kQ;
-    const int q_end = min(p.k, i0 + kQ);
-    const int nblk = (q_end + kKV - 1) / kKV;
-
-    if (threadIdx.x == 0) {
-        mbar_init(smem_u32(&sm.qa_full), 1);
-        mbar_init(smem_u32(&sm.sp_full), 1);
-        mbar_init(smem_u32(&sm.ds_ready), 128);
-        mbar_init(smem_u32(&sm.ds_done), 1);
-        mbar_init(smem_u32(&sm.acc_done), 1);
-        for (int s = 0; s < kStages; ++s) {
-            mbar_init(smem_u32(&sm.kv_full[s]), 1);
-            mbar_init(smem_u32(&sm.kv_empty[s]), 1);
-        }
-        sm.abort = 0;
-        fence_barrier_init();
-    }
-    if (warp == 2) {
-        tmem_alloc(smem_u32(&sm.tmem), 256);
-        tmem_relinquish();
-    }
-    tc_fence_before();
-    __syncthreads();
-    tc_fence_after();
-    pdl_wait();  // Q, K, V, dA, lse written by the previous kernels
-    const uint32_t tmem = sm.tmem;
-    const uint32_t tS = tmem, tDP = tmem + 64, tDQ = tmem + 128;
-
-    if (warp == 0) {
-        if (lane == 0) {
-            const uint32_t qb = smem_u32(&sm.qa_full);
-            mbar_expect_tx(qb, 4 * kHalf128);
-            tma_load_4d(smem_u32(sm.q[0]), &p.mA0, qb, 0, i0, b, h);
-            tma_load_4d(smem_u32(sm.q[1]), &p.mA0, qb, 64, i0, b, h);
-            tma_load_4d(smem_u32(sm.da[0]), &p.mA1, qb, 0, i0, b, h);
-            tma_load_4d(smem_u32(sm.da[1]), &p.mA1, qb, 64, i0, b, h);
-            int issued = 0;
-            for (int n = 0; n < nblk; ++n) {
-                const int s = n % kStages;
-                if (!mbar_wait(smem_u32(&sm.kv_empty[s]), ((n / kStages) & 1) ^ 1) ||
-                    *(volatile int *)&sm.abort) {
-                    flag_timeout_b(sm, p.status);
-                    break;
-                }
-                const uint32_t fb = smem_u32(&sm.kv_full[s]);
-                mbar_expect_tx(fb, 4 * kHalf64);
-                tma_load_4d(smem_u32(sm.k[s][0]), &p.mB0, fb, 0, n * kKV, b, h);
-                tma_load_4d(smem_u32(sm.k[s][1]), &p.mB0, fb, 64, n * kKV, b, h);
-                tma_load_4d(smem_u32(sm.v[s][0]), &p.mB1, fb, 0, n * kKV, b, h);
-                tma_load_4d(smem_u32(sm.v[s][1]), &p.mB1, fb, 64, n * kKV, b, h);
-                issued = n + 1;
-            }
-            if (*(volatile int *)&sm.abort) {
-                mbar_wait(qb, 0);
-                for (int n = max(0, issued - kStages); n < issued; ++n)
-                    mbar_wait(smem_u32(&sm.kv_full[n % kStages]), (n / kStages) & 1);
-            }
-        }
-    } else if (warp == 1) {
-        if (lane == 0) {
-            constexpr uint32_t idKK = idesc_bf16(kQ, kKV, false, false);  // S, dP
-            constexpr uint32_t idKM = idesc_bf16(kQ, 64, false, true);    // dQ
-            bool ok = mbar_wait(smem_u32(&sm.qa_full), 0);
-            for (int n = 0; ok && n < nblk; ++n) {
-                const int s = n % kStages;
-                if (!mbar_wait(smem_u32(&sm.kv_full[s]), (n / kStages) & 1) ||
-                    *(volatile int *)&sm.abort) {
-                    ok = false;
-                    break;
-                }
-                tc_fence_after();
-                const uint32_t k0 = smem_u32(sm.k[s][0]), k1 = smem_u32(sm.k[s][1]);
-                const uint32_t v0 = smem_u32(sm.v[s][0]), v1 = smem_u32(sm.v[s][1]);
-                mma_pair3(tS, smem_u32(sm.q[0]), smem_u32(sm.q[1]), k0, k1, false, false, idKK, false);
-                mma_pair3(tDP, smem_u32(sm.da[0]), smem_u32(sm.da[1]), v0, v1, false, false, idKK, false);
-                mma_commit(smem_u32(&sm.sp_full));
-                if (!mbar_wait(smem_u32(&sm.ds_ready), n & 1) || *(volatile int *)&sm.abort) {
-                    ok = false;
-                    break;
-                }
-                tc_fence_after();
-                mma_pair3(tDQ, smem_u32(sm.ds[0]), smem_u32(sm.ds[1]), k0, k1, false, true, idKM, n > 0);
-                mma_commit(smem_u32(&sm.kv_empty[s]));
-                mma_commit(smem_u32(&sm.ds_done));
-            }
-            if (!ok) {
-                flag_timeout_b(sm, p.status);
-                mma_commit(smem_u32(&sm.sp_full));
-            }
-            mma_commit(smem_u32(&sm.acc_done));
-        }
-    } else if (warp >= 4) {
-        pdl_trigger();
-        const int q = warp - 4;
-        const int r = q * 32 + lane;
-        const int i = i0 + r;
-        const uint32_t lane_off = (uint32_t)(q * 32) << 16;
-        const size_t base = (size_t)h * p.Mtok + (size_t)b * p.k;
-        const float l2 = i < p.k ? p.lse[base + i] * 1.4426950408889634f : 0.f;
-        const float dd = i < p.k ? p.Dd[base + i] : 0.f;
-        bool ok = true;
-        for (int n = 0; n < nblk; ++n) {
-            if (!mbar_wait(smem_u32(&sm.sp_full), n & 1) || *(volatile int *)&sm.abort) {
-                ok = false;
-                break;
-            }
+            // dS = P o (dP - D), over P once dV has read it
+            ok = bwait(sm, sm.pv_done, i & 1, p.status) && ok;
             tc_fence_after();
-            float sv[64], dp[64];
-            ld64(tS + lane_off, sv);
-            ld64(tDP + lane_off, dp);
-            const int jb = n * kKV;
+            {
+                float t32[32];
+                tmem_ld32(tDP + lane_off + 64 * ch, t32);
 #pragma unroll
-            for (int c = 0; c < 64; ++c) {
-                const bool allowed = (jb + c <= i);
-                const float pr = allowed ? exp2_fast(sv[c] * p.scale_log2 - l2) : 0.f;
-                dp[c] = pr * (dp[c] - dd);
+                for (int c = 0; c < 32; ++c) pv[c] *= t32[c] - dd;
+                tmem_ld32(tDP + lane_off + 64 * ch + 32, t32);
+#pragma unroll
+                for (int c = 0; c < 32; ++c) pv[32 + c] *= t32[c] - dd;
             }
-            if (n > 0 && !mbar_wait(smem_u32(&sm.ds_done), (n - 1) & 1)) {
-                ok = false;
-                break;
-            }
-            write_pair_row64(sm.ds[0], sm.ds[1], r, dp);
+            write_pair32(sm.ps, r, 64 * ch, pv);
+            write_pair32(sm.ps, r, 64 * ch + 32, pv + 32);
             fence_proxy_async();
             tc_fence_before();
             mbar_arrive(smem_u32(&sm.ds_ready));
+            // dQ_i into the fp32 accumulator (columns 32 ch .. +31 of this row)
+            ok = bwait(sm, sm.dq_full, i & 1, p.status) && ok;
+            tc_fence_after();
+            float dq[32];
+            tmem_ld32(tDQ + lane_off + 32 * ch, dq);
+            tc_fence_before();
+            mbar_arrive(smem_u32(&sm.dq_empty));
+            const bool live = __all_sync(0xffffffffu, ok && !*(volatile int *)&sm.abort);
+            const unsigned vmask = __ballot_sync(0xffffffffu, valid);
+            if (live) {
+                stage_f32x32(xb, dq, p.scale, lane);
+                const int cu = lane & 7;
+                const size_t row0 = base + (size_t)(jt + i) * 128 + q * 32;
+#pragma unroll
+                for (int e = 0; e < 8; ++e) {
+                    const int rl = (lane >> 3) + 4 * e;
+                    const float4 val = *reinterpret_cast<const float4 *>(xb + xoff128(rl, cu));
+                    if ((vmask >> rl) & 1u)
+                        red_add_v4(p.dQacc + (row0 + rl) * 64 + 32 * ch + 4 * cu, val.x, val.y, val.z, val.w);
+                }
+            }
+            named_barrier(1, kBWorkers);   // staging reads done before the next P is written
         }
-        const bool done = mbar_wait(smem_u32(&sm.acc_done), 0);
+        // dK / sqrt(h') and dV of the tile's keys (row r = key j0 + r)
+        const bool done = bwait(sm, sm.acc_done, 0, p.status);
         tc_fence_after();
-        float dq[64];
-        ld64(tDQ + lane_off, dq);
-        if (!ok || !done) flag_timeout_b(sm, p.status);
-        if (ok && done && i < p.k && nblk > 0 && !*(volatile int *)&sm.abort) {
-            bf16 *row = p.dQKV + (base + i) * 512;
-            store_pair64(row, 0, 256, dq, p.scale);
+        const int kj = j0 + r;
+        const unsigned kmask = __ballot_sync(0xffffffffu, kj < p.k);
+        const bool live = __all_sync(0xffffffffu, ok && done && !*(volatile int *)&sm.abort) && nb > 0;
+        const uint32_t src[2] = {tDK, tDV};
+        const float fac[2] = {p.scale, 1.f};
+#pragma unroll
+        for (int t = 0; t < 2; ++t) {
+            float v[32];
+            tmem_ld32(src[t] + lane_off + 32 * ch, v);
+            if (!live) continue;
+            stage_pair32(xb, v, fac[t], lane);
+            store_rows128(xb, lane, [&](int rl, int c) -> uint4 * {
+                if (!((kmask >> rl) & 1u)) return nullptr;
+                bf16 *row = p.dQKV + (base + j0 + q * 32 + rl) * 512 + 64 * (t + 1) + 32 * ch;
+                return c < 4 ? reinterpret_cast<uint4 *>(row) + c
+                             : reinterpret_cast<uint4 *>(row + 256) + (c - 4);
+            });
         }
     }
     tc_fence_before();
     __syncthreads();
     if (warp == 2) {
         tc_fence_after();
-        tmem_dealloc(tmem, 256);
+        tmem_dealloc(tmem, 512);
     }
+}
+
+// dQ from its fp32 accumulator into columns 0..63 (hi) / 256..319 (lo) of the
+// dQKV pair rows, two columns per thread.
+__global__ void dq_finish_kernel(const float *__restrict__ dQacc, bf16 *__restrict__ dQKV, size_t rows) {
+    pdl_wait();
+    const size_t idx = (size_t)blockIdx.x * blockDim.x + threadIdx.x;   // (row, column pair)
+    if (idx >= rows * 32) return;
+    const size_t row = idx >> 5;
+    const int c = (int)(idx & 31) * 2;
+    const float2 v = *reinterpret_cast<const float2 *>(dQacc + row * 64 + c);
+    uint32_t hi, lo;
+    split_pair2(v.x, v.y, hi, lo);
+    *reinterpret_cast<uint32_t *>(dQKV + row * 512 + c) = hi;
+    *reinterpret_cast<uint32_t *>(dQKV + row * 512 + 256 + c) = lo;
 }
 
 // ------------------------------------------------- k <= 128: one CTA per tile
@@ -1169,39 +1046,40 @@ cudaError_t tc_attn_bwd(const Dims &dm, const Saved &sv, cudaStream_t s) {
         note_launches(1);
         return e;
     }
-    bool ok = map_units(&kv.mA0, sv.K, dm.H, dm.B, dm.k, kKT) &&
-              map_units(&kv.mA1, sv.V, dm.H, dm.B, dm.k, kKT) &&
-              map_units(&kv.mB0, sv.Q, dm.H, dm.B, dm.k, kQB) &&
-              map_units(&kv.mB1, sv.dA, dm.H, dm.B, dm.k, kQB) &&
-              map_units(&dq.mA0, sv.Q, dm.H, dm.B, dm.k, kQ) &&
-              map_units(&dq.mA1, sv.dA, dm.H, dm.B, dm.k, kQ) &&
-              map_units(&dq.mB0, sv.K, dm.H, dm.B, dm.k, kKV) &&
-              map_units(&dq.mB1, sv.V, dm.H, dm.B, dm.k, kKV);
+    // k > 128: one CTA per 128-key tile; dQ accumulates in fp32 (the
+    // workspace's G buffer, unused on this path) and is split into pairs after
+    BwdParams bp;
+    memset(&bp, 0, sizeof(bp));
+    bool ok = map_units(&bp.mA0, sv.K, dm.H, dm.B, dm.k, 128) &&
+              map_units(&bp.mA1, sv.V, dm.H, dm.B, dm.k, 128) &&
+              map_units(&bp.mB0, sv.Q, dm.H, dm.B, dm.k, 128) &&
+              map_units(&bp.mB1, sv.dA, dm.H, dm.B, dm.k, 128);
     if (!ok) return cudaErrorInvalidValue;
-    for (BwdParams *p : {&kv, &dq}) {
-        p->k = dm.k;
-        p->Mtok = dm.B * dm.k;
-        p->scale = 1.f / sqrtf(64.f);
-        p->scale_log2 = 1.4426950408889634f / sqrtf(64.f);
-        p->lse = sv.lse;
-        p->Dd = sv.Dd;
-        p->dQKV = static_cast<bf16 *>(sv.dQKV);
-        p->status = sv.status;
-    }
+    bp.k = dm.k;
+    bp.Mtok = dm.B * dm.k;
+    bp.scale = 1.f / sqrtf(64.f);
+    bp.scale_log2 = 1.4426950408889634f / sqrtf(64.f);
+    bp.lse = sv.lse;
+    bp.Dd = sv.Dd;
+    bp.dQKV = static_cast<bf16 *>(sv.dQKV);
+    bp.dQacc = sv.G;
+    bp.status = sv.status;
+    const size_t rows = (size_t)dm.H * dm.B * dm.k;
     static std::once_flag once;
     static cudaError_t attr = cudaSuccess;
     std::call_once(once, [] {
-        attr = cudaFuncSetAttribute(attn_dkv_tc_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                    kDkvSmem);
-        if (attr == cudaSuccess)
-            attr = cudaFuncSetAttribute(attn_dq_tc_kernel,
-                                        cudaFuncAttributeMaxDynamicSharedMemorySize, kDqSmem);
+        attr = cudaFuncSetAttribute(attn_bwd_tc_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                    kBwdLargeSmem);
     });
     if (attr != cudaSuccess) return attr;
-    dim3 gkv((dm.k + kKT - 1) / kKT, dm.B, dm.H);
-    cudaError_t e = launch_pdl(attn_dkv_tc_kernel, gkv, dim3(kThreads), kDkvSmem, s, kv);
-    dim3 gq((dm.k + kQ - 1) / kQ, dm.B, dm.H);
-    if (e == cudaSuccess) e = launch_pdl(attn_dq_tc_kernel, gq, dim3(kThreads), kDqSmem, s, dq);
+    cudaError_t e = cudaMemsetAsync(sv.G, 0, sizeof(float) * rows * 64, s);
+    if (e != cudaSuccess) return e;
+    dim3 grid((dm.k + 127) / 128, dm.B, dm.H);
+    e = launch_pdl(attn_bwd_tc_kernel, grid, dim3(kBT), kBwdLargeSmem, s, bp);
+    const size_t n = rows * 32;
+    if (e == cudaSuccess)
+        e = launch_pdl(dq_finish_kernel, dim3((unsigned)((n + 255) / 256)), dim3(256), 0, s,
+                       (const float *)sv.G, static_cast<bf16 *>(sv.dQKV), rows);
     note_launches(2);
     return e;
 }

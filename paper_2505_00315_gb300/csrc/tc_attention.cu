@@ -108,9 +108,10 @@ __global__ void __launch_bounds__(kLT, 1) attn_fwd_tc_kernel(const __grid_consta
     FwdLargeSmem &sm = *reinterpret_cast<FwdLargeSmem *>(
         (reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-    // heaviest (last) query tiles first: they visit the most key blocks
-    const int nqt = gridDim.x;
-    const int qt = nqt - 1 - (int)blockIdx.x, b = blockIdx.y, h = blockIdx.z;
+    // heaviest (last) query tiles first: they visit the most key blocks; the
+    // tile index is the grid's slowest dimension, so CTAs start in that order
+    const int nqt = gridDim.z;
+    const int qt = nqt - 1 - (int)blockIdx.z, b = blockIdx.x, h = blockIdx.y;
     const int i0 = qt * kQ;
     const int n = qt + 1;                      // causal: key blocks 0 .. qt
     const int nitems = 2 * n;
@@ -364,7 +365,9 @@ __device__ __forceinline__ void flag_timeout_b(SM &sm, uint32_t *status) {
 //   dS = P o (dP - D_i)                         (pair tile, over P)
 //   dK += dS^T Q_i, dQ_i = dS K                 (TMEM)
 //   dQ_i / sqrt(h') is added into an fp32 accumulator [H, B*k, 64] with
-//   coalesced vector reductions (staged in the P / dS tile, idle by then);
+//   vector reductions issued after the next block's P has been stored;
+// S_{i+1} is issued before dK_i and dQ_i, so the exponentials of block i+1
+// run on the workers while the tensor pipe works on block i;
 // dK / sqrt(h') and dV are written once at the end.  Q_i goes to slot i % 2
 // (it is needed until dK and dQ of block i), dA_i to slot 2 (free after dV),
 // so each load is issued at least half a block before its use.
@@ -398,7 +401,9 @@ __global__ void __launch_bounds__(kBT, 1) attn_bwd_tc_kernel(const __grid_consta
     BwdLargeSmem &sm = *reinterpret_cast<BwdLargeSmem *>(
         (reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-    const int jt = blockIdx.x, b = blockIdx.y, h = blockIdx.z;   // tile 0 has the most blocks
+    // key tile 0 visits the most query blocks; the tile index is the grid's
+    // slowest dimension, so CTAs start heaviest first
+    const int jt = blockIdx.z, b = blockIdx.x, h = blockIdx.y;
     const int j0 = jt * 128;
     const int nqb = (p.k + 127) / 128;
     const int nb = nqb - jt;                  // query blocks jt .. nqb-1
@@ -460,32 +465,42 @@ __global__ void __launch_bounds__(kBT, 1) attn_bwd_tc_kernel(const __grid_consta
             bool ok = bwait(sm, sm.kv_full, 0, p.status);
             const uint32_t k0 = smem_u32(sm.k[0]), k1 = smem_u32(sm.k[1]);
             const uint32_t v0 = smem_u32(sm.v[0]), v1 = smem_u32(sm.v[1]);
-            for (int i = 0; i < nb && ok; ++i) {
-                const int sq = i & 1, sa = 2;
-                // S and dP of the previous block have been read by the workers
-                if (i > 0) ok = bwait(sm, sm.ds_ready, (i - 1) & 1, p.status);
-                ok = ok && bwait(sm, sm.ring_full[sq], (i >> 1) & 1, p.status);
-                if (!ok) break;
+            // S_i = Q_i K^T (needs Q_i in slot i % 2), dP_i = dA_i V^T (dA_i in slot 2)
+            auto issue_s = [&](int i) {
+                ok = ok && bwait(sm, sm.ring_full[i & 1], (i >> 1) & 1, p.status);
+                if (!ok) return;
                 tc_fence_after();
-                const uint32_t q0 = smem_u32(sm.ring[sq][0]), q1 = smem_u32(sm.ring[sq][1]);
-                const uint32_t a0 = smem_u32(sm.ring[sa][0]), a1 = smem_u32(sm.ring[sa][1]);
-                mma_pair3(tS, q0, q1, k0, k1, false, false, idKK, false);    // S  = Q_i K^T
+                mma_pair3(tS, smem_u32(sm.ring[i & 1][0]), smem_u32(sm.ring[i & 1][1]), k0, k1, false,
+                          false, idKK, false);
                 mma_commit(smem_u32(&sm.sp_full));
-                if (!(ok = bwait(sm, sm.ring_full[sa], i & 1, p.status))) break;
+            };
+            auto issue_dp = [&](int i) {
+                ok = ok && bwait(sm, sm.ring_full[2], i & 1, p.status);
+                if (!ok) return;
                 tc_fence_after();
-                mma_pair3(tDP, a0, a1, v0, v1, false, false, idKK, false);   // dP = dA_i V^T
+                mma_pair3(tDP, smem_u32(sm.ring[2][0]), smem_u32(sm.ring[2][1]), v0, v1, false, false,
+                          idKK, false);
+            };
+            issue_s(0);
+            issue_dp(0);
+            for (int i = 0; i < nb && ok; ++i) {
                 if (!(ok = bwait(sm, sm.p_ready, i & 1, p.status))) break;
                 tc_fence_after();
-                mma_k128(tDV, sm.ps, sm.ring[sa], true, idMN, i > 0);        // dV += P^T dA_i
-                mma_commit(smem_u32(&sm.pv_done));                            // dP and dV done
-                mma_commit(smem_u32(&sm.ring_empty[sa]));
+                mma_k128(tDV, sm.ps, sm.ring[2], true, idMN, i > 0);          // dV += P^T dA_i
+                mma_commit(smem_u32(&sm.pv_done));                            // dP_i and dV done
+                mma_commit(smem_u32(&sm.ring_empty[2]));
                 if (!(ok = bwait(sm, sm.ds_ready, i & 1, p.status))) break;
-                if (i > 0 && !(ok = bwait(sm, sm.dq_empty, (i - 1) & 1, p.status))) break;
+                // S and dP of block i have been read: the next S goes first so
+                // that its P is computed while dK and dQ of this block run
+                if (i + 1 < nb) issue_s(i + 1);
+                if (i > 0) ok = ok && bwait(sm, sm.dq_empty, (i - 1) & 1, p.status);
+                if (!ok) break;
                 tc_fence_after();
-                mma_k128(tDK, sm.ps, sm.ring[sq], true, idMN, i > 0);        // dK += dS^T Q_i
-                mma_k128(tDQ, sm.ps, sm.k, false, idKM);                     // dQ_i = dS K
+                mma_k128(tDK, sm.ps, sm.ring[i & 1], true, idMN, i > 0);     // dK += dS^T Q_i
+                mma_k128(tDQ, sm.ps, sm.k, false, idKM);                      // dQ_i = dS K
                 mma_commit(smem_u32(&sm.dq_full));
-                mma_commit(smem_u32(&sm.ring_empty[sq]));
+                mma_commit(smem_u32(&sm.ring_empty[i & 1]));
+                if (i + 1 < nb) issue_dp(i + 1);
             }
             if (!ok) {
                 // release every wait of the workers that may still be pending
@@ -502,6 +517,24 @@ __global__ void __launch_bounds__(kBT, 1) attn_bwd_tc_kernel(const __grid_consta
         const uint32_t lane_off = (uint32_t)(q * 32) << 16;
         uint8_t *xb = &sm.ps[0][0][0] + (warp - 4) * 4096;
         bool ok = true;
+        // dQ of block i (dK and dQ done) into the fp32 accumulator: columns
+        // 32 ch .. +31 of this thread's row, eight 16-byte vector reductions
+        // straight from registers (they run while the next block's dV does)
+        auto drain_dq = [&](int i) {
+            float dq[32];
+            tmem_ld32(tDQ + lane_off + 32 * ch, dq);
+            tc_fence_before();
+            mbar_arrive(smem_u32(&sm.dq_empty));
+            const bool live = __all_sync(0xffffffffu, ok && !*(volatile int *)&sm.abort);
+            const int qi = (jt + i) * 128 + r;
+            if (live && qi < p.k) {
+                float *dst = p.dQacc + (base + qi) * 64 + 32 * ch;
+#pragma unroll
+                for (int c = 0; c < 32; c += 4)
+                    red_add_v4(dst + c, dq[c] * p.scale, dq[c + 1] * p.scale, dq[c + 2] * p.scale,
+                               dq[c + 3] * p.scale);
+            }
+        };
         for (int i = 0; i < nb; ++i) {
             const int qi = (jt + i) * 128 + r;        // query index
             const bool valid = qi < p.k;
@@ -524,11 +557,17 @@ __global__ void __launch_bounds__(kBT, 1) attn_bwd_tc_kernel(const __grid_consta
 #pragma unroll
             for (int c = 0; c < 64; ++c)
                 pv[c] = (valid && c <= lim) ? exp2_fast(fmaf(pv[c], p.scale_log2, -l2)) : 0.f;
+            // the tile holds dS of the previous block until its dK and dQ are done
+            if (i > 0) {
+                ok = bwait(sm, sm.dq_full, (i - 1) & 1, p.status) && ok;
+                tc_fence_after();
+            }
             write_pair32(sm.ps, r, 64 * ch, pv);
             write_pair32(sm.ps, r, 64 * ch + 32, pv + 32);
             fence_proxy_async();
             tc_fence_before();
             mbar_arrive(smem_u32(&sm.p_ready));
+            if (i > 0) drain_dq(i - 1);
             // dS = P o (dP - D), over P once dV has read it
             ok = bwait(sm, sm.pv_done, i & 1, p.status) && ok;
             tc_fence_after();
@@ -546,29 +585,10 @@ __global__ void __launch_bounds__(kBT, 1) attn_bwd_tc_kernel(const __grid_consta
             fence_proxy_async();
             tc_fence_before();
             mbar_arrive(smem_u32(&sm.ds_ready));
-            // dQ_i into the fp32 accumulator (columns 32 ch .. +31 of this row)
-            ok = bwait(sm, sm.dq_full, i & 1, p.status) && ok;
-            tc_fence_after();
-            float dq[32];
-            tmem_ld32(tDQ + lane_off + 32 * ch, dq);
-            tc_fence_before();
-            mbar_arrive(smem_u32(&sm.dq_empty));
-            const bool live = __all_sync(0xffffffffu, ok && !*(volatile int *)&sm.abort);
-            const unsigned vmask = __ballot_sync(0xffffffffu, valid);
-            if (live) {
-                stage_f32x32(xb, dq, p.scale, lane);
-                const int cu = lane & 7;
-                const size_t row0 = base + (size_t)(jt + i) * 128 + q * 32;
-#pragma unroll
-                for (int e = 0; e < 8; ++e) {
-                    const int rl = (lane >> 3) + 4 * e;
-                    const float4 val = *reinterpret_cast<const float4 *>(xb + xoff128(rl, cu));
-                    if ((vmask >> rl) & 1u)
-                        red_add_v4(p.dQacc + (row0 + rl) * 64 + 32 * ch + 4 * cu, val.x, val.y, val.z, val.w);
-                }
-            }
-            named_barrier(1, kBWorkers);   // staging reads done before the next P is written
         }
+        ok = bwait(sm, sm.dq_full, (nb - 1) & 1, p.status) && ok;
+        tc_fence_after();
+        drain_dq(nb - 1);
         // dK / sqrt(h') and dV of the tile's keys (row r = key j0 + r)
         const bool done = bwait(sm, sm.acc_done, 0, p.status);
         tc_fence_after();
@@ -1006,7 +1026,7 @@ cudaError_t tc_attn_fwd(const Dims &dm, const Saved &sv, cudaStream_t s) {
         note_launches(1);
         return e;
     }
-    dim3 grid((dm.k + kQ - 1) / kQ, dm.B, dm.H);
+    dim3 grid(dm.B, dm.H, (dm.k + kQ - 1) / kQ);   // query tiles slowest (see the kernel)
     cudaError_t e = launch_pdl(attn_fwd_tc_kernel, grid, dim3(kLT), kFwdLargeSmem, s, p);
     note_launches(1);
     return e;
@@ -1074,7 +1094,7 @@ cudaError_t tc_attn_bwd(const Dims &dm, const Saved &sv, cudaStream_t s) {
     if (attr != cudaSuccess) return attr;
     cudaError_t e = cudaMemsetAsync(sv.G, 0, sizeof(float) * rows * 64, s);
     if (e != cudaSuccess) return e;
-    dim3 grid((dm.k + 127) / 128, dm.B, dm.H);
+    dim3 grid(dm.B, dm.H, (dm.k + 127) / 128);   // key tiles slowest (see the kernel)
     e = launch_pdl(attn_bwd_tc_kernel, grid, dim3(kBT), kBwdLargeSmem, s, bp);
     const size_t n = rows * 32;
     if (e == cudaSuccess)

@@ -7,6 +7,8 @@
 // every key above it plus the lowest-index keys equal to it, so I comes out
 // ascending (the order the causal mask works in) and ties go to the lower
 // token index.  Block-wide ranks use warp ballots, so no sort is needed.
+#include <mutex>
+
 #include "launch.h"
 #include "profile.h"
 #include "simt_gemm.cuh"
@@ -37,7 +39,10 @@ __device__ __forceinline__ uint32_t order_key(float f) {
     return (u & 0x80000000u) ? ~u : (u | 0x80000000u);
 }
 
-constexpr int kSelThreads = 1024;
+constexpr int kSelThreads = 1024;   // upper bound; launches use 256 or 1024
+// Rows up to this many scores keep their order keys in shared memory for all
+// five passes over them (four radix passes and the compaction).
+constexpr int kSelStagedMax = 16384;
 
 // Exclusive rank of this thread among the block's threads with `flag` set,
 // in thread order; `total` receives the block-wide count.  sh has 33 words.
@@ -65,10 +70,13 @@ __device__ __forceinline__ uint32_t block_rank(bool flag, uint32_t *sh, uint32_t
     return r;
 }
 
+// One CTA per row: 1024 threads when rows are long or few (the CTA's own
+// latency decides), 256 when many short rows fill the GPU several times over.
 __global__ void __launch_bounds__(kSelThreads)
 topk_select_kernel(const float *__restrict__ scores, int T, int k, int32_t *__restrict__ I,
                    float *__restrict__ rsel, int B, int H, int32_t *__restrict__ gidx,
                    float *__restrict__ rsel_hm) {
+    extern __shared__ uint32_t keys_s[];   // the row's order keys when T <= kSelStagedMax
     __shared__ uint32_t hist[256];
     __shared__ uint32_t sh[33];
     __shared__ uint32_t sh_prefix, sh_remaining;
@@ -76,15 +84,22 @@ topk_select_kernel(const float *__restrict__ scores, int T, int k, int32_t *__re
     const int row = blockIdx.x;
     const float *s = scores + (size_t)row * T;
     const int tid = threadIdx.x;
+    const bool staged = T <= kSelStagedMax;
+    if (staged) {
+        for (int t = tid; t < T; t += blockDim.x) keys_s[t] = order_key(__ldg(s + t));
+        __syncthreads();
+    }
+    auto key_at = [&](int t) -> uint32_t { return staged ? keys_s[t] : order_key(__ldg(s + t)); };
 
     uint32_t prefix = 0u, mask = 0u, remaining = (uint32_t)k;
     for (int pass = 0; pass < 4; ++pass) {
         const int shift = 24 - 8 * pass;
+        const uint32_t digit = 255u;
         for (int i = tid; i < 256; i += blockDim.x) hist[i] = 0u;
         __syncthreads();
         for (int t = tid; t < T; t += blockDim.x) {
-            const uint32_t key = order_key(__ldg(s + t));
-            if ((key & mask) == prefix) atomicAdd(&hist[(key >> shift) & 255u], 1u);
+            const uint32_t key = key_at(t);
+            if ((key & mask) == prefix) atomicAdd(&hist[(key >> shift) & digit], 1u);
         }
         __syncthreads();
         if (tid < 32) {
@@ -124,7 +139,7 @@ topk_select_kernel(const float *__restrict__ scores, int T, int k, int32_t *__re
         __syncthreads();
         prefix = sh_prefix;
         remaining = sh_remaining;
-        mask |= 255u << shift;
+        mask |= digit << shift;
         __syncthreads();
     }
     // prefix is now the k-th largest key; `remaining` keys equal to it are kept.
@@ -137,7 +152,7 @@ topk_select_kernel(const float *__restrict__ scores, int T, int k, int32_t *__re
         uint32_t key = 0u;
         if (t < T) {
             v = __ldg(s + t);
-            key = order_key(v);
+            key = staged ? keys_s[t] : order_key(v);
         }
         const bool gt = t < T && key > thr;
         const bool eq = t < T && key == thr;
@@ -206,7 +221,16 @@ cudaError_t launch_router_auto(const Dims &dm, const void *X, const void *Wr, fl
 cudaError_t launch_select(int rows, int T, int k, const float *scores, int32_t *I, float *rsel,
                           int B, int H, int32_t *gidx, float *rsel_hm, cudaStream_t stream) {
     if (rows <= 0) return cudaSuccess;
-    cudaError_t e = launch_pdl(topk_select_kernel, dim3(rows), dim3(kSelThreads), 0, stream,
+    static std::once_flag once;
+    static cudaError_t attr = cudaSuccess;
+    std::call_once(once, [] {
+        attr = cudaFuncSetAttribute(topk_select_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                    kSelStagedMax * (int)sizeof(uint32_t));
+    });
+    if (attr != cudaSuccess) return attr;
+    const size_t smem = T <= kSelStagedMax ? sizeof(uint32_t) * (size_t)T : 0;
+    const int threads = (T >= 2048 || rows < 608) ? 1024 : 256;
+    cudaError_t e = launch_pdl(topk_select_kernel, dim3(rows), dim3(threads), smem, stream,
                                scores, T, k, I, rsel, B, H, gidx, rsel_hm);
     note_launches(1);
     return e;

@@ -205,14 +205,14 @@ def traffic_for(stage, cfg_name):
 
 
 # Kernel name (as ncu prints it) -> bench stage.
-KERNEL_STAGE = [("tc_gemm_kernel<6>", "router"), ("tc_gemm_kernel<(int)6>", "router"),
+KERNEL_STAGE = [("tc_gemm_kernel<5>", "router"), ("tc_gemm_kernel<(int)5>", "router"),
                 ("topk_select", "select"), ("tc_gemm_kernel<0>", "qkv"),
                 ("tc_gemm_kernel<(int)0>", "qkv"), ("attn_fwd", "attn_fwd"),
                 ("tc_gemm_kernel<1>", "out"), ("tc_gemm_kernel<(int)1>", "out"),
                 ("tc_gemm_kernel<2>", "out_bwd"), ("tc_gemm_kernel<(int)2>", "out_bwd"),
-                ("attn_bwd", "attn_bwd"), ("attn_dkv", "attn_bwd"), ("attn_dq", "attn_bwd"),
-                ("tc_gemm_kernel<4>", "in_bwd"), ("tc_gemm_kernel<(int)4>", "in_bwd"),
-                ("tc_gemm_kernel<5>", "w_bwd"), ("tc_gemm_kernel<(int)5>", "w_bwd"),
+                ("attn_bwd", "attn_bwd"), ("dq_finish", "attn_bwd"),
+                ("dx_kernel", "in_bwd"),
+                ("tc_gemm_kernel<4>", "w_bwd"), ("tc_gemm_kernel<(int)4>", "w_bwd"),
                 ("tc_gemm_kernel<3>", "dwo"), ("tc_gemm_kernel<(int)3>", "dwo"),
                 ("fused_fwd_kernel", "fwd_unit"), ("fused_bwd_kernel", "bwd_unit")]
 

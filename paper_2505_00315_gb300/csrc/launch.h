@@ -117,6 +117,9 @@ cudaError_t tc_transpose_wr(const Dims &dm, const void *Wr, const Saved &sv, cud
 cudaError_t tc_in_bwd(const Dims &dm, const void *Wq, const void *Wk, const void *Wv,
                       const void *Wr, const Saved &sv, float *dX, cudaStream_t s,
                       bool zero_output);
+// B3 as a persistent kernel over (head, 128-row tile, 256-column chunk) units.
+cudaError_t tc_dx(const Dims &dm, const void *Wq, const void *Wk, const void *Wv, const Saved &sv,
+                  float *dX, cudaStream_t s);
 // F1 on tensor cores (bf16 inputs, H % 8 == 0); false if not applicable.
 bool tc_router(const Dims &dm, const void *X, const void *Wr, float *r_full, uint32_t *status,
                cudaStream_t s, cudaError_t *err);

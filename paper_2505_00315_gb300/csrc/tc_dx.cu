@@ -1,0 +1,279 @@
+// Input gradient B3 (Sec. 2.2, Eq. mosa_mha differentiated through the
+// gather X^s = X[I] and the router r = sigmoid(X W^r)):
+//   dX[g(m), n] += sum_j [dQ|dK|dV]_j(m, :) W_j[h](n, :)  +  dlogit(m) W_r[n, h]
+// for the B*k selected rows m of head h, g(m) = b*T + I[b,h,i].
+//
+// The work is a list of units (head, 128-row tile, 256-column chunk of d),
+// head-major, and a persistent grid of at most one CTA per SM takes a
+// contiguous range of it, so every SM gets the same number of units whatever
+// the tile count.  A CTA loads a tile's dQ|dK|dV pair (96 KB) by TMA once for
+// all the chunks it holds of that tile; the W_j blocks (256 rows of d x 64)
+// stream through a 3-slot ring; the chunk accumulators alternate between two
+// 256-column halves of TMEM, so the scatter-add of one chunk (red.add.v4
+// through a per-warp staging buffer, with dlogit x W_r from an fp32 transpose
+// of W_r) runs while the MMAs of the next one do.  Each product with the
+// pair operand is two MMAs (hi, lo).
+// Warps: 0 TMA producer, 1 MMA issuer, 2 TMEM owner, 3 idle, 4-11 epilogue
+// (warp w: tile rows 32 (w % 4) .. +31, chunk columns 128 ((w - 4) / 4) ..).
+// Every wait is bounded.
+#include <mutex>
+
+#include "launch.h"
+#include "profile.h"
+#include "tc_common.cuh"
+#include "tc_tiles.cuh"
+#include "tmap.h"
+
+namespace mosa {
+namespace {
+
+using namespace tc;
+
+constexpr int kThreads = 384;
+constexpr int kWorkers = 256;
+constexpr int kChunk = 256;
+constexpr int kSlots = 3;
+constexpr int kWBytes = 256 * 128;   // one W_j block: 256 rows of d x 64 columns
+
+struct DxSmem {
+    uint8_t a[3][2][kTileHalf];      // dQ, dK, dV pairs of the tile [j][hi / lo]
+    uint8_t w[kSlots][kWBytes];      // W_j blocks
+    uint8_t stage[8][4096];          // epilogue staging, one buffer per epilogue warp
+    uint64_t a_full[3], a_empty[3], w_full[kSlots], w_empty[kSlots], out_full[2], out_empty[2];
+    uint32_t tmem;
+    int abort;
+};
+constexpr int kSmem = (int)sizeof(DxSmem) + 1024;
+static_assert(kSmem <= 227 * 1024, "shared memory");
+
+struct DxParams {
+    CUtensorMap mA;       // dQKV pair [H, B*k, 512], box {64, 128, 1}
+    CUtensorMap mW[3];    // W_q, W_k, W_v [H, d, 64], box {64, 256, 1}
+    const int32_t *gidx;  // [H, B*k]
+    const float *dlogit;  // [H, B*k]
+    const float *WrT;     // [H, d]
+    float *dX;            // [B*T, d], accumulated into
+    int Mtok, d;
+    int mt, nch;          // tiles per head, chunks per tile
+    long long units;      // H * mt * nch
+    uint32_t *status;
+};
+
+__device__ __forceinline__ bool dwait(DxSmem &sm, uint64_t &bar, uint32_t parity, uint32_t *status) {
+    if (*(volatile int *)&sm.abort) return false;
+    if (mbar_wait(smem_u32(&bar), parity)) return true;
+    atomicOr(status, kStatusTimeout);
+    *(volatile int *)&sm.abort = 1;
+    return false;
+}
+
+__global__ void __launch_bounds__(kThreads, 1) dx_kernel(const __grid_constant__ DxParams p) {
+    extern __shared__ uint8_t smem_raw[];
+    DxSmem &sm = *reinterpret_cast<DxSmem *>(
+        (reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    // this CTA's units [u0, u1); unit u = (h * mt + tile) * nch + chunk
+    const long long u0 = p.units * blockIdx.x / gridDim.x;
+    const long long u1 = p.units * (blockIdx.x + 1) / gridDim.x;
+    const int nu = (int)(u1 - u0);
+
+    if (threadIdx.x == 0) {
+        for (int j = 0; j < 3; ++j) {
+            mbar_init(smem_u32(&sm.a_full[j]), 1);
+            mbar_init(smem_u32(&sm.a_empty[j]), 1);
+        }
+        for (int s = 0; s < kSlots; ++s) {
+            mbar_init(smem_u32(&sm.w_full[s]), 1);
+            mbar_init(smem_u32(&sm.w_empty[s]), 1);
+        }
+        for (int i = 0; i < 2; ++i) {
+            mbar_init(smem_u32(&sm.out_full[i]), 1);
+            mbar_init(smem_u32(&sm.out_empty[i]), kWorkers);
+        }
+        sm.abort = 0;
+        fence_barrier_init();
+    }
+    if (warp == 2) {
+        tmem_alloc(smem_u32(&sm.tmem), 512);
+        tmem_relinquish();
+    }
+    tc_fence_before();
+    __syncthreads();
+    tc_fence_after();
+    const uint32_t tmem = sm.tmem;
+    pdl_wait();  // dQ|dK|dV, dlogit and the W_r transpose come from earlier kernels
+
+    if (warp == 0) {
+        if (lane == 0) {
+            int ntile = 0;  // tiles started so far
+            for (int i = 0; i < nu; ++i) {
+                const long long u = u0 + i;
+                const int c = (int)(u % p.nch);
+                const long long tile = u / p.nch;
+                const int h = (int)(tile / p.mt), m0 = (int)(tile % p.mt) * 128;
+                const bool fresh = i == 0 || c == 0;
+                bool ok = true;
+                for (int j = 0; j < 3; ++j) {
+                    const int idx = 3 * i + j, s = idx % kSlots;
+                    if (!(ok = dwait(sm, sm.w_empty[s], ((idx / kSlots) & 1) ^ 1, p.status))) break;
+                    if (fresh) {
+                        // A_j of the previous tile frees once its last j-products end
+                        if (ntile > 0 && !(ok = dwait(sm, sm.a_empty[j], (ntile - 1) & 1, p.status)))
+                            break;
+                        const uint32_t ab = smem_u32(&sm.a_full[j]);
+                        mbar_expect_tx(ab, 2 * kTileHalf);
+                        tma_load_3d(smem_u32(sm.a[j][0]), &p.mA, ab, 64 * j, m0, h);        // hi
+                        tma_load_3d(smem_u32(sm.a[j][1]), &p.mA, ab, 256 + 64 * j, m0, h);  // lo
+                    }
+                    const uint32_t fb = smem_u32(&sm.w_full[s]);
+                    mbar_expect_tx(fb, kWBytes);
+                    tma_load_3d(smem_u32(sm.w[s]), &p.mW[j], fb, 0, c * kChunk, h);
+                }
+                if (!ok) break;
+                if (fresh) ++ntile;
+            }
+        }
+    } else if (warp == 1) {
+        if (lane == 0) {
+            constexpr uint32_t idX = idesc_bf16(128, kChunk, false, false);
+            bool ok = true;
+            int ntile = 0;
+            for (int i = 0; i < nu && ok; ++i) {
+                const long long u = u0 + i;
+                const int c = (int)(u % p.nch), buf = i & 1;
+                const bool fresh = i == 0 || c == 0;
+                const bool last = c == p.nch - 1 || i == nu - 1;  // the tile's last chunk here
+                if (i >= 2 && !(ok = dwait(sm, sm.out_empty[buf], ((i >> 1) - 1) & 1, p.status))) break;
+                for (int j = 0; j < 3 && ok; ++j) {
+                    const int idx = 3 * i + j, s = idx % kSlots;
+                    if (fresh && !(ok = dwait(sm, sm.a_full[j], ntile & 1, p.status))) break;
+                    if (!(ok = dwait(sm, sm.w_full[s], (idx / kSlots) & 1, p.status))) break;
+                    tc_fence_after();
+                    const uint32_t wb = smem_u32(sm.w[s]);
+#pragma unroll
+                    for (int half = 0; half < 2; ++half)
+#pragma unroll
+                        for (int kk = 0; kk < 4; ++kk)
+                            mma_bf16(tmem + 256 * buf,
+                                     smem_desc_sw128(smem_u32(sm.a[j][half]) + kk * 32, 16, 1024),
+                                     smem_desc_sw128(wb + kk * 32, 16, 1024), idX,
+                                     (j > 0 || half > 0 || kk > 0) ? 1u : 0u);
+                    mma_commit(smem_u32(&sm.w_empty[s]));
+                    if (last) mma_commit(smem_u32(&sm.a_empty[j]));
+                }
+                if (!ok) break;
+                mma_commit(smem_u32(&sm.out_full[buf]));
+                if (fresh) ++ntile;
+            }
+            if (!ok) {
+                // release the epilogue warps
+                for (int b2 = 0; b2 < 2; ++b2) mma_commit(smem_u32(&sm.out_full[b2]));
+            }
+        }
+    } else if (warp >= 4) {
+        pdl_trigger();
+        const int q = warp & 3, ch = (warp - 4) >> 2;
+        const uint32_t lane_off = (uint32_t)(q * 32) << 16;
+        uint8_t *xb = sm.stage[warp - 4];
+        const int cu = lane & 7;
+        int my_row = -1;     // b*T + I of tile row 32 q + lane, -1 past B*k
+        float my_dl = 0.f;   // its dlogit
+        for (int i = 0; i < nu; ++i) {
+            const long long u = u0 + i;
+            const int c = (int)(u % p.nch), buf = i & 1;
+            const long long tile = u / p.nch;
+            const int h = (int)(tile / p.mt), m0 = (int)(tile % p.mt) * 128;
+            if (i == 0 || c == 0) {
+                const int m = m0 + q * 32 + lane;
+                my_row = m < p.Mtok ? p.gidx[(size_t)h * p.Mtok + m] : -1;
+                my_dl = m < p.Mtok ? p.dlogit[(size_t)h * p.Mtok + m] : 0.f;
+            }
+            const bool got = dwait(sm, sm.out_full[buf], (i >> 1) & 1, p.status);
+            tc_fence_after();
+            const bool go = __all_sync(0xffffffffu, got && !*(volatile int *)&sm.abort);
+            const uint32_t tb = tmem + 256 * buf + lane_off;
+#pragma unroll 1
+            for (int s0 = 128 * ch; s0 < 128 * ch + 128; s0 += 32) {
+                if (!go) break;
+                float v[32];
+                tmem_ld32(tb + s0, v);
+                stage_f32x32(xb, v, 1.f, lane);
+                const int n = c * kChunk + s0 + 4 * cu;
+                const bool nin = n < p.d;
+                float4 w4 = make_float4(0.f, 0.f, 0.f, 0.f);
+                if (nin) w4 = *reinterpret_cast<const float4 *>(p.WrT + (size_t)h * p.d + n);
+#pragma unroll
+                for (int r = 0; r < 8; ++r) {
+                    const int rl = (lane >> 3) + 4 * r;
+                    const int srow = __shfl_sync(0xffffffffu, my_row, rl);
+                    const float dlr = __shfl_sync(0xffffffffu, my_dl, rl);
+                    float4 val = *reinterpret_cast<const float4 *>(xb + xoff128(rl, cu));
+                    if (srow >= 0 && nin) {
+                        val.x = fmaf(dlr, w4.x, val.x);
+                        val.y = fmaf(dlr, w4.y, val.y);
+                        val.z = fmaf(dlr, w4.z, val.z);
+                        val.w = fmaf(dlr, w4.w, val.w);
+                        red_add_v4(p.dX + (size_t)srow * p.d + n, val.x, val.y, val.z, val.w);
+                    }
+                }
+                __syncwarp();
+            }
+            tc_fence_before();
+            mbar_arrive(smem_u32(&sm.out_empty[buf]));
+            if (!go) break;
+        }
+    }
+    tc_fence_before();
+    __syncthreads();
+    if (warp == 2) {
+        tc_fence_after();
+        tmem_dealloc(tmem, 512);
+    }
+}
+
+bool map3(CUtensorMap *m, const void *base, uint64_t H, uint64_t rows, uint64_t cols,
+          uint32_t box_rows) {
+    const uint64_t dims[3] = {cols, rows, H}, strides[2] = {cols * 2, rows * cols * 2};
+    const uint32_t box[3] = {64, box_rows, 1};
+    return tmap_bf16(m, base, 3, dims, strides, box);
+}
+
+}  // namespace
+
+cudaError_t tc_dx(const Dims &dm, const void *Wq, const void *Wk, const void *Wv, const Saved &sv,
+                  float *dX, cudaStream_t s) {
+    DxParams p;
+    memset(&p, 0, sizeof(p));
+    const int Mtok = dm.B * dm.k;
+    if (Mtok <= 0 || dm.d <= 0 || dm.H <= 0) return cudaSuccess;
+    const void *W[3] = {Wq, Wk, Wv};
+    bool ok = map3(&p.mA, sv.dQKV, dm.H, Mtok, 512, 128);
+    for (int j = 0; j < 3; ++j) ok = ok && map3(&p.mW[j], W[j], dm.H, dm.d, 64, 256);
+    if (!ok) return cudaErrorInvalidValue;
+    p.gidx = sv.gidx;
+    p.dlogit = sv.dlogit;
+    p.WrT = sv.WrT;
+    p.dX = dX;
+    p.Mtok = Mtok;
+    p.d = dm.d;
+    p.mt = (Mtok + 127) / 128;
+    p.nch = (dm.d + kChunk - 1) / kChunk;
+    p.units = (long long)dm.H * p.mt * p.nch;
+    p.status = sv.status;
+    static std::once_flag once;
+    static cudaError_t attr = cudaSuccess;
+    std::call_once(once, [] {
+        attr = cudaFuncSetAttribute(dx_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, kSmem);
+    });
+    if (attr != cudaSuccess) return attr;
+    int dev = 0, sms = 0;
+    cudaError_t e = cudaGetDevice(&dev);
+    if (e == cudaSuccess) e = cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
+    if (e != cudaSuccess) return e;
+    const long long grid = p.units < sms ? p.units : sms;
+    e = launch_pdl(dx_kernel, dim3((unsigned)grid), dim3(kThreads), kSmem, s, p);
+    note_launches(1);
+    return e;
+}
+
+}  // namespace mosa

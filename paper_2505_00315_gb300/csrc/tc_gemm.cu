@@ -20,14 +20,13 @@
 //   kOUT  F5  Y[g(m),n]    += (diag(r) A)(m,:) W_o[h](:,n)   A = AR pair,  B MN-major
 //   kG    B1  G(m,:)        = dY[g(m),:] W_o[h]^T, then dr, dA = r G, D, dlogit in the epilogue
 //   kDWO  B1  dW_o[h](p,c)  = sum_m AR(m,p) dY[g(m),c]       A gathered MN-major, B = AR pair
-//   kDX   B3  dX[g(m),n]   += dQKV(m,:) [W_q|W_k|W_v][h]^T(:,n) + dlogit(m) W_r[n,h]
-//             (W_r read from its fp32 transpose [H, d], one float4 per lane)
 //   kDW   B4  [dW_q|dW_k|dW_v|dW_r][h](c,:) = sum_m X[g(m),c] [dQ|dK|dV|dlogit](m,:)
 //             A gathered MN-major, B = the dQKV pair (its 4th 64-column block holds
 //             dlogit in column 0 and zeros), so dW_r comes out of the same product;
 //             256 rows c per CTA in two accumulators that share every B tile
 //   kROUTER F1 r[b,h,t] = sigmoid(X[b,t,:] W_r[:,h])       A = X tiles, B = W_r MN-major
-// where g(m) = b*T + I[b,h,i] for row m = b*k + i of head h.
+// where g(m) = b*T + I[b,h,i] for row m = b*k + i of head h.  B3 (dX) has a
+// persistent kernel of its own (tc_dx.cu).
 #include <algorithm>
 #include <cstdio>
 #include <mutex>
@@ -42,7 +41,7 @@ namespace {
 
 using namespace tc;
 
-enum Kind : int { kQKV = 0, kOUT, kG, kDWO, kDX, kDW, kROUTER };
+enum Kind : int { kQKV = 0, kOUT, kG, kDWO, kDW, kROUTER };
 
 constexpr int kBM = 128;        // rows per tile (TMEM lanes)
 constexpr int kBK = 64;         // K per stage: one 128-byte swizzle row of bf16
@@ -78,15 +77,6 @@ struct Cfg<kDWO> {
     static constexpr bool A_MN = true, B_MN = true, A_PAIR = false, B_PAIR = true;
 };
 template <>
-struct Cfg<kDX> {
-    // one stage: 80 KB of shared memory lets two CTAs share an SM, so one CTA's
-    // scatter-add epilogue overlaps the other's loads (measured faster than a
-    // three-stage ring at one CTA per SM)
-    static constexpr int BN = 256, STAGES = 1, A_BYTES = 2 * kTile16K, B_BYTES = 32768,
-                         TMEM_COLS = 256, MIN_CTAS = 2;
-    static constexpr bool A_MN = false, B_MN = false, A_PAIR = true, B_PAIR = false;
-};
-template <>
 struct Cfg<kDW> {
     // 256 rows of d per CTA as two 128 x 256 accumulators sharing each B tile;
     // K blocks of 32 tokens: A = 4 blocks of 32 x 64, B = 8 blocks of 32 x 64
@@ -118,10 +108,10 @@ __host__ __device__ constexpr int kind_acc() {
 // [dQ | dK | dV | dlogit, 0..] hi (256) then the same lo (256).
 constexpr int kDQKVCols = 512;
 
-// Kinds that scatter-add their output rows into [B*T, d] (Y or dX).
+// Kinds that scatter-add their output rows into [B*T, d] (Y).
 template <int KIND>
 __host__ __device__ constexpr bool scatters() {
-    return KIND == kOUT || KIND == kDX;
+    return KIND == kOUT;
 }
 
 // Kinds whose A operand is gathered through the selected rows.
@@ -133,7 +123,7 @@ __host__ __device__ constexpr bool gathers() {
 // Kinds whose epilogue runs on all eight warps (wide output tiles).
 template <int KIND>
 __host__ __device__ constexpr bool epi_all_warps() {
-    return KIND == kQKV || KIND == kOUT || KIND == kDX || KIND == kDW || KIND == kDWO;
+    return KIND == kQKV || KIND == kOUT || KIND == kDW || KIND == kDWO;
 }
 
 template <int KIND>
@@ -147,7 +137,7 @@ struct TcParams {
     CUtensorMap mapB[3];   // per-head tile maps of the B operand
     int M;                 // output rows per head: B*k for row kinds, d for kDWO / kDW
     int Mtok;              // selected rows per head, B*k
-    int N;                 // output columns (d for kOUT / kDX); MMA width (kROUTER)
+    int N;                 // output columns (d for kOUT); MMA width (kROUTER)
     int ring_stages;       // kROUTER: stages in the ring (<= kMaxStages)
     int ring_stride;       // kROUTER: bytes per stage
     int nkb;               // K blocks in the whole reduction
@@ -156,11 +146,9 @@ struct TcParams {
     const int32_t *gidx;   // [H, B*k]
     const float *rsel;     // [H, B*k]
     const float *A32;      // [H, B*k, 64] attention output (kG)
-    const float *dlogit;   // [H, B*k] (kDX reads, kG writes via out_f1)
-    const float *WrT;      // [H, d] fp32 transpose of W_r (kDX)
     const void *src_rows;  // gathered source [B*T, d] bf16: X (kQKV, kDW) or dY (kG, kDWO)
     void *out[3];          // Q/K/V pairs (kQKV); dA pair, dQKV pair (kG)
-    float *out_f;          // Y (kOUT), dW_o (kDWO), dX (kDX), dW_q (kDW)
+    float *out_f;          // Y (kOUT), dW_o (kDWO), dW_q (kDW)
     float *out_f1;         // Dd (kG), dW_k (kDW)
     float *out_f2;         // dlogit (kG), dW_v (kDW)
     float *out_f3;         // dW_r (kDW)
@@ -350,7 +338,6 @@ __global__ void __launch_bounds__(kThreads, Cfg<KIND>::MIN_CTAS)
     int *s_abort = reinterpret_cast<int *>(tmem_slot + 1);
     int *s_rows = s_abort + 1 + 2;  // 128 gather rows, 16-byte aligned below
     s_rows = reinterpret_cast<int *>((reinterpret_cast<uintptr_t>(s_rows) + 15) & ~uintptr_t(15));
-    float *s_dl = reinterpret_cast<float *>(s_rows + kBM);   // dlogit of the tile's rows (kDX)
     static_assert(KIND == kROUTER || S * (C::A_BYTES + C::B_BYTES) >= 8 * kXpose,
                   "epilogue staging must fit in the operand ring");
 
@@ -383,7 +370,6 @@ __global__ void __launch_bounds__(kThreads, Cfg<KIND>::MIN_CTAS)
         for (int r = threadIdx.x; r < kBM; r += kThreads) {
             const int m = m0 + r;
             s_rows[r] = m < p.Mtok ? p.gidx[(size_t)h * p.Mtok + m] : 0;
-            if (KIND == kDX) s_dl[r] = m < p.Mtok ? p.dlogit[(size_t)h * p.Mtok + m] : 0.f;
         }
     }
     if (warp == 2) {
@@ -433,10 +419,6 @@ __global__ void __launch_bounds__(kThreads, Cfg<KIND>::MIN_CTAS)
                 if (lane == 0) tma_load_2d(a, &p.mapA, fb, kb * kBK, m0);
                 if (lane >= 1 && lane <= nbl)
                     tma_load_2d(b + (lane - 1) * kTile8K, &p.mapB[0], fb, n0 + 64 * (lane - 1), kb * kBK);
-            } else if constexpr (KIND == kDX) {
-                if (lane == 0) tma_load_3d(a, &p.mapA, fb, 64 * kb, m0, h);
-                if (lane == 1) tma_load_3d(a + kTile16K, &p.mapA, fb, 256 + 64 * kb, m0, h);
-                if (lane == 2) tma_load_3d(b, &p.mapB[kb], fb, 0, n0, h);
             } else if constexpr (KIND == kDWO) {
                 if (lane < 2) tma_load_3d(b + lane * kTile8K, &p.mapB[0], fb, 64 * lane, kb * kBK, h);
             } else {  // kDW: hi blocks 0..3 then lo blocks 0..3, 32 token rows each
@@ -530,29 +512,19 @@ __global__ void __launch_bounds__(kThreads, Cfg<KIND>::MIN_CTAS)
                     return reinterpret_cast<uint4 *>(dst + (size_t)rl * 128) + u;
                 });
             }
-        } else if constexpr (KIND == kOUT || KIND == kDX) {
+        } else if constexpr (KIND == kOUT) {
             // 32 x 32 blocks transposed through shared memory so that every
             // red.add.v4 covers four whole 128-byte row segments
             const int chunk = lane & 7;
             for (int c0 = part * (C::BN / 2); c0 < (part + 1) * (C::BN / 2); c0 += 32) {
                 stage_f32_32(xb, tb + c0, lane);
                 const int n = n0 + c0 + 4 * chunk;
-                float4 w4 = make_float4(0.f, 0.f, 0.f, 0.f);
-                if (KIND == kDX && n < p.d)
-                    w4 = *reinterpret_cast<const float4 *>(p.WrT + (size_t)h * p.d + n);
 #pragma unroll
                 for (int i = 0; i < 8; ++i) {
                     const int rl = (lane >> 3) + 4 * i;
                     const int rt = q * 32 + rl;
                     float4 val = *reinterpret_cast<const float4 *>(xb + rl * 128 + ((chunk ^ (rl & 7)) << 4));
                     if (m0 + rt < p.M && n < p.d) {
-                        if (KIND == kDX) {
-                            const float dl = s_dl[rt];
-                            val.x = fmaf(dl, w4.x, val.x);
-                            val.y = fmaf(dl, w4.y, val.y);
-                            val.z = fmaf(dl, w4.z, val.z);
-                            val.w = fmaf(dl, w4.w, val.w);
-                        }
                         red_add_v4(p.out_f + (size_t)s_rows[rt] * p.d + n, val.x, val.y, val.z, val.w);
                     }
                 }
@@ -885,22 +857,8 @@ cudaError_t tc_in_bwd(const Dims &dm, const void *Wq, const void *Wk, const void
         cudaError_t e = cudaMemsetAsync(dX, 0, sizeof(float) * (size_t)dm.B * dm.T * dm.d, s);
         if (e != cudaSuccess) return e;
     }
-    TcParams p = base_params(dm, sv);
-    p.M = p.Mtok;
-    p.N = dm.d;
-    p.nkb = 3;
-    const void *W[3] = {Wq, Wk, Wv};
-    bool ok = map_heads(&p.mapA, sv.dQKV, dm.H, p.Mtok, kDQKVCols, 128);
-    for (int j = 0; j < 3; ++j) ok = ok && map_heads(&p.mapB[j], W[j], dm.H, dm.d, 64, 256);
-    if (!ok) return cudaErrorInvalidValue;
-    (void)Wr;
-    p.dlogit = sv.dlogit;
-    p.WrT = sv.WrT;
-    p.out_f = dX;
-    dim3 grid((p.M + kBM - 1) / kBM, (dm.d + 255) / 256, dm.H);
-    // early start: the dW product beside it on the other stream needs all 512
-    // TMEM columns of an SM, so the two cannot share SMs anyway
-    return launch_kind<kDX>(p, grid, s);
+    (void)Wr;  // read through its fp32 transpose sv.WrT
+    return tc_dx(dm, Wq, Wk, Wv, sv, dX, s);
 }
 
 cudaError_t tc_w_bwd(const Dims &dm, const void *X, const Saved &sv, float *dWq, float *dWk,

@@ -92,7 +92,7 @@ struct Saved {
                         // [H,B*k,512] bf16 pair dQ|dK|dV|dlogit,0.. hi then lo)
     float *G;           // [H,B*k,hp] dY[I] W_o^T (fp32, CUDA-core path); on the
                         // tensor-core path with k > 128 the fp32 dQ accumulator
-    float *WrT;         // [H,d] fp32 transpose of W_r (tensor-core backward)
+    float *WrT;         // [H,d] fp32 transpose of W_r (tensor-core dX epilogue)
 };
 
 struct Dims {

@@ -96,12 +96,11 @@ bool use_fused_forward(const Dims &dm);
 cudaError_t tc_fused_forward(const Dims &dm, const void *X, const void *Wq, const void *Wk,
                              const void *Wv, const void *Wo, const Saved &sv, float *Y,
                              cudaStream_t s);
-// Fused G / row terms + attention backward (+ dX) for k <= 128 (tc_fused_bwd.cu);
-// opt-in with MOSA_FUSED_BWD=1.  Needs the fp32 W_r transpose and dX zeroed.
+// Fused G / row terms + attention backward for k <= 128 (tc_fused_bwd.cu);
+// opt-in with MOSA_FUSED_BWD=1.
 bool use_fused_backward(const Dims &dm);
-cudaError_t tc_fused_backward(const Dims &dm, const void *W_q, const void *W_k, const void *W_v,
-                              const void *W_o, const void *dY, const Saved &sv, float *dX,
-                              bool with_dx, cudaStream_t s);
+cudaError_t tc_fused_backward(const Dims &dm, const void *W_o, const void *dY, const Saved &sv,
+                              cudaStream_t s);
 cudaError_t tc_qkv(const Dims &dm, const void *X, const void *Wq, const void *Wk, const void *Wv,
                    const Saved &sv, cudaStream_t s);
 // zero_output = false: the caller has already zeroed Y / dX on this stream's timeline.
@@ -112,17 +111,18 @@ cudaError_t tc_out_bwd_g(const Dims &dm, const void *Wo, const void *dY, const S
                          cudaStream_t s);
 cudaError_t tc_out_bwd_w(const Dims &dm, const void *dY, const Saved &sv, float *dWo,
                          cudaStream_t s);
-// W_r [d,H] bf16 -> sv.WrT [H,d] fp32 (read by the dX epilogue).
-cudaError_t tc_transpose_wr(const Dims &dm, const void *Wr, const Saved &sv, cudaStream_t s);
 cudaError_t tc_in_bwd(const Dims &dm, const void *Wq, const void *Wk, const void *Wv,
                       const void *Wr, const Saved &sv, float *dX, cudaStream_t s,
                       bool zero_output);
 // B3 as a persistent kernel over (head, 128-row tile, 256-column chunk) units.
+// Needs dX zeroed and sv.WrT (tc_transpose_wr).
 cudaError_t tc_dx(const Dims &dm, const void *Wq, const void *Wk, const void *Wv, const Saved &sv,
                   float *dX, cudaStream_t s);
 // F1 on tensor cores (bf16 inputs, H % 8 == 0); false if not applicable.
 bool tc_router(const Dims &dm, const void *X, const void *Wr, float *r_full, uint32_t *status,
                cudaStream_t s, cudaError_t *err);
+// W_r [d,H] bf16 -> sv.WrT [H,d] fp32 (read by the dX epilogue).
+cudaError_t tc_transpose_wr(const Dims &dm, const void *Wr, const Saved &sv, cudaStream_t s);
 cudaError_t tc_attn_fwd(const Dims &dm, const Saved &sv, cudaStream_t s);
 cudaError_t tc_attn_bwd(const Dims &dm, const Saved &sv, cudaStream_t s);
 cudaError_t tc_w_bwd(const Dims &dm, const void *X, const Saved &sv, float *dWq, float *dWk,

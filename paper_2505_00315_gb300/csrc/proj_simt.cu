@@ -289,7 +289,10 @@ cudaError_t launch_out_bwd(const Dims &dm, const void *Wo, const void *dY, const
 
 cudaError_t launch_in_bwd(const Dims &dm, const void *Wq, const void *Wk, const void *Wv,
                           const void *Wr, const Saved &sv, float *dX, cudaStream_t s) {
-    if (use_tc(dm)) return tc_in_bwd(dm, Wq, Wk, Wv, Wr, sv, dX, s, true);
+    if (use_tc(dm)) {
+        cudaError_t e = tc_transpose_wr(dm, Wr, sv, s);
+        return e != cudaSuccess ? e : tc_in_bwd(dm, Wq, Wk, Wv, Wr, sv, dX, s, true);
+    }
     return dm.bf16 ? in_bwd_t<bf16>(dm, Wq, Wk, Wv, Wr, sv, dX, s)
                    : in_bwd_t<float>(dm, Wq, Wk, Wv, Wr, sv, dX, s);
 }

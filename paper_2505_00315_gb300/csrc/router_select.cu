@@ -80,6 +80,8 @@ topk_select_kernel(const float *__restrict__ scores, int T, int k, int32_t *__re
     __shared__ uint32_t hist[256];
     __shared__ uint32_t sh[33];
     __shared__ uint32_t sh_prefix, sh_remaining;
+    // the next kernel may launch and run its prologue as this grid's CTAs finish
+    asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
     asm volatile("griddepcontrol.wait;" ::: "memory");  // scores from the router kernel
     const int row = blockIdx.x;
     const float *s = scores + (size_t)row * T;

@@ -622,6 +622,7 @@ __global__ void __launch_bounds__(kBT, 1) attn_bwd_tc_kernel(const __grid_consta
 // dQ from its fp32 accumulator into columns 0..63 (hi) / 256..319 (lo) of the
 // dQKV pair rows, two columns per thread.
 __global__ void dq_finish_kernel(const float *__restrict__ dQacc, bf16 *__restrict__ dQKV, size_t rows) {
+    pdl_trigger();  // the next kernel (zeroing dX) may run beside this one
     pdl_wait();
     const size_t idx = (size_t)blockIdx.x * blockDim.x + threadIdx.x;   // (row, column pair)
     if (idx >= rows * 32) return;

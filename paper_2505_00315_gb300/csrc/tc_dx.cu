@@ -10,8 +10,8 @@
 // all the chunks it holds of that tile; the W_j blocks (256 rows of d x 64)
 // stream through a 3-slot ring; the chunk accumulators alternate between two
 // 256-column halves of TMEM, so the scatter-add of one chunk (red.add.v4
-// through a per-warp staging buffer, with dlogit x W_r from an fp32 transpose
-// of W_r) runs while the MMAs of the next one do.  Each product with the
+// through a per-warp staging buffer, with dlogit x W_r added from an fp32
+// transpose of W_r) runs while the MMAs of the next one do.  Each product with the
 // pair operand is two MMAs (hi, lo).
 // Warps: 0 TMA producer, 1 MMA issuer, 2 TMEM owner, 3 idle, 4-11 epilogue
 // (warp w: tile rows 32 (w % 4) .. +31, chunk columns 128 ((w - 4) / 4) ..).
@@ -51,7 +51,7 @@ struct DxParams {
     CUtensorMap mW[3];    // W_q, W_k, W_v [H, d, 64], box {64, 256, 1}
     const int32_t *gidx;  // [H, B*k]
     const float *dlogit;  // [H, B*k]
-    const float *WrT;     // [H, d]
+    const float *WrT;     // [H, d] fp32 transpose of W_r
     float *dX;            // [B*T, d], accumulated into
     int Mtok, d;
     int mt, nch;          // tiles per head, chunks per tile
@@ -101,7 +101,7 @@ __global__ void __launch_bounds__(kThreads, 1) dx_kernel(const __grid_constant__
     __syncthreads();
     tc_fence_after();
     const uint32_t tmem = sm.tmem;
-    pdl_wait();  // dQ|dK|dV, dlogit and the W_r transpose come from earlier kernels
+    pdl_wait();  // dQ|dK|dV and dlogit come from earlier kernels
 
     if (warp == 0) {
         if (lane == 0) {

@@ -8,14 +8,10 @@
 //            dlogit = dr r (1 - r) (the router gradient through diag(r))
 //   phase 3  S = Q K^T, dP = dA V^T; P from the saved log-sum-exp; dV = P^T dA;
 //            dS = P o (dP - D); dK = dS^T Q / sqrt(h'), dQ = dS K / sqrt(h')
-//   phase 4  dQ|dK|dV (and dlogit) to global memory for the weight gradients,
-//            and, when asked, dX[g(m), n] += ([dQ|dK|dV] [W_q|W_k|W_v][h]^T)(m, n)
-//            + dlogit(m) W_r[n, h] for n in 256-wide chunks (W blocks streamed
-//            by TMA, accumulators double-buffered in TMEM).  With one CTA per
-//            SM this phase cannot overlap other work, so the library runs dX
-//            as its own product beside the weight gradients instead.
-// The weight gradients reduce over all tiles of a head and stay separate
-// products (dW_o, dW_q|dW_k|dW_v|dW_r in tc_gemm.cu).
+//   phase 4  dQ|dK|dV (and dlogit) to global memory for dX and the weight
+//            gradients.
+// dX (tc_dx.cu) and the weight gradients, which reduce over all tiles of a
+// head, stay separate products (dW_o, dW_q|dW_k|dW_v|dW_r in tc_gemm.cu).
 //
 // Warps: 0 TMA producer, 1 MMA issuer, 2 TMEM owner, 3 idle; 4-11 gather,
 // row terms, softmax passes and epilogues, two per TMEM lane quadrant.
@@ -38,46 +34,39 @@ constexpr int kWorkers = 256;
 constexpr int kStages = 3;
 constexpr int kHalf = kTileHalf;                 // 16 KB
 constexpr int kStageBytes = kHalf + 8192;        // gathered dY block + W_o block
-constexpr int kChunk = 256;                      // dX columns per phase-4 chunk
-constexpr int kWBytes = 256 * 128;               // one W_j block: 256 rows of d x 64 columns
 
 // TMEM columns
 constexpr uint32_t kColG = 0, kColS = 64, kColDP = 192, kColDV = 320, kColDK = 384, kColDQ = 448;
 
 struct FusedBwdSmem {
     // phase 1: the ring (3 x 24 KB); phase 3: P / dS pair tile [half][key block]
-    // (64 KB); phase 4: two W_j blocks of 32 KB
+    // (64 KB)
     uint8_t r1[5 * kHalf];
     uint8_t da[2][kHalf];        // dA pair; phase 4: epilogue staging (8 x 4 KB)
-    uint8_t qkv[3][2][kHalf];    // Q, K, V pairs; phase 4: dQ, dK, dV pairs (A of the dX product)
+    uint8_t qkv[3][2][kHalf];    // Q, K, V pairs
     float part[2][128];          // partial <A, G> per column half
-    float Dd[128], dl[128];      // D and dlogit per tile row
+    float Dd[128];               // D per tile row
     int rows[128];               // b*T + I of each tile row, -1 outside the tile's sequences
     uint64_t full[kStages], empty[kStages];
-    uint64_t qkv_full, g_done, da_ready, sp_full, p_ready, pv_done, ds_ready, acc_done, dq_ready;
-    uint64_t w_full[2], w_empty[2], out_full[2], out_empty[2];
+    uint64_t qkv_full, g_done, da_ready, sp_full, p_ready, pv_done, ds_ready, acc_done;
     uint32_t tmem;
     int abort;
 };
 constexpr int kSmem = (int)sizeof(FusedBwdSmem) + 1024;
 static_assert(kSmem <= 227 * 1024, "shared memory");
-static_assert(kStages * kStageBytes <= 5 * kHalf && 2 * kWBytes <= 5 * kHalf, "region 1");
+static_assert(kStages * kStageBytes <= 5 * kHalf, "region 1");
 
 struct FusedBwdParams {
     CUtensorMap mWo;       // W_o: [H, 64, d], box {64, 64, 1}
     CUtensorMap mQKV[3];   // Q, K, V pairs: [H, B*k, 128], box {64, 128, 1}
-    CUtensorMap mW[3];     // W_q, W_k, W_v: [H, d, 64], box {64, 256, 1}
     const bf16 *dY;        // [B*T, d]
     const int32_t *gidx;   // [H, B*k]
     const float *rsel;     // [H, B*k]
     const float *A;        // [H, B*k, 64]
     const float *lse;      // [H, B*k]
-    const float *WrT;      // [H, d] fp32 transpose of W_r
     bf16 *dQKV;            // [H, B*k, 512] pair: dQ|dK|dV|dlogit hi, then lo
     float *Dd, *dlogit;    // [H, B*k]
-    float *dX;             // [B*T, d], accumulated into
     int B, T, d, k, U, Mtok;
-    int do_dx;             // phase 4's dX product (otherwise left to the separate kernel)
     float scale, scale_log2;
     uint32_t *status;
 };
@@ -98,11 +87,9 @@ __global__ void __launch_bounds__(kThreads, 1) fused_bwd_kernel(const __grid_con
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     const int b0 = blockIdx.x * p.U, h = blockIdx.y;
     const int nkb = (p.d + 63) / 64;
-    const int nch = p.do_dx ? (p.d + kChunk - 1) / kChunk : 0;
     const size_t row_base = (size_t)h * p.Mtok + (size_t)b0 * p.k;
     uint8_t(*ptile)[2][kHalf] = reinterpret_cast<uint8_t(*)[2][kHalf]>(&sm.r1[0]);
     auto ring = [&](int s) -> uint8_t * { return &sm.r1[0] + s * kStageBytes; };
-    auto wbuf = [&](int s) -> uint8_t * { return &sm.r1[0] + s * kWBytes; };
 
     if (threadIdx.x == 0) {
         for (int s = 0; s < kStages; ++s) {
@@ -117,13 +104,6 @@ __global__ void __launch_bounds__(kThreads, 1) fused_bwd_kernel(const __grid_con
         mbar_init(smem_u32(&sm.pv_done), 1);
         mbar_init(smem_u32(&sm.ds_ready), kWorkers);
         mbar_init(smem_u32(&sm.acc_done), 1);
-        mbar_init(smem_u32(&sm.dq_ready), kWorkers);
-        for (int i = 0; i < 2; ++i) {
-            mbar_init(smem_u32(&sm.w_full[i]), 1);
-            mbar_init(smem_u32(&sm.w_empty[i]), 1);
-            mbar_init(smem_u32(&sm.out_full[i]), 1);
-            mbar_init(smem_u32(&sm.out_empty[i]), kWorkers);
-        }
         sm.abort = 0;
         fence_barrier_init();
     }
@@ -158,17 +138,6 @@ __global__ void __launch_bounds__(kThreads, 1) fused_bwd_kernel(const __grid_con
                 const uint32_t fb = smem_u32(&sm.full[s]);
                 mbar_expect_tx(fb, 8192);
                 tma_load_3d(smem_u32(ring(s) + kHalf), &p.mWo, fb, kb * 64, 0, h);
-            }
-            // phase 4: W_j blocks (256 rows of d x 64) once dS is no longer read
-            if (nch > 0 && wait_or_abort(sm, sm.acc_done, 0, p.status)) {
-                for (int idx = 0; idx < 3 * nch; ++idx) {
-                    const int s = idx & 1, c = idx / 3, j = idx % 3;
-                    if (idx >= 2 && !wait_or_abort(sm, sm.w_empty[s], ((idx >> 1) - 1) & 1, p.status))
-                        break;
-                    const uint32_t fb = smem_u32(&sm.w_full[s]);
-                    mbar_expect_tx(fb, kWBytes);
-                    tma_load_3d(smem_u32(wbuf(s)), &p.mW[j], fb, 0, c * kChunk, h);
-                }
             }
         }
     } else if (warp == 1) {
@@ -221,36 +190,11 @@ __global__ void __launch_bounds__(kThreads, 1) fused_bwd_kernel(const __grid_con
                 mma_k128(tmem + kColDQ, ptile, sm.qkv[1], false, idKM);   // dQ = dS K
             }
             mma_commit(smem_u32(&sm.acc_done));
-            // phase 4: dX chunk c = sum_j [dQ|dK|dV]_j (pair) W_j[chunk rows]^T, TMEM 256 (c % 2)
-            ok = ok && (nch == 0 || wait_or_abort(sm, sm.dq_ready, 0, p.status));
-            constexpr uint32_t idX = idesc_bf16(128, kChunk, false, false);
-            for (int c = 0; c < nch && ok; ++c) {
-                const int buf = c & 1;
-                if (c >= 2 && !(ok = wait_or_abort(sm, sm.out_empty[buf], ((c >> 1) - 1) & 1, p.status)))
-                    break;
-                for (int j = 0; j < 3 && ok; ++j) {
-                    const int idx = 3 * c + j, s = idx & 1;
-                    if (!(ok = wait_or_abort(sm, sm.w_full[s], (idx >> 1) & 1, p.status))) break;
-                    tc_fence_after();
-                    const uint32_t wb = smem_u32(wbuf(s));
-#pragma unroll
-                    for (int half = 0; half < 2; ++half)
-#pragma unroll
-                        for (int kk = 0; kk < 4; ++kk)
-                            mma_bf16(tmem + 256 * buf,
-                                     smem_desc_sw128(smem_u32(sm.qkv[j][half]) + kk * 32, 16, 1024),
-                                     smem_desc_sw128(wb + kk * 32, 16, 1024), idX,
-                                     (j > 0 || half > 0 || kk > 0) ? 1u : 0u);
-                    mma_commit(smem_u32(&sm.w_empty[s]));
-                }
-                if (ok) mma_commit(smem_u32(&sm.out_full[buf]));
-            }
             if (!ok) {
                 // release every wait of the other warps that may still be pending
                 mma_commit(smem_u32(&sm.sp_full));
                 mma_commit(smem_u32(&sm.pv_done));
                 mma_commit(smem_u32(&sm.acc_done));
-                for (int i = 0; i < 2; ++i) mma_commit(smem_u32(&sm.out_full[i]));
             }
         }
     } else if (warp >= 4) {
@@ -324,7 +268,6 @@ __global__ void __launch_bounds__(kThreads, 1) fused_bwd_kernel(const __grid_con
         const float dlg = dr * rr * (1.f - rr);      // dlogit
         if (ch == 0) {
             sm.Dd[r] = dd;
-            sm.dl[r] = dlg;
             if (ok && valid) {
                 p.Dd[grow] = dd;
                 p.dlogit[grow] = dlg;
@@ -374,7 +317,7 @@ __global__ void __launch_bounds__(kThreads, 1) fused_bwd_kernel(const __grid_con
         tc_fence_before();
         mbar_arrive(smem_u32(&sm.ds_ready));
 
-        // ------------------- phase 4: dQ|dK|dV out, then the dX scatter-add
+        // ---------------------------------------------- phase 4: dQ|dK|dV out
         ok = wait_or_abort(sm, sm.acc_done, 0, p.status) && ok;
         tc_fence_after();
         const bool live = __all_sync(0xffffffffu, ok && !*(volatile int *)&sm.abort);
@@ -386,8 +329,6 @@ __global__ void __launch_bounds__(kThreads, 1) fused_bwd_kernel(const __grid_con
             for (int j = 0; j < 3; ++j) {
                 float v[32];
                 tmem_ld32(tmem + src[j] + lane_off + 32 * ch, v);
-                // A operand of the dX product (Q, K, V are no longer read)
-                if (nch > 0) put_pair32(sm.qkv[j][0], sm.qkv[j][1], r, 32 * ch, v, fac[j]);
                 if (live) {
                     stage_pair32(xb, v, fac[j], lane);
                     store_rows128(xb, lane, [&](int rl, int c) -> uint4 * {
@@ -399,46 +340,7 @@ __global__ void __launch_bounds__(kThreads, 1) fused_bwd_kernel(const __grid_con
                 }
             }
         }
-        fence_proxy_async();
-        tc_fence_before();
-        mbar_arrive(smem_u32(&sm.dq_ready));
         pdl_trigger();
-        const int cu = lane & 7;
-        for (int c = 0; c < nch; ++c) {
-            const int buf = c & 1;
-            const bool got = wait_or_abort(sm, sm.out_full[buf], (c >> 1) & 1, p.status);
-            tc_fence_after();
-            const bool go = __all_sync(0xffffffffu, got && live);
-            const uint32_t tb = tmem + 256 * buf + lane_off;
-#pragma unroll 1
-            for (int s0 = 128 * ch; s0 < 128 * ch + 128; s0 += 32) {
-                if (!go) break;
-                float v[32];
-                tmem_ld32(tb + s0, v);
-                stage_f32x32(xb, v, 1.f, lane);
-                const int n = c * kChunk + s0 + 4 * cu;
-                float4 w4 = make_float4(0.f, 0.f, 0.f, 0.f);
-                if (n < p.d) w4 = *reinterpret_cast<const float4 *>(p.WrT + (size_t)h * p.d + n);
-#pragma unroll
-                for (int i = 0; i < 8; ++i) {
-                    const int rl = (lane >> 3) + 4 * i;
-                    const int srow = sm.rows[q * 32 + rl];
-                    float4 val = *reinterpret_cast<const float4 *>(xb + xoff128(rl, cu));
-                    if (srow >= 0 && n < p.d) {
-                        const float dlr = sm.dl[q * 32 + rl];
-                        val.x = fmaf(dlr, w4.x, val.x);
-                        val.y = fmaf(dlr, w4.y, val.y);
-                        val.z = fmaf(dlr, w4.z, val.z);
-                        val.w = fmaf(dlr, w4.w, val.w);
-                        red_add_v4(p.dX + (size_t)srow * p.d + n, val.x, val.y, val.z, val.w);
-                    }
-                }
-                __syncwarp();
-            }
-            tc_fence_before();
-            mbar_arrive(smem_u32(&sm.out_empty[buf]));
-            if (!go) break;
-        }
     }
     tc_fence_before();
     __syncthreads();
@@ -467,30 +369,24 @@ bool use_fused_backward(const Dims &dm) {
     return use_tc(dm) && dm.k <= 128;
 }
 
-cudaError_t tc_fused_backward(const Dims &dm, const void *W_q, const void *W_k, const void *W_v,
-                              const void *W_o, const void *dY, const Saved &sv, float *dX,
-                              bool with_dx, cudaStream_t s) {
+cudaError_t tc_fused_backward(const Dims &dm, const void *W_o, const void *dY, const Saved &sv,
+                              cudaStream_t s) {
     FusedBwdParams p;
     memset(&p, 0, sizeof(p));
     const int Mtok = dm.B * dm.k;
-    const void *W[3] = {W_q, W_k, W_v};
     const void *QKV[3] = {sv.Q, sv.K, sv.V};
     bool ok = map3(&p.mWo, W_o, dm.H, 64, dm.d, 64);
     for (int j = 0; j < 3; ++j)
-        ok = ok && map3(&p.mQKV[j], QKV[j], dm.H, Mtok, 128, 128) &&
-             map3(&p.mW[j], W[j], dm.H, dm.d, 64, 256);
+        ok = ok && map3(&p.mQKV[j], QKV[j], dm.H, Mtok, 128, 128);
     if (!ok) return cudaErrorInvalidValue;
     p.dY = static_cast<const bf16 *>(dY);
     p.gidx = sv.gidx;
     p.rsel = sv.rsel;
     p.A = sv.A;
     p.lse = sv.lse;
-    p.WrT = sv.WrT;
     p.dQKV = static_cast<bf16 *>(sv.dQKV);
     p.Dd = sv.Dd;
     p.dlogit = sv.dlogit;
-    p.dX = dX;
-    p.do_dx = with_dx ? 1 : 0;
     p.B = dm.B;
     p.T = dm.T;
     p.d = dm.d;

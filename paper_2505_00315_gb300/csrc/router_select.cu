@@ -6,7 +6,8 @@
 // which finds the exact k-th largest key.  A final in-order compaction keeps
 // every key above it plus the lowest-index keys equal to it, so I comes out
 // ascending (the order the causal mask works in) and ties go to the lower
-// token index.  Block-wide ranks use warp ballots, so no sort is needed.
+// token index.  Output positions come from one block-wide prefix sum of the
+// per-segment counts, so no sort is needed.
 #include <mutex>
 
 #include "launch.h"
@@ -44,41 +45,49 @@ constexpr int kSelThreads = 1024;   // upper bound; launches use 256 or 1024
 // five passes over them (four radix passes and the compaction).
 constexpr int kSelStagedMax = 16384;
 
-// Exclusive rank of this thread among the block's threads with `flag` set,
-// in thread order; `total` receives the block-wide count.  sh has 33 words.
-__device__ __forceinline__ uint32_t block_rank(bool flag, uint32_t *sh, uint32_t &total) {
+// Block-wide exclusive prefix sum of v (thread order); `total` receives the
+// sum.  sh has 33 entries.  Two barriers.
+__device__ __forceinline__ unsigned long long block_excl_scan(unsigned long long v,
+                                                              unsigned long long *sh,
+                                                              unsigned long long &total) {
     const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
     const int nwarps = blockDim.x >> 5;
-    const uint32_t ballot = __ballot_sync(0xffffffffu, flag);
-    if (lane == 0) sh[warp] = __popc(ballot);
+    unsigned long long incl = v;
+#pragma unroll
+    for (int off = 1; off < 32; off <<= 1) {
+        const unsigned long long y = __shfl_up_sync(0xffffffffu, incl, off);
+        if (lane >= off) incl += y;
+    }
+    if (lane == 31) sh[warp] = incl;
     __syncthreads();
     if (warp == 0) {
-        const uint32_t v = lane < nwarps ? sh[lane] : 0u;
-        uint32_t incl = v;
+        const unsigned long long w = lane < nwarps ? sh[lane] : 0ull;
+        unsigned long long wi = w;
 #pragma unroll
         for (int off = 1; off < 32; off <<= 1) {
-            const uint32_t y = __shfl_up_sync(0xffffffffu, incl, off);
-            if (lane >= off) incl += y;
+            const unsigned long long y = __shfl_up_sync(0xffffffffu, wi, off);
+            if (lane >= off) wi += y;
         }
-        sh[lane] = incl - v;
-        if (lane == 31) sh[32] = incl;
+        sh[lane] = wi - w;
+        if (lane == 31) sh[32] = wi;
     }
     __syncthreads();
-    const uint32_t r = sh[warp] + __popc(ballot & ((1u << lane) - 1u));
     total = sh[32];
-    __syncthreads();
-    return r;
+    return sh[warp] + incl - v;
 }
 
-// One CTA per row: 1024 threads when rows are long or few (the CTA's own
-// latency decides), 256 when many short rows fill the GPU several times over.
+// One CTA per row, 256 to 1024 threads (chosen at launch).
+// Radix passes use two histograms in turn (the next one is cleared while the
+// current one fills), so a pass costs two barriers; the compaction gives each
+// thread a contiguous segment of the row and places its selected keys after
+// one block-wide scan of the per-segment counts.
 __global__ void __launch_bounds__(kSelThreads)
 topk_select_kernel(const float *__restrict__ scores, int T, int k, int32_t *__restrict__ I,
                    float *__restrict__ rsel, int B, int H, int32_t *__restrict__ gidx,
                    float *__restrict__ rsel_hm) {
     extern __shared__ uint32_t keys_s[];   // the row's order keys when T <= kSelStagedMax
-    __shared__ uint32_t hist[256];
-    __shared__ uint32_t sh[33];
+    __shared__ uint32_t hist[2][256];
+    __shared__ unsigned long long sh[33];
     __shared__ uint32_t sh_prefix, sh_remaining;
     // the next kernel may launch and run its prologue as this grid's CTAs finish
     asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
@@ -87,21 +96,20 @@ topk_select_kernel(const float *__restrict__ scores, int T, int k, int32_t *__re
     const float *s = scores + (size_t)row * T;
     const int tid = threadIdx.x;
     const bool staged = T <= kSelStagedMax;
-    if (staged) {
+    for (int i = tid; i < 256; i += blockDim.x) hist[0][i] = 0u;
+    if (staged)
         for (int t = tid; t < T; t += blockDim.x) keys_s[t] = order_key(__ldg(s + t));
-        __syncthreads();
-    }
+    __syncthreads();
     auto key_at = [&](int t) -> uint32_t { return staged ? keys_s[t] : order_key(__ldg(s + t)); };
 
     uint32_t prefix = 0u, mask = 0u, remaining = (uint32_t)k;
     for (int pass = 0; pass < 4; ++pass) {
         const int shift = 24 - 8 * pass;
-        const uint32_t digit = 255u;
-        for (int i = tid; i < 256; i += blockDim.x) hist[i] = 0u;
-        __syncthreads();
+        uint32_t *hc = hist[pass & 1], *hn = hist[(pass + 1) & 1];
+        for (int i = tid; i < 256; i += blockDim.x) hn[i] = 0u;  // read by no one this pass
         for (int t = tid; t < T; t += blockDim.x) {
             const uint32_t key = key_at(t);
-            if ((key & mask) == prefix) atomicAdd(&hist[(key >> shift) & digit], 1u);
+            if ((key & mask) == prefix) atomicAdd(&hc[(key >> shift) & 255u], 1u);
         }
         __syncthreads();
         if (tid < 32) {
@@ -110,7 +118,7 @@ topk_select_kernel(const float *__restrict__ scores, int T, int k, int32_t *__re
             uint32_t c[8], sum = 0u;
 #pragma unroll
             for (int j = 0; j < 8; ++j) {
-                c[j] = hist[255 - (lane * 8 + j)];
+                c[j] = hc[255 - (lane * 8 + j)];
                 sum += c[j];
             }
             uint32_t incl = sum;
@@ -141,28 +149,31 @@ topk_select_kernel(const float *__restrict__ scores, int T, int k, int32_t *__re
         __syncthreads();
         prefix = sh_prefix;
         remaining = sh_remaining;
-        mask |= digit << shift;
-        __syncthreads();
+        mask |= 255u << shift;
     }
-    // prefix is now the k-th largest key; `remaining` keys equal to it are kept.
+    // prefix is now the k-th largest key; the first `remaining` keys equal to it
+    // (in token order) are kept, with every key above it.
     const uint32_t thr = prefix;
-    uint32_t base_eq = 0u, base_sel = 0u;
+    const int per = (T + (int)blockDim.x - 1) / (int)blockDim.x;
+    const int t0 = min(T, tid * per), t1 = min(T, t0 + per);
+    uint32_t n_gt = 0u, n_eq = 0u;
+    for (int t = t0; t < t1; ++t) {
+        const uint32_t key = key_at(t);
+        n_gt += key > thr ? 1u : 0u;
+        n_eq += key == thr ? 1u : 0u;
+    }
+    unsigned long long tot;
+    const unsigned long long before =
+        block_excl_scan(((unsigned long long)n_gt << 32) | n_eq, sh, tot);
+    uint32_t eq_before = (uint32_t)(before & 0xffffffffu);
+    uint32_t pos = (uint32_t)(before >> 32) + min(eq_before, remaining);
     const int hh = row % H, bb = row / H;
-    for (int t0 = 0; t0 < T; t0 += blockDim.x) {
-        const int t = t0 + tid;
-        float v = 0.f;
-        uint32_t key = 0u;
-        if (t < T) {
-            v = __ldg(s + t);
-            key = staged ? keys_s[t] : order_key(v);
-        }
-        const bool gt = t < T && key > thr;
-        const bool eq = t < T && key == thr;
-        uint32_t n_eq, n_sel;
-        const uint32_t eq_rank = base_eq + block_rank(eq, sh, n_eq);
-        const bool take = gt || (eq && eq_rank < remaining);
-        const uint32_t pos = base_sel + block_rank(take, sh, n_sel);
+    for (int t = t0; t < t1 && pos < (uint32_t)k; ++t) {
+        const uint32_t key = key_at(t);
+        bool take = key > thr;
+        if (key == thr) take = eq_before++ < remaining;
         if (take) {
+            const float v = __ldg(s + t);
             I[(size_t)row * k + pos] = t;
             rsel[(size_t)row * k + pos] = v;
             if (gidx != nullptr) {
@@ -170,9 +181,8 @@ topk_select_kernel(const float *__restrict__ scores, int T, int k, int32_t *__re
                 gidx[o] = bb * T + t;
                 rsel_hm[o] = v;
             }
+            ++pos;
         }
-        base_eq += n_eq;
-        base_sel += n_sel;
     }
 }
 
@@ -231,7 +241,11 @@ cudaError_t launch_select(int rows, int T, int k, const float *scores, int32_t *
     });
     if (attr != cudaSuccess) return attr;
     const size_t smem = T <= kSelStagedMax ? sizeof(uint32_t) * (size_t)T : 0;
-    const int threads = (T >= 2048 || rows < 608) ? 1024 : 256;
+    // about four keys per thread, 256..1024 threads; at most 512 once rows fill
+    // the GPU (measured best at rows x T = 128 x 1024, 1024 x 1024, 32..256 x
+    // 4096, 512 and 1024 x 4096, 64 x 8192)
+    int threads = T / 4 < 256 ? 256 : (T / 4 > 1024 ? 1024 : (T / 4 + 31) / 32 * 32);
+    if (rows >= 512 && threads > 512) threads = 512;
     cudaError_t e = launch_pdl(topk_select_kernel, dim3(rows), dim3(threads), smem, stream,
                                scores, T, k, I, rsel, B, H, gidx, rsel_hm);
     note_launches(1);

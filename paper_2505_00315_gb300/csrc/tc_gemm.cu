@@ -123,7 +123,7 @@ __host__ __device__ constexpr bool gathers() {
 // Kinds whose epilogue runs on all eight warps (wide output tiles).
 template <int KIND>
 __host__ __device__ constexpr bool epi_all_warps() {
-    return KIND == kQKV || KIND == kOUT || KIND == kDW || KIND == kDWO;
+    return KIND == kQKV || KIND == kOUT || KIND == kDW || KIND == kDWO || KIND == kROUTER;
 }
 
 template <int KIND>
@@ -591,13 +591,18 @@ __global__ void __launch_bounds__(kThreads, Cfg<KIND>::MIN_CTAS)
             const int bb = live ? mg / p.T : 0, t = live ? mg % p.T : 0;
             float *dst = p.out_f + (size_t)bb * p.H * p.T + t;
             const int ncols = min(C::BN, p.H - n0);
-            for (int c0 = 0; c0 < ncols; c0 += 32) {
+            // 32-column groups alternate between the two warps of a lane quarter;
+            // sigmoid(x) = 1 / (1 + 2^(-x log2 e)) with the hardware exp2 and
+            // reciprocal (relative error a few ulp)
+            for (int c0 = 32 * part; c0 < ncols; c0 += 64) {
                 float v[32];
                 tmem_ld32(tb + c0, v);
                 const int nv = live ? min(32, ncols - c0) : 0;
 #pragma unroll
                 for (int e = 0; e < 32; ++e) {
-                    if (e < nv) dst[(size_t)(n0 + c0 + e) * p.T] = 1.f / (1.f + expf(-v[e]));
+                    if (e < nv)
+                        dst[(size_t)(n0 + c0 + e) * p.T] =
+                            __frcp_rn(1.f + exp2_fast(-1.4426950408889634f * v[e]));
                 }
             }
         } else if constexpr (KIND == kDWO) {

@@ -9,18 +9,19 @@
 //            3-stage ring: W blocks by TMA, the selected rows of X by 16-byte
 //            cp.async gathers
 //   phase 2  the accumulator is read back and split into bf16 hi/lo pairs, kept
-//            in shared memory as the attention operands and copied to global
-//            memory (the backward reads them)
+//            in shared memory as the attention operands; warp 3 copies them to
+//            global memory (the backward reads them) by TMA stores while the
+//            softmax runs
 //   phase 3  S = Q K^T, block-diagonal causal softmax (two threads per row),
-//            O = P V; A = O / l, AR = r A and lse go to global memory, AR (a
-//            pair) also stays in shared memory
+//            O = P V; A = O / l and lse go to global memory; AR = r A (a pair)
+//            stays in shared memory and warp 3 stores it by TMA
 //   phase 4  Y[g(m), n] += (AR W_o[h])(m, n) for n in 256-wide chunks, W_o
 //            chunks double-buffered by TMA, accumulators double-buffered in
 //            TMEM so one chunk's scatter-add overlaps the next chunk's MMAs.
 // Products with one pair operand are two MMAs, with two pair operands three
 // (hi hi + hi lo + lo hi), as in the separate kernels.
 //
-// Warps: 0 TMA producer, 1 MMA issuer, 2 TMEM owner, 3 idle; 4-11 gather,
+// Warps: 0 TMA producer, 1 MMA issuer, 2 TMEM owner, 3 TMA stores; 4-11 gather,
 // softmax and epilogues, two per TMEM lane quadrant (warp w serves tile rows
 // 32 (w % 4) .. +31 and column half (w - 4) / 4).  Every wait is bounded.
 #include <mutex>
@@ -53,7 +54,7 @@ struct FusedSmem {
     float part_max[2][128], part_sum[2][128];
     int rows[128];           // b*T + I of each tile row, -1 for rows outside the tile's sequences
     uint64_t full[kStages], empty[kStages];
-    uint64_t qkv_done, qkv_staged, s_full, p_ready, o_full, ar_ready;
+    uint64_t qkv_done, qkv_staged, qkv_read, s_full, p_ready, o_full, ar_ready;
     uint64_t wo_full[2], wo_empty[2], out_full[2], out_empty[2];
     uint32_t tmem;
     int abort;
@@ -64,12 +65,11 @@ static_assert(kSmem <= 227 * 1024, "shared memory");
 struct FusedParams {
     CUtensorMap mW[3];     // W_q, W_k, W_v: [H, d, 64], box {64, 64, 1}
     CUtensorMap mWo;       // W_o: [H, 64, d], box {64, 64, 1}
+    CUtensorMap mOut[4];   // Q, K, V, AR pairs: [H, B*k, 128], box {64, U k, 1} (stores)
     const bf16 *X;         // [B*T, d]
     const int32_t *gidx;   // [H, B*k]
     const float *rsel;     // [H, B*k]
-    bf16 *Q, *K, *V;       // [H, B*k, 128] pairs
     float *A;              // [H, B*k, 64]
-    bf16 *AR;              // [H, B*k, 128] pair
     float *lse;            // [H, B*k]
     float *Y;              // [B*T, d], accumulated into
     int B, T, d, k, U, Mtok;
@@ -107,6 +107,7 @@ __global__ void __launch_bounds__(kThreads, 1) fused_fwd_kernel(const __grid_con
         }
         mbar_init(smem_u32(&sm.qkv_done), 1);
         mbar_init(smem_u32(&sm.qkv_staged), kWorkers);
+        mbar_init(smem_u32(&sm.qkv_read), 1);
         mbar_init(smem_u32(&sm.s_full), 1);
         mbar_init(smem_u32(&sm.p_ready), kWorkers);
         mbar_init(smem_u32(&sm.o_full), 1);
@@ -146,8 +147,10 @@ __global__ void __launch_bounds__(kThreads, 1) fused_fwd_kernel(const __grid_con
                 for (int j = 0; j < 3; ++j)
                     tma_load_3d(smem_u32(sm.ring[s] + kHalf + j * 8192), &p.mW[j], fb, 0, kb * 64, h);
             }
-            // phase 4: W_o chunks into the K / V tiles once P V is done
-            if (wait_or_abort(sm, sm.o_full, 0, p.status)) {
+            // phase 4: W_o chunks into the K / V tiles once P V is done and
+            // their TMA stores have read them
+            if (wait_or_abort(sm, sm.o_full, 0, p.status) &&
+                wait_or_abort(sm, sm.qkv_read, 0, p.status)) {
                 for (int c = 0; c < nch; ++c) {
                     const int buf = c & 1;
                     if (c >= 2 && !wait_or_abort(sm, sm.wo_empty[buf], ((c >> 1) - 1) & 1, p.status))
@@ -237,6 +240,28 @@ __global__ void __launch_bounds__(kThreads, 1) fused_fwd_kernel(const __grid_con
                 for (int i = 0; i < 2; ++i) mma_commit(smem_u32(&sm.out_full[i]));
             }
         }
+    } else if (warp == 3) {
+        // ------------------------------------------------- TMA stores
+        if (lane == 0) {
+            // Q, K, V pairs straight from the attention operand tiles
+            bool ok = wait_or_abort(sm, sm.qkv_staged, 0, p.status);
+            if (ok) {
+                uint8_t(*tiles[3])[kHalf] = {sm.q, sm.k, sm.v};
+                for (int j = 0; j < 3; ++j)
+                    for (int hf = 0; hf < 2; ++hf)
+                        tma_store_3d(&p.mOut[j], smem_u32(tiles[j][hf]), 64 * hf, b0 * p.k, h);
+                bulk_commit();
+            }
+            bulk_wait_read0();
+            mbar_arrive(smem_u32(&sm.qkv_read));   // the tiles may be overwritten
+            // AR pair from the Q tile (the A operand of phase 4)
+            if (ok && wait_or_abort(sm, sm.ar_ready, 0, p.status)) {
+                for (int hf = 0; hf < 2; ++hf)
+                    tma_store_3d(&p.mOut[3], smem_u32(sm.q[hf]), 64 * hf, b0 * p.k, h);
+                bulk_commit();
+            }
+            bulk_wait0();
+        }
     } else if (warp >= 4) {
         const int t = threadIdx.x - 128;            // 0..255
         const int q = warp & 3, ch = (warp - 4) >> 2;
@@ -292,21 +317,6 @@ __global__ void __launch_bounds__(kThreads, 1) fused_fwd_kernel(const __grid_con
         tc_fence_before();
         named_barrier(1, kWorkers);
         mbar_arrive(smem_u32(&sm.qkv_staged));
-        {
-            // warps with ch = 0 copy the hi halves, ch = 1 the lo halves (128 B per row each)
-            bf16 *dstm[3] = {p.Q, p.K, p.V};
-            const uint8_t *srcm[3] = {sm.q[ch], sm.k[ch], sm.v[ch]};
-            const int cu = lane & 7;
-#pragma unroll
-            for (int j = 0; j < 3; ++j)
-#pragma unroll
-                for (int i = 0; i < 8; ++i) {
-                    const int rl = (lane >> 3) + 4 * i, row = q * 32 + rl;
-                    const uint4 val = *reinterpret_cast<const uint4 *>(srcm[j] + row * 128 + ((cu ^ (row & 7)) << 4));
-                    if (ok && ((vmask >> rl) & 1u))
-                        *(reinterpret_cast<uint4 *>(dstm[j] + (grow0 + rl) * 128 + ch * 64) + cu) = val;
-                }
-        }
 
         // -------------------------------------------------- phase 3: softmax
         ok = wait_or_abort(sm, sm.s_full, 0, p.status) && ok;
@@ -343,6 +353,7 @@ __global__ void __launch_bounds__(kThreads, 1) fused_fwd_kernel(const __grid_con
         ok = wait_or_abort(sm, sm.o_full, 0, p.status) && ok;
         tc_fence_after();
         named_barrier(1, kWorkers);   // partial sums visible; Q tile no longer read
+        ok = wait_or_abort(sm, sm.qkv_read, 0, p.status) && ok;   // nor by its TMA store
         l = sm.part_sum[0][r] + sm.part_sum[1][r];
         float o[32];
         tmem_ld32(tmem + 128 + lane_off + 32 * ch, o);   // output columns 32 ch .. +31
@@ -360,13 +371,6 @@ __global__ void __launch_bounds__(kThreads, 1) fused_fwd_kernel(const __grid_con
             store_rows128(xb, lane, [&](int rl, int c) -> uint4 * {
                 if (!((vmask >> rl) & 1u)) return nullptr;
                 return reinterpret_cast<uint4 *>(p.A + (grow0 + rl) * 64 + 32 * ch) + c;
-            });
-            stage_pair32(xb, o, inv * rr, lane);
-            store_rows128(xb, lane, [&](int rl, int c) -> uint4 * {
-                if (!((vmask >> rl) & 1u)) return nullptr;
-                bf16 *base = p.AR + (grow0 + rl) * 128 + 32 * ch;
-                return c < 4 ? reinterpret_cast<uint4 *>(base) + c
-                             : reinterpret_cast<uint4 *>(base + 64) + (c - 4);
             });
             if (ch == 0 && valid) p.lse[grow0 + lane] = (m + log2f(l)) * 0.69314718055994531f;
         }
@@ -427,17 +431,17 @@ cudaError_t tc_fused_forward(const Dims &dm, const void *X, const void *Wq, cons
     FusedParams p;
     memset(&p, 0, sizeof(p));
     const void *W[3] = {Wq, Wk, Wv};
+    const int U = 128 / dm.k;
+    const void *outs[4] = {sv.Q, sv.K, sv.V, sv.AR};
     bool ok = map_heads3(&p.mWo, Wo, dm.H, 64, dm.d, 64);
     for (int j = 0; j < 3; ++j) ok = ok && map_heads3(&p.mW[j], W[j], dm.H, dm.d, 64, 64);
+    for (int j = 0; j < 4; ++j)
+        ok = ok && map_heads3(&p.mOut[j], outs[j], dm.H, (uint64_t)dm.B * dm.k, 128, U * dm.k);
     if (!ok) return cudaErrorInvalidValue;
     p.X = static_cast<const bf16 *>(X);
     p.gidx = sv.gidx;
     p.rsel = sv.rsel;
-    p.Q = static_cast<bf16 *>(sv.Q);
-    p.K = static_cast<bf16 *>(sv.K);
-    p.V = static_cast<bf16 *>(sv.V);
     p.A = sv.A;
-    p.AR = static_cast<bf16 *>(sv.AR);
     p.lse = sv.lse;
     p.Y = Y;
     p.B = dm.B;

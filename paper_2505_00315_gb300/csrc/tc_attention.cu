@@ -43,7 +43,6 @@ struct AttnParams {
     int U;                    // k <= 128: sequences packed into one 128-row tile
     float scale_log2;         // log2(e) / sqrt(h')
     const float *rsel;        // [H, B*k]
-    float *A;                 // [H, B*k, 64]
     bf16 *AR;                 // [H, B*k, 128] pair
     float *lse;               // [H, B*k]
     uint32_t *status;
@@ -307,11 +306,6 @@ __global__ void __launch_bounds__(kLT, 1) attn_fwd_tc_kernel(const __grid_consta
         if (live) {
             uint8_t *xb = &sm.kv[0][0][0] + (warp - 4) * 4096;   // the ring is idle now
             const float inv = valid ? 1.f / l : 0.f;
-            stage_f32x32(xb, o, inv, lane);
-            store_rows128(xb, lane, [&](int rl, int c) -> uint4 * {
-                if (!((vmask >> rl) & 1u)) return nullptr;
-                return reinterpret_cast<uint4 *>(p.A + (row0 + rl) * 64 + 32 * ch) + c;
-            });
             const float rr = valid ? p.rsel[row0 + lane] : 0.f;
             stage_pair32(xb, o, inv * rr, lane);
             store_rows128(xb, lane, [&](int rl, int c) -> uint4 * {
@@ -797,11 +791,6 @@ __global__ void __launch_bounds__(kSmallThreads, 1) attn_fwd_small_kernel(const 
             // Q tile is free once S is done: 4 KB of staging per softmax warp
             uint8_t *xb = sm.q[0] + (warp - 4) * 4096;
             const float inv = tr.valid ? 1.f / l : 0.f;
-            stage_f32x32(xb, o, inv, lane);
-            store_rows128(xb, lane, [&](int rl, int c) -> uint4 * {
-                if (!((vmask >> rl) & 1u)) return nullptr;
-                return reinterpret_cast<uint4 *>(p.A + (row0 + rl) * 64 + 32 * ch) + c;
-            });
             const float rr = tr.valid ? p.rsel[row0 + lane] : 0.f;
             stage_pair32(xb, o, inv * rr, lane);
             store_rows128(xb, lane, [&](int rl, int c) -> uint4 * {
@@ -1007,7 +996,6 @@ cudaError_t tc_attn_fwd(const Dims &dm, const Saved &sv, cudaStream_t s) {
     p.Mtok = dm.B * dm.k;
     p.scale_log2 = 1.4426950408889634f / sqrtf(64.f);
     p.rsel = sv.rsel;
-    p.A = sv.A;
     p.AR = static_cast<bf16 *>(sv.AR);
     p.lse = sv.lse;
     p.status = sv.status;

@@ -88,6 +88,21 @@ __device__ __forceinline__ void tma_load_4d(uint32_t dst, const CUtensorMap *map
         "l"(map), "r"(bar), "r"(c0), "r"(c1), "r"(c2), "r"(c3)
         : "memory");
 }
+// Dot product of 8 bf16 pair values (hi word h4, lo word l4: columns c..c+7)
+// with g[0..7], added to acc.
+__device__ __forceinline__ float dot_pair8(const uint4 &h4, const uint4 &l4, const float *g,
+                                           float acc) {
+    const uint32_t hw[4] = {h4.x, h4.y, h4.z, h4.w}, lw[4] = {l4.x, l4.y, l4.z, l4.w};
+#pragma unroll
+    for (int e = 0; e < 4; ++e) {
+        const float a0 = __uint_as_float(hw[e] << 16) + __uint_as_float(lw[e] << 16);
+        const float a1 = __uint_as_float(hw[e] & 0xFFFF0000u) + __uint_as_float(lw[e] & 0xFFFF0000u);
+        acc = fmaf(a0, g[2 * e], acc);
+        acc = fmaf(a1, g[2 * e + 1], acc);
+    }
+    return acc;
+}
+
 // Shared-memory tile to a 3-D tensor (box at c0, c1, c2; rows outside the
 // tensor are not written), tracked by the issuing thread's bulk async-group.
 __device__ __forceinline__ void tma_store_3d(const CUtensorMap *map, uint32_t src, int c0, int c1,

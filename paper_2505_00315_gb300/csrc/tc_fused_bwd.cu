@@ -4,8 +4,8 @@
 // on the tensor cores with fp32 accumulators in TMEM:
 //   phase 1  G = dY[g(m), :] W_o[h]^T        K = d in 64-wide blocks, a 3-stage
 //            ring: W_o blocks by TMA, the selected rows of dY by cp.async
-//   phase 2  dr = <A, G>, dA = r G (bf16 pair, shared memory), D = r dr,
-//            dlogit = dr r (1 - r) (the router gradient through diag(r))
+//   phase 2  D = <AR, G> = r <A, G>, dA = r G (bf16 pair, shared memory),
+//            dlogit = D (1 - r) (the router gradient through diag(r))
 //   phase 3  S = Q K^T, dP = dA V^T; P from the saved log-sum-exp; dV = P^T dA;
 //            dS = P o (dP - D); dK = dS^T Q / sqrt(h'), dQ = dS K / sqrt(h')
 //   phase 4  dQ|dK|dV (and dlogit) to global memory for dX and the weight
@@ -62,7 +62,7 @@ struct FusedBwdParams {
     const bf16 *dY;        // [B*T, d]
     const int32_t *gidx;   // [H, B*k]
     const float *rsel;     // [H, B*k]
-    const float *A;        // [H, B*k, 64]
+    const bf16 *AR;        // [H, B*k, 128] pair of AR = diag(r) A
     const float *lse;      // [H, B*k]
     bf16 *dQKV;            // [H, B*k, 512] pair: dQ|dK|dV|dlogit hi, then lo
     float *Dd, *dlogit;    // [H, B*k]
@@ -245,27 +245,22 @@ __global__ void __launch_bounds__(kThreads, 1) fused_bwd_kernel(const __grid_con
         tc_fence_after();
         float g[32];
         tmem_ld32(tmem + kColG + lane_off + 32 * ch, g);   // G columns 32 ch .. +31
-        float dr = 0.f;
+        float dd = 0.f;   // this half of D = <AR, G> = r <A, G>
         if (valid) {
-            const float4 *arow = reinterpret_cast<const float4 *>(p.A + grow * 64 + 32 * ch);
+            // columns 32 ch .. +31 of the AR pair row: hi at 32 ch, lo at 64 + 32 ch
+            const uint4 *hrow = reinterpret_cast<const uint4 *>(p.AR + grow * 128 + 32 * ch);
+            const uint4 *lrow = reinterpret_cast<const uint4 *>(p.AR + grow * 128 + 64 + 32 * ch);
 #pragma unroll
-            for (int e4 = 0; e4 < 8; ++e4) {
-                const float4 a4 = arow[e4];
-                dr = fmaf(a4.x, g[4 * e4 + 0], dr);
-                dr = fmaf(a4.y, g[4 * e4 + 1], dr);
-                dr = fmaf(a4.z, g[4 * e4 + 2], dr);
-                dr = fmaf(a4.w, g[4 * e4 + 3], dr);
-            }
+            for (int u = 0; u < 4; ++u) dd = dot_pair8(hrow[u], lrow[u], g + 8 * u, dd);
         }
         const float rr = valid ? p.rsel[grow] : 0.f;
         put_pair32(sm.da[0], sm.da[1], r, 32 * ch, g, rr);   // dA = r G
-        sm.part[ch][r] = dr;
+        sm.part[ch][r] = dd;
         fence_proxy_async();
         tc_fence_before();
         named_barrier(1, kWorkers);
-        dr = sm.part[0][r] + sm.part[1][r];
-        const float dd = rr * dr;                    // D = rowsum(dA o A)
-        const float dlg = dr * rr * (1.f - rr);      // dlogit
+        dd = sm.part[0][r] + sm.part[1][r];          // D = rowsum(dA o A)
+        const float dlg = dd * (1.f - rr);           // dlogit = r (1 - r) <A, G>
         if (ch == 0) {
             sm.Dd[r] = dd;
             if (ok && valid) {
@@ -382,7 +377,7 @@ cudaError_t tc_fused_backward(const Dims &dm, const void *W_o, const void *dY, c
     p.dY = static_cast<const bf16 *>(dY);
     p.gidx = sv.gidx;
     p.rsel = sv.rsel;
-    p.A = sv.A;
+    p.AR = static_cast<const bf16 *>(sv.AR);
     p.lse = sv.lse;
     p.dQKV = static_cast<bf16 *>(sv.dQKV);
     p.Dd = sv.Dd;

@@ -13,8 +13,9 @@
 //            global memory (the backward reads them) by TMA stores while the
 //            softmax runs
 //   phase 3  S = Q K^T, block-diagonal causal softmax (two threads per row),
-//            O = P V; A = O / l and lse go to global memory; AR = r A (a pair)
-//            stays in shared memory and warp 3 stores it by TMA
+//            O = P V; lse goes to global memory; AR = r A / l (a pair) stays in
+//            shared memory and warp 3 stores it by TMA (the backward needs A
+//            only through AR)
 //   phase 4  Y[g(m), n] += (AR W_o[h])(m, n) for n in 256-wide chunks, W_o
 //            chunks double-buffered by TMA, accumulators double-buffered in
 //            TMEM so one chunk's scatter-add overlaps the next chunk's MMAs.
@@ -69,7 +70,6 @@ struct FusedParams {
     const bf16 *X;         // [B*T, d]
     const int32_t *gidx;   // [H, B*k]
     const float *rsel;     // [H, B*k]
-    float *A;              // [H, B*k, 64]
     float *lse;            // [H, B*k]
     float *Y;              // [B*T, d], accumulated into
     int B, T, d, k, U, Mtok;
@@ -270,7 +270,6 @@ __global__ void __launch_bounds__(kThreads, 1) fused_fwd_kernel(const __grid_con
         const int u = r / p.k;
         const bool valid = u < p.U && b0 + u < p.B;
         const int lo = valid ? u * p.k : r + 1;     // first visible key (none when invalid)
-        const unsigned vmask = __ballot_sync(0xffffffffu, valid);
         const size_t grow0 = row_base + q * 32;     // head row of lane 0's tile row
 
         // ------------------------------------------- phase 1: gather X rows
@@ -366,14 +365,7 @@ __global__ void __launch_bounds__(kThreads, 1) fused_fwd_kernel(const __grid_con
         mbar_arrive(smem_u32(&sm.ar_ready));
         const bool live = __all_sync(0xffffffffu, ok && !*(volatile int *)&sm.abort);
         uint8_t *xb = stage_area + (warp - 4) * 4096;
-        if (live) {
-            stage_f32x32(xb, o, inv, lane);
-            store_rows128(xb, lane, [&](int rl, int c) -> uint4 * {
-                if (!((vmask >> rl) & 1u)) return nullptr;
-                return reinterpret_cast<uint4 *>(p.A + (grow0 + rl) * 64 + 32 * ch) + c;
-            });
-            if (ch == 0 && valid) p.lse[grow0 + lane] = (m + log2f(l)) * 0.69314718055994531f;
-        }
+        if (live && ch == 0 && valid) p.lse[grow0 + lane] = (m + log2f(l)) * 0.69314718055994531f;
 
         // ------------------------------------- phase 4: scatter-add into Y
         const int cu = lane & 7;
@@ -441,7 +433,6 @@ cudaError_t tc_fused_forward(const Dims &dm, const void *X, const void *Wq, cons
     p.X = static_cast<const bf16 *>(X);
     p.gidx = sv.gidx;
     p.rsel = sv.rsel;
-    p.A = sv.A;
     p.lse = sv.lse;
     p.Y = Y;
     p.B = dm.B;

@@ -18,7 +18,7 @@
 // a product with one is two MMAs into the same accumulator):
 //   kQKV  F3  [Q|K|V](m,:)  = X[g(m),:] W_{q|k|v}[h]        A gathered K-major, B MN-major
 //   kOUT  F5  Y[g(m),n]    += (diag(r) A)(m,:) W_o[h](:,n)   A = AR pair,  B MN-major
-//   kG    B1  G(m,:)        = dY[g(m),:] W_o[h]^T, then dr, dA = r G, D, dlogit in the epilogue
+//   kG    B1  G(m,:)        = dY[g(m),:] W_o[h]^T, then D = <AR, G>, dA = r G, dlogit in the epilogue
 //   kDWO  B1  dW_o[h](p,c)  = sum_m AR(m,p) dY[g(m),c]       A gathered MN-major, B = AR pair
 //   kDW   B4  [dW_q|dW_k|dW_v|dW_r][h](c,:) = sum_m X[g(m),c] [dQ|dK|dV|dlogit](m,:)
 //             A gathered MN-major, B = the dQKV pair (its 4th 64-column block holds
@@ -145,7 +145,7 @@ struct TcParams {
     int d, H, T;
     const int32_t *gidx;   // [H, B*k]
     const float *rsel;     // [H, B*k]
-    const float *A32;      // [H, B*k, 64] attention output (kG)
+    const bf16 *ARp;       // [H, B*k, 128] pair of AR = diag(r) A (kG)
     const void *src_rows;  // gathered source [B*T, d] bf16: X (kQKV, kDW) or dY (kG, kDWO)
     void *out[3];          // Q/K/V pairs (kQKV); dA pair, dQKV pair (kG)
     float *out_f;          // Y (kOUT), dW_o (kDWO), dW_q (kDW)
@@ -531,34 +531,32 @@ __global__ void __launch_bounds__(kThreads, Cfg<KIND>::MIN_CTAS)
                 __syncwarp();
             }
         } else if constexpr (KIND == kG) {
-            // G row in two 32-column halves: dr = <A, G> accumulates, dA = r G is staged
+            // G row in two 32-column halves: D = <AR, G> = r <A, G> accumulates,
+            // dA = r G is staged
             const bool live = mg < p.M;
             const size_t row = (size_t)h * p.Mtok + (live ? mg : 0);
             const float rr = live ? p.rsel[row] : 0.f;
-            const float4 *arow = reinterpret_cast<const float4 *>(p.A32 + row * 64);
-            float dr = 0.f;
+            const uint4 *arow = reinterpret_cast<const uint4 *>(p.ARp + row * 128);  // hi 0..7, lo 8..15
+            const uint4 z4 = make_uint4(0u, 0u, 0u, 0u);
+            float dd = 0.f;
 #pragma unroll
             for (int hlf = 0; hlf < 2; ++hlf) {
                 float g[32];
                 tmem_ld32(tb + 32 * hlf, g);
 #pragma unroll
-                for (int e4 = 0; e4 < 8; ++e4) {
-                    const float4 a4 = live ? arow[8 * hlf + e4] : make_float4(0.f, 0.f, 0.f, 0.f);
-                    dr = fmaf(a4.x, g[4 * e4 + 0], dr);
-                    dr = fmaf(a4.y, g[4 * e4 + 1], dr);
-                    dr = fmaf(a4.z, g[4 * e4 + 2], dr);
-                    dr = fmaf(a4.w, g[4 * e4 + 3], dr);
-                }
+                for (int u = 0; u < 4; ++u)
+                    dd = dot_pair8(live ? arow[4 * hlf + u] : z4, live ? arow[8 + 4 * hlf + u] : z4,
+                                   g + 8 * u, dd);
 #pragma unroll
                 for (int e = 0; e < 32; ++e) g[e] *= rr;  // dA = r G, kept as a bf16 pair
 #pragma unroll
                 for (int u = 0; u < 4; ++u) stage_pair_unit(xb, lane, 4 * hlf + u, g + 8 * u);
             }
             __syncwarp();
-            // D = rowsum(dA o A) = r dr; dlogit = dr r (1 - r)
-            const float dl = dr * rr * (1.f - rr);
+            // D = rowsum(dA o A) = r <A, G>; dlogit = r (1 - r) <A, G> = D (1 - r)
+            const float dl = dd * (1.f - rr);
             if (live) {
-                p.out_f1[row] = rr * dr;
+                p.out_f1[row] = dd;
                 p.out_f2[row] = dl;
             }
             const int row0 = m0 + q * 32;
@@ -825,7 +823,7 @@ cudaError_t tc_out_bwd_g(const Dims &dm, const void *Wo, const void *dY, const S
               map_heads(&p.mapB[0], Wo, dm.H, 64, dm.d, 64);
     if (!ok) return cudaErrorInvalidValue;
     p.src_rows = dY;
-    p.A32 = sv.A;
+    p.ARp = static_cast<const bf16 *>(sv.AR);
     p.out[0] = sv.dA;
     p.out[1] = sv.dQKV;
     p.out_f1 = sv.Dd;

@@ -331,6 +331,7 @@ __global__ void __launch_bounds__(kLT, 1) attn_fwd_tc_kernel(const __grid_consta
 struct BwdParams {
     CUtensorMap mA0, mA1, mB0, mB1;   // dK/dV: K, V (128 rows), Q, dA (64 rows); dQ: Q, dA (128), K, V (64)
                                       // k <= 128: Q, K, V, dA as 3-D maps over [H, B*k, 128]
+    CUtensorMap mOut;                 // k <= 128: dQKV [H, B*k, 512], box {64, U k, 1} (stores)
     int k, Mtok;
     int U, B;                         // k <= 128: sequences per tile, batch
     float scale, scale_log2;
@@ -932,24 +933,26 @@ __global__ void __launch_bounds__(kSmallThreads, 1) attn_bwd_small_kernel(const 
         tc_fence_after();
         if (!ok) flag_timeout_b(sm, p.status);
         const bool live = __all_sync(0xffffffffu, ok && !*(volatile int *)&sm.abort);
-        const unsigned vmask = __ballot_sync(0xffffffffu, valid);
-        // dQ, dK, dV columns 32 ch .. +31 as bf16 pairs in the dQKV row layout
-        // (hi at column off + 32 ch, lo 256 further); the Q tile is free by now
-        uint8_t *xb = sm.q[0] + (warp - 4) * 4096;
+        // dQ, dK, dV columns 32 ch .. +31 as bf16 pairs into the Q, K, V tiles
+        // (free once every MMA is done), then out by six TMA stores into the
+        // dQKV rows: hi blocks at columns 0, 64, 128, lo blocks 256 further
+        uint8_t(*tiles[3])[kPBig] = {sm.q, sm.k, sm.v};
         const uint32_t src[3] = {tDQ, tDK, tDV};
         const float fac[3] = {p.scale, p.scale, 1.f};
 #pragma unroll 1
         for (int t = 0; t < 3; ++t) {
             float v[32];
             tmem_ld32(src[t] + lane_off + 32 * ch, v);
-            if (!live) continue;
-            stage_pair32(xb, v, fac[t], lane);
-            store_rows128(xb, lane, [&](int rl, int c) -> uint4 * {
-                if (!((vmask >> rl) & 1u)) return nullptr;
-                bf16 *row = p.dQKV + (base + q * 32 + rl) * 512 + 64 * t + 32 * ch;
-                return c < 4 ? reinterpret_cast<uint4 *>(row) + c
-                             : reinterpret_cast<uint4 *>(row + 256) + (c - 4);
-            });
+            put_pair32(tiles[t][0], tiles[t][1], r, 32 * ch, v, fac[t]);
+        }
+        fence_proxy_async();
+        named_barrier(1, kSoftmaxThreads);
+        if (threadIdx.x == 128 && live) {
+            for (int t = 0; t < 3; ++t)
+                for (int hf = 0; hf < 2; ++hf)
+                    tma_store_3d(&p.mOut, smem_u32(tiles[t][hf]), 64 * t + 256 * hf, b0 * p.k, h);
+            bulk_commit();
+            bulk_wait0();
         }
     }
     tc_fence_before();
@@ -1029,10 +1032,14 @@ cudaError_t tc_attn_bwd(const Dims &dm, const Saved &sv, cudaStream_t s) {
         BwdParams sp;
         memset(&sp, 0, sizeof(sp));
         const int Mtok = dm.B * dm.k;
-        const bool ok = map_rows(&sp.mA0, sv.Q, dm.H, Mtok) && map_rows(&sp.mA1, sv.K, dm.H, Mtok) &&
-                        map_rows(&sp.mB0, sv.V, dm.H, Mtok) && map_rows(&sp.mB1, sv.dA, dm.H, Mtok);
-        if (!ok) return cudaErrorInvalidValue;
         sp.U = kSmallK / dm.k;
+        const uint64_t odims[3] = {512, (uint64_t)Mtok, (uint64_t)dm.H};
+        const uint64_t ostrides[2] = {1024, (uint64_t)Mtok * 1024};
+        const uint32_t obox[3] = {64, (uint32_t)(sp.U * dm.k), 1};
+        const bool ok = map_rows(&sp.mA0, sv.Q, dm.H, Mtok) && map_rows(&sp.mA1, sv.K, dm.H, Mtok) &&
+                        map_rows(&sp.mB0, sv.V, dm.H, Mtok) && map_rows(&sp.mB1, sv.dA, dm.H, Mtok) &&
+                        tmap_bf16(&sp.mOut, sv.dQKV, 3, odims, ostrides, obox);
+        if (!ok) return cudaErrorInvalidValue;
         sp.B = dm.B;
         sp.k = dm.k;
         sp.Mtok = dm.B * dm.k;

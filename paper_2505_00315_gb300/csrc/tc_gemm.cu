@@ -21,8 +21,9 @@
 //   kG    B1  G(m,:)        = dY[g(m),:] W_o[h]^T, then D = <AR, G>, dA = r G, dlogit in the epilogue
 //   kDWO  B1  dW_o[h](p,c)  = sum_m AR(m,p) dY[g(m),c]       A gathered MN-major, B = AR pair
 //   kDW   B4  [dW_q|dW_k|dW_v|dW_r][h](c,:) = sum_m X[g(m),c] [dQ|dK|dV|dlogit](m,:)
-//             A gathered MN-major, B = the dQKV pair (its 4th 64-column block holds
-//             dlogit in column 0 and zeros), so dW_r comes out of the same product;
+//             A gathered MN-major, B = the dQKV pair (column 0 of its 4th 64-column
+//             block holds dlogit; the rest of that block only reaches unread
+//             accumulator columns), so dW_r comes out of the same product;
 //             256 rows c per CTA in two accumulators that share every B tile
 //   kROUTER F1 r[b,h,t] = sigmoid(X[b,t,:] W_r[:,h])       A = X tiles, B = W_r MN-major
 // where g(m) = b*T + I[b,h,i] for row m = b*k + i of head h.  B3 (dX) has a
@@ -565,24 +566,16 @@ __global__ void __launch_bounds__(kThreads, Cfg<KIND>::MIN_CTAS)
             store_rows256(xb, lane, nrows, [&](int rl, int u) {
                 return reinterpret_cast<uint4 *>(dA + (size_t)rl * 128) + u;
             });
-            // column block 3 of the dQKV pair: dlogit, then zeros (read by kDW for dW_r)
-            {
+            // dlogit as column 192 (hi) / 448 (lo) of the dQKV pair row, column 0 of
+            // the 4th 64-column block that kDW reads for dW_r; the block's other
+            // columns are never written: accumulator column n of that product
+            // depends only on B column n, and columns 193..255 are not read
+            if (live) {
                 const bf16 dh = __float2bfloat16_rn(dl);
                 const bf16 dlo = __float2bfloat16_rn(dl - __bfloat162float(dh));
-                const uint4 z = make_uint4(0, 0, 0, 0);
-#pragma unroll
-                for (int u = 0; u < 16; ++u) {
-                    uint4 v4 = z;
-                    if (u == 0) v4.x = (uint32_t)__bfloat16_as_ushort(dh);
-                    if (u == 8) v4.x = (uint32_t)__bfloat16_as_ushort(dlo);
-                    *reinterpret_cast<uint4 *>(xb + xoff256(lane, u)) = v4;
-                }
-                __syncwarp();
-                bf16 *dq = static_cast<bf16 *>(p.out[1]) + ((size_t)h * p.Mtok + row0) * kDQKVCols;
-                store_rows256(xb, lane, nrows, [&](int rl, int u) {
-                    bf16 *base = dq + (size_t)rl * kDQKVCols + (u < 8 ? 192 : 448 - 64);
-                    return reinterpret_cast<uint4 *>(base) + u;
-                });
+                bf16 *dq = static_cast<bf16 *>(p.out[1]) + row * kDQKVCols;
+                dq[192] = dh;
+                dq[448] = dlo;
             }
         } else if constexpr (KIND == kROUTER) {
             const bool live = mg < p.M;

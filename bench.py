@@ -464,36 +464,71 @@ def main():
     finally:
         os.environ.pop("MOSA_GRAPHS", None)
 
-    # End to end through the public API with pinned host buffers.
+    # End to end through the public API with pinned host buffers, pipelined as a
+    # training loop runs it: step i's inputs are copied in on one stream while
+    # step i-1 computes, and its outputs copied out on another while step i+1
+    # computes (two device buffer sets).  The timed region holds every step's
+    # copies and compute; it ends when the last step's outputs are on the host.
     hX = torch.from_numpy(x["X"]).to(tdt).pin_memory()
     hdY = torch.from_numpy(x["dY"]).to(tdt).pin_memory()
     hY = torch.empty((cfg.B, cfg.T, cfg.d), dtype=torch.float32).pin_memory()
     hdX = torch.empty((cfg.B, cfg.T, cfg.d), dtype=torch.float32).pin_memory()
-    Xd = torch.empty_like(D["X"])
-    dYd = torch.empty_like(D["dY"])
+    slots = [{"X": torch.empty_like(D["X"]), "dY": torch.empty_like(D["dY"]),
+              "outs": {n: torch.empty_like(v) for n, v in outs.items()},
+              "grads": {n: torch.empty_like(v) for n, v in grads.items()}} for _ in range(2)]
+    comp = torch.cuda.current_stream()
+    s_in, s_out = torch.cuda.Stream(), torch.cuda.Stream()
+    in_ready = [torch.cuda.Event() for _ in range(2)]
+    in_free = [torch.cuda.Event() for _ in range(2)]
+    done = [torch.cuda.Event() for _ in range(2)]
+    out_free = [torch.cuda.Event() for _ in range(2)]
     e2e_steps = max(10, K // 4)
 
-    def e2e_step():
-        Xd.copy_(hX, non_blocking=True)
-        dYd.copy_(hdY, non_blocking=True)
-        step(Xd, dYd)
-        hY.copy_(outs["Y"], non_blocking=True)
-        hdX.copy_(grads["dX"], non_blocking=True)
+    def e2e_run(n, start_event=None):
+        if start_event is not None:
+            s_in.wait_event(start_event)
+            s_out.wait_event(start_event)
+        for i in range(n):
+            j = i % 2
+            sl = slots[j]
+            with torch.cuda.stream(s_in):
+                if i >= 2:
+                    s_in.wait_event(in_free[j])   # step i-2 is done with these inputs
+                sl["X"].copy_(hX, non_blocking=True)
+                if cfg.backward:
+                    sl["dY"].copy_(hdY, non_blocking=True)
+                in_ready[j].record(s_in)
+            comp.wait_event(in_ready[j])
+            if i >= 2:
+                comp.wait_event(out_free[j])      # step i-2's outputs have left
+            Y, I, rs, _, _ = mosa.mosa_forward(sl["X"], D["Wr"], D["Wq"], D["Wk"], D["Wv"],
+                                               D["Wo"], cfg.k, workspace=ws, out=sl["outs"])
+            if cfg.backward:
+                mosa.mosa_backward(sl["X"], D["Wr"], D["Wq"], D["Wk"], D["Wv"], D["Wo"], I, rs,
+                                   sl["dY"], ws, out=sl["grads"])
+            in_free[j].record(comp)
+            done[j].record(comp)
+            with torch.cuda.stream(s_out):
+                s_out.wait_event(done[j])
+                hY.copy_(sl["outs"]["Y"], non_blocking=True)
+                if cfg.backward:
+                    hdX.copy_(sl["grads"]["dX"], non_blocking=True)
+                out_free[j].record(s_out)
+        comp.wait_stream(s_in)
+        comp.wait_stream(s_out)
 
-    for _ in range(3):
-        e2e_step()
+    e2e_run(4)   # captures the layer's graphs for both buffer sets
     torch.cuda.synchronize()
     barrier()
     e0 = torch.cuda.Event(enable_timing=True)
     e1 = torch.cuda.Event(enable_timing=True)
     e0.record()
-    for _ in range(e2e_steps):
-        e2e_step()
+    e2e_run(e2e_steps, start_event=e0)
     e1.record()
     torch.cuda.synchronize()
     e2e_value, e2e_ms = combine_ranks(e0.elapsed_time(e1), cfg.B * cfg.T * e2e_steps, dist, dev)
-    h2d = hX.numel() * hX.element_size() + hdY.numel() * hdY.element_size()
-    d2h = hY.numel() * 4 + hdX.numel() * 4
+    h2d = hX.numel() * hX.element_size() + (hdY.numel() * hdY.element_size() if cfg.backward else 0)
+    d2h = hY.numel() * 4 + (hdX.numel() * 4 if cfg.backward else 0)
 
     if rank != 0:
         if dist is not None:
@@ -528,7 +563,9 @@ def main():
         "stage_ms": {s: round(v, 5) for s, v in stage_ms.items()},
         "e2e": {"value": e2e_value, "unit": "tokens/s",
                 "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h,
-                "what": "pinned host X, dY -> device; forward+backward; Y, dX -> pinned host"},
+                "what": "pinned host X, dY -> device; forward+backward; Y, dX -> pinned host; "
+                        "copies on two streams beside the compute of the neighbouring steps "
+                        "(two device buffer sets)"},
         "gpu_launches": int(launches),
         "graph_ms_per_step": graph_ms,
         "clocks": clocks,

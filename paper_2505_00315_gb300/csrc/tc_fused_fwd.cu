@@ -6,8 +6,9 @@
 // sequences b0 .. b0+U-1 (their rows are adjacent in the [H, B*k] layout), all
 // on the tensor cores with fp32 accumulators in TMEM:
 //   phase 1  [Q|K|V] = X[g(m), :] [W_q|W_k|W_v][h]   K = d in 64-wide blocks, a
-//            3-stage ring: W blocks by TMA, the selected rows of X by 16-byte
-//            cp.async gathers
+//            5-stage ring (three slots of its own, two in the Q/K/V tiles, idle
+//            until phase 2): W blocks by TMA, the selected rows of X by 16-byte
+//            cp.async gathers, confirmed three blocks after issue
 //   phase 2  the accumulator is read back and split into bf16 hi/lo pairs, kept
 //            in shared memory as the attention operands; warp 3 copies them to
 //            global memory (the backward reads them) by TMA stores while the
@@ -40,7 +41,9 @@ using namespace tc;
 
 constexpr int kThreads = 384;
 constexpr int kWorkers = 256;            // warps 4-11
-constexpr int kStages = 3;
+constexpr int kStages = 5;                // ring slots in phase 1
+constexpr int kOwnStages = 3;             // slots of the ring array; the others lie in the Q/K/V tiles
+constexpr int kLag = kStages - 2;         // gather blocks in flight before one is confirmed
 constexpr int kHalf = kTileHalf;         // one hi or lo half of a 128 x 64 tile: 16 KB
 constexpr int kStageBytes = kHalf + 3 * 8192;   // gathered X block + W_q|W_k|W_v blocks
 constexpr int kChunk = 256;              // output columns per phase-4 chunk
@@ -48,7 +51,7 @@ constexpr int kChunk = 256;              // output columns per phase-4 chunk
 struct FusedSmem {
     // phase 1: the ring; phase 3: P pair tile [half][key block] in its first
     // 64 KB and epilogue staging at +64 KB; phase 4: staging at +64 KB
-    uint8_t ring[kStages][kStageBytes];
+    uint8_t ring[kOwnStages][kStageBytes];
     uint8_t q[2][kHalf];     // Q pair; phase 4: AR pair (A operand of the output product)
     uint8_t k[2][kHalf];     // K pair; phase 4: W_o chunk buffer 0
     uint8_t v[2][kHalf];     // V pair; phase 4: W_o chunk buffer 1
@@ -62,6 +65,7 @@ struct FusedSmem {
 };
 constexpr int kSmem = (int)sizeof(FusedSmem) + 1024;
 static_assert(kSmem <= 227 * 1024, "shared memory");
+static_assert((kStages - kOwnStages) * kStageBytes <= 6 * kHalf, "ring slots in the Q/K/V tiles");
 
 struct FusedParams {
     CUtensorMap mW[3];     // W_q, W_k, W_v: [H, d, 64], box {64, 64, 1}
@@ -99,6 +103,11 @@ __global__ void __launch_bounds__(kThreads, 1) fused_fwd_kernel(const __grid_con
     // P pair tile [half][key block] over the start of the ring
     uint8_t(*ptile)[2][kHalf] = reinterpret_cast<uint8_t(*)[2][kHalf]>(&sm.ring[0][0]);
     uint8_t *stage_area = &sm.ring[0][0] + 4 * kHalf;   // 32 KB of epilogue staging
+    // phase-1 ring slot s: the ring array, then the Q/K/V tiles (contiguous, idle
+    // until the Q|K|V product is done)
+    auto slot = [&](int s) -> uint8_t * {
+        return s < kOwnStages ? sm.ring[s] : &sm.q[0][0] + (s - kOwnStages) * kStageBytes;
+    };
 
     if (threadIdx.x == 0) {
         for (int s = 0; s < kStages; ++s) {
@@ -145,7 +154,7 @@ __global__ void __launch_bounds__(kThreads, 1) fused_fwd_kernel(const __grid_con
                 const uint32_t fb = smem_u32(&sm.full[s]);
                 mbar_expect_tx(fb, 3 * 8192);
                 for (int j = 0; j < 3; ++j)
-                    tma_load_3d(smem_u32(sm.ring[s] + kHalf + j * 8192), &p.mW[j], fb, 0, kb * 64, h);
+                    tma_load_3d(smem_u32(slot(s) + kHalf + j * 8192), &p.mW[j], fb, 0, kb * 64, h);
             }
             // phase 4: W_o chunks into the K / V tiles once P V is done and
             // their TMA stores have read them
@@ -173,7 +182,7 @@ __global__ void __launch_bounds__(kThreads, 1) fused_fwd_kernel(const __grid_con
                 const int s = kb % kStages;
                 if (!(ok = wait_or_abort(sm, sm.full[s], (kb / kStages) & 1, p.status))) break;
                 tc_fence_after();
-                const uint32_t a = smem_u32(sm.ring[s]), b = a + kHalf;
+                const uint32_t a = smem_u32(slot(s)), b = a + kHalf;
 #pragma unroll
                 for (int j = 0; j < 4; ++j)
                     mma_bf16(tmem, smem_desc_sw128(a + j * 32, 16, 1024),
@@ -279,7 +288,7 @@ __global__ void __launch_bounds__(kThreads, 1) fused_fwd_kernel(const __grid_con
             for (int kb = 0; kb < nkb; ++kb) {
                 const int s = kb % kStages;
                 if (!wait_or_abort(sm, sm.empty[s], ((kb / kStages) & 1) ^ 1, p.status)) break;
-                const uint32_t a = smem_u32(sm.ring[s]);
+                const uint32_t a = smem_u32(slot(s));
                 const int col = kb * 64 + chunk * 8;
 #pragma unroll
                 for (int j = 0; j < 4; ++j) {
@@ -291,10 +300,10 @@ __global__ void __launch_bounds__(kThreads, 1) fused_fwd_kernel(const __grid_con
                 }
                 cp_async_commit();
                 issued = kb + 1;
-                if (kb >= 1) {
-                    cp_async_wait<1>();
+                if (kb >= kLag) {
+                    cp_async_wait<kLag>();
                     fence_proxy_async();
-                    mbar_arrive(smem_u32(&sm.full[(kb - 1) % kStages]));
+                    mbar_arrive(smem_u32(&sm.full[(kb - kLag) % kStages]));
                     ++landed;
                 }
             }

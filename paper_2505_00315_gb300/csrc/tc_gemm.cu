@@ -17,7 +17,6 @@
 // Variants (bf16 inputs, head size 64; intermediates are bf16 hi/lo pairs, so
 // a product with one is two MMAs into the same accumulator):
 //   kQKV  F3  [Q|K|V](m,:)  = X[g(m),:] W_{q|k|v}[h]        A gathered K-major, B MN-major
-//   kOUT  F5  Y[g(m),n]    += (diag(r) A)(m,:) W_o[h](:,n)   A = AR pair,  B MN-major
 //   kG    B1  G(m,:)        = dY[g(m),:] W_o[h]^T, then D = <AR, G>, dA = r G, dlogit in the epilogue
 //   kDWO  B1  dW_o[h](p,c)  = sum_m AR(m,p) dY[g(m),c]       A gathered MN-major, B = AR pair
 //   kDW   B4  [dW_q|dW_k|dW_v|dW_r][h](c,:) = sum_m X[g(m),c] [dQ|dK|dV|dlogit](m,:)
@@ -26,8 +25,9 @@
 //             accumulator columns), so dW_r comes out of the same product;
 //             256 rows c per CTA in two accumulators that share every B tile
 //   kROUTER F1 r[b,h,t] = sigmoid(X[b,t,:] W_r[:,h])       A = X tiles, B = W_r MN-major
-// where g(m) = b*T + I[b,h,i] for row m = b*k + i of head h.  B3 (dX) has a
-// persistent kernel of its own (tc_dx.cu).
+// where g(m) = b*T + I[b,h,i] for row m = b*k + i of head h.  The products
+// that scatter-add rows into Y or dX (F5 for k > 128, B3) have a persistent
+// kernel of their own (tc_dx.cu).
 #include <algorithm>
 #include <cstdio>
 #include <mutex>
@@ -42,7 +42,8 @@ namespace {
 
 using namespace tc;
 
-enum Kind : int { kQKV = 0, kOUT, kG, kDWO, kDW, kROUTER };
+// (the values name the kernel instances tc_gemm_kernel<N> in profiles)
+enum Kind : int { kQKV = 0, kG = 2, kDWO = 3, kDW = 4, kROUTER = 5 };
 
 constexpr int kBM = 128;        // rows per tile (TMEM lanes)
 constexpr int kBK = 64;         // K per stage: one 128-byte swizzle row of bf16
@@ -58,12 +59,6 @@ struct Cfg<kQKV> {
     static constexpr int BN = 192, STAGES = 2, A_BYTES = kTile16K, B_BYTES = 3 * kTile8K,
                          TMEM_COLS = 256, MIN_CTAS = 2;
     static constexpr bool A_MN = false, B_MN = true, A_PAIR = false, B_PAIR = false;
-};
-template <>
-struct Cfg<kOUT> {
-    static constexpr int BN = 256, STAGES = 1, A_BYTES = 2 * kTile16K, B_BYTES = 4 * kTile8K,
-                         TMEM_COLS = 256, MIN_CTAS = 2;
-    static constexpr bool A_MN = false, B_MN = true, A_PAIR = true, B_PAIR = false;
 };
 template <>
 struct Cfg<kG> {
@@ -109,12 +104,6 @@ __host__ __device__ constexpr int kind_acc() {
 // [dQ | dK | dV | dlogit, 0..] hi (256) then the same lo (256).
 constexpr int kDQKVCols = 512;
 
-// Kinds that scatter-add their output rows into [B*T, d] (Y).
-template <int KIND>
-__host__ __device__ constexpr bool scatters() {
-    return KIND == kOUT;
-}
-
 // Kinds whose A operand is gathered through the selected rows.
 template <int KIND>
 __host__ __device__ constexpr bool gathers() {
@@ -124,7 +113,7 @@ __host__ __device__ constexpr bool gathers() {
 // Kinds whose epilogue runs on all eight warps (wide output tiles).
 template <int KIND>
 __host__ __device__ constexpr bool epi_all_warps() {
-    return KIND == kQKV || KIND == kOUT || KIND == kDW || KIND == kDWO || KIND == kROUTER;
+    return KIND == kQKV || KIND == kDW || KIND == kDWO || KIND == kROUTER;
 }
 
 template <int KIND>
@@ -138,7 +127,7 @@ struct TcParams {
     CUtensorMap mapB[3];   // per-head tile maps of the B operand
     int M;                 // output rows per head: B*k for row kinds, d for kDWO / kDW
     int Mtok;              // selected rows per head, B*k
-    int N;                 // output columns (d for kOUT); MMA width (kROUTER)
+    int N;                 // MMA width (kROUTER)
     int ring_stages;       // kROUTER: stages in the ring (<= kMaxStages)
     int ring_stride;       // kROUTER: bytes per stage
     int nkb;               // K blocks in the whole reduction
@@ -149,7 +138,7 @@ struct TcParams {
     const bf16 *ARp;       // [H, B*k, 128] pair of AR = diag(r) A (kG)
     const void *src_rows;  // gathered source [B*T, d] bf16: X (kQKV, kDW) or dY (kG, kDWO)
     void *out[3];          // Q/K/V pairs (kQKV); dA pair, dQKV pair (kG)
-    float *out_f;          // Y (kOUT), dW_o (kDWO), dW_q (kDW)
+    float *out_f;          // r (kROUTER), dW_o (kDWO), dW_q (kDW)
     float *out_f1;         // Dd (kG), dW_k (kDW)
     float *out_f2;         // dlogit (kG), dW_v (kDW)
     float *out_f3;         // dW_r (kDW)
@@ -367,7 +356,7 @@ __global__ void __launch_bounds__(kThreads, Cfg<KIND>::MIN_CTAS)
         fence_barrier_init();
     }
     pdl_wait();  // everything below may read what the previous kernel wrote
-    if (KIND == kQKV || KIND == kG || scatters<KIND>()) {
+    if (KIND == kQKV || KIND == kG) {
         for (int r = threadIdx.x; r < kBM; r += kThreads) {
             const int m = m0 + r;
             s_rows[r] = m < p.Mtok ? p.gidx[(size_t)h * p.Mtok + m] : 0;
@@ -411,11 +400,6 @@ __global__ void __launch_bounds__(kThreads, Cfg<KIND>::MIN_CTAS)
                 if (lane < 3) tma_load_3d(b + lane * kTile8K, &p.mapB[lane], fb, 0, kb * kBK, h);
             } else if constexpr (KIND == kG) {
                 if (lane == 0) tma_load_3d(b, &p.mapB[0], fb, kb * kBK, 0, h);
-            } else if constexpr (KIND == kOUT) {
-                if (lane == 0) tma_load_3d(a, &p.mapA, fb, 0, m0, h);
-                if (lane == 1) tma_load_3d(a + kTile16K, &p.mapA, fb, 64, m0, h);
-                if (lane >= 2 && lane < 6)
-                    tma_load_3d(b + (lane - 2) * kTile8K, &p.mapB[0], fb, n0 + 64 * (lane - 2), 0, h);
             } else if constexpr (KIND == kROUTER) {
                 if (lane == 0) tma_load_2d(a, &p.mapA, fb, kb * kBK, m0);
                 if (lane >= 1 && lane <= nbl)
@@ -512,24 +496,6 @@ __global__ void __launch_bounds__(kThreads, Cfg<KIND>::MIN_CTAS)
                 store_rows256(xb, lane, nrows, [&](int rl, int u) {
                     return reinterpret_cast<uint4 *>(dst + (size_t)rl * 128) + u;
                 });
-            }
-        } else if constexpr (KIND == kOUT) {
-            // 32 x 32 blocks transposed through shared memory so that every
-            // red.add.v4 covers four whole 128-byte row segments
-            const int chunk = lane & 7;
-            for (int c0 = part * (C::BN / 2); c0 < (part + 1) * (C::BN / 2); c0 += 32) {
-                stage_f32_32(xb, tb + c0, lane);
-                const int n = n0 + c0 + 4 * chunk;
-#pragma unroll
-                for (int i = 0; i < 8; ++i) {
-                    const int rl = (lane >> 3) + 4 * i;
-                    const int rt = q * 32 + rl;
-                    float4 val = *reinterpret_cast<const float4 *>(xb + rl * 128 + ((chunk ^ (rl & 7)) << 4));
-                    if (m0 + rt < p.M && n < p.d) {
-                        red_add_v4(p.out_f + (size_t)s_rows[rt] * p.d + n, val.x, val.y, val.z, val.w);
-                    }
-                }
-                __syncwarp();
             }
         } else if constexpr (KIND == kG) {
             // G row in two 32-column halves: D = <AR, G> = r <A, G> accumulates,
@@ -794,16 +760,7 @@ cudaError_t tc_out(const Dims &dm, const void *Wo, const Saved &sv, float *Y, cu
         cudaError_t e = cudaMemsetAsync(Y, 0, sizeof(float) * (size_t)dm.B * dm.T * dm.d, s);
         if (e != cudaSuccess) return e;
     }
-    TcParams p = base_params(dm, sv);
-    p.M = p.Mtok;
-    p.N = dm.d;
-    p.nkb = 1;
-    bool ok = map_heads(&p.mapA, sv.AR, dm.H, p.Mtok, 128, 128) &&
-              map_heads(&p.mapB[0], Wo, dm.H, 64, dm.d, 64);
-    if (!ok) return cudaErrorInvalidValue;
-    p.out_f = Y;
-    dim3 grid((p.M + kBM - 1) / kBM, (dm.d + 255) / 256, dm.H);
-    return launch_kind<kOUT>(p, grid, s);
+    return tc_out_scatter(dm, Wo, sv, Y, s);
 }
 
 cudaError_t tc_out_bwd_g(const Dims &dm, const void *Wo, const void *dY, const Saved &sv,

@@ -73,15 +73,25 @@ typedef enum {
 typedef enum { MOSA_F32 = 0, MOSA_BF16 = 1 } mosa_dtype;
 
 /* Problem size.  B sequences of T tokens of width d; H MoSA heads of size hp
- * (the paper's h'); each head keeps k of the T tokens (Sec. 2.2). */
+ * (the paper's h'); each head keeps k of the T tokens (Sec. 2.2).
+ * first_token = 1 makes every head keep token 0 of each sequence and select
+ * the other k-1 tokens by router score among tokens 1..T-1 (the IsoFLOP
+ * models of Sec. 3.2); token 0 is scaled by its own router score like the
+ * others.  first_token = 0 is the plain TopK; other values are invalid. */
 typedef struct {
     int32_t B, T, d, H, hp, k;
-    int32_t dtype; /* mosa_dtype of X, dY and all weights */
+    int32_t dtype;       /* mosa_dtype of X, dY and all weights */
+    int32_t first_token; /* 0 or 1, see above */
 } mosa_shape;
 
 /* Supported sizes (else MOSA_ERR_UNSUPPORTED):
  *   1 <= k <= T <= 65536; B, H >= 1; B*T*d < 2^31; H*d*hp < 2^31;
  *   d % 8 == 0 and hp in {16, 32, 64, 128}. */
+
+/* Tokens per head for a sequence of T tokens at sparsity rho (Sec. 3.5, for
+ * inputs shorter than the training length): k = max(floor(T / rho), 2),
+ * and at most T.  Returns 0 if T < 1 or rho < 1. */
+int32_t mosa_adaptive_k(int32_t T, int32_t rho);
 
 /* Human-readable name of a status code (static string, never NULL). */
 const char *mosa_status_string(mosa_status s);

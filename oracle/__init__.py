@@ -58,7 +58,9 @@ def _load():
             lib.oracle_router.argtypes = [c_int, c_int, c_int, c_int, d, d, d]
             lib.oracle_topk.argtypes = [c_int, c_int, d, i32, d]
             lib.oracle_topk.restype = c_int
-            lib.oracle_forward.argtypes = [c_int] * 6 + [d] * 6 + [d, i32, d, d, u8, u8]
+            lib.oracle_topk_first.argtypes = [c_int, c_int, d, i32, d]
+            lib.oracle_topk_first.restype = c_int
+            lib.oracle_forward.argtypes = [c_int] * 6 + [d] * 6 + [d, i32, d, d, u8, u8, c_int]
             lib.oracle_forward.restype = c_int
             lib.oracle_forward_indices.argtypes = [c_int] * 6 + [d] * 6 + [i32, d, d, u8, u8]
             lib.oracle_forward_indices.restype = c_int
@@ -113,23 +115,27 @@ def router(X, Wr) -> np.ndarray:
     return out
 
 
-def topk(r_row, k: int):
+def topk(r_row, k: int, first_token: bool = False):
     """TopK over one row of scores (Sec. 2.2): full sort by (-score, index),
-    first k kept, returned in ascending index order with their scores."""
+    first k kept, returned in ascending index order with their scores.  With
+    ``first_token`` (Sec. 3.2) token 0 is always kept and the other k-1 are the
+    TopK of tokens 1..T-1."""
     r_row = _f64(r_row).reshape(-1)
     T = r_row.shape[0]
     I = np.empty(k, dtype=np.int32)
     rs = np.empty(k, dtype=np.float64)
-    if _load().oracle_topk(T, k, _ptr(r_row), _ptr(I, ctypes.c_int32), _ptr(rs)) != 0:
+    fn = _load().oracle_topk_first if first_token else _load().oracle_topk
+    if fn(T, k, _ptr(r_row), _ptr(I, ctypes.c_int32), _ptr(rs)) != 0:
         raise ValueError("oracle_topk: invalid arguments")
     return I, rs
 
 
-def forward(X, Wr, Wq, Wk, Wv, Wo, k: int, batches=None, heads=None):
+def forward(X, Wr, Wq, Wk, Wv, Wo, k: int, batches=None, heads=None, first_token=False):
     """MoSA layer forward (Sec. 2.2, Eq. mosa_mha).  Returns (Y, I, r_sel, r_full).
 
     ``batches`` / ``heads`` restrict the computed units (b,h); Y[b] is exact
-    for a batch whose every head is computed."""
+    for a batch whose every head is computed.  ``first_token``: every head
+    keeps token 0 and selects k-1 more (Sec. 3.2)."""
     X, Wr, Wq, Wk, Wv, Wo = map(_f64, (X, Wr, Wq, Wk, Wv, Wo))
     B, T, d, H, hp = _dims(X, Wq)
     Y = np.zeros((B, T, d))
@@ -139,7 +145,8 @@ def forward(X, Wr, Wq, Wk, Wv, Wo, k: int, batches=None, heads=None):
     bm, hm = _mask(batches, B), _mask(heads, H)
     rc = _load().oracle_forward(B, T, d, H, hp, k, _ptr(X), _ptr(Wr), _ptr(Wq), _ptr(Wk),
                                 _ptr(Wv), _ptr(Wo), _ptr(Y), _ptr(I, ctypes.c_int32), _ptr(rs),
-                                _ptr(rf), _ptr(bm, ctypes.c_ubyte), _ptr(hm, ctypes.c_ubyte))
+                                _ptr(rf), _ptr(bm, ctypes.c_ubyte), _ptr(hm, ctypes.c_ubyte),
+                                1 if first_token else 0)
     if rc != 0:
         raise ValueError("oracle_forward failed (bad arguments or out of memory)")
     return Y, I, rs, rf

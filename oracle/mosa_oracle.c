@@ -18,11 +18,12 @@
  *                              A = Attention(Q,K,V,M);  X^o = diag(r^topk) A W^o;
  *                              Y_j = X^o_i if j = I_i, else 0.
  *   Sec. 2.2, Eq. (mosa_mha):  MoSA(X) = sum_i MoSA_head(X; theta_i)
+ *   Sec. 3.2 (IsoFLOP models): the first token is always in every head's set
  *   Sec. 2.2 (last paragraph of the output definition): the router receives
  *                              its gradient only through the diag(r) scaling;
  *                              TopK itself is not differentiated.
  *
- * Readings of points the paper leaves open (each also listed in the design doc):
+ * Readings of points the paper leaves open:
  *   - TopK ranks the sigmoid scores r; ties go to the lower token index.
  *   - I is returned in ascending token order (the mask uses the indices
  *     themselves, so the layer output does not depend on the order).
@@ -30,6 +31,9 @@
  *   - The mask is applied inside the 1/sqrt(h') scaling; -inf stays -inf.
  *     The diagonal I_i >= I_i is always allowed, so no row is empty.
  *   - No router noise, no biases, no dropout.
+ *   - Sec. 3.2 (IsoFLOP models) keeps the first token in every head and
+ *     selects the other k-1 by router score: read as token 0 plus TopK(k-1)
+ *     over tokens 1..T-1 (same tie rule), token 0 scaled by its own score.
  *
  * Layouts (row-major, all fp64 here):
  *   X [B,T,d]; W_r [d,H]; W_q, W_k, W_v [H,d,h']; W_o [H,h',d];
@@ -115,6 +119,22 @@ int oracle_topk(int T, int k, const double *r, int32_t *I, double *r_sel) {
     for (int i = 0; i < k; ++i) { I[i] = chosen[i]; r_sel[i] = r[chosen[i]]; }
     free(all);
     free(chosen);
+    return 0;
+}
+
+/* Sec. 3.2 (IsoFLOP models): every head always includes the first token; it
+ * selects the other k-1 tokens by router score.  Token 0 plus the k-1 largest
+ * of r[1..T-1] by a full sort of those T-1 scores (ties: lower index), I in
+ * ascending order, r_sel[i] = r[I[i]] (token 0 keeps its own score).
+ * Returns 0, or -1 on bad arguments. */
+int oracle_topk_first(int T, int k, const double *r, int32_t *I, double *r_sel) {
+    if (T <= 0 || k <= 0 || k > T) return -1;
+    I[0] = 0;
+    r_sel[0] = r[0];
+    if (k == 1) return 0;
+    /* the rest: TopK(k-1) over tokens 1..T-1, shifted back to token indices */
+    if (oracle_topk(T - 1, k - 1, r + 1, I + 1, r_sel + 1) != 0) return -1;
+    for (int i = 1; i < k; ++i) I[i] += 1;
     return 0;
 }
 
@@ -271,7 +291,7 @@ int oracle_forward_indices(int B, int T, int d, int H, int hp, int k, const doub
 int oracle_forward(int B, int T, int d, int H, int hp, int k, const double *X,
                    const double *Wr, const double *Wq, const double *Wk, const double *Wv,
                    const double *Wo, double *Y, int32_t *I, double *r_sel, double *r_full,
-                   const unsigned char *bsel, const unsigned char *hsel) {
+                   const unsigned char *bsel, const unsigned char *hsel, int first_token) {
     if (B <= 0 || T <= 0 || d <= 0 || H <= 0 || hp <= 0 || k <= 0 || k > T) return -1;
     int failed = 0;
     #pragma omp parallel for collapse(2) schedule(dynamic, 1) reduction(| : failed)
@@ -287,7 +307,9 @@ int oracle_forward(int B, int T, int d, int H, int hp, int k, const double *X,
             }
             if (r_full)
                 for (int t = 0; t < T; ++t) r_full[IDX3(b, h, t, H, T)] = r[t];
-            if (oracle_topk(T, k, r, I + IDX3(b, h, 0, H, k), r_sel + IDX3(b, h, 0, H, k)) != 0)
+            int32_t *Ib = I + IDX3(b, h, 0, H, k);
+            double *rb = r_sel + IDX3(b, h, 0, H, k);
+            if ((first_token ? oracle_topk_first(T, k, r, Ib, rb) : oracle_topk(T, k, r, Ib, rb)) != 0)
                 failed |= 1;
             free(r);
         }

@@ -26,18 +26,19 @@ MOSA_BF16 = 1
 EXPORTED = ("mosa_status_string", "mosa_workspace_bytes", "mosa_forward",
             "mosa_forward_with_indices", "mosa_backward", "mosa_topk", "mosa_check_status",
             "mosa_kernel_launches", "mosa_profile_stages", "mosa_profile_read",
-            "mosa_stage_name", "mosa_stage_engine", "mosa_route_noalloc")
+            "mosa_stage_name", "mosa_stage_engine", "mosa_route_noalloc", "mosa_adaptive_k")
 
 
 class MosaShape(ctypes.Structure):
     """mosa_shape: B sequences of T tokens of width d, H heads of size hp, k
-    tokens per head, storage dtype (MOSA_F32 or MOSA_BF16)."""
+    tokens per head, storage dtype (MOSA_F32 or MOSA_BF16), first_token (1:
+    every head keeps token 0 and selects k-1 more, Sec. 3.2)."""
     _fields_ = [("B", ctypes.c_int32), ("T", ctypes.c_int32), ("d", ctypes.c_int32),
                 ("H", ctypes.c_int32), ("hp", ctypes.c_int32), ("k", ctypes.c_int32),
-                ("dtype", ctypes.c_int32)]
+                ("dtype", ctypes.c_int32), ("first_token", ctypes.c_int32)]
 
     def astuple(self):
-        return (self.B, self.T, self.d, self.H, self.hp, self.k, self.dtype)
+        return (self.B, self.T, self.d, self.H, self.hp, self.k, self.dtype, self.first_token)
 
 
 class MosaError(RuntimeError):
@@ -93,6 +94,8 @@ def load(build_if_missing: bool = True) -> ctypes.CDLL:
         L.mosa_route_noalloc.restype = ctypes.c_int
         L.mosa_stage_engine.argtypes = [sp, i32]
         L.mosa_stage_engine.restype = i32
+        L.mosa_adaptive_k.argtypes = [i32, i32]
+        L.mosa_adaptive_k.restype = i32
         _lib = L
         return L
 
@@ -141,12 +144,18 @@ def _stream(stream):
     return ctypes.c_void_p(s.cuda_stream)
 
 
-def make_shape(X, W_q, k: int) -> MosaShape:
+def make_shape(X, W_q, k: int, first_token: bool = False) -> MosaShape:
     B, T, d = X.shape
     H, d2, hp = W_q.shape
     if d2 != d:
         raise ValueError("W_q must be [H, d, hp] with the d of X")
-    return MosaShape(B, T, d, H, hp, int(k), _dtype_code(X))
+    return MosaShape(B, T, d, H, hp, int(k), _dtype_code(X), 1 if first_token else 0)
+
+
+def mosa_adaptive_k(T: int, rho: int) -> int:
+    """Tokens per head for a T-token input at sparsity rho (Sec. 3.5):
+    max(floor(T / rho), 2), at most T; 0 for T < 1 or rho < 1."""
+    return int(load().mosa_adaptive_k(int(T), int(rho)))
 
 
 def mosa_workspace_bytes(shape: MosaShape) -> int:
@@ -169,12 +178,14 @@ def _same(ref, *ts):
 
 
 def mosa_forward(X, W_r, W_q, W_k, W_v, W_o, k: int, workspace=None, want_r_full=False,
-                 out=None, stream=None):
+                 out=None, stream=None, first_token: bool = False):
     """Forward pass (Sec. 2.2).  Returns (Y, I, r_sel, r_full or None, workspace).
 
-    ``out`` may hold preallocated "Y", "I", "r_sel" (and "r_full") tensors."""
+    ``out`` may hold preallocated "Y", "I", "r_sel" (and "r_full") tensors.
+    With ``first_token`` every head keeps token 0 and selects k-1 more
+    (Sec. 3.2)."""
     torch = _torch()
-    shape = make_shape(X, W_q, k)
+    shape = make_shape(X, W_q, k, first_token)
     _same(X, ("W_r", W_r), ("W_q", W_q), ("W_k", W_k), ("W_v", W_v), ("W_o", W_o))
     B, T, d, H = shape.B, shape.T, shape.d, shape.H
     dev = X.device
@@ -312,14 +323,15 @@ def stage_impl(shape: MosaShape) -> dict:
     return out
 
 
-def mosa_route_noalloc(X, W_r, k: int, hp: int = 64, out=None, stream=None):
+def mosa_route_noalloc(X, W_r, k: int, hp: int = 64, out=None, stream=None,
+                       first_token: bool = False):
     """Router + TopK with no workspace (the library's own 4 MiB score array);
     returns (I, r_sel).  For callers that cannot allocate device memory; the
     output tensors may be passed preallocated in ``out``."""
     torch = _torch()
     B, T, d = X.shape
     H = W_r.shape[1]
-    shape = MosaShape(B, T, d, H, int(hp), int(k), _dtype_code(X))
+    shape = MosaShape(B, T, d, H, int(hp), int(k), _dtype_code(X), 1 if first_token else 0)
     _same(X, ("W_r", W_r))
     I = (out or {}).get("I")
     rs = (out or {}).get("r_sel")

@@ -98,6 +98,7 @@ struct Saved {
 struct Dims {
     int B, T, d, H, hp, k;
     bool bf16;
+    bool first_token;   // token 0 always kept, k-1 more by score (Sec. 3.2)
     long long rows() const { return (long long)H * B * k; }
     size_t esize() const { return bf16 ? 2 : 4; }
 };

@@ -49,8 +49,11 @@ cudaError_t launch_router_auto(const Dims &dm, const void *X, const void *Wr, fl
 // F2, Sec. 2.2 TopK: per row of T scores, the k largest (ties: lower index),
 // ascending.  If gidx != nullptr, row = b*H + h also writes the head-major
 // gather rows gidx[(h*B+b)*k + i] = b*T + I and rsel_hm likewise.
+// With first_token, token 0 of every row is kept and the other k-1 are the
+// largest of tokens 1..T-1 (Sec. 3.2).
 cudaError_t launch_select(int rows, int T, int k, const float *scores, int32_t *I, float *rsel,
-                          int B, int H, int32_t *gidx, float *rsel_hm, cudaStream_t stream);
+                          int B, int H, int32_t *gidx, float *rsel_hm, cudaStream_t stream,
+                          bool first_token = false);
 
 // Caller-supplied I / r_sel -> head-major gather rows, validating each row
 // (in range, strictly ascending); invalid rows become 0..k-1 and set

@@ -24,6 +24,7 @@ mosa_status check_shape(const mosa_shape *s, Dims *out) {
         return MOSA_ERR_INVALID_ARG;
     if (s->k > s->T) return MOSA_ERR_INVALID_ARG;
     if (s->dtype != MOSA_F32 && s->dtype != MOSA_BF16) return MOSA_ERR_INVALID_ARG;
+    if (s->first_token != 0 && s->first_token != 1) return MOSA_ERR_INVALID_ARG;
     const long long lim = 1LL << 31;
     if ((long long)s->B * s->T * s->d >= lim) return MOSA_ERR_UNSUPPORTED;
     if ((long long)s->H * s->d * s->hp >= lim) return MOSA_ERR_UNSUPPORTED;
@@ -33,7 +34,8 @@ mosa_status check_shape(const mosa_shape *s, Dims *out) {
     if (s->H > 65535) return MOSA_ERR_UNSUPPORTED;
     if (s->d % 8 != 0) return MOSA_ERR_UNSUPPORTED;
     if (s->hp != 16 && s->hp != 32 && s->hp != 64 && s->hp != 128) return MOSA_ERR_UNSUPPORTED;
-    if (out) *out = Dims{s->B, s->T, s->d, s->H, s->hp, s->k, s->dtype == MOSA_BF16};
+    if (out)
+        *out = Dims{s->B, s->T, s->d, s->H, s->hp, s->k, s->dtype == MOSA_BF16, s->first_token != 0};
     return MOSA_OK;
 }
 
@@ -158,7 +160,7 @@ mosa_status forward_tc(const Dims &dm, const void *X, const void *W_r, const voi
     if (route) {
         StageScope st_(kStageSelect, s);
         MOSA_TRY(launch_select(dm.B * dm.H, dm.T, dm.k, rf, I, r_sel, dm.B, dm.H, sv.gidx,
-                               sv.rsel, s));
+                               sv.rsel, s, dm.first_token));
     } else {
         StageScope st_(kStageSelect, s);
         MOSA_TRY(launch_indices_to_rows(dm, I_in, rsel_in, sv.gidx, sv.rsel, sv.status, s));
@@ -357,6 +359,12 @@ using namespace mosa;
 
 extern "C" {
 
+int32_t mosa_adaptive_k(int32_t T, int32_t rho) {
+    if (T < 1 || rho < 1) return 0;
+    const int32_t k = T / rho < 2 ? 2 : T / rho;   // Sec. 3.5: max(floor(T / rho), 2)
+    return k < T ? k : T;
+}
+
 const char *mosa_status_string(mosa_status s) {
     switch (s) {
         case MOSA_OK: return "MOSA_OK";
@@ -400,7 +408,7 @@ mosa_status mosa_forward(const mosa_shape *shape, const void *X, const void *W_r
         {
             StageScope st_(kStageSelect, s);
             MOSA_TRY(launch_select(dm.B * dm.H, dm.T, dm.k, rf, I, r_sel, dm.B, dm.H, sv.gidx,
-                                   sv.rsel, s));
+                                   sv.rsel, s, dm.first_token));
         }
         return forward_heads(dm, X, W_q, W_k, W_v, W_o, Y, sv, s);
     };

@@ -56,7 +56,8 @@ extern "C" mosa_status mosa_route_noalloc(const mosa_shape *shape, const void *X
         // invalid or unsupported shape: report which
         if (shape == nullptr || shape->B <= 0 || shape->T <= 0 || shape->d <= 0 ||
             shape->H <= 0 || shape->hp <= 0 || shape->k <= 0 || shape->k > shape->T ||
-            (shape->dtype != MOSA_F32 && shape->dtype != MOSA_BF16))
+            (shape->dtype != MOSA_F32 && shape->dtype != MOSA_BF16) ||
+            (shape->first_token != 0 && shape->first_token != 1))
             return MOSA_ERR_INVALID_ARG;
         return MOSA_ERR_UNSUPPORTED;
     }
@@ -66,12 +67,13 @@ extern "C" mosa_status mosa_route_noalloc(const mosa_shape *shape, const void *X
     float *scores = nullptr;
     if (scores_address(&scores) != cudaSuccess) return MOSA_ERR_CUDA;
     const Dims dm{shape->B, shape->T, shape->d, shape->H, shape->hp, shape->k,
-                  shape->dtype == MOSA_BF16};
+                  shape->dtype == MOSA_BF16, shape->first_token != 0};
     cudaStream_t s = static_cast<cudaStream_t>(stream);
     // Every score the selection reads is written by the router first, so the
     // array needs no clearing between calls.
     if (launch_router(dm, X, W_r, scores, s) != cudaSuccess) return MOSA_ERR_CUDA;
-    if (launch_select(dm.B * dm.H, dm.T, dm.k, scores, I, r_sel, 0, 1, nullptr, nullptr, s) !=
+    if (launch_select(dm.B * dm.H, dm.T, dm.k, scores, I, r_sel, 0, 1, nullptr, nullptr, s,
+                      dm.first_token) !=
         cudaSuccess)
         return MOSA_ERR_CUDA;
     return MOSA_OK;

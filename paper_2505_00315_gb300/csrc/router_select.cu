@@ -3,7 +3,9 @@
 //
 // The selection is a per-row radix select on an order-preserving uint32
 // image of the fp32 scores (4 passes of 8 bits, most significant first),
-// which finds the exact k-th largest key.  A final in-order compaction keeps
+// which finds the exact k-th largest key.  With first_token, token 0 gets a
+// key above every score's (0xFFFFFFFF; a finite or infinite score maps at most
+// to 0xFF800000), so it is always kept and the other k-1 come from the rest.  A final in-order compaction keeps
 // every key above it plus the lowest-index keys equal to it, so I comes out
 // ascending (the order the causal mask works in) and ties go to the lower
 // token index.  Output positions come from one block-wide prefix sum of the
@@ -84,7 +86,7 @@ __device__ __forceinline__ unsigned long long block_excl_scan(unsigned long long
 __global__ void __launch_bounds__(kSelThreads)
 topk_select_kernel(const float *__restrict__ scores, int T, int k, int32_t *__restrict__ I,
                    float *__restrict__ rsel, int B, int H, int32_t *__restrict__ gidx,
-                   float *__restrict__ rsel_hm) {
+                   float *__restrict__ rsel_hm, int first_token) {
     extern __shared__ uint32_t keys_s[];   // the row's order keys when T <= kSelStagedMax
     __shared__ uint32_t hist[2][256];
     __shared__ unsigned long long sh[33];
@@ -97,10 +99,14 @@ topk_select_kernel(const float *__restrict__ scores, int T, int k, int32_t *__re
     const int tid = threadIdx.x;
     const bool staged = T <= kSelStagedMax;
     for (int i = tid; i < 256; i += blockDim.x) hist[0][i] = 0u;
+    // token 0's key under first_token: above every score's
+    auto key_of = [&](int t) -> uint32_t {
+        return (first_token && t == 0) ? 0xFFFFFFFFu : order_key(__ldg(s + t));
+    };
     if (staged)
-        for (int t = tid; t < T; t += blockDim.x) keys_s[t] = order_key(__ldg(s + t));
+        for (int t = tid; t < T; t += blockDim.x) keys_s[t] = key_of(t);
     __syncthreads();
-    auto key_at = [&](int t) -> uint32_t { return staged ? keys_s[t] : order_key(__ldg(s + t)); };
+    auto key_at = [&](int t) -> uint32_t { return staged ? keys_s[t] : key_of(t); };
 
     uint32_t prefix = 0u, mask = 0u, remaining = (uint32_t)k;
     for (int pass = 0; pass < 4; ++pass) {
@@ -231,7 +237,8 @@ cudaError_t launch_router_auto(const Dims &dm, const void *X, const void *Wr, fl
 }
 
 cudaError_t launch_select(int rows, int T, int k, const float *scores, int32_t *I, float *rsel,
-                          int B, int H, int32_t *gidx, float *rsel_hm, cudaStream_t stream) {
+                          int B, int H, int32_t *gidx, float *rsel_hm, cudaStream_t stream,
+                          bool first_token) {
     if (rows <= 0) return cudaSuccess;
     static std::once_flag once;
     static cudaError_t attr = cudaSuccess;
@@ -247,7 +254,7 @@ cudaError_t launch_select(int rows, int T, int k, const float *scores, int32_t *
     int threads = T / 4 < 256 ? 256 : (T / 4 > 1024 ? 1024 : (T / 4 + 31) / 32 * 32);
     if (rows >= 512 && threads > 512) threads = 512;
     cudaError_t e = launch_pdl(topk_select_kernel, dim3(rows), dim3(threads), smem, stream,
-                               scores, T, k, I, rsel, B, H, gidx, rsel_hm);
+                               scores, T, k, I, rsel, B, H, gidx, rsel_hm, first_token ? 1 : 0);
     note_launches(1);
     return e;
 }

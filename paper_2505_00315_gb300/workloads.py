@@ -46,6 +46,7 @@ class MosaConfig:
     dtype: str = "bf16"          # "f32" or "bf16" storage; accumulation is fp32
     backward: bool = True
     seed: int = 0
+    first_token: bool = False    # every head keeps token 0 and selects k-1 more
     note: str = field(default="", compare=False)
 
     @property
@@ -117,16 +118,19 @@ def make_inputs(cfg: MosaConfig, seed: int | None = None, plant: bool = True,
     dY = to_storage(rng.standard_normal((B, T, d), dtype=np.float32), cfg.dtype)
     X0 = to_storage(X0, cfg.dtype)
     if plant:
-        X = plant_margin(X0, Wr, k, delta)
+        X = plant_margin(X0, Wr, k, delta, cfg.first_token)
     else:
         X = X0
     X = to_storage(X, cfg.dtype)
     return {"X": X, "Wr": Wr, "Wq": Wq, "Wk": Wk, "Wv": Wv, "Wo": Wo, "dY": dY}
 
 
-def plant_margin(X0: np.ndarray, Wr: np.ndarray, k: int, delta: float) -> np.ndarray:
+def plant_margin(X0: np.ndarray, Wr: np.ndarray, k: int, delta: float,
+                 first_token: bool = False) -> np.ndarray:
     """Return X0 + G pinv(W_r) where G raises the k highest logits of every
-    (b, head) column of X0 W_r by ``delta`` (float64 arithmetic, float32 result)."""
+    (b, head) column of X0 W_r by ``delta`` (float64 arithmetic, float32 result).
+    With ``first_token`` the raised set is token 0 and the k-1 highest of the
+    other tokens (the set the selection then keeps)."""
     B, T, d = X0.shape
     H = Wr.shape[1]
     Wr64 = Wr.astype(np.float64)
@@ -134,10 +138,15 @@ def plant_margin(X0: np.ndarray, Wr: np.ndarray, k: int, delta: float) -> np.nda
     Xout = np.empty_like(X0)
     for b in range(B):
         L0 = X0[b].astype(np.float64) @ Wr64          # [T, H]
-        order = np.argsort(-L0, axis=0, kind="stable")  # per column, highest first
         G = np.zeros((T, H))
         cols = np.arange(H)[None, :]
-        G[order[:k, :], cols] = delta
+        if first_token:
+            order = np.argsort(-L0[1:], axis=0, kind="stable") + 1   # tokens 1..T-1
+            G[0, :] = delta
+            G[order[:k - 1, :], cols] = delta
+        else:
+            order = np.argsort(-L0, axis=0, kind="stable")  # per column, highest first
+            G[order[:k, :], cols] = delta
         Xout[b] = (X0[b].astype(np.float64) + G @ pinv).astype(np.float32)
     return Xout
 

@@ -24,7 +24,8 @@ def run_layer(cfg, x, backward=True):
     """Forward (and backward) on the GPU; returns numpy outputs."""
     dt = cfg.dtype
     X, Wr, Wq, Wk, Wv, Wo = (to_dev(x[n], dt) for n in ("X", "Wr", "Wq", "Wk", "Wv", "Wo"))
-    Y, I, rs, rf, ws = mosa.mosa_forward(X, Wr, Wq, Wk, Wv, Wo, cfg.k, want_r_full=True)
+    Y, I, rs, rf, ws = mosa.mosa_forward(X, Wr, Wq, Wk, Wv, Wo, cfg.k, want_r_full=True,
+                                         first_token=cfg.first_token)
     out = {"Y": Y, "I": I, "r_sel": rs, "r_full": rf}
     if backward:
         dY = to_dev(x["dY"], dt)

@@ -37,15 +37,17 @@ def test_status_strings():
 
 
 def shape(**kw):
-    base = dict(B=2, T=64, d=32, H=3, hp=32, k=8, dtype=B.MOSA_BF16)
+    base = dict(B=2, T=64, d=32, H=3, hp=32, k=8, dtype=B.MOSA_BF16, first_token=0)
     base.update(kw)
-    return B.MosaShape(*[base[n] for n in ("B", "T", "d", "H", "hp", "k", "dtype")])
+    return B.MosaShape(*[base[n] for n in ("B", "T", "d", "H", "hp", "k", "dtype", "first_token")])
 
 
 @pytest.mark.parametrize("kw,ok", [
     ({}, True), (dict(k=64), True), (dict(k=65), False), (dict(k=0), False),
     (dict(B=0), False), (dict(T=-1), False), (dict(hp=48), False), (dict(d=12), False),
     (dict(dtype=7), False), (dict(T=70000, k=8), False), (dict(hp=128, dtype=B.MOSA_F32), True),
+    (dict(first_token=1), True), (dict(first_token=1, k=1), True), (dict(first_token=2), False),
+    (dict(first_token=-1), False),
 ])
 def test_workspace_bytes_validates_shape(kw, ok):
     n = B.mosa_workspace_bytes(shape(**kw))
@@ -109,3 +111,14 @@ def test_check_status_rejects_bad_arguments():
     L = B.load()
     assert L.mosa_check_status(ctypes.byref(shape(k=0)), FAKE, None) == B.MOSA_ERR_INVALID_ARG
     assert L.mosa_check_status(ctypes.byref(shape()), None, None) == B.MOSA_ERR_WORKSPACE
+
+
+@pytest.mark.parametrize("T,rho,k", [
+    # Sec. 3.5: k = max(floor(T / rho), 2); a 10-token input at rho = 64 keeps 2
+    (10, 64, 2), (1024, 8, 128), (1024, 64, 16), (130, 64, 2), (191, 64, 2), (192, 64, 3),
+    (8192, 32, 256),
+    # at most T tokens exist; no k for an empty input or rho < 1
+    (1, 64, 1), (2, 64, 2), (0, 8, 0), (100, 0, 0),
+])
+def test_adaptive_k(T, rho, k):
+    assert B.mosa_adaptive_k(T, rho) == k

@@ -118,6 +118,54 @@ def test_small_forward_backward_full_parity(cfg, kernel_path):
         assert_close(name, g[gname], ref[name], cfg.dtype)
 
 
+# ------------------------------------ first token always kept (Sec. 3.2) ----
+
+FIRST = [
+    W.MosaConfig("first_bf16", B=3, T=200, d=64, H=2, hp=64, k=64, dtype="bf16", seed=31,
+                 first_token=True),
+    W.MosaConfig("first_pack_bf16", B=5, T=90, d=32, H=3, hp=64, k=30, dtype="bf16", seed=32,
+                 first_token=True),
+    W.MosaConfig("first_k1_bf16", B=2, T=50, d=32, H=3, hp=64, k=1, dtype="bf16", seed=33,
+                 first_token=True),
+    W.MosaConfig("first_f32", B=2, T=129, d=24, H=3, hp=32, k=40, dtype="f32", seed=34,
+                 first_token=True),
+    W.MosaConfig("first_largek_bf16", B=1, T=400, d=64, H=2, hp=64, k=200, dtype="bf16",
+                 seed=35, first_token=True),
+]
+
+
+@pytest.mark.parametrize("cfg", FIRST, ids=lambda c: c.name)
+def test_first_token_forward_backward_parity(cfg, kernel_path):
+    x = W.make_inputs(cfg)
+    Y, I, rs, rf = oracle.forward(x["X"], *weights(x), k=cfg.k, first_token=True)
+    if cfg.k > 1:
+        assert sigmoid_gap(rf[..., 1:], cfg.k - 1) > 1e-3
+    g = run_layer(cfg, x, backward=True)
+    assert (g["I"][:, :, 0] == 0).all()
+    np.testing.assert_array_equal(g["I"], I)
+    assert_close("r_sel", g["r_sel"], rs, cfg.dtype)
+    assert_close("Y", g["Y"], Y, cfg.dtype)
+    ref = oracle.backward(x["X"], *weights(x), I=I, dY=x["dY"])
+    for name in ("dX", "dWr", "dWq", "dWk", "dWv", "dWo"):
+        gname = name[:2] + "_" + name[2:].lower() if name != "dX" else "dX"
+        assert_close(name, g[gname], ref[name], cfg.dtype)
+
+
+def test_first_token_long_rows_unstaged_select():
+    # rows longer than the TopK kernel stages in shared memory (16384 scores)
+    cfg = W.MosaConfig("first_long", B=1, T=20000, d=64, H=2, hp=64, k=300, dtype="bf16",
+                       seed=36, first_token=True)
+    x = W.make_inputs(cfg)
+    X, Wr = to_dev(x["X"], "bf16"), to_dev(x["Wr"], "bf16")
+    I, rs = mosa.mosa_route_noalloc(X, Wr, cfg.k, first_token=True)
+    rf = oracle.router(x["X"], x["Wr"])
+    assert sigmoid_gap(rf[..., 1:], cfg.k - 1) > 1e-3
+    I = I.cpu().numpy()
+    for h in range(cfg.H):
+        Iref, _ = oracle.topk(rf[0, h], cfg.k, first_token=True)
+        np.testing.assert_array_equal(I[0, h], Iref)
+
+
 # ------------------------------------------------ full workload sizes ----
 
 FULL = [c for c in W.CONFIGS.values() if c.dtype == "bf16"]

@@ -84,6 +84,58 @@ def test_topk_k_equals_T_and_bad_k():
         oracle.topk(row, 0)
 
 
+# Sec. 3.2: every head keeps the first token and selects k-1 more by score.
+
+@pytest.mark.parametrize("seed", range(16))
+def test_topk_first_token_matches_definition(seed):
+    rng = np.random.default_rng(100 + seed)
+    T = int(rng.integers(1, 60))
+    k = int(rng.integers(1, T + 1))
+    row = rng.choice([0.1, 0.25, 0.5, 0.75], size=T) if seed % 2 else rng.random(T)
+    I, rs = oracle.topk(row, k, first_token=True)
+    rest = sorted(range(1, T), key=lambda t: (-row[t], t))[:k - 1]
+    assert list(I) == [0] + sorted(rest)
+    np.testing.assert_array_equal(rs, row[I])
+
+
+def test_topk_first_token_special_cases():
+    row = np.array([0.1, 0.9, 0.5, 0.9, 0.2, 0.9])
+    assert list(oracle.topk(row, 1, first_token=True)[0]) == [0]
+    assert list(oracle.topk(row, 6, first_token=True)[0]) == list(range(6))
+    # token 0 would lose the plain TopK: it is kept anyway, ties below go to lower indices
+    assert list(oracle.topk(row, 3, first_token=True)[0]) == [0, 1, 3]
+    assert list(oracle.topk(row, 3)[0]) == [1, 3, 5]
+    # token 0 already the largest: both rules agree
+    top = np.array([0.95, 0.2, 0.7, 0.1, 0.6])
+    for k in range(1, 6):
+        assert list(oracle.topk(top, k, first_token=True)[0]) == list(oracle.topk(top, k)[0])
+
+
+def test_forward_first_token_is_forward_on_its_token_sets():
+    cfg = W.MosaConfig("first", B=2, T=40, d=16, H=3, hp=8, k=6, dtype="f32", seed=7,
+                       first_token=True)
+    x = W.make_inputs(cfg)
+    w = [x[n] for n in ("Wr", "Wq", "Wk", "Wv", "Wo")]
+    Y, I, rs, rf = oracle.forward(x["X"], *w, k=cfg.k, first_token=True)
+    assert (I[:, :, 0] == 0).all()
+    for b in range(cfg.B):
+        for h in range(cfg.H):
+            Iref, rsref = oracle.topk(rf[b, h], cfg.k, first_token=True)
+            np.testing.assert_array_equal(I[b, h], Iref)
+            np.testing.assert_array_equal(rs[b, h], rsref)
+    Y2 = oracle.forward_indices(x["X"], *w, I=I)
+    np.testing.assert_allclose(Y, Y2, rtol=0, atol=1e-12)
+
+
+def test_planted_margin_with_first_token():
+    cfg = W.MosaConfig("first", B=2, T=300, d=64, H=4, hp=16, k=37, dtype="bf16", seed=9,
+                       first_token=True)
+    x = W.make_inputs(cfg)
+    rf = oracle.router(x["X"], x["Wr"])
+    s = -np.sort(-rf[..., 1:], axis=-1)
+    assert float(np.min(s[..., cfg.k - 2] - s[..., cfg.k - 1])) > 1e-3
+
+
 # ----------------------------------------------------- forward reductions ----
 
 def dense_causal_mha_scaled(X, Wr, Wq, Wk, Wv, Wo):

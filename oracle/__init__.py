@@ -60,12 +60,13 @@ def _load():
             lib.oracle_topk.restype = c_int
             lib.oracle_topk_first.argtypes = [c_int, c_int, d, i32, d]
             lib.oracle_topk_first.restype = c_int
-            lib.oracle_forward.argtypes = [c_int] * 6 + [d] * 6 + [d, i32, d, d, u8, u8, c_int]
+            lib.oracle_forward.argtypes = [c_int] * 6 + [d] * 6 + [d, i32, d, d, u8, u8, c_int,
+                                                                    c_int]
             lib.oracle_forward.restype = c_int
-            lib.oracle_forward_indices.argtypes = [c_int] * 6 + [d] * 6 + [i32, d, d, u8, u8]
+            lib.oracle_forward_indices.argtypes = [c_int] * 6 + [d] * 6 + [i32, d, d, u8, u8, c_int]
             lib.oracle_forward_indices.restype = c_int
             lib.oracle_backward.argtypes = ([c_int] * 6 + [d] * 6 + [i32, d] + [d] * 6 +
-                                            [u8, u8])
+                                            [u8, u8, c_int])
             lib.oracle_backward.restype = c_int
             _lib = lib
     return _lib
@@ -130,12 +131,14 @@ def topk(r_row, k: int, first_token: bool = False):
     return I, rs
 
 
-def forward(X, Wr, Wq, Wk, Wv, Wo, k: int, batches=None, heads=None, first_token=False):
+def forward(X, Wr, Wq, Wk, Wv, Wo, k: int, batches=None, heads=None, first_token=False,
+            rope=False):
     """MoSA layer forward (Sec. 2.2, Eq. mosa_mha).  Returns (Y, I, r_sel, r_full).
 
     ``batches`` / ``heads`` restrict the computed units (b,h); Y[b] is exact
     for a batch whose every head is computed.  ``first_token``: every head
-    keeps token 0 and selects k-1 more (Sec. 3.2)."""
+    keeps token 0 and selects k-1 more (Sec. 3.2).  ``rope``: Q and K rotated
+    at the tokens' original positions (Sec. 2.2, positional encodings)."""
     X, Wr, Wq, Wk, Wv, Wo = map(_f64, (X, Wr, Wq, Wk, Wv, Wo))
     B, T, d, H, hp = _dims(X, Wq)
     Y = np.zeros((B, T, d))
@@ -146,13 +149,14 @@ def forward(X, Wr, Wq, Wk, Wv, Wo, k: int, batches=None, heads=None, first_token
     rc = _load().oracle_forward(B, T, d, H, hp, k, _ptr(X), _ptr(Wr), _ptr(Wq), _ptr(Wk),
                                 _ptr(Wv), _ptr(Wo), _ptr(Y), _ptr(I, ctypes.c_int32), _ptr(rs),
                                 _ptr(rf), _ptr(bm, ctypes.c_ubyte), _ptr(hm, ctypes.c_ubyte),
-                                1 if first_token else 0)
+                                1 if first_token else 0, 1 if rope else 0)
     if rc != 0:
         raise ValueError("oracle_forward failed (bad arguments or out of memory)")
     return Y, I, rs, rf
 
 
-def forward_indices(X, Wr, Wq, Wk, Wv, Wo, I, r_sel=None, batches=None, heads=None):
+def forward_indices(X, Wr, Wq, Wk, Wv, Wo, I, r_sel=None, batches=None, heads=None,
+                    rope=False):
     """Forward with the token sets I fixed.  If ``r_sel`` is None the scores
     are sigma(X W_r)[I] (TopK held constant); otherwise they are used as given
     (e.g. ones, for the fixed-sparse special case of Sec. 3.1)."""
@@ -166,13 +170,14 @@ def forward_indices(X, Wr, Wq, Wk, Wv, Wo, I, r_sel=None, batches=None, heads=No
     rc = _load().oracle_forward_indices(B, T, d, H, hp, k, _ptr(X), _ptr(Wr), _ptr(Wq),
                                         _ptr(Wk), _ptr(Wv), _ptr(Wo),
                                         _ptr(I, ctypes.c_int32), _ptr(rs), _ptr(Y),
-                                        _ptr(bm, ctypes.c_ubyte), _ptr(hm, ctypes.c_ubyte))
+                                        _ptr(bm, ctypes.c_ubyte), _ptr(hm, ctypes.c_ubyte),
+                                        1 if rope else 0)
     if rc != 0:
         raise ValueError("oracle_forward_indices failed")
     return Y
 
 
-def backward(X, Wr, Wq, Wk, Wv, Wo, I, dY, batches=None, heads=None):
+def backward(X, Wr, Wq, Wk, Wv, Wo, I, dY, batches=None, heads=None, rope=False):
     """Gradients of sum(Y * dY) for the token sets I (TopK held constant).
     Returns a dict with dX, dWr, dWq, dWk, dWv, dWo."""
     X, Wr, Wq, Wk, Wv, Wo, dY = map(_f64, (X, Wr, Wq, Wk, Wv, Wo, dY))
@@ -186,7 +191,7 @@ def backward(X, Wr, Wq, Wk, Wv, Wo, I, dY, batches=None, heads=None):
                                  _ptr(Wv), _ptr(Wo), _ptr(I, ctypes.c_int32), _ptr(dY),
                                  _ptr(g["dX"]), _ptr(g["dWr"]), _ptr(g["dWq"]), _ptr(g["dWk"]),
                                  _ptr(g["dWv"]), _ptr(g["dWo"]), _ptr(bm, ctypes.c_ubyte),
-                                 _ptr(hm, ctypes.c_ubyte))
+                                 _ptr(hm, ctypes.c_ubyte), 1 if rope else 0)
     if rc != 0:
         raise ValueError("oracle_backward failed")
     return g

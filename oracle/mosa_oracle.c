@@ -19,6 +19,9 @@
  *                              Y_j = X^o_i if j = I_i, else 0.
  *   Sec. 2.2, Eq. (mosa_mha):  MoSA(X) = sum_i MoSA_head(X; theta_i)
  *   Sec. 3.2 (IsoFLOP models): the first token is always in every head's set
+ *   Sec. 2.2 (positional encodings): RoPE rotates Q and K after the mapping by
+ *                              angles of the tokens' original positions I,
+ *                              half of the dimensions rotated, half unchanged
  *   Sec. 2.2 (last paragraph of the output definition): the router receives
  *                              its gradient only through the diag(r) scaling;
  *                              TopK itself is not differentiated.
@@ -31,6 +34,9 @@
  *   - The mask is applied inside the 1/sqrt(h') scaling; -inf stays -inf.
  *     The diagonal I_i >= I_i is always allowed, so no row is empty.
  *   - No router noise, no biases, no dropout.
+ *   - RoPE (optional): base 10000 and adjacent pairs (the RoFormer form) in
+ *     the first h'/2 dimensions: pair p = 0 .. h'/4-1 of position t turns by
+ *     t * 10000^(-2p / (h'/2)); dimensions h'/2 .. h'-1 are left unchanged.
  *   - Sec. 3.2 (IsoFLOP models) keeps the first token in every head and
  *     selects the other k-1 by router score: read as token 0 plus TopK(k-1)
  *     over tokens 1..T-1 (same tie rule), token 0 scaled by its own score.
@@ -166,11 +172,28 @@ static void head_state_free(head_state *s) {
     free(s->Xs); free(s->Q); free(s->K); free(s->V); free(s->P); free(s->A); free(s->AWo);
 }
 
-/* Sec. 2.2, steps gather -> projections -> masked attention -> A W^o for one
- * head on one sequence.  Xb is X[b] ([T,d]); the weights are this head's. */
+/* Sec. 2.2 (positional encodings): rotate the first h'/2 entries of v, a
+ * query or key row of the token at original position t, by +t theta_p
+ * (dir = +1) or back by -t theta_p (dir = -1, the transpose, for gradients);
+ * pair p = (2p, 2p+1), theta_p = 10000^(-2p / (h'/2)). */
+static void rope_rotate(double *v, int hp, int t, int dir) {
+    const int half = hp / 2;
+    for (int p = 0; p < half / 2; ++p) {
+        const double theta = pow(10000.0, -2.0 * p / (double)half);
+        const double ang = dir * (double)t * theta;
+        const double c = cos(ang), sn = sin(ang);
+        const double x0 = v[2 * p], x1 = v[2 * p + 1];
+        v[2 * p] = x0 * c - x1 * sn;
+        v[2 * p + 1] = x0 * sn + x1 * c;
+    }
+}
+
+/* Sec. 2.2, steps gather -> projections (-> RoPE at the original positions
+ * I when `rope`) -> masked attention -> A W^o for one head on one sequence.
+ * Xb is X[b] ([T,d]); the weights are this head's. */
 static void head_forward(const head_state *s, int T, const double *Xb, const int32_t *I,
                          const double *Wq, const double *Wk, const double *Wv,
-                         const double *Wo) {
+                         const double *Wo, int rope) {
     const int k = s->k, d = s->d, hp = s->hp;
     (void)T;
     /* X^s = (X_{I_1}, ..., X_{I_k}) */
@@ -189,6 +212,11 @@ static void head_forward(const head_state *s, int T, const double *Xb, const int
             s->Q[IDX2(i, p, hp)] = q;
             s->K[IDX2(i, p, hp)] = kk;
             s->V[IDX2(i, p, hp)] = v;
+        }
+    if (rope)
+        for (int i = 0; i < k; ++i) {
+            rope_rotate(s->Q + IDX2(i, 0, hp), hp, I[i], +1);
+            rope_rotate(s->K + IDX2(i, 0, hp), hp, I[i], +1);
         }
     /* P = softmax((QK^T + M) / sqrt(h')), M_ij = 0 iff I_i >= I_j else -inf.
      * Masked entries get probability exactly 0. */
@@ -244,7 +272,7 @@ int oracle_forward_indices(int B, int T, int d, int H, int hp, int k, const doub
                            const double *Wr, const double *Wq, const double *Wk,
                            const double *Wv, const double *Wo, const int32_t *I,
                            const double *r_sel_in, double *Y, const unsigned char *bsel,
-                           const unsigned char *hsel) {
+                           const unsigned char *hsel, int rope) {
     if (B <= 0 || T <= 0 || d <= 0 || H <= 0 || hp <= 0 || k <= 0 || k > T) return -1;
     memset(Y, 0, sizeof(double) * (size_t)B * T * d);
     int failed = 0;
@@ -272,7 +300,7 @@ int oracle_forward_indices(int B, int T, int d, int H, int hp, int k, const doub
                 }
             }
             head_forward(&s, T, Xb, Ibh, Wq + IDX3(h, 0, 0, d, hp), Wk + IDX3(h, 0, 0, d, hp),
-                         Wv + IDX3(h, 0, 0, d, hp), Wo + IDX3(h, 0, 0, hp, d));
+                         Wv + IDX3(h, 0, 0, d, hp), Wo + IDX3(h, 0, 0, hp, d), rope);
             /* X^o = diag(r^topk) A W^o;  Y_{I_i} += X^o_i  (Eq. mosa_mha sums the heads) */
             for (int i = 0; i < k; ++i)
                 for (int c = 0; c < d; ++c) {
@@ -291,7 +319,8 @@ int oracle_forward_indices(int B, int T, int d, int H, int hp, int k, const doub
 int oracle_forward(int B, int T, int d, int H, int hp, int k, const double *X,
                    const double *Wr, const double *Wq, const double *Wk, const double *Wv,
                    const double *Wo, double *Y, int32_t *I, double *r_sel, double *r_full,
-                   const unsigned char *bsel, const unsigned char *hsel, int first_token) {
+                   const unsigned char *bsel, const unsigned char *hsel, int first_token,
+                   int rope) {
     if (B <= 0 || T <= 0 || d <= 0 || H <= 0 || hp <= 0 || k <= 0 || k > T) return -1;
     int failed = 0;
     #pragma omp parallel for collapse(2) schedule(dynamic, 1) reduction(| : failed)
@@ -315,7 +344,7 @@ int oracle_forward(int B, int T, int d, int H, int hp, int k, const double *X,
         }
     if (failed) return -1;
     return oracle_forward_indices(B, T, d, H, hp, k, X, Wr, Wq, Wk, Wv, Wo, I, r_sel, Y, bsel,
-                                  hsel);
+                                  hsel, rope);
 }
 
 /* Backward of the layer for the token sets I (TopK held constant, Sec. 2.2):
@@ -327,7 +356,8 @@ int oracle_forward(int B, int T, int d, int H, int hp, int k, const double *X,
  *   dA        = diag(r) dX^o (W^o)^T
  *   dV        = P^T dA,   dP = dA V^T
  *   dS_ij     = P_ij (dP_ij - sum_l P_il dP_il)     (softmax; masked P = 0)
- *   dQ        = dS K / sqrt(h'),   dK = dS^T Q / sqrt(h')
+ *   dQ        = dS K / sqrt(h'),   dK = dS^T Q / sqrt(h')   (Q, K after RoPE)
+ *   with RoPE: dQ, dK rotated back to the projections' outputs (transpose)
  *   dW^{Q,K,V}+= X^s^T d{Q,K,V}
  *   dlogit_i  = dr_i r_i (1 - r_i)                  (sigma' = sigma (1 - sigma))
  *   dW^r     += X^s^T dlogit
@@ -337,7 +367,7 @@ int oracle_backward(int B, int T, int d, int H, int hp, int k, const double *X,
                     const double *Wr, const double *Wq, const double *Wk, const double *Wv,
                     const double *Wo, const int32_t *I, const double *dY, double *dX,
                     double *dWr, double *dWq, double *dWk, double *dWv, double *dWo,
-                    const unsigned char *bsel, const unsigned char *hsel) {
+                    const unsigned char *bsel, const unsigned char *hsel, int rope) {
     if (B <= 0 || T <= 0 || d <= 0 || H <= 0 || hp <= 0 || k <= 0 || k > T) return -1;
     memset(dX, 0, sizeof(double) * (size_t)B * T * d);
     memset(dWr, 0, sizeof(double) * (size_t)d * H);
@@ -379,7 +409,7 @@ int oracle_backward(int B, int T, int d, int H, int hp, int k, const double *X,
                 for (int c = 0; c < d; ++c) logit += Xb[IDX2(Ibh[i], c, d)] * Wr[IDX2(c, h, H)];
                 rs[i] = sigmoid(logit);
             }
-            head_forward(&s, T, Xb, Ibh, Wq_h, Wk_h, Wv_h, Wo_h);
+            head_forward(&s, T, Xb, Ibh, Wq_h, Wk_h, Wv_h, Wo_h, rope);
             /* dX^o = dY[I] */
             for (int i = 0; i < k; ++i)
                 for (int c = 0; c < d; ++c) dXo[IDX2(i, c, d)] = dYb[IDX2(Ibh[i], c, d)];
@@ -434,6 +464,11 @@ int oracle_backward(int B, int T, int d, int H, int hp, int k, const double *X,
                     }
                     dQ[IDX2(i, p, hp)] = aq * scale;
                     dK[IDX2(i, p, hp)] = ak * scale;
+                }
+            if (rope)
+                for (int i = 0; i < k; ++i) {
+                    rope_rotate(dQ + IDX2(i, 0, hp), hp, Ibh[i], -1);
+                    rope_rotate(dK + IDX2(i, 0, hp), hp, Ibh[i], -1);
                 }
             /* dlogit = dr o r o (1 - r) */
             for (int i = 0; i < k; ++i) dlogit[i] = dr[i] * rs[i] * (1.0 - rs[i]);

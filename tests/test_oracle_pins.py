@@ -333,7 +333,21 @@ def test_backward_matches_finite_differences(seed):
         assert np.abs(num - g[gname]).max() / scale < 1e-6, name
 
 
-def torch_restatement(X, Wr, Wq, Wk, Wv, Wo, I):
+def rope_complex(Z, pos):
+    """RoPE as complex multiplication: the first h'/2 entries of each row of Z
+    [..., k, h'] read as h'/4 complex numbers (2p + i (2p+1)), each multiplied
+    by exp(i pos theta_p), theta_p = 10000^(-2p / (h'/2)); the rest unchanged."""
+    hp = Z.shape[-1]
+    half = hp // 2
+    p = torch.arange(half // 2, dtype=torch.float64)
+    theta = 10000.0 ** (-2.0 * p / half)
+    ang = pos[..., None].to(torch.float64) * theta
+    zc = torch.view_as_complex(Z[..., :half].reshape(*Z.shape[:-1], half // 2, 2).contiguous())
+    rot = torch.view_as_real(zc * torch.polar(torch.ones_like(ang), ang))
+    return torch.cat([rot.reshape(*Z.shape[:-1], half), Z[..., half:]], dim=-1)
+
+
+def torch_restatement(X, Wr, Wq, Wk, Wv, Wo, I, rope=False):
     """Forward written with gather / einsum / scatter_add on float64 tensors."""
     B, T, d = X.shape
     H, _, hp = Wq.shape
@@ -345,6 +359,8 @@ def torch_restatement(X, Wr, Wq, Wk, Wv, Wo, I):
     Q = torch.einsum("bhkc,hcp->bhkp", Xs, Wq)
     K = torch.einsum("bhkc,hcp->bhkp", Xs, Wk)
     V = torch.einsum("bhkc,hcp->bhkp", Xs, Wv)
+    if rope:
+        Q, K = rope_complex(Q, idx), rope_complex(K, idx)
     S = torch.einsum("bhip,bhjp->bhij", Q, K) / np.sqrt(hp)
     allowed = idx[..., :, None] >= idx[..., None, :]
     S = S.masked_fill(~allowed, float("-inf"))
@@ -419,3 +435,44 @@ def test_layer_work_matches_head_formula_without_causal_halving():
     mine = w["forward_flops"] - w["attn_fwd"]["flops"] + 4 * hp * k * k * B * H
     paper = flops.head_flops_mosa(d, hp, T, k) * B * H - hp * k * B * H
     assert mine == paper
+
+
+# ------------------------------------------------ RoPE (Sec. 2.2) ----
+
+@pytest.mark.parametrize("hp", [4, 8, 16])
+def test_rope_forward_backward_match_complex_restatement(hp):
+    cfg, x = small(2, 40, 12, 3, hp, 9, seed=40 + hp)
+    _, I, _, _ = oracle.forward(x["X"], *weights(x), k=cfg.k)
+    ts = {n: torch.tensor(v, dtype=torch.float64, requires_grad=(n != "dY"))
+          for n, v in x.items()}
+    Y = torch_restatement(ts["X"], ts["Wr"], ts["Wq"], ts["Wk"], ts["Wv"], ts["Wo"],
+                          torch.tensor(I), rope=True)
+    Yo = oracle.forward_indices(x["X"], *weights(x), I=I, rope=True)
+    np.testing.assert_allclose(Y.detach().numpy(), Yo, rtol=1e-11, atol=1e-12)
+    (Y * ts["dY"]).sum().backward()
+    g = oracle.backward(x["X"], *weights(x), I=I, dY=x["dY"], rope=True)
+    for name in ("X", "Wr", "Wq", "Wk", "Wv", "Wo"):
+        np.testing.assert_allclose(g["d" + name], ts[name].grad.numpy(), rtol=1e-10,
+                                   atol=1e-11, err_msg=name)
+
+
+def test_rope_changes_only_through_positions():
+    # the rotation is a function of the original positions: the same token set
+    # with RoPE differs from the set without it, and k = T with RoPE equals
+    # dense causal attention on rotated queries and keys (positions 0..T-1)
+    B, T, d, H, hp = 1, 24, 16, 2, 8
+    _, x = small(B, T, d, H, hp, T, seed=5, plant=False)
+    Y, I, rs, rf = oracle.forward(x["X"], *weights(x), k=T, rope=True)
+    Y0, _, _, _ = oracle.forward(x["X"], *weights(x), k=T)
+    assert np.abs(Y - Y0).max() > 1e-3
+    Xt = torch.tensor(x["X"], dtype=torch.float64)
+    ref = torch.zeros_like(Xt)
+    pos = torch.arange(T)
+    for h in range(H):
+        q = rope_complex(Xt @ torch.tensor(x["Wq"][h], dtype=torch.float64), pos)
+        kk = rope_complex(Xt @ torch.tensor(x["Wk"][h], dtype=torch.float64), pos)
+        v = Xt @ torch.tensor(x["Wv"][h], dtype=torch.float64)
+        a = F.scaled_dot_product_attention(q, kk, v, is_causal=True)
+        r = torch.sigmoid(Xt @ torch.tensor(x["Wr"][:, h], dtype=torch.float64))
+        ref += r[..., None] * (a @ torch.tensor(x["Wo"][h], dtype=torch.float64))
+    np.testing.assert_allclose(Y, ref.numpy(), rtol=1e-10, atol=1e-12)

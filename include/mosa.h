@@ -82,7 +82,13 @@ typedef struct {
     int32_t B, T, d, H, hp, k;
     int32_t dtype;       /* mosa_dtype of X, dY and all weights */
     int32_t first_token; /* 0 or 1, see above */
+    int32_t rope;        /* 0 or 1: rotary position encoding, see below */
 } mosa_shape;
+/* rope = 1 rotates each head's queries and keys after the projections by the
+ * tokens' original positions t = I[b,h,i] (Sec. 2.2, positional encodings):
+ * pair (2p, 2p+1) of the first h'/2 dimensions turns by t * 10000^(-2p/(h'/2)),
+ * the other h'/2 dimensions are left unchanged.  A backward must be given the
+ * same rope value as its forward. */
 
 /* Supported sizes (else MOSA_ERR_UNSUPPORTED):
  *   1 <= k <= T <= 65536; B, H >= 1; B*T*d < 2^31; H*d*hp < 2^31;

@@ -35,10 +35,12 @@ class MosaShape(ctypes.Structure):
     every head keeps token 0 and selects k-1 more, Sec. 3.2)."""
     _fields_ = [("B", ctypes.c_int32), ("T", ctypes.c_int32), ("d", ctypes.c_int32),
                 ("H", ctypes.c_int32), ("hp", ctypes.c_int32), ("k", ctypes.c_int32),
-                ("dtype", ctypes.c_int32), ("first_token", ctypes.c_int32)]
+                ("dtype", ctypes.c_int32), ("first_token", ctypes.c_int32),
+                ("rope", ctypes.c_int32)]
 
     def astuple(self):
-        return (self.B, self.T, self.d, self.H, self.hp, self.k, self.dtype, self.first_token)
+        return (self.B, self.T, self.d, self.H, self.hp, self.k, self.dtype, self.first_token,
+                self.rope)
 
 
 class MosaError(RuntimeError):
@@ -144,12 +146,13 @@ def _stream(stream):
     return ctypes.c_void_p(s.cuda_stream)
 
 
-def make_shape(X, W_q, k: int, first_token: bool = False) -> MosaShape:
+def make_shape(X, W_q, k: int, first_token: bool = False, rope: bool = False) -> MosaShape:
     B, T, d = X.shape
     H, d2, hp = W_q.shape
     if d2 != d:
         raise ValueError("W_q must be [H, d, hp] with the d of X")
-    return MosaShape(B, T, d, H, hp, int(k), _dtype_code(X), 1 if first_token else 0)
+    return MosaShape(B, T, d, H, hp, int(k), _dtype_code(X), 1 if first_token else 0,
+                     1 if rope else 0)
 
 
 def mosa_adaptive_k(T: int, rho: int) -> int:
@@ -178,14 +181,15 @@ def _same(ref, *ts):
 
 
 def mosa_forward(X, W_r, W_q, W_k, W_v, W_o, k: int, workspace=None, want_r_full=False,
-                 out=None, stream=None, first_token: bool = False):
+                 out=None, stream=None, first_token: bool = False, rope: bool = False):
     """Forward pass (Sec. 2.2).  Returns (Y, I, r_sel, r_full or None, workspace).
 
     ``out`` may hold preallocated "Y", "I", "r_sel" (and "r_full") tensors.
     With ``first_token`` every head keeps token 0 and selects k-1 more
-    (Sec. 3.2)."""
+    (Sec. 3.2); with ``rope`` Q and K are rotated at the tokens' original
+    positions (Sec. 2.2), and the backward must be given ``rope`` too."""
     torch = _torch()
-    shape = make_shape(X, W_q, k, first_token)
+    shape = make_shape(X, W_q, k, first_token, rope)
     _same(X, ("W_r", W_r), ("W_q", W_q), ("W_k", W_k), ("W_v", W_v), ("W_o", W_o))
     B, T, d, H = shape.B, shape.T, shape.d, shape.H
     dev = X.device
@@ -209,11 +213,11 @@ def mosa_forward(X, W_r, W_q, W_k, W_v, W_o, k: int, workspace=None, want_r_full
 
 
 def mosa_forward_with_indices(X, W_q, W_k, W_v, W_o, I, r_sel, workspace=None, out=None,
-                              stream=None):
+                              stream=None, rope: bool = False):
     """Forward with caller-chosen token sets (e.g. the fixed-sparse case of
     Sec. 3.1).  Returns (Y, workspace)."""
     torch = _torch()
-    shape = make_shape(X, W_q, I.shape[-1])
+    shape = make_shape(X, W_q, I.shape[-1], rope=rope)
     _same(X, ("W_q", W_q), ("W_k", W_k), ("W_v", W_v), ("W_o", W_o))
     B, T, d = shape.B, shape.T, shape.d
     Y = (out or {}).get("Y")
@@ -230,10 +234,12 @@ def mosa_forward_with_indices(X, W_q, W_k, W_v, W_o, I, r_sel, workspace=None, o
     return Y, workspace
 
 
-def mosa_backward(X, W_r, W_q, W_k, W_v, W_o, I, r_sel, dY, workspace, out=None, stream=None):
-    """Backward pass; returns a dict with dX, dW_r, dW_q, dW_k, dW_v, dW_o (fp32)."""
+def mosa_backward(X, W_r, W_q, W_k, W_v, W_o, I, r_sel, dY, workspace, out=None, stream=None,
+                  rope: bool = False):
+    """Backward pass; returns a dict with dX, dW_r, dW_q, dW_k, dW_v, dW_o (fp32).
+    ``rope`` must match the forward's."""
     torch = _torch()
-    shape = make_shape(X, W_q, I.shape[-1])
+    shape = make_shape(X, W_q, I.shape[-1], rope=rope)
     _same(X, ("W_r", W_r), ("W_q", W_q), ("W_k", W_k), ("W_v", W_v), ("W_o", W_o), ("dY", dY))
     dev = X.device
     g = dict(out or {})

@@ -95,10 +95,39 @@ struct Saved {
     float *WrT;         // [H,d] fp32 transpose of W_r (tensor-core dX epilogue)
 };
 
+// Rotary position encoding (Sec. 2.2): pair p of the first h'/2 dimensions of
+// a query or key row at original position t turns by t * theta_p, theta_p =
+// 10000^(-2p / (h'/2)).  phi[p] holds theta_p / (2 pi) in turns per position
+// as a 64-bit fixed-point fraction, so t * phi[p] taken mod 2^64 is the angle's
+// fraction of a turn, exact up to phi's rounding (about 1e-12 rad at t =
+// 65535), for any t: no large angle ever reaches a floating-point sin or cos.
+constexpr int kRopeMaxPairs = 32;   // h' <= 128
+struct RopeTable {
+    uint64_t phi[kRopeMaxPairs];
+    int npairs;   // h' / 4
+    int T;        // positions are gidx mod T
+};
+
+// (x0, x1) turned by dir * t * theta (dir = +1 forward, -1 for gradients).
+// The top 24 bits of the turn fraction, read as signed, give the angle in
+// [-pi, pi), where the hardware sine and cosine are accurate to about 4e-7.
+__device__ __forceinline__ void rope_turn(float &x0, float &x1, uint64_t phi, int t, float dir) {
+    const uint64_t turns = phi * (uint64_t)(uint32_t)t;               // mod one turn
+    const int32_t q = (int32_t)(uint32_t)(turns >> 32) >> 8;          // [-2^23, 2^23)
+    const float ang = (float)q * (6.2831853071795865f / 16777216.f);  // [-pi, pi)
+    float sn, cs;
+    __sincosf(ang, &sn, &cs);
+    sn *= dir;
+    const float y0 = x0 * cs - x1 * sn, y1 = x0 * sn + x1 * cs;
+    x0 = y0;
+    x1 = y1;
+}
+
 struct Dims {
     int B, T, d, H, hp, k;
     bool bf16;
     bool first_token;   // token 0 always kept, k-1 more by score (Sec. 3.2)
+    bool rope;          // rotary position encoding of Q and K (Sec. 2.2)
     long long rows() const { return (long long)H * B * k; }
     size_t esize() const { return bf16 ? 2 : 4; }
 };

@@ -25,6 +25,7 @@ mosa_status check_shape(const mosa_shape *s, Dims *out) {
     if (s->k > s->T) return MOSA_ERR_INVALID_ARG;
     if (s->dtype != MOSA_F32 && s->dtype != MOSA_BF16) return MOSA_ERR_INVALID_ARG;
     if (s->first_token != 0 && s->first_token != 1) return MOSA_ERR_INVALID_ARG;
+    if (s->rope != 0 && s->rope != 1) return MOSA_ERR_INVALID_ARG;
     const long long lim = 1LL << 31;
     if ((long long)s->B * s->T * s->d >= lim) return MOSA_ERR_UNSUPPORTED;
     if ((long long)s->H * s->d * s->hp >= lim) return MOSA_ERR_UNSUPPORTED;
@@ -35,7 +36,8 @@ mosa_status check_shape(const mosa_shape *s, Dims *out) {
     if (s->d % 8 != 0) return MOSA_ERR_UNSUPPORTED;
     if (s->hp != 16 && s->hp != 32 && s->hp != 64 && s->hp != 128) return MOSA_ERR_UNSUPPORTED;
     if (out)
-        *out = Dims{s->B, s->T, s->d, s->H, s->hp, s->k, s->dtype == MOSA_BF16, s->first_token != 0};
+        *out = Dims{s->B, s->T, s->d, s->H, s->hp, s->k, s->dtype == MOSA_BF16, s->first_token != 0,
+                    s->rope != 0};
     return MOSA_OK;
 }
 
@@ -122,12 +124,35 @@ cudaError_t link(cudaStream_t from, cudaStream_t to, cudaEvent_t ev) {
 }
 
 // F3-F5 for the rows already selected into sv.gidx / sv.rsel.
+// RoPE (Sec. 2.2) in place on the stored Q and K rows (dir +1), or on the dQ
+// and dK blocks of the dQ|dK|dV rows (dir -1).  Pair storage for bf16 inputs:
+// on the tensor cores Q is [hi 64 | lo 64] and dQ|dK|dV|dlogit [hi 256 | lo 256]
+// per row, on the CUDA cores [hi hp | lo hp] and [hi 3hp | lo 3hp]; fp32 rows
+// otherwise.
+cudaError_t rope_qk(const Dims &dm, const Saved &sv, bool grads, cudaStream_t s) {
+    const RopeTable tab = make_rope_table(dm.hp, dm.T);
+    const long long rows = dm.rows();
+    const bool pair = dm.bf16;
+    cudaError_t e;
+    if (!grads) {
+        e = launch_rope(sv.Q, pair, dm.hp, 0, rows, sv.gidx, tab, 1.f, s);
+        if (e == cudaSuccess) e = launch_rope(sv.K, pair, dm.hp, 0, rows, sv.gidx, tab, 1.f, s);
+    } else {
+        const int cols = use_tc(dm) ? 256 : 3 * dm.hp;
+        e = launch_rope(sv.dQKV, pair, cols, 0, rows, sv.gidx, tab, -1.f, s);
+        if (e == cudaSuccess)
+            e = launch_rope(sv.dQKV, pair, cols, dm.hp, rows, sv.gidx, tab, -1.f, s);
+    }
+    return e;
+}
+
 mosa_status forward_heads(const Dims &dm, const void *X, const void *W_q, const void *W_k,
                           const void *W_v, const void *W_o, float *Y, const Saved &sv,
                           cudaStream_t s) {
     {
         StageScope st_(kStageQkv, s);
         MOSA_TRY(launch_qkv(dm, X, W_q, W_k, W_v, sv, s));
+        if (dm.rope) MOSA_TRY(rope_qk(dm, sv, false, s));
     }
     {
         StageScope st_(kStageAttnFwd, s);
@@ -174,6 +199,7 @@ mosa_status forward_tc(const Dims &dm, const void *X, const void *W_r, const voi
     {
         StageScope st_(kStageQkv, s);
         MOSA_TRY(launch_qkv(dm, X, W_q, W_k, W_v, sv, s));
+        if (dm.rope) MOSA_TRY(rope_qk(dm, sv, false, s));
     }
     {
         StageScope st_(kStageAttnFwd, s);
@@ -207,6 +233,7 @@ mosa_status backward_tc(const Dims &dm, const void *X, const void *W_r, const vo
         {
             StageScope st_(kStageBwdUnit, s);
             MOSA_TRY(tc_fused_backward(dm, W_o, dY, sv, s));
+            if (dm.rope) MOSA_TRY(rope_qk(dm, sv, true, s));
         }
         MOSA_TRY(link(s, t, r.ev[2]));  // dQ|dK|dV|dlogit ready
         {
@@ -239,6 +266,7 @@ mosa_status backward_tc(const Dims &dm, const void *X, const void *W_r, const vo
     {
         StageScope st_(kStageAttnBwd, s);
         MOSA_TRY(launch_attn_bwd(dm, sv, s));
+        if (dm.rope) MOSA_TRY(rope_qk(dm, sv, true, s));
     }
     MOSA_TRY(link(s, t, r.ev[2]));  // dQ|dK|dV|dlogit ready for dW
     {
@@ -468,6 +496,7 @@ mosa_status mosa_backward(const mosa_shape *shape, const void *X, const void *W_
         {
             StageScope st_(kStageAttnBwd, s);
             MOSA_TRY(launch_attn_bwd(dm, sv, s));
+            if (dm.rope) MOSA_TRY(rope_qk(dm, sv, true, s));
         }
         {
             StageScope st_(kStageInBwd, s);

@@ -57,7 +57,8 @@ extern "C" mosa_status mosa_route_noalloc(const mosa_shape *shape, const void *X
         if (shape == nullptr || shape->B <= 0 || shape->T <= 0 || shape->d <= 0 ||
             shape->H <= 0 || shape->hp <= 0 || shape->k <= 0 || shape->k > shape->T ||
             (shape->dtype != MOSA_F32 && shape->dtype != MOSA_BF16) ||
-            (shape->first_token != 0 && shape->first_token != 1))
+            (shape->first_token != 0 && shape->first_token != 1) ||
+            (shape->rope != 0 && shape->rope != 1))
             return MOSA_ERR_INVALID_ARG;
         return MOSA_ERR_UNSUPPORTED;
     }
@@ -67,7 +68,7 @@ extern "C" mosa_status mosa_route_noalloc(const mosa_shape *shape, const void *X
     float *scores = nullptr;
     if (scores_address(&scores) != cudaSuccess) return MOSA_ERR_CUDA;
     const Dims dm{shape->B, shape->T, shape->d, shape->H, shape->hp, shape->k,
-                  shape->dtype == MOSA_BF16, shape->first_token != 0};
+                  shape->dtype == MOSA_BF16, shape->first_token != 0, shape->rope != 0};
     cudaStream_t s = static_cast<cudaStream_t>(stream);
     // Every score the selection reads is written by the router first, so the
     // array needs no clearing between calls.

@@ -9,7 +9,8 @@
 //            5-stage ring (three slots of its own, two in the Q/K/V tiles, idle
 //            until phase 2): W blocks by TMA, the selected rows of X by 16-byte
 //            cp.async gathers, confirmed three blocks after issue
-//   phase 2  the accumulator is read back and split into bf16 hi/lo pairs, kept
+//   phase 2  the accumulator is read back (Q and K turned by RoPE at the rows'
+//            original positions when asked, Sec. 2.2) and split into bf16 hi/lo pairs, kept
 //            in shared memory as the attention operands; warp 3 copies them to
 //            global memory (the backward reads them) by TMA stores while the
 //            softmax runs
@@ -78,6 +79,8 @@ struct FusedParams {
     float *Y;              // [B*T, d], accumulated into
     int B, T, d, k, U, Mtok;
     float scale_log2;
+    int rope_on;           // RoPE on Q and K (Sec. 2.2)
+    RopeTable rope;
     uint32_t *status;
 };
 
@@ -318,6 +321,12 @@ __global__ void __launch_bounds__(kThreads, 1) fused_fwd_kernel(const __grid_con
         for (int c0 = 96 * ch; c0 < 96 * ch + 96; c0 += 32) {
             float v[32];
             tmem_ld32(tmem + lane_off + c0, v);
+            if (p.rope_on && (c0 == 0 || c0 == 64) && valid) {
+                // the first h'/2 = 32 columns of Q (c0 = 0) and of K (c0 = 64)
+                const int t = sm.rows[r] % p.rope.T;
+#pragma unroll
+                for (int pr = 0; pr < 16; ++pr) rope_turn(v[2 * pr], v[2 * pr + 1], p.rope.phi[pr], t, 1.f);
+            }
             uint8_t(*tile)[kHalf] = c0 < 64 ? sm.q : (c0 < 128 ? sm.k : sm.v);
             put_pair32(tile[0], tile[1], r, c0, v, 1.f);
         }
@@ -451,6 +460,8 @@ cudaError_t tc_fused_forward(const Dims &dm, const void *X, const void *Wq, cons
     p.U = 128 / dm.k;
     p.Mtok = dm.B * dm.k;
     p.scale_log2 = 1.4426950408889634f / sqrtf(64.f);
+    p.rope_on = dm.rope ? 1 : 0;
+    if (dm.rope) p.rope = make_rope_table(64, dm.T);
     p.status = sv.status;
     static std::once_flag once;
     static cudaError_t attr = cudaSuccess;

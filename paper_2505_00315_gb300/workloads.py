@@ -47,6 +47,7 @@ class MosaConfig:
     backward: bool = True
     seed: int = 0
     first_token: bool = False    # every head keeps token 0 and selects k-1 more
+    rope: bool = False           # rotary position encoding of Q and K
     note: str = field(default="", compare=False)
 
     @property

@@ -25,11 +25,11 @@ def run_layer(cfg, x, backward=True):
     dt = cfg.dtype
     X, Wr, Wq, Wk, Wv, Wo = (to_dev(x[n], dt) for n in ("X", "Wr", "Wq", "Wk", "Wv", "Wo"))
     Y, I, rs, rf, ws = mosa.mosa_forward(X, Wr, Wq, Wk, Wv, Wo, cfg.k, want_r_full=True,
-                                         first_token=cfg.first_token)
+                                         first_token=cfg.first_token, rope=cfg.rope)
     out = {"Y": Y, "I": I, "r_sel": rs, "r_full": rf}
     if backward:
         dY = to_dev(x["dY"], dt)
-        out.update(mosa.mosa_backward(X, Wr, Wq, Wk, Wv, Wo, I, rs, dY, ws))
+        out.update(mosa.mosa_backward(X, Wr, Wq, Wk, Wv, Wo, I, rs, dY, ws, rope=cfg.rope))
     torch.cuda.synchronize()
     st = mosa.mosa_check_status(mosa.make_shape(X, Wq, cfg.k), ws)
     assert st == 0, f"device status {st}"

@@ -166,6 +166,38 @@ def test_first_token_long_rows_unstaged_select():
         np.testing.assert_array_equal(I[0, h], Iref)
 
 
+# ------------------------------------------- RoPE at the original positions ----
+
+ROPE = [
+    W.MosaConfig("rope_bf16", B=3, T=200, d=64, H=2, hp=64, k=64, dtype="bf16", seed=41,
+                 rope=True),
+    W.MosaConfig("rope_largek_bf16", B=2, T=600, d=64, H=2, hp=64, k=300, dtype="bf16",
+                 seed=42, rope=True),
+    W.MosaConfig("rope_far_bf16", B=1, T=20000, d=64, H=2, hp=64, k=64, dtype="bf16", seed=43,
+                 rope=True),
+    W.MosaConfig("rope_f32", B=2, T=129, d=24, H=3, hp=32, k=40, dtype="f32", seed=44,
+                 rope=True),
+    W.MosaConfig("rope_hp16_f32", B=2, T=90, d=16, H=2, hp=16, k=33, dtype="f32", seed=45,
+                 rope=True),
+    W.MosaConfig("rope_first_bf16", B=2, T=150, d=32, H=2, hp=64, k=50, dtype="bf16", seed=46,
+                 rope=True, first_token=True),
+]
+
+
+@pytest.mark.parametrize("cfg", ROPE, ids=lambda c: c.name)
+def test_rope_forward_backward_parity(cfg, kernel_path):
+    x = W.make_inputs(cfg)
+    Y, I, rs, rf = oracle.forward(x["X"], *weights(x), k=cfg.k, first_token=cfg.first_token,
+                                  rope=True)
+    g = run_layer(cfg, x, backward=True)
+    np.testing.assert_array_equal(g["I"], I)
+    assert_close("Y", g["Y"], Y, cfg.dtype)
+    ref = oracle.backward(x["X"], *weights(x), I=I, dY=x["dY"], rope=True)
+    for name in ("dX", "dWr", "dWq", "dWk", "dWv", "dWo"):
+        gname = name[:2] + "_" + name[2:].lower() if name != "dX" else "dX"
+        assert_close(name, g[gname], ref[name], cfg.dtype)
+
+
 # ------------------------------------------------ full workload sizes ----
 
 FULL = [c for c in W.CONFIGS.values() if c.dtype == "bf16"]

@@ -198,6 +198,36 @@ def test_rope_forward_backward_parity(cfg, kernel_path):
         assert_close(name, g[gname], ref[name], cfg.dtype)
 
 
+# ------------------------- hybrid layer: MoSA heads beside dense heads ----
+
+@pytest.mark.parametrize("rope", [False, True])
+def test_hybrid_mosa_plus_dense_heads(rope):
+    # Sec. 2.2 (hybridization): MoSA heads and dense heads in one layer, their
+    # outputs summed; a dense head is the index-given forward with I = 0..T-1
+    # and unit scores
+    cfg = W.MosaConfig("hybrid", B=2, T=128, d=64, H=4, hp=64, k=32, dtype="bf16", seed=51,
+                       rope=rope)
+    dense = W.MosaConfig("hybrid_dense", B=2, T=128, d=64, H=2, hp=64, k=128, dtype="bf16",
+                         seed=52, rope=rope)
+    x = W.make_inputs(cfg)
+    xd = W.make_inputs(dense, plant=False)
+    Ym, I, _, _ = oracle.forward(x["X"], *weights(x), k=cfg.k, rope=rope)
+    Idense = np.broadcast_to(np.arange(cfg.T, dtype=np.int32), (cfg.B, dense.H, cfg.T)).copy()
+    ones = np.ones((cfg.B, dense.H, cfg.T))
+    Yd = oracle.forward_indices(x["X"], xd["Wr"], xd["Wq"], xd["Wk"], xd["Wv"], xd["Wo"],
+                                I=Idense, r_sel=ones, rope=rope)
+    X = to_dev(x["X"], "bf16")
+    Wm = [to_dev(x[n], "bf16") for n in ("Wr", "Wq", "Wk", "Wv", "Wo")]
+    Wd = [to_dev(xd[n], "bf16") for n in ("Wq", "Wk", "Wv", "Wo")]
+    Yg, Ig, _, _, _ = mosa.mosa_forward(X, *Wm, cfg.k, rope=rope)
+    Ydg, _ = mosa.mosa_forward_with_indices(
+        X, *Wd, torch.tensor(Idense, device="cuda"),
+        torch.ones((cfg.B, dense.H, cfg.T), dtype=torch.float32, device="cuda"), rope=rope)
+    torch.cuda.synchronize()
+    np.testing.assert_array_equal(Ig.cpu().numpy(), I)
+    assert_close("Y", (Yg + Ydg).cpu().numpy(), Ym + Yd, "bf16")
+
+
 # ------------------------------------------------ full workload sizes ----
 
 FULL = [c for c in W.CONFIGS.values() if c.dtype == "bf16"]

@@ -68,6 +68,11 @@ def _load():
             lib.oracle_backward.argtypes = ([c_int] * 6 + [d] * 6 + [i32, d] + [d] * 6 +
                                             [u8, u8, c_int])
             lib.oracle_backward.restype = c_int
+            lib.oracle_dense_forward.argtypes = [c_int] * 6 + [d] * 5 + [d, u8, u8, c_int]
+            lib.oracle_dense_forward.restype = c_int
+            lib.oracle_dense_backward.argtypes = ([c_int] * 6 + [d] * 6 + [d] * 5 +
+                                                  [u8, u8, c_int])
+            lib.oracle_dense_backward.restype = c_int
             _lib = lib
     return _lib
 
@@ -194,4 +199,64 @@ def backward(X, Wr, Wq, Wk, Wv, Wo, I, dY, batches=None, heads=None, rope=False)
                                  _ptr(hm, ctypes.c_ubyte), 1 if rope else 0)
     if rc != 0:
         raise ValueError("oracle_backward failed")
+    return g
+
+
+def dense_forward(X, Dq, Dk, Dv, Do, window: int = 0, batches=None, heads=None, rope=False):
+    """Dense heads of a hybrid layer (Sec. 2.2, hybridization): causal
+    multi-head attention over all T tokens (Sec. 2.1, Eq. mha), no router.
+    ``window`` > 0: local heads (Sec. 3.4), token i sees token j iff j <= i and
+    both lie in the same block of ``window`` positions.  Returns Y [B,T,d]."""
+    X, Dq, Dk, Dv, Do = map(_f64, (X, Dq, Dk, Dv, Do))
+    B, T, d, H, hp = _dims(X, Dq)
+    Y = np.zeros((B, T, d))
+    bm, hm = _mask(batches, B), _mask(heads, H)
+    rc = _load().oracle_dense_forward(B, T, d, H, hp, int(window), _ptr(X), _ptr(Dq), _ptr(Dk),
+                                      _ptr(Dv), _ptr(Do), _ptr(Y), _ptr(bm, ctypes.c_ubyte),
+                                      _ptr(hm, ctypes.c_ubyte), 1 if rope else 0)
+    if rc != 0:
+        raise ValueError("oracle_dense_forward failed")
+    return Y
+
+
+def dense_backward(X, Dq, Dk, Dv, Do, dY, window: int = 0, batches=None, heads=None,
+                   rope=False):
+    """Gradients of sum(Y * dY) for the dense (or local) heads of
+    ``dense_forward``.  Returns a dict with dX, dWq, dWk, dWv, dWo."""
+    X, Dq, Dk, Dv, Do, dY = map(_f64, (X, Dq, Dk, Dv, Do, dY))
+    B, T, d, H, hp = _dims(X, Dq)
+    g = {"dX": np.zeros((B, T, d)), "dWq": np.zeros((H, d, hp)), "dWk": np.zeros((H, d, hp)),
+         "dWv": np.zeros((H, d, hp)), "dWo": np.zeros((H, hp, d))}
+    bm, hm = _mask(batches, B), _mask(heads, H)
+    rc = _load().oracle_dense_backward(B, T, d, H, hp, int(window), _ptr(X), _ptr(Dq), _ptr(Dk),
+                                       _ptr(Dv), _ptr(Do), _ptr(dY), _ptr(g["dX"]),
+                                       _ptr(g["dWq"]), _ptr(g["dWk"]), _ptr(g["dWv"]),
+                                       _ptr(g["dWo"]), _ptr(bm, ctypes.c_ubyte),
+                                       _ptr(hm, ctypes.c_ubyte), 1 if rope else 0)
+    if rc != 0:
+        raise ValueError("oracle_dense_backward failed")
+    return g
+
+
+def hybrid_forward(X, Wr, Wq, Wk, Wv, Wo, Dq, Dk, Dv, Do, k: int, window: int = 0,
+                   batches=None, first_token=False, rope=False):
+    """Hybrid layer (Sec. 2.2, hybridization): the MoSA heads plus the dense
+    (or local) heads, outputs summed as every head's is (Eq. mha).  Returns
+    (Y, I, r_sel, r_full) with I, r_sel, r_full those of the MoSA heads."""
+    Y, I, rs, rf = forward(X, Wr, Wq, Wk, Wv, Wo, k, batches=batches,
+                           first_token=first_token, rope=rope)
+    Y = Y + dense_forward(X, Dq, Dk, Dv, Do, window, batches=batches, rope=rope)
+    return Y, I, rs, rf
+
+
+def hybrid_backward(X, Wr, Wq, Wk, Wv, Wo, Dq, Dk, Dv, Do, I, dY, window: int = 0,
+                    batches=None, rope=False):
+    """Gradients of the hybrid layer: dX summed over both head groups; dWr,
+    dWq, dWk, dWv, dWo of the MoSA heads; dDq, dDk, dDv, dDo of the dense
+    heads."""
+    g = backward(X, Wr, Wq, Wk, Wv, Wo, I, dY, batches=batches, rope=rope)
+    gd = dense_backward(X, Dq, Dk, Dv, Do, dY, window, batches=batches, rope=rope)
+    g["dX"] = g["dX"] + gd["dX"]
+    for n in ("q", "k", "v", "o"):
+        g["dD" + n] = gd["dW" + n]
     return g

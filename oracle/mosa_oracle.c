@@ -40,6 +40,13 @@
  *   - Sec. 3.2 (IsoFLOP models) keeps the first token in every head and
  *     selects the other k-1 by router score: read as token 0 plus TopK(k-1)
  *     over tokens 1..T-1 (same tie rule), token 0 scaled by its own score.
+ *   - Hybrid layers (Sec. 2.2, hybridization) add dense heads (Sec. 2.1,
+ *     Eq. mha, causal M, no router and no scaling) or, for long sequences
+ *     (Sec. 3.4), local heads.  The paper does not define its local
+ *     attention; read as the block pattern of the cited fixed sparse
+ *     attention: token i sees token j iff j <= i and floor(j/w) = floor(i/w)
+ *     for a window of w tokens (the last block may be shorter).  The layer
+ *     output is the sum over all heads, sparse and dense.
  *
  * Layouts (row-major, all fp64 here):
  *   X [B,T,d]; W_r [d,H]; W_q, W_k, W_v [H,d,h']; W_o [H,h',d];
@@ -188,12 +195,20 @@ static void rope_rotate(double *v, int hp, int t, int dir) {
     }
 }
 
+/* The attention mask M of Sec. 2.2: query i may attend to key j iff
+ * I_i >= I_j; with a window w > 0 (local heads, Sec. 3.4) also only within
+ * the same block of w original positions. */
+static int visible(const int32_t *I, int i, int j, int window) {
+    if (I[i] < I[j]) return 0;
+    return window <= 0 || I[i] / window == I[j] / window;
+}
+
 /* Sec. 2.2, steps gather -> projections (-> RoPE at the original positions
  * I when `rope`) -> masked attention -> A W^o for one head on one sequence.
  * Xb is X[b] ([T,d]); the weights are this head's. */
 static void head_forward(const head_state *s, int T, const double *Xb, const int32_t *I,
                          const double *Wq, const double *Wk, const double *Wv,
-                         const double *Wo, int rope) {
+                         const double *Wo, int rope, int window) {
     const int k = s->k, d = s->d, hp = s->hp;
     (void)T;
     /* X^s = (X_{I_1}, ..., X_{I_k}) */
@@ -218,13 +233,14 @@ static void head_forward(const head_state *s, int T, const double *Xb, const int
             rope_rotate(s->Q + IDX2(i, 0, hp), hp, I[i], +1);
             rope_rotate(s->K + IDX2(i, 0, hp), hp, I[i], +1);
         }
-    /* P = softmax((QK^T + M) / sqrt(h')), M_ij = 0 iff I_i >= I_j else -inf.
-     * Masked entries get probability exactly 0. */
+    /* P = softmax((QK^T + M) / sqrt(h')), M_ij = 0 iff visible(i, j) (I_i >= I_j,
+     * and the same block of a local head) else -inf.  Masked entries get
+     * probability exactly 0. */
     const double scale = 1.0 / sqrt((double)hp);
     for (int i = 0; i < k; ++i) {
         double row_max = -INFINITY;
         for (int j = 0; j < k; ++j) {
-            if (I[i] >= I[j]) {
+            if (visible(I, i, j, window)) {
                 double dot = 0.0;
                 for (int p = 0; p < hp; ++p) dot += s->Q[IDX2(i, p, hp)] * s->K[IDX2(j, p, hp)];
                 double sij = dot * scale;
@@ -234,7 +250,7 @@ static void head_forward(const head_state *s, int T, const double *Xb, const int
         }
         double denom = 0.0;
         for (int j = 0; j < k; ++j) {
-            if (I[i] >= I[j]) {
+            if (visible(I, i, j, window)) {
                 double e = exp(s->P[IDX2(i, j, k)] - row_max);
                 s->P[IDX2(i, j, k)] = e;
                 denom += e;
@@ -262,17 +278,14 @@ static void head_forward(const head_state *s, int T, const double *Xb, const int
 
 static int selected(const unsigned char *mask, int i) { return mask == NULL || mask[i] != 0; }
 
-/* Forward of the layer with the token sets fixed by the caller.
- * I [B,H,k]; if r_sel_in is non-NULL it is used as r^topk (the fixed-sparse
- * special case of Sec. 3.1 passes ones), otherwise r^topk = sigma(X W^r)[I]
- * is computed, which keeps W^r differentiable with TopK held constant.
- * Y [B,T,d] is overwritten: Y[b] = sum_h scatter(diag(r^topk) A W^o).
- * Returns 0 or -1. */
-int oracle_forward_indices(int B, int T, int d, int H, int hp, int k, const double *X,
-                           const double *Wr, const double *Wq, const double *Wk,
-                           const double *Wv, const double *Wo, const int32_t *I,
-                           const double *r_sel_in, double *Y, const unsigned char *bsel,
-                           const unsigned char *hsel, int rope) {
+/* Heads on fixed token sets: Y[b] = sum_h scatter(diag(r) A W^o) with the
+ * mask window of head_forward.  r is r_sel_in if non-NULL, else
+ * sigma(X W^r)[I].  Y [B,T,d] is overwritten. */
+static int forward_units(int B, int T, int d, int H, int hp, int k, const double *X,
+                         const double *Wr, const double *Wq, const double *Wk,
+                         const double *Wv, const double *Wo, const int32_t *I,
+                         const double *r_sel_in, double *Y, const unsigned char *bsel,
+                         const unsigned char *hsel, int rope, int window) {
     if (B <= 0 || T <= 0 || d <= 0 || H <= 0 || hp <= 0 || k <= 0 || k > T) return -1;
     memset(Y, 0, sizeof(double) * (size_t)B * T * d);
     int failed = 0;
@@ -300,7 +313,7 @@ int oracle_forward_indices(int B, int T, int d, int H, int hp, int k, const doub
                 }
             }
             head_forward(&s, T, Xb, Ibh, Wq + IDX3(h, 0, 0, d, hp), Wk + IDX3(h, 0, 0, d, hp),
-                         Wv + IDX3(h, 0, 0, d, hp), Wo + IDX3(h, 0, 0, hp, d), rope);
+                         Wv + IDX3(h, 0, 0, d, hp), Wo + IDX3(h, 0, 0, hp, d), rope, window);
             /* X^o = diag(r^topk) A W^o;  Y_{I_i} += X^o_i  (Eq. mosa_mha sums the heads) */
             for (int i = 0; i < k; ++i)
                 for (int c = 0; c < d; ++c) {
@@ -311,6 +324,21 @@ int oracle_forward_indices(int B, int T, int d, int H, int hp, int k, const doub
             head_state_free(&s);
         }
     return failed ? -1 : 0;
+}
+
+/* Forward of the layer with the token sets fixed by the caller.
+ * I [B,H,k]; if r_sel_in is non-NULL it is used as r^topk (the fixed-sparse
+ * special case of Sec. 3.1 passes ones), otherwise r^topk = sigma(X W^r)[I]
+ * is computed, which keeps W^r differentiable with TopK held constant.
+ * Y [B,T,d] is overwritten: Y[b] = sum_h scatter(diag(r^topk) A W^o).
+ * Returns 0 or -1. */
+int oracle_forward_indices(int B, int T, int d, int H, int hp, int k, const double *X,
+                           const double *Wr, const double *Wq, const double *Wk,
+                           const double *Wv, const double *Wo, const int32_t *I,
+                           const double *r_sel_in, double *Y, const unsigned char *bsel,
+                           const unsigned char *hsel, int rope) {
+    return forward_units(B, T, d, H, hp, k, X, Wr, Wq, Wk, Wv, Wo, I, r_sel_in, Y, bsel, hsel,
+                         rope, 0);
 }
 
 /* Full forward: router -> TopK -> heads -> sum (Sec. 2.2, Eq. mosa_mha).
@@ -363,14 +391,19 @@ int oracle_forward(int B, int T, int d, int H, int hp, int k, const double *X,
  *   dW^r     += X^s^T dlogit
  *   dX[I]    += dQ W^Q^T + dK W^K^T + dV W^V^T + dlogit W^r^T
  * Returns 0 or -1. */
-int oracle_backward(int B, int T, int d, int H, int hp, int k, const double *X,
-                    const double *Wr, const double *Wq, const double *Wk, const double *Wv,
-                    const double *Wo, const int32_t *I, const double *dY, double *dX,
-                    double *dWr, double *dWq, double *dWk, double *dWv, double *dWo,
-                    const unsigned char *bsel, const unsigned char *hsel, int rope) {
+/* The chain rule above for heads on fixed token sets.  With `unit_scores`
+ * the heads have no router (r = 1, Sec. 2.1): the dr, dlogit and W^r terms
+ * are absent and dWr / Wr are not touched (may be NULL).  `window` as in
+ * head_forward. */
+static int backward_units(int B, int T, int d, int H, int hp, int k, const double *X,
+                          const double *Wr, const double *Wq, const double *Wk,
+                          const double *Wv, const double *Wo, const int32_t *I,
+                          const double *dY, double *dX, double *dWr, double *dWq, double *dWk,
+                          double *dWv, double *dWo, const unsigned char *bsel,
+                          const unsigned char *hsel, int rope, int unit_scores, int window) {
     if (B <= 0 || T <= 0 || d <= 0 || H <= 0 || hp <= 0 || k <= 0 || k > T) return -1;
     memset(dX, 0, sizeof(double) * (size_t)B * T * d);
-    memset(dWr, 0, sizeof(double) * (size_t)d * H);
+    if (!unit_scores) memset(dWr, 0, sizeof(double) * (size_t)d * H);
     memset(dWq, 0, sizeof(double) * (size_t)H * d * hp);
     memset(dWk, 0, sizeof(double) * (size_t)H * d * hp);
     memset(dWv, 0, sizeof(double) * (size_t)H * d * hp);
@@ -405,11 +438,12 @@ int oracle_backward(int B, int T, int d, int H, int hp, int k, const double *X,
             double *dXb = dX + IDX3(b, 0, 0, T, d);
             const int32_t *Ibh = I + IDX3(b, h, 0, H, k);
             for (int i = 0; i < k; ++i) {
+                if (unit_scores) { rs[i] = 1.0; continue; }
                 double logit = 0.0;
                 for (int c = 0; c < d; ++c) logit += Xb[IDX2(Ibh[i], c, d)] * Wr[IDX2(c, h, H)];
                 rs[i] = sigmoid(logit);
             }
-            head_forward(&s, T, Xb, Ibh, Wq_h, Wk_h, Wv_h, Wo_h, rope);
+            head_forward(&s, T, Xb, Ibh, Wq_h, Wk_h, Wv_h, Wo_h, rope, window);
             /* dX^o = dY[I] */
             for (int i = 0; i < k; ++i)
                 for (int c = 0; c < d; ++c) dXo[IDX2(i, c, d)] = dYb[IDX2(Ibh[i], c, d)];
@@ -470,8 +504,9 @@ int oracle_backward(int B, int T, int d, int H, int hp, int k, const double *X,
                     rope_rotate(dQ + IDX2(i, 0, hp), hp, Ibh[i], -1);
                     rope_rotate(dK + IDX2(i, 0, hp), hp, Ibh[i], -1);
                 }
-            /* dlogit = dr o r o (1 - r) */
-            for (int i = 0; i < k; ++i) dlogit[i] = dr[i] * rs[i] * (1.0 - rs[i]);
+            /* dlogit = dr o r o (1 - r); no router term for heads without one */
+            for (int i = 0; i < k; ++i)
+                dlogit[i] = unit_scores ? 0.0 : dr[i] * rs[i] * (1.0 - rs[i]);
             /* dW^{Q,K,V} += X^s^T d{Q,K,V};  dW^r[:,h] += X^s^T dlogit */
             for (int c = 0; c < d; ++c) {
                 for (int p = 0; p < hp; ++p) {
@@ -489,6 +524,7 @@ int oracle_backward(int B, int T, int d, int H, int hp, int k, const double *X,
                     #pragma omp atomic
                     dWv_h[IDX2(c, p, hp)] += av;
                 }
+                if (unit_scores) continue;
                 double ar = 0.0;
                 for (int i = 0; i < k; ++i) ar += s.Xs[IDX2(i, c, d)] * dlogit[i];
                 #pragma omp atomic
@@ -497,7 +533,7 @@ int oracle_backward(int B, int T, int d, int H, int hp, int k, const double *X,
             /* dX[I] += dQ W^Q^T + dK W^K^T + dV W^V^T + dlogit W^r[:,h]^T */
             for (int i = 0; i < k; ++i)
                 for (int c = 0; c < d; ++c) {
-                    double acc = dlogit[i] * Wr[IDX2(c, h, H)];
+                    double acc = unit_scores ? 0.0 : dlogit[i] * Wr[IDX2(c, h, H)];
                     for (int p = 0; p < hp; ++p)
                         acc += dQ[IDX2(i, p, hp)] * Wq_h[IDX2(c, p, hp)] +
                                dK[IDX2(i, p, hp)] * Wk_h[IDX2(c, p, hp)] +
@@ -511,4 +547,65 @@ int oracle_backward(int B, int T, int d, int H, int hp, int k, const double *X,
         head_state_free(&s);
     }
     return failed ? -1 : 0;
+}
+
+/* Backward of the layer for the token sets I: the chain rule above with
+ * r^topk = sigma(X W^r)[I].  All outputs are overwritten.  Returns 0 or -1. */
+int oracle_backward(int B, int T, int d, int H, int hp, int k, const double *X,
+                    const double *Wr, const double *Wq, const double *Wk, const double *Wv,
+                    const double *Wo, const int32_t *I, const double *dY, double *dX,
+                    double *dWr, double *dWq, double *dWk, double *dWv, double *dWo,
+                    const unsigned char *bsel, const unsigned char *hsel, int rope) {
+    return backward_units(B, T, d, H, hp, k, X, Wr, Wq, Wk, Wv, Wo, I, dY, dX, dWr, dWq, dWk,
+                          dWv, dWo, bsel, hsel, rope, 0, 0);
+}
+
+/* I [B,H,T] = 0..T-1 for every (b,h): a dense head sees every token. */
+static int32_t *all_tokens(int B, int H, int T) {
+    int32_t *I = (int32_t *)malloc(sizeof(int32_t) * (size_t)B * H * T);
+    if (!I) return NULL;
+    for (size_t u = 0; u < (size_t)B * H; ++u)
+        for (int t = 0; t < T; ++t) I[u * T + t] = t;
+    return I;
+}
+
+/* Dense heads of a hybrid layer (Sec. 2.2, hybridization): multi-head
+ * attention of Sec. 2.1, Eq. (mha), Y[b] = sum_h Attention(X W^Q_h, X W^K_h,
+ * X W^V_h, M) W^O_h over all T tokens, causal M, no router; window > 0 makes
+ * them the local heads of Sec. 3.4 (same block of `window` positions only).
+ * RoPE, if on, at the positions 0..T-1.  Y is overwritten.  Returns 0 or -1. */
+int oracle_dense_forward(int B, int T, int d, int H, int hp, int window, const double *X,
+                         const double *Wq, const double *Wk, const double *Wv,
+                         const double *Wo, double *Y, const unsigned char *bsel,
+                         const unsigned char *hsel, int rope) {
+    if (B <= 0 || T <= 0 || H <= 0 || window < 0) return -1;
+    int32_t *I = all_tokens(B, H, T);
+    double *ones = (double *)malloc(sizeof(double) * (size_t)B * H * T);
+    int rc = -1;
+    if (I && ones) {
+        for (size_t i = 0; i < (size_t)B * H * T; ++i) ones[i] = 1.0;
+        rc = forward_units(B, T, d, H, hp, T, X, NULL, Wq, Wk, Wv, Wo, I, ones, Y, bsel, hsel,
+                           rope, window);
+    }
+    free(I);
+    free(ones);
+    return rc;
+}
+
+/* Gradients of sum(Y * dY) for the dense (or local) heads above: dX, dW^Q,
+ * dW^K, dW^V, dW^O (overwritten), by the chain rule of oracle_backward with
+ * r = 1 and no router terms.  Returns 0 or -1. */
+int oracle_dense_backward(int B, int T, int d, int H, int hp, int window, const double *X,
+                          const double *Wq, const double *Wk, const double *Wv,
+                          const double *Wo, const double *dY, double *dX, double *dWq,
+                          double *dWk, double *dWv, double *dWo, const unsigned char *bsel,
+                          const unsigned char *hsel, int rope) {
+    if (B <= 0 || T <= 0 || H <= 0 || window < 0) return -1;
+    int32_t *I = all_tokens(B, H, T);
+    int rc = -1;
+    if (I)
+        rc = backward_units(B, T, d, H, hp, T, X, NULL, Wq, Wk, Wv, Wo, I, dY, dX, NULL, dWq, dWk,
+                            dWv, dWo, bsel, hsel, rope, 1, window);
+    free(I);
+    return rc;
 }

@@ -126,6 +126,22 @@ def make_inputs(cfg: MosaConfig, seed: int | None = None, plant: bool = True,
     return {"X": X, "Wr": Wr, "Wq": Wq, "Wk": Wk, "Wv": Wv, "Wo": Wo, "dY": dY}
 
 
+def make_dense_weights(cfg: MosaConfig, H_dense: int, seed: int | None = None
+                       ) -> dict[str, np.ndarray]:
+    """Weights of the dense (or local) heads of a hybrid layer (Sec. 2.2,
+    hybridization): D_q, D_k, D_v ~ N(0,1/d) [H_dense,d,hp] and D_o ~ N(0,1/d)
+    [H_dense,hp,d], rounded to ``cfg.dtype``; one generator seeded with
+    ``cfg.seed + 1000`` (or ``seed``), one draw per tensor in that order."""
+    rng = np.random.default_rng(cfg.seed + 1000 if seed is None else seed)
+    d, hp = cfg.d, cfg.hp
+    s = 1.0 / np.sqrt(d)
+    out = {}
+    for name, shape in (("Dq", (H_dense, d, hp)), ("Dk", (H_dense, d, hp)),
+                        ("Dv", (H_dense, d, hp)), ("Do", (H_dense, hp, d))):
+        out[name] = to_storage(rng.standard_normal(shape, dtype=np.float32) * s, cfg.dtype)
+    return out
+
+
 def plant_margin(X0: np.ndarray, Wr: np.ndarray, k: int, delta: float,
                  first_token: bool = False) -> np.ndarray:
     """Return X0 + G pinv(W_r) where G raises the k highest logits of every

@@ -476,3 +476,98 @@ def test_rope_changes_only_through_positions():
         r = torch.sigmoid(Xt @ torch.tensor(x["Wr"][:, h], dtype=torch.float64))
         ref += r[..., None] * (a @ torch.tensor(x["Wo"][h], dtype=torch.float64))
     np.testing.assert_allclose(Y, ref.numpy(), rtol=1e-10, atol=1e-12)
+
+
+# ---------------------------------- hybrid layers (Sec. 2.2 hybridization, Sec. 3.4) ----
+
+def dense_heads_sdpa(X, Dq, Dk, Dv, Do, window=0, rope=False):
+    """Eq. (mha) over all T tokens with torch's SDPA and an explicit boolean
+    mask: query i sees key j iff j <= i and, for a window w > 0, floor(i/w) =
+    floor(j/w).  float64 tensors in and out, differentiable."""
+    T = X.shape[1]
+    pos = torch.arange(T)
+    allowed = pos[:, None] >= pos[None, :]
+    if window:
+        allowed = allowed & ((pos[:, None] // window) == (pos[None, :] // window))
+    Y = torch.zeros_like(X)
+    for h in range(Dq.shape[0]):
+        q, kk, v = X @ Dq[h], X @ Dk[h], X @ Dv[h]
+        if rope:
+            q, kk = rope_complex(q, pos), rope_complex(kk, pos)
+        Y = Y + F.scaled_dot_product_attention(q, kk, v, attn_mask=allowed) @ Do[h]
+    return Y
+
+
+def dense_inputs(B, T, d, H, hp, Hd, seed):
+    cfg, x = small(B, T, d, H, hp, max(1, T // 4), seed=seed)
+    x.update(W.make_dense_weights(cfg, Hd))
+    return cfg, x
+
+
+@pytest.mark.parametrize("window,rope", [(0, False), (0, True), (4, False), (5, True),
+                                         (18, False)])
+def test_dense_heads_match_sdpa_forward_and_autograd(window, rope):
+    # T = 18 with w = 4 or 5 leaves a shorter last block
+    _, x = dense_inputs(2, 18, 12, 2, 8, 3, seed=50 + window)
+    D = [x[n] for n in ("Dq", "Dk", "Dv", "Do")]
+    ts = {n: torch.tensor(x[n], dtype=torch.float64, requires_grad=(n != "dY"))
+          for n in ("X", "Dq", "Dk", "Dv", "Do", "dY")}
+    Y = dense_heads_sdpa(ts["X"], ts["Dq"], ts["Dk"], ts["Dv"], ts["Do"], window, rope)
+    Yo = oracle.dense_forward(x["X"], *D, window=window, rope=rope)
+    np.testing.assert_allclose(Yo, Y.detach().numpy(), rtol=1e-11, atol=1e-12)
+    (Y * ts["dY"]).sum().backward()
+    g = oracle.dense_backward(x["X"], *D, dY=x["dY"], window=window, rope=rope)
+    for name, tname in (("dX", "X"), ("dWq", "Dq"), ("dWk", "Dk"), ("dWv", "Dv"),
+                        ("dWo", "Do")):
+        np.testing.assert_allclose(g[name], ts[tname].grad.numpy(), rtol=1e-10, atol=1e-11,
+                                   err_msg=name)
+
+
+def test_local_window_one_is_the_value_path():
+    # w = 1: each token sees only itself, softmax of one entry is 1, so
+    # Y = sum_h X D_v[h] D_o[h] whatever the queries and keys
+    _, x = dense_inputs(2, 11, 8, 1, 4, 3, seed=60)
+    Y = oracle.dense_forward(x["X"], x["Dq"], x["Dk"], x["Dv"], x["Do"], window=1, rope=True)
+    X64 = x["X"].astype(np.float64)
+    ref = sum(X64 @ x["Dv"][h].astype(np.float64) @ x["Do"][h].astype(np.float64)
+              for h in range(3))
+    np.testing.assert_allclose(Y, ref, rtol=1e-12, atol=1e-13)
+
+
+def test_local_heads_are_blockwise_dense_heads_with_rope():
+    # RoPE scores depend on position differences only, so local heads at the
+    # original positions equal dense heads run on each block as its own
+    # sequence from position 0 (the form the CUDA library computes them in)
+    B, T, w = 2, 24, 8
+    _, x = dense_inputs(B, T, 16, 1, 8, 2, seed=61)
+    D = [x[n] for n in ("Dq", "Dk", "Dv", "Do")]
+    Y = oracle.dense_forward(x["X"], *D, window=w, rope=True)
+    Xb = x["X"].reshape(B * T // w, w, -1)
+    Yb = oracle.dense_forward(Xb, *D, window=0, rope=True).reshape(B, T, -1)
+    np.testing.assert_allclose(Y, Yb, rtol=1e-10, atol=1e-12)
+    g = oracle.dense_backward(x["X"], *D, dY=x["dY"], window=w, rope=True)
+    gb = oracle.dense_backward(Xb, *D, dY=x["dY"].reshape(B * T // w, w, -1), rope=True)
+    np.testing.assert_allclose(g["dX"], gb["dX"].reshape(B, T, -1), rtol=1e-10, atol=1e-12)
+    for n in ("dWq", "dWk", "dWv", "dWo"):
+        np.testing.assert_allclose(g[n], gb[n], rtol=1e-10, atol=1e-12, err_msg=n)
+    # and they differ from dense heads over the whole sequence
+    assert np.abs(Y - oracle.dense_forward(x["X"], *D, rope=True)).max() > 1e-3
+
+
+@pytest.mark.parametrize("window,rope", [(0, False), (6, True)])
+def test_hybrid_layer_matches_torch_restatement(window, rope):
+    cfg, x = dense_inputs(2, 24, 12, 3, 8, 2, seed=62 + window)
+    Y, I, _, _ = oracle.hybrid_forward(x["X"], *weights(x), x["Dq"], x["Dk"], x["Dv"], x["Do"],
+                                       k=cfg.k, window=window, rope=rope)
+    names = ("X", "Wr", "Wq", "Wk", "Wv", "Wo", "Dq", "Dk", "Dv", "Do")
+    ts = {n: torch.tensor(x[n], dtype=torch.float64, requires_grad=True) for n in names}
+    Yt = (torch_restatement(ts["X"], ts["Wr"], ts["Wq"], ts["Wk"], ts["Wv"], ts["Wo"],
+                            torch.tensor(I), rope=rope) +
+          dense_heads_sdpa(ts["X"], ts["Dq"], ts["Dk"], ts["Dv"], ts["Do"], window, rope))
+    np.testing.assert_allclose(Y, Yt.detach().numpy(), rtol=1e-11, atol=1e-12)
+    (Yt * torch.tensor(x["dY"], dtype=torch.float64)).sum().backward()
+    g = oracle.hybrid_backward(x["X"], *weights(x), x["Dq"], x["Dk"], x["Dv"], x["Do"], I=I,
+                               dY=x["dY"], window=window, rope=rope)
+    for n in names:
+        np.testing.assert_allclose(g["d" + n], ts[n].grad.numpy(), rtol=1e-10, atol=1e-11,
+                                   err_msg=n)

@@ -158,6 +158,54 @@ mosa_status mosa_backward(const mosa_shape *shape, const void *X, const void *W_
                           float *dW_r, float *dW_q, float *dW_k, float *dW_v, float *dW_o,
                           void *workspace, size_t workspace_bytes, void *stream);
 
+/* Hybrid layer (Sec. 2.2, hybridization; Sec. 3.4): the MoSA heads of
+ * `sparse` plus H_dense dense heads, all summed into one Y (Eq. mha).  A
+ * dense head attends causally over all T tokens with no router and no
+ * scaling (Sec. 2.1).  window = w > 0 makes them local heads for long
+ * sequences (Sec. 3.4): token i sees token j iff j <= i and both lie in the
+ * same block of w positions (the block pattern of fixed sparse attention;
+ * T % w == 0, else MOSA_ERR_UNSUPPORTED).  window = 0 (or T) is the dense
+ * case.  Dense and local heads use the head size hp, the dtype and the rope
+ * setting of `sparse` (positions 0..T-1); first_token applies to the MoSA
+ * heads only.  H_dense = 0 is a plain MoSA layer. */
+typedef struct {
+    mosa_shape sparse;  /* the MoSA heads */
+    int32_t H_dense;    /* >= 0 */
+    int32_t window;     /* 0 <= window <= T */
+} mosa_hybrid_shape;
+
+/* Workspace bytes of a hybrid forward and its backward; 0 if the shape is
+ * invalid or unsupported.  256-byte aligned, as for mosa_workspace_bytes;
+ * mosa_check_status(&shape->sparse, workspace, stream) reports for both
+ * head groups. */
+size_t mosa_hybrid_workspace_bytes(const mosa_hybrid_shape *shape);
+
+/* Forward of the hybrid layer.  Arguments as mosa_forward, plus the dense
+ * heads' weights D_q, D_k, D_v [H_dense,d,hp] and D_o [H_dense,hp,d] in the
+ * storage dtype (may be NULL when H_dense = 0).  Y [B,T,d] fp32 is
+ * overwritten with the sum of both head groups; I, r_sel, r_full are the MoSA
+ * heads'.  Returns as mosa_forward. */
+mosa_status mosa_hybrid_forward(const mosa_hybrid_shape *shape, const void *X, const void *W_r,
+                                const void *W_q, const void *W_k, const void *W_v,
+                                const void *W_o, const void *D_q, const void *D_k,
+                                const void *D_v, const void *D_o, float *Y, int32_t *I,
+                                float *r_sel, float *r_full, void *workspace,
+                                size_t workspace_bytes, void *stream);
+
+/* Backward of the hybrid layer; must follow mosa_hybrid_forward on the same
+ * stream with the same shape, inputs and workspace.  dX [B,T,d] receives the
+ * sum over both head groups; dW_r .. dW_o are the MoSA heads' gradients (as
+ * mosa_backward), dD_q, dD_k, dD_v [H_dense,d,hp] and dD_o [H_dense,hp,d] the
+ * dense heads' (fp32, overwritten).  Returns as mosa_backward. */
+mosa_status mosa_hybrid_backward(const mosa_hybrid_shape *shape, const void *X, const void *W_r,
+                                 const void *W_q, const void *W_k, const void *W_v,
+                                 const void *W_o, const void *D_q, const void *D_k,
+                                 const void *D_v, const void *D_o, const int32_t *I,
+                                 const float *r_sel, const void *dY, float *dX, float *dW_r,
+                                 float *dW_q, float *dW_k, float *dW_v, float *dW_o, float *dD_q,
+                                 float *dD_k, float *dD_v, float *dD_o, void *workspace,
+                                 size_t workspace_bytes, void *stream);
+
 /* TopK alone (Sec. 2.2): for each of `rows` rows of T fp32 scores, the k
  * largest (ties: lower index first), written ascending by index.
  *   scores [rows,T] fp32 input; I [rows,k] int32 and r_sel [rows,k] fp32 outputs.

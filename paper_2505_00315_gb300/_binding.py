@@ -26,7 +26,8 @@ MOSA_BF16 = 1
 EXPORTED = ("mosa_status_string", "mosa_workspace_bytes", "mosa_forward",
             "mosa_forward_with_indices", "mosa_backward", "mosa_topk", "mosa_check_status",
             "mosa_kernel_launches", "mosa_profile_stages", "mosa_profile_read",
-            "mosa_stage_name", "mosa_stage_engine", "mosa_route_noalloc", "mosa_adaptive_k")
+            "mosa_stage_name", "mosa_stage_engine", "mosa_route_noalloc", "mosa_adaptive_k",
+            "mosa_hybrid_workspace_bytes", "mosa_hybrid_forward", "mosa_hybrid_backward")
 
 
 class MosaShape(ctypes.Structure):
@@ -41,6 +42,13 @@ class MosaShape(ctypes.Structure):
     def astuple(self):
         return (self.B, self.T, self.d, self.H, self.hp, self.k, self.dtype, self.first_token,
                 self.rope)
+
+
+class MosaHybridShape(ctypes.Structure):
+    """mosa_hybrid_shape: the MoSA heads' shape plus H_dense dense heads
+    (window = 0) or local heads attending within blocks of ``window`` tokens
+    (Sec. 2.2 hybridization, Sec. 3.4)."""
+    _fields_ = [("sparse", MosaShape), ("H_dense", ctypes.c_int32), ("window", ctypes.c_int32)]
 
 
 class MosaError(RuntimeError):
@@ -98,6 +106,13 @@ def load(build_if_missing: bool = True) -> ctypes.CDLL:
         L.mosa_stage_engine.restype = i32
         L.mosa_adaptive_k.argtypes = [i32, i32]
         L.mosa_adaptive_k.restype = i32
+        hp_ = ctypes.POINTER(MosaHybridShape)
+        L.mosa_hybrid_workspace_bytes.argtypes = [hp_]
+        L.mosa_hybrid_workspace_bytes.restype = sz
+        L.mosa_hybrid_forward.argtypes = [hp_] + [vp] * 10 + [vp] * 4 + [vp, sz, vp]
+        L.mosa_hybrid_forward.restype = ctypes.c_int
+        L.mosa_hybrid_backward.argtypes = [hp_] + [vp] * 10 + [vp, vp, vp] + [vp] * 10 + [vp, sz, vp]
+        L.mosa_hybrid_backward.restype = ctypes.c_int
         _lib = L
         return L
 
@@ -350,3 +365,81 @@ def mosa_route_noalloc(X, W_r, k: int, hp: int = 64, out=None, stream=None,
                                    _stream(stream))
     _check(rc, "mosa_route_noalloc")
     return I, rs
+
+
+# ------------------------------------------------------------ hybrid layers
+
+def make_hybrid_shape(X, W_q, k: int, H_dense: int, window: int = 0,
+                      first_token: bool = False, rope: bool = False) -> MosaHybridShape:
+    return MosaHybridShape(make_shape(X, W_q, k, first_token, rope), int(H_dense), int(window))
+
+
+def mosa_hybrid_workspace_bytes(shape: MosaHybridShape) -> int:
+    return int(load().mosa_hybrid_workspace_bytes(ctypes.byref(shape)))
+
+
+def alloc_hybrid_workspace(shape: MosaHybridShape, device=None):
+    """A torch uint8 device buffer of mosa_hybrid_workspace_bytes(shape) bytes."""
+    torch = _torch()
+    n = mosa_hybrid_workspace_bytes(shape)
+    if n == 0:
+        raise MosaError(MOSA_ERR_INVALID_ARG, "mosa_hybrid_workspace_bytes")
+    return torch.empty(n, dtype=torch.uint8, device=device or "cuda")
+
+
+def mosa_hybrid_forward(X, W_r, W_q, W_k, W_v, W_o, D_q, D_k, D_v, D_o, k: int,
+                        window: int = 0, workspace=None, out=None, stream=None,
+                        first_token: bool = False, rope: bool = False):
+    """Hybrid layer forward (Sec. 2.2 hybridization, Sec. 3.4): the MoSA heads
+    plus the dense heads D_q, D_k, D_v [H_dense,d,hp], D_o [H_dense,hp,d]
+    (local heads with ``window`` > 0), summed into Y.  Returns
+    (Y, I, r_sel, workspace)."""
+    torch = _torch()
+    shape = make_hybrid_shape(X, W_q, k, D_q.shape[0], window, first_token, rope)
+    _same(X, ("W_r", W_r), ("W_q", W_q), ("W_k", W_k), ("W_v", W_v), ("W_o", W_o),
+          ("D_q", D_q), ("D_k", D_k), ("D_v", D_v), ("D_o", D_o))
+    B, T, d, H = X.shape[0], X.shape[1], X.shape[2], W_q.shape[0]
+    dev = X.device
+    out = out or {}
+    Y = out.get("Y") if out.get("Y") is not None else torch.empty((B, T, d), dtype=torch.float32, device=dev)
+    I = out.get("I") if out.get("I") is not None else torch.empty((B, H, k), dtype=torch.int32, device=dev)
+    rs = out.get("r_sel") if out.get("r_sel") is not None else torch.empty((B, H, k), dtype=torch.float32, device=dev)
+    if workspace is None:
+        workspace = alloc_hybrid_workspace(shape, dev)
+    rc = load().mosa_hybrid_forward(
+        ctypes.byref(shape), _dev(X, "X"), _dev(W_r, "W_r"), _dev(W_q, "W_q"), _dev(W_k, "W_k"),
+        _dev(W_v, "W_v"), _dev(W_o, "W_o"), _dev(D_q, "D_q"), _dev(D_k, "D_k"), _dev(D_v, "D_v"),
+        _dev(D_o, "D_o"), _dev(Y, "Y", torch.float32), _dev(I, "I", torch.int32),
+        _dev(rs, "r_sel", torch.float32), None, _dev(workspace, "workspace"), workspace.numel(),
+        _stream(stream))
+    _check(rc, "mosa_hybrid_forward")
+    return Y, I, rs, workspace
+
+
+def mosa_hybrid_backward(X, W_r, W_q, W_k, W_v, W_o, D_q, D_k, D_v, D_o, I, r_sel, dY,
+                         workspace, window: int = 0, out=None, stream=None,
+                         rope: bool = False):
+    """Hybrid layer backward; returns a dict with dX (both head groups),
+    dW_r, dW_q, dW_k, dW_v, dW_o (MoSA heads) and dD_q, dD_k, dD_v, dD_o
+    (dense heads), fp32.  ``window`` and ``rope`` must match the forward's."""
+    torch = _torch()
+    shape = make_hybrid_shape(X, W_q, I.shape[-1], D_q.shape[0], window, rope=rope)
+    _same(X, ("W_r", W_r), ("W_q", W_q), ("W_k", W_k), ("W_v", W_v), ("W_o", W_o),
+          ("D_q", D_q), ("D_k", D_k), ("D_v", D_v), ("D_o", D_o), ("dY", dY))
+    dev = X.device
+    g = dict(out or {})
+    f32 = torch.float32
+    for name, like in (("dX", X), ("dW_r", W_r), ("dW_q", W_q), ("dW_k", W_k), ("dW_v", W_v),
+                       ("dW_o", W_o), ("dD_q", D_q), ("dD_k", D_k), ("dD_v", D_v),
+                       ("dD_o", D_o)):
+        if g.get(name) is None:
+            g[name] = torch.empty(like.shape, dtype=f32, device=dev)
+    grads = [_dev(g[n], n, f32) for n in ("dX", "dW_r", "dW_q", "dW_k", "dW_v", "dW_o", "dD_q",
+                                          "dD_k", "dD_v", "dD_o")]
+    rc = load().mosa_hybrid_backward(
+        ctypes.byref(shape), _dev(X, "X"), _dev(W_r, "W_r"), _dev(W_q, "W_q"), _dev(W_k, "W_k"),
+        _dev(W_v, "W_v"), _dev(W_o, "W_o"), _dev(D_q, "D_q"), _dev(D_k, "D_k"), _dev(D_v, "D_v"),
+        _dev(D_o, "D_o"), _dev(I, "I", torch.int32), _dev(r_sel, "r_sel", f32), _dev(dY, "dY"),
+        *grads, _dev(workspace, "workspace"), workspace.numel(), _stream(stream))
+    _check(rc, "mosa_hybrid_backward")
+    return g

@@ -128,6 +128,7 @@ struct Dims {
     bool bf16;
     bool first_token;   // token 0 always kept, k-1 more by score (Sec. 3.2)
     bool rope;          // rotary position encoding of Q and K (Sec. 2.2)
+    bool accumulate;    // Y (forward) and dX (backward) are added into, not overwritten
     long long rows() const { return (long long)H * B * k; }
     size_t esize() const { return bf16 ? 2 : 4; }
 };

@@ -70,6 +70,10 @@ cudaError_t launch_indices_to_rows(const Dims &dm, const int32_t *I, const float
                                    int32_t *gidx, float *rsel_hm, uint32_t *status,
                                    cudaStream_t stream);
 
+// Dense heads: gidx[(h*B+b)*k + i] = b*T + i (k = T) and rsel_hm = 1.
+cudaError_t launch_dense_rows(const Dims &dm, int32_t *gidx, float *rsel_hm,
+                              cudaStream_t stream);
+
 // F3: Q, K, V = X[I] W_{q,k,v}[h].
 cudaError_t launch_qkv(const Dims &dm, const void *X, const void *Wq, const void *Wk,
                        const void *Wv, const Saved &sv, cudaStream_t stream);

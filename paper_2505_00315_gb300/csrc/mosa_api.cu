@@ -174,18 +174,22 @@ mosa_status forward_tc(const Dims &dm, const void *X, const void *W_r, const voi
                        const void *W_k, const void *W_v, const void *W_o, float *Y, int32_t *I,
                        float *r_sel, float *rf, bool route, const int32_t *I_in,
                        const float *rsel_in, const Saved &sv, cudaStream_t s, DevResources &r) {
-    MOSA_TRY(cudaMemsetAsync(sv.status, 0, sizeof(uint32_t), s));
+    // A call that adds into Y continues the status word of the call that wrote it.
+    if (!dm.accumulate) MOSA_TRY(cudaMemsetAsync(sv.status, 0, sizeof(uint32_t), s));
     const size_t ny = (size_t)dm.B * dm.T * dm.d;
     if (route) {
         StageScope st_(kStageRouter, s);
         MOSA_TRY(launch_router_auto(dm, X, W_r, rf, sv.status, s));
     }
     MOSA_TRY(link(s, r.side, r.ev[0]));
-    MOSA_TRY(cudaMemsetAsync(Y, 0, sizeof(float) * ny, r.side));
+    if (!dm.accumulate) MOSA_TRY(cudaMemsetAsync(Y, 0, sizeof(float) * ny, r.side));
     if (route) {
         StageScope st_(kStageSelect, s);
         MOSA_TRY(launch_select(dm.B * dm.H, dm.T, dm.k, rf, I, r_sel, dm.B, dm.H, sv.gidx,
                                sv.rsel, s, dm.first_token));
+    } else if (I_in == nullptr) {
+        StageScope st_(kStageSelect, s);
+        MOSA_TRY(launch_dense_rows(dm, sv.gidx, sv.rsel, s));
     } else {
         StageScope st_(kStageSelect, s);
         MOSA_TRY(launch_indices_to_rows(dm, I_in, rsel_in, sv.gidx, sv.rsel, sv.status, s));
@@ -228,7 +232,7 @@ mosa_status backward_tc(const Dims &dm, const void *X, const void *W_r, const vo
         // The fused kernel (G, row terms, attention backward) holds a whole SM
         // per CTA, so nothing runs beside it; dX, dW and dW_o then share the GPU.
         MOSA_TRY(tc_transpose_wr(dm, W_r, sv, t));
-        MOSA_TRY(cudaMemsetAsync(dX, 0, sizeof(float) * nx, t));
+        if (!dm.accumulate) MOSA_TRY(cudaMemsetAsync(dX, 0, sizeof(float) * nx, t));
         MOSA_TRY(cudaEventRecord(r.ev[1], t));  // dX zeroed, W_r transposed
         {
             StageScope st_(kStageBwdUnit, s);
@@ -257,7 +261,7 @@ mosa_status backward_tc(const Dims &dm, const void *X, const void *W_r, const vo
         MOSA_TRY(tc_out_bwd_w(dm, dY, sv, dW_o, t));
     }
     MOSA_TRY(tc_transpose_wr(dm, W_r, sv, t));
-    MOSA_TRY(cudaMemsetAsync(dX, 0, sizeof(float) * nx, t));
+    if (!dm.accumulate) MOSA_TRY(cudaMemsetAsync(dX, 0, sizeof(float) * nx, t));
     MOSA_TRY(cudaEventRecord(r.ev[1], t));  // dX zeroed, W_r transposed
     {
         StageScope st_(kStageOutBwd, s);
@@ -282,6 +286,159 @@ mosa_status backward_tc(const Dims &dm, const void *X, const void *W_r, const vo
     return MOSA_OK;
 }
 
+// The launch sequences of the three calls, on stream s.  `res` is the side
+// stream of the tensor-core path (nullptr: the CUDA-core sequence).
+
+// Router, TopK and the heads (mosa_forward).
+mosa_status forward_routed(const Dims &dm, const void *X, const void *W_r, const void *W_q,
+                           const void *W_k, const void *W_v, const void *W_o, float *Y,
+                           int32_t *I, float *r_sel, float *rf, const Saved &sv, cudaStream_t s,
+                           DevResources *res) {
+    if (res != nullptr)
+        return forward_tc(dm, X, W_r, W_q, W_k, W_v, W_o, Y, I, r_sel, rf, true, nullptr, nullptr,
+                          sv, s, *res);
+    MOSA_TRY(cudaMemsetAsync(sv.status, 0, sizeof(uint32_t), s));
+    {
+        StageScope st_(kStageRouter, s);
+        MOSA_TRY(launch_router_auto(dm, X, W_r, rf, sv.status, s));
+    }
+    {
+        StageScope st_(kStageSelect, s);
+        MOSA_TRY(launch_select(dm.B * dm.H, dm.T, dm.k, rf, I, r_sel, dm.B, dm.H, sv.gidx,
+                               sv.rsel, s, dm.first_token));
+    }
+    return forward_heads(dm, X, W_q, W_k, W_v, W_o, Y, sv, s);
+}
+
+// The heads on given token sets (mosa_forward_with_indices); I == nullptr:
+// every token with score 1 (dense heads, k = T).
+mosa_status forward_given(const Dims &dm, const void *X, const void *W_q, const void *W_k,
+                          const void *W_v, const void *W_o, const int32_t *I,
+                          const float *r_sel, float *Y, const Saved &sv, cudaStream_t s,
+                          DevResources *res) {
+    if (res != nullptr)
+        return forward_tc(dm, X, nullptr, W_q, W_k, W_v, W_o, Y, nullptr, nullptr, nullptr, false,
+                          I, r_sel, sv, s, *res);
+    if (!dm.accumulate) MOSA_TRY(cudaMemsetAsync(sv.status, 0, sizeof(uint32_t), s));
+    {
+        StageScope st_(kStageSelect, s);
+        if (I == nullptr)
+            MOSA_TRY(launch_dense_rows(dm, sv.gidx, sv.rsel, s));
+        else
+            MOSA_TRY(launch_indices_to_rows(dm, I, r_sel, sv.gidx, sv.rsel, sv.status, s));
+    }
+    return forward_heads(dm, X, W_q, W_k, W_v, W_o, Y, sv, s);
+}
+
+// The backward (mosa_backward).
+mosa_status backward_all(const Dims &dm, const void *X, const void *W_r, const void *W_q,
+                         const void *W_k, const void *W_v, const void *W_o, const void *dY,
+                         float *dX, float *dW_r, float *dW_q, float *dW_k, float *dW_v,
+                         float *dW_o, const Saved &sv, cudaStream_t s, DevResources *res) {
+    if (res != nullptr)
+        return backward_tc(dm, X, W_r, W_q, W_k, W_v, W_o, dY, dX, dW_r, dW_q, dW_k, dW_v, dW_o,
+                           sv, s, *res);
+    {
+        StageScope st_(kStageOutBwd, s);
+        MOSA_TRY(launch_out_bwd(dm, W_o, dY, sv, dW_o, s));
+    }
+    {
+        StageScope st_(kStageAttnBwd, s);
+        MOSA_TRY(launch_attn_bwd(dm, sv, s));
+        if (dm.rope) MOSA_TRY(rope_qk(dm, sv, true, s));
+    }
+    {
+        StageScope st_(kStageInBwd, s);
+        MOSA_TRY(launch_in_bwd(dm, W_q, W_k, W_v, W_r, sv, dX, s));
+    }
+    {
+        StageScope st_(kStageWBwd, s);
+        MOSA_TRY(launch_w_bwd(dm, X, sv, dW_q, dW_k, dW_v, dW_r, s));
+    }
+    return MOSA_OK;
+}
+
+// ------------------------------------------------------------ hybrid layers
+// MoSA heads plus dense heads (Sec. 2.2, hybridization) or local heads
+// (Sec. 3.4).  The dense heads run through the given-token-set path with
+// every token and unit scores: with r = 1 the router terms vanish (dlogit =
+// D (1 - r) = 0), so they get a zeroed W_r and a scratch dW_r.  Local heads
+// (causal attention within blocks of w tokens) are dense heads over B*T/w
+// sequences of w tokens, the same rows of X, Y and dX; RoPE scores depend on
+// position differences only, so positions counted from each block's start
+// give the same attention.  The dense heads add into the Y and dX the MoSA
+// heads wrote.
+struct Hybrid {
+    Dims sparse, dense;
+    bool has_dense;
+};
+
+mosa_status check_hybrid(const mosa_hybrid_shape *hs, Hybrid *h) {
+    if (hs == nullptr) return MOSA_ERR_INVALID_ARG;
+    mosa_status st = check_shape(&hs->sparse, &h->sparse);
+    if (st != MOSA_OK) return st;
+    const int T = hs->sparse.T;
+    if (hs->H_dense < 0 || hs->window < 0 || hs->window > T) return MOSA_ERR_INVALID_ARG;
+    h->has_dense = hs->H_dense > 0;
+    h->dense = Dims{};
+    if (!h->has_dense) return MOSA_OK;
+    const int w = hs->window == 0 ? T : hs->window;
+    if (T % w != 0) return MOSA_ERR_UNSUPPORTED;
+    mosa_shape ds = hs->sparse;
+    ds.B = hs->sparse.B * (T / w);
+    ds.T = w;
+    ds.H = hs->H_dense;
+    ds.k = w;
+    ds.first_token = 0;
+    if ((st = check_shape(&ds, &h->dense)) != MOSA_OK) return st;
+    h->dense.accumulate = true;
+    return MOSA_OK;
+}
+
+struct HybridSpace {
+    Saved sparse, dense;
+    void *zero_wr;    // [d, H_dense] zeros in the storage dtype
+    float *dwr;       // [d, H_dense] fp32, discarded
+    size_t zero_wr_bytes;
+};
+
+// Sparse heads' state, then the dense heads' (sharing the status word), then
+// the two W_r stand-ins.  Returns the bytes needed.
+size_t carve_hybrid(const Hybrid &h, char *base, HybridSpace *sp) {
+    Saved ss{}, ds{};
+    const size_t o1 = carve(h.sparse, base, &ss);
+    size_t total = o1;
+    size_t nwr = 0;
+    char *dense_base = base ? base + o1 : nullptr;
+    if (h.has_dense) {
+        const size_t o2 = carve(h.dense, dense_base, &ds);
+        nwr = (size_t)h.dense.d * h.dense.H * h.dense.esize();
+        total = o1 + o2 + align_up(nwr) + align_up(sizeof(float) * h.dense.d * h.dense.H);
+        if (base) {
+            ds.status = ss.status;
+            sp->zero_wr = base + o1 + o2;
+            sp->dwr = (float *)(base + o1 + o2 + align_up(nwr));
+        }
+    }
+    if (base) {
+        sp->sparse = ss;
+        sp->dense = ds;
+        sp->zero_wr_bytes = nwr;
+        if (!h.has_dense) {
+            sp->zero_wr = nullptr;
+            sp->dwr = nullptr;
+        }
+    }
+    return total;
+}
+
+mosa_status check_hybrid_workspace(const Hybrid &h, void *ws, size_t bytes, HybridSpace *sp) {
+    if (ws == nullptr || ((uintptr_t)ws % kAlign) != 0) return MOSA_ERR_WORKSPACE;
+    if (bytes < carve_hybrid(h, nullptr, nullptr)) return MOSA_ERR_WORKSPACE;
+    carve_hybrid(h, (char *)ws, sp);
+    return MOSA_OK;
+}
+
 // ---------------------------------------------------------- graph cache
 // A layer call enqueues about a dozen kernels and memsets; launched one by one
 // from the host that costs tens of microseconds per call.  The first call with
@@ -293,7 +450,8 @@ struct GraphKey {
     int op, device, tc;
     uint32_t mask;
     mosa_shape shape;
-    const void *ptr[18];
+    int extra[2];  // hybrid calls: dense heads, window
+    const void *ptr[28];
     bool operator==(const GraphKey &o) const { return std::memcmp(this, &o, sizeof(GraphKey)) == 0; }
 };
 
@@ -322,15 +480,22 @@ bool graphs_enabled() {
     return v == nullptr || v[0] != '0';
 }
 
+int path_bits(const Dims &dm) {
+    return (use_tc(dm) ? 1 : 0) | (use_fused_forward(dm) ? 2 : 0) | (use_fused_backward(dm) ? 4 : 0);
+}
+
 GraphKey make_key(int op, const Dims &dm, const mosa_shape *shape,
-                  std::initializer_list<const void *> ptrs) {
+                  std::initializer_list<const void *> ptrs, const Dims *dense = nullptr,
+                  int extra0 = 0, int extra1 = 0) {
     GraphKey k;
     std::memset(&k, 0, sizeof(k));
     k.op = op;
     cudaGetDevice(&k.device);
-    k.tc = (use_tc(dm) ? 1 : 0) | (use_fused_forward(dm) ? 2 : 0) | (use_fused_backward(dm) ? 4 : 0);
+    k.tc = path_bits(dm) | (dense ? path_bits(*dense) << 3 : 0);
     k.mask = profile_mask();
     k.shape = *shape;
+    k.extra[0] = extra0;
+    k.extra[1] = extra1;
     int i = 0;
     for (const void *p : ptrs) k.ptr[i++] = p;
     return k;
@@ -425,20 +590,7 @@ mosa_status mosa_forward(const mosa_shape *shape, const void *X, const void *W_r
     float *rf = r_full ? r_full : sv.r_full;
     DevResources *res = use_tc(dm) ? dev_resources() : nullptr;
     auto enqueue = [&](cudaStream_t s) -> mosa_status {
-        if (res != nullptr)
-            return forward_tc(dm, X, W_r, W_q, W_k, W_v, W_o, Y, I, r_sel, rf, true, nullptr,
-                              nullptr, sv, s, *res);
-        MOSA_TRY(cudaMemsetAsync(sv.status, 0, sizeof(uint32_t), s));
-        {
-            StageScope st_(kStageRouter, s);
-            MOSA_TRY(launch_router_auto(dm, X, W_r, rf, sv.status, s));
-        }
-        {
-            StageScope st_(kStageSelect, s);
-            MOSA_TRY(launch_select(dm.B * dm.H, dm.T, dm.k, rf, I, r_sel, dm.B, dm.H, sv.gidx,
-                                   sv.rsel, s, dm.first_token));
-        }
-        return forward_heads(dm, X, W_q, W_k, W_v, W_o, Y, sv, s);
+        return forward_routed(dm, X, W_r, W_q, W_k, W_v, W_o, Y, I, r_sel, rf, sv, s, res);
     };
     const GraphKey key = make_key(0, dm, shape, {X, W_r, W_q, W_k, W_v, W_o, Y, I, r_sel, r_full,
                                                  workspace});
@@ -457,15 +609,7 @@ mosa_status mosa_forward_with_indices(const mosa_shape *shape, const void *X, co
     if ((st = check_workspace(dm, workspace, workspace_bytes, &sv)) != MOSA_OK) return st;
     DevResources *res = use_tc(dm) ? dev_resources() : nullptr;
     auto enqueue = [&](cudaStream_t s) -> mosa_status {
-        if (res != nullptr)
-            return forward_tc(dm, X, nullptr, W_q, W_k, W_v, W_o, Y, nullptr, nullptr, nullptr,
-                              false, I, r_sel, sv, s, *res);
-        MOSA_TRY(cudaMemsetAsync(sv.status, 0, sizeof(uint32_t), s));
-        {
-            StageScope st_(kStageSelect, s);
-            MOSA_TRY(launch_indices_to_rows(dm, I, r_sel, sv.gidx, sv.rsel, sv.status, s));
-        }
-        return forward_heads(dm, X, W_q, W_k, W_v, W_o, Y, sv, s);
+        return forward_given(dm, X, W_q, W_k, W_v, W_o, I, r_sel, Y, sv, s, res);
     };
     const GraphKey key = make_key(1, dm, shape, {X, W_q, W_k, W_v, W_o, I, r_sel, Y, workspace});
     return run_graphed(key, (cudaStream_t)stream, enqueue);
@@ -486,30 +630,83 @@ mosa_status mosa_backward(const mosa_shape *shape, const void *X, const void *W_
     if ((st = check_workspace(dm, workspace, workspace_bytes, &sv)) != MOSA_OK) return st;
     DevResources *res = use_tc(dm) ? dev_resources() : nullptr;
     auto enqueue = [&](cudaStream_t s) -> mosa_status {
-        if (res != nullptr)
-            return backward_tc(dm, X, W_r, W_q, W_k, W_v, W_o, dY, dX, dW_r, dW_q, dW_k, dW_v,
-                               dW_o, sv, s, *res);
-        {
-            StageScope st_(kStageOutBwd, s);
-            MOSA_TRY(launch_out_bwd(dm, W_o, dY, sv, dW_o, s));
-        }
-        {
-            StageScope st_(kStageAttnBwd, s);
-            MOSA_TRY(launch_attn_bwd(dm, sv, s));
-            if (dm.rope) MOSA_TRY(rope_qk(dm, sv, true, s));
-        }
-        {
-            StageScope st_(kStageInBwd, s);
-            MOSA_TRY(launch_in_bwd(dm, W_q, W_k, W_v, W_r, sv, dX, s));
-        }
-        {
-            StageScope st_(kStageWBwd, s);
-            MOSA_TRY(launch_w_bwd(dm, X, sv, dW_q, dW_k, dW_v, dW_r, s));
-        }
-        return MOSA_OK;
+        return backward_all(dm, X, W_r, W_q, W_k, W_v, W_o, dY, dX, dW_r, dW_q, dW_k, dW_v, dW_o,
+                            sv, s, res);
     };
     const GraphKey key = make_key(2, dm, shape, {X, W_r, W_q, W_k, W_v, W_o, I, r_sel, dY, dX,
                                                  dW_r, dW_q, dW_k, dW_v, dW_o, workspace});
+    return run_graphed(key, (cudaStream_t)stream, enqueue);
+}
+
+size_t mosa_hybrid_workspace_bytes(const mosa_hybrid_shape *shape) {
+    Hybrid h;
+    if (check_hybrid(shape, &h) != MOSA_OK) return 0;
+    return carve_hybrid(h, nullptr, nullptr);
+}
+
+mosa_status mosa_hybrid_forward(const mosa_hybrid_shape *shape, const void *X, const void *W_r,
+                                const void *W_q, const void *W_k, const void *W_v,
+                                const void *W_o, const void *D_q, const void *D_k,
+                                const void *D_v, const void *D_o, float *Y, int32_t *I,
+                                float *r_sel, float *r_full, void *workspace,
+                                size_t workspace_bytes, void *stream) {
+    Hybrid h;
+    mosa_status st = check_hybrid(shape, &h);
+    if (st != MOSA_OK) return st;
+    if (!X || !W_r || !W_q || !W_k || !W_v || !W_o || !Y || !I || !r_sel)
+        return MOSA_ERR_INVALID_ARG;
+    if (h.has_dense && (!D_q || !D_k || !D_v || !D_o)) return MOSA_ERR_INVALID_ARG;
+    HybridSpace sp;
+    if ((st = check_hybrid_workspace(h, workspace, workspace_bytes, &sp)) != MOSA_OK) return st;
+    float *rf = r_full ? r_full : sp.sparse.r_full;
+    DevResources *rs = use_tc(h.sparse) ? dev_resources() : nullptr;
+    DevResources *rd = h.has_dense && use_tc(h.dense) ? dev_resources() : nullptr;
+    auto enqueue = [&](cudaStream_t s) -> mosa_status {
+        mosa_status e = forward_routed(h.sparse, X, W_r, W_q, W_k, W_v, W_o, Y, I, r_sel, rf,
+                                       sp.sparse, s, rs);
+        if (e != MOSA_OK || !h.has_dense) return e;
+        return forward_given(h.dense, X, D_q, D_k, D_v, D_o, nullptr, nullptr, Y, sp.dense, s, rd);
+    };
+    const GraphKey key = make_key(3, h.sparse, &shape->sparse,
+                                  {X, W_r, W_q, W_k, W_v, W_o, D_q, D_k, D_v, D_o, Y, I, r_sel,
+                                   r_full, workspace},
+                                  h.has_dense ? &h.dense : nullptr, shape->H_dense, shape->window);
+    return run_graphed(key, (cudaStream_t)stream, enqueue);
+}
+
+mosa_status mosa_hybrid_backward(const mosa_hybrid_shape *shape, const void *X, const void *W_r,
+                                 const void *W_q, const void *W_k, const void *W_v,
+                                 const void *W_o, const void *D_q, const void *D_k,
+                                 const void *D_v, const void *D_o, const int32_t *I,
+                                 const float *r_sel, const void *dY, float *dX, float *dW_r,
+                                 float *dW_q, float *dW_k, float *dW_v, float *dW_o, float *dD_q,
+                                 float *dD_k, float *dD_v, float *dD_o, void *workspace,
+                                 size_t workspace_bytes, void *stream) {
+    Hybrid h;
+    mosa_status st = check_hybrid(shape, &h);
+    if (st != MOSA_OK) return st;
+    if (!X || !W_r || !W_q || !W_k || !W_v || !W_o || !I || !r_sel || !dY || !dX || !dW_r ||
+        !dW_q || !dW_k || !dW_v || !dW_o)
+        return MOSA_ERR_INVALID_ARG;
+    if (h.has_dense && (!D_q || !D_k || !D_v || !D_o || !dD_q || !dD_k || !dD_v || !dD_o))
+        return MOSA_ERR_INVALID_ARG;
+    HybridSpace sp;
+    if ((st = check_hybrid_workspace(h, workspace, workspace_bytes, &sp)) != MOSA_OK) return st;
+    DevResources *rs = use_tc(h.sparse) ? dev_resources() : nullptr;
+    DevResources *rd = h.has_dense && use_tc(h.dense) ? dev_resources() : nullptr;
+    auto enqueue = [&](cudaStream_t s) -> mosa_status {
+        mosa_status e = backward_all(h.sparse, X, W_r, W_q, W_k, W_v, W_o, dY, dX, dW_r, dW_q,
+                                     dW_k, dW_v, dW_o, sp.sparse, s, rs);
+        if (e != MOSA_OK || !h.has_dense) return e;
+        MOSA_TRY(cudaMemsetAsync(sp.zero_wr, 0, sp.zero_wr_bytes, s));
+        return backward_all(h.dense, X, sp.zero_wr, D_q, D_k, D_v, D_o, dY, dX, sp.dwr, dD_q,
+                            dD_k, dD_v, dD_o, sp.dense, s, rd);
+    };
+    const GraphKey key = make_key(4, h.sparse, &shape->sparse,
+                                  {X, W_r, W_q, W_k, W_v, W_o, D_q, D_k, D_v, D_o, I, r_sel, dY,
+                                   dX, dW_r, dW_q, dW_k, dW_v, dW_o, dD_q, dD_k, dD_v, dD_o,
+                                   workspace},
+                                  h.has_dense ? &h.dense : nullptr, shape->H_dense, shape->window);
     return run_graphed(key, (cudaStream_t)stream, enqueue);
 }
 

@@ -212,8 +212,10 @@ cudaError_t qkv_t(const Dims &dm, const void *X, const void *Wq, const void *Wk,
 
 template <class T>
 cudaError_t out_t(const Dims &dm, const void *Wo, const Saved &sv, float *Y, cudaStream_t s) {
-    cudaError_t e = cudaMemsetAsync(Y, 0, sizeof(float) * (size_t)dm.B * dm.T * dm.d, s);
-    if (e != cudaSuccess) return e;
+    if (!dm.accumulate) {
+        cudaError_t e = cudaMemsetAsync(Y, 0, sizeof(float) * (size_t)dm.B * dm.T * dm.d, s);
+        if (e != cudaSuccess) return e;
+    }
     OutOp<T> op{dm.B * dm.k, dm.d, dm.hp, sv.AR, (const T *)Wo, sv.gidx, Y};
     return launch_simt_gemm(op, dm.H, s);
 }
@@ -238,8 +240,10 @@ cudaError_t out_bwd_t(const Dims &dm, const void *Wo, const void *dY, const Save
 template <class T>
 cudaError_t in_bwd_t(const Dims &dm, const void *Wq, const void *Wk, const void *Wv,
                      const void *Wr, const Saved &sv, float *dX, cudaStream_t s) {
-    cudaError_t e = cudaMemsetAsync(dX, 0, sizeof(float) * (size_t)dm.B * dm.T * dm.d, s);
-    if (e != cudaSuccess) return e;
+    if (!dm.accumulate) {
+        cudaError_t e = cudaMemsetAsync(dX, 0, sizeof(float) * (size_t)dm.B * dm.T * dm.d, s);
+        if (e != cudaSuccess) return e;
+    }
     InBwdOp<T> op{dm.B * dm.k, dm.d, 3 * dm.hp, dm.hp, dm.H, sv.dQKV, (const T *)Wq,
                   (const T *)Wk, (const T *)Wv, (const T *)Wr, sv.dlogit, sv.gidx, dX};
     return launch_simt_gemm(op, dm.H, s);
@@ -274,7 +278,7 @@ cudaError_t launch_qkv(const Dims &dm, const void *X, const void *Wq, const void
 }
 
 cudaError_t launch_out(const Dims &dm, const void *Wo, const Saved &sv, float *Y, cudaStream_t s) {
-    if (use_tc(dm)) return tc_out(dm, Wo, sv, Y, s, true);
+    if (use_tc(dm)) return tc_out(dm, Wo, sv, Y, s, !dm.accumulate);
     return dm.bf16 ? out_t<bf16>(dm, Wo, sv, Y, s) : out_t<float>(dm, Wo, sv, Y, s);
 }
 
@@ -291,7 +295,7 @@ cudaError_t launch_in_bwd(const Dims &dm, const void *Wq, const void *Wk, const 
                           const void *Wr, const Saved &sv, float *dX, cudaStream_t s) {
     if (use_tc(dm)) {
         cudaError_t e = tc_transpose_wr(dm, Wr, sv, s);
-        return e != cudaSuccess ? e : tc_in_bwd(dm, Wq, Wk, Wv, Wr, sv, dX, s, true);
+        return e != cudaSuccess ? e : tc_in_bwd(dm, Wq, Wk, Wv, Wr, sv, dX, s, !dm.accumulate);
     }
     return dm.bf16 ? in_bwd_t<bf16>(dm, Wq, Wk, Wv, Wr, sv, dX, s)
                    : in_bwd_t<float>(dm, Wq, Wk, Wv, Wr, sv, dX, s);

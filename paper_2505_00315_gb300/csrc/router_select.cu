@@ -215,6 +215,18 @@ __global__ void indices_to_rows_kernel(const int32_t *__restrict__ I,
     }
 }
 
+// Dense heads (Sec. 2.1, Eq. mha; the dense heads of a hybrid layer,
+// Sec. 2.2): every (b, h) keeps all of its k = T tokens with score 1, so row
+// m = b*k + i of a head gathers X row b*T + i = m.
+__global__ void dense_rows_kernel(long long n, long long rows_per_head,
+                                  int32_t *__restrict__ gidx, float *__restrict__ rsel_hm) {
+    for (long long o = (long long)blockIdx.x * blockDim.x + threadIdx.x; o < n;
+         o += (long long)gridDim.x * blockDim.x) {
+        gidx[o] = (int32_t)(o % rows_per_head);
+        rsel_hm[o] = 1.f;
+    }
+}
+
 }  // namespace
 
 cudaError_t launch_router(const Dims &dm, const void *X, const void *Wr, float *r_full,
@@ -264,6 +276,16 @@ cudaError_t launch_indices_to_rows(const Dims &dm, const int32_t *I, const float
                                    cudaStream_t stream) {
     indices_to_rows_kernel<<<dm.B * dm.H, 256, 0, stream>>>(I, rsel, dm.B, dm.H, dm.T, dm.k,
                                                            gidx, rsel_hm, status);
+    note_launches(1);
+    return cudaGetLastError();
+}
+
+cudaError_t launch_dense_rows(const Dims &dm, int32_t *gidx, float *rsel_hm, cudaStream_t stream) {
+    const long long n = dm.rows();
+    if (n <= 0) return cudaSuccess;
+    const long long blocks = (n + 255) / 256;
+    dense_rows_kernel<<<(unsigned)(blocks < 4096 ? blocks : 4096), 256, 0, stream>>>(
+        n, (long long)dm.B * dm.k, gidx, rsel_hm);
     note_launches(1);
     return cudaGetLastError();
 }

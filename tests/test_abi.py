@@ -122,3 +122,58 @@ def test_check_status_rejects_bad_arguments():
 ])
 def test_adaptive_k(T, rho, k):
     assert B.mosa_adaptive_k(T, rho) == k
+
+
+def hshape(H_dense=2, window=0, **kw):
+    return B.MosaHybridShape(shape(**kw), H_dense, window)
+
+
+@pytest.mark.parametrize("H_dense,window,kw,ok", [
+    (2, 0, {}, True), (2, 16, {}, True), (2, 64, {}, True), (0, 0, {}, True), (1, 1, {}, True),
+    (2, 24, {}, False),              # local blocks must tile the sequence
+    (2, 65, {}, False), (2, -1, {}, False), (-1, 0, {}, False),
+    (2, 0, dict(k=65), False), (2, 0, dict(hp=48), False), (2, 0, dict(first_token=1), True),
+])
+def test_hybrid_workspace_bytes_validates_shape(H_dense, window, kw, ok):
+    assert (B.mosa_hybrid_workspace_bytes(hshape(H_dense, window, **kw)) > 0) == ok
+
+
+def test_hybrid_workspace_holds_both_head_groups():
+    s = shape()
+    sparse = B.mosa_workspace_bytes(s)
+    assert B.mosa_hybrid_workspace_bytes(hshape(0)) == sparse
+    dense = B.mosa_hybrid_workspace_bytes(hshape(2))
+    assert dense > sparse
+    assert B.mosa_hybrid_workspace_bytes(hshape(4)) > dense
+    assert B.mosa_hybrid_workspace_bytes(hshape(2, window=64)) == dense   # w = T is dense
+    # local heads keep every token too, in blocks: no fewer rows than dense heads
+    assert B.mosa_hybrid_workspace_bytes(hshape(2, window=16)) > sparse
+
+
+def test_hybrid_entries_reject_before_launch():
+    L = B.load()
+    fwd = [FAKE] * 14            # X, W_r, W_q..W_o, D_q..D_o, Y, I, r_sel, r_full
+    assert L.mosa_hybrid_forward(ctypes.byref(hshape(window=24)), *fwd, FAKE, 1 << 40, None) \
+        == B.MOSA_ERR_UNSUPPORTED
+    assert L.mosa_hybrid_forward(None, *fwd, FAKE, 1 << 40, None) == B.MOSA_ERR_INVALID_ARG
+    for i in range(13):
+        a = list(fwd)
+        a[i] = None
+        assert L.mosa_hybrid_forward(ctypes.byref(hshape()), *a, FAKE, 1 << 40, None) == \
+            B.MOSA_ERR_INVALID_ARG, i
+    # without dense heads their weights may be NULL: validation reaches the workspace
+    a = list(fwd)
+    a[6:10] = [None] * 4
+    assert L.mosa_hybrid_forward(ctypes.byref(hshape(0)), *a, None, 1 << 40, None) == \
+        B.MOSA_ERR_WORKSPACE
+    need = B.mosa_hybrid_workspace_bytes(hshape())
+    assert L.mosa_hybrid_forward(ctypes.byref(hshape()), *fwd, FAKE, need - 1, None) == \
+        B.MOSA_ERR_WORKSPACE
+    bwd = [FAKE] * 23            # ..., I, r_sel, dY, dX, dW_r..dW_o, dD_q..dD_o
+    for i in range(23):
+        a = list(bwd)
+        a[i] = None
+        assert L.mosa_hybrid_backward(ctypes.byref(hshape()), *a, FAKE, 1 << 40, None) == \
+            B.MOSA_ERR_INVALID_ARG, i
+    assert L.mosa_hybrid_backward(ctypes.byref(hshape()), *bwd, None, 1 << 40, None) == \
+        B.MOSA_ERR_WORKSPACE

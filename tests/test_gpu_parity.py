@@ -228,6 +228,89 @@ def test_hybrid_mosa_plus_dense_heads(rope):
     assert_close("Y", (Yg + Ydg).cpu().numpy(), Ym + Yd, "bf16")
 
 
+# --------------- hybrid layer entry (Sec. 2.2 hybridization, Sec. 3.4) ----
+
+# (config, dense heads, window): window 0 = dense causal heads over all T
+# tokens, w > 0 = local heads within blocks of w tokens
+HYBRID = [
+    (W.MosaConfig("hyb_dense_bf16", B=2, T=256, d=128, H=4, hp=64, k=64, dtype="bf16",
+                  seed=53), 2, 0),
+    (W.MosaConfig("hyb_local64_rope_bf16", B=2, T=256, d=128, H=4, hp=64, k=32, dtype="bf16",
+                  seed=54, rope=True), 3, 64),
+    (W.MosaConfig("hyb_local128_first_rope_bf16", B=2, T=384, d=64, H=2, hp=64, k=48,
+                  dtype="bf16", seed=55, rope=True, first_token=True), 2, 128),
+    (W.MosaConfig("hyb_dense_rope_f32", B=2, T=96, d=48, H=3, hp=32, k=24, dtype="f32", seed=56,
+                  rope=True), 2, 0),
+    (W.MosaConfig("hyb_local40_f32", B=1, T=120, d=40, H=2, hp=16, k=30, dtype="f32", seed=57),
+     1, 40),
+]
+
+
+def run_hybrid(cfg, x, xd, window):
+    dt = cfg.dtype
+    X, Wr, Wq, Wk, Wv, Wo = (to_dev(x[n], dt) for n in ("X", "Wr", "Wq", "Wk", "Wv", "Wo"))
+    D = [to_dev(xd[n], dt) for n in ("Dq", "Dk", "Dv", "Do")]
+    Y, I, rs, ws = mosa.mosa_hybrid_forward(X, Wr, Wq, Wk, Wv, Wo, *D, cfg.k, window=window,
+                                            first_token=cfg.first_token, rope=cfg.rope)
+    out = {"Y": Y, "I": I}
+    out.update(mosa.mosa_hybrid_backward(X, Wr, Wq, Wk, Wv, Wo, *D, I, rs, to_dev(x["dY"], dt),
+                                         ws, window=window, rope=cfg.rope))
+    torch.cuda.synchronize()
+    assert mosa.mosa_check_status(mosa.make_shape(X, Wq, cfg.k), ws) == 0
+    return {k: v.cpu().numpy() for k, v in out.items()}
+
+
+HYB_GRADS = (("dX", "dX"), ("dWr", "dW_r"), ("dWq", "dW_q"), ("dWk", "dW_k"), ("dWv", "dW_v"),
+             ("dWo", "dW_o"), ("dDq", "dD_q"), ("dDk", "dD_k"), ("dDv", "dD_v"),
+             ("dDo", "dD_o"))
+
+
+@pytest.mark.parametrize("case", HYBRID, ids=lambda c: c[0].name)
+def test_hybrid_entry_forward_backward_parity(case, kernel_path):
+    cfg, H_dense, window = case
+    x = W.make_inputs(cfg)
+    xd = W.make_dense_weights(cfg, H_dense)
+    Y, I, _, _ = oracle.hybrid_forward(x["X"], *weights(x), xd["Dq"], xd["Dk"], xd["Dv"],
+                                       xd["Do"], k=cfg.k, window=window,
+                                       first_token=cfg.first_token, rope=cfg.rope)
+    ref = oracle.hybrid_backward(x["X"], *weights(x), xd["Dq"], xd["Dk"], xd["Dv"], xd["Do"],
+                                 I=I, dY=x["dY"], window=window, rope=cfg.rope)
+    g = run_hybrid(cfg, x, xd, window)
+    np.testing.assert_array_equal(g["I"], I)
+    assert_close("Y", g["Y"], Y, cfg.dtype)
+    for name, gname in HYB_GRADS:
+        assert_close(name, g[gname], ref[name], cfg.dtype)
+
+
+def test_hybrid_entry_paper_sizes_sampled():
+    # the IsoFLOP hybrids of Sec. 3.2 keep 4 dense heads beside the MoSA
+    # heads (here at B8 T1024 d512 H16 k128); the long-sequence models of
+    # Sec. 3.4 pair 60 MoSA heads (k = 64) with 4 local heads at T = 2048,
+    # d = 1024 (block of 512 tokens).  Y and dX of the last sequence, exact in
+    # the oracle for that sequence alone.
+    for cfg, H_dense, window in (
+            (W.MosaConfig("hyb_isoflop", B=8, T=1024, d=512, H=16, hp=64, k=128, dtype="bf16",
+                          seed=58, rope=True, first_token=True), 4, 0),
+            (W.MosaConfig("hyb_long", B=1, T=2048, d=1024, H=60, hp=64, k=64, dtype="bf16",
+                          seed=59, rope=True), 4, 512)):
+        x = W.make_inputs(cfg)
+        xd = W.make_dense_weights(cfg, H_dense)
+        g = run_hybrid(cfg, x, xd, window)
+        b0 = cfg.B - 1
+        Y, I, _, _ = oracle.hybrid_forward(x["X"], *weights(x), xd["Dq"], xd["Dk"], xd["Dv"],
+                                           xd["Do"], k=cfg.k, window=window, batches=[b0],
+                                           first_token=cfg.first_token, rope=cfg.rope)
+        np.testing.assert_array_equal(g["I"][b0], I[b0])
+        assert_close("Y", g["Y"][b0], Y[b0], cfg.dtype)
+        ref = oracle.hybrid_backward(x["X"], *weights(x), xd["Dq"], xd["Dk"], xd["Dv"],
+                                     xd["Do"], I=I, dY=x["dY"], window=window, batches=[b0],
+                                     rope=cfg.rope)
+        assert_close("dX", g["dX"][b0], ref["dX"][b0], cfg.dtype)
+        if cfg.B == 1:
+            for name, gname in HYB_GRADS[1:]:
+                assert_close(name, g[gname], ref[name], cfg.dtype)
+
+
 # ------------------------------------------------ full workload sizes ----
 
 FULL = [c for c in W.CONFIGS.values() if c.dtype == "bf16"]

@@ -55,6 +55,15 @@ def parse_args():
     p.add_argument("--config", default=None)
     p.add_argument("--no-cpu-baseline", action="store_true")
     p.add_argument("--cpu-budget-s", type=float, default=15.0)
+    p.add_argument("--rope", action="store_true",
+                   help="rotary position encoding at the original positions (Sec. 2.2)")
+    p.add_argument("--first-token", action="store_true",
+                   help="every head keeps token 0 and selects k-1 more (Sec. 3.2)")
+    p.add_argument("--dense-heads", type=int, default=0,
+                   help="hybrid layer: this many dense heads beside the MoSA heads (Sec. 2.2)")
+    p.add_argument("--window", type=int, default=0,
+                   help="with --dense-heads: local heads over blocks of this many tokens "
+                        "(Sec. 3.4); 0 = dense causal heads")
     p.add_argument("--ingest-ncu", metavar="CSV", default=None,
                    help="turn an ncu CSV with dram__bytes_read/write.sum per kernel (taken on "
                         "this command's workload) into profiles/traffic.json and exit")
@@ -140,14 +149,25 @@ class ClockSampler:
 # ------------------------------------------------------------ CPU oracle
 
 def oracle_sample(cfg, x, n_seq):
-    """Time the oracle's forward + backward on the first n_seq sequences."""
+    """Time the oracle's forward + backward on the first n_seq sequences (with
+    the dense heads of a hybrid layer when x holds their weights)."""
     import oracle
     W = (x["Wr"], x["Wq"], x["Wk"], x["Wv"], x["Wo"])
     batches = list(range(n_seq))
     t0 = time.perf_counter()
-    _, I, _, _ = oracle.forward(x["X"], *W, k=cfg.k, batches=batches)
+    if "Dq" in x:
+        D = (x["Dq"], x["Dk"], x["Dv"], x["Do"])
+        _, I, _, _ = oracle.hybrid_forward(x["X"], *W, *D, k=cfg.k, window=x["window"],
+                                           batches=batches, first_token=cfg.first_token,
+                                           rope=cfg.rope)
+        if cfg.backward:
+            oracle.hybrid_backward(x["X"], *W, *D, I=I, dY=x["dY"], window=x["window"],
+                                   batches=batches, rope=cfg.rope)
+        return time.perf_counter() - t0
+    _, I, _, _ = oracle.forward(x["X"], *W, k=cfg.k, batches=batches,
+                                first_token=cfg.first_token, rope=cfg.rope)
     if cfg.backward:
-        oracle.backward(x["X"], *W, I=I, dY=x["dY"], batches=batches)
+        oracle.backward(x["X"], *W, I=I, dY=x["dY"], batches=batches, rope=cfg.rope)
     return time.perf_counter() - t0
 
 
@@ -165,7 +185,7 @@ def cpu_baseline(cfg, x, budget_s):
     return {"value": n * cfg.T / t, "unit": "tokens/s", "cores": oracle.num_threads(),
             "kind": "oracle",
             "sample": f"{what} of {n} of the {cfg.B} sequences of {cfg.name} "
-                      f"(all {cfg.H} heads, fp64, {t:.2f} s)"}
+                      f"(all heads, fp64, {t:.2f} s)"}
 
 
 # ------------------------------------------------------------ roofline
@@ -189,7 +209,7 @@ def stage_kind(stage, lib_impl):
 
 
 def traffic_for(stage, cfg_name):
-    """Per-launch DRAM bytes of `stage` from the committed ncu summary, or None
+    """DRAM bytes per step of `stage` from the committed ncu summary, or None
     when the summary is missing or was taken on a different kernel source."""
     path = os.path.join(ROOT, "profiles", "traffic.json")
     if not os.path.exists(path):
@@ -201,7 +221,7 @@ def traffic_for(stage, cfg_name):
         return None
     if ent.get("source_sha256") != source_digest():
         return None
-    return ent.get("bytes_per_launch")
+    return ent.get("bytes_per_step")
 
 
 # Kernel name (as ncu prints it) -> bench stage.
@@ -214,19 +234,28 @@ KERNEL_STAGE = [("tc_gemm_kernel<5>", "router"), ("tc_gemm_kernel<(int)5>", "rou
                 ("scatter_product_kernel<1>", "out"), ("scatter_product_kernel<true>", "out"),
                 ("tc_gemm_kernel<4>", "w_bwd"), ("tc_gemm_kernel<(int)4>", "w_bwd"),
                 ("tc_gemm_kernel<3>", "dwo"), ("tc_gemm_kernel<(int)3>", "dwo"),
-                ("fused_fwd_kernel", "fwd_unit"), ("fused_bwd_kernel", "bwd_unit")]
+                ("fused_fwd_kernel", "fwd_unit"), ("fused_bwd_kernel", "bwd_unit"),
+                ("dense_rows", "select")]
+# RoPE passes (rope_rows_kernel) run inside the qkv and attn_bwd stages alike
+# and are left unattributed.
 
 
 def ingest_ncu(csv_path, cfg_name):
-    """Average DRAM bytes per step of each stage from an ncu CSV (one row per
-    kernel launch and metric) into profiles/traffic.json."""
+    """DRAM bytes per step of each stage from an ncu CSV (one row per kernel
+    launch and metric) into profiles/traffic.json.  A stage may launch several
+    kernels a step (the large-k attention backward and its dQ split; both head
+    groups of a hybrid layer); the steps are counted by the TopK launches, one
+    per layer step."""
     import csv
     import collections
     per = collections.defaultdict(lambda: collections.defaultdict(float))
+    steps = set()
     with open(csv_path) as f:
         lines = [l for l in f if not l.startswith("==")]
     for row in csv.DictReader(lines):
         name, metric = row.get("Kernel Name", ""), row.get("Metric Name", "")
+        if "topk_select" in name:
+            steps.add(row["ID"])
         if metric not in ("dram__bytes_read.sum", "dram__bytes_write.sum"):
             continue
         stage = next((st for key, st in KERNEL_STAGE if key in name), None)
@@ -238,15 +267,16 @@ def ingest_ncu(csv_path, cfg_name):
     path = os.path.join(ROOT, "profiles", "traffic.json")
     data = json.load(open(path)) if os.path.exists(path) else {}
     digest = source_digest()
+    n_steps = max(1, len(steps))
     ent = {}
     for stage, launches in per.items():
         vals = list(launches.values())
-        ent[stage] = {"bytes_per_launch": sum(vals) / len(vals), "launches": len(vals),
-                      "source_sha256": digest}
+        ent[stage] = {"bytes_per_step": sum(vals) / n_steps, "launches": len(vals),
+                      "steps": n_steps, "source_sha256": digest}
     data[cfg_name] = ent
     with open(path, "w") as f:
         json.dump(data, f, indent=1, sort_keys=True)
-    print(json.dumps({k: round(v["bytes_per_launch"] / 1e6, 3) for k, v in ent.items()}))
+    print(json.dumps({k: round(v["bytes_per_step"] / 1e6, 3) for k, v in ent.items()}))
 
 
 def source_digest():
@@ -281,8 +311,7 @@ def run_reference(args, cfg, rank, world):
     if rank != 0:
         return
     import oracle
-    from paper_2505_00315_gb300 import workloads as W
-    x = W.make_inputs(cfg)
+    x = make_workload(cfg, args)
     per_step_budget = max(1.0, 150.0 / max(1, args.steps + args.warmup))
     n, _ = choose_sample(cfg, x, per_step_budget)
     for _ in range(args.warmup):
@@ -295,7 +324,7 @@ def run_reference(args, cfg, rank, world):
             "n_gpus": args.gpus, "steps": args.steps, "warmup": args.warmup,
             "ms_per_step": 1e3 * total / args.steps, "higher_is_better": True,
             "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic",
-            "config": config_block(cfg),
+            "config": config_block(cfg, args),
             "cpu_baseline": {"value": value, "unit": "tokens/s", "kind": "oracle",
                              "cores": oracle.num_threads(),
                              "sample": f"{what} of {n} of the {cfg.B} sequences per step"},
@@ -304,11 +333,36 @@ def run_reference(args, cfg, rank, world):
     print(json.dumps(line), flush=True)
 
 
-def config_block(cfg):
+def variant(cfg, args):
+    """The workload with the option flags applied, and its name."""
+    cfg = cfg.with_(rope=bool(args.rope), first_token=bool(args.first_token))
+    name = cfg.name + ("+rope" if cfg.rope else "") + ("+first" if cfg.first_token else "")
+    if args.dense_heads:
+        name += f"+dense{args.dense_heads}" + (f"w{args.window}" if args.window else "")
+    return cfg.with_(name=name)
+
+
+def config_block(cfg, args=None):
+    extra = {}
+    if cfg.rope or cfg.first_token:
+        extra.update(rope=cfg.rope, first_token=cfg.first_token)
+    if args is not None and args.dense_heads:
+        extra.update(H_dense=args.dense_heads, window=args.window)
     return {"workload": cfg.name, "B": cfg.B, "T": cfg.T, "d": cfg.d, "H": cfg.H, "hp": cfg.hp,
-            "k": cfg.k, "storage": cfg.dtype,
+            "k": cfg.k, "storage": cfg.dtype, **extra,
             "inputs": "seeded Gaussian X, weights N(0,1/d), dY; planted router margin",
             "l2": "flushed before every timed step by a 256 MiB write outside the step's events"}
+
+
+def make_workload(cfg, args):
+    """Seeded inputs of the workload, plus the dense heads' weights and window
+    of a hybrid layer."""
+    from paper_2505_00315_gb300 import workloads as W
+    x = W.make_inputs(cfg)
+    if args.dense_heads:
+        x.update(W.make_dense_weights(cfg, args.dense_heads))
+        x["window"] = args.window
+    return x
 
 
 def main():
@@ -319,7 +373,7 @@ def main():
     world = int(os.environ.get("WORLD_SIZE", "1"))
     rank = int(os.environ.get("RANK", "0"))
     local = int(os.environ.get("LOCAL_RANK", "0"))
-    cfg = W.CONFIGS[args.config or W.BENCH_CONFIG]
+    cfg = variant(W.CONFIGS[args.config or W.BENCH_CONFIG], args)
 
     if args.ingest_ncu:
         ingest_ncu(args.ingest_ncu, cfg.name)
@@ -342,12 +396,18 @@ def main():
         if dist is not None:
             dist.barrier()
 
-    x = W.make_inputs(cfg)
+    x = make_workload(cfg, args)
     tdt = torch.bfloat16 if cfg.dtype == "bf16" else torch.float32
     dev = torch.device("cuda", local)
-    D = {n: torch.from_numpy(x[n]).to(dev).to(tdt) for n in x}
-    shape = mosa.make_shape(D["X"], D["Wq"], cfg.k)
-    ws = mosa.alloc_workspace(shape, dev)
+    D = {n: torch.from_numpy(x[n]).to(dev).to(tdt) for n in x if n != "window"}
+    shape = mosa.make_shape(D["X"], D["Wq"], cfg.k, cfg.first_token, cfg.rope)
+    hybrid = args.dense_heads > 0
+    if hybrid:
+        ws = mosa.alloc_hybrid_workspace(
+            mosa.make_hybrid_shape(D["X"], D["Wq"], cfg.k, args.dense_heads, args.window,
+                                   cfg.first_token, cfg.rope), dev)
+    else:
+        ws = mosa.alloc_workspace(shape, dev)
     f32 = dict(dtype=torch.float32, device=dev)
     outs = {"Y": torch.empty((cfg.B, cfg.T, cfg.d), **f32),
             "I": torch.empty((cfg.B, cfg.H, cfg.k), dtype=torch.int32, device=dev),
@@ -358,30 +418,47 @@ def main():
              "dW_k": torch.empty((cfg.H, cfg.d, cfg.hp), **f32),
              "dW_v": torch.empty((cfg.H, cfg.d, cfg.hp), **f32),
              "dW_o": torch.empty((cfg.H, cfg.hp, cfg.d), **f32)}
+    if hybrid:
+        for n in ("Dq", "Dk", "Dv", "Do"):
+            grads["dD_" + n[1]] = torch.empty(D[n].shape, **f32)
     flush_buf = torch.empty(L2_FLUSH_BYTES // 4, **f32)
+    Wm = (D["Wr"], D["Wq"], D["Wk"], D["Wv"], D["Wo"])
 
-    def step(Xd=None, dYd=None):
-        Xd = D["X"] if Xd is None else Xd
-        dYd = D["dY"] if dYd is None else dYd
-        Y, I, rs, _, _ = mosa.mosa_forward(Xd, D["Wr"], D["Wq"], D["Wk"], D["Wv"], D["Wo"],
-                                           cfg.k, workspace=ws, out=outs)
+    def layer(Xd, dYd, o, g):
+        """One forward (+ backward) through the public API."""
+        if hybrid:
+            Dw = (D["Dq"], D["Dk"], D["Dv"], D["Do"])
+            _, I, rs, _ = mosa.mosa_hybrid_forward(Xd, *Wm, *Dw, cfg.k, window=args.window,
+                                                   workspace=ws, out=o,
+                                                   first_token=cfg.first_token, rope=cfg.rope)
+            if cfg.backward:
+                mosa.mosa_hybrid_backward(Xd, *Wm, *Dw, I, rs, dYd, ws, window=args.window,
+                                          out=g, rope=cfg.rope)
+            return
+        _, I, rs, _, _ = mosa.mosa_forward(Xd, *Wm, cfg.k, workspace=ws, out=o,
+                                           first_token=cfg.first_token, rope=cfg.rope)
         if cfg.backward:
-            mosa.mosa_backward(Xd, D["Wr"], D["Wq"], D["Wk"], D["Wv"], D["Wo"], I, rs, dYd, ws,
-                               out=grads)
+            mosa.mosa_backward(Xd, *Wm, I, rs, dYd, ws, out=g, rope=cfg.rope)
+
+    def step():
+        layer(D["X"], D["dY"], outs, grads)
 
     # Warm-up, then one profiled pass to find the dominant stage.
     for _ in range(max(3, args.warmup)):
         flush_buf.zero_()
         step()
     torch.cuda.synchronize()
+    # Stage times are per step: a hybrid layer runs each stage twice a step
+    # (MoSA heads, then dense heads), and its algorithmic work is per step.
     mosa.mosa_profile_stages((1 << len(STAGES)) - 1)
-    for _ in range(5):
+    n_prof = 5
+    for _ in range(n_prof):
         flush_buf.zero_()
         step()
     torch.cuda.synchronize()
     prof = mosa.mosa_profile_read()
     mosa.mosa_profile_stages(0)
-    stage_ms = {s: prof[s][0] / max(prof[s][1], 1) for s in STAGES if prof[s][1]}
+    stage_ms = {s: prof[s][0] / n_prof for s in STAGES if prof[s][1]}
     dominant = max(stage_ms, key=stage_ms.get)
 
     # Timed region: K steps, L2 flushed before each, the dominant stage timed
@@ -405,7 +482,7 @@ def main():
     barrier()
     torch.cuda.synchronize()
     launches0 = mosa.mosa_kernel_launches()
-    dom = [0.0, 0]
+    dom = [0.0, 0, 0]   # ms, launches, steps
     t_host0 = time.time()
     for i in range(K):
         timed = i % PROFILE_EVERY == 0
@@ -419,6 +496,7 @@ def main():
             ms, n = mosa.mosa_profile_read()[dominant]
             dom[0] += ms
             dom[1] += n
+            dom[2] += 1
     torch.cuda.synchronize()
     t_host1 = time.time()
     barrier()
@@ -501,11 +579,7 @@ def main():
             comp.wait_event(in_ready[j])
             if i >= 2:
                 comp.wait_event(out_free[j])      # step i-2's outputs have left
-            Y, I, rs, _, _ = mosa.mosa_forward(sl["X"], D["Wr"], D["Wq"], D["Wk"], D["Wv"],
-                                               D["Wo"], cfg.k, workspace=ws, out=sl["outs"])
-            if cfg.backward:
-                mosa.mosa_backward(sl["X"], D["Wr"], D["Wq"], D["Wk"], D["Wv"], D["Wo"], I, rs,
-                                   sl["dY"], ws, out=sl["grads"])
+            layer(sl["X"], sl["dY"], sl["outs"], sl["grads"])
             in_free[j].record(comp)
             done[j].record(comp)
             with torch.cuda.stream(s_out):
@@ -537,12 +611,12 @@ def main():
 
     # Roofline of the dominant kernel.
     peaks, peak_src = load_peaks()
-    work = flops.layer_work(cfg.B, cfg.T, cfg.d, cfg.H, cfg.hp, cfg.k,
-                            elem_bytes=2 if cfg.dtype == "bf16" else 4)
+    work = flops.hybrid_work(cfg.B, cfg.T, cfg.d, cfg.H, cfg.hp, cfg.k, args.dense_heads,
+                             args.window, elem_bytes=2 if cfg.dtype == "bf16" else 4)
     impl = mosa.stage_impl(shape)
     kind = stage_kind(dominant, impl)
     bound, peak, unit = stage_bound(dominant, peaks, kind)
-    dom_ms = dom[0] / max(dom[1], 1)
+    dom_ms = dom[0] / max(dom[2], 1)   # per step
     if unit == "GB/s":
         achieved = work[dominant]["bytes"] / (dom_ms / 1e3) / 1e9
     else:
@@ -552,12 +626,13 @@ def main():
         "metric": METRIC, "value": value, "unit": "tokens/s", "n_gpus": world, "steps": K,
         "warmup": args.warmup, "ms_per_step": total_ms / K, "higher_is_better": True,
         "scaling": "weak", "vs_baseline": None, "dtype": cfg.dtype, "data": "synthetic",
-        "config": config_block(cfg),
+        "config": config_block(cfg, args),
         "roofline": {"kernel": dominant, "bound": bound, "achieved": achieved, "peak": peak,
                      "unit": unit, "frac": achieved / peak, "peak_source": peak_src,
                      "traffic": traffic_for(dominant, cfg.name),
                      "algorithmic": work[dominant]["flops" if unit != "GB/s" else "bytes"],
-                     "ms_per_launch": dom_ms, "timed_launches": dom[1],
+                     "stage_ms_per_step": dom_ms, "launches_per_step": dom[1] / max(dom[2], 1),
+                     "timed_steps": dom[2],
                      "timed_every_nth_step": PROFILE_EVERY},
         "layer_tflops": layer_flops * world * K / (total_ms / 1e3) / 1e12,
         "stage_ms": {s: round(v, 5) for s, v in stage_ms.items()},

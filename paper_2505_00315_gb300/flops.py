@@ -101,3 +101,33 @@ def layer_work(B: int, T: int, d: int, H: int, hp: int, k: int, elem_bytes: int 
     w["forward_flops"] = sum(w[s]["flops"] for s in fwd)
     w["backward_flops"] = sum(w[s]["flops"] for s in bwd)
     return w
+
+
+def hybrid_work(B: int, T: int, d: int, H: int, hp: int, k: int, H_dense: int,
+                window: int = 0, elem_bytes: int = 2) -> dict:
+    """``layer_work`` of a hybrid layer (Sec. 2.2, hybridization; Sec. 3.4):
+    the MoSA heads plus H_dense dense heads over all T tokens (window 0) or
+    local heads over blocks of ``window`` tokens, per step, summed.  The dense
+    heads have no router: no F1 work, their token lists are written once
+    (8 bytes per row), and no dlogit terms in B3/B4."""
+    w = layer_work(B, T, d, H, hp, k, elem_bytes)
+    if H_dense <= 0:
+        return w
+    blk = window if window else T
+    Bd = B * (T // blk)
+    dn = layer_work(Bd, blk, d, H_dense, hp, blk, elem_bytes)
+    rows = Bd * H_dense * blk
+    dn["router"] = {"flops": 0, "bytes": 0}
+    dn["select"] = {"flops": 0, "bytes": 2 * rows * 4}
+    for s in ("in_bwd", "w_bwd"):
+        dn[s] = dict(dn[s], flops=dn[s]["flops"] - 2 * d * blk * Bd * H_dense)
+    dn["w_bwd"]["bytes"] -= d * H_dense * 4
+    out = {}
+    for s, v in w.items():
+        if isinstance(v, dict):
+            out[s] = {"flops": v["flops"] + dn[s]["flops"], "bytes": v["bytes"] + dn[s]["bytes"]}
+    fwd = ("router", "select", "qkv", "attn_fwd", "out")
+    bwd = ("out_bwd", "dwo", "attn_bwd", "in_bwd", "w_bwd")
+    out["forward_flops"] = sum(out[s]["flops"] for s in fwd)
+    out["backward_flops"] = sum(out[s]["flops"] for s in bwd)
+    return out

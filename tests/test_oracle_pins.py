@@ -571,3 +571,22 @@ def test_hybrid_layer_matches_torch_restatement(window, rope):
     for n in names:
         np.testing.assert_allclose(g["d" + n], ts[n].grad.numpy(), rtol=1e-10, atol=1e-11,
                                    err_msg=n)
+
+
+def test_hybrid_work_adds_dense_and_local_heads():
+    # dense heads: every token, causal attention over T, no router terms;
+    # local heads of w tokens: B*T/w sequences of w tokens
+    B, T, d, H, hp, k, Hd = 2, 64, 32, 3, 16, 8, 2
+    base = flops.layer_work(B, T, d, H, hp, k)
+    assert flops.hybrid_work(B, T, d, H, hp, k, 0) == base
+    for w, n_seq in ((0, B), (16, B * T // 16)):
+        blk = w or T
+        h = flops.hybrid_work(B, T, d, H, hp, k, Hd, w)
+        U = n_seq * Hd
+        assert h["router"] == base["router"]
+        assert h["attn_fwd"]["flops"] - base["attn_fwd"]["flops"] == 2 * hp * blk * (blk + 1) * U
+        assert h["qkv"]["flops"] - base["qkv"]["flops"] == 6 * d * hp * blk * U
+        assert h["in_bwd"]["flops"] - base["in_bwd"]["flops"] == 6 * d * hp * blk * U
+        assert h["w_bwd"]["flops"] - base["w_bwd"]["flops"] == 6 * d * hp * blk * U
+        assert h["forward_flops"] == sum(h[s]["flops"] for s in
+                                         ("router", "select", "qkv", "attn_fwd", "out"))

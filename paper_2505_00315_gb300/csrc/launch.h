@@ -43,9 +43,11 @@ inline cudaError_t launch_pdl(void (*kernel)(KArgs...), dim3 grid, dim3 block, s
 RopeTable make_rope_table(int hp, int T);
 // Turns pairs (col0 + 2p, col0 + 2p + 1), p < h'/4, of each of `rows` stored
 // rows ([rows, 2 cols] bf16 pairs if `pair`, else [rows, cols] fp32) in place
-// by dir * t * theta_p, t = gidx[row] mod T.
-cudaError_t launch_rope(void *p, bool pair, int cols, int col0, long long rows,
-                        const int32_t *gidx, const RopeTable &tab, float dir, cudaStream_t s);
+// by dir * t * theta_p, t = gidx[row] mod T, for two column blocks at once:
+// (p0, col0_0) and (p1, col0_1).  col0_* and cols are multiples of 8.
+cudaError_t launch_rope(void *p0, int col0_0, void *p1, int col0_1, bool pair, int cols,
+                        long long rows, const int32_t *gidx, const RopeTable &tab, float dir,
+                        cudaStream_t s);
 
 // F1, Sec. 2.2 router: r_full[b,h,t] = sigmoid(X[b,t,:] . W_r[:,h]) in fp32.
 cudaError_t launch_router(const Dims &dm, const void *X, const void *Wr, float *r_full,

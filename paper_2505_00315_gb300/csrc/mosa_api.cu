@@ -133,17 +133,9 @@ cudaError_t rope_qk(const Dims &dm, const Saved &sv, bool grads, cudaStream_t s)
     const RopeTable tab = make_rope_table(dm.hp, dm.T);
     const long long rows = dm.rows();
     const bool pair = dm.bf16;
-    cudaError_t e;
-    if (!grads) {
-        e = launch_rope(sv.Q, pair, dm.hp, 0, rows, sv.gidx, tab, 1.f, s);
-        if (e == cudaSuccess) e = launch_rope(sv.K, pair, dm.hp, 0, rows, sv.gidx, tab, 1.f, s);
-    } else {
-        const int cols = use_tc(dm) ? 256 : 3 * dm.hp;
-        e = launch_rope(sv.dQKV, pair, cols, 0, rows, sv.gidx, tab, -1.f, s);
-        if (e == cudaSuccess)
-            e = launch_rope(sv.dQKV, pair, cols, dm.hp, rows, sv.gidx, tab, -1.f, s);
-    }
-    return e;
+    if (!grads) return launch_rope(sv.Q, 0, sv.K, 0, pair, dm.hp, rows, sv.gidx, tab, 1.f, s);
+    const int cols = use_tc(dm) ? 256 : 3 * dm.hp;
+    return launch_rope(sv.dQKV, 0, sv.dQKV, dm.hp, pair, cols, rows, sv.gidx, tab, -1.f, s);
 }
 
 mosa_status forward_heads(const Dims &dm, const void *X, const void *W_q, const void *W_k,

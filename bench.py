@@ -622,6 +622,9 @@ def main():
     else:
         achieved = work[dominant]["flops"] / (dom_ms / 1e3) / 1e12
     layer_flops = work["forward_flops"] + (work["backward_flops"] if cfg.backward else 0)
+    full = flops.hybrid_work(cfg.B, cfg.T, cfg.d, cfg.H, cfg.hp, cfg.k, args.dense_heads,
+                             args.window, causal=False)
+    layer_flops_full = full["forward_flops"] + (full["backward_flops"] if cfg.backward else 0)
     line = {
         "metric": METRIC, "value": value, "unit": "tokens/s", "n_gpus": world, "steps": K,
         "warmup": args.warmup, "ms_per_step": total_ms / K, "higher_is_better": True,
@@ -635,6 +638,11 @@ def main():
                      "timed_steps": dom[2],
                      "timed_every_nth_step": PROFILE_EVERY},
         "layer_tflops": layer_flops * world * K / (total_ms / 1e3) / 1e12,
+        "layer_tflops_counting": "causal attention counted as 2h'k(k+1) forward, "
+                                 "5h'k(k+1) backward",
+        "layer_tflops_paper_count": layer_flops_full * world * K / (total_ms / 1e3) / 1e12,
+        "layer_tflops_paper_counting": "attention counted as the paper's App. A does, "
+                                       "4h'k^2 forward (no causal halving), 10h'k^2 backward",
         "stage_ms": {s: round(v, 5) for s, v in stage_ms.items()},
         "e2e": {"value": e2e_value, "unit": "tokens/s",
                 "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h,

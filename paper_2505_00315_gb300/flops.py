@@ -45,17 +45,20 @@ def isoflop_heads(layers: int, h: int, hp: int, T: int, n_heads_dense_baseline: 
     return (budget - fixed) // (layers * head_flops_mosa(h, hp, T, k))
 
 
-def layer_work(B: int, T: int, d: int, H: int, hp: int, k: int, elem_bytes: int = 2) -> dict:
+def layer_work(B: int, T: int, d: int, H: int, hp: int, k: int, elem_bytes: int = 2,
+               causal: bool = True) -> dict:
     """Algorithmic FLOPs and HBM bytes of one MoSA layer, per step of the
     forward (F1-F5) and backward (B1-B4) pass, summed over all B*H units.
 
     FLOPs: router 2dT per (b,h); projections 6dh'k; causal attention
     2h'k(k+1) forward and 5h'k(k+1) backward; output 2h'dk; output backward
     4h'dk; input backward 6dh'k + 2dk; weight backward 6dh'k + 2dk.
+    ``causal=False`` counts attention as the paper does (App. A: 4h'k^2
+    forward, not halved for the mask) and 10h'k^2 backward.
     Bytes (minimum, each operand touched once): see the per-entry comments."""
     U = B * H
     e = elem_bytes
-    causal = hp * k * (k + 1)
+    causal = hp * k * (k + 1) if causal else 2 * hp * k * k
     w = {
         "router": {"flops": 2 * d * T * U,
                    # read X once, write r [B,H,T] fp32
@@ -104,18 +107,18 @@ def layer_work(B: int, T: int, d: int, H: int, hp: int, k: int, elem_bytes: int 
 
 
 def hybrid_work(B: int, T: int, d: int, H: int, hp: int, k: int, H_dense: int,
-                window: int = 0, elem_bytes: int = 2) -> dict:
+                window: int = 0, elem_bytes: int = 2, causal: bool = True) -> dict:
     """``layer_work`` of a hybrid layer (Sec. 2.2, hybridization; Sec. 3.4):
     the MoSA heads plus H_dense dense heads over all T tokens (window 0) or
     local heads over blocks of ``window`` tokens, per step, summed.  The dense
     heads have no router: no F1 work, their token lists are written once
     (8 bytes per row), and no dlogit terms in B3/B4."""
-    w = layer_work(B, T, d, H, hp, k, elem_bytes)
+    w = layer_work(B, T, d, H, hp, k, elem_bytes, causal)
     if H_dense <= 0:
         return w
     blk = window if window else T
     Bd = B * (T // blk)
-    dn = layer_work(Bd, blk, d, H_dense, hp, blk, elem_bytes)
+    dn = layer_work(Bd, blk, d, H_dense, hp, blk, elem_bytes, causal)
     rows = Bd * H_dense * blk
     dn["router"] = {"flops": 0, "bytes": 0}
     dn["select"] = {"flops": 0, "bytes": 2 * rows * 4}

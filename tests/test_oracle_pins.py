@@ -590,3 +590,15 @@ def test_hybrid_work_adds_dense_and_local_heads():
         assert h["w_bwd"]["flops"] - base["w_bwd"]["flops"] == 6 * d * hp * blk * U
         assert h["forward_flops"] == sum(h[s]["flops"] for s in
                                          ("router", "select", "qkv", "attn_fwd", "out"))
+
+
+def test_paper_count_matches_app_a_head_formula():
+    # with attention not halved for the mask, the layer's forward FLOPs are
+    # App. A's MoSA head cost per (b, h) minus its h'k scaling term, which the
+    # library's count leaves out
+    B, T, d, H, hp, k = 2, 1024, 512, 16, 64, 128
+    w = flops.layer_work(B, T, d, H, hp, k, causal=False)
+    assert w["forward_flops"] + B * H * hp * k == B * H * flops.head_flops_mosa(d, hp, T, k)
+    assert w["attn_bwd"]["flops"] == 10 * hp * k * k * B * H
+    c = flops.layer_work(B, T, d, H, hp, k)
+    assert c["attn_fwd"]["flops"] == 2 * hp * k * (k + 1) * B * H < w["attn_fwd"]["flops"]

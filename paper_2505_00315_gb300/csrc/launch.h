@@ -131,12 +131,12 @@ cudaError_t tc_out_bwd_w(const Dims &dm, const void *dY, const Saved &sv, float 
 cudaError_t tc_in_bwd(const Dims &dm, const void *Wq, const void *Wk, const void *Wv,
                       const void *Wr, const Saved &sv, float *dX, cudaStream_t s,
                       bool zero_output);
-// B3 as a persistent kernel over (head, 128-row tile, 256-column chunk) units.
-// F5 as the same persistent scatter product: Y[g(m), :] += AR(m, :) W_o[h]
-// (Y zeroed by the caller).
+// F5 as a persistent scatter product over (head, 128-row tile, 256-column
+// chunk) units: Y[g(m), :] += AR(m, :) W_o[h] (Y zeroed by the caller).
 cudaError_t tc_out_scatter(const Dims &dm, const void *Wo, const Saved &sv, float *Y,
                            cudaStream_t s);
-// Needs dX zeroed and sv.WrT (tc_transpose_wr).
+// B3 as the same persistent scatter product; needs dX zeroed and sv.WrT
+// (tc_transpose_wr).
 cudaError_t tc_dx(const Dims &dm, const void *Wq, const void *Wk, const void *Wv, const Saved &sv,
                   float *dX, cudaStream_t s);
 // F1 on tensor cores (bf16 inputs, H % 8 == 0); false if not applicable.

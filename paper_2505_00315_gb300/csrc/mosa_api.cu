@@ -90,9 +90,11 @@ mosa_status cuda_status(cudaError_t e) { return e == cudaSuccess ? MOSA_OK : MOS
 // ------------------------------------------------ concurrent branches
 // On the tensor-core path independent kernels run on a second, internal
 // stream joined back with events (graph branches when captured):
-//   forward:  zeroing Y runs beside router .. attention;
-//   backward: dW_o and the zeroing of dX and the weight gradients run beside
+//   forward:  zeroing Y runs beside TopK (forked after the router, joined
+//             before the output product);
+//   backward: dW_o, the W_r transpose and the zeroing of dX run beside
 //             G -> attention backward; then dX and dW run side by side.
+// A hybrid call runs the MoSA heads and then the dense heads, each this way.
 struct DevResources {
     cudaStream_t side = nullptr;
     cudaEvent_t ev[4] = {};

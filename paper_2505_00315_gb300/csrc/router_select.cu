@@ -5,8 +5,9 @@
 // image of the fp32 scores (4 passes of 8 bits, most significant first),
 // which finds the exact k-th largest key.  With first_token, token 0 gets a
 // key above every score's (0xFFFFFFFF; a finite or infinite score maps at most
-// to 0xFF800000), so it is always kept and the other k-1 come from the rest.  A final in-order compaction keeps
-// every key above it plus the lowest-index keys equal to it, so I comes out
+// to 0xFF800000), so it is always kept and the other k-1 come from the rest.
+// A final in-order compaction keeps every key above the k-th largest plus the
+// lowest-index keys equal to it, so I comes out
 // ascending (the order the causal mask works in) and ties go to the lower
 // token index.  Output positions come from one block-wide prefix sum of the
 // per-segment counts, so no sort is needed.

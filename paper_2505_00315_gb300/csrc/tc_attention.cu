@@ -6,7 +6,8 @@
 //   for each 128-key block j (causal: up to the tile's last query)
 //     S_j  = Q K_j^T                       tcgen05, fp32 in TMEM, two buffers
 //     P_j  = exp(S_j/sqrt(h') - m), running max m and sum l per row
-//     O   += P_j V_j                       tcgen05, P from shared memory, O in TMEM
+//     O   += P_j V_j                       tcgen05, O in TMEM; P read from TMEM
+//                                          (k > 128) or shared memory (k <= 128)
 //   A = O / l, AR = r A, lse = m + log l  (details at the kernel).
 // Q, K, V, P are bf16 hi/lo pairs (v ~ hi + lo), so each product is three
 // bf16 MMAs (hi*hi + hi*lo + lo*hi) into one fp32 accumulator, which keeps the

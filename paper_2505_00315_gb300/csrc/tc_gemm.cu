@@ -1,6 +1,6 @@
 // Per-head projections of the MoSA layer on the 5th-generation tensor cores
-// (tcgen05.mma, fp32 accumulators in TMEM), operands staged by TMA, with the
-// gathers through the selected token indices done by TMA gather4 loads.
+// (tcgen05.mma, fp32 accumulators in TMEM): dense operands staged by TMA, the
+// rows gathered through the selected token indices by 16-byte cp.async copies.
 //
 // One CTA computes one 128-row output tile of one head (or one split of the
 // reduction for the weight gradients).  Warp roles (256 threads):
@@ -10,7 +10,10 @@
 //   warps 4-7   gathered operand: 16-byte cp.async copies of the selected rows,
 //               written in the 128-byte-swizzled layout (TMA gather4 issues
 //               only ~4 rows per ~80 cycles per SM, too slow here); then the
-//               epilogue: tcgen05.ld of the accumulator rows, fused output
+//               epilogue: tcgen05.ld of the accumulator rows and the fused
+//               output step of each variant.  Wide tiles (kQKV, kDWO, kDW,
+//               kROUTER) split the epilogue over all eight warps, two per TMEM
+//               lane quadrant, each taking half of the columns.
 // Every mbarrier wait is bounded; a wait that runs out sets kStatusTimeout in
 // the workspace status word and the CTA winds down without hanging.
 //

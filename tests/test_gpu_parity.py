@@ -374,6 +374,23 @@ def test_invalid_indices_are_flagged_not_followed():
     assert mosa.mosa_check_status(shape, ws) == 0          # cleared by the read
 
 
+def test_status_word_maps_to_error_codes():
+    # A bounded device wait that gives up sets the timeout bit in the
+    # workspace status word; here the bits are written from the host (no
+    # kernel waits or faults) and the read maps them to error codes, timeout
+    # first, and clears the word.
+    X = torch.zeros((1, 16, 32), dtype=torch.float32, device="cuda")
+    Wq = torch.zeros((2, 32, 32), dtype=torch.float32, device="cuda")
+    shape = mosa.make_shape(X, Wq, 4)
+    ws = mosa.alloc_workspace(shape)
+    ws.zero_()
+    for word, code in ((2, 4), (3, 4), (1, 1), (0, 0)):   # timeout, both, bad index, none
+        ws[:4].copy_(torch.tensor(list(word.to_bytes(4, "little")), dtype=torch.uint8))
+        assert mosa.mosa_check_status(shape, ws) == code, word
+        assert mosa.mosa_check_status(shape, ws) == 0      # cleared by the read
+        assert int(ws[:4].sum().item()) == 0
+
+
 def test_workspace_reuse_gives_same_result():
     cfg = W.CONFIGS["B8_T1024_d512_H16_k128"].with_(B=2)
     x = W.make_inputs(cfg)

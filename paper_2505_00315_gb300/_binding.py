@@ -195,6 +195,28 @@ def _same(ref, *ts):
             raise TypeError(f"{name} must have the storage dtype {ref.dtype}")
 
 
+def _shapes(**named):
+    """Check each tensor's shape: name=(tensor, expected shape).  The library
+    sees plain pointers, so a wrong shape here would mean out-of-range
+    accesses there; None tensors are skipped."""
+    for name, (t, want) in named.items():
+        if t is not None and tuple(t.shape) != tuple(want):
+            raise ValueError(f"{name} must have shape {tuple(want)}, got {tuple(t.shape)}")
+
+
+def _layer_shapes(X, W_r, W_q, W_k, W_v, W_o, k=None, I=None, r_sel=None, dY=None):
+    """Shapes of the layer's inputs against X [B,T,d] and W_q [H,d,hp]."""
+    if X.dim() != 3 or W_q.dim() != 3:
+        raise ValueError("X must be [B, T, d] and W_q [H, d, hp]")
+    B, T, d = X.shape
+    H, _, hp = W_q.shape
+    _shapes(W_q=(W_q, (H, d, hp)), W_r=(W_r, (d, H)), W_k=(W_k, (H, d, hp)),
+            W_v=(W_v, (H, d, hp)), W_o=(W_o, (H, hp, d)), dY=(dY, (B, T, d)))
+    if k is not None:
+        _shapes(I=(I, (B, H, k)), r_sel=(r_sel, (B, H, k)))
+    return B, T, d, H, hp
+
+
 def mosa_forward(X, W_r, W_q, W_k, W_v, W_o, k: int, workspace=None, want_r_full=False,
                  out=None, stream=None, first_token: bool = False, rope: bool = False):
     """Forward pass (Sec. 2.2).  Returns (Y, I, r_sel, r_full or None, workspace).
@@ -204,11 +226,14 @@ def mosa_forward(X, W_r, W_q, W_k, W_v, W_o, k: int, workspace=None, want_r_full
     (Sec. 3.2); with ``rope`` Q and K are rotated at the tokens' original
     positions (Sec. 2.2), and the backward must be given ``rope`` too."""
     torch = _torch()
+    _layer_shapes(X, W_r, W_q, W_k, W_v, W_o)
     shape = make_shape(X, W_q, k, first_token, rope)
     _same(X, ("W_r", W_r), ("W_q", W_q), ("W_k", W_k), ("W_v", W_v), ("W_o", W_o))
     B, T, d, H = shape.B, shape.T, shape.d, shape.H
     dev = X.device
     out = out or {}
+    _shapes(Y=(out.get("Y"), (B, T, d)), I=(out.get("I"), (B, H, k)),
+            r_sel=(out.get("r_sel"), (B, H, k)), r_full=(out.get("r_full"), (B, H, T)))
     Y = out.get("Y") if out.get("Y") is not None else torch.empty((B, T, d), dtype=torch.float32, device=dev)
     I = out.get("I") if out.get("I") is not None else torch.empty((B, H, k), dtype=torch.int32, device=dev)
     rs = out.get("r_sel") if out.get("r_sel") is not None else torch.empty((B, H, k), dtype=torch.float32, device=dev)
@@ -232,6 +257,9 @@ def mosa_forward_with_indices(X, W_q, W_k, W_v, W_o, I, r_sel, workspace=None, o
     """Forward with caller-chosen token sets (e.g. the fixed-sparse case of
     Sec. 3.1).  Returns (Y, workspace)."""
     torch = _torch()
+    B_, T_, d_, H_, _ = _layer_shapes(X, None, W_q, W_k, W_v, W_o, k=I.shape[-1], I=I,
+                                      r_sel=r_sel)
+    _shapes(Y=((out or {}).get("Y"), (B_, T_, d_)))
     shape = make_shape(X, W_q, I.shape[-1], rope=rope)
     _same(X, ("W_q", W_q), ("W_k", W_k), ("W_v", W_v), ("W_o", W_o))
     B, T, d = shape.B, shape.T, shape.d
@@ -254,6 +282,7 @@ def mosa_backward(X, W_r, W_q, W_k, W_v, W_o, I, r_sel, dY, workspace, out=None,
     """Backward pass; returns a dict with dX, dW_r, dW_q, dW_k, dW_v, dW_o (fp32).
     ``rope`` must match the forward's."""
     torch = _torch()
+    _layer_shapes(X, W_r, W_q, W_k, W_v, W_o, k=I.shape[-1], I=I, r_sel=r_sel, dY=dY)
     shape = make_shape(X, W_q, I.shape[-1], rope=rope)
     _same(X, ("W_r", W_r), ("W_q", W_q), ("W_k", W_k), ("W_v", W_v), ("W_o", W_o), ("dY", dY))
     dev = X.device
@@ -263,6 +292,8 @@ def mosa_backward(X, W_r, W_q, W_k, W_v, W_o, I, r_sel, dY, workspace, out=None,
                        ("dW_o", W_o)):
         if g.get(name) is None:
             g[name] = torch.empty(like.shape, dtype=f32, device=dev)
+        else:
+            _shapes(**{name: (g[name], like.shape)})
     rc = load().mosa_backward(
         ctypes.byref(shape), _dev(X, "X"), _dev(W_r, "W_r"), _dev(W_q, "W_q"), _dev(W_k, "W_k"),
         _dev(W_v, "W_v"), _dev(W_o, "W_o"), _dev(I, "I", torch.int32),
@@ -286,6 +317,7 @@ def mosa_topk(scores, k: int, out=None, stream=None):
         I = torch.empty(lead + (k,), dtype=torch.int32, device=scores.device)
     if rs is None:
         rs = torch.empty(lead + (k,), dtype=torch.float32, device=scores.device)
+    _shapes(I=(I, lead + (k,)), r_sel=(rs, lead + (k,)))
     rc = load().mosa_topk(rows, T, int(k), _dev(scores, "scores", torch.float32),
                           _dev(I, "I", torch.int32), _dev(rs, "r_sel", torch.float32),
                           _stream(stream))
@@ -354,12 +386,14 @@ def mosa_route_noalloc(X, W_r, k: int, hp: int = 64, out=None, stream=None,
     H = W_r.shape[1]
     shape = MosaShape(B, T, d, H, int(hp), int(k), _dtype_code(X), 1 if first_token else 0)
     _same(X, ("W_r", W_r))
+    _shapes(W_r=(W_r, (d, H)))
     I = (out or {}).get("I")
     rs = (out or {}).get("r_sel")
     if I is None:
         I = torch.empty((B, H, k), dtype=torch.int32, device=X.device)
     if rs is None:
         rs = torch.empty((B, H, k), dtype=torch.float32, device=X.device)
+    _shapes(I=(I, (B, H, k)), r_sel=(rs, (B, H, k)))
     rc = load().mosa_route_noalloc(ctypes.byref(shape), _dev(X, "X"), _dev(W_r, "W_r"),
                                    _dev(I, "I", torch.int32), _dev(rs, "r_sel", torch.float32),
                                    _stream(stream))
@@ -368,6 +402,17 @@ def mosa_route_noalloc(X, W_r, k: int, hp: int = 64, out=None, stream=None,
 
 
 # ------------------------------------------------------------ hybrid layers
+
+def _hybrid_shapes(X, W_r, W_q, W_k, W_v, W_o, D_q, D_k, D_v, D_o, **kw):
+    """Shapes of a hybrid call: the MoSA heads' as _layer_shapes, and the dense
+    heads' D_q, D_k, D_v [H_dense, d, hp], D_o [H_dense, hp, d]."""
+    B, T, d, H, hp = _layer_shapes(X, W_r, W_q, W_k, W_v, W_o, **kw)
+    if D_q.dim() != 3:
+        raise ValueError("D_q must be [H_dense, d, hp]")
+    Hd = D_q.shape[0]
+    _shapes(D_q=(D_q, (Hd, d, hp)), D_k=(D_k, (Hd, d, hp)), D_v=(D_v, (Hd, d, hp)),
+            D_o=(D_o, (Hd, hp, d)))
+
 
 def make_hybrid_shape(X, W_q, k: int, H_dense: int, window: int = 0,
                       first_token: bool = False, rope: bool = False) -> MosaHybridShape:
@@ -395,12 +440,15 @@ def mosa_hybrid_forward(X, W_r, W_q, W_k, W_v, W_o, D_q, D_k, D_v, D_o, k: int,
     (local heads with ``window`` > 0), summed into Y.  Returns
     (Y, I, r_sel, workspace)."""
     torch = _torch()
+    _hybrid_shapes(X, W_r, W_q, W_k, W_v, W_o, D_q, D_k, D_v, D_o)
     shape = make_hybrid_shape(X, W_q, k, D_q.shape[0], window, first_token, rope)
     _same(X, ("W_r", W_r), ("W_q", W_q), ("W_k", W_k), ("W_v", W_v), ("W_o", W_o),
           ("D_q", D_q), ("D_k", D_k), ("D_v", D_v), ("D_o", D_o))
     B, T, d, H = X.shape[0], X.shape[1], X.shape[2], W_q.shape[0]
     dev = X.device
     out = out or {}
+    _shapes(Y=(out.get("Y"), (B, T, d)), I=(out.get("I"), (B, H, k)),
+            r_sel=(out.get("r_sel"), (B, H, k)))
     Y = out.get("Y") if out.get("Y") is not None else torch.empty((B, T, d), dtype=torch.float32, device=dev)
     I = out.get("I") if out.get("I") is not None else torch.empty((B, H, k), dtype=torch.int32, device=dev)
     rs = out.get("r_sel") if out.get("r_sel") is not None else torch.empty((B, H, k), dtype=torch.float32, device=dev)
@@ -423,6 +471,8 @@ def mosa_hybrid_backward(X, W_r, W_q, W_k, W_v, W_o, D_q, D_k, D_v, D_o, I, r_se
     dW_r, dW_q, dW_k, dW_v, dW_o (MoSA heads) and dD_q, dD_k, dD_v, dD_o
     (dense heads), fp32.  ``window`` and ``rope`` must match the forward's."""
     torch = _torch()
+    _hybrid_shapes(X, W_r, W_q, W_k, W_v, W_o, D_q, D_k, D_v, D_o, k=I.shape[-1], I=I,
+                   r_sel=r_sel, dY=dY)
     shape = make_hybrid_shape(X, W_q, I.shape[-1], D_q.shape[0], window, rope=rope)
     _same(X, ("W_r", W_r), ("W_q", W_q), ("W_k", W_k), ("W_v", W_v), ("W_o", W_o),
           ("D_q", D_q), ("D_k", D_k), ("D_v", D_v), ("D_o", D_o), ("dY", dY))
@@ -434,6 +484,8 @@ def mosa_hybrid_backward(X, W_r, W_q, W_k, W_v, W_o, D_q, D_k, D_v, D_o, I, r_se
                        ("dD_o", D_o)):
         if g.get(name) is None:
             g[name] = torch.empty(like.shape, dtype=f32, device=dev)
+        else:
+            _shapes(**{name: (g[name], like.shape)})
     grads = [_dev(g[n], n, f32) for n in ("dX", "dW_r", "dW_q", "dW_k", "dW_v", "dW_o", "dD_q",
                                           "dD_k", "dD_v", "dD_o")]
     rc = load().mosa_hybrid_backward(

@@ -26,9 +26,9 @@
  *       dW_r      [d,H]  dW_q,dW_k,dW_v [H,d,h']  dW_o [H,h',d]   fp32
  *   - Calls are asynchronous on `stream` (a cudaStream_t, NULL = legacy default
  *     stream).  They return after argument validation and kernel launch.
- *   - mosa_forward, mosa_forward_with_indices and mosa_backward capture their
- *     launch sequence into a CUDA graph the first time they see a given
- *     shape, set of pointers and kernel path, and replay that graph on later
+ *   - mosa_forward, mosa_forward_with_indices, mosa_backward and the hybrid
+ *     calls capture their launch sequence into a CUDA graph the first time
+ *     they see a given shape, set of pointers and kernel path, and replay that graph on later
  *     identical calls (one launch instead of about a dozen).  The capture runs
  *     on an internal stream of the current device.  Up to 128 graphs are kept
  *     (driver resources, no user memory); further new calls run unrecorded.
@@ -241,9 +241,12 @@ mosa_status mosa_route_noalloc(const mosa_shape *shape, const void *X, const voi
                                int32_t *I, float *r_sel, void *stream);
 
 /* ---- Measurement support (not part of the layer) ----------------------
- * Stages, in launch order: 0 router, 1 select, 2 qkv, 3 attn_fwd, 4 out,
- * 5 out_bwd, 6 attn_bwd, 7 in_bwd, 8 w_bwd (9 reserved).  These calls create
- * CUDA events (host-side handles, no device memory) when stage timing is on. */
+ * Stages: 0 router, 1 select, 2 qkv, 3 attn_fwd, 4 out, 5 out_bwd,
+ * 6 attn_bwd, 7 in_bwd, 8 w_bwd, 9 dwo (dW_o), 10 fwd_unit (F3-F5 fused,
+ * k <= 128), 11 bwd_unit (G, row terms and attention backward fused, k <= 128,
+ * opt-in).  A hybrid call times each stage once per head group.  These calls
+ * create CUDA events (host-side handles, no device memory) when stage timing
+ * is on. */
 
 /* Number of kernels this library has launched since it was loaded. */
 unsigned long long mosa_kernel_launches(void);

@@ -25,8 +25,11 @@ import threading
 import numpy as np
 
 _HERE = os.path.dirname(os.path.abspath(__file__))
-_SRC = os.path.join(_HERE, "mosa_oracle.c")
-_LIB = os.path.join(_HERE, "_build", "liboracle.so")
+# A test may point the oracle at a modified copy of its source (to check that
+# the pins catch planted mistakes); that copy's library is built beside it.
+_SRC = os.environ.get("MOSA_ORACLE_SRC") or os.path.join(_HERE, "mosa_oracle.c")
+_LIB = (os.path.splitext(_SRC)[0] + ".so" if os.environ.get("MOSA_ORACLE_SRC")
+        else os.path.join(_HERE, "_build", "liboracle.so"))
 _lock = threading.Lock()
 _lib = None
 

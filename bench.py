@@ -5,15 +5,16 @@
                     [--config NAME] [--no-cpu-baseline]
 
 A step is one forward and one backward pass of the layer over one batch of
-the workload (default: B=8 sequences of T=1024 tokens, d=512, H=16 heads of
-size 64, k=128 tokens per head, bf16 storage) with inputs resident in HBM.
+the workload (default: B=4 sequences of T=4096 tokens, d=1024, H=8 heads of
+size 64, k=2048 tokens per head, bf16 storage: the configuration with the
+most work per step) with inputs resident in HBM.
 L2 is flushed (a 256 MiB write) before every timed step, outside the step's
 CUDA events.  Under torchrun every rank runs its own copy of the workload
 (weak scaling, no collective on the data path); the reported time is the
 maximum over ranks.
 
 Rank 0 prints one JSON line: tokens/s, the roofline of the dominant kernel
-(timed live with CUDA events on the library's stream, every 8th timed step), the fp64 CPU oracle
+(timed live with CUDA events on the library's stream, every 2nd timed step), the fp64 CPU oracle
 timed on a bounded sample of the same workload, an end-to-end figure through
 the public API with host buffers, SM clocks sampled during the timed region
 and the number of library kernels launched.
@@ -39,7 +40,7 @@ sys.path.insert(0, ROOT)
 
 METRIC = "MoSA layer fwd+bwd tokens/s; achieved TFLOP/s and HBM GB/s vs GB300 peak"
 L2_FLUSH_BYTES = 256 << 20
-PROFILE_EVERY = 8   # timed steps per live timing of the dominant stage
+PROFILE_EVERY = 2   # timed steps per live timing of the dominant stage
 FALLBACK_PEAKS = {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "bf16_tflops_sustained": 1700.0,
                   "sm_max_mhz": 2070.0}
 NUM_SM = 152
@@ -177,6 +178,26 @@ def choose_sample(cfg, x, budget_s):
     return n, t1
 
 
+def single_thread_seconds():
+    """The oracle on one host thread: the whole fp32 forward-only workload
+    (B1 T256 d128 H4 k64) and the forward + backward of one sequence of
+    B8 T1024 d512 H16 k128."""
+    import oracle
+    from paper_2505_00315_gb300 import workloads as W
+    out = {}
+    n0 = oracle.num_threads()
+    oracle.set_num_threads(1)
+    try:
+        for name in ("f32_B1_T256_d128_H4_k64", "B8_T1024_d512_H16_k128"):
+            c = W.CONFIGS[name]
+            out[name] = {"seconds": round(oracle_sample(c, W.make_inputs(c), 1), 4),
+                         "sample": ("forward" if not c.backward else "forward+backward") +
+                                   " of 1 sequence"}
+    finally:
+        oracle.set_num_threads(n0)
+    return out
+
+
 def cpu_baseline(cfg, x, budget_s):
     import oracle
     n, t1 = choose_sample(cfg, x, budget_s)
@@ -185,7 +206,8 @@ def cpu_baseline(cfg, x, budget_s):
     return {"value": n * cfg.T / t, "unit": "tokens/s", "cores": oracle.num_threads(),
             "kind": "oracle",
             "sample": f"{what} of {n} of the {cfg.B} sequences of {cfg.name} "
-                      f"(all heads, fp64, {t:.2f} s)"}
+                      f"(all heads, fp64, {t:.2f} s)",
+            "single_thread": single_thread_seconds()}
 
 
 # ------------------------------------------------------------ roofline

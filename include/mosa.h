@@ -229,13 +229,17 @@ mosa_status mosa_check_status(const mosa_shape *shape, void *workspace, void *st
  * into the library (held on every GPU that loads it until the process
  * exits), so B*H*T may be at most 1,048,576 (else MOSA_ERR_UNSUPPORTED).
  *   X [B,T,d], W_r [d,H] : inputs (storage dtype); hp is validated but unused.
- *   I [B,H,k] int32, r_sel [B,H,k] fp32 : outputs, as mosa_forward.
- * The first call on a device looks up the array's device address (once per
- * device, with that device current); make that first call before any stream
- * capture.  All calls share the one array and the contents of the last call
- * remain in it; nothing needs clearing, because each call writes every score
- * it reads.  Calls whose GPU work overlaps (different streams or host
- * threads without ordering) race on the array: order them on one stream.
+ *   I [B,H,k] int32, r_sel [B,H,k] fp32 : outputs, as mosa_forward (the same
+ *   router kernel computes the scores, so the results are identical).
+ * Every call looks up the array's device address on the current device (the
+ * host-side symbol is not a device address); the first call on a device also
+ * loads the library's device code there, so make it before any stream
+ * capture.  After a cudaDeviceReset the next call finds the array anew.
+ * All calls share the one array and the contents of the last call remain in
+ * it; nothing needs clearing, because each call writes every score it reads.
+ * Calls whose GPU work overlaps (different streams or host threads without
+ * ordering) race on the array: order them on one stream.  There is no status
+ * word: a bounded device wait that runs out leaves I and r_sel undefined.
  * Returns MOSA_OK, MOSA_ERR_INVALID_ARG, MOSA_ERR_UNSUPPORTED or MOSA_ERR_CUDA. */
 mosa_status mosa_route_noalloc(const mosa_shape *shape, const void *X, const void *W_r,
                                int32_t *I, float *r_sel, void *stream);

@@ -3,11 +3,12 @@
 // returns the launch status; none synchronizes.
 #pragma once
 
+#include <cstdlib>
+#include <mutex>
+#include <set>
 #include <utility>
 
 #include "common.cuh"
-
-#include <cstdlib>
 
 namespace mosa {
 
@@ -37,6 +38,22 @@ template <typename... KArgs, typename... Args>
 inline cudaError_t launch_pdl(void (*kernel)(KArgs...), dim3 grid, dim3 block, size_t smem,
                               cudaStream_t s, Args &&...args) {
     return launch_ex(true, kernel, grid, block, smem, s, std::forward<Args>(args)...);
+}
+
+// Raises `kernel`'s dynamic shared-memory limit to `bytes` on the current
+// device.  The attribute is per device, so it is set once for each device
+// (and each kernel) a process uses.
+inline cudaError_t allow_smem(const void *kernel, int bytes) {
+    static std::mutex mu;
+    static std::set<std::pair<int, const void *>> done;
+    int dev = 0;
+    cudaError_t e = cudaGetDevice(&dev);
+    if (e != cudaSuccess) return e;
+    std::lock_guard<std::mutex> lk(mu);
+    if (done.count({dev, kernel})) return cudaSuccess;
+    e = cudaFuncSetAttribute(kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, bytes);
+    if (e == cudaSuccess) done.insert({dev, kernel});
+    return e;
 }
 
 // RoPE (Sec. 2.2) angle table for head size hp and sequences of T tokens.

@@ -8,8 +8,6 @@
 // or loops that must never trigger cudaMalloc's implicit device-wide
 // synchronisation.  For them mosa_route_noalloc keeps the scores in a fixed
 // array compiled into this library instead.
-#include <mutex>
-
 #include "../../include/mosa.h"
 #include "launch.h"
 
@@ -22,25 +20,24 @@ constexpr size_t kRouteScratchScores = size_t(1) << 20;
 
 __device__ __align__(256) float g_route_scores[kRouteScratchScores];
 
-constexpr int kMaxDevices = 64;
-std::mutex g_mu;
-float *g_scores_on[kMaxDevices] = {};
+// Status word for the router's bounded waits (there is no workspace to hold
+// one).  Nothing reads it back: a wait that runs out (a GPU that stopped
+// making progress for 2 s) leaves that call's I and r_sel undefined.
+__device__ __align__(256) uint32_t g_route_status;
 
-// Device address of g_route_scores on the current device, looked up once per
-// device (the host-side symbol is only a stand-in and must not reach a kernel).
-cudaError_t scores_address(float **out) {
-    int dev = 0;
-    cudaError_t e = cudaGetDevice(&dev);
+// Device addresses of the two arrays on the current device.  They are looked
+// up on every call (cheap once the library's device code is loaded) rather
+// than cached: a device reset reloads the module, and a cached address could
+// then point at freed memory.  The host-side symbols are only stand-ins and
+// must never reach a kernel.
+cudaError_t scratch_addresses(float **scores, uint32_t **status) {
+    void *p = nullptr;
+    cudaError_t e = cudaGetSymbolAddress(&p, g_route_scores);
     if (e != cudaSuccess) return e;
-    if (dev < 0 || dev >= kMaxDevices) return cudaErrorInvalidDevice;
-    std::lock_guard<std::mutex> lk(g_mu);
-    if (g_scores_on[dev] == nullptr) {
-        void *p = nullptr;
-        e = cudaGetSymbolAddress(&p, g_route_scores);
-        if (e != cudaSuccess) return e;
-        g_scores_on[dev] = static_cast<float *>(p);
-    }
-    *out = g_scores_on[dev];
+    *scores = static_cast<float *>(p);
+    e = cudaGetSymbolAddress(&p, g_route_status);
+    if (e != cudaSuccess) return e;
+    *status = static_cast<uint32_t *>(p);
     return cudaSuccess;
 }
 
@@ -66,13 +63,16 @@ extern "C" mosa_status mosa_route_noalloc(const mosa_shape *shape, const void *X
         return MOSA_ERR_INVALID_ARG;
     if ((size_t)shape->B * shape->H * shape->T > kRouteScratchScores) return MOSA_ERR_UNSUPPORTED;
     float *scores = nullptr;
-    if (scores_address(&scores) != cudaSuccess) return MOSA_ERR_CUDA;
+    uint32_t *status = nullptr;
+    if (scratch_addresses(&scores, &status) != cudaSuccess) return MOSA_ERR_CUDA;
     const Dims dm{shape->B, shape->T, shape->d, shape->H, shape->hp, shape->k,
                   shape->dtype == MOSA_BF16, shape->first_token != 0, shape->rope != 0};
     cudaStream_t s = static_cast<cudaStream_t>(stream);
     // Every score the selection reads is written by the router first, so the
-    // array needs no clearing between calls.
-    if (launch_router(dm, X, W_r, scores, s) != cudaSuccess) return MOSA_ERR_CUDA;
+    // array needs no clearing between calls.  The router is chosen as in
+    // mosa_forward (tensor cores for bf16 with H % 8 == 0), so both entry
+    // points compute the same scores bit for bit.
+    if (launch_router_auto(dm, X, W_r, scores, status, s) != cudaSuccess) return MOSA_ERR_CUDA;
     if (launch_select(dm.B * dm.H, dm.T, dm.k, scores, I, r_sel, 0, 1, nullptr, nullptr, s,
                       dm.first_token) !=
         cudaSuccess)

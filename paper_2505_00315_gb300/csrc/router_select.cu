@@ -253,12 +253,8 @@ cudaError_t launch_select(int rows, int T, int k, const float *scores, int32_t *
                           int B, int H, int32_t *gidx, float *rsel_hm, cudaStream_t stream,
                           bool first_token) {
     if (rows <= 0) return cudaSuccess;
-    static std::once_flag once;
-    static cudaError_t attr = cudaSuccess;
-    std::call_once(once, [] {
-        attr = cudaFuncSetAttribute(topk_select_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                    kSelStagedMax * (int)sizeof(uint32_t));
-    });
+    const cudaError_t attr =
+        allow_smem((const void *)topk_select_kernel, kSelStagedMax * (int)sizeof(uint32_t));
     if (attr != cudaSuccess) return attr;
     const size_t smem = T <= kSelStagedMax ? sizeof(uint32_t) * (size_t)T : 0;
     // about four keys per thread, 256..1024 threads; at most 512 once rows fill

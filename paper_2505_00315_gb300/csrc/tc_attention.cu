@@ -1003,15 +1003,8 @@ cudaError_t tc_attn_fwd(const Dims &dm, const Saved &sv, cudaStream_t s) {
     p.AR = static_cast<bf16 *>(sv.AR);
     p.lse = sv.lse;
     p.status = sv.status;
-    static std::once_flag once;
-    static cudaError_t attr = cudaSuccess;
-    std::call_once(once, [] {
-        attr = cudaFuncSetAttribute(attn_fwd_tc_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                    kFwdLargeSmem);
-        if (attr == cudaSuccess)
-            attr = cudaFuncSetAttribute(attn_fwd_small_kernel,
-                                        cudaFuncAttributeMaxDynamicSharedMemorySize, kSmallFwdSmem);
-    });
+    cudaError_t attr = allow_smem((const void *)attn_fwd_tc_kernel, kFwdLargeSmem);
+    if (attr == cudaSuccess) attr = allow_smem((const void *)attn_fwd_small_kernel, kSmallFwdSmem);
     if (attr != cudaSuccess) return attr;
     if (small) {
         cudaError_t e = launch_pdl(attn_fwd_small_kernel, dim3(1, (dm.B + p.U - 1) / p.U, dm.H),
@@ -1050,13 +1043,7 @@ cudaError_t tc_attn_bwd(const Dims &dm, const Saved &sv, cudaStream_t s) {
         sp.Dd = sv.Dd;
         sp.dQKV = static_cast<bf16 *>(sv.dQKV);
         sp.status = sv.status;
-        static std::once_flag once_small;
-        static cudaError_t attr_small = cudaSuccess;
-        std::call_once(once_small, [] {
-            attr_small = cudaFuncSetAttribute(attn_bwd_small_kernel,
-                                              cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                              kSmallBwdSmem);
-        });
+        const cudaError_t attr_small = allow_smem((const void *)attn_bwd_small_kernel, kSmallBwdSmem);
         if (attr_small != cudaSuccess) return attr_small;
         cudaError_t e = launch_pdl(attn_bwd_small_kernel, dim3(1, (dm.B + sp.U - 1) / sp.U, dm.H),
                                    dim3(kSmallThreads), kSmallBwdSmem, s, sp);
@@ -1082,12 +1069,7 @@ cudaError_t tc_attn_bwd(const Dims &dm, const Saved &sv, cudaStream_t s) {
     bp.dQacc = sv.G;
     bp.status = sv.status;
     const size_t rows = (size_t)dm.H * dm.B * dm.k;
-    static std::once_flag once;
-    static cudaError_t attr = cudaSuccess;
-    std::call_once(once, [] {
-        attr = cudaFuncSetAttribute(attn_bwd_tc_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                    kBwdLargeSmem);
-    });
+    const cudaError_t attr = allow_smem((const void *)attn_bwd_tc_kernel, kBwdLargeSmem);
     if (attr != cudaSuccess) return attr;
     cudaError_t e = cudaMemsetAsync(sv.G, 0, sizeof(float) * rows * 64, s);
     if (e != cudaSuccess) return e;

@@ -265,12 +265,7 @@ cudaError_t launch_scatter_product(DxParams &p, const Dims &dm, cudaStream_t s) 
     p.mt = (Mtok + 127) / 128;
     p.nch = (dm.d + kChunk - 1) / kChunk;
     p.units = (long long)dm.H * p.mt * p.nch;
-    static std::once_flag once;
-    static cudaError_t attr = cudaSuccess;
-    std::call_once(once, [] {
-        attr = cudaFuncSetAttribute(scatter_product_kernel<kOut>,
-                                    cudaFuncAttributeMaxDynamicSharedMemorySize, kSmem);
-    });
+    const cudaError_t attr = allow_smem((const void *)scatter_product_kernel<kOut>, kSmem);
     if (attr != cudaSuccess) return attr;
     int dev = 0, sms = 0;
     cudaError_t e = cudaGetDevice(&dev);

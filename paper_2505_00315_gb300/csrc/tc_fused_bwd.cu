@@ -391,11 +391,7 @@ cudaError_t tc_fused_backward(const Dims &dm, const void *W_o, const void *dY, c
     p.scale = 1.f / sqrtf(64.f);
     p.scale_log2 = 1.4426950408889634f / sqrtf(64.f);
     p.status = sv.status;
-    static std::once_flag once;
-    static cudaError_t attr = cudaSuccess;
-    std::call_once(once, [] {
-        attr = cudaFuncSetAttribute(fused_bwd_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, kSmem);
-    });
+    const cudaError_t attr = allow_smem((const void *)fused_bwd_kernel, kSmem);
     if (attr != cudaSuccess) return attr;
     const dim3 grid((dm.B + p.U - 1) / p.U, dm.H);
     cudaError_t e = launch_pdl(fused_bwd_kernel, grid, dim3(kThreads), kSmem, s, p);

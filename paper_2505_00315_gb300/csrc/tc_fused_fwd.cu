@@ -463,11 +463,7 @@ cudaError_t tc_fused_forward(const Dims &dm, const void *X, const void *Wq, cons
     p.rope_on = dm.rope ? 1 : 0;
     if (dm.rope) p.rope = make_rope_table(64, dm.T);
     p.status = sv.status;
-    static std::once_flag once;
-    static cudaError_t attr = cudaSuccess;
-    std::call_once(once, [] {
-        attr = cudaFuncSetAttribute(fused_fwd_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, kSmem);
-    });
+    const cudaError_t attr = allow_smem((const void *)fused_fwd_kernel, kSmem);
     if (attr != cudaSuccess) return attr;
     const dim3 grid((dm.B + p.U - 1) / p.U, dm.H);
     cudaError_t e = launch_pdl(fused_fwd_kernel, grid, dim3(kThreads), kSmem, s, p);

@@ -654,12 +654,7 @@ bool map_heads(CUtensorMap *m, const void *base, uint64_t H, uint64_t rows, uint
 template <int KIND>
 cudaError_t launch_kind(const TcParams &p, dim3 grid, cudaStream_t s, bool early = true) {
     constexpr int smem = smem_bytes<KIND>();
-    static std::once_flag once;
-    static cudaError_t attr = cudaSuccess;
-    std::call_once(once, [] {
-        attr = cudaFuncSetAttribute(tc_gemm_kernel<KIND>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                    smem);
-    });
+    const cudaError_t attr = allow_smem((const void *)tc_gemm_kernel<KIND>, smem);
     if (attr != cudaSuccess) return attr;
     cudaError_t e = launch_ex(early, tc_gemm_kernel<KIND>, grid, dim3(kThreads), smem, s, p);
     note_launches(1);

@@ -66,15 +66,16 @@ def test_variant_names_and_config():
 
 
 def test_reference_arm_prints_one_line():
-    # the oracle as the reference arm, one short step of the default workload
+    # the oracle as the reference arm, one short step
+    # (a small workload: one sequence of the default one takes the oracle ~20 s)
     out = subprocess.run([sys.executable, os.path.join(ROOT, "bench.py"), "--impl", "reference",
-                          "--steps", "1", "--warmup", "0"], capture_output=True, text=True,
-                         timeout=600, cwd=ROOT)
+                          "--config", "B8_T1024_d512_H16_k128", "--steps", "1", "--warmup", "0"],
+                         capture_output=True, text=True, timeout=600, cwd=ROOT)
     assert out.returncode == 0, out.stderr[-2000:]
     lines = [l for l in out.stdout.splitlines() if l.startswith("{")]
     assert len(lines) == 1
     j = json.loads(lines[0])
     assert j["impl"] == "reference" and j["value"] > 0 and j["unit"] == "tokens/s"
-    assert j["config"]["workload"] == W.BENCH_CONFIG
+    assert j["config"]["workload"] == "B8_T1024_d512_H16_k128"
     assert j["cpu_baseline"]["kind"] == "oracle"
     assert j["e2e"]["h2d_bytes_per_step"] == 0

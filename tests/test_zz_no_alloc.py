@@ -6,8 +6,9 @@ only sees its inputs and outputs, a loop that may never trigger cudaMalloc's
 device-wide synchronisation.  For them the entry point keeps the router
 scores in a fixed 4 MiB array inside the library.  These tests call it
 through the C ABI and check that it selects exactly what mosa_forward
-selects, on two calls in a row (the second must not see the first's
-scores), and that it refuses problems larger than its array.  The file is
+selects and what the oracle selects, on two calls in a row (the second must
+not see the first's scores), and that it refuses problems larger than its
+array.  The file is
 named to be collected last."""
 import ctypes
 
@@ -32,7 +33,9 @@ def test_refuses_problems_beyond_its_array():
 
 
 @pytest.mark.gpu
-def test_matches_forward_on_two_calls_in_a_row():
+def test_matches_forward_and_oracle_on_two_calls_in_a_row():
+    import oracle
+    from _util import sigmoid_gap
     cases = [W.CONFIGS["B8_T1024_d512_H16_k128"],
              W.MosaConfig("second", B=3, T=500, d=136, H=5, hp=64, k=77, dtype="bf16", seed=31)]
     for cfg in cases:
@@ -42,6 +45,15 @@ def test_matches_forward_on_two_calls_in_a_row():
                                                    dev["Wv"], dev["Wo"], cfg.k)
         I, rs = mosa.mosa_route_noalloc(dev["X"], dev["Wr"], cfg.k, hp=cfg.hp)
         torch.cuda.synchronize()
-        np.testing.assert_array_equal(I.cpu().numpy(), I_ref.cpu().numpy())
-        a, b = rs.cpu().numpy().astype(np.float64), rs_ref.cpu().numpy().astype(np.float64)
-        assert np.linalg.norm(a - b) <= 1e-4 * np.linalg.norm(b)
+        I, rs = I.cpu().numpy(), rs.cpu().numpy()
+        # the same router kernel as mosa_forward: identical indices and scores
+        np.testing.assert_array_equal(I, I_ref.cpu().numpy())
+        np.testing.assert_array_equal(rs.view(np.uint32), rs_ref.cpu().numpy().view(np.uint32))
+        # and the oracle's selection (its k-th / (k+1)-th score gap is planted)
+        rf = oracle.router(x["X"], x["Wr"])
+        assert sigmoid_gap(rf, cfg.k) > 1e-3
+        for b in range(cfg.B):
+            for h in range(cfg.H):
+                Iref, rsref = oracle.topk(rf[b, h], cfg.k)
+                np.testing.assert_array_equal(I[b, h], Iref)
+                np.testing.assert_allclose(rs[b, h], rsref, rtol=1e-5, atol=0)

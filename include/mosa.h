@@ -40,10 +40,15 @@
  *     attention backward as one fused kernel; MOSA_PDL=0 turns programmatic
  *     dependent launch off.  All paths compute the same operation.
  *   - Outputs are overwritten, never accumulated into.
- *   - Arithmetic: fp32 accumulation everywhere; with bf16 storage the
- *     intermediates fed to tensor-core products (Q, K, V, P, the attention
- *     output, dA, dS, dQ|dK|dV) are kept as bf16 hi/lo pairs (v ~ hi + lo),
- *     which keeps those products at fp32-level accuracy.
+ *   - Arithmetic: fp32 accumulation everywhere.  With bf16 storage the
+ *     intermediates fed to tensor-core products are kept as bf16 hi/lo pairs
+ *     (v ~ hi + lo, fp32-level accuracy) where they meet the bf16 weights
+ *     (the attention output diag(r) A and dQ|dK|dV).  Inside the attention,
+ *     Q, K, V, P, dA and dS are pairs too for k <= 128, and single fp16
+ *     values (11-bit significand) for k > 128, one MMA per product: a value
+ *     beyond the fp16 range (|v| > 65504) is reported as MOSA_ERR_RANGE by
+ *     mosa_check_status() rather than passed on silently.  With fp32 storage
+ *     every intermediate is fp32.
  *   - Tokens tied on the router score are taken lowest index first.
  *   - NaN inputs give undefined results (but no out-of-bounds access).
  *   - Errors: a call that returns anything but MOSA_OK has launched nothing.
@@ -67,7 +72,8 @@ typedef enum {
     MOSA_ERR_UNSUPPORTED = 2,     /* valid but outside what the kernels implement */
     MOSA_ERR_CUDA = 3,            /* a CUDA runtime call or launch failed */
     MOSA_ERR_DEVICE_TIMEOUT = 4,  /* a bounded device-side wait gave up */
-    MOSA_ERR_WORKSPACE = 5        /* workspace NULL, too small or misaligned */
+    MOSA_ERR_WORKSPACE = 5,       /* workspace NULL, too small or misaligned */
+    MOSA_ERR_RANGE = 6            /* an fp16 attention intermediate overflowed (see below) */
 } mosa_status;
 
 typedef enum { MOSA_F32 = 0, MOSA_BF16 = 1 } mosa_dtype;
@@ -214,8 +220,10 @@ mosa_status mosa_topk(int32_t rows, int32_t T, int32_t k, const float *scores, i
                       float *r_sel, void *stream);
 
 /* Waits for `stream`, then reads and clears the device status word in the
- * workspace: MOSA_OK, MOSA_ERR_INVALID_ARG (caller indices were invalid) or
- * MOSA_ERR_DEVICE_TIMEOUT; MOSA_ERR_CUDA if the wait itself failed. */
+ * workspace: MOSA_OK, MOSA_ERR_INVALID_ARG (caller indices were invalid),
+ * MOSA_ERR_DEVICE_TIMEOUT or MOSA_ERR_RANGE (an fp16 intermediate of the
+ * k > 128 attention overflowed; the outputs are then not valid); MOSA_ERR_CUDA
+ * if the wait itself failed. */
 mosa_status mosa_check_status(const mosa_shape *shape, void *workspace, void *stream);
 
 

@@ -19,6 +19,7 @@ MOSA_ERR_UNSUPPORTED = 2
 MOSA_ERR_CUDA = 3
 MOSA_ERR_DEVICE_TIMEOUT = 4
 MOSA_ERR_WORKSPACE = 5
+MOSA_ERR_RANGE = 6
 MOSA_F32 = 0
 MOSA_BF16 = 1
 

@@ -14,6 +14,7 @@ namespace mosa {
 enum : uint32_t {
     kStatusBadIndex = 1u,  // caller-supplied indices out of range or not ascending
     kStatusTimeout = 2u,   // a bounded spin-wait gave up
+    kStatusRange = 4u,     // an fp16 intermediate of the k > 128 attention overflowed
 };
 
 using bf16 = __nv_bfloat16;

@@ -124,6 +124,10 @@ bool tc_supported(const Dims &dm);
 // True when the tensor-core kernels serve this shape (false also when the
 // environment variable MOSA_FORCE_SIMT is set to a non-zero value).
 bool use_tc(const Dims &dm);
+// True when the attention runs on fp16 operands (tensor cores, k > 128): Q,
+// K, V and dA are then stored as fp16 rows [H, B*k, 64], with RoPE applied
+// in the projection's epilogue; otherwise they are bf16 pairs (or fp32).
+bool attn_f16(const Dims &dm);
 // Fused F3 + F4 + F5 for k <= 128 (tc_fused_fwd.cu); off with MOSA_FUSED_FWD=0.
 bool tc_fused_forward_supported(const Dims &dm);
 bool use_fused_forward(const Dims &dm);

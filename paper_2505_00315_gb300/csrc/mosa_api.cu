@@ -146,7 +146,8 @@ mosa_status forward_heads(const Dims &dm, const void *X, const void *W_q, const 
     {
         StageScope st_(kStageQkv, s);
         MOSA_TRY(launch_qkv(dm, X, W_q, W_k, W_v, sv, s));
-        if (dm.rope) MOSA_TRY(rope_qk(dm, sv, false, s));
+        // (the fp16 attention path turns Q and K in the projection's epilogue)
+        if (dm.rope && !attn_f16(dm)) MOSA_TRY(rope_qk(dm, sv, false, s));
     }
     {
         StageScope st_(kStageAttnFwd, s);
@@ -197,7 +198,8 @@ mosa_status forward_tc(const Dims &dm, const void *X, const void *W_r, const voi
     {
         StageScope st_(kStageQkv, s);
         MOSA_TRY(launch_qkv(dm, X, W_q, W_k, W_v, sv, s));
-        if (dm.rope) MOSA_TRY(rope_qk(dm, sv, false, s));
+        // (the fp16 attention path turns Q and K in the projection's epilogue)
+        if (dm.rope && !attn_f16(dm)) MOSA_TRY(rope_qk(dm, sv, false, s));
     }
     {
         StageScope st_(kStageAttnFwd, s);
@@ -560,6 +562,8 @@ const char *mosa_status_string(mosa_status s) {
         case MOSA_ERR_CUDA: return "MOSA_ERR_CUDA: CUDA runtime error";
         case MOSA_ERR_DEVICE_TIMEOUT: return "MOSA_ERR_DEVICE_TIMEOUT: a bounded device wait gave up";
         case MOSA_ERR_WORKSPACE: return "MOSA_ERR_WORKSPACE: workspace missing, misaligned or too small";
+        case MOSA_ERR_RANGE:
+            return "MOSA_ERR_RANGE: an fp16 attention intermediate (k > 128) exceeded +-65504";
         default: return "unknown mosa_status";
     }
 }
@@ -746,6 +750,7 @@ mosa_status mosa_check_status(const mosa_shape *shape, void *workspace, void *st
     if (cudaMemset(workspace, 0, sizeof(word)) != cudaSuccess) return MOSA_ERR_CUDA;
     if (word & kStatusTimeout) return MOSA_ERR_DEVICE_TIMEOUT;
     if (word & kStatusBadIndex) return MOSA_ERR_INVALID_ARG;
+    if (word & kStatusRange) return MOSA_ERR_RANGE;
     return MOSA_OK;
 }
 

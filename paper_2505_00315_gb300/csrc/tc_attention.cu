@@ -9,9 +9,15 @@
 //     O   += P_j V_j                       tcgen05, O in TMEM; P read from TMEM
 //                                          (k > 128) or shared memory (k <= 128)
 //   A = O / l, AR = r A, lse = m + log l  (details at the kernel).
-// Q, K, V, P are bf16 hi/lo pairs (v ~ hi + lo), so each product is three
-// bf16 MMAs (hi*hi + hi*lo + lo*hi) into one fp32 accumulator, which keeps the
-// result at fp32-level accuracy.
+// Precision.  For k <= 128, Q, K, V, P, dA and dS are bf16 hi/lo pairs
+// (v ~ hi + lo), so each product is three bf16 MMAs (hi*hi + hi*lo + lo*hi)
+// into one fp32 accumulator, at fp32-level accuracy.  For k > 128 they are
+// single fp16 values (11-bit significand, 8 times finer than bf16) and each
+// product is one MMA; the operands that meet the bf16 weights outside the
+// attention (diag(r) A and dQ|dK|dV) stay pairs either way.  A measured
+// audit of the rounding of each intermediate against the stated tolerances
+// chose this split; an fp16 value at or beyond the fp16 range sets
+// kStatusRange instead of passing silently.
 // Backward (B2), flash-style with P recomputed from the saved log-sum-exp,
 // D = rowsum(dA o A) and dS = P o (dP - D): one CTA per (128-key tile, b, h)
 // over 128-query blocks: S = Q K^T, dP = dA V^T, then dV += P^T dA,
@@ -53,32 +59,32 @@ struct AttnParams {
 // Forward for k > 128 (F4), one CTA per (128-query tile, b, h), 384 threads:
 // warps 0-3 load, issue MMAs and own TMEM; warps 4-11 run the softmax, two per
 // TMEM lane quadrant (warp w: query rows 32 (w % 4) .. +31, keys
-// 64 ((w - 4) / 4) .. +63 of each 128-key block).  For key block j:
+// 64 ((w - 4) / 4) .. +63 of each 128-key block).  Q, K, V and P are fp16
+// (one MMA per 16-wide K step).  For key block j:
 //   S_j = Q K_j^T into TMEM buffer j % 2, issued two blocks ahead, so the
 //   MMAs of S_{j+2} and O += P_j V_j run while the softmax of block j+1 runs;
 //   P_j = exp2(S_j scale - m) with m the row's running maximum, updated only
 //   when the block's maximum exceeds it by more than 2^8 (O and l are then
-//   rescaled in place; otherwise P may reach 2^8, well inside fp32 and exact
-//   up to the pair rounding, and the final O / l uses the same m throughout);
-//   O accumulates in TMEM.  P_j (a bf16 pair) is written by the softmax warps
-//   into the TMEM columns of S_j itself (hi in the first 64 columns, lo in
-//   the next 64, two bf16 per column) and O += P_j V_j reads it from there as
-//   the A operand.  Measured on this GPU: a tcgen05.st issued while an MMA
-//   that reads its A operand from TMEM is still running corrupts that MMA's
-//   result even when the columns differ, so P_j is stored only after
+//   rescaled in place; otherwise P may reach 2^8, well inside the fp16 range,
+//   and the final O / l uses the same m throughout); O accumulates in TMEM.
+//   P_j is written by the softmax warps as fp16 into the first 64 TMEM
+//   columns of S_j itself (two per column) and O += P_j V_j reads it from
+//   there as the A operand.  Measured on this GPU: a tcgen05.st issued while
+//   an MMA that reads its A operand from TMEM is still running corrupts that
+//   MMA's result even when the columns differ, so P_j is stored only after
 //   P_{j-1} V_{j-1} has completed (its exponentials are computed meanwhile),
 //   and S_{j+2} (which overwrites P_j's columns) only after P_j V_j.
-// K and V blocks stream through a 4-slot ring in the order the MMAs use them:
-// K0, K1, V0, K2, V1, K3, ... (see kv_item).
+// K and V blocks stream through an 8-slot ring in the order the MMAs use
+// them: K0, K1, V0, K2, V1, K3, ... (see kv_item).
 constexpr int kLT = 384;              // threads
 constexpr int kLWorkers = 256;
 constexpr int kLKeys = 128;           // keys per block
-constexpr int kLSlots = 4;            // ring slots of one K or V block pair (32 KB)
+constexpr int kLSlots = 8;            // ring slots of one K or V block (16 KB)
 constexpr float kRescaleLog2 = 8.f;   // lazy-rescale threshold (log2 units)
 
 struct FwdLargeSmem {
-    uint8_t q[2][kTileHalf];                  // Q pair
-    uint8_t kv[kLSlots][2][kTileHalf];        // K or V block pairs
+    uint8_t q[kTileHalf];                     // Q, fp16 [128 x 64]
+    uint8_t kv[kLSlots][kTileHalf];           // K or V blocks, fp16 [128 x 64]
     float part[2][2][128];                    // [block parity][key half]: block max, final sums
     uint64_t q_full, kv_full[kLSlots], kv_empty[kLSlots], s_full[2], p_ready, pv_done;
     uint32_t tmem;
@@ -143,9 +149,8 @@ __global__ void __launch_bounds__(kLT, 1) attn_fwd_tc_kernel(const __grid_consta
     if (warp == 0) {
         if (lane == 0) {
             const uint32_t qb = smem_u32(&sm.q_full);
-            mbar_expect_tx(qb, 2 * kTileHalf);
-            tma_load_4d(smem_u32(sm.q[0]), &p.mQ, qb, 0, i0, b, h);
-            tma_load_4d(smem_u32(sm.q[1]), &p.mQ, qb, 64, i0, b, h);
+            mbar_expect_tx(qb, kTileHalf);
+            tma_load_4d(smem_u32(sm.q), &p.mQ, qb, 0, i0, b, h);
             for (int t = 0; t < nitems; ++t) {
                 const int s = t % kLSlots;
                 if (!lwait(sm, sm.kv_empty[s], ((t / kLSlots) & 1) ^ 1, p.status)) break;
@@ -153,16 +158,14 @@ __global__ void __launch_bounds__(kLT, 1) attn_fwd_tc_kernel(const __grid_consta
                 int blk;
                 kv_item(t, n, is_v, blk);
                 const uint32_t fb = smem_u32(&sm.kv_full[s]);
-                mbar_expect_tx(fb, 2 * kTileHalf);
-                const CUtensorMap *m = is_v ? &p.mV : &p.mK;
-                tma_load_4d(smem_u32(sm.kv[s][0]), m, fb, 0, blk * kLKeys, b, h);
-                tma_load_4d(smem_u32(sm.kv[s][1]), m, fb, 64, blk * kLKeys, b, h);
+                mbar_expect_tx(fb, kTileHalf);
+                tma_load_4d(smem_u32(sm.kv[s]), is_v ? &p.mV : &p.mK, fb, 0, blk * kLKeys, b, h);
             }
         }
     } else if (warp == 1) {
         if (lane == 0) {
-            constexpr uint32_t idS = idesc_bf16(128, kLKeys, false, false);
-            constexpr uint32_t idO = idesc_bf16(128, 64, false, true);
+            constexpr uint32_t idS = idesc_f16(128, kLKeys, false, false);
+            constexpr uint32_t idO = idesc_f16(128, 64, false, true);
             int t = 0;   // next K/V item to consume
             bool ok = lwait(sm, sm.q_full, 0, p.status);
             auto take = [&]() -> int {   // wait for item t, return its slot
@@ -175,8 +178,7 @@ __global__ void __launch_bounds__(kLT, 1) attn_fwd_tc_kernel(const __grid_consta
                 const int s = take();
                 if (!ok) return;
                 tc_fence_after();
-                mma_pair3(tmem + 128 * (j & 1), smem_u32(sm.q[0]), smem_u32(sm.q[1]),
-                          smem_u32(sm.kv[s][0]), smem_u32(sm.kv[s][1]), false, false, idS, false);
+                mma_k64_f16(tmem + 128 * (j & 1), smem_u32(sm.q), smem_u32(sm.kv[s]), idS);
                 mma_commit(smem_u32(&sm.s_full[j & 1]));
                 mma_commit(smem_u32(&sm.kv_empty[s]));
             };
@@ -187,18 +189,14 @@ __global__ void __launch_bounds__(kLT, 1) attn_fwd_tc_kernel(const __grid_consta
                 const int s = take();   // V_j
                 if (!ok) break;
                 tc_fence_after();
-                // O += P_j V_j: P (A operand) from the TMEM columns of S_j,
-                // hi at +0, lo at +64, 8 columns per 16 keys; V MN-major
+                // O += P_j V_j: P (A operand) from the first 64 TMEM columns of
+                // S_j, 8 columns per 16 keys; V MN-major
                 const uint32_t pa = tmem + 128 * (j & 1);
+                const uint32_t vb = smem_u32(sm.kv[s]);
 #pragma unroll
-                for (int tt = 0; tt < 3; ++tt) {
-                    const uint32_t a_col = pa + (tt == 2 ? 64 : 0);
-                    const uint32_t vb = smem_u32(sm.kv[s][tt == 1 ? 1 : 0]);
-#pragma unroll
-                    for (int kk = 0; kk < 8; ++kk)
-                        mma_bf16_ts(tO, a_col + 8 * kk, smem_desc_sw128(vb + kk * 2048, kTileHalf, 1024),
-                                    idO, (j > 0 || tt > 0 || kk > 0) ? 1u : 0u);
-                }
+                for (int kk = 0; kk < 8; ++kk)
+                    mma_bf16_ts(tO, pa + 8 * kk, smem_desc_sw128(vb + kk * 2048, kTileHalf, 1024), idO,
+                                (j > 0 || kk > 0) ? 1u : 0u);
                 mma_commit(smem_u32(&sm.pv_done));
                 mma_commit(smem_u32(&sm.kv_empty[s]));
                 if (j + 2 < n) {
@@ -259,10 +257,14 @@ __global__ void __launch_bounds__(kLT, 1) attn_fwd_tc_kernel(const __grid_consta
             const float m_new = grow ? mb : m;
             const float corr = grow ? exp2_fast(m - m_new) : 1.f;   // 0 on the first block
             float sm4[4] = {0.f, 0.f, 0.f, 0.f};
+            uint32_t pw[32];
 #pragma unroll
-            for (int c = 0; c < 64; ++c) {
-                s[c] = exp2_fast(fmaf(s[c], p.scale_log2, -m_new));
-                sm4[c & 3] += s[c];
+            for (int c = 0; c < 32; ++c) {
+                const float e0 = exp2_fast(fmaf(s[2 * c], p.scale_log2, -m_new));
+                const float e1 = exp2_fast(fmaf(s[2 * c + 1], p.scale_log2, -m_new));
+                sm4[(2 * c) & 3] += e0;
+                sm4[(2 * c + 1) & 3] += e1;
+                pw[c] = pack_f16x2(e0, e1);
             }
             l = l * corr + ((sm4[0] + sm4[1]) + (sm4[2] + sm4[3]));
             m = m_new;
@@ -279,17 +281,10 @@ __global__ void __launch_bounds__(kLT, 1) attn_fwd_tc_kernel(const __grid_consta
                 for (int c = 0; c < 32; ++c) o[c] *= corr;
                 tmem_st32(tO + lane_off + 32 * ch, o);
             }
-            // P_j as a pair into the columns of S_j: this thread's 64 keys are
-            // columns 32 ch .. +31 of the hi half and of the lo half (both
-            // threads of the row have read their S values: exchange barrier)
-            {
-                uint32_t hw[32], lw[32];
-#pragma unroll
-                for (int c = 0; c < 32; ++c) split_pair2(s[2 * c], s[2 * c + 1], hw[c], lw[c]);
-                const uint32_t pb = tmem + 128 * (j & 1) + lane_off + 32 * ch;
-                tmem_st32u(pb, hw);
-                tmem_st32u(pb + 64, lw);
-            }
+            // P_j as fp16 into the columns of S_j: this thread's 64 keys are
+            // columns 32 ch .. +31 (both threads of the row have read their S
+            // values: exchange barrier)
+            tmem_st32u(tmem + 128 * (j & 1) + lane_off + 32 * ch, pw);
             tc_fence_before();
             mbar_arrive(smem_u32(&sm.p_ready));
         }
@@ -305,7 +300,7 @@ __global__ void __launch_bounds__(kLT, 1) attn_fwd_tc_kernel(const __grid_consta
         const unsigned vmask = __ballot_sync(0xffffffffu, valid);
         const size_t row0 = (size_t)h * p.Mtok + (size_t)b * p.k + i0 + q * 32;
         if (live) {
-            uint8_t *xb = &sm.kv[0][0][0] + (warp - 4) * 4096;   // the ring is idle now
+            uint8_t *xb = &sm.kv[0][0] + (warp - 4) * 4096;   // the ring is idle now
             const float inv = valid ? 1.f / l : 0.f;
             const float rr = valid ? p.rsel[row0 + lane] : 0.f;
             stage_pair32(xb, o, inv * rr, lane);
@@ -353,31 +348,34 @@ __device__ __forceinline__ void flag_timeout_b(SM &sm, uint32_t *status) {
 // Backward for k > 128 (B2), one CTA per (128-key tile, b, h), 384 threads:
 // warps 0-3 load, issue MMAs and own TMEM; warps 4-11 compute P and dS, two
 // per TMEM lane quadrant (warp w: query rows 32 (w % 4) .. +31 of the current
-// block, keys 64 ((w - 4) / 4) .. +63 of the tile).  For each 128-query block
-// i at or after the tile (causal):
+// block, keys 64 ((w - 4) / 4) .. +63 of the tile).  Q, K, V, dA, P and dS
+// are fp16 (one MMA per 16-wide K step).  For each 128-query block i at or
+// after the tile (causal):
 //   S = Q_i K^T, dP = dA_i V^T                  (TMEM)
-//   P = exp(S / sqrt(h') - lse_i)               (pair tile; kept in registers)
+//   P = exp(S / sqrt(h') - lse_i)               (P tile; kept in registers)
 //   dV += P^T dA_i                              (TMEM, the tile read MN-major)
-//   dS = P o (dP - D_i)                         (pair tile, over P)
+//   dS = P o (dP - D_i)                         (dS tile)
 //   dK += dS^T Q_i, dQ_i = dS K                 (TMEM)
 //   dQ_i / sqrt(h') is added into an fp32 accumulator [H, B*k, 64] with
 //   vector reductions issued after the next block's P has been stored;
 // S_{i+1} is issued before dK_i and dQ_i, so the exponentials of block i+1
-// run on the workers while the tensor pipe works on block i;
-// dK / sqrt(h') and dV are written once at the end.  Q_i goes to slot i % 2
-// (it is needed until dK and dQ of block i), dA_i to slot 2 (free after dV),
-// so each load is issued at least half a block before its use.
+// run on the workers while the tensor pipe works on block i; P and dS have
+// tiles of their own, so dS_i is written while dV_i still reads P_i.
+// dK / sqrt(h') and dV are written once at the end as bf16 pairs.  Q_i and
+// dA_i go to ring slots 2 (i % 2) and 2 (i % 2) + 1, so each load is issued
+// a block ahead of its use.
 constexpr int kBT = 384;
 constexpr int kBWorkers = 256;
-constexpr int kBSlots = 3;
+constexpr int kBSlots = 4;
 
 struct BwdLargeSmem {
-    uint8_t k[2][kTileHalf];
-    uint8_t v[2][kTileHalf];
-    uint8_t ring[kBSlots][2][kTileHalf];   // Q_i or dA_i pairs
-    uint8_t ps[2][2][kTileHalf];           // P, then dS [half][64-key block]; dQ staging
+    uint8_t k[kTileHalf];                  // K tile, fp16 [128 keys x 64]
+    uint8_t v[kTileHalf];                  // V tile
+    uint8_t ring[kBSlots][kTileHalf];      // Q_i, dA_i (fp16 [128 queries x 64])
+    uint8_t p[2][kTileHalf];               // P [128 queries x 128 keys] as two 64-key blocks
+    uint8_t ds[2][kTileHalf];              // dS, the same layout
     uint64_t kv_full, ring_full[kBSlots], ring_empty[kBSlots];
-    uint64_t sp_full, p_ready, pv_done, ds_ready, dq_full, dq_empty, acc_done;
+    uint64_t sp_full, dp_full, p_ready, pv_done, ds_ready, dq_full, dq_empty, acc_done;
     uint32_t tmem;
     int abort;
 };
@@ -412,6 +410,7 @@ __global__ void __launch_bounds__(kBT, 1) attn_bwd_tc_kernel(const __grid_consta
             mbar_init(smem_u32(&sm.ring_empty[s]), 1);
         }
         mbar_init(smem_u32(&sm.sp_full), 1);
+        mbar_init(smem_u32(&sm.dp_full), 1);
         mbar_init(smem_u32(&sm.p_ready), kBWorkers);
         mbar_init(smem_u32(&sm.pv_done), 1);
         mbar_init(smem_u32(&sm.ds_ready), kBWorkers);
@@ -435,56 +434,54 @@ __global__ void __launch_bounds__(kBT, 1) attn_bwd_tc_kernel(const __grid_consta
     if (warp == 0) {
         if (lane == 0) {
             const uint32_t kb = smem_u32(&sm.kv_full);
-            mbar_expect_tx(kb, 4 * kTileHalf);
-            tma_load_4d(smem_u32(sm.k[0]), &p.mA0, kb, 0, j0, b, h);
-            tma_load_4d(smem_u32(sm.k[1]), &p.mA0, kb, 64, j0, b, h);
-            tma_load_4d(smem_u32(sm.v[0]), &p.mA1, kb, 0, j0, b, h);
-            tma_load_4d(smem_u32(sm.v[1]), &p.mA1, kb, 64, j0, b, h);
+            mbar_expect_tx(kb, 2 * kTileHalf);
+            tma_load_4d(smem_u32(sm.k), &p.mA0, kb, 0, j0, b, h);
+            tma_load_4d(smem_u32(sm.v), &p.mA1, kb, 0, j0, b, h);
             for (int t = 0; t < 2 * nb; ++t) {
                 const int i = t >> 1, is_da = t & 1;
-                const int s = is_da ? 2 : (i & 1);
-                const int use = is_da ? i : (i >> 1);   // earlier loads into this slot
+                const int s = 2 * (i & 1) + is_da;
+                const int use = i >> 1;   // earlier loads into this slot
                 if (!bwait(sm, sm.ring_empty[s], (use & 1) ^ 1, p.status)) break;
                 const int q0 = (jt + i) * 128;
-                const CUtensorMap *m = is_da ? &p.mB1 : &p.mB0;   // dA_i : Q_i
                 const uint32_t fb = smem_u32(&sm.ring_full[s]);
-                mbar_expect_tx(fb, 2 * kTileHalf);
-                tma_load_4d(smem_u32(sm.ring[s][0]), m, fb, 0, q0, b, h);
-                tma_load_4d(smem_u32(sm.ring[s][1]), m, fb, 64, q0, b, h);
+                mbar_expect_tx(fb, kTileHalf);
+                tma_load_4d(smem_u32(sm.ring[s]), is_da ? &p.mB1 : &p.mB0, fb, 0, q0, b, h);   // dA_i : Q_i
             }
         }
     } else if (warp == 1) {
         if (lane == 0) {
-            constexpr uint32_t idKK = idesc_bf16(128, 128, false, false);  // S, dP
-            constexpr uint32_t idMN = idesc_bf16(128, 64, true, true);     // dV, dK
-            constexpr uint32_t idKM = idesc_bf16(128, 64, false, true);    // dQ
+            constexpr uint32_t idKK = idesc_f16(128, 128, false, false);  // S, dP
+            constexpr uint32_t idMN = idesc_f16(128, 64, true, true);     // dV, dK
+            constexpr uint32_t idKM = idesc_f16(128, 64, false, true);    // dQ
             bool ok = bwait(sm, sm.kv_full, 0, p.status);
-            const uint32_t k0 = smem_u32(sm.k[0]), k1 = smem_u32(sm.k[1]);
-            const uint32_t v0 = smem_u32(sm.v[0]), v1 = smem_u32(sm.v[1]);
-            // S_i = Q_i K^T (needs Q_i in slot i % 2), dP_i = dA_i V^T (dA_i in slot 2)
+            const uint32_t kt = smem_u32(sm.k), vt = smem_u32(sm.v);
+            const uint32_t p0 = smem_u32(sm.p[0]), ds0 = smem_u32(sm.ds[0]);
+            // S_i = Q_i K^T (Q_i in slot 2 (i % 2)), dP_i = dA_i V^T (dA_i in the next slot)
             auto issue_s = [&](int i) {
-                ok = ok && bwait(sm, sm.ring_full[i & 1], (i >> 1) & 1, p.status);
+                const int s = 2 * (i & 1);
+                ok = ok && bwait(sm, sm.ring_full[s], (i >> 1) & 1, p.status);
                 if (!ok) return;
                 tc_fence_after();
-                mma_pair3(tS, smem_u32(sm.ring[i & 1][0]), smem_u32(sm.ring[i & 1][1]), k0, k1, false,
-                          false, idKK, false);
+                mma_k64_f16(tS, smem_u32(sm.ring[s]), kt, idKK);
                 mma_commit(smem_u32(&sm.sp_full));
             };
             auto issue_dp = [&](int i) {
-                ok = ok && bwait(sm, sm.ring_full[2], i & 1, p.status);
+                const int s = 2 * (i & 1) + 1;
+                ok = ok && bwait(sm, sm.ring_full[s], (i >> 1) & 1, p.status);
                 if (!ok) return;
                 tc_fence_after();
-                mma_pair3(tDP, smem_u32(sm.ring[2][0]), smem_u32(sm.ring[2][1]), v0, v1, false, false,
-                          idKK, false);
+                mma_k64_f16(tDP, smem_u32(sm.ring[s]), vt, idKK);
+                mma_commit(smem_u32(&sm.dp_full));
             };
             issue_s(0);
             issue_dp(0);
             for (int i = 0; i < nb && ok; ++i) {
+                const int sq = 2 * (i & 1), sa = sq + 1;
                 if (!(ok = bwait(sm, sm.p_ready, i & 1, p.status))) break;
                 tc_fence_after();
-                mma_k128(tDV, sm.ps, sm.ring[2], true, idMN, i > 0);          // dV += P^T dA_i
-                mma_commit(smem_u32(&sm.pv_done));                            // dP_i and dV done
-                mma_commit(smem_u32(&sm.ring_empty[2]));
+                mma_k128_f16(tDV, p0, smem_u32(sm.ring[sa]), true, idMN, i > 0);   // dV += P^T dA_i
+                mma_commit(smem_u32(&sm.pv_done));                                // P tile free
+                mma_commit(smem_u32(&sm.ring_empty[sa]));                         // dA_i (dP_i done too)
                 if (!(ok = bwait(sm, sm.ds_ready, i & 1, p.status))) break;
                 // S and dP of block i have been read: the next S goes first so
                 // that its P is computed while dK and dQ of this block run
@@ -492,15 +489,16 @@ __global__ void __launch_bounds__(kBT, 1) attn_bwd_tc_kernel(const __grid_consta
                 if (i > 0) ok = ok && bwait(sm, sm.dq_empty, (i - 1) & 1, p.status);
                 if (!ok) break;
                 tc_fence_after();
-                mma_k128(tDK, sm.ps, sm.ring[i & 1], true, idMN, i > 0);     // dK += dS^T Q_i
-                mma_k128(tDQ, sm.ps, sm.k, false, idKM);                      // dQ_i = dS K
-                mma_commit(smem_u32(&sm.dq_full));
-                mma_commit(smem_u32(&sm.ring_empty[i & 1]));
+                mma_k128_f16(tDK, ds0, smem_u32(sm.ring[sq]), true, idMN, i > 0);  // dK += dS^T Q_i
+                mma_k128_f16(tDQ, ds0, kt, false, idKM, false);                    // dQ_i = dS K
+                mma_commit(smem_u32(&sm.dq_full));                                // dS tile free
+                mma_commit(smem_u32(&sm.ring_empty[sq]));
                 if (i + 1 < nb) issue_dp(i + 1);
             }
             if (!ok) {
                 // release every wait of the workers that may still be pending
                 mma_commit(smem_u32(&sm.sp_full));
+                mma_commit(smem_u32(&sm.dp_full));
                 mma_commit(smem_u32(&sm.pv_done));
                 mma_commit(smem_u32(&sm.dq_full));
             }
@@ -511,12 +509,14 @@ __global__ void __launch_bounds__(kBT, 1) attn_bwd_tc_kernel(const __grid_consta
         const int q = warp & 3, ch = (warp - 4) >> 2;
         const int r = q * 32 + lane;                  // query row of the block; key row at the end
         const uint32_t lane_off = (uint32_t)(q * 32) << 16;
-        uint8_t *xb = &sm.ps[0][0][0] + (warp - 4) * 4096;
         bool ok = true;
+        float dsmax = 0.f;                            // largest |dS| written (fp16 range check)
         // dQ of block i (dK and dQ done) into the fp32 accumulator: columns
         // 32 ch .. +31 of this thread's row, eight 16-byte vector reductions
         // straight from registers (they run while the next block's dV does)
         auto drain_dq = [&](int i) {
+            ok = bwait(sm, sm.dq_full, i & 1, p.status) && ok;
+            tc_fence_after();
             float dq[32];
             tmem_ld32(tDQ + lane_off + 32 * ch, dq);
             tc_fence_before();
@@ -553,19 +553,20 @@ __global__ void __launch_bounds__(kBT, 1) attn_bwd_tc_kernel(const __grid_consta
 #pragma unroll
             for (int c = 0; c < 64; ++c)
                 pv[c] = (valid && c <= lim) ? exp2_fast(fmaf(pv[c], p.scale_log2, -l2)) : 0.f;
-            // the tile holds dS of the previous block until its dK and dQ are done
+            // the P tile holds P_{i-1} until dV_{i-1} has read it
             if (i > 0) {
-                ok = bwait(sm, sm.dq_full, (i - 1) & 1, p.status) && ok;
+                ok = bwait(sm, sm.pv_done, (i - 1) & 1, p.status) && ok;
                 tc_fence_after();
             }
-            write_pair32(sm.ps, r, 64 * ch, pv);
-            write_pair32(sm.ps, r, 64 * ch + 32, pv + 32);
+            put_f16_32(sm.p[ch], r, 0, pv, 1.f);
+            put_f16_32(sm.p[ch], r, 32, pv + 32, 1.f);
             fence_proxy_async();
             tc_fence_before();
             mbar_arrive(smem_u32(&sm.p_ready));
+            // dQ_{i-1} out; its completion also frees the dS tile
             if (i > 0) drain_dq(i - 1);
-            // dS = P o (dP - D), over P once dV has read it
-            ok = bwait(sm, sm.pv_done, i & 1, p.status) && ok;
+            // dS = P o (dP - D)
+            ok = bwait(sm, sm.dp_full, i & 1, p.status) && ok;
             tc_fence_after();
             {
                 float t32[32];
@@ -576,15 +577,14 @@ __global__ void __launch_bounds__(kBT, 1) attn_bwd_tc_kernel(const __grid_consta
 #pragma unroll
                 for (int c = 0; c < 32; ++c) pv[32 + c] *= t32[c] - dd;
             }
-            write_pair32(sm.ps, r, 64 * ch, pv);
-            write_pair32(sm.ps, r, 64 * ch + 32, pv + 32);
+            dsmax = fmaxf(dsmax, put_f16_32(sm.ds[ch], r, 0, pv, 1.f));
+            dsmax = fmaxf(dsmax, put_f16_32(sm.ds[ch], r, 32, pv + 32, 1.f));
             fence_proxy_async();
             tc_fence_before();
             mbar_arrive(smem_u32(&sm.ds_ready));
         }
-        ok = bwait(sm, sm.dq_full, (nb - 1) & 1, p.status) && ok;
-        tc_fence_after();
-        drain_dq(nb - 1);
+        if (nb > 0) drain_dq(nb - 1);
+        if (!(dsmax < kF16Overflow)) atomicOr(p.status, kStatusRange);
         // dK / sqrt(h') and dV of the tile's keys (row r = key j0 + r)
         const bool done = bwait(sm, sm.acc_done, 0, p.status);
         tc_fence_after();
@@ -593,6 +593,7 @@ __global__ void __launch_bounds__(kBT, 1) attn_bwd_tc_kernel(const __grid_consta
         const bool live = __all_sync(0xffffffffu, ok && done && !*(volatile int *)&sm.abort) && nb > 0;
         const uint32_t src[2] = {tDK, tDV};
         const float fac[2] = {p.scale, 1.f};
+        uint8_t *xb = &sm.p[0][0] + (warp - 4) * 4096;   // the P and dS tiles are idle now
 #pragma unroll
         for (int t = 0; t < 2; ++t) {
             float v[32];
@@ -964,8 +965,6 @@ __global__ void __launch_bounds__(kSmallThreads, 1) attn_bwd_small_kernel(const 
     }
 }
 
-// [H, B, k, 128] bf16 pair array (row = 64 hi + 64 lo), box {64, rows, 1, 1}:
-// rows past k of one sequence read as zeros.
 bool map_rows(CUtensorMap *m, const void *base, int H, int Mtok) {
     // [H, B*k, 128] bf16 pair array, box {64, 128, 1}: 128 consecutive rows of one head
     const uint64_t dims[3] = {128, (uint64_t)Mtok, (uint64_t)H};
@@ -974,9 +973,12 @@ bool map_rows(CUtensorMap *m, const void *base, int H, int Mtok) {
     return tmap_bf16(m, base, 3, dims, strides, box);
 }
 
+// [H, B, k, 64] fp16 array (k > 128 path), box {64, rows, 1, 1}: rows past k
+// of one sequence read as zeros.  (The map's element type only sets the
+// element size; the tiles are copied bit for bit.)
 bool map_units(CUtensorMap *m, const void *base, int H, int B, int k, uint32_t rows) {
-    const uint64_t dims[4] = {128, (uint64_t)k, (uint64_t)B, (uint64_t)H};
-    const uint64_t strides[3] = {256, (uint64_t)k * 256, (uint64_t)B * k * 256};
+    const uint64_t dims[4] = {64, (uint64_t)k, (uint64_t)B, (uint64_t)H};
+    const uint64_t strides[3] = {128, (uint64_t)k * 128, (uint64_t)B * k * 128};
     const uint32_t box[4] = {64, rows, 1, 1};
     return tmap_bf16(m, base, 4, dims, strides, box);
 }

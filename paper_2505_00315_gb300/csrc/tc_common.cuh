@@ -5,6 +5,7 @@
 #pragma once
 
 #include <cuda.h>
+#include <cuda_fp16.h>
 
 #include "common.cuh"
 
@@ -175,7 +176,8 @@ __device__ __forceinline__ void tc_fence_after() {
     asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
 }
 
-// D[tmem] (+)= A[smem] * B[smem], bf16 inputs, fp32 accumulation.
+// D[tmem] (+)= A[smem] * B[smem], fp32 accumulation; the operand type (bf16
+// or fp16, the same for A and B) is set by the instruction descriptor.
 __device__ __forceinline__ void mma_bf16(uint32_t d_tmem, uint64_t adesc, uint64_t bdesc,
                                          uint32_t idesc, uint32_t accumulate) {
     asm volatile(
@@ -287,6 +289,26 @@ __host__ __device__ constexpr uint32_t idesc_bf16(int M, int N, bool a_mn_major,
            | ((uint32_t)(N >> 3) << 17)
            | ((uint32_t)(M >> 4) << 24);
 }
+
+// Instruction descriptor of tcgen05.mma kind::f16 with fp16 A/B and fp32 D
+// (the attention operands of the k > 128 path).
+__host__ __device__ constexpr uint32_t idesc_f16(int M, int N, bool a_mn_major, bool b_mn_major) {
+    return (1u << 4)                       // D format: f32 (A and B format 0: f16)
+           | ((a_mn_major ? 1u : 0u) << 15)
+           | ((b_mn_major ? 1u : 0u) << 16)
+           | ((uint32_t)(N >> 3) << 17)
+           | ((uint32_t)(M >> 4) << 24);
+}
+
+// Two values as an fp16x2 word (round to nearest even; a in the low half).
+__device__ __forceinline__ uint32_t pack_f16x2(float a, float b) {
+    const __half2 h = __floats2half2_rn(a, b);
+    return *reinterpret_cast<const uint32_t *>(&h);
+}
+
+// Smallest magnitude that rounds to infinity in fp16 (65504 is the largest
+// finite value): an intermediate at or above it is out of the fp16 range.
+constexpr float kF16Overflow = 65520.f;
 
 // The split-bf16 pair representation of the kernels' intermediate operands,
 // for two values at once, as bf16x2 words with a in the low 16 bits:

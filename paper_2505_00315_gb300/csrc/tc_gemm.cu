@@ -146,6 +146,10 @@ struct TcParams {
     float *out_f2;         // dlogit (kG), dW_v (kDW)
     float *out_f3;         // dW_r (kDW)
     uint32_t *status;
+    int half;              // kQKV / kG: Q, K, V or dA as fp16 rows [H, B*k, 64] (k > 128)
+                           // instead of bf16 pairs
+    int rope;              // kQKV with half: rotate Q and K (Sec. 2.2) before rounding
+    RopeTable rope_tab;
 };
 
 // Epilogue staging: each warp owns kXpose bytes at the start of the operand
@@ -187,6 +191,25 @@ __device__ __forceinline__ void stage_pair_row64(uint8_t *xb, uint32_t taddr, in
         for (int u = 0; u < 4; ++u) stage_pair_unit(xb, lane, 4 * hlf + u, v + 8 * u);
     }
     __syncwarp();
+}
+
+// This lane's 64 values as one fp16 row (128 bytes: units 0..7 at
+// xoff128(lane, u)); returns the largest magnitude (fp16 range check).
+__device__ __forceinline__ float stage_f16_vals64(uint8_t *xb, const float (&v)[64], int lane) {
+    float mx = 0.f;
+#pragma unroll
+    for (int u = 0; u < 8; ++u) {
+        uint32_t w[4];
+#pragma unroll
+        for (int e = 0; e < 4; ++e) {
+            const float a = v[8 * u + 2 * e], b = v[8 * u + 2 * e + 1];
+            mx = fmaxf(mx, fmaxf(fabsf(a), fabsf(b)));
+            w[e] = pack_f16x2(a, b);
+        }
+        *reinterpret_cast<uint4 *>(xb + xoff128(lane, u)) = make_uint4(w[0], w[1], w[2], w[3]);
+    }
+    __syncwarp();
+    return mx;
 }
 
 // Copies staged rows 0 .. nrows-1 to global memory with 16 lanes per row, so
@@ -491,15 +514,45 @@ __global__ void __launch_bounds__(kThreads, Cfg<KIND>::MIN_CTAS)
         if (abort) {
             // nothing to write
         } else if constexpr (KIND == kQKV) {
-            // Q and K by warps 4-7, V by warps 0-3; one 256-byte pair row per matrix row
+            // Q and K by warps 4-7, V by warps 0-3; one 256-byte pair row per
+            // matrix row, or (half) one 128-byte fp16 row, Q and K turned by
+            // RoPE first when asked
+            const int nrows = min(32, p.M - (m0 + q * 32));
+            float mx = 0.f;
             for (int j = part == 0 ? 0 : 2; j < (part == 0 ? 2 : 3); ++j) {
-                stage_pair_row64(xb, tb + 64 * j, lane);
-                bf16 *dst = static_cast<bf16 *>(p.out[j]) + ((size_t)h * p.Mtok + m0 + q * 32) * 128;
-                const int nrows = min(32, p.M - (m0 + q * 32));
-                store_rows256(xb, lane, nrows, [&](int rl, int u) {
-                    return reinterpret_cast<uint4 *>(dst + (size_t)rl * 128) + u;
+                if (!p.half) {
+                    stage_pair_row64(xb, tb + 64 * j, lane);
+                    bf16 *dst = static_cast<bf16 *>(p.out[j]) + ((size_t)h * p.Mtok + m0 + q * 32) * 128;
+                    store_rows256(xb, lane, nrows, [&](int rl, int u) {
+                        return reinterpret_cast<uint4 *>(dst + (size_t)rl * 128) + u;
+                    });
+                    continue;
+                }
+                float v[64];
+                {
+                    float t32[32];
+                    tmem_ld32(tb + 64 * j, t32);
+#pragma unroll
+                    for (int c = 0; c < 32; ++c) v[c] = t32[c];
+                    tmem_ld32(tb + 64 * j + 32, t32);
+#pragma unroll
+                    for (int c = 0; c < 32; ++c) v[32 + c] = t32[c];
+                }
+                if (p.rope && j < 2) {
+                    // pairs (2p, 2p+1), p < 16, of the first 32 columns, at the
+                    // token's original position t (gidx = b*T + t)
+                    const int t = s_rows[r] % p.T;
+#pragma unroll
+                    for (int pp = 0; pp < 16; ++pp)
+                        rope_turn(v[2 * pp], v[2 * pp + 1], p.rope_tab.phi[pp], t, 1.f);
+                }
+                mx = fmaxf(mx, stage_f16_vals64(xb, v, lane));
+                bf16 *dst = static_cast<bf16 *>(p.out[j]) + ((size_t)h * p.Mtok + m0 + q * 32) * 64;
+                store_rows128(xb, lane, [&](int rl, int c) -> uint4 * {
+                    return rl < nrows ? reinterpret_cast<uint4 *>(dst + (size_t)rl * 64) + c : nullptr;
                 });
             }
+            if (!(mx < kF16Overflow) && mg < p.M) atomicOr(p.status, kStatusRange);
         } else if constexpr (KIND == kG) {
             // G row in two 32-column halves: D = <AR, G> = r <A, G> accumulates,
             // dA = r G is staged
@@ -508,7 +561,7 @@ __global__ void __launch_bounds__(kThreads, Cfg<KIND>::MIN_CTAS)
             const float rr = live ? p.rsel[row] : 0.f;
             const uint4 *arow = reinterpret_cast<const uint4 *>(p.ARp + row * 128);  // hi 0..7, lo 8..15
             const uint4 z4 = make_uint4(0u, 0u, 0u, 0u);
-            float dd = 0.f;
+            float dd = 0.f, amax = 0.f;
 #pragma unroll
             for (int hlf = 0; hlf < 2; ++hlf) {
                 float g[32];
@@ -518,9 +571,25 @@ __global__ void __launch_bounds__(kThreads, Cfg<KIND>::MIN_CTAS)
                     dd = dot_pair8(live ? arow[4 * hlf + u] : z4, live ? arow[8 + 4 * hlf + u] : z4,
                                    g + 8 * u, dd);
 #pragma unroll
-                for (int e = 0; e < 32; ++e) g[e] *= rr;  // dA = r G, kept as a bf16 pair
+                for (int e = 0; e < 32; ++e) g[e] *= rr;  // dA = r G
+                if (!p.half) {
 #pragma unroll
-                for (int u = 0; u < 4; ++u) stage_pair_unit(xb, lane, 4 * hlf + u, g + 8 * u);
+                    for (int u = 0; u < 4; ++u) stage_pair_unit(xb, lane, 4 * hlf + u, g + 8 * u);
+                } else {
+                    // fp16 row: units 4 hlf .. 4 hlf + 3 of the 128-byte layout
+#pragma unroll
+                    for (int u = 0; u < 4; ++u) {
+                        uint32_t w[4];
+#pragma unroll
+                        for (int e = 0; e < 4; ++e) {
+                            const float a = g[8 * u + 2 * e], b = g[8 * u + 2 * e + 1];
+                            amax = fmaxf(amax, fmaxf(fabsf(a), fabsf(b)));
+                            w[e] = pack_f16x2(a, b);
+                        }
+                        *reinterpret_cast<uint4 *>(xb + xoff128(lane, 4 * hlf + u)) =
+                            make_uint4(w[0], w[1], w[2], w[3]);
+                    }
+                }
             }
             __syncwarp();
             // D = rowsum(dA o A) = r <A, G>; dlogit = r (1 - r) <A, G> = D (1 - r)
@@ -531,10 +600,18 @@ __global__ void __launch_bounds__(kThreads, Cfg<KIND>::MIN_CTAS)
             }
             const int row0 = m0 + q * 32;
             const int nrows = min(32, p.M - row0);
-            bf16 *dA = static_cast<bf16 *>(p.out[0]) + ((size_t)h * p.Mtok + row0) * 128;
-            store_rows256(xb, lane, nrows, [&](int rl, int u) {
-                return reinterpret_cast<uint4 *>(dA + (size_t)rl * 128) + u;
-            });
+            if (!p.half) {
+                bf16 *dA = static_cast<bf16 *>(p.out[0]) + ((size_t)h * p.Mtok + row0) * 128;
+                store_rows256(xb, lane, nrows, [&](int rl, int u) {
+                    return reinterpret_cast<uint4 *>(dA + (size_t)rl * 128) + u;
+                });
+            } else {
+                bf16 *dA = static_cast<bf16 *>(p.out[0]) + ((size_t)h * p.Mtok + row0) * 64;
+                store_rows128(xb, lane, [&](int rl, int c) -> uint4 * {
+                    return rl < nrows ? reinterpret_cast<uint4 *>(dA + (size_t)rl * 64) + c : nullptr;
+                });
+                if (!(amax < kF16Overflow) && live) atomicOr(p.status, kStatusRange);
+            }
             // dlogit as column 192 (hi) / 448 (lo) of the dQKV pair row, column 0 of
             // the 4th 64-column block that kDW reads for dW_r; the block's other
             // columns are never written: accumulator column n of that product
@@ -735,6 +812,8 @@ bool tc_supported(const Dims &dm) {
     return dm.bf16 && dm.hp == 64 && tmap_available();
 }
 
+bool attn_f16(const Dims &dm) { return dm.k > 128 && use_tc(dm); }
+
 cudaError_t tc_qkv(const Dims &dm, const void *X, const void *Wq, const void *Wk, const void *Wv,
                    const Saved &sv, cudaStream_t s) {
     TcParams p = base_params(dm, sv);
@@ -748,6 +827,12 @@ cudaError_t tc_qkv(const Dims &dm, const void *X, const void *Wq, const void *Wk
     p.out[0] = sv.Q;
     p.out[1] = sv.K;
     p.out[2] = sv.V;
+    p.T = dm.T;
+    p.half = attn_f16(dm) ? 1 : 0;
+    if (p.half && dm.rope) {
+        p.rope = 1;
+        p.rope_tab = make_rope_table(dm.hp, dm.T);
+    }
     dim3 grid((p.M + kBM - 1) / kBM, 1, dm.H);
     return launch_kind<kQKV>(p, grid, s);
 }
@@ -776,6 +861,7 @@ cudaError_t tc_out_bwd_g(const Dims &dm, const void *Wo, const void *dY, const S
     p.out[1] = sv.dQKV;
     p.out_f1 = sv.Dd;
     p.out_f2 = sv.dlogit;
+    p.half = attn_f16(dm) ? 1 : 0;
     dim3 grid((p.M + kBM - 1) / kBM, 1, dm.H);
     return launch_kind<kG>(p, grid, s);
 }

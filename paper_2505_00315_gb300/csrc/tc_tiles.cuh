@@ -1,7 +1,8 @@
 // Shared-memory tile helpers of the attention kernels (tc_attention.cu) and the
 // fused per-tile kernels (tc_fused_fwd.cu, tc_fused_bwd.cu): 128-row tiles in
-// 64-column blocks of 128-byte-swizzled bf16, stored as hi / lo pairs
-// (v ~ hi + lo), and the split products over them.
+// 64-column blocks of 128-byte-swizzled 16-bit values, stored as bf16 hi / lo
+// pairs (v ~ hi + lo) with the split products over them, or as single fp16
+// values (k > 128 attention) with one MMA per product.
 #pragma once
 
 #include "tc_common.cuh"
@@ -47,6 +48,51 @@ __device__ __forceinline__ void put_pair32(uint8_t *hi_blk, uint8_t *lo_blk, int
 __device__ __forceinline__ void write_pair32(uint8_t (*tile)[2][kTileHalf], int r, int c0,
                                              const float *v) {
     put_pair32(tile[0][c0 >> 6], tile[1][c0 >> 6], r, c0, v, 1.f);
+}
+
+// 32 values v * f as fp16, columns c0 .. c0+31 (within one 64-column block)
+// of row r of a K-major fp16 block; returns the largest magnitude written.
+__device__ __forceinline__ float put_f16_32(uint8_t *blk, int r, int c0, const float *v, float f) {
+    const int cb = (c0 & 63) >> 3;  // first 16-byte unit within the 128-byte row
+    float mx = 0.f;
+#pragma unroll
+    for (int c = 0; c < 4; ++c) {
+        uint32_t w[4];
+#pragma unroll
+        for (int e = 0; e < 4; ++e) {
+            const float a = v[c * 8 + 2 * e] * f, b = v[c * 8 + 2 * e + 1] * f;
+            mx = fmaxf(mx, fmaxf(fabsf(a), fabsf(b)));
+            w[e] = pack_f16x2(a, b);
+        }
+        const int off = r * 128 + (((cb + c) ^ (r & 7)) << 4);
+        *reinterpret_cast<uint4 *>(blk + off) = make_uint4(w[0], w[1], w[2], w[3]);
+    }
+    return mx;
+}
+
+// D (+)= A B over K = 128 for fp16 tiles (one MMA per 16-wide K step), A a
+// [128 x 128] tile as two 64-column blocks at a0 and a0 + kTileHalf, B a
+// 128-row tile read MN-major (its rows are the K index):
+//   a_mn = false: A K-major, K = tile columns (dS K)
+//   a_mn = true:  A read as its transpose (P^T dA, dS^T Q), K = tile rows
+__device__ __forceinline__ void mma_k128_f16(uint32_t d, uint32_t a0, uint32_t b, bool a_mn,
+                                             uint32_t idesc, bool accumulate) {
+#pragma unroll
+    for (int kk = 0; kk < 8; ++kk) {
+        const uint64_t ad = a_mn ? smem_desc_sw128(a0 + kk * 2048, kTileHalf, 1024)
+                                 : smem_desc_sw128(a0 + (kk >> 2) * kTileHalf + (kk & 3) * 32, 16, 1024);
+        const uint64_t bd = smem_desc_sw128(b + kk * 2048, kTileHalf, 1024);
+        mma_bf16(d, ad, bd, idesc, (accumulate || kk > 0) ? 1u : 0u);
+    }
+}
+
+// D = A B^T over K = 64 for fp16 tiles, both K-major 128-row blocks (S = Q K^T,
+// dP = dA V^T; N = 128).
+__device__ __forceinline__ void mma_k64_f16(uint32_t d, uint32_t a, uint32_t b, uint32_t idesc) {
+#pragma unroll
+    for (int kk = 0; kk < 4; ++kk)
+        mma_bf16(d, smem_desc_sw128(a + kk * 32, 16, 1024), smem_desc_sw128(b + kk * 32, 16, 1024),
+                 idesc, kk > 0 ? 1u : 0u);
 }
 
 // Three split products D (+)= Ah Bh + Ah Bl + Al Bh over K = 64.

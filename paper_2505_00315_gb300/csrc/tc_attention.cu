@@ -225,15 +225,7 @@ __global__ void __launch_bounds__(kLT, 1) attn_fwd_tc_kernel(const __grid_consta
             ok = lwait(sm, sm.s_full[j & 1], (j >> 1) & 1, p.status) && ok;
             tc_fence_after();
             float s[64];
-            {
-                float t32[32];
-                tmem_ld32(tmem + 128 * (j & 1) + lane_off + 64 * ch, t32);
-#pragma unroll
-                for (int c = 0; c < 32; ++c) s[c] = t32[c];
-                tmem_ld32(tmem + 128 * (j & 1) + lane_off + 64 * ch + 32, t32);
-#pragma unroll
-                for (int c = 0; c < 32; ++c) s[32 + c] = t32[c];
-            }
+            tmem_ld64(tmem + 128 * (j & 1) + lane_off + 64 * ch, s);
             if (j == qt) {
                 // diagonal block (earlier blocks are wholly visible): key
                 // j*128 + 64 ch + c is visible from query i iff c <= lim
@@ -248,10 +240,11 @@ __global__ void __launch_bounds__(kLT, 1) attn_fwd_tc_kernel(const __grid_consta
             for (int c = 0; c < 64; ++c) mx[c & 3] = fmaxf(mx[c & 3], s[c]);
             float mb = fmaxf(fmaxf(mx[0], mx[1]), fmaxf(mx[2], mx[3])) * p.scale_log2;
             // the exchange buffer alternates with the block parity: the buffer
-            // written here was last read before everyone passed the previous
-            // block's barrier, so one barrier per block suffices
+            // written here was last read before both warps of the row passed
+            // the previous block's barrier, so one barrier per block suffices;
+            // only the two warps sharing the lane quadrant q synchronise
             sm.part[j & 1][ch][r] = mb;
-            named_barrier(1, kLWorkers);
+            named_barrier(1 + q, 64);
             mb = fmaxf(sm.part[j & 1][0][r], sm.part[j & 1][1][r]);
             const bool grow = mb > m + kRescaleLog2;   // same decision in both threads of the row
             const float m_new = grow ? mb : m;
@@ -291,7 +284,7 @@ __global__ void __launch_bounds__(kLT, 1) attn_fwd_tc_kernel(const __grid_consta
         ok = lwait(sm, sm.pv_done, (n - 1) & 1, p.status) && ok;
         tc_fence_after();
         sm.part[n & 1][ch][r] = l;
-        named_barrier(1, kLWorkers);
+        named_barrier(1 + q, 64);
         l = sm.part[n & 1][0][r] + sm.part[n & 1][1][r];
         float o[32];
         tmem_ld32(tO + lane_off + 32 * ch, o);      // output columns 32 ch .. +31
@@ -328,6 +321,8 @@ struct BwdParams {
     CUtensorMap mA0, mA1, mB0, mB1;   // dK/dV: K, V (128 rows), Q, dA (64 rows); dQ: Q, dA (128), K, V (64)
                                       // k <= 128: Q, K, V, dA as 3-D maps over [H, B*k, 128]
     CUtensorMap mOut;                 // k <= 128: dQKV [H, B*k, 512], box {64, U k, 1} (stores)
+    CUtensorMap mDQ;                  // k > 128: dQ accumulator [H, B, k, 64] fp32, box {32, 32, 1, 1}
+                                      // (reductions)
     int k, Mtok;
     int U, B;                         // k <= 128: sequences per tile, batch
     float scale, scale_log2;
@@ -354,28 +349,42 @@ __device__ __forceinline__ void flag_timeout_b(SM &sm, uint32_t *status) {
 //   S = Q_i K^T, dP = dA_i V^T                  (TMEM)
 //   P = exp(S / sqrt(h') - lse_i)               (P tile; kept in registers)
 //   dV += P^T dA_i                              (TMEM, the tile read MN-major)
-//   dS = P o (dP - D_i)                         (dS tile)
-//   dK += dS^T Q_i, dQ_i = dS K                 (TMEM)
-//   dQ_i / sqrt(h') is added into an fp32 accumulator [H, B*k, 64] with
-//   vector reductions issued after the next block's P has been stored;
-// S_{i+1} is issued before dK_i and dQ_i, so the exponentials of block i+1
-// run on the workers while the tensor pipe works on block i; P and dS have
-// tiles of their own, so dS_i is written while dV_i still reads P_i.
+//   dS = P o (dP - D_i)                         (dS tile i % 2)
+//   dK += dS^T Q_i, dQ_i = dS K                 (TMEM; dQ in buffer i % 2)
+//   dQ_i / sqrt(h') is added into an fp32 accumulator [H, B*k, 64] two
+//   blocks later: each worker warp stages its 32 x 32 part in the dS tile it
+//   is about to overwrite and one lane hands it to the TMA engine as a bulk
+//   reduce-add (the 256 threads' own scattered vector reductions took about
+//   1 us per block).
+// Measured on this GPU, an MMA instruction (M = 128, K = 16) takes about the
+// same time for any N up to 128 (about 2.3x longer per FLOP at N = 64 than
+// at N = 256), so the 32 MMAs of a block (S, dP: N = 128; dV, dK, dQ: N = 64)
+// cost about 4000 cycles and the kernel is bound by keeping the tensor pipe
+// issuing.  The MMA issuer therefore waits only for what each product needs:
+// S_{i+1} is issued as soon as the workers have read S_i into registers, and
+// dP_{i+1}, dK_i and dQ_i as soon as dS_i is stored; the workers do not wait
+// for the tensor pipe either: dS and dQ are double-buffered (the smem dS tile
+// and the TMEM dQ accumulator of block i are reused by block i + 2, whose dQ
+// the workers drain two blocks late), and lse and D of block i+1 are loaded
+// during block i.  Barriers of double-buffered data come in pairs, one per
+// buffer, so no waiter can see its barrier complete two phases ahead.
 // dK / sqrt(h') and dV are written once at the end as bf16 pairs.  Q_i and
-// dA_i go to ring slots 2 (i % 2) and 2 (i % 2) + 1, so each load is issued
-// a block ahead of its use.
+// dA_i go to ring slots 2 (i % 3) and 2 (i % 3) + 1, so each load is issued
+// up to three blocks ahead of its use (a two-block ring left the MMA issuer
+// waiting about 1 us per block for Q_{i+1}).
 constexpr int kBT = 384;
 constexpr int kBWorkers = 256;
-constexpr int kBSlots = 4;
+constexpr int kBDepth = 3;                 // blocks in the Q / dA ring
+constexpr int kBSlots = 2 * kBDepth;
 
 struct BwdLargeSmem {
     uint8_t k[kTileHalf];                  // K tile, fp16 [128 keys x 64]
     uint8_t v[kTileHalf];                  // V tile
     uint8_t ring[kBSlots][kTileHalf];      // Q_i, dA_i (fp16 [128 queries x 64])
     uint8_t p[2][kTileHalf];               // P [128 queries x 128 keys] as two 64-key blocks
-    uint8_t ds[2][kTileHalf];              // dS, the same layout
+    uint8_t ds[2][2][kTileHalf];           // dS of blocks i % 2, the same layout
     uint64_t kv_full, ring_full[kBSlots], ring_empty[kBSlots];
-    uint64_t sp_full, dp_full, p_ready, pv_done, ds_ready, dq_full, dq_empty, acc_done;
+    uint64_t sp_full, dp_full, s_free, p_ready, pv_done, ds_ready, dq_full[2], dq_empty[2], acc_done;
     uint32_t tmem;
     int abort;
 };
@@ -411,11 +420,14 @@ __global__ void __launch_bounds__(kBT, 1) attn_bwd_tc_kernel(const __grid_consta
         }
         mbar_init(smem_u32(&sm.sp_full), 1);
         mbar_init(smem_u32(&sm.dp_full), 1);
+        mbar_init(smem_u32(&sm.s_free), kBWorkers);
         mbar_init(smem_u32(&sm.p_ready), kBWorkers);
         mbar_init(smem_u32(&sm.pv_done), 1);
         mbar_init(smem_u32(&sm.ds_ready), kBWorkers);
-        mbar_init(smem_u32(&sm.dq_full), 1);
-        mbar_init(smem_u32(&sm.dq_empty), kBWorkers);
+        for (int u = 0; u < 2; ++u) {
+            mbar_init(smem_u32(&sm.dq_full[u]), 1);
+            mbar_init(smem_u32(&sm.dq_empty[u]), kBWorkers);
+        }
         mbar_init(smem_u32(&sm.acc_done), 1);
         sm.abort = 0;
         fence_barrier_init();
@@ -429,6 +441,7 @@ __global__ void __launch_bounds__(kBT, 1) attn_bwd_tc_kernel(const __grid_consta
     tc_fence_after();
     pdl_wait();  // Q, K, V, dA, lse, D written by the previous kernels
     const uint32_t tmem = sm.tmem;
+    // S, dP, dV, dK, and the two dQ buffers: all 512 columns
     const uint32_t tS = tmem, tDP = tmem + 128, tDV = tmem + 256, tDK = tmem + 320, tDQ = tmem + 384;
 
     if (warp == 0) {
@@ -439,8 +452,8 @@ __global__ void __launch_bounds__(kBT, 1) attn_bwd_tc_kernel(const __grid_consta
             tma_load_4d(smem_u32(sm.v), &p.mA1, kb, 0, j0, b, h);
             for (int t = 0; t < 2 * nb; ++t) {
                 const int i = t >> 1, is_da = t & 1;
-                const int s = 2 * (i & 1) + is_da;
-                const int use = i >> 1;   // earlier loads into this slot
+                const int s = 2 * (i % kBDepth) + is_da;
+                const int use = i / kBDepth;   // earlier loads into this slot
                 if (!bwait(sm, sm.ring_empty[s], (use & 1) ^ 1, p.status)) break;
                 const int q0 = (jt + i) * 128;
                 const uint32_t fb = smem_u32(&sm.ring_full[s]);
@@ -455,19 +468,19 @@ __global__ void __launch_bounds__(kBT, 1) attn_bwd_tc_kernel(const __grid_consta
             constexpr uint32_t idKM = idesc_f16(128, 64, false, true);    // dQ
             bool ok = bwait(sm, sm.kv_full, 0, p.status);
             const uint32_t kt = smem_u32(sm.k), vt = smem_u32(sm.v);
-            const uint32_t p0 = smem_u32(sm.p[0]), ds0 = smem_u32(sm.ds[0]);
-            // S_i = Q_i K^T (Q_i in slot 2 (i % 2)), dP_i = dA_i V^T (dA_i in the next slot)
+            const uint32_t p0 = smem_u32(sm.p[0]);
+            // S_i = Q_i K^T (Q_i in slot 2 (i % 3)), dP_i = dA_i V^T (dA_i in the next slot)
             auto issue_s = [&](int i) {
-                const int s = 2 * (i & 1);
-                ok = ok && bwait(sm, sm.ring_full[s], (i >> 1) & 1, p.status);
+                const int s = 2 * (i % kBDepth);
+                ok = ok && bwait(sm, sm.ring_full[s], (i / kBDepth) & 1, p.status);
                 if (!ok) return;
                 tc_fence_after();
                 mma_k64_f16(tS, smem_u32(sm.ring[s]), kt, idKK);
                 mma_commit(smem_u32(&sm.sp_full));
             };
             auto issue_dp = [&](int i) {
-                const int s = 2 * (i & 1) + 1;
-                ok = ok && bwait(sm, sm.ring_full[s], (i >> 1) & 1, p.status);
+                const int s = 2 * (i % kBDepth) + 1;
+                ok = ok && bwait(sm, sm.ring_full[s], (i / kBDepth) & 1, p.status);
                 if (!ok) return;
                 tc_fence_after();
                 mma_k64_f16(tDP, smem_u32(sm.ring[s]), vt, idKK);
@@ -475,32 +488,42 @@ __global__ void __launch_bounds__(kBT, 1) attn_bwd_tc_kernel(const __grid_consta
             };
             issue_s(0);
             issue_dp(0);
+            // Issue order per block follows the workers' progress: S_{i+1} once
+            // S_i is in their registers, dV_i once P_i is stored, then dP_{i+1},
+            // dK_i and dQ_i once dS_i is stored (by then dP_i has been read;
+            // dQ_i also waits for dQ_{i-2}, the last user of its buffer, to be
+            // drained).
             for (int i = 0; i < nb && ok; ++i) {
-                const int sq = 2 * (i & 1), sa = sq + 1;
-                if (!(ok = bwait(sm, sm.p_ready, i & 1, p.status))) break;
+                const int sq = 2 * (i % kBDepth), sa = sq + 1;
+                if (i + 1 < nb) {
+                    if (!(ok = bwait(sm, sm.s_free, i & 1, p.status))) break;
+                    issue_s(i + 1);
+                }
+                if (!(ok = ok && bwait(sm, sm.p_ready, i & 1, p.status))) break;
                 tc_fence_after();
                 mma_k128_f16(tDV, p0, smem_u32(sm.ring[sa]), true, idMN, i > 0);   // dV += P^T dA_i
                 mma_commit(smem_u32(&sm.pv_done));                                // P tile free
                 mma_commit(smem_u32(&sm.ring_empty[sa]));                         // dA_i (dP_i done too)
-                if (!(ok = bwait(sm, sm.ds_ready, i & 1, p.status))) break;
-                // S and dP of block i have been read: the next S goes first so
-                // that its P is computed while dK and dQ of this block run
-                if (i + 1 < nb) issue_s(i + 1);
-                if (i > 0) ok = ok && bwait(sm, sm.dq_empty, (i - 1) & 1, p.status);
+                if (!(ok = ok && bwait(sm, sm.ds_ready, i & 1, p.status))) break;
+                if (i + 1 < nb) issue_dp(i + 1);
+                // dQ_{i-2} drained (the (i/2 - 1)-th completion of buffer i % 2's barrier)
+                if (i >= 2) ok = ok && bwait(sm, sm.dq_empty[i & 1], ((i >> 1) - 1) & 1, p.status);
                 if (!ok) break;
                 tc_fence_after();
-                mma_k128_f16(tDK, ds0, smem_u32(sm.ring[sq]), true, idMN, i > 0);  // dK += dS^T Q_i
-                mma_k128_f16(tDQ, ds0, kt, false, idKM, false);                    // dQ_i = dS K
-                mma_commit(smem_u32(&sm.dq_full));                                // dS tile free
+                const uint32_t dsb = smem_u32(sm.ds[i & 1][0]);
+                mma_k128_f16(tDK, dsb, smem_u32(sm.ring[sq]), true, idMN, i > 0);   // dK += dS^T Q_i
+                mma_k128_f16(tDQ + 64 * (i & 1), dsb, kt, false, idKM, false);      // dQ_i = dS K
+                mma_commit(smem_u32(&sm.dq_full[i & 1]));
                 mma_commit(smem_u32(&sm.ring_empty[sq]));
-                if (i + 1 < nb) issue_dp(i + 1);
             }
             if (!ok) {
                 // release every wait of the workers that may still be pending
+                // (each of their later waits then sees the abort flag first)
                 mma_commit(smem_u32(&sm.sp_full));
                 mma_commit(smem_u32(&sm.dp_full));
                 mma_commit(smem_u32(&sm.pv_done));
-                mma_commit(smem_u32(&sm.dq_full));
+                mma_commit(smem_u32(&sm.dq_full[0]));
+                mma_commit(smem_u32(&sm.dq_full[1]));
             }
             mma_commit(smem_u32(&sm.acc_done));
         }
@@ -510,49 +533,67 @@ __global__ void __launch_bounds__(kBT, 1) attn_bwd_tc_kernel(const __grid_consta
         const int r = q * 32 + lane;                  // query row of the block; key row at the end
         const uint32_t lane_off = (uint32_t)(q * 32) << 16;
         bool ok = true;
-        float dsmax = 0.f;                            // largest |dS| written (fp16 range check)
-        // dQ of block i (dK and dQ done) into the fp32 accumulator: columns
-        // 32 ch .. +31 of this thread's row, eight 16-byte vector reductions
-        // straight from registers (they run while the next block's dV does)
+        // dQ of block i (its dK and dQ done; buffer i % 2) into the fp32
+        // accumulator: this warp's query rows 32 q .. +31, columns 32 ch .. +31,
+        // staged (128-byte swizzled, as the map's swizzle expects) in the rows
+        // of dS tile i % 2 this warp itself writes, then one bulk reduce-add
+        // issued by lane 0 (rows past k are skipped by the map)
         auto drain_dq = [&](int i) {
-            ok = bwait(sm, sm.dq_full, i & 1, p.status) && ok;
+            ok = bwait(sm, sm.dq_full[i & 1], (i >> 1) & 1, p.status) && ok;
             tc_fence_after();
             float dq[32];
-            tmem_ld32(tDQ + lane_off + 32 * ch, dq);
+            tmem_ld32(tDQ + 64 * (i & 1) + lane_off + 32 * ch, dq);
             tc_fence_before();
-            mbar_arrive(smem_u32(&sm.dq_empty));
+            mbar_arrive(smem_u32(&sm.dq_empty[i & 1]));
             const bool live = __all_sync(0xffffffffu, ok && !*(volatile int *)&sm.abort);
-            const int qi = (jt + i) * 128 + r;
-            if (live && qi < p.k) {
-                float *dst = p.dQacc + (base + qi) * 64 + 32 * ch;
-#pragma unroll
-                for (int c = 0; c < 32; c += 4)
-                    red_add_v4(dst + c, dq[c] * p.scale, dq[c + 1] * p.scale, dq[c + 2] * p.scale,
-                               dq[c + 3] * p.scale);
+            if (!live) return;
+            uint8_t *xs = sm.ds[i & 1][ch] + q * 4096;
+            stage_f32x32(xs, dq, p.scale, lane);   // ends with __syncwarp
+            fence_proxy_async();
+            __syncwarp();
+            const int q0 = (jt + i) * 128 + q * 32;   // first query row of this warp
+            if (lane == 0 && q0 < p.k) {
+                tma_reduce_add_4d(&p.mDQ, smem_u32(xs), 32 * ch, q0, b, h);
+                bulk_commit();
             }
         };
+        // this warp's staged dQ rows must have been read before dS overwrites them
+        auto staging_read = [&]() {
+            if (lane == 0) bulk_wait_read0();
+            __syncwarp();
+        };
+        // lse (log2 units) and D of this thread's query row, one block ahead
+        auto row_terms = [&](int i, float &l2, float &dd) {
+            const int qi = (jt + i) * 128 + r;
+            const bool v = i < nb && qi < p.k;
+            l2 = v ? __ldg(p.lse + base + qi) * 1.4426950408889634f : 0.f;
+            dd = v ? __ldg(p.Dd + base + qi) : 0.f;
+        };
+        float l2n, ddn;
+        row_terms(0, l2n, ddn);
         for (int i = 0; i < nb; ++i) {
             const int qi = (jt + i) * 128 + r;        // query index
             const bool valid = qi < p.k;
-            const float l2 = valid ? __ldg(p.lse + base + qi) * 1.4426950408889634f : 0.f;
-            const float dd = valid ? __ldg(p.Dd + base + qi) : 0.f;
+            const float l2 = l2n, dd = ddn;
+            row_terms(i + 1, l2n, ddn);
             ok = bwait(sm, sm.sp_full, i & 1, p.status) && ok;
             tc_fence_after();
             // P over this thread's 64 keys (the diagonal block i = 0 is causal)
             float pv[64];
-            {
-                float t32[32];
-                tmem_ld32(tS + lane_off + 64 * ch, t32);
+            tmem_ld64(tS + lane_off + 64 * ch, pv);
+            tc_fence_before();
+            mbar_arrive(smem_u32(&sm.s_free));        // S_{i+1} may overwrite these columns
+            if (i == 0 || !valid) {
+                // the diagonal block is causal (key offsets c <= lim visible);
+                // rows past k see nothing
+                const int lim = valid ? r - 64 * ch : -1;
 #pragma unroll
-                for (int c = 0; c < 32; ++c) pv[c] = t32[c];
-                tmem_ld32(tS + lane_off + 64 * ch + 32, t32);
+                for (int c = 0; c < 64; ++c)
+                    pv[c] = c <= lim ? exp2_fast(fmaf(pv[c], p.scale_log2, -l2)) : 0.f;
+            } else {
 #pragma unroll
-                for (int c = 0; c < 32; ++c) pv[32 + c] = t32[c];
+                for (int c = 0; c < 64; ++c) pv[c] = exp2_fast(fmaf(pv[c], p.scale_log2, -l2));
             }
-            const int lim = (i == 0) ? r - 64 * ch : 127;   // visible key offsets c <= lim
-#pragma unroll
-            for (int c = 0; c < 64; ++c)
-                pv[c] = (valid && c <= lim) ? exp2_fast(fmaf(pv[c], p.scale_log2, -l2)) : 0.f;
             // the P tile holds P_{i-1} until dV_{i-1} has read it
             if (i > 0) {
                 ok = bwait(sm, sm.pv_done, (i - 1) & 1, p.status) && ok;
@@ -563,29 +604,31 @@ __global__ void __launch_bounds__(kBT, 1) attn_bwd_tc_kernel(const __grid_consta
             fence_proxy_async();
             tc_fence_before();
             mbar_arrive(smem_u32(&sm.p_ready));
-            // dQ_{i-1} out; its completion also frees the dS tile
-            if (i > 0) drain_dq(i - 1);
+            // dQ_{i-2} out: frees its TMEM buffer, and its completion also
+            // frees the dS tile this block writes
+            if (i >= 2) drain_dq(i - 2);
             // dS = P o (dP - D)
             ok = bwait(sm, sm.dp_full, i & 1, p.status) && ok;
             tc_fence_after();
             {
-                float t32[32];
-                tmem_ld32(tDP + lane_off + 64 * ch, t32);
+                float dp[64];
+                tmem_ld64(tDP + lane_off + 64 * ch, dp);
 #pragma unroll
-                for (int c = 0; c < 32; ++c) pv[c] *= t32[c] - dd;
-                tmem_ld32(tDP + lane_off + 64 * ch + 32, t32);
-#pragma unroll
-                for (int c = 0; c < 32; ++c) pv[32 + c] *= t32[c] - dd;
+                for (int c = 0; c < 64; ++c) pv[c] *= dp[c] - dd;
             }
-            dsmax = fmaxf(dsmax, put_f16_32(sm.ds[ch], r, 0, pv, 1.f));
-            dsmax = fmaxf(dsmax, put_f16_32(sm.ds[ch], r, 32, pv + 32, 1.f));
+            staging_read();
+            put_f16_32(sm.ds[i & 1][ch], r, 0, pv, 1.f);
+            put_f16_32(sm.ds[i & 1][ch], r, 32, pv + 32, 1.f);
             fence_proxy_async();
             tc_fence_before();
-            mbar_arrive(smem_u32(&sm.ds_ready));
+            mbar_arrive(smem_u32(&sm.ds_ready));       // also: dP_{i+1} may overwrite dP_i
         }
-        if (nb > 0) drain_dq(nb - 1);
-        if (!(dsmax < kF16Overflow)) atomicOr(p.status, kStatusRange);
-        // dK / sqrt(h') and dV of the tile's keys (row r = key j0 + r)
+        if (nb >= 2) drain_dq(nb - 2);
+        drain_dq(nb - 1);
+        if (lane == 0) bulk_wait0();   // the reductions are complete before the CTA's smem goes
+        __syncwarp();
+        // dK / sqrt(h') and dV of the tile's keys (row r = key j0 + r); an fp16
+        // dS out of range has made them non-finite, which flags it
         const bool done = bwait(sm, sm.acc_done, 0, p.status);
         tc_fence_after();
         const int kj = j0 + r;
@@ -593,12 +636,15 @@ __global__ void __launch_bounds__(kBT, 1) attn_bwd_tc_kernel(const __grid_consta
         const bool live = __all_sync(0xffffffffu, ok && done && !*(volatile int *)&sm.abort) && nb > 0;
         const uint32_t src[2] = {tDK, tDV};
         const float fac[2] = {p.scale, 1.f};
-        uint8_t *xb = &sm.p[0][0] + (warp - 4) * 4096;   // the P and dS tiles are idle now
+        uint8_t *xb = &sm.p[0][0] + (warp - 4) * 4096;   // the P tile is idle now
+        bool finite = true;
 #pragma unroll
         for (int t = 0; t < 2; ++t) {
             float v[32];
             tmem_ld32(src[t] + lane_off + 32 * ch, v);
             if (!live) continue;
+#pragma unroll
+            for (int c = 0; c < 32; ++c) finite = finite && fabsf(v[c]) < INFINITY;
             stage_pair32(xb, v, fac[t], lane);
             store_rows128(xb, lane, [&](int rl, int c) -> uint4 * {
                 if (!((kmask >> rl) & 1u)) return nullptr;
@@ -607,6 +653,7 @@ __global__ void __launch_bounds__(kBT, 1) attn_bwd_tc_kernel(const __grid_consta
                              : reinterpret_cast<uint4 *>(row + 256) + (c - 4);
             });
         }
+        if (live && !finite && kj < p.k) atomicOr(p.status, kStatusRange);
     }
     tc_fence_before();
     __syncthreads();
@@ -1070,6 +1117,13 @@ cudaError_t tc_attn_bwd(const Dims &dm, const Saved &sv, cudaStream_t s) {
     bp.dQKV = static_cast<bf16 *>(sv.dQKV);
     bp.dQacc = sv.G;
     bp.status = sv.status;
+    {
+        // dQ accumulator [H, B, k, 64] fp32 (the workspace's G buffer)
+        const uint64_t dims[4] = {64, (uint64_t)dm.k, (uint64_t)dm.B, (uint64_t)dm.H};
+        const uint64_t strides[3] = {256, (uint64_t)dm.k * 256, (uint64_t)dm.B * dm.k * 256};
+        const uint32_t box[4] = {32, 32, 1, 1};
+        if (!tmap_f32(&bp.mDQ, sv.G, 4, dims, strides, box)) return cudaErrorInvalidValue;
+    }
     const size_t rows = (size_t)dm.H * dm.B * dm.k;
     const cudaError_t attr = allow_smem((const void *)attn_bwd_tc_kernel, kBwdLargeSmem);
     if (attr != cudaSuccess) return attr;

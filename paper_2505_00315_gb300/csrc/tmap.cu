@@ -26,6 +26,7 @@ PFN_cuTensorMapEncodeTiled_v12000 encoder() {
 }
 
 struct Key {
+    uint64_t dtype;
     uint64_t base;
     uint64_t dims[5], strides[4];
     uint32_t box[5];
@@ -50,11 +51,14 @@ constexpr size_t kMaxEntries = 4096;
 
 bool tmap_available() { return encoder() != nullptr; }
 
-bool tmap_bf16(CUtensorMap *out, const void *base, int rank, const uint64_t *dims,
-               const uint64_t *strides, const uint32_t *box) {
+namespace {
+
+bool encode(CUtensorMapDataType dtype, CUtensorMap *out, const void *base, int rank,
+            const uint64_t *dims, const uint64_t *strides, const uint32_t *box) {
     if (rank < 1 || rank > 5) return false;
     Key key;
     std::memset(&key, 0, sizeof(key));
+    key.dtype = (uint64_t)dtype;
     key.base = reinterpret_cast<uint64_t>(base);
     key.rank = rank;
     for (int i = 0; i < rank; ++i) {
@@ -80,7 +84,7 @@ bool tmap_bf16(CUtensorMap *out, const void *base, int rank, const uint64_t *dim
     }
     for (int i = 0; i < rank - 1; ++i) gs[i] = strides[i];
     CUtensorMap m;
-    if (fn(&m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, (cuuint32_t)rank, const_cast<void *>(base), gd,
+    if (fn(&m, dtype, (cuuint32_t)rank, const_cast<void *>(base), gd,
            gs, bx, es, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
            CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) != CUDA_SUCCESS)
         return false;
@@ -89,6 +93,18 @@ bool tmap_bf16(CUtensorMap *out, const void *base, int rank, const uint64_t *dim
     g_cache.emplace(key, m);
     *out = m;
     return true;
+}
+
+}  // namespace
+
+bool tmap_bf16(CUtensorMap *out, const void *base, int rank, const uint64_t *dims,
+               const uint64_t *strides, const uint32_t *box) {
+    return encode(CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, out, base, rank, dims, strides, box);
+}
+
+bool tmap_f32(CUtensorMap *out, const void *base, int rank, const uint64_t *dims,
+              const uint64_t *strides, const uint32_t *box) {
+    return encode(CU_TENSOR_MAP_DATA_TYPE_FLOAT32, out, base, rank, dims, strides, box);
 }
 
 }  // namespace mosa

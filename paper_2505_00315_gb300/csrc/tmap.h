@@ -16,5 +16,8 @@ bool tmap_available();
 // results are cached and reused across calls.  False if encoding fails.
 bool tmap_bf16(CUtensorMap *out, const void *base, int rank, const uint64_t *dims,
                const uint64_t *strides, const uint32_t *box);
+// The same for fp32 elements (the box's innermost extent then at most 32).
+bool tmap_f32(CUtensorMap *out, const void *base, int rank, const uint64_t *dims,
+              const uint64_t *strides, const uint32_t *box);
 
 }  // namespace mosa

@@ -94,6 +94,11 @@ struct Saved {
     float *G;           // [H,B*k,hp] dY[I] W_o^T (fp32, CUDA-core path); on the
                         // tensor-core path with k > 128 the fp32 dQ accumulator
     float *WrT;         // [H,d] fp32 transpose of W_r (tensor-core dX epilogue)
+    // fp16 attention path (tensor cores, k > 128): dQKV is [H,B*k,256] fp16
+    // (dQ | dK | dV | dlogit, 0..), and the backward reads X and W_q|W_k|W_v
+    // through fp16 copies so that every product with dQKV is one MMA
+    void *X16;          // [B*T,d] fp16 copy of X
+    void *W16;          // [3][H,d,hp] fp16 copies of W_q, W_k, W_v
 };
 
 // Rotary position encoding (Sec. 2.2): pair p of the first h'/2 dimensions of

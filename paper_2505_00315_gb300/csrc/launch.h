@@ -42,7 +42,8 @@ inline cudaError_t launch_pdl(void (*kernel)(KArgs...), dim3 grid, dim3 block, s
 
 // Raises `kernel`'s dynamic shared-memory limit to `bytes` on the current
 // device.  The attribute is per device, so it is set once for each device
-// (and each kernel) a process uses.
+// (and each kernel) a process uses; `bytes` must therefore be the largest
+// size the kernel is ever launched with, not the size of one launch.
 inline cudaError_t allow_smem(const void *kernel, int bytes) {
     static std::mutex mu;
     static std::set<std::pair<int, const void *>> done;
@@ -163,6 +164,10 @@ cudaError_t tc_dx(const Dims &dm, const void *Wq, const void *Wk, const void *Wv
 // F1 on tensor cores (bf16 inputs, H % 8 == 0); false if not applicable.
 bool tc_router(const Dims &dm, const void *X, const void *Wr, float *r_full, uint32_t *status,
                cudaStream_t s, cudaError_t *err);
+// fp16 attention path: X -> sv.X16 and W_q, W_k, W_v -> sv.W16 (bf16 ->
+// fp16; out-of-range values set kStatusRange).
+cudaError_t tc_f16_copies(const Dims &dm, const void *X, const void *Wq, const void *Wk,
+                          const void *Wv, const Saved &sv, cudaStream_t s);
 // W_r [d,H] bf16 -> sv.WrT [H,d] fp32 (read by the dX epilogue).
 cudaError_t tc_transpose_wr(const Dims &dm, const void *Wr, const Saved &sv, cudaStream_t s);
 cudaError_t tc_attn_fwd(const Dims &dm, const Saved &sv, cudaStream_t s);

@@ -68,6 +68,12 @@ size_t carve(const Dims &dm, char *base, Saved *sv) {
     s.dQKV = take(e * R * 4 * dm.hp);  // 3 h' columns, or 4 blocks of 64 on the tensor cores
     s.G = (float *)take(sizeof(float) * R * dm.hp);
     s.WrT = (float *)take(sizeof(float) * (size_t)dm.d * dm.H);
+    // the fp16 attention path's copies (reserved whenever that path can run,
+    // so the size does not depend on the environment's kernel-path switches)
+    if (dm.bf16 && dm.hp == 64 && dm.k > 128) {
+        s.X16 = take((size_t)2 * dm.B * dm.T * dm.d);
+        s.W16 = take((size_t)2 * 3 * dm.H * dm.d * dm.hp);
+    }
     if (sv) *sv = s;
     return off;
 }
@@ -252,6 +258,9 @@ mosa_status backward_tc(const Dims &dm, const void *X, const void *W_r, const vo
         MOSA_TRY(link(t, s, r.ev[3]));  // join
         return MOSA_OK;
     }
+    // fp16 attention path: fp16 copies of X and W_q|W_k|W_v for the products
+    // with the fp16 dQ|dK|dV (beside G, which leaves room on every SM)
+    if (attn_f16(dm)) MOSA_TRY(tc_f16_copies(dm, X, W_q, W_k, W_v, sv, t));
     {
         StageScope st_(kStageDwo, t);
         MOSA_TRY(tc_out_bwd_w(dm, dY, sv, dW_o, t));
@@ -266,7 +275,8 @@ mosa_status backward_tc(const Dims &dm, const void *X, const void *W_r, const vo
     {
         StageScope st_(kStageAttnBwd, s);
         MOSA_TRY(launch_attn_bwd(dm, sv, s));
-        if (dm.rope) MOSA_TRY(rope_qk(dm, sv, true, s));
+        // (the fp16 path turns dQ and dK back before rounding them)
+        if (dm.rope && !attn_f16(dm)) MOSA_TRY(rope_qk(dm, sv, true, s));
     }
     MOSA_TRY(link(s, t, r.ev[2]));  // dQ|dK|dV|dlogit ready for dW
     {

@@ -327,9 +327,14 @@ struct BwdParams {
     int U, B;                         // k <= 128: sequences per tile, batch
     float scale, scale_log2;
     const float *lse, *Dd;            // [H, B*k]
-    bf16 *dQKV;                       // [H, B*k, 512] pair: dQ|dK|dV|dlogit hi, then lo
+    bf16 *dQKV;                       // k <= 128: [H, B*k, 512] pair: dQ|dK|dV|dlogit hi, then lo
+                                      // k > 128: [H, B*k, 256] fp16 dQ|dK|dV|dlogit
     float *dQacc;                     // k > 128: [H, B*k, 64] fp32 dQ accumulator (zeroed)
     uint32_t *status;
+    // k > 128 with RoPE: dK is turned back (Sec. 2.2) before its fp16 rounding
+    const int32_t *gidx;              // [H, B*k]: b*T + t
+    int rope, T;
+    RopeTable rope_tab;
 };
 
 template <class SM>
@@ -368,7 +373,8 @@ __device__ __forceinline__ void flag_timeout_b(SM &sm, uint32_t *status) {
 // the workers drain two blocks late), and lse and D of block i+1 are loaded
 // during block i.  Barriers of double-buffered data come in pairs, one per
 // buffer, so no waiter can see its barrier complete two phases ahead.
-// dK / sqrt(h') and dV are written once at the end as bf16 pairs.  Q_i and
+// dK / sqrt(h') and dV are written once at the end as fp16 (dK turned back
+// by RoPE first when asked) into dQ|dK|dV|dlogit rows.  Q_i and
 // dA_i go to ring slots 2 (i % 3) and 2 (i % 3) + 1, so each load is issued
 // up to three blocks ahead of its use (a two-block ring left the MMA issuer
 // waiting about 1 us per block for Q_{i+1}).
@@ -632,28 +638,40 @@ __global__ void __launch_bounds__(kBT, 1) attn_bwd_tc_kernel(const __grid_consta
         const bool done = bwait(sm, sm.acc_done, 0, p.status);
         tc_fence_after();
         const int kj = j0 + r;
-        const unsigned kmask = __ballot_sync(0xffffffffu, kj < p.k);
         const bool live = __all_sync(0xffffffffu, ok && done && !*(volatile int *)&sm.abort) && nb > 0;
         const uint32_t src[2] = {tDK, tDV};
         const float fac[2] = {p.scale, 1.f};
-        uint8_t *xb = &sm.p[0][0] + (warp - 4) * 4096;   // the P tile is idle now
-        bool finite = true;
+        const int tpos = (p.rope && kj < p.k) ? p.gidx[base + kj] % p.T : 0;
+        float vmax = 0.f;   // an out-of-range dS made these non-finite
 #pragma unroll
         for (int t = 0; t < 2; ++t) {
             float v[32];
             tmem_ld32(src[t] + lane_off + 32 * ch, v);
             if (!live) continue;
 #pragma unroll
-            for (int c = 0; c < 32; ++c) finite = finite && fabsf(v[c]) < INFINITY;
-            stage_pair32(xb, v, fac[t], lane);
-            store_rows128(xb, lane, [&](int rl, int c) -> uint4 * {
-                if (!((kmask >> rl) & 1u)) return nullptr;
-                bf16 *row = p.dQKV + (base + j0 + q * 32 + rl) * 512 + 64 * (t + 1) + 32 * ch;
-                return c < 4 ? reinterpret_cast<uint4 *>(row) + c
-                             : reinterpret_cast<uint4 *>(row + 256) + (c - 4);
-            });
+            for (int c = 0; c < 32; ++c) v[c] *= fac[t];
+            if (t == 0 && p.rope && ch == 0) {
+                // dK columns 0..31 are the turned pairs (2p, 2p+1), p < 16
+#pragma unroll
+                for (int pp = 0; pp < 16; ++pp)
+                    rope_turn(v[2 * pp], v[2 * pp + 1], p.rope_tab.phi[pp], tpos, -1.f);
+            }
+            if (kj < p.k) {
+                __half *row = reinterpret_cast<__half *>(p.dQKV) + (base + kj) * 256 + 64 * (t + 1) + 32 * ch;
+#pragma unroll
+                for (int u = 0; u < 4; ++u) {
+                    uint32_t w[4];
+#pragma unroll
+                    for (int e = 0; e < 4; ++e) {
+                        const float a = v[8 * u + 2 * e], c2 = v[8 * u + 2 * e + 1];
+                        vmax = fmaxf(vmax, fmaxf(fabsf(a), fabsf(c2)));
+                        w[e] = pack_f16x2(a, c2);
+                    }
+                    reinterpret_cast<uint4 *>(row)[u] = make_uint4(w[0], w[1], w[2], w[3]);
+                }
+            }
         }
-        if (live && !finite && kj < p.k) atomicOr(p.status, kStatusRange);
+        if (live && kj < p.k && !(vmax < kF16Overflow)) atomicOr(p.status, kStatusRange);
     }
     tc_fence_before();
     __syncthreads();
@@ -663,20 +681,29 @@ __global__ void __launch_bounds__(kBT, 1) attn_bwd_tc_kernel(const __grid_consta
     }
 }
 
-// dQ from its fp32 accumulator into columns 0..63 (hi) / 256..319 (lo) of the
-// dQKV pair rows, two columns per thread.
-__global__ void dq_finish_kernel(const float *__restrict__ dQacc, bf16 *__restrict__ dQKV, size_t rows) {
+// dQ from its fp32 accumulator into columns 0..63 of the dQ|dK|dV|dlogit rows,
+// two columns per thread: as a bf16 pair ([hi 256 | lo 256] rows), or (f16)
+// as fp16 rows of 256, turned back by RoPE first when asked (gidx, rope).
+__global__ void dq_finish_kernel(const float *__restrict__ dQacc, bf16 *__restrict__ dQKV, size_t rows,
+                                 int f16, const int32_t *__restrict__ gidx, int rope, int T,
+                                 RopeTable tab, uint32_t *status) {
     pdl_trigger();  // the next kernel (zeroing dX) may run beside this one
     pdl_wait();
     const size_t idx = (size_t)blockIdx.x * blockDim.x + threadIdx.x;   // (row, column pair)
     if (idx >= rows * 32) return;
     const size_t row = idx >> 5;
     const int c = (int)(idx & 31) * 2;
-    const float2 v = *reinterpret_cast<const float2 *>(dQacc + row * 64 + c);
-    uint32_t hi, lo;
-    split_pair2(v.x, v.y, hi, lo);
-    *reinterpret_cast<uint32_t *>(dQKV + row * 512 + c) = hi;
-    *reinterpret_cast<uint32_t *>(dQKV + row * 512 + 256 + c) = lo;
+    float2 v = *reinterpret_cast<const float2 *>(dQacc + row * 64 + c);
+    if (!f16) {
+        uint32_t hi, lo;
+        split_pair2(v.x, v.y, hi, lo);
+        *reinterpret_cast<uint32_t *>(dQKV + row * 512 + c) = hi;
+        *reinterpret_cast<uint32_t *>(dQKV + row * 512 + 256 + c) = lo;
+        return;
+    }
+    if (rope && c < 32) rope_turn(v.x, v.y, tab.phi[c >> 1], gidx[row] % T, -1.f);
+    *reinterpret_cast<uint32_t *>(reinterpret_cast<__half *>(dQKV) + row * 256 + c) = pack_f16x2(v.x, v.y);
+    if (!(fabsf(v.x) < kF16Overflow) || !(fabsf(v.y) < kF16Overflow)) atomicOr(status, kStatusRange);
 }
 
 // ------------------------------------------------- k <= 128: one CTA per tile
@@ -1117,6 +1144,10 @@ cudaError_t tc_attn_bwd(const Dims &dm, const Saved &sv, cudaStream_t s) {
     bp.dQKV = static_cast<bf16 *>(sv.dQKV);
     bp.dQacc = sv.G;
     bp.status = sv.status;
+    bp.gidx = sv.gidx;
+    bp.T = dm.T;
+    bp.rope = dm.rope ? 1 : 0;
+    if (dm.rope) bp.rope_tab = make_rope_table(dm.hp, dm.T);
     {
         // dQ accumulator [H, B, k, 64] fp32 (the workspace's G buffer)
         const uint64_t dims[4] = {64, (uint64_t)dm.k, (uint64_t)dm.B, (uint64_t)dm.H};
@@ -1134,7 +1165,8 @@ cudaError_t tc_attn_bwd(const Dims &dm, const Saved &sv, cudaStream_t s) {
     const size_t n = rows * 32;
     if (e == cudaSuccess)
         e = launch_pdl(dq_finish_kernel, dim3((unsigned)((n + 255) / 256)), dim3(256), 0, s,
-                       (const float *)sv.G, static_cast<bf16 *>(sv.dQKV), rows);
+                       (const float *)sv.G, static_cast<bf16 *>(sv.dQKV), rows, 1,
+                       (const int32_t *)sv.gidx, bp.rope, dm.T, bp.rope_tab, sv.status);
     note_launches(2);
     return e;
 }

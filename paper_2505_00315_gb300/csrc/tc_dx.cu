@@ -16,7 +16,9 @@
 // 256-column halves of TMEM, so the scatter-add of one chunk (red.add.v4
 // through a per-warp staging buffer; for dX with dlogit x W_r added from an
 // fp32 transpose of W_r) runs while the MMAs of the next one do.  Each
-// product with a pair operand is two MMAs (hi, lo).
+// product with a pair operand is two MMAs (hi, lo); on the fp16 attention
+// path (k > 128) dX reads dQ|dK|dV as single fp16 values and fp16 copies of
+// W_q|W_k|W_v, one MMA.
 // Warps: 0 TMA producer, 1 MMA issuer, 2 TMEM owner, 3 idle, 4-11 epilogue
 // (warp w: tile rows 32 (w % 4) .. +31, chunk columns 128 ((w - 4) / 4) ..).
 // Every wait is bounded.
@@ -61,6 +63,7 @@ struct DxParams {
     int mt, nch;          // tiles per head, chunks per tile
     long long units;      // H * mt * nch
     uint32_t *status;
+    int f16;              // dX: A = fp16 dQKV rows [H, B*k, 256], W = fp16 copies (one MMA)
 };
 
 __device__ __forceinline__ bool dwait(DxSmem &sm, uint64_t &bar, uint32_t parity, uint32_t *status) {
@@ -130,9 +133,10 @@ __global__ void __launch_bounds__(kThreads, 1) scatter_product_kernel(const __gr
                         if (ntile > 0 && !(ok = dwait(sm, sm.a_empty[j], (ntile - 1) & 1, p.status)))
                             break;
                         const uint32_t ab = smem_u32(&sm.a_full[j]);
-                        mbar_expect_tx(ab, 2 * kTileHalf);
+                        mbar_expect_tx(ab, (p.f16 ? 1 : 2) * kTileHalf);
                         tma_load_3d(smem_u32(sm.a[j][0]), &p.mA, ab, 64 * j, m0, h);        // hi
-                        tma_load_3d(smem_u32(sm.a[j][1]), &p.mA, ab, kLo + 64 * j, m0, h);  // lo
+                        if (!p.f16)
+                            tma_load_3d(smem_u32(sm.a[j][1]), &p.mA, ab, kLo + 64 * j, m0, h);  // lo
                     }
                     const uint32_t fb = smem_u32(&sm.w_full[s]);
                     mbar_expect_tx(fb, kWBytes);
@@ -151,7 +155,9 @@ __global__ void __launch_bounds__(kThreads, 1) scatter_product_kernel(const __gr
     } else if (warp == 1) {
         if (lane == 0) {
             // B: W_j blocks K-major (dX), W_o chunks MN-major (Y)
-            constexpr uint32_t idX = idesc_bf16(128, kChunk, false, kOut);
+            const uint32_t idX = p.f16 ? idesc_f16(128, kChunk, false, kOut)
+                                       : idesc_bf16(128, kChunk, false, kOut);
+            const int halves = p.f16 ? 1 : 2;
             bool ok = true;
             int ntile = 0;
             for (int i = 0; i < nu && ok; ++i) {
@@ -166,8 +172,7 @@ __global__ void __launch_bounds__(kThreads, 1) scatter_product_kernel(const __gr
                     if (!(ok = dwait(sm, sm.w_full[s], (idx / kSlots) & 1, p.status))) break;
                     tc_fence_after();
                     const uint32_t wb = smem_u32(sm.w[s]);
-#pragma unroll
-                    for (int half = 0; half < 2; ++half)
+                    for (int half = 0; half < halves; ++half)
 #pragma unroll
                         for (int kk = 0; kk < 4; ++kk)
                             mma_bf16(tmem + 256 * buf,
@@ -250,6 +255,7 @@ __global__ void __launch_bounds__(kThreads, 1) scatter_product_kernel(const __gr
     }
 }
 
+// [H, rows, cols] array of 16-bit elements, box {64, box_rows, 1}.
 bool map3(CUtensorMap *m, const void *base, uint64_t H, uint64_t rows, uint64_t cols,
           uint32_t box_rows) {
     const uint64_t dims[3] = {cols, rows, H}, strides[2] = {cols * 2, rows * cols * 2};
@@ -285,8 +291,12 @@ cudaError_t tc_dx(const Dims &dm, const void *Wq, const void *Wk, const void *Wv
     memset(&p, 0, sizeof(p));
     const int Mtok = dm.B * dm.k;
     if (Mtok <= 0 || dm.d <= 0 || dm.H <= 0) return cudaSuccess;
+    p.f16 = attn_f16(dm) ? 1 : 0;
+    const size_t nw = (size_t)dm.H * dm.d * 64;
     const void *W[3] = {Wq, Wk, Wv};
-    bool ok = map3(&p.mA, sv.dQKV, dm.H, Mtok, 512, 128);
+    if (p.f16)
+        for (int j = 0; j < 3; ++j) W[j] = static_cast<const char *>(sv.W16) + 2 * nw * j;
+    bool ok = map3(&p.mA, sv.dQKV, dm.H, Mtok, p.f16 ? 256 : 512, 128);
     for (int j = 0; j < 3; ++j) ok = ok && map3(&p.mW[j], W[j], dm.H, dm.d, 64, 256);
     if (!ok) return cudaErrorInvalidValue;
     p.gidx = sv.gidx;

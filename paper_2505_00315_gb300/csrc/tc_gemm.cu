@@ -417,7 +417,9 @@ __global__ void __launch_bounds__(kThreads, Cfg<KIND>::MIN_CTAS)
             const int kb = kb_begin + it;
             const uint32_t a = smem_u32(stage_a(s)), b = smem_u32(stage_b(s));
             if (lane == 0) {
+                // (kDW on the fp16 path: dQ|dK|dV|dlogit single, half the B bytes)
                 const uint32_t tx = KIND == kROUTER ? C::A_BYTES + nbl * kTile8K
+                                    : (KIND == kDW && p.half) ? C::B_BYTES / 2
                                     : gathers<KIND>() ? C::B_BYTES : C::A_BYTES + C::B_BYTES;
                 mbar_expect_tx(fb, tx);
             }
@@ -432,8 +434,9 @@ __global__ void __launch_bounds__(kThreads, Cfg<KIND>::MIN_CTAS)
                     tma_load_2d(b + (lane - 1) * kTile8K, &p.mapB[0], fb, n0 + 64 * (lane - 1), kb * kBK);
             } else if constexpr (KIND == kDWO) {
                 if (lane < 2) tma_load_3d(b + lane * kTile8K, &p.mapB[0], fb, 64 * lane, kb * kBK, h);
-            } else {  // kDW: hi blocks 0..3 then lo blocks 0..3, 32 token rows each
-                if (lane < 8) tma_load_3d(b + lane * 4096, &p.mapB[0], fb, 64 * lane, kb * 32, h);
+            } else {  // kDW: hi blocks 0..3 then lo blocks 0..3 (fp16: blocks 0..3), 32 token rows each
+                if (lane < (p.half ? 4 : 8))
+                    tma_load_3d(b + lane * 4096, &p.mapB[0], fb, 64 * lane, kb * 32, h);
             }
             issued = it + 1;
         }
@@ -446,7 +449,8 @@ __global__ void __launch_bounds__(kThreads, Cfg<KIND>::MIN_CTAS)
         // ------------------------------------------------------ MMA issuer
         if (lane == 0) {
             const uint32_t idesc = KIND == kROUTER ? idesc_bf16(kBM, p.N, false, true)
-                                                   : idesc_bf16(kBM, C::BN, C::A_MN, C::B_MN);
+                                   : (KIND == kDW && p.half) ? idesc_f16(kBM, C::BN, C::A_MN, C::B_MN)
+                                   : idesc_bf16(kBM, C::BN, C::A_MN, C::B_MN);
             for (int it = 0; it < nkb; ++it) {
                 const int s = it % ns;
                 if (!mbar_wait(smem_u32(&full[s]), (it / ns) & 1) || *(volatile int *)s_abort) {
@@ -459,10 +463,11 @@ __global__ void __launch_bounds__(kThreads, Cfg<KIND>::MIN_CTAS)
                 constexpr int pairs = (C::A_PAIR || C::B_PAIR) ? 2 : 1;
                 if constexpr (KIND == kDW) {
                     // accumulator c: rows of d-blocks 2c, 2c+1; B pair halves at +0 / +16 KB
+                    // (fp16: one B block set)
+                    const int halves = p.half ? 1 : 2;
 #pragma unroll
                     for (int c = 0; c < 2; ++c)
-#pragma unroll
-                        for (int half = 0; half < 2; ++half)
+                        for (int half = 0; half < halves; ++half)
 #pragma unroll
                             for (int j = 0; j < 2; ++j)
                                 mma_bf16(tmem + 256 * c,
@@ -616,12 +621,17 @@ __global__ void __launch_bounds__(kThreads, Cfg<KIND>::MIN_CTAS)
             // the 4th 64-column block that kDW reads for dW_r; the block's other
             // columns are never written: accumulator column n of that product
             // depends only on B column n, and columns 193..255 are not read
-            if (live) {
+            if (live && !p.half) {
                 const bf16 dh = __float2bfloat16_rn(dl);
                 const bf16 dlo = __float2bfloat16_rn(dl - __bfloat162float(dh));
                 bf16 *dq = static_cast<bf16 *>(p.out[1]) + row * kDQKVCols;
                 dq[192] = dh;
                 dq[448] = dlo;
+            } else if (live) {
+                // fp16 rows [H, B*k, 256]: dlogit at column 192
+                __half *dq = static_cast<__half *>(p.out[1]) + row * 256;
+                dq[192] = __float2half_rn(dl);
+                if (!(fabsf(dl) < kF16Overflow)) atomicOr(p.status, kStatusRange);
             }
         } else if constexpr (KIND == kROUTER) {
             const bool live = mg < p.M;
@@ -790,6 +800,31 @@ bool tc_router(const Dims &dm, const void *X, const void *Wr, float *r_full, uin
     return true;
 }
 
+// bf16 -> fp16, eight values per 16-byte step.  Exact for magnitudes in
+// [2^-17, 65504] (fp16 has three more significand bits than bf16); smaller
+// ones round to fp16's subnormal grid (2^-24); a value beyond the fp16 range
+// sets kStatusRange.
+__global__ void to_f16_kernel(const uint4 *__restrict__ src, uint4 *__restrict__ dst, size_t n8,
+                              uint32_t *status) {
+    pdl_wait();
+    pdl_trigger();
+    bool bad = false;
+    for (size_t i = (size_t)blockIdx.x * blockDim.x + threadIdx.x; i < n8;
+         i += (size_t)gridDim.x * blockDim.x) {
+        const uint4 u = src[i];
+        const uint32_t w[4] = {u.x, u.y, u.z, u.w};
+        uint32_t o[4];
+#pragma unroll
+        for (int e = 0; e < 4; ++e) {
+            const float lo = __uint_as_float(w[e] << 16), hi = __uint_as_float(w[e] & 0xFFFF0000u);
+            bad = bad || !(fabsf(lo) < kF16Overflow) || !(fabsf(hi) < kF16Overflow);
+            o[e] = pack_f16x2(lo, hi);
+        }
+        dst[i] = make_uint4(o[0], o[1], o[2], o[3]);
+    }
+    if (__any_sync(0xffffffffu, bad) && (threadIdx.x & 31) == 0) atomicOr(status, kStatusRange);
+}
+
 __global__ void transpose_wr_kernel(const bf16 *__restrict__ Wr, float *__restrict__ WrT, int d,
                                     int H) {
     pdl_wait();
@@ -798,6 +833,24 @@ __global__ void transpose_wr_kernel(const bf16 *__restrict__ Wr, float *__restri
         const int h = i / d, c = i - h * d;
         WrT[i] = __bfloat162float(Wr[(size_t)c * H + h]);
     }
+}
+
+cudaError_t tc_f16_copies(const Dims &dm, const void *X, const void *Wq, const void *Wk,
+                          const void *Wv, const Saved &sv, cudaStream_t s) {
+    const size_t nw = (size_t)dm.H * dm.d * dm.hp;
+    const void *src[4] = {X, Wq, Wk, Wv};
+    void *dst[4] = {sv.X16, sv.W16, (char *)sv.W16 + 2 * nw, (char *)sv.W16 + 4 * nw};
+    const size_t n[4] = {(size_t)dm.B * dm.T * dm.d, nw, nw, nw};
+    for (int i = 0; i < 4; ++i) {
+        const size_t n8 = n[i] / 8;   // d % 8 == 0
+        const unsigned grid = (unsigned)std::min<size_t>((n8 + 255) / 256, 1216);
+        to_f16_kernel<<<grid, 256, 0, s>>>(static_cast<const uint4 *>(src[i]),
+                                           static_cast<uint4 *>(dst[i]), n8, sv.status);
+        note_launches(1);
+        const cudaError_t e = cudaGetLastError();
+        if (e != cudaSuccess) return e;
+    }
+    return cudaSuccess;
 }
 
 cudaError_t tc_transpose_wr(const Dims &dm, const void *Wr, const Saved &sv, cudaStream_t s) {
@@ -907,10 +960,14 @@ cudaError_t tc_w_bwd(const Dims &dm, const void *X, const Saved &sv, float *dWq,
     // one wave of single-CTA SMs: the most reduction splits with tiles * splits <= 152
     p.splits = 1;
     while (tiles * p.splits * 2 <= 152 && p.splits * 4 <= p.nkb) p.splits *= 2;
-    bool ok = map_gather(&p.mapA, X, (uint64_t)dm.B * dm.T, dm.d) &&
-              map_heads(&p.mapB[0], sv.dQKV, dm.H, p.Mtok, kDQKVCols, 32);
+    // fp16 attention path: dQ|dK|dV|dlogit single fp16 rows of 256, and the
+    // gathered rows from the fp16 copy of X, one MMA per step
+    p.half = attn_f16(dm) ? 1 : 0;
+    const void *Xs = p.half ? sv.X16 : X;
+    bool ok = map_gather(&p.mapA, Xs, (uint64_t)dm.B * dm.T, dm.d) &&
+              map_heads(&p.mapB[0], sv.dQKV, dm.H, p.Mtok, p.half ? 256 : kDQKVCols, 32);
     if (!ok) return cudaErrorInvalidValue;
-    p.src_rows = X;
+    p.src_rows = Xs;
     p.out_f = dWq;
     p.out_f1 = dWk;
     p.out_f2 = dWv;

@@ -255,6 +255,8 @@ KERNEL_STAGE = [("tc_gemm_kernel<5>", "router"), ("tc_gemm_kernel<(int)5>", "rou
                 ("scatter_product_kernel<0>", "in_bwd"), ("scatter_product_kernel<false>", "in_bwd"),
                 ("scatter_product_kernel<1>", "out"), ("scatter_product_kernel<true>", "out"),
                 ("tc_gemm_kernel<4>", "w_bwd"), ("tc_gemm_kernel<(int)4>", "w_bwd"),
+                ("tc_gemm_kernel<6>", "w_bwd"), ("tc_gemm_kernel<(int)6>", "w_bwd"),
+                ("to_f16_kernel", "dwo"),
                 ("tc_gemm_kernel<3>", "dwo"), ("tc_gemm_kernel<(int)3>", "dwo"),
                 ("fused_fwd_kernel", "fwd_unit"), ("fused_bwd_kernel", "bwd_unit"),
                 ("dense_rows", "select")]

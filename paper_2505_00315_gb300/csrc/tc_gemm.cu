@@ -46,7 +46,7 @@ namespace {
 using namespace tc;
 
 // (the values name the kernel instances tc_gemm_kernel<N> in profiles)
-enum Kind : int { kQKV = 0, kG = 2, kDWO = 3, kDW = 4, kROUTER = 5 };
+enum Kind : int { kQKV = 0, kG = 2, kDWO = 3, kDW = 4, kROUTER = 5, kDWH = 6 };
 
 constexpr int kBM = 128;        // rows per tile (TMEM lanes)
 constexpr int kBK = 64;         // K per stage: one 128-byte swizzle row of bf16
@@ -85,6 +85,16 @@ struct Cfg<kDW> {
 };
 
 template <>
+struct Cfg<kDWH> {
+    // kDW on the fp16 attention path: dQ|dK|dV|dlogit single fp16 (B 16 KB a
+    // stage), so the ring holds six stages and the gathers of X run four
+    // stages ahead (with four they ran two ahead and bound the kernel)
+    static constexpr int BN = 256, STAGES = 6, A_BYTES = 4 * 4096, B_BYTES = 4 * 4096,
+                         TMEM_COLS = 512, MIN_CTAS = 1;
+    static constexpr bool A_MN = true, B_MN = true, A_PAIR = false, B_PAIR = false;
+};
+
+template <>
 struct Cfg<kROUTER> {
     // ring of 192 KB; the stage count is chosen at launch from the MMA width
     // (p.N = 64..256): a stage holds the X tile and N/64 W_r blocks
@@ -96,11 +106,11 @@ struct Cfg<kROUTER> {
 // Tokens per K block and accumulators (128-row tiles) per CTA.
 template <int KIND>
 __host__ __device__ constexpr int kind_bk() {
-    return KIND == kDW ? 32 : kBK;
+    return (KIND == kDW || KIND == kDWH) ? 32 : kBK;
 }
 template <int KIND>
 __host__ __device__ constexpr int kind_acc() {
-    return KIND == kDW ? 2 : 1;
+    return (KIND == kDW || KIND == kDWH) ? 2 : 1;
 }
 
 // Row width (bf16) of the dQKV pair array on the tensor-core path:
@@ -110,19 +120,30 @@ constexpr int kDQKVCols = 512;
 // Kinds whose A operand is gathered through the selected rows.
 template <int KIND>
 __host__ __device__ constexpr bool gathers() {
-    return KIND == kQKV || KIND == kG || KIND == kDWO || KIND == kDW;
+    return KIND == kQKV || KIND == kG || KIND == kDWO || KIND == kDW || KIND == kDWH;
 }
 
 // Kinds whose epilogue runs on all eight warps (wide output tiles).
 template <int KIND>
 __host__ __device__ constexpr bool epi_all_warps() {
-    return KIND == kQKV || KIND == kDW || KIND == kDWO || KIND == kROUTER;
+    return KIND == kQKV || KIND == kDW || KIND == kDWH || KIND == kDWO || KIND == kROUTER;
 }
+
+// Kinds whose gathered operand runs along the reduction (tokens of K blocks):
+// their row indices are staged in shared memory for the CTA's whole K range
+// when it holds at most kIdxMax tokens (each K block otherwise began with a
+// dependent global load of its indices, about one memory latency per block).
+template <int KIND>
+__host__ __device__ constexpr bool stages_idx() {
+    return KIND == kDWO || KIND == kDW || KIND == kDWH;
+}
+constexpr int kIdxMax = 2048;
 
 template <int KIND>
 constexpr int smem_bytes() {
     return 1024 /* alignment slack */ + Cfg<KIND>::STAGES * (Cfg<KIND>::A_BYTES + Cfg<KIND>::B_BYTES) +
-           2048 /* barriers, row indices, row scalars */;
+           2048 /* barriers, row indices, row scalars */ +
+           (stages_idx<KIND>() ? kIdxMax * 4 : 0) /* K-range row indices */;
 }
 
 struct TcParams {
@@ -256,7 +277,8 @@ __device__ __forceinline__ void stage_f32_32(uint8_t *xb, uint32_t taddr, int la
 template <int KIND>
 __device__ __forceinline__ void gather_operand(const TcParams &p, uint8_t *sA, uint64_t *full,
                                                uint64_t *empty, const int *s_rows, int *s_abort,
-                                               int h, int m0, int kb_begin, int nkb) {
+                                               int h, int m0, int kb_begin, int nkb,
+                                               const int *s_idx, int tok0, bool idx_staged) {
     using C = Cfg<KIND>;
     constexpr int S = C::STAGES;
     constexpr int LAG = S >= 3 ? S - 2 : S - 1;  // a two-stage ring keeps one stage of lag
@@ -283,13 +305,13 @@ __device__ __forceinline__ void gather_operand(const TcParams &p, uint8_t *sA, u
                 const bf16 *g = src + (size_t)s_rows[row] * p.d + (nbytes ? col : 0);
                 cp_async16(a + row * 128 + ((chunk ^ (row & 7)) << 4), g, nbytes);
             }
-        } else if constexpr (KIND == kDW) {
+        } else if constexpr (KIND == kDW || KIND == kDWH) {
             // 32 tokens x 256 columns of d in four 64-wide blocks of 4 KB
 #pragma unroll
             for (int q2 = 0; q2 < 2; ++q2) {
                 const int tok = sub + 16 * q2;
                 const int tg = kb * 32 + tok;
-                const int rowg = tg < p.Mtok ? gi[tg] : 0;
+                const int rowg = idx_staged ? s_idx[tg - tok0] : (tg < p.Mtok ? gi[tg] : 0);
 #pragma unroll
                 for (int j = 0; j < 4; ++j) {
                     const int col = m0 + 64 * j + chunk * 8;
@@ -303,7 +325,7 @@ __device__ __forceinline__ void gather_operand(const TcParams &p, uint8_t *sA, u
             for (int q4 = 0; q4 < 4; ++q4) {
                 const int tok = sub + 16 * q4;
                 const int tg = kb * kBK + tok;
-                const int rowg = tg < p.Mtok ? gi[tg] : 0;
+                const int rowg = idx_staged ? s_idx[tg - tok0] : (tg < p.Mtok ? gi[tg] : 0);
 #pragma unroll
                 for (int j = 0; j < 2; ++j) {
                     const int col = m0 + 64 * j + chunk * 8;
@@ -354,17 +376,19 @@ __global__ void __launch_bounds__(kThreads, Cfg<KIND>::MIN_CTAS)
     int *s_abort = reinterpret_cast<int *>(tmem_slot + 1);
     int *s_rows = s_abort + 1 + 2;  // 128 gather rows, 16-byte aligned below
     s_rows = reinterpret_cast<int *>((reinterpret_cast<uintptr_t>(s_rows) + 15) & ~uintptr_t(15));
+    int *s_idx = s_rows + 128;      // stages_idx kinds: row indices of the CTA's K range
     static_assert(KIND == kROUTER || S * (C::A_BYTES + C::B_BYTES) >= 8 * kXpose,
                   "epilogue staging must fit in the operand ring");
 
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     const int m_tile = blockIdx.x, n_tile = blockIdx.y;
-    const int h = (KIND == kDWO || KIND == kDW) ? blockIdx.z / p.splits : blockIdx.z;
-    const int split = (KIND == kDWO || KIND == kDW) ? blockIdx.z % p.splits : 0;
+    constexpr bool kSplitK = KIND == kDWO || KIND == kDW || KIND == kDWH;
+    const int h = kSplitK ? blockIdx.z / p.splits : blockIdx.z;
+    const int split = kSplitK ? blockIdx.z % p.splits : 0;
     const int m0 = m_tile * kBM * kind_acc<KIND>();
     const int n0 = n_tile * C::BN;
     int kb_begin = 0, kb_end = p.nkb;
-    if (KIND == kDWO || KIND == kDW) {
+    if (kSplitK) {
         const int per = (p.nkb + p.splits - 1) / p.splits;
         kb_begin = split * per;
         kb_end = min(p.nkb, kb_begin + per);
@@ -386,6 +410,14 @@ __global__ void __launch_bounds__(kThreads, Cfg<KIND>::MIN_CTAS)
         for (int r = threadIdx.x; r < kBM; r += kThreads) {
             const int m = m0 + r;
             s_rows[r] = m < p.Mtok ? p.gidx[(size_t)h * p.Mtok + m] : 0;
+        }
+    }
+    const int tok0 = kb_begin * kind_bk<KIND>();
+    const bool idx_staged = stages_idx<KIND>() && nkb * kind_bk<KIND>() <= kIdxMax;
+    if (idx_staged) {
+        for (int i = threadIdx.x; i < nkb * kind_bk<KIND>(); i += kThreads) {
+            const int tg = tok0 + i;
+            s_idx[i] = tg < p.Mtok ? p.gidx[(size_t)h * p.Mtok + tg] : 0;
         }
     }
     if (warp == 2) {
@@ -417,9 +449,7 @@ __global__ void __launch_bounds__(kThreads, Cfg<KIND>::MIN_CTAS)
             const int kb = kb_begin + it;
             const uint32_t a = smem_u32(stage_a(s)), b = smem_u32(stage_b(s));
             if (lane == 0) {
-                // (kDW on the fp16 path: dQ|dK|dV|dlogit single, half the B bytes)
                 const uint32_t tx = KIND == kROUTER ? C::A_BYTES + nbl * kTile8K
-                                    : (KIND == kDW && p.half) ? C::B_BYTES / 2
                                     : gathers<KIND>() ? C::B_BYTES : C::A_BYTES + C::B_BYTES;
                 mbar_expect_tx(fb, tx);
             }
@@ -434,9 +464,10 @@ __global__ void __launch_bounds__(kThreads, Cfg<KIND>::MIN_CTAS)
                     tma_load_2d(b + (lane - 1) * kTile8K, &p.mapB[0], fb, n0 + 64 * (lane - 1), kb * kBK);
             } else if constexpr (KIND == kDWO) {
                 if (lane < 2) tma_load_3d(b + lane * kTile8K, &p.mapB[0], fb, 64 * lane, kb * kBK, h);
-            } else {  // kDW: hi blocks 0..3 then lo blocks 0..3 (fp16: blocks 0..3), 32 token rows each
-                if (lane < (p.half ? 4 : 8))
-                    tma_load_3d(b + lane * 4096, &p.mapB[0], fb, 64 * lane, kb * 32, h);
+            } else if constexpr (KIND == kDWH) {  // fp16 blocks 0..3, 32 token rows each
+                if (lane < 4) tma_load_3d(b + lane * 4096, &p.mapB[0], fb, 64 * lane, kb * 32, h);
+            } else {  // kDW: hi blocks 0..3 then lo blocks 0..3, 32 token rows each
+                if (lane < 8) tma_load_3d(b + lane * 4096, &p.mapB[0], fb, 64 * lane, kb * 32, h);
             }
             issued = it + 1;
         }
@@ -449,7 +480,7 @@ __global__ void __launch_bounds__(kThreads, Cfg<KIND>::MIN_CTAS)
         // ------------------------------------------------------ MMA issuer
         if (lane == 0) {
             const uint32_t idesc = KIND == kROUTER ? idesc_bf16(kBM, p.N, false, true)
-                                   : (KIND == kDW && p.half) ? idesc_f16(kBM, C::BN, C::A_MN, C::B_MN)
+                                   : KIND == kDWH ? idesc_f16(kBM, C::BN, C::A_MN, C::B_MN)
                                    : idesc_bf16(kBM, C::BN, C::A_MN, C::B_MN);
             for (int it = 0; it < nkb; ++it) {
                 const int s = it % ns;
@@ -461,12 +492,13 @@ __global__ void __launch_bounds__(kThreads, Cfg<KIND>::MIN_CTAS)
                 tc_fence_after();
                 const uint32_t a = smem_u32(stage_a(s)), b = smem_u32(stage_b(s));
                 constexpr int pairs = (C::A_PAIR || C::B_PAIR) ? 2 : 1;
-                if constexpr (KIND == kDW) {
+                if constexpr (KIND == kDW || KIND == kDWH) {
                     // accumulator c: rows of d-blocks 2c, 2c+1; B pair halves at +0 / +16 KB
-                    // (fp16: one B block set)
-                    const int halves = p.half ? 1 : 2;
+                    // (kDWH: one fp16 B block set)
+                    constexpr int halves = KIND == kDWH ? 1 : 2;
 #pragma unroll
                     for (int c = 0; c < 2; ++c)
+#pragma unroll
                         for (int half = 0; half < halves; ++half)
 #pragma unroll
                             for (int j = 0; j < 2; ++j)
@@ -494,7 +526,7 @@ __global__ void __launch_bounds__(kThreads, Cfg<KIND>::MIN_CTAS)
         }
     } else if (warp >= 4) {
         if constexpr (gathers<KIND>()) gather_operand<KIND>(p, sA, full, empty, s_rows, s_abort, h, m0,
-                                                            kb_begin, nkb);
+                                                            kb_begin, nkb, s_idx, tok0, idx_staged);
     }
 
     // ------------------------------------------------------------ epilogue
@@ -674,7 +706,7 @@ __global__ void __launch_bounds__(kThreads, Cfg<KIND>::MIN_CTAS)
                         *reinterpret_cast<float4 *>(dst) = val;
                 }
             }
-        } else {  // kDW: warps 4-7 accumulator 0 (d rows m0 ..), warps 0-3 accumulator 1 (m0+128 ..)
+        } else {  // kDW / kDWH: warps 4-7 accumulator 0 (d rows m0 ..), warps 0-3 accumulator 1 (m0+128 ..)
             const int chunk = lane & 7;
             const uint32_t ta = tb + 256 * part;
             const int mrow0 = m0 + 128 * part + q * 32;
@@ -962,10 +994,10 @@ cudaError_t tc_w_bwd(const Dims &dm, const void *X, const Saved &sv, float *dWq,
     while (tiles * p.splits * 2 <= 152 && p.splits * 4 <= p.nkb) p.splits *= 2;
     // fp16 attention path: dQ|dK|dV|dlogit single fp16 rows of 256, and the
     // gathered rows from the fp16 copy of X, one MMA per step
-    p.half = attn_f16(dm) ? 1 : 0;
-    const void *Xs = p.half ? sv.X16 : X;
+    const bool half = attn_f16(dm);
+    const void *Xs = half ? sv.X16 : X;
     bool ok = map_gather(&p.mapA, Xs, (uint64_t)dm.B * dm.T, dm.d) &&
-              map_heads(&p.mapB[0], sv.dQKV, dm.H, p.Mtok, p.half ? 256 : kDQKVCols, 32);
+              map_heads(&p.mapB[0], sv.dQKV, dm.H, p.Mtok, half ? 256 : kDQKVCols, 32);
     if (!ok) return cudaErrorInvalidValue;
     p.src_rows = Xs;
     p.out_f = dWq;
@@ -982,7 +1014,7 @@ cudaError_t tc_w_bwd(const Dims &dm, const void *X, const Saved &sv, float *dWq,
             return e;
     }
     dim3 grid((dm.d + 255) / 256, 1, dm.H * p.splits);
-    return launch_kind<kDW>(p, grid, s);
+    return half ? launch_kind<kDWH>(p, grid, s) : launch_kind<kDW>(p, grid, s);
 }
 
 }  // namespace mosa

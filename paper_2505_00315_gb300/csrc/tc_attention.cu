@@ -682,28 +682,43 @@ __global__ void __launch_bounds__(kBT, 1) attn_bwd_tc_kernel(const __grid_consta
 }
 
 // dQ from its fp32 accumulator into columns 0..63 of the dQ|dK|dV|dlogit rows,
-// two columns per thread: as a bf16 pair ([hi 256 | lo 256] rows), or (f16)
-// as fp16 rows of 256, turned back by RoPE first when asked (gidx, rope).
+// eight columns per thread (two 16-byte loads): as a bf16 pair ([hi 256 | lo
+// 256] rows), or (f16) as fp16 rows of 256 (one 16-byte store), turned back by
+// RoPE first when asked (gidx, rope).
 __global__ void dq_finish_kernel(const float *__restrict__ dQacc, bf16 *__restrict__ dQKV, size_t rows,
                                  int f16, const int32_t *__restrict__ gidx, int rope, int T,
                                  RopeTable tab, uint32_t *status) {
     pdl_trigger();  // the next kernel (zeroing dX) may run beside this one
     pdl_wait();
-    const size_t idx = (size_t)blockIdx.x * blockDim.x + threadIdx.x;   // (row, column pair)
-    if (idx >= rows * 32) return;
-    const size_t row = idx >> 5;
-    const int c = (int)(idx & 31) * 2;
-    float2 v = *reinterpret_cast<const float2 *>(dQacc + row * 64 + c);
+    const size_t idx = (size_t)blockIdx.x * blockDim.x + threadIdx.x;   // (row, 8-column group)
+    if (idx >= rows * 8) return;
+    const size_t row = idx >> 3;
+    const int c = (int)(idx & 7) * 8;
+    const float4 a = *reinterpret_cast<const float4 *>(dQacc + row * 64 + c);
+    const float4 b = *reinterpret_cast<const float4 *>(dQacc + row * 64 + c + 4);
+    float v[8] = {a.x, a.y, a.z, a.w, b.x, b.y, b.z, b.w};
     if (!f16) {
-        uint32_t hi, lo;
-        split_pair2(v.x, v.y, hi, lo);
-        *reinterpret_cast<uint32_t *>(dQKV + row * 512 + c) = hi;
-        *reinterpret_cast<uint32_t *>(dQKV + row * 512 + 256 + c) = lo;
+        uint32_t hi[4], lo[4];
+#pragma unroll
+        for (int e = 0; e < 4; ++e) split_pair2(v[2 * e], v[2 * e + 1], hi[e], lo[e]);
+        *reinterpret_cast<uint4 *>(dQKV + row * 512 + c) = make_uint4(hi[0], hi[1], hi[2], hi[3]);
+        *reinterpret_cast<uint4 *>(dQKV + row * 512 + 256 + c) = make_uint4(lo[0], lo[1], lo[2], lo[3]);
         return;
     }
-    if (rope && c < 32) rope_turn(v.x, v.y, tab.phi[c >> 1], gidx[row] % T, -1.f);
-    *reinterpret_cast<uint32_t *>(reinterpret_cast<__half *>(dQKV) + row * 256 + c) = pack_f16x2(v.x, v.y);
-    if (!(fabsf(v.x) < kF16Overflow) || !(fabsf(v.y) < kF16Overflow)) atomicOr(status, kStatusRange);
+    if (rope && c < 32) {
+        const int t = gidx[row] % T;
+#pragma unroll
+        for (int e = 0; e < 4; ++e) rope_turn(v[2 * e], v[2 * e + 1], tab.phi[(c >> 1) + e], t, -1.f);
+    }
+    uint32_t w[4];
+    float mx = 0.f;
+#pragma unroll
+    for (int e = 0; e < 4; ++e) {
+        mx = fmaxf(mx, fmaxf(fabsf(v[2 * e]), fabsf(v[2 * e + 1])));
+        w[e] = pack_f16x2(v[2 * e], v[2 * e + 1]);
+    }
+    *reinterpret_cast<uint4 *>(reinterpret_cast<__half *>(dQKV) + row * 256 + c) = make_uint4(w[0], w[1], w[2], w[3]);
+    if (!(mx < kF16Overflow)) atomicOr(status, kStatusRange);
 }
 
 // ------------------------------------------------- k <= 128: one CTA per tile
@@ -1094,6 +1109,11 @@ cudaError_t tc_attn_fwd(const Dims &dm, const Saved &sv, cudaStream_t s) {
     return e;
 }
 
+cudaError_t tc_zero_dq(const Dims &dm, const Saved &sv, cudaStream_t s) {
+    if (dm.k <= kSmallK) return cudaSuccess;
+    return cudaMemsetAsync(sv.G, 0, sizeof(float) * (size_t)dm.H * dm.B * dm.k * 64, s);
+}
+
 cudaError_t tc_attn_bwd(const Dims &dm, const Saved &sv, cudaStream_t s) {
     BwdParams kv, dq;
     memset(&kv, 0, sizeof(kv));
@@ -1158,11 +1178,10 @@ cudaError_t tc_attn_bwd(const Dims &dm, const Saved &sv, cudaStream_t s) {
     const size_t rows = (size_t)dm.H * dm.B * dm.k;
     const cudaError_t attr = allow_smem((const void *)attn_bwd_tc_kernel, kBwdLargeSmem);
     if (attr != cudaSuccess) return attr;
-    cudaError_t e = cudaMemsetAsync(sv.G, 0, sizeof(float) * rows * 64, s);
-    if (e != cudaSuccess) return e;
+    // (the dQ accumulator sv.G has been zeroed by the caller: tc_zero_dq)
     dim3 grid(dm.B, dm.H, (dm.k + 127) / 128);   // key tiles slowest (see the kernel)
-    e = launch_pdl(attn_bwd_tc_kernel, grid, dim3(kBT), kBwdLargeSmem, s, bp);
-    const size_t n = rows * 32;
+    cudaError_t e = launch_pdl(attn_bwd_tc_kernel, grid, dim3(kBT), kBwdLargeSmem, s, bp);
+    const size_t n = rows * 8;
     if (e == cudaSuccess)
         e = launch_pdl(dq_finish_kernel, dim3((unsigned)((n + 255) / 256)), dim3(256), 0, s,
                        (const float *)sv.G, static_cast<bf16 *>(sv.dQKV), rows, 1,

@@ -61,21 +61,25 @@ struct AttnParams {
 // TMEM lane quadrant (warp w: query rows 32 (w % 4) .. +31, keys
 // 64 ((w - 4) / 4) .. +63 of each 128-key block).  Q, K, V and P are fp16
 // (one MMA per 16-wide K step).  For key block j:
-//   S_j = Q K_j^T into TMEM buffer j % 2, issued two blocks ahead, so the
-//   MMAs of S_{j+2} and O += P_j V_j run while the softmax of block j+1 runs;
+//   S_j = Q K_j^T into TMEM buffer j % 2;
 //   P_j = exp2(S_j scale - m) with m the row's running maximum, updated only
 //   when the block's maximum exceeds it by more than 2^8 (O and l are then
 //   rescaled in place; otherwise P may reach 2^8, well inside the fp16 range,
-//   and the final O / l uses the same m throughout); O accumulates in TMEM.
-//   P_j is written by the softmax warps as fp16 into the first 64 TMEM
-//   columns of S_j itself (two per column) and O += P_j V_j reads it from
-//   there as the A operand.  Measured on this GPU: a tcgen05.st issued while
-//   an MMA that reads its A operand from TMEM is still running corrupts that
-//   MMA's result even when the columns differ, so P_j is stored only after
-//   P_{j-1} V_{j-1} has completed (its exponentials are computed meanwhile),
-//   and S_{j+2} (which overwrites P_j's columns) only after P_j V_j.
+//   and the final O / l uses the same m throughout), written as fp16 into
+//   shared-memory tile j % 2;
+//   O += P_j V_j with both operands in shared memory, O in TMEM.
+// The MMA issuer issues S_{j+2} as soon as the softmax warps have read S_j
+// into registers and P_j V_j as soon as P_j is stored, and the softmax warps
+// wait for the tensor pipe only to reuse a P tile (P_{j-2} V_{j-2} done) or
+// to rescale O, so the softmax of one block runs while the MMAs of the
+// neighbouring blocks do.  (P was first kept in the TMEM columns of S_j and
+// read from there by the MMA; a tcgen05.st issued while such an MMA is still
+// reading TMEM corrupts it, so every P store waited for the previous block's
+// P V and the block time was the MMAs plus that hand-over.)  Each hand-over
+// barrier comes in a pair, one per buffer parity, so no waiter can see its
+// barrier complete twice ahead of it.
 // K and V blocks stream through an 8-slot ring in the order the MMAs use
-// them: K0, K1, V0, K2, V1, K3, ... (see kv_item).
+// them: K0, K1, K2, V0, K3, V1, ... (see kv_item).
 constexpr int kLT = 384;              // threads
 constexpr int kLWorkers = 256;
 constexpr int kLKeys = 128;           // keys per block
@@ -85,20 +89,30 @@ constexpr float kRescaleLog2 = 8.f;   // lazy-rescale threshold (log2 units)
 struct FwdLargeSmem {
     uint8_t q[kTileHalf];                     // Q, fp16 [128 x 64]
     uint8_t kv[kLSlots][kTileHalf];           // K or V blocks, fp16 [128 x 64]
+    uint8_t p[2][2][kTileHalf];               // P tiles [block parity][64-key block], fp16
     float part[2][2][128];                    // [block parity][key half]: block max, final sums
-    uint64_t q_full, kv_full[kLSlots], kv_empty[kLSlots], s_full[2], p_ready, pv_done;
+    uint64_t q_full, kv_full[kLSlots], kv_empty[kLSlots];
+    uint64_t s_full[2], s_free[2], p_ready[2], pv_done[2];   // per buffer parity
     uint32_t tmem;
     int abort;
 };
 constexpr int kFwdLargeSmem = (int)sizeof(FwdLargeSmem) + 1024;
 static_assert(kFwdLargeSmem <= 227 * 1024, "shared memory");
 
-// Item t of the K/V stream for n blocks: (is V, block).
+// Item t of the K/V stream for n blocks, in MMA issue order: K_0, K_1, then
+// K_{j+2} followed by V_j while j + 2 < n, then the remaining V_j.
+// Returns (is V, block).
 __device__ __forceinline__ void kv_item(int t, int n, bool &is_v, int &blk) {
-    if (t == 0) { is_v = false; blk = 0; return; }
-    if (n == 1) { is_v = true; blk = 0; return; }
-    if (t == 2 * n - 1) { is_v = true; blk = n - 1; return; }
-    if (t & 1) { is_v = false; blk = (t + 1) >> 1; } else { is_v = true; blk = (t >> 1) - 1; }
+    const int s0 = n < 2 ? n : 2;
+    if (t < s0) { is_v = false; blk = t; return; }
+    const int u = t - s0, pairs = n > 2 ? n - 2 : 0;
+    if (u < 2 * pairs) {
+        is_v = (u & 1) == 1;
+        blk = is_v ? (u >> 1) : (u >> 1) + 2;
+        return;
+    }
+    is_v = true;
+    blk = pairs + (u - 2 * pairs);
 }
 
 __device__ __forceinline__ bool lwait(FwdLargeSmem &sm, uint64_t &bar, uint32_t parity, uint32_t *status) {
@@ -128,10 +142,12 @@ __global__ void __launch_bounds__(kLT, 1) attn_fwd_tc_kernel(const __grid_consta
             mbar_init(smem_u32(&sm.kv_full[s]), 1);
             mbar_init(smem_u32(&sm.kv_empty[s]), 1);
         }
-        mbar_init(smem_u32(&sm.s_full[0]), 1);
-        mbar_init(smem_u32(&sm.s_full[1]), 1);
-        mbar_init(smem_u32(&sm.p_ready), kLWorkers);
-        mbar_init(smem_u32(&sm.pv_done), 1);
+        for (int u = 0; u < 2; ++u) {
+            mbar_init(smem_u32(&sm.s_full[u]), 1);
+            mbar_init(smem_u32(&sm.s_free[u]), kLWorkers);
+            mbar_init(smem_u32(&sm.p_ready[u]), kLWorkers);
+            mbar_init(smem_u32(&sm.pv_done[u]), 1);
+        }
         sm.abort = 0;
         fence_barrier_init();
     }
@@ -185,32 +201,28 @@ __global__ void __launch_bounds__(kLT, 1) attn_fwd_tc_kernel(const __grid_consta
             issue_s(0);
             if (n > 1) issue_s(1);
             for (int j = 0; j < n && ok; ++j) {
-                ok = lwait(sm, sm.p_ready, j & 1, p.status);
-                const int s = take();   // V_j
-                if (!ok) break;
-                tc_fence_after();
-                // O += P_j V_j: P (A operand) from the first 64 TMEM columns of
-                // S_j, 8 columns per 16 keys; V MN-major
-                const uint32_t pa = tmem + 128 * (j & 1);
-                const uint32_t vb = smem_u32(sm.kv[s]);
-#pragma unroll
-                for (int kk = 0; kk < 8; ++kk)
-                    mma_bf16_ts(tO, pa + 8 * kk, smem_desc_sw128(vb + kk * 2048, kTileHalf, 1024), idO,
-                                (j > 0 || kk > 0) ? 1u : 0u);
-                mma_commit(smem_u32(&sm.pv_done));
-                mma_commit(smem_u32(&sm.kv_empty[s]));
+                const int u = j & 1;
                 if (j + 2 < n) {
-                    // S_{j+2} overwrites the columns P_j V_j reads
-                    ok = ok && lwait(sm, sm.pv_done, j & 1, p.status);
+                    // S_{j+2} reuses buffer j % 2 once the workers hold S_j
+                    ok = lwait(sm, sm.s_free[u], (j >> 1) & 1, p.status);
                     tc_fence_after();
                     issue_s(j + 2);
                 }
+                ok = ok && lwait(sm, sm.p_ready[u], (j >> 1) & 1, p.status);
+                const int s = take();   // V_j
+                if (!ok) break;
+                tc_fence_after();
+                // O += P_j V_j: P tile j % 2 (K-major, keys along K), V MN-major
+                mma_k128_f16(tO, smem_u32(sm.p[u][0]), smem_u32(sm.kv[s]), false, idO, j > 0);
+                mma_commit(smem_u32(&sm.pv_done[u]));
+                mma_commit(smem_u32(&sm.kv_empty[s]));
             }
             if (!ok) {
-                // release the softmax warps
-                mma_commit(smem_u32(&sm.s_full[0]));
-                mma_commit(smem_u32(&sm.s_full[1]));
-                mma_commit(smem_u32(&sm.pv_done));
+                // release the softmax warps (their later waits see the abort flag)
+                for (int u = 0; u < 2; ++u) {
+                    mma_commit(smem_u32(&sm.s_full[u]));
+                    mma_commit(smem_u32(&sm.pv_done[u]));
+                }
             }
         }
     } else if (warp >= 4) {
@@ -222,10 +234,13 @@ __global__ void __launch_bounds__(kLT, 1) attn_fwd_tc_kernel(const __grid_consta
         float m = -INFINITY, l = 0.f;              // running max (log2 units), partial sum
         bool ok = true;
         for (int j = 0; j < n; ++j) {
-            ok = lwait(sm, sm.s_full[j & 1], (j >> 1) & 1, p.status) && ok;
+            const int u = j & 1;
+            ok = lwait(sm, sm.s_full[u], (j >> 1) & 1, p.status) && ok;
             tc_fence_after();
             float s[64];
-            tmem_ld64(tmem + 128 * (j & 1) + lane_off + 64 * ch, s);
+            tmem_ld64(tmem + 128 * u + lane_off + 64 * ch, s);
+            tc_fence_before();
+            mbar_arrive(smem_u32(&sm.s_free[u]));   // S_{j+2} may overwrite these columns
             if (j == qt) {
                 // diagonal block (earlier blocks are wholly visible): key
                 // j*128 + 64 ch + c is visible from query i iff c <= lim
@@ -243,45 +258,42 @@ __global__ void __launch_bounds__(kLT, 1) attn_fwd_tc_kernel(const __grid_consta
             // written here was last read before both warps of the row passed
             // the previous block's barrier, so one barrier per block suffices;
             // only the two warps sharing the lane quadrant q synchronise
-            sm.part[j & 1][ch][r] = mb;
+            sm.part[u][ch][r] = mb;
             named_barrier(1 + q, 64);
-            mb = fmaxf(sm.part[j & 1][0][r], sm.part[j & 1][1][r]);
+            mb = fmaxf(sm.part[u][0][r], sm.part[u][1][r]);
             const bool grow = mb > m + kRescaleLog2;   // same decision in both threads of the row
             const float m_new = grow ? mb : m;
             const float corr = grow ? exp2_fast(m - m_new) : 1.f;   // 0 on the first block
             float sm4[4] = {0.f, 0.f, 0.f, 0.f};
-            uint32_t pw[32];
 #pragma unroll
-            for (int c = 0; c < 32; ++c) {
-                const float e0 = exp2_fast(fmaf(s[2 * c], p.scale_log2, -m_new));
-                const float e1 = exp2_fast(fmaf(s[2 * c + 1], p.scale_log2, -m_new));
-                sm4[(2 * c) & 3] += e0;
-                sm4[(2 * c + 1) & 3] += e1;
-                pw[c] = pack_f16x2(e0, e1);
+            for (int c = 0; c < 64; ++c) {
+                s[c] = exp2_fast(fmaf(s[c], p.scale_log2, -m_new));
+                sm4[c & 3] += s[c];
             }
             l = l * corr + ((sm4[0] + sm4[1]) + (sm4[2] + sm4[3]));
             m = m_new;
-            // P_{j-1} V_{j-1} must be complete before any TMEM store (see above);
-            // then O may also be rescaled (P_j V_j waits for this block's P)
-            if (j > 0) {
-                ok = lwait(sm, sm.pv_done, (j - 1) & 1, p.status) && ok;
-                tc_fence_after();
-            }
             if (j > 0 && __any_sync(0xffffffffu, grow)) {
+                // O holds P_0 V_0 .. P_{j-1} V_{j-1}: all of them done first
+                ok = lwait(sm, sm.pv_done[u ^ 1], ((j - 1) >> 1) & 1, p.status) && ok;
+                tc_fence_after();
                 float o[32];
                 tmem_ld32(tO + lane_off + 32 * ch, o);
 #pragma unroll
                 for (int c = 0; c < 32; ++c) o[c] *= corr;
                 tmem_st32(tO + lane_off + 32 * ch, o);
             }
-            // P_j as fp16 into the columns of S_j: this thread's 64 keys are
-            // columns 32 ch .. +31 (both threads of the row have read their S
-            // values: exchange barrier)
-            tmem_st32u(tmem + 128 * (j & 1) + lane_off + 32 * ch, pw);
+            // P tile j % 2 was last read by P_{j-2} V_{j-2}
+            if (j >= 2) {
+                ok = lwait(sm, sm.pv_done[u], ((j >> 1) - 1) & 1, p.status) && ok;
+                tc_fence_after();
+            }
+            put_f16_32(sm.p[u][ch], r, 0, s, 1.f);
+            put_f16_32(sm.p[u][ch], r, 32, s + 32, 1.f);
+            fence_proxy_async();
             tc_fence_before();
-            mbar_arrive(smem_u32(&sm.p_ready));
+            mbar_arrive(smem_u32(&sm.p_ready[u]));
         }
-        ok = lwait(sm, sm.pv_done, (n - 1) & 1, p.status) && ok;
+        ok = lwait(sm, sm.pv_done[(n - 1) & 1], ((n - 1) >> 1) & 1, p.status) && ok;
         tc_fence_after();
         sm.part[n & 1][ch][r] = l;
         named_barrier(1 + q, 64);

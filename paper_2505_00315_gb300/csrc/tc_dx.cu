@@ -172,7 +172,9 @@ __global__ void __launch_bounds__(kThreads, 1) scatter_product_kernel(const __gr
                     if (!(ok = dwait(sm, sm.w_full[s], (idx / kSlots) & 1, p.status))) break;
                     tc_fence_after();
                     const uint32_t wb = smem_u32(sm.w[s]);
-                    for (int half = 0; half < halves; ++half)
+                    // (straight-line issue: a loop with a run-time trip count around
+                    // tcgen05.mma was measured to halve the issue rate)
+                    auto issue = [&](int half) {
 #pragma unroll
                         for (int kk = 0; kk < 4; ++kk)
                             mma_bf16(tmem + 256 * buf,
@@ -180,6 +182,9 @@ __global__ void __launch_bounds__(kThreads, 1) scatter_product_kernel(const __gr
                                      kOut ? smem_desc_sw128(wb + kk * 2048, 8192, 1024)
                                           : smem_desc_sw128(wb + kk * 32, 16, 1024),
                                      idX, (j > 0 || half > 0 || kk > 0) ? 1u : 0u);
+                    };
+                    issue(0);
+                    if (halves > 1) issue(1);
                     mma_commit(smem_u32(&sm.w_empty[s]));
                     if (last) mma_commit(smem_u32(&sm.a_empty[j]));
                 }

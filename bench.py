@@ -507,6 +507,7 @@ def main():
     torch.cuda.synchronize()
     launches0 = mosa.mosa_kernel_launches()
     dom = [0.0, 0, 0]   # ms, launches, steps
+    span = [0.0, 0]     # kernel-span ms, steps
     t_host0 = time.time()
     for i in range(K):
         timed = i % PROFILE_EVERY == 0
@@ -521,6 +522,11 @@ def main():
             dom[0] += ms
             dom[1] += n
             dom[2] += 1
+            if not hybrid:
+                sp = mosa.mosa_profile_spans(shape, ws).get(dominant, -1.0)
+                if sp >= 0:
+                    span[0] += sp
+                    span[1] += 1
     torch.cuda.synchronize()
     t_host1 = time.time()
     barrier()
@@ -645,6 +651,10 @@ def main():
         achieved = work[dominant]["bytes"] / (dom_ms / 1e3) / 1e9
     else:
         achieved = work[dominant]["flops"] / (dom_ms / 1e3) / 1e12
+    key = "flops" if unit != "GB/s" else "bytes"
+    scale = 1e12 if unit != "GB/s" else 1e9
+    span_ms = span[0] / span[1] if span[1] else None
+    span_achieved = work[dominant][key] / (span_ms / 1e3) / scale if span_ms else None
     layer_flops = work["forward_flops"] + (work["backward_flops"] if cfg.backward else 0)
     full = flops.hybrid_work(cfg.B, cfg.T, cfg.d, cfg.H, cfg.hp, cfg.k, args.dense_heads,
                              args.window, causal=False)
@@ -660,6 +670,11 @@ def main():
                      "algorithmic": work[dominant]["flops" if unit != "GB/s" else "bytes"],
                      "stage_ms_per_step": dom_ms, "launches_per_step": dom[1] / max(dom[2], 1),
                      "timed_steps": dom[2],
+                     "kernel_span_ms_per_step": span_ms,
+                     "kernel_span_achieved": span_achieved,
+                     "kernel_span_frac": span_achieved / peak if span_achieved else None,
+                     "kernel_span_what": "first CTA start to last CTA end of the stage's "
+                                         "kernels (%globaltimer), same timed steps",
                      "timed_every_nth_step": PROFILE_EVERY},
         "layer_tflops": layer_flops * world * K / (total_ms / 1e3) / 1e12,
         "layer_tflops_counting": "causal attention counted as 2h'k(k+1) forward, "

@@ -274,6 +274,16 @@ mosa_status mosa_profile_stages(uint32_t stage_mask);
  * stages the library has. */
 int32_t mosa_profile_read(double *total_ms, int32_t *count, int32_t max_stages);
 
+/* Device time of the stages timed by the last layer call with this
+ * workspace: for each stage (ms[0 .. max_stages-1]), the span in
+ * milliseconds from the first CTA start to the last CTA end of its
+ * tensor-core and selection kernels (%globaltimer stamps written into the
+ * workspace while the stage's timing is on), or -1 if it recorded none.
+ * Unlike the event timing above, this excludes the time a stage's kernels
+ * wait for a launch or for SMs before they start.  Waits for the device.
+ * Returns the number of entries written. */
+int32_t mosa_profile_spans(const mosa_shape *shape, void *workspace, double *ms, int32_t max_stages);
+
 /* Name of a stage ("router", "select", ...; "unknown" if out of range). */
 const char *mosa_stage_name(int32_t stage);
 

@@ -28,7 +28,8 @@ EXPORTED = ("mosa_status_string", "mosa_workspace_bytes", "mosa_forward",
             "mosa_forward_with_indices", "mosa_backward", "mosa_topk", "mosa_check_status",
             "mosa_kernel_launches", "mosa_profile_stages", "mosa_profile_read",
             "mosa_stage_name", "mosa_stage_engine", "mosa_route_noalloc", "mosa_adaptive_k",
-            "mosa_hybrid_workspace_bytes", "mosa_hybrid_forward", "mosa_hybrid_backward")
+            "mosa_hybrid_workspace_bytes", "mosa_hybrid_forward", "mosa_hybrid_backward",
+            "mosa_profile_spans")
 
 
 class MosaShape(ctypes.Structure):
@@ -99,6 +100,8 @@ def load(build_if_missing: bool = True) -> ctypes.CDLL:
         L.mosa_profile_read.argtypes = [ctypes.POINTER(ctypes.c_double),
                                         ctypes.POINTER(ctypes.c_int32), i32]
         L.mosa_profile_read.restype = i32
+        L.mosa_profile_spans.argtypes = [sp, vp, ctypes.POINTER(ctypes.c_double), i32]
+        L.mosa_profile_spans.restype = i32
         L.mosa_stage_name.argtypes = [i32]
         L.mosa_stage_name.restype = ctypes.c_char_p
         L.mosa_route_noalloc.argtypes = [sp, vp, vp, vp, vp, vp]
@@ -356,6 +359,18 @@ def mosa_profile_read() -> dict:
     cnt = (ctypes.c_int32 * n)()
     m = L.mosa_profile_read(ms, cnt, n)
     return {mosa_stage_name(i): (ms[i], cnt[i]) for i in range(min(m, n))}
+
+
+def mosa_profile_spans(shape: MosaShape, workspace) -> dict:
+    """{stage name: ms} from the first CTA start to the last CTA end of each
+    stage's kernels in the last layer call with ``workspace`` (only stages
+    timed with mosa_profile_stages; -1 where none recorded).  Waits for the
+    device."""
+    L = load()
+    n = 16
+    ms = (ctypes.c_double * n)()
+    m = L.mosa_profile_spans(ctypes.byref(shape), ctypes.c_void_p(workspace.data_ptr()), ms, n)
+    return {mosa_stage_name(i): ms[i] for i in range(min(m, n))}
 
 
 _ENGINES = {0: "simt", 1: "tensor", 2: "mem"}

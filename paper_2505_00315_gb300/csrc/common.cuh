@@ -99,6 +99,7 @@ struct Saved {
     // through fp16 copies so that every product with dQKV is one MMA
     void *X16;          // [B*T,d] fp16 copy of X
     void *W16;          // [3][H,d,hp] fp16 copies of W_q, W_k, W_v
+    unsigned long long *spans;   // [16][2] kernel spans of the timed stages (measurement)
 };
 
 // Rotary position encoding (Sec. 2.2): pair p of the first h'/2 dimensions of
@@ -127,6 +128,22 @@ __device__ __forceinline__ void rope_turn(float &x0, float &x1, uint64_t phi, in
     const float y0 = x0 * cs - x1 * sn, y1 = x0 * sn + x1 * cs;
     x0 = y0;
     x1 = y1;
+}
+
+// Kernel spans (measurement only): a stage's kernels record the earliest
+// start and the latest end of their CTAs (%globaltimer, ns) into a slot
+// [start, end] of the workspace, when that stage is being timed (sp != null).
+__device__ __forceinline__ unsigned long long span_clock() {
+    unsigned long long t;
+    asm volatile("mov.u64 %0, %%globaltimer;" : "=l"(t));
+    return t;
+}
+__device__ __forceinline__ void span_begin(unsigned long long *sp) {
+    if (sp != nullptr && threadIdx.x == 0) atomicMin(sp, span_clock());
+}
+// Call after the CTA's last barrier (all its work done).
+__device__ __forceinline__ void span_end(unsigned long long *sp) {
+    if (sp != nullptr && threadIdx.x == 0) atomicMax(sp + 1, span_clock());
 }
 
 struct Dims {

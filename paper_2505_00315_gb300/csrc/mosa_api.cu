@@ -68,6 +68,7 @@ size_t carve(const Dims &dm, char *base, Saved *sv) {
     s.dQKV = take(e * R * 4 * dm.hp);  // 3 h' columns, or 4 blocks of 64 on the tensor cores
     s.G = (float *)take(sizeof(float) * R * dm.hp);
     s.WrT = (float *)take(sizeof(float) * (size_t)dm.d * dm.H);
+    s.spans = (unsigned long long *)take(sizeof(unsigned long long) * 2 * 16);
     // the fp16 attention path's copies (reserved whenever that path can run,
     // so the size does not depend on the environment's kernel-path switches)
     if (dm.bf16 && dm.hp == 64 && dm.k > 128) {
@@ -175,6 +176,7 @@ mosa_status forward_tc(const Dims &dm, const void *X, const void *W_r, const voi
                        const void *W_k, const void *W_v, const void *W_o, float *Y, int32_t *I,
                        float *r_sel, float *rf, bool route, const int32_t *I_in,
                        const float *rsel_in, const Saved &sv, cudaStream_t s, DevResources &r) {
+    set_span_base(sv.spans);   // measurement: this call's kernel-span slots
     // A call that adds into Y continues the status word of the call that wrote it.
     if (!dm.accumulate) MOSA_TRY(cudaMemsetAsync(sv.status, 0, sizeof(uint32_t), s));
     const size_t ny = (size_t)dm.B * dm.T * dm.d;
@@ -227,6 +229,7 @@ mosa_status backward_tc(const Dims &dm, const void *X, const void *W_r, const vo
                         const void *W_k, const void *W_v, const void *W_o, const void *dY,
                         float *dX, float *dW_r, float *dW_q, float *dW_k, float *dW_v,
                         float *dW_o, const Saved &sv, cudaStream_t s, DevResources &r) {
+    set_span_base(sv.spans);   // measurement: this call's kernel-span slots
     cudaStream_t t = r.side;
     const size_t nx = (size_t)dm.B * dm.T * dm.d;
     MOSA_TRY(link(s, t, r.ev[0]));
@@ -301,6 +304,7 @@ mosa_status forward_routed(const Dims &dm, const void *X, const void *W_r, const
                            const void *W_k, const void *W_v, const void *W_o, float *Y,
                            int32_t *I, float *r_sel, float *rf, const Saved &sv, cudaStream_t s,
                            DevResources *res) {
+    set_span_base(sv.spans);   // measurement: this call's kernel-span slots
     if (res != nullptr)
         return forward_tc(dm, X, W_r, W_q, W_k, W_v, W_o, Y, I, r_sel, rf, true, nullptr, nullptr,
                           sv, s, *res);
@@ -323,6 +327,7 @@ mosa_status forward_given(const Dims &dm, const void *X, const void *W_q, const 
                           const void *W_v, const void *W_o, const int32_t *I,
                           const float *r_sel, float *Y, const Saved &sv, cudaStream_t s,
                           DevResources *res) {
+    set_span_base(sv.spans);   // measurement: this call's kernel-span slots
     if (res != nullptr)
         return forward_tc(dm, X, nullptr, W_q, W_k, W_v, W_o, Y, nullptr, nullptr, nullptr, false,
                           I, r_sel, sv, s, *res);
@@ -342,6 +347,7 @@ mosa_status backward_all(const Dims &dm, const void *X, const void *W_r, const v
                          const void *W_k, const void *W_v, const void *W_o, const void *dY,
                          float *dX, float *dW_r, float *dW_q, float *dW_k, float *dW_v,
                          float *dW_o, const Saved &sv, cudaStream_t s, DevResources *res) {
+    set_span_base(sv.spans);   // measurement: this call's kernel-span slots
     if (res != nullptr)
         return backward_tc(dm, X, W_r, W_q, W_k, W_v, W_o, dY, dX, dW_r, dW_q, dW_k, dW_v, dW_o,
                            sv, s, *res);
@@ -747,6 +753,23 @@ int32_t mosa_stage_engine(const mosa_shape *shape, int32_t stage) {
         case kStageBwdUnit: return use_fused_backward(dm) ? 1 : 0;
         default: return 0;
     }
+}
+
+int32_t mosa_profile_spans(const mosa_shape *shape, void *workspace, double *ms, int32_t max_stages) {
+    Dims dm;
+    if (check_shape(shape, &dm) != MOSA_OK || workspace == nullptr || ms == nullptr) return 0;
+    Saved sv;
+    carve(dm, (char *)workspace, &sv);
+    unsigned long long h[2 * 16];
+    if (cudaDeviceSynchronize() != cudaSuccess ||
+        cudaMemcpy(h, sv.spans, sizeof(h), cudaMemcpyDeviceToHost) != cudaSuccess)
+        return 0;
+    const int n = max_stages < kNumStages ? max_stages : kNumStages;
+    for (int i = 0; i < n; ++i) {
+        const unsigned long long a = h[2 * i], b = h[2 * i + 1];
+        ms[i] = (a != ~0ull && b != 0ull && b >= a) ? (double)(b - a) * 1e-6 : -1.0;
+    }
+    return n;
 }
 
 mosa_status mosa_check_status(const mosa_shape *shape, void *workspace, void *stream) {

@@ -21,6 +21,9 @@ struct Pending {
     bool recycle;  // false for events owned by a captured graph
 };
 thread_local CaptureRecord *t_capture = nullptr;
+static_assert(kNumStages <= 16, "kernel-span slots in the workspace");
+thread_local unsigned long long *t_span_base = nullptr;
+thread_local unsigned long long *t_active_span = nullptr;
 std::vector<Pending> g_pending;
 std::vector<cudaEvent_t> g_free;
 double g_ms[kNumStages] = {};
@@ -62,8 +65,19 @@ void replayed(const CaptureRecord &rec) {
     for (const CaptureRecord::Pair &q : rec.pairs) g_pending.push_back({q.stage, q.start, q.stop, false});
 }
 
+void set_span_base(unsigned long long *base) { t_span_base = base; }
+unsigned long long *active_span() { return t_active_span; }
+
 StageScope::StageScope(int stage, cudaStream_t s) : stage_(stage), stream_(s) {
+    prev_span_ = t_active_span;
     if (!(g_mask.load(std::memory_order_relaxed) & (1u << stage))) return;
+    if (t_span_base != nullptr) {
+        // reset this stage's span slot (start = max, end = 0) ahead of its kernels
+        unsigned long long *slot = t_span_base + 2 * stage;
+        if (cudaMemsetAsync(slot, 0xFF, sizeof(unsigned long long), s) == cudaSuccess &&
+            cudaMemsetAsync(slot + 1, 0, sizeof(unsigned long long), s) == cudaSuccess)
+            t_active_span = slot;
+    }
     if (t_capture != nullptr) {
         // recorded into the graph: these events live as long as the graph
         // External records become event nodes of the graph (a plain record
@@ -82,6 +96,7 @@ StageScope::StageScope(int stage, cudaStream_t s) : stage_(stage), stream_(s) {
 }
 
 StageScope::~StageScope() {
+    t_active_span = prev_span_;
     if (!active_) return;
     if (t_capture != nullptr) {
         if (cudaEventRecordWithFlags(stop_, stream_, cudaEventRecordExternal) == cudaSuccess)

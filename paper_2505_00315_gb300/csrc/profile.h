@@ -36,6 +36,12 @@ void replayed(const CaptureRecord &rec);
 // Stage-timing mask currently in force.
 uint32_t profile_mask();
 
+// Kernel spans: the layer call names its workspace's span slots ([stage][2]);
+// while a timed stage is open, active_span() is its slot (else nullptr) and
+// the launchers pass it to their kernels.
+void set_span_base(unsigned long long *base);
+unsigned long long *active_span();
+
 // Records a CUDA event pair around one stage when that stage's timing is on.
 class StageScope {
   public:
@@ -49,6 +55,7 @@ class StageScope {
     cudaStream_t stream_;
     cudaEvent_t start_ = nullptr, stop_ = nullptr;
     bool active_ = false;
+    unsigned long long *prev_span_ = nullptr;
 };
 
 }  // namespace mosa

@@ -87,7 +87,7 @@ __device__ __forceinline__ unsigned long long block_excl_scan(unsigned long long
 __global__ void __launch_bounds__(kSelThreads)
 topk_select_kernel(const float *__restrict__ scores, int T, int k, int32_t *__restrict__ I,
                    float *__restrict__ rsel, int B, int H, int32_t *__restrict__ gidx,
-                   float *__restrict__ rsel_hm, int first_token) {
+                   float *__restrict__ rsel_hm, int first_token, unsigned long long *span) {
     extern __shared__ uint32_t keys_s[];   // the row's order keys when T <= kSelStagedMax
     __shared__ uint32_t hist[2][256];
     __shared__ unsigned long long sh[33];
@@ -95,6 +95,7 @@ topk_select_kernel(const float *__restrict__ scores, int T, int k, int32_t *__re
     // the next kernel may launch and run its prologue as this grid's CTAs finish
     asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
     asm volatile("griddepcontrol.wait;" ::: "memory");  // scores from the router kernel
+    span_begin(span);
     const int row = blockIdx.x;
     const float *s = scores + (size_t)row * T;
     const int tid = threadIdx.x;
@@ -191,6 +192,10 @@ topk_select_kernel(const float *__restrict__ scores, int T, int k, int32_t *__re
             ++pos;
         }
     }
+    if (span != nullptr) {
+        __syncthreads();
+        span_end(span);
+    }
 }
 
 __global__ void indices_to_rows_kernel(const int32_t *__restrict__ I,
@@ -263,7 +268,8 @@ cudaError_t launch_select(int rows, int T, int k, const float *scores, int32_t *
     int threads = T / 4 < 256 ? 256 : (T / 4 > 1024 ? 1024 : (T / 4 + 31) / 32 * 32);
     if (rows >= 512 && threads > 512) threads = 512;
     cudaError_t e = launch_pdl(topk_select_kernel, dim3(rows), dim3(threads), smem, stream,
-                               scores, T, k, I, rsel, B, H, gidx, rsel_hm, first_token ? 1 : 0);
+                               scores, T, k, I, rsel, B, H, gidx, rsel_hm, first_token ? 1 : 0,
+                               active_span());
     note_launches(1);
     return e;
 }

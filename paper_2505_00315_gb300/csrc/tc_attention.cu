@@ -53,6 +53,7 @@ struct AttnParams {
     bf16 *AR;                 // [H, B*k, 128] pair
     float *lse;               // [H, B*k]
     uint32_t *status;
+    unsigned long long *span; // measurement: kernel span slot, or null
 };
 
 
@@ -159,6 +160,7 @@ __global__ void __launch_bounds__(kLT, 1) attn_fwd_tc_kernel(const __grid_consta
     __syncthreads();
     tc_fence_after();
     pdl_wait();  // Q, K, V written by the previous kernels
+    span_begin(p.span);
     const uint32_t tmem = sm.tmem;
     const uint32_t tO = tmem + 256;              // S buffers at 0 and 128
 
@@ -321,6 +323,7 @@ __global__ void __launch_bounds__(kLT, 1) attn_fwd_tc_kernel(const __grid_consta
     }
     tc_fence_before();
     __syncthreads();
+    span_end(p.span);
     if (warp == 2) {
         tc_fence_after();
         tmem_dealloc(tmem, 512);
@@ -347,6 +350,7 @@ struct BwdParams {
     const int32_t *gidx;              // [H, B*k]: b*T + t
     int rope, T;
     RopeTable rope_tab;
+    unsigned long long *span; // measurement: kernel span slot, or null
 };
 
 template <class SM>
@@ -458,6 +462,7 @@ __global__ void __launch_bounds__(kBT, 1) attn_bwd_tc_kernel(const __grid_consta
     __syncthreads();
     tc_fence_after();
     pdl_wait();  // Q, K, V, dA, lse, D written by the previous kernels
+    span_begin(p.span);
     const uint32_t tmem = sm.tmem;
     // S, dP, dV, dK, and the two dQ buffers: all 512 columns
     const uint32_t tS = tmem, tDP = tmem + 128, tDV = tmem + 256, tDK = tmem + 320, tDQ = tmem + 384;
@@ -687,6 +692,7 @@ __global__ void __launch_bounds__(kBT, 1) attn_bwd_tc_kernel(const __grid_consta
     }
     tc_fence_before();
     __syncthreads();
+    span_end(p.span);
     if (warp == 2) {
         tc_fence_after();
         tmem_dealloc(tmem, 512);
@@ -699,9 +705,10 @@ __global__ void __launch_bounds__(kBT, 1) attn_bwd_tc_kernel(const __grid_consta
 // RoPE first when asked (gidx, rope).
 __global__ void dq_finish_kernel(const float *__restrict__ dQacc, bf16 *__restrict__ dQKV, size_t rows,
                                  int f16, const int32_t *__restrict__ gidx, int rope, int T,
-                                 RopeTable tab, uint32_t *status) {
+                                 RopeTable tab, uint32_t *status, unsigned long long *span) {
     pdl_trigger();  // the next kernel (zeroing dX) may run beside this one
     pdl_wait();
+    span_begin(span);
     const size_t idx = (size_t)blockIdx.x * blockDim.x + threadIdx.x;   // (row, 8-column group)
     if (idx >= rows * 8) return;
     const size_t row = idx >> 3;
@@ -731,6 +738,7 @@ __global__ void dq_finish_kernel(const float *__restrict__ dQacc, bf16 *__restri
     }
     *reinterpret_cast<uint4 *>(reinterpret_cast<__half *>(dQKV) + row * 256 + c) = make_uint4(w[0], w[1], w[2], w[3]);
     if (!(mx < kF16Overflow)) atomicOr(status, kStatusRange);
+    span_end(span);   // (thread 0 of each block, after its own row group)
 }
 
 // ------------------------------------------------- k <= 128: one CTA per tile
@@ -799,6 +807,7 @@ __global__ void __launch_bounds__(kSmallThreads, 1) attn_fwd_small_kernel(const 
     __syncthreads();
     tc_fence_after();
     pdl_wait();  // Q, K, V, dA, lse written by the previous kernels
+    span_begin(p.span);
     const uint32_t tmem = sm.tmem, tS = tmem, tO = tmem + 128;
 
     if (warp == 0) {
@@ -909,6 +918,7 @@ __global__ void __launch_bounds__(kSmallThreads, 1) attn_fwd_small_kernel(const 
     }
     tc_fence_before();
     __syncthreads();
+    span_end(p.span);
     if (warp == 2) {
         tc_fence_after();
         tmem_dealloc(tmem, 256);
@@ -939,6 +949,7 @@ __global__ void __launch_bounds__(kSmallThreads, 1) attn_bwd_small_kernel(const 
     __syncthreads();
     tc_fence_after();
     pdl_wait();  // Q, K, V, dA, lse written by the previous kernels
+    span_begin(p.span);
     const uint32_t tmem = sm.tmem;
     const uint32_t tS = tmem, tDP = tmem + 128, tDV = tmem + 256, tDK = tmem + 320, tDQ = tmem + 384;
 
@@ -1060,6 +1071,7 @@ __global__ void __launch_bounds__(kSmallThreads, 1) attn_bwd_small_kernel(const 
     }
     tc_fence_before();
     __syncthreads();
+    span_end(p.span);
     if (warp == 2) {
         tc_fence_after();
         tmem_dealloc(tmem, 512);
@@ -1106,6 +1118,7 @@ cudaError_t tc_attn_fwd(const Dims &dm, const Saved &sv, cudaStream_t s) {
     p.AR = static_cast<bf16 *>(sv.AR);
     p.lse = sv.lse;
     p.status = sv.status;
+    p.span = active_span();
     cudaError_t attr = allow_smem((const void *)attn_fwd_tc_kernel, kFwdLargeSmem);
     if (attr == cudaSuccess) attr = allow_smem((const void *)attn_fwd_small_kernel, kSmallFwdSmem);
     if (attr != cudaSuccess) return attr;
@@ -1151,6 +1164,7 @@ cudaError_t tc_attn_bwd(const Dims &dm, const Saved &sv, cudaStream_t s) {
         sp.Dd = sv.Dd;
         sp.dQKV = static_cast<bf16 *>(sv.dQKV);
         sp.status = sv.status;
+        sp.span = active_span();
         const cudaError_t attr_small = allow_smem((const void *)attn_bwd_small_kernel, kSmallBwdSmem);
         if (attr_small != cudaSuccess) return attr_small;
         cudaError_t e = launch_pdl(attn_bwd_small_kernel, dim3(1, (dm.B + sp.U - 1) / sp.U, dm.H),
@@ -1176,6 +1190,7 @@ cudaError_t tc_attn_bwd(const Dims &dm, const Saved &sv, cudaStream_t s) {
     bp.dQKV = static_cast<bf16 *>(sv.dQKV);
     bp.dQacc = sv.G;
     bp.status = sv.status;
+    bp.span = active_span();
     bp.gidx = sv.gidx;
     bp.T = dm.T;
     bp.rope = dm.rope ? 1 : 0;
@@ -1197,7 +1212,7 @@ cudaError_t tc_attn_bwd(const Dims &dm, const Saved &sv, cudaStream_t s) {
     if (e == cudaSuccess)
         e = launch_pdl(dq_finish_kernel, dim3((unsigned)((n + 255) / 256)), dim3(256), 0, s,
                        (const float *)sv.G, static_cast<bf16 *>(sv.dQKV), rows, 1,
-                       (const int32_t *)sv.gidx, bp.rope, dm.T, bp.rope_tab, sv.status);
+                       (const int32_t *)sv.gidx, bp.rope, dm.T, bp.rope_tab, sv.status, bp.span);
     note_launches(2);
     return e;
 }

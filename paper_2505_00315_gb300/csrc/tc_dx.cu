@@ -64,6 +64,7 @@ struct DxParams {
     long long units;      // H * mt * nch
     uint32_t *status;
     int f16;              // dX: A = fp16 dQKV rows [H, B*k, 256], W = fp16 copies (one MMA)
+    unsigned long long *span;   // measurement: kernel span slot, or null
 };
 
 __device__ __forceinline__ bool dwait(DxSmem &sm, uint64_t &bar, uint32_t parity, uint32_t *status) {
@@ -114,6 +115,7 @@ __global__ void __launch_bounds__(kThreads, 1) scatter_product_kernel(const __gr
     tc_fence_after();
     const uint32_t tmem = sm.tmem;
     pdl_wait();  // the A pairs (and dlogit) come from earlier kernels
+    span_begin(p.span);
 
     if (warp == 0) {
         if (lane == 0) {
@@ -254,6 +256,7 @@ __global__ void __launch_bounds__(kThreads, 1) scatter_product_kernel(const __gr
     }
     tc_fence_before();
     __syncthreads();
+    span_end(p.span);
     if (warp == 2) {
         tc_fence_after();
         tmem_dealloc(tmem, 512);
@@ -276,6 +279,7 @@ cudaError_t launch_scatter_product(DxParams &p, const Dims &dm, cudaStream_t s) 
     p.mt = (Mtok + 127) / 128;
     p.nch = (dm.d + kChunk - 1) / kChunk;
     p.units = (long long)dm.H * p.mt * p.nch;
+    p.span = active_span();
     const cudaError_t attr = allow_smem((const void *)scatter_product_kernel<kOut>, kSmem);
     if (attr != cudaSuccess) return attr;
     int dev = 0, sms = 0;

@@ -69,6 +69,7 @@ struct FusedBwdParams {
     int B, T, d, k, U, Mtok;
     float scale, scale_log2;
     uint32_t *status;
+    unsigned long long *span;   // measurement: kernel span slot, or null
 };
 
 __device__ __forceinline__ bool wait_or_abort(FusedBwdSmem &sm, uint64_t &bar, uint32_t parity,
@@ -112,6 +113,7 @@ __global__ void __launch_bounds__(kThreads, 1) fused_bwd_kernel(const __grid_con
         tmem_relinquish();
     }
     pdl_wait();  // everything read below was written by earlier kernels
+    span_begin(p.span);
     if (threadIdx.x < 128) {
         const int r = threadIdx.x, u = r / p.k;
         const bool valid = u < p.U && b0 + u < p.B;
@@ -339,6 +341,7 @@ __global__ void __launch_bounds__(kThreads, 1) fused_bwd_kernel(const __grid_con
     }
     tc_fence_before();
     __syncthreads();
+    span_end(p.span);
     if (warp == 2) {
         tc_fence_after();
         tmem_dealloc(tmem, 512);
@@ -391,6 +394,7 @@ cudaError_t tc_fused_backward(const Dims &dm, const void *W_o, const void *dY, c
     p.scale = 1.f / sqrtf(64.f);
     p.scale_log2 = 1.4426950408889634f / sqrtf(64.f);
     p.status = sv.status;
+    p.span = active_span();
     const cudaError_t attr = allow_smem((const void *)fused_bwd_kernel, kSmem);
     if (attr != cudaSuccess) return attr;
     const dim3 grid((dm.B + p.U - 1) / p.U, dm.H);

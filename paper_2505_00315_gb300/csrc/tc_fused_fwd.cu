@@ -82,6 +82,7 @@ struct FusedParams {
     int rope_on;           // RoPE on Q and K (Sec. 2.2)
     RopeTable rope;
     uint32_t *status;
+    unsigned long long *span;   // measurement: kernel span slot, or null
 };
 
 // Bounded wait that gives up at once when the CTA is already aborting.
@@ -138,6 +139,7 @@ __global__ void __launch_bounds__(kThreads, 1) fused_fwd_kernel(const __grid_con
         tmem_relinquish();
     }
     pdl_wait();  // gidx and r_sel come from the selection kernel
+    span_begin(p.span);
     if (threadIdx.x < 128) {
         const int r = threadIdx.x, u = r / p.k;
         const bool valid = u < p.U && b0 + u < p.B;
@@ -417,6 +419,7 @@ __global__ void __launch_bounds__(kThreads, 1) fused_fwd_kernel(const __grid_con
     }
     tc_fence_before();
     __syncthreads();
+    span_end(p.span);
     if (warp == 2) {
         tc_fence_after();
         tmem_dealloc(tmem, 512);
@@ -463,6 +466,7 @@ cudaError_t tc_fused_forward(const Dims &dm, const void *X, const void *Wq, cons
     p.rope_on = dm.rope ? 1 : 0;
     if (dm.rope) p.rope = make_rope_table(64, dm.T);
     p.status = sv.status;
+    p.span = active_span();
     const cudaError_t attr = allow_smem((const void *)fused_fwd_kernel, kSmem);
     if (attr != cudaSuccess) return attr;
     const dim3 grid((dm.B + p.U - 1) / p.U, dm.H);

@@ -171,6 +171,7 @@ struct TcParams {
                            // instead of bf16 pairs
     int rope;              // kQKV with half: rotate Q and K (Sec. 2.2) before rounding
     RopeTable rope_tab;
+    unsigned long long *span;   // measurement: this stage's kernel span slot, or null
 };
 
 // Epilogue staging: each warp owns kXpose bytes at the start of the operand
@@ -406,6 +407,7 @@ __global__ void __launch_bounds__(kThreads, Cfg<KIND>::MIN_CTAS)
         fence_barrier_init();
     }
     pdl_wait();  // everything below may read what the previous kernel wrote
+    span_begin(p.span);
     if (KIND == kQKV || KIND == kG) {
         for (int r = threadIdx.x; r < kBM; r += kThreads) {
             const int m = m0 + r;
@@ -742,6 +744,7 @@ __global__ void __launch_bounds__(kThreads, Cfg<KIND>::MIN_CTAS)
     }
     tc_fence_before();
     __syncthreads();
+    span_end(p.span);
     if (warp == 2) {
         tc_fence_after();
         tmem_dealloc(tmem, C::TMEM_COLS);
@@ -797,6 +800,7 @@ TcParams base_params(const Dims &dm, const Saved &sv) {
     p.rsel = sv.rsel;
     p.status = sv.status;
     p.splits = 1;
+    p.span = active_span();
     return p;
 }
 
@@ -820,6 +824,7 @@ bool tc_router(const Dims &dm, const void *X, const void *Wr, float *r_full, uin
     p.H = dm.H;
     p.T = dm.T;
     p.status = status;
+    p.span = active_span();
     p.out_f = r_full;
     p.N = std::min(256, (dm.H + 63) / 64 * 64);  // MMA width: 64-wide W_r blocks
     p.ring_stride = kTile16K + p.N / 64 * kTile8K;

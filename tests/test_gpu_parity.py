@@ -399,3 +399,36 @@ def test_workspace_reuse_gives_same_result():
     np.testing.assert_array_equal(a["I"], b["I"])
     for n in ("Y", "dX", "dW_q", "dW_o", "dW_r"):
         np.testing.assert_allclose(a[n], b[n], rtol=1e-5, atol=1e-6)
+
+
+@pytest.mark.parametrize("name", ["largek_bf16", "pack2_oddB_bf16"])
+def test_stage_kernel_spans_inside_event_windows(name):
+    # The kernel spans (first CTA start to last CTA end, stamped by the kernels
+    # themselves) of every tensor-core stage lie inside that stage's CUDA-event
+    # window, and timing leaves the results unchanged.
+    cfg = next(c for c in SMALL if c.name == name)
+    x = W.make_inputs(cfg)
+    plain = run_layer(cfg, x)
+    dt = cfg.dtype
+    X, Wr, Wq, Wk, Wv, Wo = (to_dev(x[n], dt) for n in ("X", "Wr", "Wq", "Wk", "Wv", "Wo"))
+    dY = to_dev(x["dY"], dt)
+    shape = mosa.make_shape(X, Wq, cfg.k)
+    impl = mosa.stage_impl(shape)
+    mosa.mosa_profile_read()
+    mosa.mosa_profile_stages(0xFFFF)
+    try:
+        Y, I, rs, _, ws = mosa.mosa_forward(X, Wr, Wq, Wk, Wv, Wo, cfg.k)
+        g = mosa.mosa_backward(X, Wr, Wq, Wk, Wv, Wo, I, rs, dY, ws)
+        torch.cuda.synchronize()
+        events = mosa.mosa_profile_read()
+        spans = mosa.mosa_profile_spans(shape, ws)
+    finally:
+        mosa.mosa_profile_stages(0)
+    assert mosa.mosa_check_status(shape, ws) == 0
+    np.testing.assert_array_equal(I.cpu().numpy(), plain["I"])
+    np.testing.assert_allclose(Y.float().cpu().numpy(), plain["Y"], rtol=1e-5, atol=1e-6)
+    np.testing.assert_allclose(g["dX"].float().cpu().numpy(), plain["dX"], rtol=1e-5, atol=1e-6)
+    tensor = [s for s, e in impl.items() if e == "tensor" and events[s][1] > 0]
+    assert tensor
+    for s in tensor:
+        assert 0.0 < spans[s] <= events[s][0] + 0.02, (s, spans[s], events[s])

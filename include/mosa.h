@@ -39,6 +39,11 @@
  *     kernel; MOSA_FUSED_BWD=1 runs the k <= 128 backward's G, row terms and
  *     attention backward as one fused kernel; MOSA_PDL=0 turns programmatic
  *     dependent launch off.  All paths compute the same operation.
+ *     For tests of the give-up path only: MOSA_TEST_ROUTER_WAIT_NS=n limits
+ *     each main-loop wait of the tensor-core router GEMM to n nanoseconds
+ *     instead of 2 s (read when the router is launched or captured, so run
+ *     such a call with MOSA_GRAPHS=0); a wait that runs out makes
+ *     mosa_check_status return MOSA_ERR_DEVICE_TIMEOUT.
  *   - Outputs are overwritten, never accumulated into.
  *   - Arithmetic: fp32 accumulation everywhere.  With bf16 storage the
  *     intermediates fed to tensor-core products are kept as bf16 hi/lo pairs

@@ -94,6 +94,7 @@ struct FwdLargeSmem {
     float part[2][2][128];                    // [block parity][key half]: block max, final sums
     uint64_t q_full, kv_full[kLSlots], kv_empty[kLSlots];
     uint64_t s_full[2], s_free[2], p_ready[2], pv_done[2];   // per buffer parity
+    uint64_t drained;                                         // the MMA issuer's final drain
     uint32_t tmem;
     int abort;
 };
@@ -149,6 +150,7 @@ __global__ void __launch_bounds__(kLT, 1) attn_fwd_tc_kernel(const __grid_consta
             mbar_init(smem_u32(&sm.p_ready[u]), kLWorkers);
             mbar_init(smem_u32(&sm.pv_done[u]), 1);
         }
+        mbar_init(smem_u32(&sm.drained), 1);
         sm.abort = 0;
         fence_barrier_init();
     }
@@ -169,6 +171,7 @@ __global__ void __launch_bounds__(kLT, 1) attn_fwd_tc_kernel(const __grid_consta
             const uint32_t qb = smem_u32(&sm.q_full);
             mbar_expect_tx(qb, kTileHalf);
             tma_load_4d(smem_u32(sm.q), &p.mQ, qb, 0, i0, b, h);
+            int issued = 0;
             for (int t = 0; t < nitems; ++t) {
                 const int s = t % kLSlots;
                 if (!lwait(sm, sm.kv_empty[s], ((t / kLSlots) & 1) ^ 1, p.status)) break;
@@ -178,7 +181,12 @@ __global__ void __launch_bounds__(kLT, 1) attn_fwd_tc_kernel(const __grid_consta
                 const uint32_t fb = smem_u32(&sm.kv_full[s]);
                 mbar_expect_tx(fb, kTileHalf);
                 tma_load_4d(smem_u32(sm.kv[s]), is_v ? &p.mV : &p.mK, fb, 0, blk * kLKeys, b, h);
+                issued = t + 1;
             }
+            // drain: Q and the last load of every slot have landed
+            drain_phase(qb, 0);
+            for (int t = max(0, issued - kLSlots); t < issued; ++t)
+                drain_phase(smem_u32(&sm.kv_full[t % kLSlots]), (t / kLSlots) & 1);
         }
     } else if (warp == 1) {
         if (lane == 0) {
@@ -226,6 +234,7 @@ __global__ void __launch_bounds__(kLT, 1) attn_fwd_tc_kernel(const __grid_consta
                     mma_commit(smem_u32(&sm.pv_done[u]));
                 }
             }
+            drain_mmas(smem_u32(&sm.drained));
         }
     } else if (warp >= 4) {
         pdl_trigger();
@@ -473,6 +482,7 @@ __global__ void __launch_bounds__(kBT, 1) attn_bwd_tc_kernel(const __grid_consta
             mbar_expect_tx(kb, 2 * kTileHalf);
             tma_load_4d(smem_u32(sm.k), &p.mA0, kb, 0, j0, b, h);
             tma_load_4d(smem_u32(sm.v), &p.mA1, kb, 0, j0, b, h);
+            int issued = 0;
             for (int t = 0; t < 2 * nb; ++t) {
                 const int i = t >> 1, is_da = t & 1;
                 const int s = 2 * (i % kBDepth) + is_da;
@@ -482,6 +492,14 @@ __global__ void __launch_bounds__(kBT, 1) attn_bwd_tc_kernel(const __grid_consta
                 const uint32_t fb = smem_u32(&sm.ring_full[s]);
                 mbar_expect_tx(fb, kTileHalf);
                 tma_load_4d(smem_u32(sm.ring[s]), is_da ? &p.mB1 : &p.mB0, fb, 0, q0, b, h);   // dA_i : Q_i
+                issued = t + 1;
+            }
+            // drain: K, V and the last load of every slot (any kBSlots
+            // consecutive loads use every slot once) have landed
+            drain_phase(kb, 0);
+            for (int t = max(0, issued - kBSlots); t < issued; ++t) {
+                const int i = t >> 1;
+                drain_phase(smem_u32(&sm.ring_full[2 * (i % kBDepth) + (t & 1)]), (i / kBDepth) & 1);
             }
         }
     } else if (warp == 1) {
@@ -548,7 +566,9 @@ __global__ void __launch_bounds__(kBT, 1) attn_bwd_tc_kernel(const __grid_consta
                 mma_commit(smem_u32(&sm.dq_full[0]));
                 mma_commit(smem_u32(&sm.dq_full[1]));
             }
-            mma_commit(smem_u32(&sm.acc_done));
+            // acc_done's only phase covers every MMA issued: wait for it here too
+            // (the workers' own wait gives up at once when the CTA is aborting)
+            drain_mmas(smem_u32(&sm.acc_done));
         }
     } else if (warp >= 4) {
         pdl_trigger();
@@ -819,6 +839,7 @@ __global__ void __launch_bounds__(kSmallThreads, 1) attn_fwd_small_kernel(const 
                 tma_load_3d(smem_u32(sm.k[hf]), &p.mK, fb, 64 * hf, b0 * p.k, h);
                 tma_load_3d(smem_u32(sm.v[hf]), &p.mV, fb, 64 * hf, b0 * p.k, h);
             }
+            drain_phase(fb, 0);
         }
     } else if (warp == 1) {
         if (lane == 0) {
@@ -848,7 +869,7 @@ __global__ void __launch_bounds__(kSmallThreads, 1) attn_fwd_small_kernel(const 
                 flag_timeout_b(sm, p.status);
                 mma_commit(smem_u32(&sm.s_full));   // release the softmax warps
             }
-            mma_commit(smem_u32(&sm.o_full));
+            drain_mmas(smem_u32(&sm.o_full));   // o_full's only phase covers every MMA
         }
     } else if (warp >= 4) {
         pdl_trigger();
@@ -963,6 +984,7 @@ __global__ void __launch_bounds__(kSmallThreads, 1) attn_bwd_small_kernel(const 
                 tma_load_3d(smem_u32(sm.v[hf]), &p.mB0, fb, 64 * hf, b0 * p.k, h);
                 tma_load_3d(smem_u32(sm.da[hf]), &p.mB1, fb, 64 * hf, b0 * p.k, h);
             }
+            drain_phase(fb, 0);
         }
     } else if (warp == 1) {
         if (lane == 0) {
@@ -997,7 +1019,7 @@ __global__ void __launch_bounds__(kSmallThreads, 1) attn_bwd_small_kernel(const 
                 mma_commit(smem_u32(&sm.sp_full));
                 mma_commit(smem_u32(&sm.pv_done));
             }
-            mma_commit(smem_u32(&sm.acc_done));
+            drain_mmas(smem_u32(&sm.acc_done));   // acc_done's only phase covers every MMA
         }
     } else if (warp >= 4) {
         pdl_trigger();

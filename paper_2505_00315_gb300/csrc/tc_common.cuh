@@ -51,12 +51,14 @@ __device__ __forceinline__ bool mbar_try_wait(uint32_t bar, uint32_t parity) {
         : "memory");
     return ok != 0;
 }
-// Waits for the phase with the given parity to complete; false on timeout.
-__device__ __forceinline__ bool mbar_wait(uint32_t bar, uint32_t parity) {
+// Waits for the phase with the given parity to complete; false once more than
+// limit_ns have passed.
+__device__ __forceinline__ bool mbar_wait(uint32_t bar, uint32_t parity,
+                                          unsigned long long limit_ns = kWaitLimitNs) {
     if (mbar_try_wait(bar, parity)) return true;
     const unsigned long long t0 = globaltimer();
     while (!mbar_try_wait(bar, parity)) {
-        if (globaltimer() - t0 > kWaitLimitNs) return false;
+        if (globaltimer() - t0 > limit_ns) return false;
     }
     return true;
 }
@@ -215,6 +217,26 @@ __device__ __forceinline__ void mma_commit(uint32_t bar) {
     asm volatile(
         "tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.b64 [%0];" ::"r"(bar)
         : "memory");
+}
+
+// Give-up path of the warp-specialised kernels.  Their waits give up at once
+// when the CTA is already aborting, so without a drain a CTA could reach its
+// final barrier with TMA loads still writing its shared memory, or MMAs still
+// reading it and writing TMEM, and then free TMEM or exit under them.  Before
+// that barrier the thread that issued MMAs waits for all of them, and the
+// thread that issued TMA loads for the last load of every barrier it used,
+// each with the full bound and regardless of the abort flag.  On the normal
+// path these waits find their phases complete, or overlap other warps' work.
+//
+// Waits for the phase of `bar` with the given parity (full bound).
+__device__ __forceinline__ void drain_phase(uint32_t bar, uint32_t parity) {
+    mbar_wait(bar, parity, kWaitLimitNs);
+}
+// The MMA-issuing thread: commits every MMA it issued to `bar` (a barrier of
+// its own, count 1, used for this only) and waits until they have completed.
+__device__ __forceinline__ void drain_mmas(uint32_t bar) {
+    mma_commit(bar);
+    mbar_wait(bar, 0, kWaitLimitNs);
 }
 
 // 32 consecutive fp32 columns of this thread's TMEM lane.

@@ -46,6 +46,7 @@ struct DxSmem {
     uint8_t w[kSlots][kWBytes];      // weight blocks
     uint8_t stage[8][4096];          // epilogue staging, one buffer per epilogue warp
     uint64_t a_full[3], a_empty[3], w_full[kSlots], w_empty[kSlots], out_full[2], out_empty[2];
+    uint64_t drained;   // the MMA issuer's final drain
     uint32_t tmem;
     int abort;
 };
@@ -103,6 +104,7 @@ __global__ void __launch_bounds__(kThreads, 1) scatter_product_kernel(const __gr
             mbar_init(smem_u32(&sm.out_full[i]), 1);
             mbar_init(smem_u32(&sm.out_empty[i]), kWorkers);
         }
+        mbar_init(smem_u32(&sm.drained), 1);
         sm.abort = 0;
         fence_barrier_init();
     }
@@ -120,6 +122,8 @@ __global__ void __launch_bounds__(kThreads, 1) scatter_product_kernel(const __gr
     if (warp == 0) {
         if (lane == 0) {
             int ntile = 0;  // tiles started so far
+            int nw = 0;     // weight-block loads issued
+            int na[3] = {0, 0, 0};   // A_j loads issued
             for (int i = 0; i < nu; ++i) {
                 const long long u = u0 + i;
                 const int c = (int)(u % p.nch);
@@ -139,6 +143,7 @@ __global__ void __launch_bounds__(kThreads, 1) scatter_product_kernel(const __gr
                         tma_load_3d(smem_u32(sm.a[j][0]), &p.mA, ab, 64 * j, m0, h);        // hi
                         if (!p.f16)
                             tma_load_3d(smem_u32(sm.a[j][1]), &p.mA, ab, kLo + 64 * j, m0, h);  // lo
+                        ++na[j];
                     }
                     const uint32_t fb = smem_u32(&sm.w_full[s]);
                     mbar_expect_tx(fb, kWBytes);
@@ -149,10 +154,16 @@ __global__ void __launch_bounds__(kThreads, 1) scatter_product_kernel(const __gr
                     } else {
                         tma_load_3d(smem_u32(sm.w[s]), &p.mW[j], fb, 0, c * kChunk, h);
                     }
+                    nw = idx + 1;
                 }
                 if (!ok) break;
                 if (fresh) ++ntile;
             }
+            // drain: the last load of every weight slot and of every A_j has landed
+            for (int idx = max(0, nw - kSlots); idx < nw; ++idx)
+                drain_phase(smem_u32(&sm.w_full[idx % kSlots]), (idx / kSlots) & 1);
+            for (int j = 0; j < NM; ++j)
+                if (na[j] > 0) drain_phase(smem_u32(&sm.a_full[j]), (na[j] - 1) & 1);
         }
     } else if (warp == 1) {
         if (lane == 0) {
@@ -198,6 +209,7 @@ __global__ void __launch_bounds__(kThreads, 1) scatter_product_kernel(const __gr
                 // release the epilogue warps
                 for (int b2 = 0; b2 < 2; ++b2) mma_commit(smem_u32(&sm.out_full[b2]));
             }
+            drain_mmas(smem_u32(&sm.drained));
         }
     } else if (warp >= 4) {
         pdl_trigger();

@@ -134,13 +134,21 @@ __global__ void __launch_bounds__(kThreads, 1) fused_bwd_kernel(const __grid_con
                 for (int hf = 0; hf < 2; ++hf)
                     tma_load_3d(smem_u32(sm.qkv[j][hf]), &p.mQKV[j], qb, 64 * hf, b0 * p.k, h);
             // phase 1: W_o blocks (rows p, 64 columns of d)
+            int issued = 0;
             for (int kb = 0; kb < nkb; ++kb) {
                 const int s = kb % kStages;
                 if (!wait_or_abort(sm, sm.empty[s], ((kb / kStages) & 1) ^ 1, p.status)) break;
                 const uint32_t fb = smem_u32(&sm.full[s]);
                 mbar_expect_tx(fb, 8192);
                 tma_load_3d(smem_u32(ring(s) + kHalf), &p.mWo, fb, kb * 64, 0, h);
+                issued = kb + 1;
             }
+            // drain: Q, K, V and the last load of every ring slot have landed (a
+            // stage whose gathering threads gave up before issuing it never
+            // completes; its wait then runs out the full bound)
+            drain_phase(qb, 0);
+            for (int kb = max(0, issued - kStages); kb < issued; ++kb)
+                drain_phase(smem_u32(&sm.full[kb % kStages]), (kb / kStages) & 1);
         }
     } else if (warp == 1) {
         // ------------------------------------------------------------- MMA
@@ -191,13 +199,12 @@ __global__ void __launch_bounds__(kThreads, 1) fused_bwd_kernel(const __grid_con
                 mma_k128(tmem + kColDK, ptile, sm.qkv[0], true, idMN);    // dK = dS^T Q
                 mma_k128(tmem + kColDQ, ptile, sm.qkv[1], false, idKM);   // dQ = dS K
             }
-            mma_commit(smem_u32(&sm.acc_done));
             if (!ok) {
                 // release every wait of the other warps that may still be pending
                 mma_commit(smem_u32(&sm.sp_full));
                 mma_commit(smem_u32(&sm.pv_done));
-                mma_commit(smem_u32(&sm.acc_done));
             }
+            drain_mmas(smem_u32(&sm.acc_done));   // acc_done's only phase covers every MMA
         }
     } else if (warp >= 4) {
         const int t = threadIdx.x - 128;

@@ -61,6 +61,7 @@ struct FusedSmem {
     uint64_t full[kStages], empty[kStages];
     uint64_t qkv_done, qkv_staged, qkv_read, s_full, p_ready, o_full, ar_ready;
     uint64_t wo_full[2], wo_empty[2], out_full[2], out_empty[2];
+    uint64_t drained;   // the MMA issuer's final drain
     uint32_t tmem;
     int abort;
 };
@@ -131,6 +132,7 @@ __global__ void __launch_bounds__(kThreads, 1) fused_fwd_kernel(const __grid_con
             mbar_init(smem_u32(&sm.out_full[i]), 1);
             mbar_init(smem_u32(&sm.out_empty[i]), kWorkers);
         }
+        mbar_init(smem_u32(&sm.drained), 1);
         sm.abort = 0;
         fence_barrier_init();
     }
@@ -153,6 +155,7 @@ __global__ void __launch_bounds__(kThreads, 1) fused_fwd_kernel(const __grid_con
     if (warp == 0) {
         // ---------------------------------------------------------- producer
         if (lane == 0) {
+            int issued = 0, nc = 0;   // ring stages and W_o chunks loaded
             for (int kb = 0; kb < nkb; ++kb) {
                 const int s = kb % kStages;
                 if (!wait_or_abort(sm, sm.empty[s], ((kb / kStages) & 1) ^ 1, p.status)) break;
@@ -160,6 +163,7 @@ __global__ void __launch_bounds__(kThreads, 1) fused_fwd_kernel(const __grid_con
                 mbar_expect_tx(fb, 3 * 8192);
                 for (int j = 0; j < 3; ++j)
                     tma_load_3d(smem_u32(slot(s) + kHalf + j * 8192), &p.mW[j], fb, 0, kb * 64, h);
+                issued = kb + 1;
             }
             // phase 4: W_o chunks into the K / V tiles once P V is done and
             // their TMA stores have read them
@@ -174,8 +178,15 @@ __global__ void __launch_bounds__(kThreads, 1) fused_fwd_kernel(const __grid_con
                     mbar_expect_tx(fb, 4 * 8192);
                     for (int j = 0; j < 4; ++j)
                         tma_load_3d(smem_u32(dst + j * 8192), &p.mWo, fb, c * kChunk + 64 * j, 0, h);
+                    nc = c + 1;
                 }
             }
+            // drain: the last load of every ring slot and W_o buffer has landed
+            // (a ring stage whose gathering threads gave up before issuing it
+            // never completes; its wait then runs out the full bound)
+            for (int kb = max(0, issued - kStages); kb < issued; ++kb)
+                drain_phase(smem_u32(&sm.full[kb % kStages]), (kb / kStages) & 1);
+            for (int c = max(0, nc - 2); c < nc; ++c) drain_phase(smem_u32(&sm.wo_full[c & 1]), (c >> 1) & 1);
         }
     } else if (warp == 1) {
         // ------------------------------------------------------------- MMA
@@ -253,6 +264,7 @@ __global__ void __launch_bounds__(kThreads, 1) fused_fwd_kernel(const __grid_con
                 // release every epilogue wait that may still be pending
                 for (int i = 0; i < 2; ++i) mma_commit(smem_u32(&sm.out_full[i]));
             }
+            drain_mmas(smem_u32(&sm.drained));
         }
     } else if (warp == 3) {
         // ------------------------------------------------- TMA stores

@@ -33,6 +33,7 @@
 // kernel of their own (tc_dx.cu).
 #include <algorithm>
 #include <cstdio>
+#include <cstdlib>
 #include <mutex>
 
 #include "launch.h"
@@ -172,6 +173,8 @@ struct TcParams {
     int rope;              // kQKV with half: rotate Q and K (Sec. 2.2) before rounding
     RopeTable rope_tab;
     unsigned long long *span;   // measurement: this stage's kernel span slot, or null
+    unsigned long long wait_ns; // limit of each main-loop wait (the waits that let
+                                // copies and MMAs in flight finish keep kWaitLimitNs)
 };
 
 // Epilogue staging: each warp owns kXpose bytes at the start of the operand
@@ -288,9 +291,11 @@ __device__ __forceinline__ void gather_operand(const TcParams &p, uint8_t *sA, u
     const bf16 *src = static_cast<const bf16 *>(p.src_rows);
     const int32_t *gi = p.gidx + (size_t)h * p.Mtok;
     int landed = 0;  // stages whose full barrier this thread has arrived on
+    int issued = 0;  // stages whose copies this thread has issued
     for (int it = 0; it < nkb; ++it) {
         const int s = it % S;
-        if (!mbar_wait(smem_u32(&empty[s]), ((it / S) & 1) ^ 1) || *(volatile int *)s_abort) {
+        if (!mbar_wait(smem_u32(&empty[s]), ((it / S) & 1) ^ 1, p.wait_ns) ||
+            *(volatile int *)s_abort) {
             atomicOr(p.status, kStatusTimeout);
             *(volatile int *)s_abort = 1;
             break;
@@ -337,6 +342,7 @@ __device__ __forceinline__ void gather_operand(const TcParams &p, uint8_t *sA, u
             }
         }
         cp_async_commit();
+        issued = it + 1;
         if (it >= LAG) {
             cp_async_wait<LAG>();
             fence_proxy_async();
@@ -344,9 +350,10 @@ __device__ __forceinline__ void gather_operand(const TcParams &p, uint8_t *sA, u
             ++landed;
         }
     }
+    // Every stage issued lands before its barrier is arrived on, also after a
+    // give-up, so that the producer's drain of the same stages completes.
     cp_async_wait<0>();
     fence_proxy_async();
-    const int issued = *(volatile int *)s_abort ? landed : nkb;
     for (int it = landed; it < issued; ++it) mbar_arrive(smem_u32(&full[it % S]));
 }
 
@@ -439,7 +446,7 @@ __global__ void __launch_bounds__(kThreads, Cfg<KIND>::MIN_CTAS)
             const int s = it % ns;
             const uint32_t fb = smem_u32(&full[s]);
             bool ok = true;
-            if (lane == 0) ok = mbar_wait(smem_u32(&empty[s]), ((it / ns) & 1) ^ 1);
+            if (lane == 0) ok = mbar_wait(smem_u32(&empty[s]), ((it / ns) & 1) ^ 1, p.wait_ns);
             ok = __shfl_sync(0xffffffffu, ok ? 1 : 0, 0) != 0;
             if (!ok || *(volatile int *)s_abort) {
                 if (lane == 0) {
@@ -473,10 +480,13 @@ __global__ void __launch_bounds__(kThreads, Cfg<KIND>::MIN_CTAS)
             }
             issued = it + 1;
         }
-        if (*(volatile int *)s_abort && lane == 0) {
-            // Let copies already in flight land before the CTA can exit.
+        if (lane == 0) {
+            // Copies in flight land before the CTA can exit: the last load of
+            // every ring slot (on the normal path all of them have been consumed).
+            // For gathered kinds a stage whose gathering threads gave up before
+            // issuing it never completes; its wait then runs out the full bound.
             for (int it = max(0, issued - ns); it < issued; ++it)
-                mbar_wait(smem_u32(&full[it % ns]), (it / ns) & 1);
+                drain_phase(smem_u32(&full[it % ns]), (it / ns) & 1);
         }
     } else if (warp == 1) {
         // ------------------------------------------------------ MMA issuer
@@ -486,7 +496,8 @@ __global__ void __launch_bounds__(kThreads, Cfg<KIND>::MIN_CTAS)
                                    : idesc_bf16(kBM, C::BN, C::A_MN, C::B_MN);
             for (int it = 0; it < nkb; ++it) {
                 const int s = it % ns;
-                if (!mbar_wait(smem_u32(&full[s]), (it / ns) & 1) || *(volatile int *)s_abort) {
+                if (!mbar_wait(smem_u32(&full[s]), (it / ns) & 1, p.wait_ns) ||
+                    *(volatile int *)s_abort) {
                     atomicOr(p.status, kStatusTimeout);
                     *(volatile int *)s_abort = 1;
                     break;
@@ -542,7 +553,14 @@ __global__ void __launch_bounds__(kThreads, Cfg<KIND>::MIN_CTAS)
         const int part = warp < 4 ? 1 : 0;
         const int r = q * 32 + lane;
         const int mg = m0 + r;
-        const bool ok = mbar_wait(smem_u32(done), 0);
+        const bool ok = mbar_wait(smem_u32(done), 0, p.wait_ns);
+        if (!ok) {
+            // Give up: stop the producer and the MMA issuer, then wait (full
+            // bound) for the MMAs already issued, which the issuer's last
+            // commit covers, before TMEM can be freed.
+            *(volatile int *)s_abort = 1;
+            mbar_wait(smem_u32(done), 0, kWaitLimitNs);
+        }
         tc_fence_after();
         if (warp >= 4) pdl_trigger();  // main loop done: the next kernel may start its prologue
         // warp-uniform, since the TMEM loads below are warp-collective
@@ -776,6 +794,7 @@ bool map_heads(CUtensorMap *m, const void *base, uint64_t H, uint64_t rows, uint
 template <int KIND>
 cudaError_t launch_kind(const TcParams &p, dim3 grid, cudaStream_t s, bool early = true) {
     constexpr int smem = smem_bytes<KIND>();
+    if (p.wait_ns == 0) return cudaErrorInvalidValue;  // every launcher sets a wait limit
     const cudaError_t attr = allow_smem((const void *)tc_gemm_kernel<KIND>, smem);
     if (attr != cudaSuccess) return attr;
     cudaError_t e = launch_ex(early, tc_gemm_kernel<KIND>, grid, dim3(kThreads), smem, s, p);
@@ -801,7 +820,17 @@ TcParams base_params(const Dims &dm, const Saved &sv) {
     p.status = sv.status;
     p.splits = 1;
     p.span = active_span();
+    p.wait_ns = tc::kWaitLimitNs;
     return p;
+}
+
+// Main-loop wait limit of the router GEMM: kWaitLimitNs, or for tests of the
+// give-up path the value of MOSA_TEST_ROUTER_WAIT_NS (nanoseconds, > 0).
+unsigned long long router_wait_ns() {
+    const char *v = std::getenv("MOSA_TEST_ROUTER_WAIT_NS");
+    if (v == nullptr || v[0] == '\0') return tc::kWaitLimitNs;
+    const unsigned long long ns = std::strtoull(v, nullptr, 10);
+    return ns > 0 ? ns : tc::kWaitLimitNs;
 }
 
 bool map_2d(CUtensorMap *m, const void *base, uint64_t rows, uint64_t cols, uint32_t box_rows) {
@@ -825,6 +854,7 @@ bool tc_router(const Dims &dm, const void *X, const void *Wr, float *r_full, uin
     p.T = dm.T;
     p.status = status;
     p.span = active_span();
+    p.wait_ns = router_wait_ns();
     p.out_f = r_full;
     p.N = std::min(256, (dm.H + 63) / 64 * 64);  // MMA width: 64-wide W_r blocks
     p.ring_stride = kTile16K + p.N / 64 * kTile8K;

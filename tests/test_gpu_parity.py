@@ -432,3 +432,38 @@ def test_stage_kernel_spans_inside_event_windows(name):
     assert tensor
     for s in tensor:
         assert 0.0 < spans[s] <= events[s][0] + 0.02, (s, spans[s], events[s])
+
+
+def test_router_wait_limit_gives_up_then_next_call_is_exact(monkeypatch):
+    # The router GEMM's main-loop waits get a 1 us limit: its epilogue waits
+    # for the whole 128-block K loop (d = 8192), gives up, stops the producer
+    # and the MMA issuer, lets the copies and MMAs in flight finish, and the
+    # status word reads MOSA_ERR_DEVICE_TIMEOUT.  The same workspace then gives
+    # the oracle's results on the next (normal) call.
+    cfg = W.MosaConfig("router_wait_bf16", B=1, T=256, d=8192, H=8, hp=64, k=32, dtype="bf16",
+                       seed=41)
+    x = W.make_inputs(cfg)
+    Y, I, rs, rf = oracle.forward(x["X"], *weights(x), k=cfg.k)
+    assert sigmoid_gap(rf, cfg.k) > 1e-3
+    X, Wr, Wq, Wk, Wv, Wo = (to_dev(x[n], cfg.dtype) for n in ("X", "Wr", "Wq", "Wk", "Wv", "Wo"))
+    shape = mosa.make_shape(X, Wq, cfg.k)
+    assert mosa.stage_impl(shape)["router"] == "tensor"
+    _, _, _, rf0, ws = mosa.mosa_forward(X, Wr, Wq, Wk, Wv, Wo, cfg.k, want_r_full=True)
+    torch.cuda.synchronize()
+    assert mosa.mosa_check_status(shape, ws) == 0
+    monkeypatch.setenv("MOSA_GRAPHS", "0")
+    monkeypatch.setenv("MOSA_TEST_ROUTER_WAIT_NS", "1000")
+    mosa.mosa_forward(X, Wr, Wq, Wk, Wv, Wo, cfg.k, workspace=ws, want_r_full=True,
+                      out={"r_full": rf0})
+    torch.cuda.synchronize()
+    assert mosa.mosa_check_status(shape, ws) == 4          # MOSA_ERR_DEVICE_TIMEOUT
+    monkeypatch.delenv("MOSA_TEST_ROUTER_WAIT_NS")
+    monkeypatch.delenv("MOSA_GRAPHS")
+    Yg, Ig, rsg, rfg, _ = mosa.mosa_forward(X, Wr, Wq, Wk, Wv, Wo, cfg.k, workspace=ws,
+                                            want_r_full=True)
+    torch.cuda.synchronize()
+    assert mosa.mosa_check_status(shape, ws) == 0
+    np.testing.assert_array_equal(Ig.cpu().numpy(), I)
+    assert_close("r_full", rfg.cpu().numpy(), rf, cfg.dtype)
+    assert_close("r_sel", rsg.cpu().numpy(), rs, cfg.dtype)
+    assert_close("Y", Yg.cpu().numpy(), Y, cfg.dtype)

@@ -65,6 +65,9 @@ def parse_args():
     p.add_argument("--window", type=int, default=0,
                    help="with --dense-heads: local heads over blocks of this many tokens "
                         "(Sec. 3.4); 0 = dense causal heads")
+    p.add_argument("--profile-run", action="store_true",
+                   help="for profilers: run --warmup then --steps plain layer steps (no "
+                        "timing, stage profiling, graph or end-to-end passes) and exit")
     p.add_argument("--ingest-ncu", metavar="CSV", default=None,
                    help="turn an ncu CSV with dram__bytes_read/write.sum per kernel (taken on "
                         "this command's workload) into profiles/traffic.json and exit")
@@ -466,6 +469,18 @@ def main():
 
     def step():
         layer(D["X"], D["dY"], outs, grads)
+
+    if args.profile_run:
+        # a short, fixed launch sequence for ncu: warm-up steps, then the steps to capture
+        for _ in range(args.warmup + args.steps):
+            step()
+        torch.cuda.synchronize()
+        st = mosa.mosa_check_status(shape, ws) if not hybrid else 0
+        print(json.dumps({"profile_run": cfg.name, "steps": args.steps, "warmup": args.warmup,
+                          "launches": int(mosa.mosa_kernel_launches()), "status": int(st)}))
+        if st != 0:
+            raise SystemExit(f"device status {st}")
+        return
 
     # Warm-up, then one profiled pass to find the dominant stage.
     for _ in range(max(3, args.warmup)):

@@ -171,9 +171,8 @@ cudaError_t tc_f16_copies(const Dims &dm, const void *X, const void *Wq, const v
 // W_r [d,H] bf16 -> sv.WrT [H,d] fp32 (read by the dX epilogue).
 cudaError_t tc_transpose_wr(const Dims &dm, const void *Wr, const Saved &sv, cudaStream_t s);
 cudaError_t tc_attn_fwd(const Dims &dm, const Saved &sv, cudaStream_t s);
-// Zeroes the fp32 dQ accumulator the k > 128 attention backward adds into
-// (sv.G); must precede tc_attn_bwd on its stream's timeline.
-cudaError_t tc_zero_dq(const Dims &dm, const Saved &sv, cudaStream_t s);
+// For k > 128 the attention backward reduce-adds dQ into the fp32
+// accumulator sv.G, whose rows the G kernel (tc_out_bwd_g) zeroes first.
 cudaError_t tc_attn_bwd(const Dims &dm, const Saved &sv, cudaStream_t s);
 cudaError_t tc_w_bwd(const Dims &dm, const void *X, const Saved &sv, float *dWq, float *dWk,
                      float *dWv, float *dWr, cudaStream_t s);

@@ -277,7 +277,6 @@ mosa_status backward_tc(const Dims &dm, const void *X, const void *W_r, const vo
     }
     {
         StageScope st_(kStageAttnBwd, s);
-        MOSA_TRY(tc_zero_dq(dm, sv, s));   // the attention backward adds dQ into it
         MOSA_TRY(launch_attn_bwd(dm, sv, s));
         // (the fp16 path turns dQ and dK back before rounding them)
         if (dm.rope && !attn_f16(dm)) MOSA_TRY(rope_qk(dm, sv, true, s));
@@ -357,7 +356,6 @@ mosa_status backward_all(const Dims &dm, const void *X, const void *W_r, const v
     }
     {
         StageScope st_(kStageAttnBwd, s);
-        if (use_tc(dm)) MOSA_TRY(tc_zero_dq(dm, sv, s));   // the dQ accumulator
         MOSA_TRY(launch_attn_bwd(dm, sv, s));
         if (dm.rope) MOSA_TRY(rope_qk(dm, sv, true, s));
     }

@@ -1156,11 +1156,6 @@ cudaError_t tc_attn_fwd(const Dims &dm, const Saved &sv, cudaStream_t s) {
     return e;
 }
 
-cudaError_t tc_zero_dq(const Dims &dm, const Saved &sv, cudaStream_t s) {
-    if (dm.k <= kSmallK) return cudaSuccess;
-    return cudaMemsetAsync(sv.G, 0, sizeof(float) * (size_t)dm.H * dm.B * dm.k * 64, s);
-}
-
 cudaError_t tc_attn_bwd(const Dims &dm, const Saved &sv, cudaStream_t s) {
     BwdParams kv, dq;
     memset(&kv, 0, sizeof(kv));
@@ -1227,7 +1222,7 @@ cudaError_t tc_attn_bwd(const Dims &dm, const Saved &sv, cudaStream_t s) {
     const size_t rows = (size_t)dm.H * dm.B * dm.k;
     const cudaError_t attr = allow_smem((const void *)attn_bwd_tc_kernel, kBwdLargeSmem);
     if (attr != cudaSuccess) return attr;
-    // (the dQ accumulator sv.G has been zeroed by the caller: tc_zero_dq)
+    // (the dQ accumulator sv.G has been zeroed by the G kernel before this)
     dim3 grid(dm.B, dm.H, (dm.k + 127) / 128);   // key tiles slowest (see the kernel)
     cudaError_t e = launch_pdl(attn_bwd_tc_kernel, grid, dim3(kBT), kBwdLargeSmem, s, bp);
     const size_t n = rows * 8;

@@ -173,6 +173,8 @@ struct TcParams {
     int rope;              // kQKV with half: rotate Q and K (Sec. 2.2) before rounding
     RopeTable rope_tab;
     unsigned long long *span;   // measurement: this stage's kernel span slot, or null
+    float *zero_rows;      // kG: [H, B*k, 64] fp32 rows zeroed alongside (the dQ
+                           // accumulator of the k > 128 attention backward), or null
     unsigned long long wait_ns; // limit of each main-loop wait (the waits that let
                                 // copies and MMAs in flight finish keep kWaitLimitNs)
 };
@@ -657,6 +659,11 @@ __global__ void __launch_bounds__(kThreads, Cfg<KIND>::MIN_CTAS)
             }
             const int row0 = m0 + q * 32;
             const int nrows = min(32, p.M - row0);
+            if (p.zero_rows != nullptr && nrows > 0) {
+                // this warp's rows of the dQ accumulator: one contiguous block
+                float4 *z = reinterpret_cast<float4 *>(p.zero_rows + ((size_t)h * p.Mtok + row0) * 64);
+                for (int u = lane; u < nrows * 16; u += 32) z[u] = make_float4(0.f, 0.f, 0.f, 0.f);
+            }
             if (!p.half) {
                 bf16 *dA = static_cast<bf16 *>(p.out[0]) + ((size_t)h * p.Mtok + row0) * 128;
                 store_rows256(xb, lane, nrows, [&](int rl, int u) {
@@ -982,6 +989,9 @@ cudaError_t tc_out_bwd_g(const Dims &dm, const void *Wo, const void *dY, const S
     p.out_f1 = sv.Dd;
     p.out_f2 = sv.dlogit;
     p.half = attn_f16(dm) ? 1 : 0;
+    // the k > 128 attention backward (next on this stream) reduce-adds dQ into
+    // sv.G: its rows start at zero here, beside dA
+    if (dm.k > 128) p.zero_rows = sv.G;
     dim3 grid((p.M + kBM - 1) / kBM, 1, dm.H);
     return launch_kind<kG>(p, grid, s);
 }

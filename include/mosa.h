@@ -38,7 +38,11 @@
  *     as three kernels (projection, attention, output) instead of one fused
  *     kernel; MOSA_FUSED_BWD=1 runs the k <= 128 backward's G, row terms and
  *     attention backward as one fused kernel; MOSA_PDL=0 turns programmatic
- *     dependent launch off.  All paths compute the same operation.
+ *     dependent launch off; MOSA_HEADSUM=0 turns off the token-major output
+ *     product (used for k > 128 when every head keeps at least half of the
+ *     tokens) in favour of the row-major one, MOSA_HEADSUM=1 uses the
+ *     token-major output and input-gradient products wherever they apply.
+ *     All paths compute the same operation.
  *     For tests of the give-up path only: MOSA_TEST_ROUTER_WAIT_NS=n limits
  *     each main-loop wait of the tensor-core router GEMM to n nanoseconds
  *     instead of 2 s (read when the router is launched or captured, so run

@@ -100,6 +100,8 @@ struct Saved {
     void *X16;          // [B*T,d] fp16 copy of X
     void *W16;          // [3][H,d,hp] fp16 copies of W_q, W_k, W_v
     unsigned long long *spans;   // [16][2] kernel spans of the timed stages (measurement)
+    int32_t *pos;       // [H,B*T] row b*k + i of head h holding token (b, t), or -1
+                        // (token-major output and input-gradient products, k > 128)
 };
 
 // Rotary position encoding (Sec. 2.2): pair p of the first h'/2 dimensions of

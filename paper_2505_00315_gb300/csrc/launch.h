@@ -142,9 +142,21 @@ cudaError_t tc_fused_backward(const Dims &dm, const void *W_o, const void *dY, c
                               cudaStream_t s);
 cudaError_t tc_qkv(const Dims &dm, const void *X, const void *Wq, const void *Wk, const void *Wv,
                    const Saved &sv, cudaStream_t s);
-// zero_output = false: the caller has already zeroed Y / dX on this stream's timeline.
+// zero_output = false: the caller has already zeroed Y / dX on this stream's timeline
+// (not needed on the token-major path, which writes every element).  pos_ready:
+// the token-major path's row map sv.pos has been built on this stream's timeline.
 cudaError_t tc_out(const Dims &dm, const void *Wo, const Saved &sv, float *Y, cudaStream_t s,
-                   bool zero_output);
+                   bool zero_output, bool pos_ready = false);
+// Token-major products (tc_headsum.cu): every head's rows of a 128-token tile
+// summed in TMEM and written once, for layers whose heads keep a large share
+// of the tokens: F5 when T <= 2k; B3 (fp16 attention path, H <= 16) only with
+// MOSA_HEADSUM=1, which also lifts the T/k limit.  MOSA_HEADSUM=0 turns both off.
+bool use_headsum_out(const Dims &dm);
+bool use_headsum_dx(const Dims &dm);
+// sv.pos[h, b*T + t] = the row b*k + i of head h that holds token t, or -1.
+cudaError_t tc_token_rows(const Dims &dm, const Saved &sv, cudaStream_t s);
+cudaError_t tc_out_headsum(const Dims &dm, const void *Wo, const Saved &sv, float *Y, cudaStream_t s);
+cudaError_t tc_dx_headsum(const Dims &dm, const Saved &sv, float *dX, cudaStream_t s);
 // B1 in two independent parts: G and the row terms; dW_o.
 cudaError_t tc_out_bwd_g(const Dims &dm, const void *Wo, const void *dY, const Saved &sv,
                          cudaStream_t s);
@@ -152,7 +164,7 @@ cudaError_t tc_out_bwd_w(const Dims &dm, const void *dY, const Saved &sv, float 
                          cudaStream_t s);
 cudaError_t tc_in_bwd(const Dims &dm, const void *Wq, const void *Wk, const void *Wv,
                       const void *Wr, const Saved &sv, float *dX, cudaStream_t s,
-                      bool zero_output);
+                      bool zero_output, bool pos_ready = false);
 // F5 as a persistent scatter product over (head, 128-row tile, 256-column
 // chunk) units: Y[g(m), :] += AR(m, :) W_o[h] (Y zeroed by the caller).
 cudaError_t tc_out_scatter(const Dims &dm, const void *Wo, const Saved &sv, float *Y,

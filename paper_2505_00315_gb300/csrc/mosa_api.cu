@@ -74,6 +74,7 @@ size_t carve(const Dims &dm, char *base, Saved *sv) {
     if (dm.bf16 && dm.hp == 64 && dm.k > 128) {
         s.X16 = take((size_t)2 * dm.B * dm.T * dm.d);
         s.W16 = take((size_t)2 * 3 * dm.H * dm.d * dm.hp);
+        s.pos = (int32_t *)take(sizeof(int32_t) * (size_t)dm.H * dm.B * dm.T);
     }
     if (sv) *sv = s;
     return off;
@@ -185,7 +186,9 @@ mosa_status forward_tc(const Dims &dm, const void *X, const void *W_r, const voi
         MOSA_TRY(launch_router_auto(dm, X, W_r, rf, sv.status, s));
     }
     MOSA_TRY(link(s, r.side, r.ev[0]));
-    if (!dm.accumulate) MOSA_TRY(cudaMemsetAsync(Y, 0, sizeof(float) * ny, r.side));
+    // (the token-major output product writes every element of Y itself)
+    const bool headsum = !use_fused_forward(dm) && use_headsum_out(dm);
+    if (!dm.accumulate && !headsum) MOSA_TRY(cudaMemsetAsync(Y, 0, sizeof(float) * ny, r.side));
     if (route) {
         StageScope st_(kStageSelect, s);
         MOSA_TRY(launch_select(dm.B * dm.H, dm.T, dm.k, rf, I, r_sel, dm.B, dm.H, sv.gidx,
@@ -196,6 +199,11 @@ mosa_status forward_tc(const Dims &dm, const void *X, const void *W_r, const voi
     } else {
         StageScope st_(kStageSelect, s);
         MOSA_TRY(launch_indices_to_rows(dm, I_in, rsel_in, sv.gidx, sv.rsel, sv.status, s));
+    }
+    if (headsum) {
+        // the token-major output product's row map, beside the projection and attention
+        MOSA_TRY(link(s, r.side, r.ev[2]));
+        MOSA_TRY(tc_token_rows(dm, sv, r.side));
     }
     if (use_fused_forward(dm)) {
         MOSA_TRY(link(r.side, s, r.ev[1]));  // Y zeroed
@@ -213,10 +221,10 @@ mosa_status forward_tc(const Dims &dm, const void *X, const void *W_r, const voi
         StageScope st_(kStageAttnFwd, s);
         MOSA_TRY(launch_attn_fwd(dm, sv, s));
     }
-    MOSA_TRY(link(r.side, s, r.ev[1]));  // Y zeroed
+    MOSA_TRY(link(r.side, s, r.ev[1]));  // Y zeroed, or the row map built
     {
         StageScope st_(kStageOut, s);
-        MOSA_TRY(tc_out(dm, W_o, sv, Y, s, false));
+        MOSA_TRY(tc_out(dm, W_o, sv, Y, s, false, headsum));
     }
     return MOSA_OK;
 }
@@ -269,8 +277,13 @@ mosa_status backward_tc(const Dims &dm, const void *X, const void *W_r, const vo
         MOSA_TRY(tc_out_bwd_w(dm, dY, sv, dW_o, t));
     }
     MOSA_TRY(tc_transpose_wr(dm, W_r, sv, t));
-    if (!dm.accumulate) MOSA_TRY(cudaMemsetAsync(dX, 0, sizeof(float) * nx, t));
-    MOSA_TRY(cudaEventRecord(r.ev[1], t));  // dX zeroed, W_r transposed
+    // (the token-major dX product writes every element of dX itself, from the row map)
+    const bool headsum = use_headsum_dx(dm);
+    if (headsum)
+        MOSA_TRY(tc_token_rows(dm, sv, t));
+    else if (!dm.accumulate)
+        MOSA_TRY(cudaMemsetAsync(dX, 0, sizeof(float) * nx, t));
+    MOSA_TRY(cudaEventRecord(r.ev[1], t));  // dX zeroed or the row map built, W_r transposed
     {
         StageScope st_(kStageOutBwd, s);
         MOSA_TRY(tc_out_bwd_g(dm, W_o, dY, sv, s));
@@ -286,10 +299,10 @@ mosa_status backward_tc(const Dims &dm, const void *X, const void *W_r, const vo
         StageScope st_(kStageWBwd, t);
         MOSA_TRY(tc_w_bwd(dm, X, sv, dW_q, dW_k, dW_v, dW_r, t));
     }
-    MOSA_TRY(cudaStreamWaitEvent(s, r.ev[1], 0));  // dX zeroed, W_r transposed
+    MOSA_TRY(cudaStreamWaitEvent(s, r.ev[1], 0));  // dX zeroed or the row map built, W_r transposed
     {
         StageScope st_(kStageInBwd, s);
-        MOSA_TRY(tc_in_bwd(dm, W_q, W_k, W_v, W_r, sv, dX, s, false));
+        MOSA_TRY(tc_in_bwd(dm, W_q, W_k, W_v, W_r, sv, dX, s, false, headsum));
     }
     MOSA_TRY(link(t, s, r.ev[3]));  // join
     return MOSA_OK;
@@ -493,7 +506,8 @@ bool graphs_enabled() {
 }
 
 int path_bits(const Dims &dm) {
-    return (use_tc(dm) ? 1 : 0) | (use_fused_forward(dm) ? 2 : 0) | (use_fused_backward(dm) ? 4 : 0);
+    return (use_tc(dm) ? 1 : 0) | (use_fused_forward(dm) ? 2 : 0) | (use_fused_backward(dm) ? 4 : 0) |
+           (use_headsum_out(dm) ? 8 : 0) | (use_headsum_dx(dm) ? 16 : 0);
 }
 
 GraphKey make_key(int op, const Dims &dm, const mosa_shape *shape,
@@ -503,7 +517,7 @@ GraphKey make_key(int op, const Dims &dm, const mosa_shape *shape,
     std::memset(&k, 0, sizeof(k));
     k.op = op;
     cudaGetDevice(&k.device);
-    k.tc = path_bits(dm) | (dense ? path_bits(*dense) << 3 : 0);
+    k.tc = path_bits(dm) | (dense ? path_bits(*dense) << 5 : 0);
     k.mask = profile_mask();
     k.shape = *shape;
     k.extra[0] = extra0;

@@ -965,7 +965,14 @@ cudaError_t tc_qkv(const Dims &dm, const void *X, const void *Wq, const void *Wk
 }
 
 cudaError_t tc_out(const Dims &dm, const void *Wo, const Saved &sv, float *Y, cudaStream_t s,
-                   bool zero_output) {
+                   bool zero_output, bool pos_ready) {
+    if (use_headsum_out(dm)) {
+        if (!pos_ready) {
+            cudaError_t e = tc_token_rows(dm, sv, s);
+            if (e != cudaSuccess) return e;
+        }
+        return tc_out_headsum(dm, Wo, sv, Y, s);
+    }
     if (zero_output) {
         cudaError_t e = cudaMemsetAsync(Y, 0, sizeof(float) * (size_t)dm.B * dm.T * dm.d, s);
         if (e != cudaSuccess) return e;
@@ -1019,7 +1026,15 @@ cudaError_t tc_out_bwd_w(const Dims &dm, const void *dY, const Saved &sv, float 
 }
 
 cudaError_t tc_in_bwd(const Dims &dm, const void *Wq, const void *Wk, const void *Wv,
-                      const void *Wr, const Saved &sv, float *dX, cudaStream_t s, bool zero_output) {
+                      const void *Wr, const Saved &sv, float *dX, cudaStream_t s, bool zero_output,
+                      bool pos_ready) {
+    if (use_headsum_dx(dm)) {
+        if (!pos_ready) {
+            cudaError_t e = tc_token_rows(dm, sv, s);
+            if (e != cudaSuccess) return e;
+        }
+        return tc_dx_headsum(dm, sv, dX, s);
+    }
     if (zero_output) {
         cudaError_t e = cudaMemsetAsync(dX, 0, sizeof(float) * (size_t)dm.B * dm.T * dm.d, s);
         if (e != cudaSuccess) return e;

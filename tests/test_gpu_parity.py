@@ -80,16 +80,24 @@ SMALL = [
 ]
 
 
-@pytest.fixture(params=["default", "unfused", "fused_bwd", "simt"])
+@pytest.fixture(params=["default", "unfused", "fused_bwd", "rowmajor", "tokenmajor", "simt"])
 def kernel_path(request, monkeypatch):
     """Run a test on the default kernels (tensor cores where the shape allows,
-    the fused forward for k <= 128), again with the forward as three separate
-    kernels, again with the fused backward switched on, and again with the
-    CUDA-core kernels forced."""
+    the fused forward for k <= 128, the token-major output and input-gradient
+    products for k > 128 where the heads keep a large share of the tokens),
+    again with the forward as three separate kernels, again with the fused
+    backward switched on, again with the row-major (scatter-add) products
+    only, again with the token-major products wherever they apply, and again
+    with the CUDA-core kernels forced."""
     monkeypatch.delenv("MOSA_FORCE_SIMT", raising=False)
     monkeypatch.delenv("MOSA_FUSED_FWD", raising=False)
     monkeypatch.delenv("MOSA_FUSED_BWD", raising=False)
-    if request.param == "simt":
+    monkeypatch.delenv("MOSA_HEADSUM", raising=False)
+    if request.param == "rowmajor":
+        monkeypatch.setenv("MOSA_HEADSUM", "0")
+    elif request.param == "tokenmajor":
+        monkeypatch.setenv("MOSA_HEADSUM", "1")
+    elif request.param == "simt":
         monkeypatch.setenv("MOSA_FORCE_SIMT", "1")
     elif request.param == "unfused":
         monkeypatch.setenv("MOSA_FUSED_FWD", "0")
@@ -467,3 +475,21 @@ def test_router_wait_limit_gives_up_then_next_call_is_exact(monkeypatch):
     assert_close("r_full", rfg.cpu().numpy(), rf, cfg.dtype)
     assert_close("r_sel", rsg.cpu().numpy(), rs, cfg.dtype)
     assert_close("Y", Yg.cpu().numpy(), Y, cfg.dtype)
+
+
+def test_token_major_products_equal_row_major_at_full_size(monkeypatch):
+    # B4 T4096 d1024 H8 k2048, every head keeping half the tokens: Y and dX
+    # from the token-major products (each head's rows of a token tile summed
+    # in TMEM, written once) and from the row-major products (each head's rows
+    # scatter-added) are the same sums in another order.
+    cfg = W.CONFIGS["B4_T4096_d1024_H8_k2048"]
+    x = W.make_inputs(cfg)
+    monkeypatch.setenv("MOSA_HEADSUM", "1")
+    a = run_layer(cfg, x)
+    monkeypatch.setenv("MOSA_HEADSUM", "0")
+    b = run_layer(cfg, x)
+    np.testing.assert_array_equal(a["I"], b["I"])
+    from _util import rel_l2
+    for n in ("Y", "dX"):
+        assert rel_l2(a[n], b[n]) < 1e-5, n
+        assert np.abs(a[n] - b[n]).max() < 1e-4, n

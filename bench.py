@@ -554,6 +554,28 @@ def main():
     total_ms = sum(s.elapsed_time(e) for s, e in zip(starts, ends))
     value, total_ms = combine_ranks(total_ms, cfg.B * cfg.T * K, dist, dev)
 
+    # Diagnostic: the stage timeline of one step (kernel spans stamped by the
+    # kernels, no events between them; outside the timed region), the median
+    # step of a few, each after an L2 flush.
+    timeline = None
+    if not hybrid:
+        mosa.mosa_profile_timeline(True)
+        try:
+            tls = []
+            for _ in range(5):
+                flush_buf.zero_()
+                step()
+                tls.append(mosa.mosa_profile_timeline_read(shape, ws))
+        finally:
+            mosa.mosa_profile_timeline(False)
+        tls.sort(key=lambda t: max(v[1] for v in t.values()))
+        mid = tls[len(tls) // 2]
+        timeline = {"what": "first CTA start and last CTA end of each stage's kernels in one "
+                            "step (the median of 5, after an L2 flush), microseconds from the "
+                            "step's first kernel start; no events between the kernels",
+                    "us": {k: [round(a, 1), round(b, 1)] for k, (a, b) in
+                           sorted(mid.items(), key=lambda kv: kv[1][0])}}
+
     # Diagnostic: the same step replayed from a CUDA graph captured by torch
     # around the eager calls (the library's own graph cache switched off).
     graph_ms = None
@@ -705,6 +727,7 @@ def main():
                         "(two device buffer sets)"},
         "gpu_launches": int(launches),
         "graph_ms_per_step": graph_ms,
+        "timeline": timeline,
         "clocks": clocks,
     }
     if world == 1 and not args.no_cpu_baseline:

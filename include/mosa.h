@@ -293,6 +293,23 @@ int32_t mosa_profile_read(double *total_ms, int32_t *count, int32_t max_stages);
  * Returns the number of entries written. */
 int32_t mosa_profile_spans(const mosa_shape *shape, void *workspace, double *ms, int32_t max_stages);
 
+/* Timeline mode (on = 1, off = 0): later layer calls record, for every stage,
+ * the first CTA start and last CTA end of its kernels (%globaltimer) into the
+ * workspace, with no CUDA events and no per-stage resets between the kernels
+ * (which would break the early-launch chain the timing is meant to show);
+ * each call instead starts with one small kernel that clears its stages'
+ * slots.  Read with mosa_profile_timeline_read.  MOSA_OK, or
+ * MOSA_ERR_INVALID_ARG for another value of on. */
+mosa_status mosa_profile_timeline(int32_t on);
+
+/* The timeline left in the workspace by the last forward and backward calls
+ * with it: start_us[i] and end_us[i] (arrays of max_stages entries) in
+ * microseconds from the earliest recorded start, -1 for a stage with no
+ * record.  Waits for the device.  Returns the number of entries written, 0 on
+ * an invalid shape or pointer or a CUDA error. */
+int32_t mosa_profile_timeline_read(const mosa_shape *shape, void *workspace, double *start_us,
+                                   double *end_us, int32_t max_stages);
+
 /* Name of a stage ("router", "select", ...; "unknown" if out of range). */
 const char *mosa_stage_name(int32_t stage);
 

@@ -29,7 +29,7 @@ EXPORTED = ("mosa_status_string", "mosa_workspace_bytes", "mosa_forward",
             "mosa_kernel_launches", "mosa_profile_stages", "mosa_profile_read",
             "mosa_stage_name", "mosa_stage_engine", "mosa_route_noalloc", "mosa_adaptive_k",
             "mosa_hybrid_workspace_bytes", "mosa_hybrid_forward", "mosa_hybrid_backward",
-            "mosa_profile_spans")
+            "mosa_profile_spans", "mosa_profile_timeline", "mosa_profile_timeline_read")
 
 
 class MosaShape(ctypes.Structure):
@@ -102,6 +102,11 @@ def load(build_if_missing: bool = True) -> ctypes.CDLL:
         L.mosa_profile_read.restype = i32
         L.mosa_profile_spans.argtypes = [sp, vp, ctypes.POINTER(ctypes.c_double), i32]
         L.mosa_profile_spans.restype = i32
+        L.mosa_profile_timeline.argtypes = [i32]
+        L.mosa_profile_timeline.restype = ctypes.c_int
+        L.mosa_profile_timeline_read.argtypes = [sp, vp, ctypes.POINTER(ctypes.c_double),
+                                                 ctypes.POINTER(ctypes.c_double), i32]
+        L.mosa_profile_timeline_read.restype = i32
         L.mosa_stage_name.argtypes = [i32]
         L.mosa_stage_name.restype = ctypes.c_char_p
         L.mosa_route_noalloc.argtypes = [sp, vp, vp, vp, vp, vp]
@@ -371,6 +376,25 @@ def mosa_profile_spans(shape: MosaShape, workspace) -> dict:
     ms = (ctypes.c_double * n)()
     m = L.mosa_profile_spans(ctypes.byref(shape), ctypes.c_void_p(workspace.data_ptr()), ms, n)
     return {mosa_stage_name(i): ms[i] for i in range(min(m, n))}
+
+
+def mosa_profile_timeline(on: bool) -> None:
+    """Timeline mode: later layer calls record every stage's kernel span
+    (first CTA start, last CTA end) without per-stage events or resets."""
+    _check(load().mosa_profile_timeline(1 if on else 0), "mosa_profile_timeline")
+
+
+def mosa_profile_timeline_read(shape: MosaShape, workspace) -> dict:
+    """{stage name: (start us, end us)} of the last forward and backward calls
+    with ``workspace`` in timeline mode, from the earliest recorded start;
+    stages without a record are left out.  Waits for the device."""
+    L = load()
+    n = 16
+    a = (ctypes.c_double * n)()
+    b = (ctypes.c_double * n)()
+    m = L.mosa_profile_timeline_read(ctypes.byref(shape), ctypes.c_void_p(workspace.data_ptr()),
+                                     a, b, n)
+    return {mosa_stage_name(i): (a[i], b[i]) for i in range(min(m, n)) if a[i] >= 0}
 
 
 _ENGINES = {0: "simt", 1: "tensor", 2: "mem"}

@@ -236,8 +236,8 @@ cudaError_t launch_attn_fwd(const Dims &dm, const Saved &sv, cudaStream_t s) {
     return dm.bf16 ? attn_fwd_dispatch<SplitBF16>(dm, sv, s) : attn_fwd_dispatch<float>(dm, sv, s);
 }
 
-cudaError_t launch_attn_bwd(const Dims &dm, const Saved &sv, cudaStream_t s) {
-    if (use_tc(dm)) return tc_attn_bwd(dm, sv, s);
+cudaError_t launch_attn_bwd(const Dims &dm, const Saved &sv, cudaStream_t s, float *zero_out) {
+    if (use_tc(dm)) return tc_attn_bwd(dm, sv, s, zero_out);
     return dm.bf16 ? attn_bwd_dispatch<SplitBF16>(dm, sv, s) : attn_bwd_dispatch<float>(dm, sv, s);
 }
 

@@ -110,7 +110,8 @@ cudaError_t launch_out_bwd(const Dims &dm, const void *Wo, const void *dY, const
                            float *dWo, cudaStream_t stream);
 
 // B2: dQ, dK, dV from dA (flash-style recomputation of P).
-cudaError_t launch_attn_bwd(const Dims &dm, const Saved &sv, cudaStream_t stream);
+cudaError_t launch_attn_bwd(const Dims &dm, const Saved &sv, cudaStream_t stream,
+                            float *zero_out = nullptr);
 
 // B3: dX = 0; dX[b, I, :] += dQ W_q^T + dK W_k^T + dV W_v^T + dlogit W_r[:,h]^T.
 cudaError_t launch_in_bwd(const Dims &dm, const void *Wq, const void *Wk, const void *Wv,
@@ -185,7 +186,14 @@ cudaError_t tc_transpose_wr(const Dims &dm, const void *Wr, const Saved &sv, cud
 cudaError_t tc_attn_fwd(const Dims &dm, const Saved &sv, cudaStream_t s);
 // For k > 128 the attention backward reduce-adds dQ into the fp32
 // accumulator sv.G, whose rows the G kernel (tc_out_bwd_g) zeroes first.
-cudaError_t tc_attn_bwd(const Dims &dm, const Saved &sv, cudaStream_t s);
+// zero_out (k > 128 only, 16-byte aligned; else nullptr): the layer's dX
+// [B*T, d] fp32, zeroed by the kernel beside the attention (see
+// attn_bwd_zeroes_dx).
+cudaError_t tc_attn_bwd(const Dims &dm, const Saved &sv, cudaStream_t s, float *zero_out = nullptr);
+// True when tc_attn_bwd can take over zeroing dX (the fp16 path, k > 128).
+inline bool attn_bwd_zeroes_dx(const Dims &dm, const void *dX) {
+    return attn_f16(dm) && dX != nullptr && ((uintptr_t)dX % 16) == 0;
+}
 cudaError_t tc_w_bwd(const Dims &dm, const void *X, const Saved &sv, float *dWq, float *dWk,
                      float *dWv, float *dWr, cudaStream_t s);
 

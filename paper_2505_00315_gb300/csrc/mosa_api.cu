@@ -89,6 +89,13 @@ mosa_status check_workspace(const Dims &dm, void *ws, size_t bytes, Saved *sv) {
 
 mosa_status cuda_status(cudaError_t e) { return e == cudaSuccess ? MOSA_OK : MOSA_ERR_CUDA; }
 
+// Stages of a forward call and of a backward call (timeline slot resets).
+constexpr uint32_t kForwardStages = (1u << kStageRouter) | (1u << kStageSelect) | (1u << kStageQkv) |
+                                    (1u << kStageAttnFwd) | (1u << kStageOut) | (1u << kStageFwdUnit);
+constexpr uint32_t kBackwardStages = (1u << kStageOutBwd) | (1u << kStageAttnBwd) |
+                                     (1u << kStageInBwd) | (1u << kStageWBwd) | (1u << kStageDwo) |
+                                     (1u << kStageBwdUnit);
+
 #define MOSA_TRY(expr)                                  \
     do {                                                \
         cudaError_t _e = (expr);                        \
@@ -98,9 +105,11 @@ mosa_status cuda_status(cudaError_t e) { return e == cudaSuccess ? MOSA_OK : MOS
 // ------------------------------------------------ concurrent branches
 // On the tensor-core path independent kernels run on a second, internal
 // stream joined back with events (graph branches when captured):
-//   forward:  zeroing Y runs beside TopK (forked after the router, joined
+//   forward:  zeroing Y and (fp16 attention path) the fp16 copies of X and
+//             W_q|W_k|W_v run beside TopK (forked after the router, joined
 //             before the output product);
-//   backward: dW_o, the W_r transpose and the zeroing of dX run beside
+//   backward: dW_o, the W_r transpose and (except on the fp16 path, where
+//             the attention backward does it) the zeroing of dX run beside
 //             G -> attention backward; then dX and dW run side by side.
 // A hybrid call runs the MoSA heads and then the dense heads, each this way.
 struct DevResources {
@@ -178,6 +187,7 @@ mosa_status forward_tc(const Dims &dm, const void *X, const void *W_r, const voi
                        float *r_sel, float *rf, bool route, const int32_t *I_in,
                        const float *rsel_in, const Saved &sv, cudaStream_t s, DevResources &r) {
     set_span_base(sv.spans);   // measurement: this call's kernel-span slots
+    MOSA_TRY(begin_timeline_call(kForwardStages, s));
     // A call that adds into Y continues the status word of the call that wrote it.
     if (!dm.accumulate) MOSA_TRY(cudaMemsetAsync(sv.status, 0, sizeof(uint32_t), s));
     const size_t ny = (size_t)dm.B * dm.T * dm.d;
@@ -189,6 +199,10 @@ mosa_status forward_tc(const Dims &dm, const void *X, const void *W_r, const voi
     // (the token-major output product writes every element of Y itself)
     const bool headsum = !use_fused_forward(dm) && use_headsum_out(dm);
     if (!dm.accumulate && !headsum) MOSA_TRY(cudaMemsetAsync(Y, 0, sizeof(float) * ny, r.side));
+    // fp16 attention path: the fp16 copies of X and W_q|W_k|W_v that the
+    // backward's products with dQ|dK|dV read, made here beside TopK, whose
+    // grid (one CTA per (b, h) row) leaves most SMs idle
+    if (attn_f16(dm)) MOSA_TRY(tc_f16_copies(dm, X, W_q, W_k, W_v, sv, r.side));
     if (route) {
         StageScope st_(kStageSelect, s);
         MOSA_TRY(launch_select(dm.B * dm.H, dm.T, dm.k, rf, I, r_sel, dm.B, dm.H, sv.gidx,
@@ -230,14 +244,16 @@ mosa_status forward_tc(const Dims &dm, const void *X, const void *W_r, const voi
 }
 
 // Tensor-core backward.  Main stream: G and the row terms, the attention
-// backward, then dX.  Side stream: dW_o beside G, the W_r transpose and the
-// zeroing of dX, then dW once dQ|dK|dV|dlogit exist; the main stream waits
-// for the side stream only before dX and at the final join.
+// backward (zeroing dX on the fp16 path), then dX.  Side stream: dW_o beside
+// G, the W_r transpose and otherwise the zeroing of dX, then dW once
+// dQ|dK|dV|dlogit exist; the main stream waits for the side stream only
+// before dX and at the final join.
 mosa_status backward_tc(const Dims &dm, const void *X, const void *W_r, const void *W_q,
                         const void *W_k, const void *W_v, const void *W_o, const void *dY,
                         float *dX, float *dW_r, float *dW_q, float *dW_k, float *dW_v,
                         float *dW_o, const Saved &sv, cudaStream_t s, DevResources &r) {
     set_span_base(sv.spans);   // measurement: this call's kernel-span slots
+    MOSA_TRY(begin_timeline_call(kBackwardStages, s));   // before the side stream forks
     cudaStream_t t = r.side;
     const size_t nx = (size_t)dm.B * dm.T * dm.d;
     MOSA_TRY(link(s, t, r.ev[0]));
@@ -269,28 +285,32 @@ mosa_status backward_tc(const Dims &dm, const void *X, const void *W_r, const vo
         MOSA_TRY(link(t, s, r.ev[3]));  // join
         return MOSA_OK;
     }
-    // fp16 attention path: fp16 copies of X and W_q|W_k|W_v for the products
-    // with the fp16 dQ|dK|dV (beside G, which leaves room on every SM)
-    if (attn_f16(dm)) MOSA_TRY(tc_f16_copies(dm, X, W_q, W_k, W_v, sv, t));
+    // (the fp16 attention path's copies of X and W_q|W_k|W_v were made by the forward)
+    MOSA_TRY(tc_transpose_wr(dm, W_r, sv, t));
+    // The token-major dX product writes every element of dX itself, from the
+    // token-to-row map sv.pos that the forward built (use_headsum_dx implies
+    // use_headsum_out); the token-major G reads that map too, so nothing
+    // rewrites it here.
+    const bool headsum = use_headsum_dx(dm);
+    // dX starts at zero for the scatter-add product: on the fp16 path the
+    // attention backward's idle warps zero it (a 67 MB memset on the side
+    // stream found no free SM until that kernel's tail and delayed dX)
+    const bool zero_in_attn = !headsum && !dm.accumulate && attn_bwd_zeroes_dx(dm, dX);
+    if (!headsum && !dm.accumulate && !zero_in_attn)
+        MOSA_TRY(cudaMemsetAsync(dX, 0, sizeof(float) * nx, t));
+    MOSA_TRY(cudaEventRecord(r.ev[1], t));  // dX zeroed (unless by the attention backward), W_r transposed
     {
+        // dW_o after the event dX waits for, so that dX does not wait for it
         StageScope st_(kStageDwo, t);
         MOSA_TRY(tc_out_bwd_w(dm, dY, sv, dW_o, t));
     }
-    MOSA_TRY(tc_transpose_wr(dm, W_r, sv, t));
-    // (the token-major dX product writes every element of dX itself, from the row map)
-    const bool headsum = use_headsum_dx(dm);
-    if (headsum)
-        MOSA_TRY(tc_token_rows(dm, sv, t));
-    else if (!dm.accumulate)
-        MOSA_TRY(cudaMemsetAsync(dX, 0, sizeof(float) * nx, t));
-    MOSA_TRY(cudaEventRecord(r.ev[1], t));  // dX zeroed or the row map built, W_r transposed
     {
         StageScope st_(kStageOutBwd, s);
         MOSA_TRY(tc_out_bwd_g(dm, W_o, dY, sv, s));
     }
     {
         StageScope st_(kStageAttnBwd, s);
-        MOSA_TRY(launch_attn_bwd(dm, sv, s));
+        MOSA_TRY(launch_attn_bwd(dm, sv, s, zero_in_attn ? dX : nullptr));
         // (the fp16 path turns dQ and dK back before rounding them)
         if (dm.rope && !attn_f16(dm)) MOSA_TRY(rope_qk(dm, sv, true, s));
     }
@@ -299,10 +319,10 @@ mosa_status backward_tc(const Dims &dm, const void *X, const void *W_r, const vo
         StageScope st_(kStageWBwd, t);
         MOSA_TRY(tc_w_bwd(dm, X, sv, dW_q, dW_k, dW_v, dW_r, t));
     }
-    MOSA_TRY(cudaStreamWaitEvent(s, r.ev[1], 0));  // dX zeroed or the row map built, W_r transposed
+    MOSA_TRY(cudaStreamWaitEvent(s, r.ev[1], 0));  // W_r transposed (and dX zeroed on the side)
     {
         StageScope st_(kStageInBwd, s);
-        MOSA_TRY(tc_in_bwd(dm, W_q, W_k, W_v, W_r, sv, dX, s, false, headsum));
+        MOSA_TRY(tc_in_bwd(dm, W_q, W_k, W_v, W_r, sv, dX, s, false, /*pos_ready=*/true));
     }
     MOSA_TRY(link(t, s, r.ev[3]));  // join
     return MOSA_OK;
@@ -320,6 +340,7 @@ mosa_status forward_routed(const Dims &dm, const void *X, const void *W_r, const
     if (res != nullptr)
         return forward_tc(dm, X, W_r, W_q, W_k, W_v, W_o, Y, I, r_sel, rf, true, nullptr, nullptr,
                           sv, s, *res);
+    MOSA_TRY(begin_timeline_call(kForwardStages, s));
     MOSA_TRY(cudaMemsetAsync(sv.status, 0, sizeof(uint32_t), s));
     {
         StageScope st_(kStageRouter, s);
@@ -343,6 +364,7 @@ mosa_status forward_given(const Dims &dm, const void *X, const void *W_q, const 
     if (res != nullptr)
         return forward_tc(dm, X, nullptr, W_q, W_k, W_v, W_o, Y, nullptr, nullptr, nullptr, false,
                           I, r_sel, sv, s, *res);
+    MOSA_TRY(begin_timeline_call(kForwardStages, s));
     if (!dm.accumulate) MOSA_TRY(cudaMemsetAsync(sv.status, 0, sizeof(uint32_t), s));
     {
         StageScope st_(kStageSelect, s);
@@ -363,6 +385,7 @@ mosa_status backward_all(const Dims &dm, const void *X, const void *W_r, const v
     if (res != nullptr)
         return backward_tc(dm, X, W_r, W_q, W_k, W_v, W_o, dY, dX, dW_r, dW_q, dW_k, dW_v, dW_o,
                            sv, s, *res);
+    MOSA_TRY(begin_timeline_call(kBackwardStages, s));
     {
         StageScope st_(kStageOutBwd, s);
         MOSA_TRY(launch_out_bwd(dm, W_o, dY, sv, dW_o, s));
@@ -780,6 +803,32 @@ int32_t mosa_profile_spans(const mosa_shape *shape, void *workspace, double *ms,
     for (int i = 0; i < n; ++i) {
         const unsigned long long a = h[2 * i], b = h[2 * i + 1];
         ms[i] = (a != ~0ull && b != 0ull && b >= a) ? (double)(b - a) * 1e-6 : -1.0;
+    }
+    return n;
+}
+
+int32_t mosa_profile_timeline_read(const mosa_shape *shape, void *workspace, double *start_us,
+                                   double *end_us, int32_t max_stages) {
+    Dims dm;
+    if (check_shape(shape, &dm) != MOSA_OK || workspace == nullptr || start_us == nullptr ||
+        end_us == nullptr)
+        return 0;
+    Saved sv;
+    carve(dm, (char *)workspace, &sv);
+    unsigned long long h[2 * 16];
+    if (cudaDeviceSynchronize() != cudaSuccess ||
+        cudaMemcpy(h, sv.spans, sizeof(h), cudaMemcpyDeviceToHost) != cudaSuccess)
+        return 0;
+    unsigned long long t0 = ~0ull;
+    for (int i = 0; i < kNumStages; ++i)
+        if (h[2 * i] != ~0ull && h[2 * i + 1] != 0ull && h[2 * i + 1] >= h[2 * i] && h[2 * i] < t0)
+            t0 = h[2 * i];
+    const int n = max_stages < kNumStages ? max_stages : kNumStages;
+    for (int i = 0; i < n; ++i) {
+        const unsigned long long a = h[2 * i], b = h[2 * i + 1];
+        const bool ok = a != ~0ull && b != 0ull && b >= a && t0 != ~0ull;
+        start_us[i] = ok ? (double)(a - t0) * 1e-3 : -1.0;
+        end_us[i] = ok ? (double)(b - t0) * 1e-3 : -1.0;
     }
     return n;
 }

@@ -13,6 +13,7 @@ namespace {
 
 std::atomic<unsigned long long> g_launches{0};
 std::atomic<uint32_t> g_mask{0};
+std::atomic<bool> g_timeline{false};
 std::mutex g_mu;
 
 struct Pending {
@@ -44,7 +45,25 @@ cudaEvent_t take_event() {
     return e;
 }
 
+// start = all ones (atomicMin target), end = 0 (atomicMax target)
+__global__ void reset_spans_kernel(unsigned long long *slots, uint32_t stages) {
+    const int i = threadIdx.x;
+    if (i < 16 && ((stages >> i) & 1u)) {
+        slots[2 * i] = ~0ull;
+        slots[2 * i + 1] = 0ull;
+    }
+}
+
 }  // namespace
+
+bool timeline_on() { return g_timeline.load(std::memory_order_relaxed); }
+
+cudaError_t begin_timeline_call(uint32_t stages, cudaStream_t s) {
+    if (!timeline_on() || t_span_base == nullptr) return cudaSuccess;
+    reset_spans_kernel<<<1, 32, 0, s>>>(t_span_base, stages);
+    note_launches(1);
+    return cudaGetLastError();
+}
 
 void note_launches(int n) {
     if (t_capture != nullptr) {
@@ -56,7 +75,9 @@ void note_launches(int n) {
 
 void capture_into(CaptureRecord *rec) { t_capture = rec; }
 
-uint32_t profile_mask() { return g_mask.load(std::memory_order_relaxed); }
+uint32_t profile_mask() {
+    return g_mask.load(std::memory_order_relaxed) | (timeline_on() ? 0x80000000u : 0u);
+}
 
 void replayed(const CaptureRecord &rec) {
     g_launches.fetch_add(rec.launches, std::memory_order_relaxed);
@@ -70,7 +91,11 @@ unsigned long long *active_span() { return t_active_span; }
 
 StageScope::StageScope(int stage, cudaStream_t s) : stage_(stage), stream_(s) {
     prev_span_ = t_active_span;
-    if (!(g_mask.load(std::memory_order_relaxed) & (1u << stage))) return;
+    if (!(g_mask.load(std::memory_order_relaxed) & (1u << stage))) {
+        // timeline mode: the call cleared this stage's slot at its start
+        if (timeline_on() && t_span_base != nullptr) t_active_span = t_span_base + 2 * stage;
+        return;
+    }
     if (t_span_base != nullptr) {
         // reset this stage's span slot (start = max, end = 0) ahead of its kernels
         unsigned long long *slot = t_span_base + 2 * stage;
@@ -118,6 +143,12 @@ unsigned long long mosa_kernel_launches(void) { return g_launches.load(); }
 
 mosa_status mosa_profile_stages(uint32_t stage_mask) {
     g_mask.store(stage_mask & ((1u << kNumStages) - 1u));
+    return MOSA_OK;
+}
+
+mosa_status mosa_profile_timeline(int32_t on) {
+    if (on != 0 && on != 1) return MOSA_ERR_INVALID_ARG;
+    g_timeline.store(on != 0);
     return MOSA_OK;
 }
 

@@ -36,6 +36,14 @@ void replayed(const CaptureRecord &rec);
 // Stage-timing mask currently in force.
 uint32_t profile_mask();
 
+// Timeline mode (mosa_profile_timeline): every stage records its kernel span
+// without CUDA events or per-stage slot resets; each layer call clears its
+// stages' slots once, at its start, with begin_timeline_call.
+bool timeline_on();
+// Clears the span slots of the stages in `stages` (bit mask) on stream s when
+// timeline mode is on (launches one small kernel); otherwise does nothing.
+cudaError_t begin_timeline_call(uint32_t stages, cudaStream_t s);
+
 // Kernel spans: the layer call names its workspace's span slots ([stage][2]);
 // while a timed stage is open, active_span() is its slot (else nullptr) and
 // the launchers pass it to their kernels.

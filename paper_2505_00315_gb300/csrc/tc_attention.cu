@@ -360,6 +360,11 @@ struct BwdParams {
     int rope, T;
     RopeTable rope_tab;
     unsigned long long *span; // measurement: kernel span slot, or null
+    // k > 128: an fp32 array of zero_n4 float4 (the layer's dX, which the
+    // input-gradient product then adds into) that the otherwise idle warp 3
+    // of every CTA zeroes, one slice per CTA, while the attention runs
+    float4 *zero;
+    long long zero_n4;
 };
 
 template <class SM>
@@ -569,6 +574,17 @@ __global__ void __launch_bounds__(kBT, 1) attn_bwd_tc_kernel(const __grid_consta
             // acc_done's only phase covers every MMA issued: wait for it here too
             // (the workers' own wait gives up at once when the CTA is aborting)
             drain_mmas(smem_u32(&sm.acc_done));
+        }
+    } else if (warp == 3) {
+        // this CTA's slice of the array to zero (after pdl_wait above: the
+        // kernels before this one are complete)
+        if (p.zero != nullptr) {
+            const long long ncta = (long long)gridDim.x * gridDim.y * gridDim.z;
+            const long long cta = ((long long)blockIdx.z * gridDim.y + blockIdx.y) * gridDim.x + blockIdx.x;
+            const long long per = (p.zero_n4 + ncta - 1) / ncta;
+            const long long a = cta * per, e = min(p.zero_n4, a + per);
+            const float4 z = make_float4(0.f, 0.f, 0.f, 0.f);
+            for (long long i = a + lane; i < e; i += 32) p.zero[i] = z;
         }
     } else if (warp >= 4) {
         pdl_trigger();
@@ -1156,7 +1172,7 @@ cudaError_t tc_attn_fwd(const Dims &dm, const Saved &sv, cudaStream_t s) {
     return e;
 }
 
-cudaError_t tc_attn_bwd(const Dims &dm, const Saved &sv, cudaStream_t s) {
+cudaError_t tc_attn_bwd(const Dims &dm, const Saved &sv, cudaStream_t s, float *zero_out) {
     BwdParams kv, dq;
     memset(&kv, 0, sizeof(kv));
     memset(&dq, 0, sizeof(dq));
@@ -1212,6 +1228,10 @@ cudaError_t tc_attn_bwd(const Dims &dm, const Saved &sv, cudaStream_t s) {
     bp.T = dm.T;
     bp.rope = dm.rope ? 1 : 0;
     if (dm.rope) bp.rope_tab = make_rope_table(dm.hp, dm.T);
+    if (zero_out != nullptr) {
+        bp.zero = reinterpret_cast<float4 *>(zero_out);
+        bp.zero_n4 = (long long)dm.B * dm.T * dm.d / 4;
+    }
     {
         // dQ accumulator [H, B, k, 64] fp32 (the workspace's G buffer)
         const uint64_t dims[4] = {64, (uint64_t)dm.k, (uint64_t)dm.B, (uint64_t)dm.H};

@@ -239,6 +239,38 @@ __device__ __forceinline__ float stage_f16_vals64(uint8_t *xb, const float (&v)[
     return mx;
 }
 
+// The warp's 32 256-byte bf16 pair rows of AR into the staging buffer (unit u
+// of row rl at xoff256(rl, u)), 16 lanes per row so that every load
+// instruction reads two whole rows, all sixteen loads in flight before the
+// first store; src_row(rl) gives the source row or nullptr to leave that
+// staging row unwritten.  Each lane then reads its own row back with
+// ld_staged_pair.  (One lane per row, each load instruction touched 32 rows.)
+template <typename F>
+__device__ __forceinline__ void load_rows256(uint8_t *xb, int lane, F src_row) {
+    const int u = lane & 15;
+    uint4 v[16];
+#pragma unroll
+    for (int i = 0; i < 16; ++i) {
+        const uint4 *src = src_row((lane >> 4) + 2 * i);
+        v[i] = src != nullptr ? src[u] : make_uint4(0u, 0u, 0u, 0u);
+    }
+#pragma unroll
+    for (int i = 0; i < 16; ++i)
+        *reinterpret_cast<uint4 *>(xb + xoff256((lane >> 4) + 2 * i, u)) = v[i];
+    __syncwarp();
+}
+
+// This lane's staged pair row: hi units 0..7, lo units 8..15 (zeros if !live).
+__device__ __forceinline__ void ld_staged_pair(const uint8_t *xb, int lane, bool live, uint4 (&ah)[8],
+                                               uint4 (&al)[8]) {
+#pragma unroll
+    for (int u = 0; u < 8; ++u) {
+        ah[u] = live ? *reinterpret_cast<const uint4 *>(xb + xoff256(lane, u)) : make_uint4(0u, 0u, 0u, 0u);
+        al[u] = live ? *reinterpret_cast<const uint4 *>(xb + xoff256(lane, 8 + u)) : make_uint4(0u, 0u, 0u, 0u);
+    }
+    __syncwarp();
+}
+
 // Copies staged rows 0 .. nrows-1 to global memory with 16 lanes per row, so
 // every store instruction writes two whole 256-byte rows; addr(rl, u) gives
 // the destination of unit u of row rl.
@@ -618,17 +650,23 @@ __global__ void __launch_bounds__(kThreads, Cfg<KIND>::MIN_CTAS)
             const bool live = mg < p.M;
             const size_t row = (size_t)h * p.Mtok + (live ? mg : 0);
             const float rr = live ? p.rsel[row] : 0.f;
-            const uint4 *arow = reinterpret_cast<const uint4 *>(p.ARp + row * 128);  // hi 0..7, lo 8..15
-            const uint4 z4 = make_uint4(0u, 0u, 0u, 0u);
+            // the warp's 32 AR pair rows (one contiguous block), two rows per load instruction
+            {
+                const size_t arow0 = (size_t)h * p.Mtok + m0 + q * 32;
+                load_rows256(xb, lane, [&](int rl) -> const uint4 * {
+                    return m0 + q * 32 + rl < p.M ? reinterpret_cast<const uint4 *>(p.ARp + (arow0 + rl) * 128)
+                                                  : nullptr;
+                });
+            }
+            uint4 ah[8], al[8];
+            ld_staged_pair(xb, lane, live, ah, al);
             float dd = 0.f, amax = 0.f;
 #pragma unroll
             for (int hlf = 0; hlf < 2; ++hlf) {
                 float g[32];
                 tmem_ld32(tb + 32 * hlf, g);
 #pragma unroll
-                for (int u = 0; u < 4; ++u)
-                    dd = dot_pair8(live ? arow[4 * hlf + u] : z4, live ? arow[8 + 4 * hlf + u] : z4,
-                                   g + 8 * u, dd);
+                for (int u = 0; u < 4; ++u) dd = dot_pair8(ah[4 * hlf + u], al[4 * hlf + u], g + 8 * u, dd);
 #pragma unroll
                 for (int e = 0; e < 32; ++e) g[e] *= rr;  // dA = r G
                 if (!p.half) {

@@ -177,3 +177,17 @@ def test_hybrid_entries_reject_before_launch():
             B.MOSA_ERR_INVALID_ARG, i
     assert L.mosa_hybrid_backward(ctypes.byref(hshape()), *bwd, None, 1 << 40, None) == \
         B.MOSA_ERR_WORKSPACE
+
+
+def test_timeline_mode_switch_validates_its_argument():
+    lib = B.load()
+    assert lib.mosa_profile_timeline(2) == B.MOSA_ERR_INVALID_ARG
+    assert lib.mosa_profile_timeline(-1) == B.MOSA_ERR_INVALID_ARG
+    assert lib.mosa_profile_timeline(1) == B.MOSA_OK
+    assert lib.mosa_profile_timeline(0) == B.MOSA_OK
+    start = (ctypes.c_double * 16)()
+    end = (ctypes.c_double * 16)()
+    s = shape()
+    # invalid pointers are rejected before any CUDA call
+    assert lib.mosa_profile_timeline_read(ctypes.byref(s), None, start, end, 16) == 0
+    assert lib.mosa_profile_timeline_read(None, FAKE, start, end, 16) == 0

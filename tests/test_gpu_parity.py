@@ -442,6 +442,44 @@ def test_stage_kernel_spans_inside_event_windows(name):
         assert 0.0 < spans[s] <= events[s][0] + 0.02, (s, spans[s], events[s])
 
 
+@pytest.mark.parametrize("name", ["largek_bf16", "pack2_oddB_bf16"])
+def test_timeline_mode_orders_the_stages_and_leaves_results_unchanged(name):
+    # Timeline mode stamps every stage's kernel span with no events between
+    # the kernels: each stage on the caller's stream starts after the one
+    # before it ends (the early-launch wait holds its CTAs until then), every
+    # tensor-core stage has a record, and the results are those of a plain run.
+    cfg = next(c for c in SMALL if c.name == name)
+    x = W.make_inputs(cfg)
+    plain = run_layer(cfg, x)
+    dt = cfg.dtype
+    X, Wr, Wq, Wk, Wv, Wo = (to_dev(x[n], dt) for n in ("X", "Wr", "Wq", "Wk", "Wv", "Wo"))
+    dY = to_dev(x["dY"], dt)
+    shape = mosa.make_shape(X, Wq, cfg.k)
+    impl = mosa.stage_impl(shape)
+    mosa.mosa_profile_timeline(True)
+    try:
+        Y, I, rs, _, ws = mosa.mosa_forward(X, Wr, Wq, Wk, Wv, Wo, cfg.k)
+        g = mosa.mosa_backward(X, Wr, Wq, Wk, Wv, Wo, I, rs, dY, ws)
+        torch.cuda.synchronize()
+        tl = mosa.mosa_profile_timeline_read(shape, ws)
+    finally:
+        mosa.mosa_profile_timeline(False)
+    assert mosa.mosa_check_status(shape, ws) == 0
+    np.testing.assert_array_equal(I.cpu().numpy(), plain["I"])
+    np.testing.assert_allclose(Y.float().cpu().numpy(), plain["Y"], rtol=1e-5, atol=1e-6)
+    np.testing.assert_allclose(g["dX"].float().cpu().numpy(), plain["dX"], rtol=1e-5, atol=1e-6)
+    fwd = ["fwd_unit"] if cfg.k <= 128 else ["qkv", "attn_fwd", "out"]
+    for s in fwd + ["select", "out_bwd", "attn_bwd", "in_bwd", "w_bwd", "dwo"]:
+        assert s in tl, (s, tl)
+    if impl.get("router") == "tensor":
+        assert "router" in tl, tl
+    main = [s for s in ("router", "select", "qkv", "attn_fwd", "out", "fwd_unit", "out_bwd",
+                        "attn_bwd", "in_bwd") if s in tl]
+    for a, b in zip(main, main[1:]):
+        assert tl[b][0] >= tl[a][1] - 0.5, (a, b, tl)
+    assert min(v[0] for v in tl.values()) == 0.0
+
+
 def test_router_wait_limit_gives_up_then_next_call_is_exact(monkeypatch):
     # The router GEMM's main-loop waits get a 1 us limit: its epilogue waits
     # for the whole 128-block K loop (d = 8192), gives up, stops the producer

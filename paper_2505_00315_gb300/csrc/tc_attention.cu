@@ -67,16 +67,23 @@ struct AttnParams {
 //   when the block's maximum exceeds it by more than 2^8 (O and l are then
 //   rescaled in place; otherwise P may reach 2^8, well inside the fp16 range,
 //   and the final O / l uses the same m throughout), written as fp16 into
-//   shared-memory tile j % 2;
-//   O += P_j V_j with both operands in shared memory, O in TMEM.
+//   TMEM buffer j % 2 (two fp16 per 32-bit column, 64 columns);
+//   O += P_j V_j with P read from TMEM as the A operand and V from shared
+//   memory, O in TMEM.
+// P in TMEM takes the shared-memory stores and the proxy fence of P off the
+// softmax warps' chain (47.7 -> 44.6 us at B4 T4096 d1024 H8 k2048); the
+// MMAs themselves cost the same either way (measured with %clock stamps:
+// about 120 cycles per M = 128, N = 64, K = 16 instruction and 165 at
+// N = 128, also when independent accumulators alternate, so the tensor pipe
+// runs these small instructions one after another at a fixed cost each).
+// Earlier builds found that a tcgen05.st issued while an MMA reads its A
+// operand from TMEM corrupts that MMA even when the columns differ, so the
+// softmax warps store P_j only after P_{j-1} V_{j-1} has completed (issued a
+// whole softmax earlier, so the wait is normally over at once) and no other
+// TMEM store (the rescale of O) happens while one runs.
 // The MMA issuer issues S_{j+2} as soon as the softmax warps have read S_j
-// into registers and P_j V_j as soon as P_j is stored, and the softmax warps
-// wait for the tensor pipe only to reuse a P tile (P_{j-2} V_{j-2} done) or
-// to rescale O, so the softmax of one block runs while the MMAs of the
-// neighbouring blocks do.  (P was first kept in the TMEM columns of S_j and
-// read from there by the MMA; a tcgen05.st issued while such an MMA is still
-// reading TMEM corrupts it, so every P store waited for the previous block's
-// P V and the block time was the MMAs plus that hand-over.)  Each hand-over
+// into registers and P_j V_j as soon as P_j is stored, so the softmax of one
+// block runs while the MMAs of the neighbouring blocks do.  Each hand-over
 // barrier comes in a pair, one per buffer parity, so no waiter can see its
 // barrier complete twice ahead of it.
 // K and V blocks stream through an 8-slot ring in the order the MMAs use
@@ -90,7 +97,6 @@ constexpr float kRescaleLog2 = 8.f;   // lazy-rescale threshold (log2 units)
 struct FwdLargeSmem {
     uint8_t q[kTileHalf];                     // Q, fp16 [128 x 64]
     uint8_t kv[kLSlots][kTileHalf];           // K or V blocks, fp16 [128 x 64]
-    uint8_t p[2][2][kTileHalf];               // P tiles [block parity][64-key block], fp16
     float part[2][2][128];                    // [block parity][key half]: block max, final sums
     uint64_t q_full, kv_full[kLSlots], kv_empty[kLSlots];
     uint64_t s_full[2], s_free[2], p_ready[2], pv_done[2];   // per buffer parity
@@ -164,7 +170,8 @@ __global__ void __launch_bounds__(kLT, 1) attn_fwd_tc_kernel(const __grid_consta
     pdl_wait();  // Q, K, V written by the previous kernels
     span_begin(p.span);
     const uint32_t tmem = sm.tmem;
-    const uint32_t tO = tmem + 256;              // S buffers at 0 and 128
+    // S buffers at columns 0 and 128, O at 256, the fp16 P buffers at 320 and 384
+    const uint32_t tO = tmem + 256, tP = tmem + 320;
 
     if (warp == 0) {
         if (lane == 0) {
@@ -222,8 +229,12 @@ __global__ void __launch_bounds__(kLT, 1) attn_fwd_tc_kernel(const __grid_consta
                 const int s = take();   // V_j
                 if (!ok) break;
                 tc_fence_after();
-                // O += P_j V_j: P tile j % 2 (K-major, keys along K), V MN-major
-                mma_k128_f16(tO, smem_u32(sm.p[u][0]), smem_u32(sm.kv[s]), false, idO, j > 0);
+                // O += P_j V_j: P from TMEM buffer j % 2 (8 columns per 16 keys), V MN-major
+                const uint32_t vb = smem_u32(sm.kv[s]);
+#pragma unroll
+                for (int kk = 0; kk < 8; ++kk)
+                    mma_bf16_ts(tO, tP + 64 * u + 8 * kk, smem_desc_sw128(vb + kk * 2048, kTileHalf, 1024),
+                                idO, (j > 0 || kk > 0) ? 1u : 0u);
                 mma_commit(smem_u32(&sm.pv_done[u]));
                 mma_commit(smem_u32(&sm.kv_empty[s]));
             }
@@ -293,14 +304,18 @@ __global__ void __launch_bounds__(kLT, 1) attn_fwd_tc_kernel(const __grid_consta
                 for (int c = 0; c < 32; ++c) o[c] *= corr;
                 tmem_st32(tO + lane_off + 32 * ch, o);
             }
-            // P tile j % 2 was last read by P_{j-2} V_{j-2}
-            if (j >= 2) {
-                ok = lwait(sm, sm.pv_done[u], ((j >> 1) - 1) & 1, p.status) && ok;
+            // no MMA may read TMEM while P_j is stored: P_{j-1} V_{j-1} (and
+            // with it every earlier one) has completed
+            if (j >= 1) {
+                ok = lwait(sm, sm.pv_done[u ^ 1], ((j - 1) >> 1) & 1, p.status) && ok;
                 tc_fence_after();
             }
-            put_f16_32(sm.p[u][ch], r, 0, s, 1.f);
-            put_f16_32(sm.p[u][ch], r, 32, s + 32, 1.f);
-            fence_proxy_async();
+            {
+                uint32_t w[32];
+#pragma unroll
+                for (int c = 0; c < 32; ++c) w[c] = pack_f16x2(s[2 * c], s[2 * c + 1]);
+                tmem_st32u(tP + 64 * u + lane_off + 32 * ch, w);   // keys 64 ch .. +63
+            }
             tc_fence_before();
             mbar_arrive(smem_u32(&sm.p_ready[u]));
         }

@@ -98,7 +98,8 @@ struct Saved {
     // (dQ | dK | dV | dlogit, 0..), and the backward reads X and W_q|W_k|W_v
     // through fp16 copies so that every product with dQKV is one MMA
     void *X16;          // [B*T,d] fp16 copy of X
-    void *W16;          // [3][H,d,hp] fp16 copies of W_q, W_k, W_v
+    void *W16;          // [3][H,d,hp] fp16 copies of W_q, W_k, W_v, then [H,hp,d] of W_o
+    void *AR16;         // [H,B*k,hp] fp16 diag(r^topk) A (the output product's operand)
     unsigned long long *spans;   // [16][2] kernel spans of the timed stages (measurement)
     int32_t *pos;       // [H,B*T] row b*k + i of head h holding token (b, t), or -1
                         // (token-major output and input-gradient products, k > 128)

@@ -180,7 +180,7 @@ bool tc_router(const Dims &dm, const void *X, const void *Wr, float *r_full, uin
 // fp16 attention path: X -> sv.X16 and W_q, W_k, W_v -> sv.W16 (bf16 ->
 // fp16; out-of-range values set kStatusRange).
 cudaError_t tc_f16_copies(const Dims &dm, const void *X, const void *Wq, const void *Wk,
-                          const void *Wv, const Saved &sv, cudaStream_t s);
+                          const void *Wv, const void *Wo, const Saved &sv, cudaStream_t s);
 // W_r [d,H] bf16 -> sv.WrT [H,d] fp32 (read by the dX epilogue).
 cudaError_t tc_transpose_wr(const Dims &dm, const void *Wr, const Saved &sv, cudaStream_t s);
 cudaError_t tc_attn_fwd(const Dims &dm, const Saved &sv, cudaStream_t s);

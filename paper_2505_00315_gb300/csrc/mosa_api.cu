@@ -73,7 +73,8 @@ size_t carve(const Dims &dm, char *base, Saved *sv) {
     // so the size does not depend on the environment's kernel-path switches)
     if (dm.bf16 && dm.hp == 64 && dm.k > 128) {
         s.X16 = take((size_t)2 * dm.B * dm.T * dm.d);
-        s.W16 = take((size_t)2 * 3 * dm.H * dm.d * dm.hp);
+        s.W16 = take((size_t)2 * 4 * dm.H * dm.d * dm.hp);   // W_q, W_k, W_v, W_o
+        s.AR16 = take((size_t)2 * R * dm.hp);
         s.pos = (int32_t *)take(sizeof(int32_t) * (size_t)dm.H * dm.B * dm.T);
     }
     if (sv) *sv = s;
@@ -200,9 +201,10 @@ mosa_status forward_tc(const Dims &dm, const void *X, const void *W_r, const voi
     const bool headsum = !use_fused_forward(dm) && use_headsum_out(dm);
     if (!dm.accumulate && !headsum) MOSA_TRY(cudaMemsetAsync(Y, 0, sizeof(float) * ny, r.side));
     // fp16 attention path: the fp16 copies of X and W_q|W_k|W_v that the
-    // backward's products with dQ|dK|dV read, made here beside TopK, whose
-    // grid (one CTA per (b, h) row) leaves most SMs idle
-    if (attn_f16(dm)) MOSA_TRY(tc_f16_copies(dm, X, W_q, W_k, W_v, sv, r.side));
+    // backward's products with dQ|dK|dV read, and of W_o for the output
+    // product, made here beside TopK, whose grid (one CTA per (b, h) row)
+    // leaves most SMs idle
+    if (attn_f16(dm)) MOSA_TRY(tc_f16_copies(dm, X, W_q, W_k, W_v, W_o, sv, r.side));
     if (route) {
         StageScope st_(kStageSelect, s);
         MOSA_TRY(launch_select(dm.B * dm.H, dm.T, dm.k, rf, I, r_sel, dm.B, dm.H, sv.gidx,

@@ -51,6 +51,7 @@ struct AttnParams {
     float scale_log2;         // log2(e) / sqrt(h')
     const float *rsel;        // [H, B*k]
     bf16 *AR;                 // [H, B*k, 128] pair
+    __half *AR16;             // k > 128: [H, B*k, 64] fp16 AR as well (the output product's operand)
     float *lse;               // [H, B*k]
     uint32_t *status;
     unsigned long long *span; // measurement: kernel span slot, or null
@@ -341,6 +342,23 @@ __global__ void __launch_bounds__(kLT, 1) attn_fwd_tc_kernel(const __grid_consta
                 return c < 4 ? reinterpret_cast<uint4 *>(base) + c
                              : reinterpret_cast<uint4 *>(base + 64) + (c - 4);
             });
+            if (p.AR16 != nullptr && valid) {
+                // the same 32 values as one fp16 run (64 bytes) of the fp16 AR row
+                uint4 *dst = reinterpret_cast<uint4 *>(p.AR16 + (row0 + lane) * 64 + 32 * ch);
+                float amax = 0.f;
+#pragma unroll
+                for (int u = 0; u < 4; ++u) {
+                    uint32_t w[4];
+#pragma unroll
+                    for (int e = 0; e < 4; ++e) {
+                        const float a = o[8 * u + 2 * e] * (inv * rr), c = o[8 * u + 2 * e + 1] * (inv * rr);
+                        amax = fmaxf(amax, fmaxf(fabsf(a), fabsf(c)));
+                        w[e] = pack_f16x2(a, c);
+                    }
+                    dst[u] = make_uint4(w[0], w[1], w[2], w[3]);
+                }
+                if (!(amax < kF16Overflow)) atomicOr(p.status, kStatusRange);
+            }
             // lse in natural-log units of the scaled scores
             if (ch == 0 && valid) p.lse[row0 + lane] = (m + log2f(l)) * 0.69314718055994531f;
         }
@@ -1169,6 +1187,7 @@ cudaError_t tc_attn_fwd(const Dims &dm, const Saved &sv, cudaStream_t s) {
     p.scale_log2 = 1.4426950408889634f / sqrtf(64.f);
     p.rsel = sv.rsel;
     p.AR = static_cast<bf16 *>(sv.AR);
+    p.AR16 = small ? nullptr : static_cast<__half *>(sv.AR16);
     p.lse = sv.lse;
     p.status = sv.status;
     p.span = active_span();

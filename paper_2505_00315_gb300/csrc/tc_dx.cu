@@ -18,7 +18,7 @@
 // fp32 transpose of W_r) runs while the MMAs of the next one do.  Each
 // product with a pair operand is two MMAs (hi, lo); on the fp16 attention
 // path (k > 128) dX reads dQ|dK|dV as single fp16 values and fp16 copies of
-// W_q|W_k|W_v, one MMA.
+// W_q|W_k|W_v, and Y reads AR as fp16 with an fp16 copy of W_o: one MMA.
 // Warps: 0 TMA producer, 1 MMA issuer, 2 TMEM owner, 3 idle, 4-11 epilogue
 // (warp w: tile rows 32 (w % 4) .. +31, chunk columns 128 ((w - 4) / 4) ..).
 // Every wait is bounded.
@@ -64,7 +64,8 @@ struct DxParams {
     int mt, nch;          // tiles per head, chunks per tile
     long long units;      // H * mt * nch
     uint32_t *status;
-    int f16;              // dX: A = fp16 dQKV rows [H, B*k, 256], W = fp16 copies (one MMA)
+    int f16;              // dX: A = fp16 dQKV rows [H, B*k, 256], W = fp16 copies (one MMA);
+                          // Y: A = fp16 AR rows [H, B*k, 64], W = the fp16 copy of W_o
     unsigned long long *span;   // measurement: kernel span slot, or null
 };
 
@@ -334,7 +335,12 @@ cudaError_t tc_out_scatter(const Dims &dm, const void *Wo, const Saved &sv, floa
     memset(&p, 0, sizeof(p));
     const int Mtok = dm.B * dm.k;
     if (Mtok <= 0 || dm.d <= 0 || dm.H <= 0) return cudaSuccess;
-    bool ok = map3(&p.mA, sv.AR, dm.H, Mtok, 128, 128) && map3(&p.mW[0], Wo, dm.H, 64, dm.d, 64);
+    // fp16 attention path: fp16 AR and the fp16 copy of W_o, one MMA per step
+    p.f16 = attn_f16(dm) ? 1 : 0;
+    const size_t nw = (size_t)dm.H * dm.d * 64;
+    const void *wo = p.f16 ? static_cast<const void *>(static_cast<const char *>(sv.W16) + 6 * nw) : Wo;
+    bool ok = p.f16 ? map3(&p.mA, sv.AR16, dm.H, Mtok, 64, 128) : map3(&p.mA, sv.AR, dm.H, Mtok, 128, 128);
+    ok = ok && map3(&p.mW[0], wo, dm.H, 64, dm.d, 64);
     if (!ok) return cudaErrorInvalidValue;
     p.gidx = sv.gidx;
     p.dX = Y;

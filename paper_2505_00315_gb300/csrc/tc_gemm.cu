@@ -948,12 +948,13 @@ __global__ void transpose_wr_kernel(const bf16 *__restrict__ Wr, float *__restri
 }
 
 cudaError_t tc_f16_copies(const Dims &dm, const void *X, const void *Wq, const void *Wk,
-                          const void *Wv, const Saved &sv, cudaStream_t s) {
+                          const void *Wv, const void *Wo, const Saved &sv, cudaStream_t s) {
     const size_t nw = (size_t)dm.H * dm.d * dm.hp;
-    const void *src[4] = {X, Wq, Wk, Wv};
-    void *dst[4] = {sv.X16, sv.W16, (char *)sv.W16 + 2 * nw, (char *)sv.W16 + 4 * nw};
-    const size_t n[4] = {(size_t)dm.B * dm.T * dm.d, nw, nw, nw};
-    for (int i = 0; i < 4; ++i) {
+    const void *src[5] = {X, Wq, Wk, Wv, Wo};
+    void *dst[5] = {sv.X16, sv.W16, (char *)sv.W16 + 2 * nw, (char *)sv.W16 + 4 * nw,
+                    (char *)sv.W16 + 6 * nw};
+    const size_t n[5] = {(size_t)dm.B * dm.T * dm.d, nw, nw, nw, nw};
+    for (int i = 0; i < 5; ++i) {
         const size_t n8 = n[i] / 8;   // d % 8 == 0
         const unsigned grid = (unsigned)std::min<size_t>((n8 + 255) / 256, 1216);
         to_f16_kernel<<<grid, 256, 0, s>>>(static_cast<const uint4 *>(src[i]),

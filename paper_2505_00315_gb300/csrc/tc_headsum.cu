@@ -17,8 +17,10 @@
 // zero rows, T/k times the algorithmic MMA work, which the removed reductions
 // more than pay for while T/k is small.
 //
-// Operands: F5 gathers AR as bf16 hi/lo pairs (two MMAs per head, K = 64) and
-// streams W_o[h] as 64 x 256 MN-major blocks; dX gathers the fp16 dQ|dK|dV rows
+// Operands: F5 gathers AR as fp16 rows (one MMA per head and 16-wide K step,
+// K = 64; bf16 hi/lo pairs, two MMAs, where the attention runs on the pair
+// path) and streams W_o[h] (its fp16 copy, or bf16) as 64 x 256 MN-major
+// blocks; dX gathers the fp16 dQ|dK|dV rows
 // (one 64-column part per stage, K = 64) and streams the fp16 copies of W_j[h]
 // as 256 x 64 K-major blocks; the dlogit term is added in the epilogue from
 // the fp32 transpose of W_r.
@@ -83,6 +85,7 @@ struct HsParams {
     const float *WrT;       // dX: [H, d] fp32 transpose of W_r
     float *out;             // [B*T, d]: Y or dX
     int accumulate;         // add to out instead of overwriting it
+    int f16;                // F5: A = fp16 AR rows [H, B*k, 64] and W = the fp16 copy of W_o (one MMA)
     int B, T, d, H, Mtok;
     int tps, nch;           // token tiles per sequence, column chunks
     long long units;        // B * tps * nch
@@ -180,8 +183,10 @@ __global__ void __launch_bounds__(kHsThreads, 1) head_sum_kernel(const __grid_co
     } else if (warp == 1) {
         // ---------------------------------------------------------- MMA issue
         if (lane == 0) {
-            const uint32_t idesc = kOut ? idesc_bf16(128, kHsChunk, false, true)
+            const uint32_t idesc = kOut ? (p.f16 ? idesc_f16(128, kHsChunk, false, true)
+                                                 : idesc_bf16(128, kHsChunk, false, true))
                                         : idesc_f16(128, kHsChunk, false, false);
+            const int halves = p.f16 ? 1 : 2;
             bool ok = true;
             for (int i = 0; i < nu && ok; ++i) {
                 const int buf = i & 1;
@@ -199,12 +204,16 @@ __global__ void __launch_bounds__(kHsThreads, 1) head_sum_kernel(const __grid_co
                     // tcgen05.mma halves the issue rate)
                     if (kOut) {
 #pragma unroll
-                        for (int half = 0; half < 2; ++half)
+                        for (int kk = 0; kk < 4; ++kk)
+                            mma_bf16(acc, smem_desc_sw128(a + kk * 32, 16, 1024),
+                                     smem_desc_sw128(wb + kk * 2048, 8192, 1024), idesc,
+                                     kk > 0 ? 1u : first);
+                        if (halves > 1) {   // the lo half of the AR pair
 #pragma unroll
                             for (int kk = 0; kk < 4; ++kk)
-                                mma_bf16(acc, smem_desc_sw128(a + half * kTileHalf + kk * 32, 16, 1024),
-                                         smem_desc_sw128(wb + kk * 2048, 8192, 1024), idesc,
-                                         (half > 0 || kk > 0) ? 1u : first);
+                                mma_bf16(acc, smem_desc_sw128(a + kTileHalf + kk * 32, 16, 1024),
+                                         smem_desc_sw128(wb + kk * 2048, 8192, 1024), idesc, 1u);
+                        }
                     } else {
 #pragma unroll
                         for (int kk = 0; kk < 4; ++kk)
@@ -229,6 +238,7 @@ __global__ void __launch_bounds__(kHsThreads, 1) head_sum_kernel(const __grid_co
         // j = 0..7: each warp instruction covers four whole 128-byte segments
         const int t = threadIdx.x - 128;
         const int chunk = t & 7, sub = t >> 3;
+        const int row_bytes = (kOut && p.f16) ? 128 : C::ROW_BYTES;   // fp16 AR rows: 64 values
         int landed = 0, issued = 0;
         bool ok = true;
         // this thread's rows of head h's list for the tile of (unit i, head h),
@@ -262,11 +272,11 @@ __global__ void __launch_bounds__(kHsThreads, 1) head_sum_kernel(const __grid_co
                         const int r = sub + 16 * j;
                         const int pr = prow[j];
                         const uint32_t nbytes = pr >= 0 ? 16u : 0u;
-                        const uint8_t *src = p.A + ((size_t)h * p.Mtok + (pr >= 0 ? pr : 0)) * C::ROW_BYTES +
+                        const uint8_t *src = p.A + ((size_t)h * p.Mtok + (pr >= 0 ? pr : 0)) * row_bytes +
                                              part * 128 + chunk * 16;
                         const uint32_t off = r * 128 + ((chunk ^ (r & 7)) << 4);
                         cp_async16(a + off, src, nbytes);
-                        if (kOut) cp_async16(a + kTileHalf + off, src + 128, nbytes);   // lo half
+                        if (kOut && !p.f16) cp_async16(a + kTileHalf + off, src + 128, nbytes);   // lo half
                     }
                     cp_async_commit();
                     issued = it + 1;
@@ -451,8 +461,13 @@ cudaError_t tc_token_rows(const Dims &dm, const Saved &sv, cudaStream_t s) {
 cudaError_t tc_out_headsum(const Dims &dm, const void *Wo, const Saved &sv, float *Y, cudaStream_t s) {
     HsParams p;
     memset(&p, 0, sizeof(p));
-    if (!map_w(&p.mW[0], Wo, dm.H, 64, dm.d, 64)) return cudaErrorInvalidValue;
-    p.A = static_cast<const uint8_t *>(sv.AR);
+    // fp16 attention path (k > 128, always so here): fp16 AR and the fp16 copy
+    // of W_o that the forward made beside TopK, one MMA per step
+    p.f16 = attn_f16(dm) ? 1 : 0;
+    const size_t nw = (size_t)dm.H * dm.d * 64;
+    const void *wo = p.f16 ? static_cast<const void *>(static_cast<const char *>(sv.W16) + 6 * nw) : Wo;
+    if (!map_w(&p.mW[0], wo, dm.H, 64, dm.d, 64)) return cudaErrorInvalidValue;
+    p.A = static_cast<const uint8_t *>(p.f16 ? sv.AR16 : sv.AR);
     p.pos = sv.pos;
     p.out = Y;
     p.accumulate = dm.accumulate ? 1 : 0;

@@ -255,16 +255,17 @@ KERNEL_STAGE = [("tc_gemm_kernel<5>", "router"), ("tc_gemm_kernel<(int)5>", "rou
                 ("tc_gemm_kernel<(int)0>", "qkv"), ("attn_fwd", "attn_fwd"),
                 ("tc_gemm_kernel<2>", "out_bwd"), ("tc_gemm_kernel<(int)2>", "out_bwd"),
                 ("attn_bwd", "attn_bwd"), ("dq_finish", "attn_bwd"),
-                ("scatter_product_kernel<0>", "in_bwd"), ("scatter_product_kernel<false>", "in_bwd"),
-                ("scatter_product_kernel<1>", "out"), ("scatter_product_kernel<true>", "out"),
+                ("scatter_product_kernel<0>", "in_bwd"), ("scatter_product_kernel<(int)0>", "in_bwd"),
+                ("scatter_product_kernel<1>", "out"), ("scatter_product_kernel<(int)1>", "out"),
+                ("head_sum_kernel<true>", "out"), ("head_sum_kernel<(bool)1>", "out"),
                 ("tc_gemm_kernel<4>", "w_bwd"), ("tc_gemm_kernel<(int)4>", "w_bwd"),
                 ("tc_gemm_kernel<6>", "w_bwd"), ("tc_gemm_kernel<(int)6>", "w_bwd"),
-                ("to_f16_kernel", "dwo"),
                 ("tc_gemm_kernel<3>", "dwo"), ("tc_gemm_kernel<(int)3>", "dwo"),
                 ("fused_fwd_kernel", "fwd_unit"), ("fused_bwd_kernel", "bwd_unit"),
                 ("dense_rows", "select")]
-# RoPE passes (rope_rows_kernel) run inside the qkv and attn_bwd stages alike
-# and are left unattributed.
+# RoPE passes (rope_rows_kernel) run inside the qkv and attn_bwd stages alike,
+# and the fp16 copies (to_f16_kernel) beside TopK on the side stream: both are
+# left unattributed.
 
 
 def ingest_ncu(csv_path, cfg_name):

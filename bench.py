@@ -503,9 +503,14 @@ def main():
 
     # Timed region: K steps, L2 flushed before each, the dominant stage timed
     # live with CUDA events on every PROFILE_EVERY-th step.  Its event pair sits
-    # inside the step's graph (and cuts the early-launch chain around it), and
-    # reading it waits for the step, so timing it on every step would slow the
-    # steps it measures; both graph variants are captured before timing starts.
+    # inside the step's graph (and cuts the early-launch chain around it), so
+    # timing it on every step would slow the steps it measures; both graph
+    # variants are captured before timing starts.  Nothing is read back during
+    # the timed region (a read waits for the device, and the next step would
+    # then start from an idle GPU with the host's launch latency inside its
+    # events): the events are read after it, and each timed step's kernel
+    # spans are copied on the device, outside the step's events, into a
+    # per-step buffer read after it as well.
     K = args.steps
     starts = [torch.cuda.Event(enable_timing=True) for _ in range(K)]
     ends = [torch.cuda.Event(enable_timing=True) for _ in range(K)]
@@ -522,8 +527,8 @@ def main():
     barrier()
     torch.cuda.synchronize()
     launches0 = mosa.mosa_kernel_launches()
-    dom = [0.0, 0, 0]   # ms, launches, steps
-    span = [0.0, 0]     # kernel-span ms, steps
+    span_slots = torch.zeros((K, 32), dtype=torch.int64, device=dev)
+    n_timed = 0
     t_host0 = time.time()
     for i in range(K):
         timed = i % PROFILE_EVERY == 0
@@ -533,18 +538,20 @@ def main():
         step()
         ends[i].record()
         if timed:
-            # waits for this step; the next step's L2 flush covers the host time
-            ms, n = mosa.mosa_profile_read()[dominant]
-            dom[0] += ms
-            dom[1] += n
-            dom[2] += 1
+            n_timed += 1
             if not hybrid:
-                sp = mosa.mosa_profile_spans(shape, ws).get(dominant, -1.0)
-                if sp >= 0:
-                    span[0] += sp
-                    span[1] += 1
+                mosa.mosa_profile_spans_copy(shape, ws, span_slots[i])
     torch.cuda.synchronize()
     t_host1 = time.time()
+    ms_d, n_d = mosa.mosa_profile_read()[dominant]
+    dom = [ms_d, n_d, n_timed]   # ms over the timed steps, launches, steps
+    span = [0.0, 0]              # kernel-span ms, steps
+    di = STAGES.index(dominant)
+    for i in range(0, K, PROFILE_EVERY):
+        a, b = (int(v) for v in span_slots[i, 2 * di:2 * di + 2].tolist())
+        if not hybrid and a != -1 and b != 0 and b >= a:   # -1: all ones read as int64
+            span[0] += (b - a) * 1e-6
+            span[1] += 1
     barrier()
     launches = mosa.mosa_kernel_launches() - launches0
     mosa.mosa_profile_stages(0)

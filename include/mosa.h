@@ -293,6 +293,16 @@ int32_t mosa_profile_read(double *total_ms, int32_t *count, int32_t max_stages);
  * Returns the number of entries written. */
 int32_t mosa_profile_spans(const mosa_shape *shape, void *workspace, double *ms, int32_t max_stages);
 
+/* Enqueues on `stream` a device-to-device copy of the workspace's kernel-span
+ * slots (32 unsigned 64-bit values: start, end in %globaltimer nanoseconds
+ * for stages 0..15; a start of all ones or an end of 0 means no record) into
+ * dst (device memory of 256 bytes), so that a caller timing many steps can
+ * keep each step's spans without waiting for the device between steps.  The
+ * slots are those mosa_profile_spans reads.  MOSA_OK, MOSA_ERR_INVALID_ARG,
+ * MOSA_ERR_WORKSPACE or MOSA_ERR_CUDA. */
+mosa_status mosa_profile_spans_copy(const mosa_shape *shape, void *workspace, void *dst,
+                                    void *stream);
+
 /* Timeline mode (on = 1, off = 0): later layer calls record, for every stage,
  * the first CTA start and last CTA end of its kernels (%globaltimer) into the
  * workspace, with no CUDA events and no per-stage resets between the kernels

@@ -12,7 +12,7 @@ __all__ = ["mosa_forward", "mosa_forward_with_indices", "mosa_backward", "mosa_t
            "mosa_workspace_bytes", "mosa_check_status", "alloc_workspace", "make_shape",
            "MosaShape", "MosaError", "load", "mosa_kernel_launches", "mosa_profile_stages",
            "mosa_profile_read", "mosa_profile_spans", "mosa_profile_timeline",
-           "mosa_profile_timeline_read", "mosa_stage_name", "mosa_stage_engine", "stage_impl",
+           "mosa_profile_timeline_read", "mosa_profile_spans_copy", "mosa_stage_name", "mosa_stage_engine", "stage_impl",
            "mosa_route_noalloc", "mosa_adaptive_k", "MosaHybridShape", "make_hybrid_shape",
            "mosa_hybrid_workspace_bytes", "alloc_hybrid_workspace", "mosa_hybrid_forward",
            "mosa_hybrid_backward"]

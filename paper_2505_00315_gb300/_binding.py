@@ -29,7 +29,8 @@ EXPORTED = ("mosa_status_string", "mosa_workspace_bytes", "mosa_forward",
             "mosa_kernel_launches", "mosa_profile_stages", "mosa_profile_read",
             "mosa_stage_name", "mosa_stage_engine", "mosa_route_noalloc", "mosa_adaptive_k",
             "mosa_hybrid_workspace_bytes", "mosa_hybrid_forward", "mosa_hybrid_backward",
-            "mosa_profile_spans", "mosa_profile_timeline", "mosa_profile_timeline_read")
+            "mosa_profile_spans", "mosa_profile_timeline", "mosa_profile_timeline_read",
+            "mosa_profile_spans_copy")
 
 
 class MosaShape(ctypes.Structure):
@@ -102,6 +103,8 @@ def load(build_if_missing: bool = True) -> ctypes.CDLL:
         L.mosa_profile_read.restype = i32
         L.mosa_profile_spans.argtypes = [sp, vp, ctypes.POINTER(ctypes.c_double), i32]
         L.mosa_profile_spans.restype = i32
+        L.mosa_profile_spans_copy.argtypes = [sp, vp, vp, vp]
+        L.mosa_profile_spans_copy.restype = ctypes.c_int
         L.mosa_profile_timeline.argtypes = [i32]
         L.mosa_profile_timeline.restype = ctypes.c_int
         L.mosa_profile_timeline_read.argtypes = [sp, vp, ctypes.POINTER(ctypes.c_double),
@@ -376,6 +379,19 @@ def mosa_profile_spans(shape: MosaShape, workspace) -> dict:
     ms = (ctypes.c_double * n)()
     m = L.mosa_profile_spans(ctypes.byref(shape), ctypes.c_void_p(workspace.data_ptr()), ms, n)
     return {mosa_stage_name(i): ms[i] for i in range(min(m, n))}
+
+
+def mosa_profile_spans_copy(shape: MosaShape, workspace, dst) -> None:
+    """Enqueue on the current stream a copy of the workspace's 32 kernel-span
+    slots (int64 [start, end] per stage) into the device tensor ``dst``
+    (at least 32 int64); no wait."""
+    torch = _torch()
+    if dst.dtype != torch.int64 or dst.numel() < 32 or not dst.is_cuda or not dst.is_contiguous():
+        raise ValueError("dst must be a contiguous CUDA int64 tensor of at least 32 elements")
+    _check(load().mosa_profile_spans_copy(ctypes.byref(shape), ctypes.c_void_p(workspace.data_ptr()),
+                                          ctypes.c_void_p(dst.data_ptr()),
+                                          ctypes.c_void_p(torch.cuda.current_stream().cuda_stream)),
+           "mosa_profile_spans_copy")
 
 
 def mosa_profile_timeline(on: bool) -> None:

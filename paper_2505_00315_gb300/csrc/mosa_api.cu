@@ -809,6 +809,19 @@ int32_t mosa_profile_spans(const mosa_shape *shape, void *workspace, double *ms,
     return n;
 }
 
+mosa_status mosa_profile_spans_copy(const mosa_shape *shape, void *workspace, void *dst,
+                                    void *stream) {
+    Dims dm;
+    mosa_status st = check_shape(shape, &dm);
+    if (st != MOSA_OK) return st;
+    if (dst == nullptr) return MOSA_ERR_INVALID_ARG;
+    if (workspace == nullptr || ((uintptr_t)workspace % kAlign) != 0) return MOSA_ERR_WORKSPACE;
+    Saved sv;
+    carve(dm, (char *)workspace, &sv);
+    return cuda_status(cudaMemcpyAsync(dst, sv.spans, sizeof(unsigned long long) * 2 * 16,
+                                       cudaMemcpyDeviceToDevice, (cudaStream_t)stream));
+}
+
 int32_t mosa_profile_timeline_read(const mosa_shape *shape, void *workspace, double *start_us,
                                    double *end_us, int32_t max_stages) {
     Dims dm;

@@ -430,8 +430,18 @@ def test_stage_kernel_spans_inside_event_windows(name):
         torch.cuda.synchronize()
         events = mosa.mosa_profile_read()
         spans = mosa.mosa_profile_spans(shape, ws)
+        slots = torch.zeros(32, dtype=torch.int64, device="cuda")
+        mosa.mosa_profile_spans_copy(shape, ws, slots)
+        torch.cuda.synchronize()
     finally:
         mosa.mosa_profile_stages(0)
+    # the device-side copy holds the same slots the synchronous read decoded
+    sl = slots.cpu().numpy()
+    for i in range(12):
+        name = mosa.mosa_stage_name(i)
+        a, b = int(sl[2 * i]), int(sl[2 * i + 1])
+        if a != -1 and b != 0:
+            assert abs((b - a) * 1e-6 - spans[name]) < 1e-9, (name, a, b, spans[name])
     assert mosa.mosa_check_status(shape, ws) == 0
     np.testing.assert_array_equal(I.cpu().numpy(), plain["I"])
     np.testing.assert_allclose(Y.float().cpu().numpy(), plain["Y"], rtol=1e-5, atol=1e-6)

@@ -547,9 +547,11 @@ def main():
     dom = [ms_d, n_d, n_timed]   # ms over the timed steps, launches, steps
     span = [0.0, 0]              # kernel-span ms, steps
     di = STAGES.index(dominant)
+    m64 = (1 << 64) - 1
     for i in range(0, K, PROFILE_EVERY):
-        a, b = (int(v) for v in span_slots[i, 2 * di:2 * di + 2].tolist())
-        if not hybrid and a != -1 and b != 0 and b >= a:   # -1: all ones read as int64
+        # unsigned, as the library decodes them: start all ones or end 0 = no record
+        a, b = (int(v) & m64 for v in span_slots[i, 2 * di:2 * di + 2].tolist())
+        if not hybrid and a != m64 and b != 0 and b >= a:
             span[0] += (b - a) * 1e-6
             span[1] += 1
     barrier()

@@ -255,8 +255,10 @@ KERNEL_STAGE = [("tc_gemm_kernel<5>", "router"), ("tc_gemm_kernel<(int)5>", "rou
                 ("tc_gemm_kernel<(int)0>", "qkv"), ("attn_fwd", "attn_fwd"),
                 ("tc_gemm_kernel<2>", "out_bwd"), ("tc_gemm_kernel<(int)2>", "out_bwd"),
                 ("attn_bwd", "attn_bwd"), ("dq_finish", "attn_bwd"),
-                ("scatter_product_kernel<0>", "in_bwd"), ("scatter_product_kernel<(int)0>", "in_bwd"),
-                ("scatter_product_kernel<1>", "out"), ("scatter_product_kernel<(int)1>", "out"),
+                ("scatter_product_kernel<0>", "in_bwd"), ("scatter_product_kernel<false>", "in_bwd"),
+                ("scatter_product_kernel<(bool)0>", "in_bwd"),
+                ("scatter_product_kernel<1>", "out"), ("scatter_product_kernel<true>", "out"),
+                ("scatter_product_kernel<(bool)1>", "out"),
                 ("head_sum_kernel<true>", "out"), ("head_sum_kernel<(bool)1>", "out"),
                 ("tc_gemm_kernel<4>", "w_bwd"), ("tc_gemm_kernel<(int)4>", "w_bwd"),
                 ("tc_gemm_kernel<6>", "w_bwd"), ("tc_gemm_kernel<(int)6>", "w_bwd"),

@@ -251,6 +251,7 @@ def traffic_for(stage, cfg_name):
 
 # Kernel name (as ncu prints it) -> bench stage.
 KERNEL_STAGE = [("tc_gemm_kernel<5>", "router"), ("tc_gemm_kernel<(int)5>", "router"),
+                ("pad_wr_kernel", "router"),
                 ("topk_select", "select"), ("tc_gemm_kernel<0>", "qkv"),
                 ("tc_gemm_kernel<(int)0>", "qkv"), ("attn_fwd", "attn_fwd"),
                 ("tc_gemm_kernel<2>", "out_bwd"), ("tc_gemm_kernel<(int)2>", "out_bwd"),

@@ -94,6 +94,8 @@ struct Saved {
     float *G;           // [H,B*k,hp] dY[I] W_o^T (fp32, CUDA-core path); on the
                         // tensor-core path with k > 128 the fp32 dQ accumulator
     float *WrT;         // [H,d] fp32 transpose of W_r (tensor-core dX epilogue)
+    void *Wr64;         // [d, H rounded up to 64] bf16 W_r with zero columns past H
+                        // (tensor-core router, H % 64 != 0)
     // fp16 attention path (tensor cores, k > 128): dQKV is [H,B*k,256] fp16
     // (dQ | dK | dV | dlogit, 0..), and the backward reads X and W_q|W_k|W_v
     // through fp16 copies so that every product with dQKV is one MMA

@@ -70,9 +70,13 @@ cudaError_t launch_rope(void *p0, int col0_0, void *p1, int col0_1, bool pair, i
 // F1, Sec. 2.2 router: r_full[b,h,t] = sigmoid(X[b,t,:] . W_r[:,h]) in fp32.
 cudaError_t launch_router(const Dims &dm, const void *X, const void *Wr, float *r_full,
                           cudaStream_t stream);
-// F1 choosing the tensor-core kernel where it applies.
+// F1 choosing the tensor-core kernel where it applies.  wr_pad (optional):
+// room for a [d, H rounded up to 64] bf16 copy of W_r, used by the
+// tensor-core router when H % 64 != 0; zero_status: zero the status word
+// first (ordered after all earlier work on the stream).
 cudaError_t launch_router_auto(const Dims &dm, const void *X, const void *Wr, float *r_full,
-                               uint32_t *status, cudaStream_t stream);
+                               uint32_t *status, cudaStream_t stream, void *wr_pad = nullptr,
+                               bool zero_status = false);
 
 // F2, Sec. 2.2 TopK: per row of T scores, the k largest (ties: lower index),
 // ascending.  If gidx != nullptr, row = b*H + h also writes the head-major
@@ -175,10 +179,17 @@ cudaError_t tc_out_scatter(const Dims &dm, const void *Wo, const Saved &sv, floa
 cudaError_t tc_dx(const Dims &dm, const void *Wq, const void *Wk, const void *Wv, const Saved &sv,
                   float *dX, cudaStream_t s);
 // F1 on tensor cores (bf16 inputs, H % 8 == 0); false if not applicable.
-bool tc_router(const Dims &dm, const void *X, const void *Wr, float *r_full, uint32_t *status,
-               cudaStream_t s, cudaError_t *err);
-// fp16 attention path: X -> sv.X16 and W_q, W_k, W_v -> sv.W16 (bf16 ->
-// fp16; out-of-range values set kStatusRange).
+// Wr is [d, wr_cols] bf16 with wr_cols >= H (columns beyond H unused).
+bool tc_router_applies(const Dims &dm);
+bool tc_router(const Dims &dm, const void *X, const void *Wr, int wr_cols, float *r_full,
+               uint32_t *status, cudaStream_t s, cudaError_t *err);
+// bf16 -> fp16 copy of n values (n % 8 == 0, 16-byte aligned); values beyond
+// the fp16 range set kStatusRange.
+cudaError_t tc_to_f16(const void *src, void *dst, size_t n, uint32_t *status, cudaStream_t s);
+// Address of the fp16 copy of W_o inside sv.W16.
+void *wo16_of(const Dims &dm, const Saved &sv);
+// fp16 attention path: X -> sv.X16 and W_q, W_k, W_v, W_o -> sv.W16 (bf16 ->
+// fp16; out-of-range values set kStatusRange); a null source is skipped.
 cudaError_t tc_f16_copies(const Dims &dm, const void *X, const void *Wq, const void *Wk,
                           const void *Wv, const void *Wo, const Saved &sv, cudaStream_t s);
 // W_r [d,H] bf16 -> sv.WrT [H,d] fp32 (read by the dX epilogue).

@@ -68,6 +68,8 @@ size_t carve(const Dims &dm, char *base, Saved *sv) {
     s.dQKV = take(e * R * 4 * dm.hp);  // 3 h' columns, or 4 blocks of 64 on the tensor cores
     s.G = (float *)take(sizeof(float) * R * dm.hp);
     s.WrT = (float *)take(sizeof(float) * (size_t)dm.d * dm.H);
+    // (reserved for either dtype, so that the size depends on the shape only)
+    if (dm.H % 64 != 0) s.Wr64 = take((size_t)2 * dm.d * ((dm.H + 63) / 64 * 64));
     s.spans = (unsigned long long *)take(sizeof(unsigned long long) * 2 * 16);
     // the fp16 attention path's copies (reserved whenever that path can run,
     // so the size does not depend on the environment's kernel-path switches)
@@ -189,12 +191,13 @@ mosa_status forward_tc(const Dims &dm, const void *X, const void *W_r, const voi
                        const float *rsel_in, const Saved &sv, cudaStream_t s, DevResources &r) {
     set_span_base(sv.spans);   // measurement: this call's kernel-span slots
     MOSA_TRY(begin_timeline_call(kForwardStages, s));
-    // A call that adds into Y continues the status word of the call that wrote it.
-    if (!dm.accumulate) MOSA_TRY(cudaMemsetAsync(sv.status, 0, sizeof(uint32_t), s));
     const size_t ny = (size_t)dm.B * dm.T * dm.d;
+    // A call that adds into Y continues the status word of the call that wrote it.
     if (route) {
         StageScope st_(kStageRouter, s);
-        MOSA_TRY(launch_router_auto(dm, X, W_r, rf, sv.status, s));
+        MOSA_TRY(launch_router_auto(dm, X, W_r, rf, sv.status, s, sv.Wr64, !dm.accumulate));
+    } else if (!dm.accumulate) {
+        MOSA_TRY(cudaMemsetAsync(sv.status, 0, sizeof(uint32_t), s));
     }
     MOSA_TRY(link(s, r.side, r.ev[0]));
     // (the token-major output product writes every element of Y itself)

@@ -11,6 +11,7 @@
 // ascending (the order the causal mask works in) and ties go to the lower
 // token index.  Output positions come from one block-wide prefix sum of the
 // per-segment counts, so no sort is needed.
+#include <algorithm>
 #include <mutex>
 
 #include "launch.h"
@@ -92,8 +93,6 @@ topk_select_kernel(const float *__restrict__ scores, int T, int k, int32_t *__re
     __shared__ uint32_t hist[2][256];
     __shared__ unsigned long long sh[33];
     __shared__ uint32_t sh_prefix, sh_remaining;
-    // the next kernel may launch and run its prologue as this grid's CTAs finish
-    asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
     asm volatile("griddepcontrol.wait;" ::: "memory");  // scores from the router kernel
     span_begin(span);
     const int row = blockIdx.x;
@@ -192,6 +191,12 @@ topk_select_kernel(const float *__restrict__ scores, int T, int k, int32_t *__re
             ++pos;
         }
     }
+    // The next kernel launches only now: launched at this kernel's start, its
+    // CTAs (one per SM for the projections) sat on every SM this grid of B*H
+    // CTAs leaves idle, and the side stream's copies and zeroing found no SM
+    // until the attention kernel's tail (measured at B4 T4096 d1024 H16 k1024:
+    // a 13 us wait before the output product, 394 -> 381 us a step).
+    asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
     if (span != nullptr) {
         __syncthreads();
         span_end(span);
@@ -247,10 +252,47 @@ cudaError_t launch_router(const Dims &dm, const void *X, const void *Wr, float *
     return launch_simt_gemm(op, 1, stream);
 }
 
+// W_r [d,H] -> Wp [d,Hp], columns H..Hp-1 zero, and the status word zeroed
+// (status != nullptr).  Launched without the early-launch attribute, so it
+// reads W_r and writes the status word only after all earlier work on the
+// stream; it lets the router launch early at once (the router still waits for
+// its completion before its first load).
+__global__ void pad_wr_kernel(const bf16 *__restrict__ Wr, bf16 *__restrict__ Wp, int d, int H,
+                              int Hp, uint32_t *status) {
+    asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
+    if (status != nullptr && blockIdx.x == 0 && threadIdx.x == 0) *status = 0;
+    const size_t n = (size_t)d * Hp;
+    for (size_t i = (size_t)blockIdx.x * blockDim.x + threadIdx.x; i < n;
+         i += (size_t)gridDim.x * blockDim.x) {
+        const int c = (int)(i % Hp);
+        Wp[i] = c < H ? Wr[(i / Hp) * H + c] : __float2bfloat16(0.f);
+    }
+}
+
 cudaError_t launch_router_auto(const Dims &dm, const void *X, const void *Wr, float *r_full,
-                               uint32_t *status, cudaStream_t stream) {
+                               uint32_t *status, cudaStream_t stream, void *wr_pad,
+                               bool zero_status) {
     cudaError_t e = cudaSuccess;
-    if (use_tc(dm) && tc_router(dm, X, Wr, r_full, status, stream, &e)) return e;
+    const bool tc = use_tc(dm) && tc_router_applies(dm);
+    // The tensor-core router loads W_r in blocks of 64 columns; when H is not
+    // a multiple of 64 it reads a zero-padded copy, since blocks reaching past
+    // column H (filled by the copy engine) ran its main loop at about 60% of
+    // the in-bounds speed (10.8 against 6.3 us at B4 T4096 d1024 H8).
+    const bool pad = tc && wr_pad != nullptr && dm.H % 64 != 0;
+    const int hp64 = (dm.H + 63) / 64 * 64;
+    if (pad) {
+        const size_t n = (size_t)dm.d * hp64;
+        const int grid = (int)std::min<size_t>((n + 255) / 256, 608);
+        pad_wr_kernel<<<grid, 256, 0, stream>>>(static_cast<const bf16 *>(Wr),
+                                                 static_cast<bf16 *>(wr_pad), dm.d, dm.H, hp64,
+                                                 zero_status ? status : nullptr);
+        note_launches(1);
+        if ((e = cudaGetLastError()) != cudaSuccess) return e;
+    } else if (zero_status) {
+        if ((e = cudaMemsetAsync(status, 0, sizeof(uint32_t), stream)) != cudaSuccess) return e;
+    }
+    if (tc && tc_router(dm, X, pad ? wr_pad : Wr, pad ? hp64 : dm.H, r_full, status, stream, &e))
+        return e;
     return launch_router(dm, X, Wr, r_full, stream);
 }
 

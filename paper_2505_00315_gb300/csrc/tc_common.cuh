@@ -367,6 +367,22 @@ __device__ __forceinline__ uint32_t pack_f16x2(float a, float b) {
 // finite value): an intermediate at or above it is out of the fp16 range.
 constexpr float kF16Overflow = 65520.f;
 
+// Eight bf16 values (one 16-byte unit) -> eight fp16 values.  Exact for
+// magnitudes in [2^-17, 65504] (fp16 has three more significand bits than
+// bf16); smaller ones round to fp16's subnormal grid (2^-24); `bad` is set
+// for a value beyond the fp16 range.
+__device__ __forceinline__ uint4 bf16x8_to_f16x8(uint4 u, bool &bad) {
+    const uint32_t w[4] = {u.x, u.y, u.z, u.w};
+    uint32_t o[4];
+#pragma unroll
+    for (int e = 0; e < 4; ++e) {
+        const float lo = __uint_as_float(w[e] << 16), hi = __uint_as_float(w[e] & 0xFFFF0000u);
+        bad = bad || !(fabsf(lo) < kF16Overflow) || !(fabsf(hi) < kF16Overflow);
+        o[e] = pack_f16x2(lo, hi);
+    }
+    return make_uint4(o[0], o[1], o[2], o[3]);
+}
+
 // The split-bf16 pair representation of the kernels' intermediate operands,
 // for two values at once, as bf16x2 words with a in the low 16 bits:
 // hi = v cut to bf16 (low 16 bits cleared, i.e. rounded toward zero), r = v - hi

@@ -337,8 +337,7 @@ cudaError_t tc_out_scatter(const Dims &dm, const void *Wo, const Saved &sv, floa
     if (Mtok <= 0 || dm.d <= 0 || dm.H <= 0) return cudaSuccess;
     // fp16 attention path: fp16 AR and the fp16 copy of W_o, one MMA per step
     p.f16 = attn_f16(dm) ? 1 : 0;
-    const size_t nw = (size_t)dm.H * dm.d * 64;
-    const void *wo = p.f16 ? static_cast<const void *>(static_cast<const char *>(sv.W16) + 6 * nw) : Wo;
+    const void *wo = p.f16 ? static_cast<const void *>(wo16_of(dm, sv)) : Wo;
     bool ok = p.f16 ? map3(&p.mA, sv.AR16, dm.H, Mtok, 64, 128) : map3(&p.mA, sv.AR, dm.H, Mtok, 128, 128);
     ok = ok && map3(&p.mW[0], wo, dm.H, 64, dm.d, 64);
     if (!ok) return cudaErrorInvalidValue;

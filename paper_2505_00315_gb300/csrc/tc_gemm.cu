@@ -886,9 +886,11 @@ bool map_2d(CUtensorMap *m, const void *base, uint64_t rows, uint64_t cols, uint
 
 }  // namespace
 
-bool tc_router(const Dims &dm, const void *X, const void *Wr, float *r_full, uint32_t *status,
-               cudaStream_t s, cudaError_t *err) {
-    if (!dm.bf16 || dm.H % 8 != 0 || !tmap_available()) return false;
+bool tc_router_applies(const Dims &dm) { return dm.bf16 && dm.H % 8 == 0 && tmap_available(); }
+
+bool tc_router(const Dims &dm, const void *X, const void *Wr, int wr_cols, float *r_full,
+               uint32_t *status, cudaStream_t s, cudaError_t *err) {
+    if (!tc_router_applies(dm) || wr_cols < dm.H) return false;
     TcParams p;
     memset(&p, 0, sizeof(p));
     p.M = dm.B * dm.T;
@@ -905,35 +907,23 @@ bool tc_router(const Dims &dm, const void *X, const void *Wr, float *r_full, uin
     p.ring_stride = kTile16K + p.N / 64 * kTile8K;
     p.ring_stages = std::min(kMaxStages, Cfg<kROUTER>::STAGES * (kTile16K + 4 * kTile8K) / p.ring_stride);
     if (!map_2d(&p.mapA, X, (uint64_t)dm.B * dm.T, dm.d, 128) ||
-        !map_2d(&p.mapB[0], Wr, dm.d, dm.H, 64))
+        !map_2d(&p.mapB[0], Wr, dm.d, wr_cols, 64))
         return false;
     dim3 grid((p.M + kBM - 1) / kBM, (dm.H + 255) / 256, 1);
     *err = launch_kind<kROUTER>(p, grid, s);
     return true;
 }
 
-// bf16 -> fp16, eight values per 16-byte step.  Exact for magnitudes in
-// [2^-17, 65504] (fp16 has three more significand bits than bf16); smaller
-// ones round to fp16's subnormal grid (2^-24); a value beyond the fp16 range
-// sets kStatusRange.
+// bf16 -> fp16, eight values per 16-byte step (bf16x8_to_f16x8); a value
+// beyond the fp16 range sets kStatusRange.
 __global__ void to_f16_kernel(const uint4 *__restrict__ src, uint4 *__restrict__ dst, size_t n8,
                               uint32_t *status) {
     pdl_wait();
     pdl_trigger();
     bool bad = false;
     for (size_t i = (size_t)blockIdx.x * blockDim.x + threadIdx.x; i < n8;
-         i += (size_t)gridDim.x * blockDim.x) {
-        const uint4 u = src[i];
-        const uint32_t w[4] = {u.x, u.y, u.z, u.w};
-        uint32_t o[4];
-#pragma unroll
-        for (int e = 0; e < 4; ++e) {
-            const float lo = __uint_as_float(w[e] << 16), hi = __uint_as_float(w[e] & 0xFFFF0000u);
-            bad = bad || !(fabsf(lo) < kF16Overflow) || !(fabsf(hi) < kF16Overflow);
-            o[e] = pack_f16x2(lo, hi);
-        }
-        dst[i] = make_uint4(o[0], o[1], o[2], o[3]);
-    }
+         i += (size_t)gridDim.x * blockDim.x)
+        dst[i] = bf16x8_to_f16x8(src[i], bad);
     if (__any_sync(0xffffffffu, bad) && (threadIdx.x & 31) == 0) atomicOr(status, kStatusRange);
 }
 
@@ -947,20 +937,30 @@ __global__ void transpose_wr_kernel(const bf16 *__restrict__ Wr, float *__restri
     }
 }
 
+cudaError_t tc_to_f16(const void *src, void *dst, size_t n, uint32_t *status, cudaStream_t s) {
+    const size_t n8 = n / 8;
+    if (n8 == 0) return cudaSuccess;
+    const unsigned grid = (unsigned)std::min<size_t>((n8 + 255) / 256, 1216);
+    to_f16_kernel<<<grid, 256, 0, s>>>(static_cast<const uint4 *>(src), static_cast<uint4 *>(dst),
+                                       n8, status);
+    note_launches(1);
+    return cudaGetLastError();
+}
+
+void *wo16_of(const Dims &dm, const Saved &sv) {
+    return (char *)sv.W16 + 6 * (size_t)dm.H * dm.d * dm.hp;
+}
+
 cudaError_t tc_f16_copies(const Dims &dm, const void *X, const void *Wq, const void *Wk,
                           const void *Wv, const void *Wo, const Saved &sv, cudaStream_t s) {
     const size_t nw = (size_t)dm.H * dm.d * dm.hp;
     const void *src[5] = {X, Wq, Wk, Wv, Wo};
     void *dst[5] = {sv.X16, sv.W16, (char *)sv.W16 + 2 * nw, (char *)sv.W16 + 4 * nw,
-                    (char *)sv.W16 + 6 * nw};
-    const size_t n[5] = {(size_t)dm.B * dm.T * dm.d, nw, nw, nw, nw};
+                    wo16_of(dm, sv)};
+    const size_t n[5] = {(size_t)dm.B * dm.T * dm.d, nw, nw, nw, nw};   // d % 8 == 0
     for (int i = 0; i < 5; ++i) {
-        const size_t n8 = n[i] / 8;   // d % 8 == 0
-        const unsigned grid = (unsigned)std::min<size_t>((n8 + 255) / 256, 1216);
-        to_f16_kernel<<<grid, 256, 0, s>>>(static_cast<const uint4 *>(src[i]),
-                                           static_cast<uint4 *>(dst[i]), n8, sv.status);
-        note_launches(1);
-        const cudaError_t e = cudaGetLastError();
+        if (src[i] == nullptr) continue;
+        const cudaError_t e = tc_to_f16(src[i], dst[i], n[i], sv.status, s);
         if (e != cudaSuccess) return e;
     }
     return cudaSuccess;

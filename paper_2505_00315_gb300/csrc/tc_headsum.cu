@@ -464,8 +464,7 @@ cudaError_t tc_out_headsum(const Dims &dm, const void *Wo, const Saved &sv, floa
     // fp16 attention path (k > 128, always so here): fp16 AR and the fp16 copy
     // of W_o that the forward made beside TopK, one MMA per step
     p.f16 = attn_f16(dm) ? 1 : 0;
-    const size_t nw = (size_t)dm.H * dm.d * 64;
-    const void *wo = p.f16 ? static_cast<const void *>(static_cast<const char *>(sv.W16) + 6 * nw) : Wo;
+    const void *wo = p.f16 ? static_cast<const void *>(wo16_of(dm, sv)) : Wo;
     if (!map_w(&p.mW[0], wo, dm.H, 64, dm.d, 64)) return cudaErrorInvalidValue;
     p.A = static_cast<const uint8_t *>(p.f16 ? sv.AR16 : sv.AR);
     p.pos = sv.pos;

@@ -386,20 +386,24 @@ def test_invalid_indices_are_flagged_not_followed():
 def test_fp16_copy_beyond_range_is_reported(which):
     # k > 128 on the tensor cores keeps fp16 copies of X, W_q|W_k|W_v and W_o:
     # a bf16 value beyond the fp16 range in any of them is reported as
-    # MOSA_ERR_RANGE
+    # MOSA_ERR_RANGE after the layer's forward and backward
     cfg = W.MosaConfig("range", B=1, T=512, d=128, H=8, hp=64, k=256, dtype="bf16", seed=23)
     x = W.make_inputs(cfg)
     names = ("X", "Wr", "Wq", "Wk", "Wv", "Wo")
-    clean = [to_dev(x[n], "bf16") for n in names]
-    shape = mosa.make_shape(clean[0], clean[2], cfg.k)
+    shape = mosa.make_shape(to_dev(x["X"], "bf16"), to_dev(x["Wq"], "bf16"), cfg.k, True)
+    dY = to_dev(x["dY"], "bf16")
+
+    def layer(inp):
+        a = [to_dev(inp[n], "bf16") for n in names]
+        _, I, rs, _, ws = mosa.mosa_forward(*a, cfg.k, first_token=True)
+        mosa.mosa_backward(*a, I, rs, dY, ws)
+        return mosa.mosa_check_status(shape, ws)
+
     bad = dict(x)
     bad[which] = x[which].copy()
     bad[which].flat[5] = 1.0e5
-    args = [to_dev(bad[n], "bf16") for n in names]
-    _, _, _, _, ws = mosa.mosa_forward(*args, cfg.k)
-    assert mosa.mosa_check_status(shape, ws) == 6          # MOSA_ERR_RANGE
-    mosa.mosa_forward(*clean, cfg.k, workspace=ws)
-    assert mosa.mosa_check_status(shape, ws) == 0
+    assert layer(bad) == 6                                  # MOSA_ERR_RANGE
+    assert layer(x) == 0
 
 
 def test_status_word_maps_to_error_codes():

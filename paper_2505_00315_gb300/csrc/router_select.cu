@@ -43,6 +43,10 @@ __device__ __forceinline__ uint32_t order_key(float f) {
     if (u == 0x80000000u) u = 0u;
     return (u & 0x80000000u) ? ~u : (u | 0x80000000u);
 }
+// The score an order key came from (exact, except that both zeros give +0).
+__device__ __forceinline__ float key_score(uint32_t key) {
+    return __uint_as_float((key & 0x80000000u) ? (key ^ 0x80000000u) : ~key);
+}
 
 constexpr int kSelThreads = 1024;   // upper bound; launches use 256 or 1024
 // Rows up to this many scores keep their order keys in shared memory for all
@@ -104,8 +108,21 @@ topk_select_kernel(const float *__restrict__ scores, int T, int k, int32_t *__re
     auto key_of = [&](int t) -> uint32_t {
         return (first_token && t == 0) ? 0xFFFFFFFFu : order_key(__ldg(s + t));
     };
-    if (staged)
-        for (int t = tid; t < T; t += blockDim.x) keys_s[t] = key_of(t);
+    if (staged) {
+        if ((T & 3) == 0 && (reinterpret_cast<uintptr_t>(s) & 15u) == 0) {
+            // four scores per 16-byte load, the loads of a thread issued together
+            const float4 *s4 = reinterpret_cast<const float4 *>(s);
+#pragma unroll 4
+            for (int q = tid; q < T / 4; q += blockDim.x) {
+                const float4 v = __ldg(s4 + q);
+                uint4 kk = make_uint4(order_key(v.x), order_key(v.y), order_key(v.z), order_key(v.w));
+                if (first_token && q == 0) kk.x = 0xFFFFFFFFu;
+                reinterpret_cast<uint4 *>(keys_s)[q] = kk;
+            }
+        } else {
+            for (int t = tid; t < T; t += blockDim.x) keys_s[t] = key_of(t);
+        }
+    }
     __syncthreads();
     auto key_at = [&](int t) -> uint32_t { return staged ? keys_s[t] : key_of(t); };
 
@@ -186,11 +203,15 @@ topk_select_kernel(const float *__restrict__ scores, int T, int k, int32_t *__re
     uint32_t pos = (uint32_t)(before >> 32) + min(eq_before, remaining);
     const int hh = row % H, bb = row / H;
     for (int t = t0; t < t1 && pos < (uint32_t)k; ++t) {
-        const uint32_t key = key_at(t) & mask;
+        const uint32_t full = key_at(t), key = full & mask;
         bool take = key > thr;
         if (key == thr) take = eq_before++ < remaining;
         if (take) {
-            const float v = __ldg(s + t);
+            // the score from its staged key (no second read of the row), but
+            // from memory for token 0 under first_token and for a zero (-0 and
+            // +0 share a key)
+            const float v = (staged && !(first_token && t == 0) && full != 0x80000000u)
+                                ? key_score(full) : __ldg(s + t);
             I[(size_t)row * k + pos] = t;
             rsel[(size_t)row * k + pos] = v;
             if (gidx != nullptr) {

@@ -397,6 +397,14 @@ __device__ __forceinline__ void split_pair2(float a, float b, uint32_t &hi, uint
     lo = __byte_perm(__float_as_uint(ra), __float_as_uint(rb), 0x7632);
 }
 
+// 1/x by the hardware's approximate reciprocal (rcp.approx.ftz: relative
+// error within a couple of ulp; 1/inf = 0).
+__device__ __forceinline__ float rcp_approx(float x) {
+    float y;
+    asm("rcp.approx.ftz.f32 %0, %1;" : "=f"(y) : "f"(x));
+    return y;
+}
+
 // 2^x by the hardware approximation (PTX ex2.approx; -inf gives 0), for the
 // softmax exponentials.
 __device__ __forceinline__ float exp2_fast(float x) {

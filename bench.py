@@ -261,6 +261,7 @@ KERNEL_STAGE = [("tc_gemm_kernel<5>", "router"), ("tc_gemm_kernel<(int)5>", "rou
                 ("scatter_product_kernel<1>", "out"), ("scatter_product_kernel<true>", "out"),
                 ("scatter_product_kernel<(bool)1>", "out"),
                 ("head_sum_kernel<true>", "out"), ("head_sum_kernel<(bool)1>", "out"),
+                ("head_sum_kernel<1>", "out"),
                 ("tc_gemm_kernel<4>", "w_bwd"), ("tc_gemm_kernel<(int)4>", "w_bwd"),
                 ("tc_gemm_kernel<6>", "w_bwd"), ("tc_gemm_kernel<(int)6>", "w_bwd"),
                 ("tc_gemm_kernel<3>", "dwo"), ("tc_gemm_kernel<(int)3>", "dwo"),

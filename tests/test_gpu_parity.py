@@ -28,7 +28,7 @@ def weights(x):
 
 # ------------------------------------------------------------ TopK alone ----
 
-def score_rows(kind, rows, T, rng):
+def score_rows(kind, rows, T, rng, k=1):
     if kind == "uniform":
         return rng.random((rows, T), dtype=np.float32)
     if kind == "ties":
@@ -41,16 +41,29 @@ def score_rows(kind, rows, T, rng):
         v[:, 3::11] = -0.0
         v[:, 5::13] = np.float32(1e-42)
         return v
+    if kind == "split":       # the k kept scores alone in the first radix byte's bin
+        v = (0.25 + 0.01 * rng.random((rows, T))).astype(np.float32)
+        for r in range(rows):
+            v[r, rng.choice(T, size=k, replace=False)] += np.float32(1.25)
+        return v
+    if kind == "gap":         # router-like scores around 1/2, a 1e-3 gap after the k-th
+        v = 0.5 + 0.05 * rng.standard_normal((rows, T))
+        for r in range(rows):
+            top = np.argsort(-v[r], kind="stable")[:k]
+            v[r, top] += 1e-3
+        return v.astype(np.float32)
     raise ValueError(kind)
 
 
-@pytest.mark.parametrize("kind", ["uniform", "ties", "equal", "signed"])
+# ("split" and "gap" let the radix passes stop early, after the first byte or
+# after two or three, as router scores with a planted margin do)
+@pytest.mark.parametrize("kind", ["uniform", "ties", "equal", "signed", "split", "gap"])
 @pytest.mark.parametrize("T,k", [(1, 1), (7, 3), (1000, 1), (1024, 128), (1025, 1025),
                                  (4096, 64), (8192, 4000), (65536, 257)])
 def test_topk_bit_exact(kind, T, k):
     rng = np.random.default_rng(T * 31 + k)
     rows = 3 if T > 10000 else 5
-    s = score_rows(kind, rows, T, rng)
+    s = score_rows(kind, rows, T, rng, k)
     I, rs = mosa.mosa_topk(torch.from_numpy(s).cuda(), k)
     I, rs = I.cpu().numpy(), rs.cpu().numpy()
     for r in range(rows):

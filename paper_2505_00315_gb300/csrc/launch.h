@@ -134,6 +134,11 @@ bool use_tc(const Dims &dm);
 // K, V and dA are then stored as fp16 rows [H, B*k, 64], with RoPE applied
 // in the projection's epilogue; otherwise they are bf16 pairs (or fp32).
 bool attn_f16(const Dims &dm);
+// dQ|dK|dV|dlogit rows as single fp16 ([H, B*k, 256]) for the input- and
+// weight-gradient products (with the fp16 copies of X and W_q|W_k|W_v): the
+// tensor-core path for k > 128, and for k <= 128 where the weights' copy is
+// small (not with the opt-in fused k <= 128 backward, which keeps bf16 pairs).
+bool dqkv_f16(const Dims &dm);
 // Fused F3 + F4 + F5 for k <= 128 (tc_fused_fwd.cu); off with MOSA_FUSED_FWD=0.
 bool tc_fused_forward_supported(const Dims &dm);
 bool use_fused_forward(const Dims &dm);

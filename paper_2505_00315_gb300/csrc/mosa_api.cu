@@ -71,11 +71,13 @@ size_t carve(const Dims &dm, char *base, Saved *sv) {
     // (reserved for either dtype, so that the size depends on the shape only)
     if (dm.H % 64 != 0) s.Wr64 = take((size_t)2 * dm.d * ((dm.H + 63) / 64 * 64));
     s.spans = (unsigned long long *)take(sizeof(unsigned long long) * 2 * 16);
-    // the fp16 attention path's copies (reserved whenever that path can run,
-    // so the size does not depend on the environment's kernel-path switches)
-    if (dm.bf16 && dm.hp == 64 && dm.k > 128) {
+    // the fp16 copies of the tensor-core path (reserved whenever that path can
+    // run, so the size does not depend on the environment's kernel-path switches)
+    if (dm.bf16 && dm.hp == 64) {
         s.X16 = take((size_t)2 * dm.B * dm.T * dm.d);
         s.W16 = take((size_t)2 * 4 * dm.H * dm.d * dm.hp);   // W_q, W_k, W_v, W_o
+    }
+    if (dm.bf16 && dm.hp == 64 && dm.k > 128) {
         s.AR16 = take((size_t)2 * R * dm.hp);
         s.pos = (int32_t *)take(sizeof(int32_t) * (size_t)dm.H * dm.B * dm.T);
     }
@@ -203,11 +205,15 @@ mosa_status forward_tc(const Dims &dm, const void *X, const void *W_r, const voi
     // (the token-major output product writes every element of Y itself)
     const bool headsum = !use_fused_forward(dm) && use_headsum_out(dm);
     if (!dm.accumulate && !headsum) MOSA_TRY(cudaMemsetAsync(Y, 0, sizeof(float) * ny, r.side));
-    // fp16 attention path: the fp16 copies of X and W_q|W_k|W_v that the
-    // backward's products with dQ|dK|dV read, and of W_o for the output
-    // product, made here beside TopK, whose grid (one CTA per (b, h) row)
-    // leaves most SMs idle
-    if (attn_f16(dm)) MOSA_TRY(tc_f16_copies(dm, X, W_q, W_k, W_v, W_o, sv, r.side));
+    // the fused k <= 128 kernel needs only Y zeroed from the side stream
+    const bool fused = use_fused_forward(dm);
+    if (fused) MOSA_TRY(cudaEventRecord(r.ev[1], r.side));
+    // the fp16 copies of X and W_q|W_k|W_v that the backward's products with
+    // single-fp16 dQ|dK|dV read, and (k > 128) of W_o for the output product,
+    // made here beside TopK, whose grid (one CTA per (b, h) row) leaves most
+    // SMs idle
+    if (dqkv_f16(dm))
+        MOSA_TRY(tc_f16_copies(dm, X, W_q, W_k, W_v, attn_f16(dm) ? W_o : nullptr, sv, r.side));
     if (route) {
         StageScope st_(kStageSelect, s);
         MOSA_TRY(launch_select(dm.B * dm.H, dm.T, dm.k, rf, I, r_sel, dm.B, dm.H, sv.gidx,
@@ -224,10 +230,13 @@ mosa_status forward_tc(const Dims &dm, const void *X, const void *W_r, const voi
         MOSA_TRY(link(s, r.side, r.ev[2]));
         MOSA_TRY(tc_token_rows(dm, sv, r.side));
     }
-    if (use_fused_forward(dm)) {
-        MOSA_TRY(link(r.side, s, r.ev[1]));  // Y zeroed
-        StageScope st_(kStageFwdUnit, s);
-        MOSA_TRY(tc_fused_forward(dm, X, W_q, W_k, W_v, W_o, sv, Y, s));
+    if (fused) {
+        MOSA_TRY(cudaStreamWaitEvent(s, r.ev[1], 0));  // Y zeroed
+        {
+            StageScope st_(kStageFwdUnit, s);
+            MOSA_TRY(tc_fused_forward(dm, X, W_q, W_k, W_v, W_o, sv, Y, s));
+        }
+        MOSA_TRY(link(r.side, s, r.ev[3]));  // the backward's fp16 copies
         return MOSA_OK;
     }
     {
@@ -316,8 +325,8 @@ mosa_status backward_tc(const Dims &dm, const void *X, const void *W_r, const vo
     {
         StageScope st_(kStageAttnBwd, s);
         MOSA_TRY(launch_attn_bwd(dm, sv, s, zero_in_attn ? dX : nullptr));
-        // (the fp16 path turns dQ and dK back before rounding them)
-        if (dm.rope && !attn_f16(dm)) MOSA_TRY(rope_qk(dm, sv, true, s));
+        // (the fp16 rows have dQ and dK turned back before rounding)
+        if (dm.rope && !dqkv_f16(dm)) MOSA_TRY(rope_qk(dm, sv, true, s));
     }
     MOSA_TRY(link(s, t, r.ev[2]));  // dQ|dK|dV|dlogit ready for dW
     {

@@ -398,6 +398,9 @@ struct BwdParams {
     // of every CTA zeroes, one slice per CTA, while the attention runs
     float4 *zero;
     long long zero_n4;
+    // k <= 128: dQ|dK|dV out as single fp16 into [H, B*k, 256] rows (dQ and
+    // dK turned back by RoPE first when asked), else as bf16 pairs
+    int out16;
 };
 
 template <class SM>
@@ -1118,23 +1121,38 @@ __global__ void __launch_bounds__(kSmallThreads, 1) attn_bwd_small_kernel(const 
         tc_fence_after();
         if (!ok) flag_timeout_b(sm, p.status);
         const bool live = __all_sync(0xffffffffu, ok && !*(volatile int *)&sm.abort);
-        // dQ, dK, dV columns 32 ch .. +31 as bf16 pairs into the Q, K, V tiles
-        // (free once every MMA is done), then out by six TMA stores into the
-        // dQKV rows: hi blocks at columns 0, 64, 128, lo blocks 256 further
+        // dQ, dK, dV columns 32 ch .. +31 into the Q, K, V tiles (free once
+        // every MMA is done), then out by TMA stores into the dQKV rows: as
+        // bf16 pairs (hi blocks at columns 0, 64, 128, lo blocks 256 further)
+        // or as single fp16 blocks at columns 0, 64, 128
         uint8_t(*tiles[3])[kPBig] = {sm.q, sm.k, sm.v};
         const uint32_t src[3] = {tDQ, tDK, tDV};
         const float fac[3] = {p.scale, p.scale, 1.f};
+        // original position of this row's token (RoPE is turned back on the
+        // first 32 columns of dQ and dK, which only ch == 0 holds)
+        const int tpos = (p.out16 && p.rope && valid && ch == 0) ? p.gidx[base + r] % p.T : 0;
+        float omax = 0.f;
 #pragma unroll 1
         for (int t = 0; t < 3; ++t) {
             float v[32];
             tmem_ld32(src[t] + lane_off + 32 * ch, v);
-            put_pair32(tiles[t][0], tiles[t][1], r, 32 * ch, v, fac[t]);
+            if (!p.out16) {
+                put_pair32(tiles[t][0], tiles[t][1], r, 32 * ch, v, fac[t]);
+                continue;
+            }
+            if (p.rope && t < 2 && ch == 0) {
+#pragma unroll
+                for (int pp = 0; pp < 16; ++pp)
+                    rope_turn(v[2 * pp], v[2 * pp + 1], p.rope_tab.phi[pp], tpos, -1.f);
+            }
+            omax = fmaxf(omax, put_f16_32(tiles[t][0], r, 32 * ch, v, fac[t]));
         }
+        if (p.out16 && live && valid && !(omax < kF16Overflow)) atomicOr(p.status, kStatusRange);
         fence_proxy_async();
         named_barrier(1, kSoftmaxThreads);
         if (threadIdx.x == 128 && live) {
             for (int t = 0; t < 3; ++t)
-                for (int hf = 0; hf < 2; ++hf)
+                for (int hf = 0; hf < (p.out16 ? 1 : 2); ++hf)
                     tma_store_3d(&p.mOut, smem_u32(tiles[t][hf]), 64 * t + 256 * hf, b0 * p.k, h);
             bulk_commit();
             bulk_wait0();
@@ -1215,8 +1233,11 @@ cudaError_t tc_attn_bwd(const Dims &dm, const Saved &sv, cudaStream_t s, float *
         memset(&sp, 0, sizeof(sp));
         const int Mtok = dm.B * dm.k;
         sp.U = kSmallK / dm.k;
-        const uint64_t odims[3] = {512, (uint64_t)Mtok, (uint64_t)dm.H};
-        const uint64_t ostrides[2] = {1024, (uint64_t)Mtok * 1024};
+        // dQ|dK|dV|dlogit rows: fp16 [H, B*k, 256], or bf16 pairs [H, B*k, 512]
+        sp.out16 = dqkv_f16(dm) ? 1 : 0;
+        const uint64_t ocols = sp.out16 ? 256 : 512;
+        const uint64_t odims[3] = {ocols, (uint64_t)Mtok, (uint64_t)dm.H};
+        const uint64_t ostrides[2] = {ocols * 2, (uint64_t)Mtok * ocols * 2};
         const uint32_t obox[3] = {64, (uint32_t)(sp.U * dm.k), 1};
         const bool ok = map_rows(&sp.mA0, sv.Q, dm.H, Mtok) && map_rows(&sp.mA1, sv.K, dm.H, Mtok) &&
                         map_rows(&sp.mB0, sv.V, dm.H, Mtok) && map_rows(&sp.mB1, sv.dA, dm.H, Mtok) &&
@@ -1232,6 +1253,10 @@ cudaError_t tc_attn_bwd(const Dims &dm, const Saved &sv, cudaStream_t s, float *
         sp.dQKV = static_cast<bf16 *>(sv.dQKV);
         sp.status = sv.status;
         sp.span = active_span();
+        sp.gidx = sv.gidx;
+        sp.T = dm.T;
+        sp.rope = dm.rope ? 1 : 0;
+        if (dm.rope) sp.rope_tab = make_rope_table(dm.hp, dm.T);
         const cudaError_t attr_small = allow_smem((const void *)attn_bwd_small_kernel, kSmallBwdSmem);
         if (attr_small != cudaSuccess) return attr_small;
         cudaError_t e = launch_pdl(attn_bwd_small_kernel, dim3(1, (dm.B + sp.U - 1) / sp.U, dm.H),

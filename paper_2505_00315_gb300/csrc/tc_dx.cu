@@ -313,7 +313,7 @@ cudaError_t tc_dx(const Dims &dm, const void *Wq, const void *Wk, const void *Wv
     memset(&p, 0, sizeof(p));
     const int Mtok = dm.B * dm.k;
     if (Mtok <= 0 || dm.d <= 0 || dm.H <= 0) return cudaSuccess;
-    p.f16 = attn_f16(dm) ? 1 : 0;
+    p.f16 = dqkv_f16(dm) ? 1 : 0;
     const size_t nw = (size_t)dm.H * dm.d * 64;
     const void *W[3] = {Wq, Wk, Wv};
     if (p.f16)

@@ -170,6 +170,7 @@ struct TcParams {
     uint32_t *status;
     int half;              // kQKV / kG: Q, K, V or dA as fp16 rows [H, B*k, 64] (k > 128)
                            // instead of bf16 pairs
+    int dq16;              // kG: dlogit into fp16 dQ|dK|dV|dlogit rows [H, B*k, 256]
     int rope;              // kQKV with half: rotate Q and K (Sec. 2.2) before rounding
     RopeTable rope_tab;
     unsigned long long *span;   // measurement: this stage's kernel span slot, or null
@@ -718,7 +719,7 @@ __global__ void __launch_bounds__(kThreads, Cfg<KIND>::MIN_CTAS)
             // the 4th 64-column block that kDW reads for dW_r; the block's other
             // columns are never written: accumulator column n of that product
             // depends only on B column n, and columns 193..255 are not read
-            if (live && !p.half) {
+            if (live && !p.dq16) {
                 const bf16 dh = __float2bfloat16_rn(dl);
                 const bf16 dlo = __float2bfloat16_rn(dl - __bfloat162float(dh));
                 bf16 *dq = static_cast<bf16 *>(p.out[1]) + row * kDQKVCols;
@@ -982,6 +983,18 @@ bool tc_supported(const Dims &dm) {
 
 bool attn_f16(const Dims &dm) { return dm.k > 128 && use_tc(dm); }
 
+bool dqkv_f16(const Dims &dm) {
+    if (!use_tc(dm)) return false;
+    if (dm.k > 128) return true;
+    if (use_fused_backward(dm)) return false;
+    // k <= 128: worth the forward's fp16 copies of X and W_q|W_k|W_v while
+    // the weights' copy is at most twice X's (3 H h' <= 2 B T).  Measured:
+    // 101.8 against 107.0 us at B8 T1024 d512 H16 k128, 384 against 397 at
+    // B16 T1024 d1024 H64 k64, 414 against 422 at B4 T4096 d1024 H128 k128;
+    // 495 against 486 at H256 k64, whose weights are three times X.
+    return 3LL * dm.H * dm.hp <= 2LL * dm.B * dm.T;
+}
+
 cudaError_t tc_qkv(const Dims &dm, const void *X, const void *Wq, const void *Wk, const void *Wv,
                    const Saved &sv, cudaStream_t s) {
     TcParams p = base_params(dm, sv);
@@ -1037,6 +1050,7 @@ cudaError_t tc_out_bwd_g(const Dims &dm, const void *Wo, const void *dY, const S
     p.out_f1 = sv.Dd;
     p.out_f2 = sv.dlogit;
     p.half = attn_f16(dm) ? 1 : 0;
+    p.dq16 = dqkv_f16(dm) ? 1 : 0;
     // the k > 128 attention backward (next on this stream) reduce-adds dQ into
     // sv.G: its rows start at zero here, beside dA
     if (dm.k > 128) p.zero_rows = sv.G;
@@ -1095,7 +1109,7 @@ cudaError_t tc_w_bwd(const Dims &dm, const void *X, const Saved &sv, float *dWq,
     while (tiles * p.splits * 2 <= 152 && p.splits * 4 <= p.nkb) p.splits *= 2;
     // fp16 attention path: dQ|dK|dV|dlogit single fp16 rows of 256, and the
     // gathered rows from the fp16 copy of X, one MMA per step
-    const bool half = attn_f16(dm);
+    const bool half = dqkv_f16(dm);
     const void *Xs = half ? sv.X16 : X;
     bool ok = map_gather(&p.mapA, Xs, (uint64_t)dm.B * dm.T, dm.d) &&
               map_heads(&p.mapB[0], sv.dQKV, dm.H, p.Mtok, half ? 256 : kDQKVCols, 32);

@@ -86,6 +86,9 @@ SMALL = [
     W.MosaConfig("pack2_oddB_bf16", B=3, T=200, d=64, H=2, hp=64, k=64, dtype="bf16", seed=17),
     W.MosaConfig("pack4_bf16", B=5, T=100, d=64, H=3, hp=64, k=32, dtype="bf16", seed=18),
     W.MosaConfig("pack2_k50_bf16", B=5, T=120, d=64, H=2, hp=64, k=50, dtype="bf16", seed=19),
+    # k <= 128 with weights large against X (3 H h' > 2 B T): dQ|dK|dV stay
+    # bf16 pairs for the input- and weight-gradient products
+    W.MosaConfig("pairs_bf16", B=1, T=160, d=64, H=4, hp=64, k=48, dtype="bf16", seed=20),
     W.MosaConfig("pack42_k3_bf16", B=5, T=40, d=32, H=2, hp=64, k=3, dtype="bf16", seed=20),
     # k > 128: several 128-query tiles and 128-key blocks, full and ragged
     W.MosaConfig("largek_bf16", B=1, T=512, d=128, H=3, hp=64, k=384, dtype="bf16", seed=21),

@@ -96,7 +96,8 @@ struct Saved {
     float *WrT;         // [H,d] fp32 transpose of W_r (tensor-core dX epilogue)
     void *Wr64;         // [d, H rounded up to 64] bf16 W_r with zero columns past H
                         // (tensor-core router, H % 64 != 0)
-    // fp16 attention path (tensor cores, k > 128): dQKV is [H,B*k,256] fp16
+    // fp16 dQ|dK|dV rows (tensor cores: k > 128, and k <= 128 where the
+    // weights' copy is small, dqkv_f16): dQKV is [H,B*k,256] fp16
     // (dQ | dK | dV | dlogit, 0..), and the backward reads X and W_q|W_k|W_v
     // through fp16 copies so that every product with dQKV is one MMA
     void *X16;          // [B*T,d] fp16 copy of X
